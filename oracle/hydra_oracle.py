@@ -1,0 +1,322 @@
+"""fp64 CPU oracle for the Hydra-PPO experience-scoring path (arXiv 2309.00754).
+
+TEST INFRASTRUCTURE, NOT PRODUCT CODE. Only the test-suite, the package's smoke check
+and the benchmark's CPU-baseline leg may import this module. The CUDA library never
+calls it, and it shares no code with the CUDA library: no kernels, helpers, tables or
+constants. Inputs arrive as plain numpy arrays (bf16 tensors as uint16 bit patterns).
+
+Everything is computed in float64 from the exact input values. Where the GPU path stores
+an intermediate in bf16 (the LoRA down-projection u, bf16 linear outputs, the bf16
+activations of the Llama block), the oracle rounds at the same tensor boundary, so that
+the two sides see the same storage format; all arithmetic between those boundaries is
+fp64. Matrix products use numpy's matmul as a library primitive, with no blocking or
+reordering of our own.
+
+Paper references (section / algorithm / appendix of "Efficient RLHF: Reducing the Memory
+Usage of PPO"):
+  * §2 "Stage 3: PPO" -- LoRA on all linear layers; ratio and clipped surrogate; GAE uses
+    V(x, y) to build the advantage estimates; critic trained on returns.
+  * §3 "Dynamic LoRA" -- the reference policy is the actor with its LoRA parameters
+    ignored, pi_ref <- LO(pi_theta); likewise the reward model is LO(critic).
+  * §3 "Stage 2: Hydra-PPO" and Algorithm 1 (J-Hydra-PPO) / Algorithm 2 (Hydra-PPO) --
+    one frozen base; "turn LoRA off ... to compute reward and reference log
+    probabilities"; "use reward and reference log probability to calculate A-hat".
+  * Appendix B "Experiment Details" -- KL coefficient beta = 0.02, GAE gamma = 1.0,
+    lambda = 0.95, LoRA rank 128.
+
+Readings where the paper is silent (the same readings the CUDA path implements):
+  * LoRA update: y_on = x W + s (x A) B (Hu et al. 2021 form); s is an argument.
+  * u = s * (x A) is stored in bf16 (the CUDA path keeps it as a bf16 operand).
+  * Per-token KL penalty uses the sampled-token estimate logp_actor - logp_ref; the
+    sequence score is added at the last valid token t = len - 1.
+  * GAE: the value after the last valid token is 0 (terminal); positions >= len are 0.
+
+Parity pins for every function live in tests/test_oracle_pins.py (closed forms,
+invariants, brute force, library routines, hand-worked fixtures in tests/golden/).
+The full 32-layer Llama composition (`llama_score`) is pinned only through its per-op
+pieces and small-size invariants: parity unpinned for the composition as a whole.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+# ---------------------------------------------------------------------------
+# bf16 storage format (IEEE binary32 with the low 16 mantissa bits dropped)
+# ---------------------------------------------------------------------------
+
+
+def bf16_to_f64(bits) -> np.ndarray:
+    """Widen bf16 bit patterns (uint16) to exact float64 values."""
+    b = np.asarray(bits, dtype=np.uint16).astype(np.uint32) << np.uint32(16)
+    return b.view(np.float32).astype(np.float64)
+
+
+def f64_to_bf16_bits(x) -> np.ndarray:
+    """Round to bf16 (nearest, ties to even, via float32) and return uint16 bits."""
+    f = np.ascontiguousarray(np.asarray(x, dtype=np.float64).astype(np.float32))
+    u = f.view(np.uint32).astype(np.uint64)
+    lsb = (u >> np.uint64(16)) & np.uint64(1)
+    u = (u + np.uint64(0x7FFF) + lsb) >> np.uint64(16)
+    return u.astype(np.uint16)
+
+
+def round_bf16(x) -> np.ndarray:
+    """Value of x after storing it as bf16 (float64 result)."""
+    return bf16_to_f64(f64_to_bf16_bits(x))
+
+
+# ---------------------------------------------------------------------------
+# a1 / a2 / a3: dual-output LoRA linear (§2 Stage 3 LoRA; §3 Dynamic LoRA)
+# Storage: x [M, K], W [N, K] (the paper's K x N weight, transposed), A [r, K], B [N, r].
+# ---------------------------------------------------------------------------
+
+
+def lora_down(x_on, A, s) -> np.ndarray:
+    """u = s * (x_on A^T), stored as bf16. x_on, A: float64 arrays."""
+    return round_bf16(s * (x_on @ A.T))
+
+
+def dual_lora_linear(x_off, x_on, W, A, B, s, out_bf16=True):
+    """(y_off, y_on) with y_off = x_off W^T (LoRA off, the reference / reward stream) and
+    y_on = x_on W^T + u B^T with u = s x_on A^T (LoRA on, the actor / critic stream).
+
+    §3 Dynamic LoRA: pi_ref <- LO(pi_theta), LO ignores the LoRA parameters, so the same
+    frozen W produces both outputs. A is None means no LoRA on this linear (y_on = x_on W^T).
+    """
+    y_off = x_off @ W.T
+    y_on = x_on @ W.T
+    if A is not None:
+        u = lora_down(x_on, A, s)
+        y_on = y_on + u @ B.T
+    if out_bf16:
+        return round_bf16(y_off), round_bf16(y_on)
+    return y_off, y_on
+
+
+# ---------------------------------------------------------------------------
+# a4: log-probability of the sampled token (Alg. 1/2 "reference log probabilities";
+# §2 ratio r(theta) = pi_theta / pi_old needs the actor's log-probabilities too)
+# ---------------------------------------------------------------------------
+
+
+def logsumexp_rows(z) -> np.ndarray:
+    """Textbook two-pass log-sum-exp per row: m = max_v z_v; m + log sum_v exp(z_v - m)."""
+    m = np.max(z, axis=-1, keepdims=True)
+    return (m + np.log(np.sum(np.exp(z - m), axis=-1, keepdims=True)))[..., 0]
+
+
+def log_softmax_gather(z, ids):
+    """(logp, lse): logp[t] = z[t, ids[t]] - lse[t], lse[t] = log sum_v exp(z[t, v])."""
+    lse = logsumexp_rows(z)
+    picked = np.take_along_axis(z, np.asarray(ids, dtype=np.int64)[:, None], axis=1)[:, 0]
+    return picked - lse, lse
+
+
+# ---------------------------------------------------------------------------
+# a5: KL-penalised per-token reward (§2 reference "used to prevent reward divergence";
+# Appendix B KL coefficient beta; Alg. 1/2 reward from the LoRA-off model)
+# ---------------------------------------------------------------------------
+
+
+def kl_penalised_reward(logp_actor, logp_ref, lengths, score, beta):
+    """r[s, t] = -beta (logp_actor - logp_ref) for t < len_s, plus score_s at t = len_s - 1;
+    0 for t >= len_s. Inputs are [S, L] (score [S] or None)."""
+    la = np.asarray(logp_actor, dtype=np.float64)
+    lr = np.asarray(logp_ref, dtype=np.float64)
+    S, L = la.shape
+    t = np.arange(L)[None, :]
+    n = np.asarray(lengths, dtype=np.int64)[:, None]
+    valid = t < n
+    r = np.where(valid, -beta * (la - lr), 0.0)
+    if score is not None:
+        last = (t == n - 1) & valid
+        r = r + np.where(last, np.asarray(score, dtype=np.float64)[:, None], 0.0)
+    return r
+
+
+def token_logprobs_kl(z_actor, z_ref, ids, lengths, score, beta, S, L):
+    """The hydra_token_logprobs_kl operation: z_* are [S*L, V] logit rows aligned with ids
+    (row t predicts ids[t]); returns dict of [S, L] arrays (zero at t >= len) plus lse."""
+    la, lse_a = log_softmax_gather(z_actor, ids)
+    lr, lse_r = log_softmax_gather(z_ref, ids)
+    la = la.reshape(S, L)
+    lr = lr.reshape(S, L)
+    if lengths is None:
+        lengths = np.full(S, L, dtype=np.int64)
+    valid = np.arange(L)[None, :] < np.asarray(lengths)[:, None]
+    return {
+        "logp_actor": np.where(valid, la, 0.0),
+        "logp_ref": np.where(valid, lr, 0.0),
+        "reward": kl_penalised_reward(la, lr, lengths, score, beta),
+        "lse_actor": np.where(valid, lse_a.reshape(S, L), 0.0),
+        "lse_ref": np.where(valid, lse_r.reshape(S, L), 0.0),
+    }
+
+
+# ---------------------------------------------------------------------------
+# a7: generalised advantage estimation (§2 "GAE uses V(x,y) to construct A-hat", critic
+# trained on returns; Appendix B gamma = 1.0, lambda = 0.95; Alg. 1/2 "calculate A-hat")
+# ---------------------------------------------------------------------------
+
+
+def gae(rewards, values, lengths, gamma, lam):
+    """Plain backward recursion, one token at a time:
+        delta_t = r_t + gamma * V_{t+1} - V_t      (V_{len} = 0: terminal)
+        A_t     = delta_t + gamma * lam * A_{t+1}  (A_{len} = 0)
+        R_t     = A_t + V_t
+    Positions t >= len are 0 in both outputs."""
+    r = np.asarray(rewards, dtype=np.float64)
+    v = np.asarray(values, dtype=np.float64)
+    S, L = r.shape
+    adv = np.zeros((S, L))
+    ret = np.zeros((S, L))
+    for s in range(S):
+        n = int(lengths[s]) if lengths is not None else L
+        a_next = 0.0
+        for t in range(n - 1, -1, -1):
+            v_next = v[s, t + 1] if t + 1 < n else 0.0
+            delta = r[s, t] + gamma * v_next - v[s, t]
+            a = delta + gamma * lam * a_next
+            adv[s, t] = a
+            ret[s, t] = a + v[s, t]
+            a_next = a
+    return adv, ret
+
+
+# ---------------------------------------------------------------------------
+# a8: Llama decoder pieces used by the full scoring pass (the paper uses Llama 7b, §4)
+# ---------------------------------------------------------------------------
+
+
+def rmsnorm(h, w, eps):
+    """RMSNorm (Zhang & Sennrich 2019): h / sqrt(mean(h^2) + eps) * w, per row."""
+    h = np.asarray(h, dtype=np.float64)
+    return h / np.sqrt(np.mean(h * h, axis=-1, keepdims=True) + eps) * w
+
+
+def rope(x, positions, theta):
+    """Rotary embedding (Su et al. 2021), rotate-half pairing: dims (i, i + D/2) of each
+    head form one plane rotated by angle pos * theta^(-2i/D). x: [T, H, D]."""
+    T, H, D = x.shape
+    half = D // 2
+    inv = theta ** (-np.arange(half, dtype=np.float64) * 2.0 / D)
+    ang = np.asarray(positions, dtype=np.float64)[:, None] * inv[None, :]  # [T, half]
+    c = np.cos(ang)[:, None, :]
+    s = np.sin(ang)[:, None, :]
+    x1 = x[..., :half]
+    x2 = x[..., half:]
+    return np.concatenate([x1 * c - x2 * s, x1 * s + x2 * c], axis=-1)
+
+
+def causal_attention(q, k, v):
+    """softmax(q k^T / sqrt(D) + causal mask) v per head. q, k, v: [T, H, D] -> [T, H, D]."""
+    T, H, D = q.shape
+    out = np.empty((T, H, D))
+    mask = np.triu(np.ones((T, T), dtype=bool), 1)
+    for h in range(H):
+        sc = (q[:, h, :] @ k[:, h, :].T) / np.sqrt(D)
+        sc = np.where(mask, -np.inf, sc)
+        m = np.max(sc, axis=1, keepdims=True)
+        p = np.exp(sc - m)
+        p = p / np.sum(p, axis=1, keepdims=True)
+        out[:, h, :] = p @ v[:, h, :]
+    return out
+
+
+def silu(x):
+    return x / (1.0 + np.exp(-x))
+
+
+def swiglu(g, u):
+    """SwiGLU gate (Shazeer 2020): silu(g) * u."""
+    return silu(g) * u
+
+
+def llama_score(weights, ids, prompt_len, cfg, seq_lengths=None, beta=0.1, gamma=1.0,
+                lam=0.95, n_layers=None):
+    """One sequence of the full J-Hydra scoring pass (Alg. 1 scoring steps), both streams.
+
+    weights: dict of float64 arrays (exact bf16 values):
+      embed [V, d]; per layer l: wq, wk, wv, wo [d, d]; wg, wu [F, d]; wd [d, F];
+      norm1, norm2 [d]; lora[name] = (A [r, in], B [out, r]) for name in q, v, g, u, d;
+      final_norm [d]; lm_head [V, d]; w_rm [d].
+    ids: [T] token ids (prompt then response); prompt_len P; response tokens are P..T-1.
+    Returns dict with logp_actor, logp_ref, reward, values, score, advantages, returns
+    (arrays of length T-P for the response) and the final normed hidden states.
+
+    Streams: "off" = LoRA ignored (reference policy and reward model, §3 Dynamic LoRA);
+    "on" = actor/critic with the single J-Hydra LoRA set (§3 J-Hydra-PPO).
+    Values: V_t = w_rm . h_on[p_t - 1]; score = w_rm . h_off[T - 1] (reward-model head on
+    the LoRA-off stream, critic = same head with LoRA on).
+    """
+    d = cfg["d"]
+    H = cfg["n_heads"]
+    Dh = d // H
+    eps = cfg["eps"]
+    s = cfg["lora_scale"]
+    T = len(ids)
+    P = prompt_len
+    L = T - P
+    n_layers = cfg["n_layers"] if n_layers is None else n_layers
+    pos = np.arange(T)
+
+    h_off = weights["embed"][np.asarray(ids)]
+    h_on = h_off.copy()
+
+    def lin(name, l, a_off, a_on):
+        W = weights[name][l]
+        ab = weights["lora"].get(name)
+        if ab is None:
+            return dual_lora_linear(a_off, a_on, W, None, None, s)
+        return dual_lora_linear(a_off, a_on, W, ab[0][l], ab[1][l], s)
+
+    for l in range(n_layers):
+        a_off = round_bf16(rmsnorm(h_off, weights["norm1"][l], eps))
+        a_on = round_bf16(rmsnorm(h_on, weights["norm1"][l], eps))
+        q = lin("wq", l, a_off, a_on)
+        k = lin("wk", l, a_off, a_on)
+        v = lin("wv", l, a_off, a_on)
+        att = []
+        for i in range(2):
+            qi = round_bf16(rope(q[i].reshape(T, H, Dh), pos, cfg["rope_theta"]))
+            ki = round_bf16(rope(k[i].reshape(T, H, Dh), pos, cfg["rope_theta"]))
+            vi = v[i].reshape(T, H, Dh)
+            att.append(round_bf16(causal_attention(qi, ki, vi).reshape(T, d)))
+        o = lin("wo", l, att[0], att[1])
+        h_off = h_off + o[0]
+        h_on = h_on + o[1]
+        a_off = round_bf16(rmsnorm(h_off, weights["norm2"][l], eps))
+        a_on = round_bf16(rmsnorm(h_on, weights["norm2"][l], eps))
+        g = lin("wg", l, a_off, a_on)
+        u = lin("wu", l, a_off, a_on)
+        m_off = round_bf16(swiglu(g[0], u[0]))
+        m_on = round_bf16(swiglu(g[1], u[1]))
+        dn = lin("wd", l, m_off, m_on)
+        h_off = h_off + dn[0]
+        h_on = h_on + dn[1]
+
+    f_off = round_bf16(rmsnorm(h_off, weights["final_norm"], eps))
+    f_on = round_bf16(rmsnorm(h_on, weights["final_norm"], eps))
+    rows = np.arange(P - 1, T - 1)                       # hidden row predicting token P+t
+    z_ref = f_off[rows] @ weights["lm_head"].T
+    z_act = f_on[rows] @ weights["lm_head"].T
+    resp_ids = np.asarray(ids)[P:]
+    la, _ = log_softmax_gather(z_act, resp_ids)
+    lr, _ = log_softmax_gather(z_ref, resp_ids)
+    n = L if seq_lengths is None else int(seq_lengths)
+    score = float(f_off[P - 1 + n] @ weights["w_rm"]) if n > 0 else 0.0
+    values = f_on[rows] @ weights["w_rm"]
+    reward = kl_penalised_reward(la[None], lr[None], [n], [score], beta)[0]
+    adv, ret = gae(reward[None], values[None], [n], gamma, lam)
+    valid = np.arange(L) < n
+    return {
+        "logp_actor": np.where(valid, la, 0.0),
+        "logp_ref": np.where(valid, lr, 0.0),
+        "reward": reward,
+        "values": np.where(valid, values, 0.0),
+        "score": score,
+        "advantages": adv[0],
+        "returns": ret[0],
+        "h_off": f_off,
+        "h_on": f_on,
+    }

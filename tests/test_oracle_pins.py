@@ -1,0 +1,376 @@
+"""Pins for the fp64 oracle: each oracle function is checked against something other than
+itself -- hand-worked fixtures (tests/golden/), closed forms, invariants, brute force on
+tiny inputs, or a library routine -- chosen so that a dropped term, a wrong sign, a wrong
+index or a transposed operand fails at least one check."""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import scipy.special
+
+import oracle as O
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _load(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        return json.load(f)
+
+
+# ---------------------------------------------------------------- bf16 storage
+
+
+def test_bf16_rounding_ties_to_even():
+    one = 1.0
+    ulp = 2.0 ** -7  # bf16 has 7 explicit mantissa bits
+    assert O.round_bf16(np.array([one]))[0] == 1.0
+    # exact half-ulp ties round to the even neighbour
+    assert O.round_bf16(np.array([one + ulp / 2]))[0] == 1.0
+    assert O.round_bf16(np.array([one + 3 * ulp / 2]))[0] == one + 2 * ulp
+    # just above a tie rounds up
+    assert O.round_bf16(np.array([one + ulp / 2 + 2.0 ** -20]))[0] == one + ulp
+    assert O.f64_to_bf16_bits(np.array([1.0, -2.0]))[0] == 0x3F80
+    assert O.f64_to_bf16_bits(np.array([1.0, -2.0]))[1] == 0xC000
+    x = np.array([3.140625, -0.0078125, 65280.0])  # bf16-representable values
+    assert np.array_equal(O.round_bf16(x), x)
+
+
+# ---------------------------------------------------------------- a1/a2 LoRA linear
+
+
+def test_lora_hand_example():
+    g = _load("lora_dual_linear.json")
+    x = np.array(g["x"], float)
+    y_off, y_on = O.dual_lora_linear(x, x, np.array(g["W"], float), np.array(g["A"], float),
+                                     np.array(g["B"], float), g["s"], out_bf16=False)
+    assert np.array_equal(y_off, np.array(g["y_off"], float))
+    assert np.array_equal(y_on, np.array(g["y_on"], float))
+
+
+def _int_problem(rng, M, K, N, r):
+    x = rng.integers(-3, 4, size=(M, K)).astype(float)
+    W = rng.integers(-3, 4, size=(N, K)).astype(float)
+    A = rng.integers(-2, 3, size=(r, K)).astype(float)
+    B = rng.integers(-2, 3, size=(N, r)).astype(float)
+    return x, W, A, B
+
+
+def test_lora_brute_force_loops_nonsquare():
+    # small integers: every product and sum is exact in fp64 and u is exact in bf16
+    rng = np.random.default_rng(1)
+    M, K, N, r, s = 5, 7, 3, 2, 2.0
+    x, W, A, B = _int_problem(rng, M, K, N, r)
+    x_off = x[::-1].copy()
+    y_off, y_on = O.dual_lora_linear(x_off, x, W, A, B, s, out_bf16=False)
+    for m in range(M):
+        for n in range(N):
+            acc_off = sum(x_off[m, k] * W[n, k] for k in range(K))
+            acc = sum(x[m, k] * W[n, k] for k in range(K))
+            for j in range(r):
+                u = s * sum(x[m, k] * A[j, k] for k in range(K))
+                acc += u * B[n, j]
+            assert y_off[m, n] == acc_off
+            assert y_on[m, n] == acc
+
+
+def test_lora_equals_dense_merged_weight():
+    # rank-r identity: x W^T + s (x A^T) B^T == x (W + s B A)^T
+    rng = np.random.default_rng(2)
+    x, W, A, B = _int_problem(rng, 6, 9, 4, 3)
+    s = 0.5
+    _, y_on = O.dual_lora_linear(x, x, W, A, B, s, out_bf16=False)
+    dense = x @ (W + s * (B @ A)).T
+    assert np.array_equal(y_on, dense)
+
+
+def test_lora_off_switch_b_zero_and_s_zero():
+    rng = np.random.default_rng(3)
+    x = O.round_bf16(rng.standard_normal((8, 16)))
+    W = O.round_bf16(0.02 * rng.standard_normal((12, 16)))
+    A = O.round_bf16(0.02 * rng.standard_normal((4, 16)))
+    B = np.zeros((12, 4))
+    y_off, y_on = O.dual_lora_linear(x, x, W, A, B, 2.0)
+    assert np.array_equal(y_off, y_on)
+    B = O.round_bf16(0.02 * rng.standard_normal((12, 4)))
+    y_off, y_on = O.dual_lora_linear(x, x, W, A, B, 0.0)
+    assert np.array_equal(y_off, y_on)
+    y_off2, y_on2 = O.dual_lora_linear(x, x, W, None, None, 2.0)
+    assert np.array_equal(y_off2, y_on2) and np.array_equal(y_off2, y_off)
+
+
+def test_lora_linear_in_s_and_bf16_output_rounding():
+    rng = np.random.default_rng(4)
+    x, W, A, B = _int_problem(rng, 4, 8, 5, 2)
+    y1 = O.dual_lora_linear(x, x, W, A, B, 1.0, out_bf16=False)[1]
+    y3 = O.dual_lora_linear(x, x, W, A, B, 3.0, out_bf16=False)[1]
+    y0 = O.dual_lora_linear(x, x, W, A, B, 0.0, out_bf16=False)[1]
+    assert np.array_equal(y3 - y0, 3.0 * (y1 - y0))
+    xr = rng.standard_normal((4, 8))
+    yb = O.dual_lora_linear(xr, xr, W, A, B, 1.0, out_bf16=True)[1]
+    assert np.array_equal(O.round_bf16(yb), yb)
+
+
+def test_lora_down_rounds_u_to_bf16():
+    x = np.array([[1.0, 1.0]])
+    A = np.array([[1.0, 2.0 ** -9]])  # s*(x A^T) = 1 + 2^-9: below half-ulp of bf16 at 1
+    u = O.lora_down(x, A, 1.0)
+    assert u[0, 0] == 1.0
+
+
+# ---------------------------------------------------------------- a4 log-softmax + gather
+
+
+def test_logsoftmax_hand_example():
+    g = _load("logsoftmax_gather.json")
+    base = np.log(np.array(g["z_is_log_of"], float))
+    z = np.stack([base, base + g["shift_row1"]])
+    logp, lse = O.log_softmax_gather(z, np.array(g["ids"]))
+    np.testing.assert_allclose(logp, g["logp"], rtol=0, atol=1e-14)
+    np.testing.assert_allclose(lse, g["lse"], rtol=0, atol=1e-14)
+
+
+def test_logsoftmax_matches_scipy_and_invariants():
+    rng = np.random.default_rng(5)
+    T, V = 16, 257
+    z = 3.0 * rng.standard_normal((T, V))
+    ids = rng.integers(0, V, size=T)
+    logp, lse = O.log_softmax_gather(z, ids)
+    ref = scipy.special.log_softmax(z, axis=1)[np.arange(T), ids]
+    np.testing.assert_allclose(logp, ref, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(lse, scipy.special.logsumexp(z, axis=1), rtol=1e-14)
+    # probabilities sum to one over the vocabulary
+    np.testing.assert_allclose(np.exp(z - lse[:, None]).sum(1), 1.0, rtol=1e-12)
+    # shift invariance per row
+    c = rng.standard_normal(T)[:, None] * 50
+    logp2, lse2 = O.log_softmax_gather(z + c, ids)
+    np.testing.assert_allclose(logp2, logp, atol=1e-10)
+    np.testing.assert_allclose(lse2, lse + c[:, 0], atol=1e-10)
+
+
+def test_logsoftmax_special_cases():
+    V = 1000
+    z = np.full((2, V), 7.25)
+    logp, _ = O.log_softmax_gather(z, np.array([0, V - 1]))
+    np.testing.assert_allclose(logp, -math.log(V), atol=1e-13)
+    logp1, lse1 = O.log_softmax_gather(np.array([[-3.5]]), np.array([0]))
+    assert logp1[0] == 0.0 and lse1[0] == -3.5
+    # brute force with exactly rounded sums on a tiny row
+    row = np.array([0.3, -1.2, 2.5, 0.0])
+    lse_bf = math.log(math.fsum(math.exp(v) for v in row))
+    lp, ls = O.log_softmax_gather(row[None], np.array([1]))
+    assert abs(ls[0] - lse_bf) < 1e-15 * 8 and abs(lp[0] - (row[1] - lse_bf)) < 1e-14
+
+
+# ---------------------------------------------------------------- a5 KL-penalised reward
+
+
+def test_kl_reward_hand_example():
+    g = _load("kl_reward.json")
+    r = O.kl_penalised_reward(np.array(g["logp_actor"]), np.array(g["logp_ref"]),
+                              g["lengths"], g["score"], g["beta"])
+    np.testing.assert_allclose(r, g["reward"], atol=1e-15)
+
+
+def test_kl_reward_lora_off_gives_score_only_and_masking():
+    rng = np.random.default_rng(6)
+    S, L, V = 3, 5, 11
+    z = rng.standard_normal((S * L, V))
+    ids = rng.integers(0, V, size=S * L)
+    lengths = np.array([5, 2, 0])
+    score = np.array([1.5, -0.25, 9.0])
+    out = O.token_logprobs_kl(z, z, ids, lengths, score, 0.1, S, L)
+    expect = np.zeros((S, L))
+    expect[0, 4] = 1.5
+    expect[1, 1] = -0.25
+    assert np.array_equal(out["reward"], expect)
+    assert np.all(out["logp_actor"][1, 2:] == 0) and np.all(out["logp_ref"][2] == 0)
+    # sign: actor more confident than reference at the sampled token -> negative penalty
+    za = z.copy()
+    za[np.arange(S * L), ids] += 2.0
+    out2 = O.token_logprobs_kl(za, z, ids, lengths, None, 0.1, S, L)
+    assert np.all(out2["reward"][0] < 0)
+
+
+# ---------------------------------------------------------------- a7 GAE
+
+
+def test_gae_hand_examples():
+    g = _load("gae.json")
+    for c in g["cases"]:
+        adv, ret = O.gae(np.array(c["rewards"]), np.array(c["values"]), c["lengths"],
+                         c["gamma"], c["lam"])
+        np.testing.assert_allclose(adv, c["advantages"], atol=1e-15)
+        np.testing.assert_allclose(ret, c["returns"], atol=1e-15)
+
+
+def _gae_problem(seed, S=4, L=37):
+    rng = np.random.default_rng(seed)
+    r = rng.standard_normal((S, L))
+    v = rng.standard_normal((S, L))
+    lengths = np.array([L, L // 2, 1, 0])[:S]
+    return r, v, lengths
+
+
+def test_gae_gamma_lambda_one_is_return_minus_value():
+    r, v, lengths = _gae_problem(7)
+    adv, ret = O.gae(r, v, lengths, 1.0, 1.0)
+    for s, n in enumerate(lengths):
+        for t in range(n):
+            assert abs(adv[s, t] - (math.fsum(r[s, t:n]) - v[s, t])) < 1e-12
+        assert np.all(adv[s, n:] == 0) and np.all(ret[s, n:] == 0)
+
+
+def test_gae_lambda_zero_is_td_residual_and_returns():
+    r, v, lengths = _gae_problem(8)
+    gamma = 0.9
+    adv, ret = O.gae(r, v, lengths, gamma, 0.0)
+    for s, n in enumerate(lengths):
+        for t in range(n):
+            vn = v[s, t + 1] if t + 1 < n else 0.0
+            assert abs(adv[s, t] - (r[s, t] + gamma * vn - v[s, t])) < 1e-14
+    np.testing.assert_allclose(ret, np.where(adv != 0, adv + v, 0.0), atol=1e-14)
+
+
+def test_gae_direct_sum_definition():
+    # A_t = sum_l (gamma lambda)^l delta_{t+l} (GAE as an exponentially weighted sum)
+    r, v, lengths = _gae_problem(9)
+    gamma, lam = 0.97, 0.95
+    adv, ret = O.gae(r, v, lengths, gamma, lam)
+    for s, n in enumerate(lengths):
+        delta = [r[s, t] + gamma * (v[s, t + 1] if t + 1 < n else 0.0) - v[s, t] for t in range(n)]
+        for t in range(n):
+            ref = math.fsum(((gamma * lam) ** l) * delta[t + l] for l in range(n - t))
+            assert abs(adv[s, t] - ref) < 1e-12
+            assert abs(ret[s, t] - (ref + v[s, t])) < 1e-12
+
+
+def test_gae_geometric_closed_form():
+    L, lam, c = 50, 0.95, 0.7
+    r = np.full((1, L), c)
+    adv, _ = O.gae(r, np.zeros((1, L)), [L], 1.0, lam)
+    for t in range(L):
+        n = L - t
+        assert abs(adv[0, t] - c * (1 - lam ** n) / (1 - lam)) < 1e-12
+
+
+# ---------------------------------------------------------------- a8 Llama pieces
+
+
+def test_rmsnorm_definition():
+    h = np.array([[3.0, 4.0], [0.0, 2.0]])
+    out = O.rmsnorm(h, np.array([1.0, 2.0]), 0.0)
+    np.testing.assert_allclose(out[0], [3 / math.sqrt(12.5), 8 / math.sqrt(12.5)], rtol=1e-15)
+    np.testing.assert_allclose(out[1], [0.0, 4 / math.sqrt(2.0)], rtol=1e-15)
+    out_eps = O.rmsnorm(np.zeros((1, 4)), np.ones(4), 1e-6)
+    assert np.all(out_eps == 0)
+
+
+def test_rope_against_rotation_matrices():
+    rng = np.random.default_rng(10)
+    T, H, D, theta = 5, 2, 8, 10000.0
+    x = rng.standard_normal((T, H, D))
+    pos = np.array([0, 1, 2, 7, 100])
+    y = O.rope(x, pos, theta)
+    half = D // 2
+    for t in range(T):
+        for h in range(H):
+            for i in range(half):
+                ang = pos[t] * theta ** (-2.0 * i / D)
+                R = np.array([[math.cos(ang), -math.sin(ang)], [math.sin(ang), math.cos(ang)]])
+                ref = R @ np.array([x[t, h, i], x[t, h, i + half]])
+                assert abs(y[t, h, i] - ref[0]) < 1e-12 and abs(y[t, h, i + half] - ref[1]) < 1e-12
+    np.testing.assert_allclose(y[0], x[0], atol=0)  # position 0 is the identity
+    # relative-position property: <rope(q, m), rope(k, n)> depends on m - n only
+    q = rng.standard_normal((1, 1, D))
+    k = rng.standard_normal((1, 1, D))
+    d1 = np.sum(O.rope(q, [9], theta) * O.rope(k, [4], theta))
+    d2 = np.sum(O.rope(q, [25], theta) * O.rope(k, [20], theta))
+    assert abs(d1 - d2) < 1e-12
+
+
+def test_causal_attention_brute_force_and_causality():
+    rng = np.random.default_rng(11)
+    T, H, D = 6, 2, 4
+    q, k, v = (rng.standard_normal((T, H, D)) for _ in range(3))
+    out = O.causal_attention(q, k, v)
+    for h in range(H):
+        for i in range(T):
+            sc = [sum(q[i, h, d] * k[j, h, d] for d in range(D)) / math.sqrt(D) for j in range(i + 1)]
+            mx = max(sc)
+            w = [math.exp(s_ - mx) for s_ in sc]
+            tot = math.fsum(w)
+            ref = [math.fsum(w[j] * v[j, h, d] for j in range(i + 1)) / tot for d in range(D)]
+            np.testing.assert_allclose(out[i, h], ref, atol=1e-12)
+    np.testing.assert_allclose(out[0], v[0], atol=1e-15)  # first query sees only itself
+    k2, v2 = k.copy(), v.copy()
+    k2[4:] += 10.0
+    v2[4:] -= 3.0
+    out2 = O.causal_attention(q, k2, v2)
+    np.testing.assert_allclose(out2[:4], out[:4], atol=0)
+
+
+def test_swiglu_against_scipy():
+    rng = np.random.default_rng(12)
+    g, u = rng.standard_normal(50) * 4, rng.standard_normal(50)
+    np.testing.assert_allclose(O.swiglu(g, u), g * scipy.special.expit(g) * u, rtol=1e-13)
+    assert O.swiglu(np.array([0.0]), np.array([5.0]))[0] == 0.0
+
+
+# ---------------------------------------------------------------- composition invariants
+
+
+def tiny_llama(seed=13, n_layers=2, d=32, H=4, F=48, V=64, r=4, zero_B=False):
+    rng = np.random.default_rng(seed)
+    bf = lambda *shape, std=0.02: O.round_bf16(std * rng.standard_normal(shape))  # noqa: E731
+    w = {
+        "embed": bf(V, d, std=1.0),
+        "wq": bf(n_layers, d, d), "wk": bf(n_layers, d, d), "wv": bf(n_layers, d, d),
+        "wo": bf(n_layers, d, d), "wg": bf(n_layers, F, d), "wu": bf(n_layers, F, d),
+        "wd": bf(n_layers, d, F),
+        "norm1": np.ones((n_layers, d)), "norm2": np.ones((n_layers, d)),
+        "final_norm": np.ones(d), "lm_head": bf(V, d, std=0.2), "w_rm": bf(d, std=0.2),
+        "lora": {},
+    }
+    dims = {"wq": (d, d), "wv": (d, d), "wg": (F, d), "wu": (F, d), "wd": (d, F)}
+    for name, (n_out, n_in) in dims.items():
+        A = bf(n_layers, r, n_in, std=0.2)
+        B = np.zeros((n_layers, n_out, r)) if zero_B else bf(n_layers, n_out, r, std=0.2)
+        w["lora"][name] = (A, B)
+    cfg = {"d": d, "n_heads": H, "eps": 1e-6, "lora_scale": 2.0, "rope_theta": 10000.0,
+           "n_layers": n_layers}
+    return w, cfg
+
+
+def test_llama_score_lora_off_invariants():
+    w, cfg = tiny_llama(zero_B=True)
+    rng = np.random.default_rng(14)
+    ids = rng.integers(0, 64, size=12)
+    out = O.llama_score(w, ids, 4, cfg)
+    assert np.array_equal(out["h_off"], out["h_on"])
+    assert np.array_equal(out["logp_actor"], out["logp_ref"])
+    expect_r = np.zeros(8)
+    expect_r[-1] = out["score"]
+    assert np.array_equal(out["reward"], expect_r)
+    adv, ret = O.gae(out["reward"][None], out["values"][None], [8], 1.0, 0.95)
+    np.testing.assert_allclose(out["advantages"], adv[0], atol=0)
+
+
+def test_llama_score_causal_and_lora_changes_actor_only():
+    w, cfg = tiny_llama()
+    rng = np.random.default_rng(15)
+    ids = rng.integers(0, 64, size=12)
+    out = O.llama_score(w, ids, 4, cfg)
+    ids2 = ids.copy()
+    ids2[-1] = (ids2[-1] + 1) % 64
+    out2 = O.llama_score(w, ids2, 4, cfg)
+    # hidden states before the last position do not see the changed last token
+    np.testing.assert_allclose(out2["h_off"][:-1], out["h_off"][:-1], atol=0)
+    np.testing.assert_allclose(out2["h_on"][:-1], out["h_on"][:-1], atol=0)
+    w0, _ = tiny_llama(zero_B=True)
+    ref0 = O.llama_score(w0, ids, 4, cfg)
+    # turning LoRA on changes the actor stream but never the reference stream
+    np.testing.assert_allclose(out["logp_ref"], ref0["logp_ref"], atol=0)
+    assert np.max(np.abs(out["logp_actor"] - ref0["logp_actor"])) > 1e-6
