@@ -1,0 +1,206 @@
+// C-ABI entry points of libhydra (declared in include/hydra.h): argument validation on
+// the host, then kernel launches on the caller's stream.
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/hydra.h"
+#include "kernels.h"
+
+namespace {
+
+// The library's device error word (one per device that loaded the library).
+__device__ int g_hydra_err = 0;
+
+constexpr int kMaxDevices = 64;
+int* g_err_ptr[kMaxDevices] = {nullptr};
+
+int* device_err_ptr() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  if (g_err_ptr[dev] == nullptr) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_hydra_err) != cudaSuccess) return nullptr;
+    g_err_ptr[dev] = static_cast<int*>(p);
+  }
+  return g_err_ptr[dev];
+}
+
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+inline size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// u_given: `workspace` already holds u = s x_on A^T (hydra_dual_linear); A is unused.
+hydra_status lora_linear_impl(const void* x_off, const void* x_on, int64_t M, int64_t K,
+                              int64_t N, const void* W, const void* A, const void* B, int64_t r,
+                              float s, void* y_off, void* y_on, int out_dtype, void* workspace,
+                              size_t workspace_bytes, int algo, void* stream,
+                              bool u_given = false) {
+  if (x_off == nullptr || W == nullptr) return HYDRA_ERR_NULL;
+  if (y_off == nullptr && y_on == nullptr) return HYDRA_ERR_NULL;
+  if (algo < 0 || algo > 2) return HYDRA_ERR_RANGE;
+  if (out_dtype != HYDRA_BF16 && out_dtype != HYDRA_F32) return HYDRA_ERR_RANGE;
+  if (M < 0 || K < 8 || N < 8 || M >= (1LL << 31) || K >= (1LL << 31) || N >= (1LL << 31))
+    return HYDRA_ERR_SHAPE;
+  if (K % 8 != 0 || N % 8 != 0) return HYDRA_ERR_ALIGN;
+  if (r < 0 || r > 256) return HYDRA_ERR_SHAPE;
+  if (r > 0 && r % 8 != 0) return HYDRA_ERR_ALIGN;
+  const bool shared_x = (x_on == nullptr || x_on == x_off);
+  if (!aligned16(x_off) || (!shared_x && !aligned16(x_on)) || !aligned16(W) ||
+      !aligned16(y_off) || !aligned16(y_on))
+    return HYDRA_ERR_ALIGN;
+  const bool lora = r > 0 && y_on != nullptr;
+  if (lora) {
+    if ((!u_given && A == nullptr) || B == nullptr) return HYDRA_ERR_NULL;
+    if ((!u_given && !aligned16(A)) || !aligned16(B)) return HYDRA_ERR_ALIGN;
+    if (workspace == nullptr) return u_given ? HYDRA_ERR_NULL : HYDRA_ERR_WORKSPACE;
+    if (!aligned16(workspace)) return HYDRA_ERR_ALIGN;
+    if (workspace_bytes < hydra_lora_linear_workspace_size(M, r)) return HYDRA_ERR_WORKSPACE;
+  }
+  const int64_t rows = shared_x ? M : 2 * M;
+  if (algo == 2 && rows > hydra::kGemvMaxRows) return HYDRA_ERR_SHAPE;
+  if (M == 0) return HYDRA_OK;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int* err = device_err_ptr();
+  if (err == nullptr) return HYDRA_ERR_CUDA;
+
+  const void* xo = shared_x ? x_off : x_on;
+  if (lora && !u_given) {
+    if (hydra::launch_lora_down(xo, M, K, A, r, s, workspace, st) != 0) return HYDRA_ERR_CUDA;
+  }
+  hydra::GemmArgs g;
+  g.x_off = x_off;
+  g.x_on = xo;
+  g.M = M;
+  g.K = K;
+  g.N = N;
+  g.W = W;
+  g.u = lora ? workspace : nullptr;
+  g.B = lora ? B : nullptr;
+  g.r = lora ? r : 0;
+  g.shared_x = shared_x;
+  g.y_off = y_off;
+  g.y_on = y_on;
+  g.out_f32 = out_dtype == HYDRA_F32 ? 1 : 0;
+  g.err = err;
+  const bool use_gemv = (algo == 2) || (algo == 0 && rows <= hydra::kGemvMaxRows);
+  const int rc = use_gemv ? hydra::launch_dual_lora_gemv(g, st) : hydra::launch_dual_lora_gemm_tc(g, st);
+  return rc == 0 ? HYDRA_OK : HYDRA_ERR_CUDA;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* hydra_status_string(int status) {
+  switch (status) {
+    case HYDRA_OK: return "HYDRA_OK";
+    case HYDRA_ERR_NULL: return "HYDRA_ERR_NULL: a required pointer is NULL";
+    case HYDRA_ERR_SHAPE: return "HYDRA_ERR_SHAPE: size out of the supported range";
+    case HYDRA_ERR_ALIGN: return "HYDRA_ERR_ALIGN: pointer or row length not 16-byte aligned";
+    case HYDRA_ERR_RANGE: return "HYDRA_ERR_RANGE: scalar or enum argument out of range";
+    case HYDRA_ERR_CUDA: return "HYDRA_ERR_CUDA: CUDA runtime or driver call failed";
+    case HYDRA_ERR_TIMEOUT: return "HYDRA_ERR_TIMEOUT: bounded device wait expired";
+    case HYDRA_ERR_WORKSPACE: return "HYDRA_ERR_WORKSPACE: workspace missing or too small";
+    case HYDRA_ERR_DEVICE: return "HYDRA_ERR_DEVICE: kernel found a bad token id or length";
+    default: return "unknown hydra status";
+  }
+}
+
+int hydra_abi_version(void) { return 1; }
+
+hydra_status hydra_device_error(int32_t* code_out, int clear) {
+  if (code_out == nullptr) return HYDRA_ERR_NULL;
+  int v = 0;
+  if (cudaDeviceSynchronize() != cudaSuccess) return HYDRA_ERR_CUDA;
+  if (cudaMemcpyFromSymbol(&v, g_hydra_err, sizeof(int)) != cudaSuccess) return HYDRA_ERR_CUDA;
+  if (clear) {
+    const int zero = 0;
+    if (cudaMemcpyToSymbol(g_hydra_err, &zero, sizeof(int)) != cudaSuccess) return HYDRA_ERR_CUDA;
+  }
+  *code_out = v;
+  return HYDRA_OK;
+}
+
+size_t hydra_lora_linear_workspace_size(int64_t M, int64_t r) {
+  if (M <= 0 || r <= 0) return 0;
+  return round_up(static_cast<size_t>(M) * static_cast<size_t>(r) * 2, 256);
+}
+
+hydra_status hydra_lora_down(const void* x_on, int64_t M, int64_t K, const void* A, int64_t r,
+                             float s, void* u, void* stream) {
+  if (x_on == nullptr || A == nullptr || u == nullptr) return HYDRA_ERR_NULL;
+  if (M < 0 || K < 8 || r < 1 || r > 256 || M >= (1LL << 31) || K >= (1LL << 31))
+    return HYDRA_ERR_SHAPE;
+  if (K % 8 != 0 || r % 8 != 0) return HYDRA_ERR_ALIGN;
+  if (!aligned16(x_on) || !aligned16(A) || !aligned16(u)) return HYDRA_ERR_ALIGN;
+  if (M == 0) return HYDRA_OK;
+  return hydra::launch_lora_down(x_on, M, K, A, r, s, u, static_cast<cudaStream_t>(stream)) == 0
+             ? HYDRA_OK
+             : HYDRA_ERR_CUDA;
+}
+
+hydra_status hydra_lora_linear(const void* x_off, const void* x_on, int64_t M, int64_t K,
+                               int64_t N, const void* W, const void* A, const void* B, int64_t r,
+                               float s, void* y_off, void* y_on, int out_dtype, void* workspace,
+                               size_t workspace_bytes, void* stream) {
+  return lora_linear_impl(x_off, x_on, M, K, N, W, A, B, r, s, y_off, y_on, out_dtype, workspace,
+                          workspace_bytes, 0, stream);
+}
+
+hydra_status hydra_lora_linear_algo(const void* x_off, const void* x_on, int64_t M, int64_t K,
+                                    int64_t N, const void* W, const void* A, const void* B,
+                                    int64_t r, float s, void* y_off, void* y_on, int out_dtype,
+                                    void* workspace, size_t workspace_bytes, int algo,
+                                    void* stream) {
+  return lora_linear_impl(x_off, x_on, M, K, N, W, A, B, r, s, y_off, y_on, out_dtype, workspace,
+                          workspace_bytes, algo, stream);
+}
+
+hydra_status hydra_dual_linear(const void* x_off, const void* x_on, int64_t M, int64_t K,
+                               int64_t N, const void* W, const void* u, const void* B, int64_t r,
+                               void* y_off, void* y_on, int out_dtype, int algo, void* stream) {
+  return lora_linear_impl(x_off, x_on, M, K, N, W, nullptr, B, r, 1.0f, y_off, y_on, out_dtype,
+                          const_cast<void*>(u), hydra_lora_linear_workspace_size(M, r), algo,
+                          stream, true);
+}
+
+hydra_status hydra_token_logprobs_kl(const void* logits_actor, const void* logits_ref,
+                                     int logits_dtype, int64_t S, int64_t L, int64_t V, int64_t ld,
+                                     const int32_t* ids, const int32_t* lengths,
+                                     const float* seq_score, float beta, float* logp_actor,
+                                     float* logp_ref, float* reward_tok, float* lse_actor,
+                                     float* lse_ref, void* stream) {
+  if (logits_dtype != HYDRA_F32 && logits_dtype != HYDRA_BF16) return HYDRA_ERR_RANGE;
+  if (S < 0 || L < 0 || V < 1 || V >= (1LL << 31) || ld < V || S * L >= (1LL << 31))
+    return HYDRA_ERR_SHAPE;
+  if (S == 0 || L == 0) return HYDRA_OK;
+  if (logits_actor == nullptr || logits_ref == nullptr || ids == nullptr ||
+      logp_actor == nullptr || logp_ref == nullptr || reward_tok == nullptr)
+    return HYDRA_ERR_NULL;
+  int* err = device_err_ptr();
+  if (err == nullptr) return HYDRA_ERR_CUDA;
+  return hydra::launch_token_logprobs_kl(logits_actor, logits_ref, logits_dtype == HYDRA_BF16, S, L,
+                                         V, ld, ids, lengths, seq_score, beta, logp_actor, logp_ref,
+                                         reward_tok, lse_actor, lse_ref, err,
+                                         static_cast<cudaStream_t>(stream)) == 0
+             ? HYDRA_OK
+             : HYDRA_ERR_CUDA;
+}
+
+hydra_status ppo_gae(const float* rewards, const float* values, const int32_t* lengths, int64_t S,
+                     int64_t L, float gamma, float lam, float* advantages, float* returns,
+                     void* stream) {
+  if (S < 0 || L < 0 || L > hydra::kGaeMaxL || S * L >= (1LL << 40) || S >= (1LL << 31))
+    return HYDRA_ERR_SHAPE;
+  if (S == 0 || L == 0) return HYDRA_OK;
+  if (rewards == nullptr || values == nullptr || advantages == nullptr || returns == nullptr)
+    return HYDRA_ERR_NULL;
+  int* err = device_err_ptr();
+  if (err == nullptr) return HYDRA_ERR_CUDA;
+  return hydra::launch_gae(rewards, values, lengths, S, L, gamma, lam, advantages, returns, err,
+                           static_cast<cudaStream_t>(stream)) == 0
+             ? HYDRA_OK
+             : HYDRA_ERR_CUDA;
+}
+
+}  // extern "C"

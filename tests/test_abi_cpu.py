@@ -1,0 +1,87 @@
+"""The C-ABI library without a GPU: it builds for sm_103a, loads, exports every function
+include/hydra.h declares, and rejects bad arguments on the host before any CUDA call."""
+import ctypes
+
+import pytest
+
+from paper_2309_00754_gb300 import build as B
+from paper_2309_00754_gb300 import hydra as H
+
+
+@pytest.fixture(scope="module")
+def lib():
+    B.build()
+    return H.load()
+
+
+def test_exports_every_declared_function(lib):
+    names = H.header_functions()
+    assert "hydra_lora_linear" in names and "hydra_token_logprobs_kl" in names and "ppo_gae" in names
+    for n in names:
+        assert hasattr(lib, n), f"libhydra.so does not export {n}"
+    assert set(names) <= set(H._SIGNATURES), "binding lacks a signature for a declared function"
+
+
+def test_status_strings_and_version(lib):
+    assert H.status_string(0) == "HYDRA_OK"
+    for code in range(1, 9):
+        assert H.status_string(code).startswith("HYDRA_ERR_")
+    assert lib.hydra_abi_version() == 1
+
+
+def test_workspace_size(lib):
+    assert H.lora_linear_workspace_size(0, 16) == 0
+    assert H.lora_linear_workspace_size(100, 0) == 0
+    assert H.lora_linear_workspace_size(2048, 16) == 2048 * 16 * 2
+    assert H.lora_linear_workspace_size(3, 8) == 256
+
+
+FAKE = 1 << 20  # a 16-byte aligned non-null value; never dereferenced on these paths
+
+
+def _lin(lib, **kw):
+    a = dict(x_off=FAKE, x_on=None, M=64, K=64, N=64, W=FAKE, A=None, B=None, r=0, s=2.0,
+             y_off=FAKE, y_on=None, dt=0, ws=None, wsb=0, algo=0)
+    a.update(kw)
+    return lib.hydra_lora_linear_algo(a["x_off"], a["x_on"], a["M"], a["K"], a["N"], a["W"], a["A"],
+                                      a["B"], a["r"], a["s"], a["y_off"], a["y_on"], a["dt"],
+                                      a["ws"], a["wsb"], a["algo"], None)
+
+
+def test_lora_linear_argument_errors(lib):
+    assert _lin(lib, x_off=None) == 1
+    assert _lin(lib, W=None) == 1
+    assert _lin(lib, y_off=None, y_on=None) == 1
+    assert _lin(lib, K=60) == 3          # K % 8
+    assert _lin(lib, N=12) == 3          # N % 8
+    assert _lin(lib, K=0) == 2
+    assert _lin(lib, M=-1) == 2
+    assert _lin(lib, M=1 << 31) == 2
+    assert _lin(lib, r=300, A=FAKE, B=FAKE, y_on=FAKE) == 2
+    assert _lin(lib, r=12, A=FAKE, B=FAKE, y_on=FAKE) == 3
+    assert _lin(lib, r=16, y_on=FAKE) == 1                      # LoRA without A/B
+    assert _lin(lib, r=16, A=FAKE, B=FAKE, y_on=FAKE) == 7      # no workspace
+    assert _lin(lib, r=16, A=FAKE, B=FAKE, y_on=FAKE, ws=FAKE, wsb=100) == 7
+    assert _lin(lib, x_off=FAKE + 8) == 3                       # misaligned pointer
+    assert _lin(lib, dt=7) == 4
+    assert _lin(lib, algo=3) == 4
+    assert _lin(lib, algo=2, M=9, x_on=FAKE * 2) == 2           # GEMV takes <= 16 rows
+    assert _lin(lib, M=0) == 0                                  # empty: no launch
+
+
+def test_logprobs_and_gae_argument_errors(lib):
+    f = lib.hydra_token_logprobs_kl
+    assert f(FAKE, FAKE, 5, 1, 1, 10, 10, FAKE, None, None, 0.1, FAKE, FAKE, FAKE, None, None, None) == 4
+    assert f(FAKE, FAKE, 1, 1, 1, 10, 9, FAKE, None, None, 0.1, FAKE, FAKE, FAKE, None, None, None) == 2
+    assert f(FAKE, FAKE, 1, 1, 1, 0, 0, FAKE, None, None, 0.1, FAKE, FAKE, FAKE, None, None, None) == 2
+    assert f(None, FAKE, 1, 1, 1, 10, 10, FAKE, None, None, 0.1, FAKE, FAKE, FAKE, None, None, None) == 1
+    assert f(FAKE, FAKE, 1, 0, 4, 10, 10, FAKE, None, None, 0.1, FAKE, FAKE, FAKE, None, None, None) == 0
+    g = lib.ppo_gae
+    assert g(FAKE, FAKE, None, 2, 20000, 1.0, 0.95, FAKE, FAKE, None) == 2
+    assert g(FAKE, FAKE, None, -1, 4, 1.0, 0.95, FAKE, FAKE, None) == 2
+    assert g(None, FAKE, None, 2, 4, 1.0, 0.95, FAKE, FAKE, None) == 1
+    assert g(FAKE, FAKE, None, 0, 4, 1.0, 0.95, FAKE, FAKE, None) == 0
+    assert lib.hydra_lora_down(None, 4, 8, FAKE, 8, 1.0, FAKE, None) == 1
+    assert lib.hydra_lora_down(FAKE, 4, 8, FAKE, 4, 1.0, FAKE, None) == 3
+    code = ctypes.c_int32(0)
+    assert lib.hydra_device_error(None, 0) == 1

@@ -1,0 +1,269 @@
+"""GPU parity: the CUDA path, called through the C-ABI, against the fp64 oracle on the same
+seeded inputs. Small cases compare every element (several tiles, ragged tails); the
+full-size workloads compare a seeded sample of rows, which the oracle computes one by
+one (outputs are row-local, so the sample is an exact check of those rows)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2309_00754_gb300 import build as B
+from paper_2309_00754_gb300 import hydra as H
+from paper_2309_00754_gb300 import synth
+from tests.helpers import (TOL_GAE, TOL_LINEAR, TOL_LOGP, assert_abs, assert_rel, dev_bf16,
+                           dev_f32, dev_i32, f64, host_f64)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    B.build()
+    L = H.load()
+    H.device_error(clear=True)
+    yield L
+    assert H.device_error(clear=True) == 0
+
+
+def sample_rows(seed, M, n=64):
+    rows = set(int(v) for v in synth.randint(seed, (n - 2,), 0, M))
+    rows.update({0, M - 1})
+    return np.array(sorted(rows))
+
+
+# ------------------------------------------------------------------ GAE (a7)
+
+
+@pytest.mark.parametrize("S,L,seed", [(4, 64, 1), (4, 512, 4), (64, 512, 5), (3, 37, 7),
+                                      (5, 1000, 8), (2, 1, 9), (7, 33, 10)])
+def test_gae_parity(S, L, seed):
+    r = synth.normal_f32(synth.tensor_seed(seed, 1), (S, L))
+    v = synth.normal_f32(synth.tensor_seed(seed, 2), (S, L))
+    lengths = synth.randint(synth.tensor_seed(seed, 3), (S,), 0, L + 1)
+    lengths[0] = L
+    if S > 2:
+        lengths[1] = 0
+        lengths[2] = min(1, L)
+    adv = torch.empty(S, L, device="cuda")
+    ret = torch.empty(S, L, device="cuda")
+    H.ppo_gae(dev_f32(r), dev_f32(v), dev_i32(lengths), 1.0, 0.95, adv, ret)
+    a_ref, r_ref = O.gae(r.astype(np.float64), v.astype(np.float64), lengths, 1.0, 0.95)
+    assert_rel(host_f64(adv), a_ref, TOL_GAE, "advantages")
+    assert_rel(host_f64(ret), r_ref, TOL_GAE, "returns")
+
+
+def test_gae_no_lengths_and_discount():
+    S, L = 3, 100
+    r = synth.normal_f32(71, (S, L))
+    v = synth.normal_f32(72, (S, L))
+    adv = torch.empty(S, L, device="cuda")
+    ret = torch.empty(S, L, device="cuda")
+    H.ppo_gae(dev_f32(r), dev_f32(v), None, 0.99, 0.9, adv, ret)
+    a_ref, r_ref = O.gae(r.astype(np.float64), v.astype(np.float64), None, 0.99, 0.9)
+    assert_rel(host_f64(adv), a_ref, TOL_GAE, "advantages")
+    assert_rel(host_f64(ret), r_ref, TOL_GAE, "returns")
+
+
+def test_gae_large_batch_sampled():
+    S, L = 65536, 512
+    r = synth.normal_f32(81, (S, L))
+    v = synth.normal_f32(82, (S, L))
+    lengths = synth.randint(83, (S,), 64, 513)
+    adv = torch.empty(S, L, device="cuda")
+    ret = torch.empty(S, L, device="cuda")
+    H.ppo_gae(dev_f32(r), dev_f32(v), dev_i32(lengths), 1.0, 0.95, adv, ret)
+    rows = sample_rows(84, S)
+    a_ref, r_ref = O.gae(r[rows].astype(np.float64), v[rows].astype(np.float64), lengths[rows], 1.0, 0.95)
+    assert_rel(host_f64(adv[rows]), a_ref, TOL_GAE, "advantages")
+    assert_rel(host_f64(ret[rows]), r_ref, TOL_GAE, "returns")
+
+
+# ------------------------------------------------------------------ log-probs + KL (a4, a5)
+
+
+def _logprobs_case(S, L, V, seed, dtype=torch.float32, ld=None, score=True, lengths=True):
+    T = S * L
+    ld = V if ld is None else ld
+    za = synth.normal_f32(synth.tensor_seed(seed, 1), (T, ld), 1.3)
+    zr = synth.normal_f32(synth.tensor_seed(seed, 2), (T, ld), 1.3)
+    ids = synth.randint(synth.tensor_seed(seed, 3), (T,), 0, V)
+    lens = synth.randint(synth.tensor_seed(seed, 4), (S,), 0, L + 1) if lengths else None
+    if lens is not None:
+        lens[0] = L
+    sc = synth.normal_f32(synth.tensor_seed(seed, 5), (S,)) if score else None
+    if dtype == torch.bfloat16:
+        za_d = dev_bf16(synth.f32_to_bf16_bits(za))
+        zr_d = dev_bf16(synth.f32_to_bf16_bits(zr))
+        za64, zr64 = host_f64(za_d), host_f64(zr_d)
+    else:
+        za_d, zr_d = dev_f32(za), dev_f32(zr)
+        za64, zr64 = za.astype(np.float64), zr.astype(np.float64)
+    outs = [torch.full((T,), 7.0, device="cuda") for _ in range(5)]
+    H.hydra_token_logprobs_kl(za_d[:, :V], zr_d[:, :V], dev_i32(ids),
+                              None if lens is None else dev_i32(lens),
+                              None if sc is None else dev_f32(sc), 0.1, S, L, *outs)
+    ref = O.token_logprobs_kl(za64[:, :V], zr64[:, :V], ids, lens, sc, 0.1, S, L)
+    names = ["logp_actor", "logp_ref", "reward", "lse_actor", "lse_ref"]
+    for o, n in zip(outs, names):
+        assert_abs(host_f64(o).reshape(S, L), ref[n], TOL_LOGP, n)
+
+
+@pytest.mark.parametrize("S,L,V,seed", [(4, 64, 4096, 11), (3, 5, 1000, 12), (2, 7, 1, 13),
+                                        (2, 9, 4099, 14), (1, 3, 3, 15)])
+def test_logprobs_kl_parity(S, L, V, seed):
+    _logprobs_case(S, L, V, seed)
+
+
+def test_logprobs_kl_strided_bf16_and_no_score():
+    _logprobs_case(3, 8, 4000, 16, ld=4096)
+    _logprobs_case(3, 8, 4001, 17, ld=4003, score=False, lengths=False)
+    _logprobs_case(2, 16, 32000, 18, dtype=torch.bfloat16)
+
+
+def test_logprobs_kl_bad_id_flags_error():
+    S, L, V = 1, 4, 64
+    z = dev_f32(synth.normal_f32(19, (S * L, V)))
+    ids = dev_i32(np.array([0, 64, 3, -1], dtype=np.int32))
+    outs = [torch.zeros(S * L, device="cuda") for _ in range(3)]
+    H.hydra_token_logprobs_kl(z, z, ids, None, None, 0.1, S, L, *outs)
+    code = H.device_error(clear=True)
+    assert code == 0x201
+    la = outs[0].cpu().numpy()
+    assert np.isfinite(la[0]) and np.isnan(la[1]) and np.isnan(la[3])
+
+
+# ------------------------------------------------------------------ dual LoRA linear (a1-a3)
+
+
+def _linear_problem(M, K, N, r, seed, std_x=1.0):
+    x = synth.normal_bf16(synth.tensor_seed(seed, 1), (M, K), std_x)
+    x2 = synth.normal_bf16(synth.tensor_seed(seed, 2), (M, K), std_x)
+    W = synth.normal_bf16(synth.tensor_seed(seed, 3), (N, K), 0.02)
+    A = synth.normal_bf16(synth.tensor_seed(seed, 4), (max(r, 1), K), 0.02)[:r]
+    Bm = synth.normal_bf16(synth.tensor_seed(seed, 5), (N, max(r, 1)), 0.02)[:, :r]
+    return x, x2, W, A, Bm
+
+
+def _run_linear(x_off, x_on, W, A, Bm, s, out=torch.bfloat16, algo=0, want=(True, True)):
+    M, K = x_off.shape
+    N = W.shape[0]
+    r = 0 if A is None else A.shape[0]
+    y_off = torch.full((M, N), float("nan"), dtype=out, device="cuda") if want[0] else None
+    y_on = torch.full((M, N), float("nan"), dtype=out, device="cuda") if want[1] else None
+    ws = torch.empty(max(1, H.lora_linear_workspace_size(M, r)), dtype=torch.uint8, device="cuda")
+    H.hydra_lora_linear(x_off, x_on, W, A, Bm, s, y_off, y_on, ws, algo=algo)
+    return y_off, y_on
+
+
+@pytest.mark.parametrize("M,K,N,r,shared,algo", [
+    (256, 512, 512, 8, True, 1),      # config-1 first linear
+    (300, 328, 520, 16, True, 1),     # ragged M, K (OOB k-block), N tail
+    (300, 328, 520, 16, False, 1),    # stacked streams
+    (129, 64, 256, 64, True, 1),
+    (130, 1024, 768, 72, False, 1),   # two LoRA k-blocks
+    (200, 512, 264, 128, True, 1),
+    (64, 256, 512, 0, True, 1),       # no LoRA
+    (96, 256, 512, 0, False, 1),
+    (1, 4096, 4096, 16, True, 2),     # decode GEMV shapes
+    (4, 4096, 1032, 16, True, 2),
+    (8, 1024, 520, 8, False, 2),
+    (16, 512, 512, 64, True, 2),
+    (3, 520, 72, 16, True, 0),
+])
+def test_lora_linear_parity(M, K, N, r, shared, algo):
+    x, x2, W, A, Bm = _linear_problem(M, K, N, r, seed=M + K + N + r)
+    xo = x if shared else x2
+    y_off, y_on = _run_linear(dev_bf16(x), None if shared else dev_bf16(x2), dev_bf16(W),
+                              dev_bf16(A) if r else None, dev_bf16(Bm) if r else None, 2.0,
+                              algo=algo)
+    ref_off, ref_on = O.dual_lora_linear(f64(x), f64(xo), f64(W), f64(A) if r else None,
+                                         f64(Bm) if r else None, 2.0)
+    assert_rel(host_f64(y_off), ref_off, TOL_LINEAR, "y_off")
+    assert_rel(host_f64(y_on), ref_on, TOL_LINEAR, "y_on")
+
+
+def test_lora_linear_fp32_out_and_single_outputs():
+    M, K, N, r = 200, 256, 264, 16
+    x, x2, W, A, Bm = _linear_problem(M, K, N, r, seed=21)
+    d = [dev_bf16(t) for t in (x, x2, W, A, Bm)]
+    ref_off, ref_on = O.dual_lora_linear(f64(x), f64(x2), f64(W), f64(A), f64(Bm), 2.0, out_bf16=False)
+    y_off, y_on = _run_linear(d[0], d[1], d[2], d[3], d[4], 2.0, out=torch.float32)
+    assert_rel(host_f64(y_off), ref_off, 1e-4, "y_off fp32")
+    assert_rel(host_f64(y_on), ref_on, 1e-4, "y_on fp32")
+    _, only_on = _run_linear(d[0], d[1], d[2], d[3], d[4], 2.0, out=torch.float32, want=(False, True))
+    assert torch.equal(only_on, y_on)
+    only_off, _ = _run_linear(d[0], d[0], d[2], d[3], d[4], 2.0, out=torch.float32, want=(True, False))
+    ref_off_s, _ = O.dual_lora_linear(f64(x), f64(x), f64(W), f64(A), f64(Bm), 2.0, out_bf16=False)
+    assert_rel(host_f64(only_off), ref_off_s, 1e-4, "y_off only")
+
+
+@pytest.mark.parametrize("algo", [1, 2])
+def test_lora_off_switch_is_bitwise(algo):
+    # §3 Dynamic LoRA: with B = 0 (or s = 0) the LoRA-on output equals the LoRA-off output
+    M = 16 if algo == 2 else 200
+    K, N, r = 512, 264, 16
+    x, _, W, A, _ = _linear_problem(M, K, N, r, seed=22)
+    Bz = torch.zeros(N, r, dtype=torch.bfloat16, device="cuda")
+    y_off, y_on = _run_linear(dev_bf16(x), None, dev_bf16(W), dev_bf16(A), Bz, 2.0, algo=algo)
+    assert torch.equal(y_off, y_on)
+    Bm = dev_bf16(synth.normal_bf16(23, (N, r), 0.02))
+    y_off2, y_on2 = _run_linear(dev_bf16(x), None, dev_bf16(W), dev_bf16(A), Bm, 0.0, algo=algo)
+    assert torch.equal(y_off2, y_on2) and torch.equal(y_off2, y_off)
+
+
+def test_stacked_equals_separate_calls_bitwise():
+    M, K, N, r = 260, 384, 520, 16
+    x, x2, W, A, Bm = _linear_problem(M, K, N, r, seed=24)
+    d = [dev_bf16(t) for t in (x, x2, W, A, Bm)]
+    st_off, st_on = _run_linear(d[0], d[1], d[2], d[3], d[4], 2.0)
+    sep_off, _ = _run_linear(d[0], None, d[2], d[3], d[4], 2.0)
+    _, sep_on = _run_linear(d[1], None, d[2], d[3], d[4], 2.0)
+    assert torch.equal(st_off, sep_off)
+    assert torch.equal(st_on, sep_on)
+
+
+def test_gemv_and_tensor_core_kernel_agree():
+    M, K, N, r = 16, 2048, 1024, 16
+    x, _, W, A, Bm = _linear_problem(M, K, N, r, seed=25)
+    d = [dev_bf16(t) for t in (x, W, A, Bm)]
+    a = _run_linear(d[0], None, d[1], d[2], d[3], 2.0, algo=1)
+    b = _run_linear(d[0], None, d[1], d[2], d[3], 2.0, algo=2)
+    for u, v in zip(a, b):
+        assert_rel(host_f64(u), host_f64(v), TOL_LINEAR, "gemv vs tcgen05")
+
+
+def test_lora_down_parity():
+    M, K, r = 300, 4096, 64
+    x, _, _, A, _ = _linear_problem(M, K, 8, r, seed=26)
+    u = torch.empty(M, r, dtype=torch.bfloat16, device="cuda")
+    H.hydra_lora_down(dev_bf16(x), dev_bf16(A), 2.0, u)
+    ref = O.lora_down(f64(x), f64(A), 2.0)
+    assert_rel(host_f64(u), ref, TOL_LINEAR, "u")
+
+
+# ------------------------------------------------------------------ full-size workloads
+
+
+@pytest.mark.parametrize("K,N", [(4096, 4096), (4096, 11008), (11008, 4096)])
+@pytest.mark.parametrize("r", [8, 16, 64])
+def test_projection_sweep_sampled(K, N, r):
+    """Llama-7B projection shapes at M = 2048 tokens (batch 4 x 512), shared input."""
+    M = 2048
+    x, _, W, A, Bm = _linear_problem(M, K, N, r, seed=2000 + K // 64 + N // 64 + r)
+    y_off, y_on = _run_linear(dev_bf16(x), None, dev_bf16(W), dev_bf16(A), dev_bf16(Bm), 2.0)
+    rows = sample_rows(2100 + r, M)
+    ref_off, ref_on = O.dual_lora_linear(f64(x[rows]), f64(x[rows]), f64(W), f64(A), f64(Bm), 2.0)
+    assert_rel(host_f64(y_off[rows]), ref_off, TOL_LINEAR, "y_off")
+    assert_rel(host_f64(y_on[rows]), ref_on, TOL_LINEAR, "y_on")
+
+
+@pytest.mark.parametrize("M", [1, 4, 8, 16])
+def test_decode_gemv_sampled(M):
+    """Decode-shaped inputs through the 4096 -> 32000 LM head and the 11008 -> 4096 down."""
+    for K, N in ((4096, 32000), (11008, 4096)):
+        x, _, W, A, Bm = _linear_problem(M, K, N, 16, seed=3000 + M + N)
+        y_off, y_on = _run_linear(dev_bf16(x), None, dev_bf16(W), dev_bf16(A), dev_bf16(Bm), 2.0)
+        ref_off, ref_on = O.dual_lora_linear(f64(x), f64(x), f64(W), f64(A), f64(Bm), 2.0)
+        assert_rel(host_f64(y_off), ref_off, TOL_LINEAR, "y_off")
+        assert_rel(host_f64(y_on), ref_on, TOL_LINEAR, "y_on")
