@@ -132,6 +132,30 @@ hydra_status hydra_lora_linear_algo(const void* x_off, const void* x_on, int64_t
                                     void* workspace, size_t workspace_bytes, int algo,
                                     void* stream);
 
+/* Largest M * r that hydra_lora_linear_noalloc accepts (u elements, bf16: 4 MiB). */
+#define HYDRA_NOALLOC_MAX_U_ELEMS (1 << 21)
+
+/*
+ * hydra_lora_linear for callers that cannot allocate device memory: a plugin inside a
+ * host framework that owns the device memory pool and passes it only its input and output
+ * buffers, or a latency-critical caller that cannot afford cudaMalloc/cudaFree (they may
+ * synchronise the device). The paper has no counterpart to this entry point.
+ * Same arguments, results and argument errors as hydra_lora_linear, without the workspace:
+ * u = s x_on A^T lives in a static device array of HYDRA_NOALLOC_MAX_U_ELEMS bf16 elements
+ * (4 MiB) that every device which loads the library holds until the process exits; the
+ * call allocates nothing.
+ *  - M * r > HYDRA_NOALLOC_MAX_U_ELEMS (with LoRA active) returns HYDRA_ERR_SHAPE and
+ *    launches nothing.
+ *  - The first call on a device resolves the array's address on that device (device set-up);
+ *    make it before any stream capture on that device.
+ *  - All calls share the array. Calls whose work overlaps on the GPU (different streams, or
+ *    unordered host threads) race on it; serialise them, e.g. on one stream.
+ */
+hydra_status hydra_lora_linear_noalloc(const void* x_off, const void* x_on, int64_t M, int64_t K,
+                                       int64_t N, const void* W, const void* A, const void* B,
+                                       int64_t r, float s, void* y_off, void* y_on, int out_dtype,
+                                       void* stream);
+
 /*
  * Per-token log-probabilities of the sampled tokens under the actor (LoRA on) and the
  * reference (LoRA off) heads, and the KL-penalised reward (Algorithm 1/2: LoRA off gives

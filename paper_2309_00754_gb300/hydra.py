@@ -34,6 +34,9 @@ _SIGNATURES = {
                                               ctypes.c_size_t, ctypes.c_int, _vp]),
     "hydra_dual_linear": (ctypes.c_int, [_vp, _vp, _c_i64, _c_i64, _c_i64, _vp, _vp, _vp, _c_i64,
                                          _vp, _vp, ctypes.c_int, ctypes.c_int, _vp]),
+    "hydra_lora_linear_noalloc": (ctypes.c_int, [_vp, _vp, _c_i64, _c_i64, _c_i64, _vp, _vp, _vp,
+                                                 _c_i64, ctypes.c_float, _vp, _vp, ctypes.c_int,
+                                                 _vp]),
     "hydra_token_logprobs_kl": (ctypes.c_int, [_vp, _vp, ctypes.c_int, _c_i64, _c_i64, _c_i64,
                                                _c_i64, _vp, _vp, _vp, ctypes.c_float, _vp, _vp,
                                                _vp, _vp, _vp, _vp]),
@@ -155,6 +158,23 @@ def hydra_dual_linear(x_off, x_on, W, u, B, y_off, y_on, algo=0, stream=None):
     _check("hydra_dual_linear", load().hydra_dual_linear(
         _p(x_off), _p(x_on), M, K, N, _p(W), _p(u), _p(B), r, _p(y_off), _p(y_on), out_dtype,
         int(algo), _stream(stream)))
+
+
+def hydra_lora_linear_noalloc(x_off, x_on, W, A, B, s, y_off, y_on, stream=None):
+    """hydra_lora_linear without a workspace: u lives in the library's static device array
+    (M * r <= HYDRA_NOALLOC_MAX_U_ELEMS), for callers that cannot allocate device memory."""
+    for t, n in ((x_off, "x_off"), (x_on, "x_on"), (W, "W"), (A, "A"), (B, "B")):
+        _req(t, torch.bfloat16, n)
+    out = y_off if y_off is not None else y_on
+    out_dtype = HYDRA_F32 if out.dtype == torch.float32 else HYDRA_BF16
+    for t, n in ((y_off, "y_off"), (y_on, "y_on")):
+        _req(t, out.dtype, n)
+    M, K = x_off.shape
+    N = W.shape[0]
+    r = 0 if A is None else A.shape[0]
+    _check("hydra_lora_linear_noalloc", load().hydra_lora_linear_noalloc(
+        _p(x_off), _p(x_on), M, K, N, _p(W), _p(A), _p(B), r, float(s), _p(y_off), _p(y_on),
+        out_dtype, _stream(stream)))
 
 
 def hydra_token_logprobs_kl(logits_actor, logits_ref, ids, lengths, seq_score, beta, S, L,
