@@ -2,23 +2,26 @@
 //
 // One frozen weight W serves both roles of the Hydra model (§3 Dynamic LoRA: the
 // reference policy is the actor with its LoRA parameters ignored):
-//     y_off = x_off W^T                 (LoRA off: reference / reward stream)
-//     y_on  = x_on  W^T + u B^T,  u = s x_on A^T   (LoRA on: actor / critic stream)
+//     y_off = x_off W^T                             (LoRA off: reference / reward stream)
+//     y_on  = x_on  W^T + u B^T,  u = s x_on A^T    (LoRA on: actor / critic stream)
 // Storage: x [M, K], W [N, K], u [M, r], B [N, r], all bf16 row-major (K-major operands).
 //
-// Two tile kinds share one kernel:
-//  * shared input (x_on == x_off): the tile's x W^T accumulates once in TMEM; the
-//    epilogue drains it to y_off, then the MMA thread accumulates u B^T on top of the same
-//    TMEM accumulator and the epilogue drains y_on. One read of each W tile yields both.
-//  * stacked streams (x_on != x_off): tiles of the off stream produce y_off; tiles of the on
-//    stream run the main loop followed by the LoRA k-blocks ([x_on | u] [W | B]^T) into one
-//    accumulator and produce y_on. Off and on tiles of the same n-block run next to each
-//    other, so each W tile is fetched from HBM once and re-read from L2.
+// Persistent kernel, one CTA per SM, tiles of 128 x 256 (k-step 64) taken round-robin.
+// Warp 0 issues TMA loads into a 4-stage shared-memory ring, warp 1 owns TMEM and issues
+// tcgen05.mma from one thread, warps 2..5 drain TMEM (warp w reads lanes 32*(w%4)..+31)
+// and store through swizzled shared memory with TMA. TMEM holds two 128 x 256 fp32
+// accumulators, so the epilogue of one tile overlaps the main loop of the next.
 //
-// CTA layout (192 threads): warp 0 = TMA producer, warp 1 = TMEM owner + MMA issuer,
-// warps 2..5 = epilogue (warp w reads TMEM lanes 32*(w%4) .. +31).
-// Tile 128 x 256 x 64, 4-stage shared-memory ring, bf16 inputs, fp32 accumulation,
-// 128-byte-swizzled K-major operands.
+// Two tile kinds:
+//  * shared input (x_on == x_off) with LoRA: the tile's x W^T is drained to y_off; the
+//    LoRA k-block(s) (u B^T) then accumulate on top of the same accumulator and the
+//    epilogue drains y_on. The LoRA k-blocks of tile j are placed in the ring a few
+//    k-blocks into tile j+1, so the y_off drain overlaps tensor-core work. One read of
+//    each W tile yields both outputs.
+//  * stacked streams (x_on != x_off): tiles of the off stream produce y_off; tiles of the
+//    on stream run the main loop followed directly by the LoRA k-blocks
+//    ([x_on | u] [W | B]^T) and produce y_on. Off and on tiles of one (m, n) block are
+//    adjacent in the schedule, so each W tile comes from HBM once and again from L2.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -33,66 +36,116 @@ constexpr int A_TILE = BM * BK * 2;  // 16 KiB
 constexpr int B_TILE = BN * BK * 2;  // 32 KiB
 constexpr int STAGE_BYTES = A_TILE + B_TILE;
 constexpr int NUM_THREADS = 192;
-constexpr uint32_t TMEM_COLS = 256;
-constexpr int NUM_BARS = 2 * STAGES + 3;
-constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + NUM_BARS * 8 + 64;
+constexpr int EPI_WARPS = 4;
+constexpr int STAGING_BYTES = 32 * 128;  // 32 rows x 128 B per epilogue-warp buffer
+constexpr uint32_t TMEM_COLS = 512;      // two accumulators of 256 fp32 columns
+constexpr int DEFER = 8;                 // LoRA k-blocks of tile j follow k-block DEFER-1 of tile j+1
+constexpr int NUM_BARS = 2 * STAGES + 7;
+constexpr int SMEM_BYTES =
+    1024 + STAGES * STAGE_BYTES + EPI_WARPS * 2 * STAGING_BYTES + NUM_BARS * 8 + 16;
 constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN);
 
 struct Params {
   int M, N, K;
-  int kb_main;   // ceil(K / BK)
-  int kb_lora;   // ceil(r / BK); 0 = no LoRA
+  int kb_main;  // ceil(K / BK)
+  int kb_lora;  // ceil(r / BK); 0 = no LoRA
   int r;
-  int shared_x;  // 1 = x_on is x_off
-  int m_tiles, n_tiles;
-  void* y_off;
-  void* y_on;
+  int shared_x;   // 1 = x_on is x_off
+  int deferred;   // shared input with LoRA and both outputs: y_off drain, then LoRA
+  int streams;    // 1 (shared) or 2 (stacked)
+  int m_tiles, n_tiles, total_tiles;
+  int has_off, has_on;
   int out_f32;
   int* err;
 };
 
-__device__ __forceinline__ void store_chunk(void* y, int out_f32, int N, int m, int n,
-                                            const uint32_t (&v)[32]) {
-  if (out_f32) {
-    float* row = reinterpret_cast<float*>(y) + static_cast<size_t>(m) * N + n;
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      if (n + 4 * j < N) {
-        float4 f = make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
-                               __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
-        *reinterpret_cast<float4*>(row + 4 * j) = f;
-      }
-    }
-  } else {
-    __nv_bfloat16* row = reinterpret_cast<__nv_bfloat16*>(y) + static_cast<size_t>(m) * N + n;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      if (n + 8 * j < N) {
-        uint4 q;
-        q.x = pack_bf16x2(__uint_as_float(v[8 * j + 0]), __uint_as_float(v[8 * j + 1]));
-        q.y = pack_bf16x2(__uint_as_float(v[8 * j + 2]), __uint_as_float(v[8 * j + 3]));
-        q.z = pack_bf16x2(__uint_as_float(v[8 * j + 4]), __uint_as_float(v[8 * j + 5]));
-        q.w = pack_bf16x2(__uint_as_float(v[8 * j + 6]), __uint_as_float(v[8 * j + 7]));
-        *reinterpret_cast<uint4*>(row + 8 * j) = q;
-      }
-    }
-  }
+struct Tile {
+  int stream, m0, n0, n_lora;
+};
+
+__device__ __forceinline__ Tile decode(const Params& p, int t) {
+  Tile tl;
+  tl.stream = t % p.streams;
+  t /= p.streams;
+  tl.m0 = (t % p.m_tiles) * BM;
+  tl.n0 = (t / p.m_tiles) * BN;
+  const bool on = p.shared_x ? true : (tl.stream == 1);
+  tl.n_lora = (p.kb_lora > 0 && on && p.has_on) ? p.kb_lora : 0;
+  return tl;
 }
 
-// Epilogue warp: read the 32 TMEM lanes of this warp (tile rows) across the tile's columns
-// and store them to up to two outputs.
-__device__ __forceinline__ void drain(uint32_t tmem_row, int m, int M, int n0, const Params& p,
-                                      void* t0, void* t1) {
-#pragma unroll 1
-  for (int c = 0; c < BN / 32; ++c) {
-    uint32_t v[32];
-    tc_ld_32x32b_x32(tmem_row + c * 32, v);
-    tc_wait_ld();
-    const int n = n0 + c * 32;
-    if (m < M && n < p.N) {
-      if (t0) store_chunk(t0, p.out_f32, p.N, m, n, v);
-      if (t1) store_chunk(t1, p.out_f32, p.N, m, n, v);
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, uint32_t src, int x, int y) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y), "r"(src)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() {
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait_read1() {
+  asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() {
+  asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+__device__ __forceinline__ void fence_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
+                                             uint32_t d) {
+  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c),
+               "r"(d)
+               : "memory");
+}
+
+// Epilogue warp: drain the warp's 32 accumulator rows (TMEM lanes) of one tile to up to two
+// outputs. Each 128-byte-wide column chunk goes registers -> 128B-swizzled staging buffer
+// -> TMA store of a [32 rows x 128 B] box; two staging buffers alternate.
+__device__ __forceinline__ void drain(uint32_t tmem_acc, int q, int lane, uint32_t staging,
+                                      uint32_t& chunk_ctr, const Params& p, int m0, int n0,
+                                      const CUtensorMap* t0, const CUtensorMap* t1) {
+  const int nchunks = p.out_f32 ? BN / 32 : BN / 64;
+  const uint32_t lane_taddr = tmem_acc + (static_cast<uint32_t>(q * 32) << 16);
+  const int y = m0 + q * 32;
+  for (int c = 0; c < nchunks; ++c) {
+    const uint32_t buf = staging + (chunk_ctr & 1u) * STAGING_BYTES;
+    if (lane == 0) bulk_wait_read1();  // the store issued two chunks ago has read `buf`
+    __syncwarp();
+    uint32_t w[32];
+    int x;
+    if (p.out_f32) {
+      tc_ld_32x32b_x32(lane_taddr + c * 32, w);
+      tc_wait_ld();
+      x = n0 + c * 32;
+    } else {
+      uint32_t v0[32], v1[32];
+      tc_ld_32x32b_x32(lane_taddr + c * 64, v0);
+      tc_ld_32x32b_x32(lane_taddr + c * 64 + 32, v1);
+      tc_wait_ld();
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        w[i] = pack_bf16x2(__uint_as_float(v0[2 * i]), __uint_as_float(v0[2 * i + 1]));
+        w[16 + i] = pack_bf16x2(__uint_as_float(v1[2 * i]), __uint_as_float(v1[2 * i + 1]));
+      }
+      x = n0 + c * 64;
     }
+    const uint32_t row = buf + lane * 128;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      st_shared_v4(row + ((j ^ (lane & 7)) << 4), w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]);
+    }
+    fence_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      if (x < p.N && y < p.M) {
+        if (t0) tma_store_2d(t0, buf, x, y);
+        if (t1) tma_store_2d(t1, buf, x, y);
+      }
+      bulk_commit();
+    }
+    ++chunk_ctr;
   }
 }
 
@@ -101,69 +154,44 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                           const __grid_constant__ CUtensorMap tm_x_on,
                           const __grid_constant__ CUtensorMap tm_w,
                           const __grid_constant__ CUtensorMap tm_u,
-                          const __grid_constant__ CUtensorMap tm_b, const Params p) {
+                          const __grid_constant__ CUtensorMap tm_b,
+                          const __grid_constant__ CUtensorMap tm_y_off,
+                          const __grid_constant__ CUtensorMap tm_y_on, const Params p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint8_t* staging_base = smem + STAGES * STAGE_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(staging_base + EPI_WARPS * 2 * STAGING_BYTES);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + NUM_BARS);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-
-  // tile -> (stream, m-block, n-block); off/on tiles of one (m, n) are adjacent
-  const int streams = p.shared_x ? 1 : 2;
-  int t = blockIdx.x;
-  const int stream = t % streams;
-  t /= streams;
-  const int m_idx = t % p.m_tiles;
-  const int n_idx = t / p.m_tiles;
-  const int m0 = m_idx * BM;
-  const int n0 = n_idx * BN;
-
-  const bool on_stream = p.shared_x ? true : (stream == 1);
-  const int n_lora = (p.kb_lora > 0 && on_stream && p.y_on != nullptr) ? p.kb_lora : 0;
-  const bool mid_drain = p.shared_x && n_lora > 0 && p.y_off != nullptr;
-  const int total_kb = p.kb_main + n_lora;
-  const CUtensorMap* tmx = (stream == 1) ? &tm_x_on : &tm_x_off;
-
-  // final drain targets
-  void* fin0;
-  void* fin1 = nullptr;
-  if (p.shared_x) {
-    if (n_lora > 0) {
-      fin0 = p.y_on;
-    } else {
-      fin0 = p.y_off;
-      fin1 = p.y_on;
-    }
-  } else {
-    fin0 = (stream == 1) ? p.y_on : p.y_off;
-  }
+  const int n_local = (p.total_tiles - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
+                      static_cast<int>(gridDim.x);
+  const int defer_at = min(DEFER, p.kb_main) - 1;
 
   const uint32_t smem_base = smem_u32(smem);
   auto full_bar = [&](int s) { return smem_u32(&bars[s]); };
   auto empty_bar = [&](int s) { return smem_u32(&bars[STAGES + s]); };
-  const uint32_t acc_full = smem_u32(&bars[2 * STAGES]);
-  const uint32_t acc_empty = smem_u32(&bars[2 * STAGES + 1]);
-  const uint32_t mma_done = smem_u32(&bars[2 * STAGES + 2]);
+  auto acc_full = [&](int b) { return smem_u32(&bars[2 * STAGES + b]); };
+  auto acc_mid = [&](int b) { return smem_u32(&bars[2 * STAGES + 2 + b]); };
+  auto acc_empty = [&](int b) { return smem_u32(&bars[2 * STAGES + 4 + b]); };
+  const uint32_t mma_done = smem_u32(&bars[2 * STAGES + 6]);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(full_bar(s), 1);
       mbar_init(empty_bar(s), 1);
     }
-    mbar_init(acc_full, 1);
-    mbar_init(acc_empty, 128);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(acc_full(b), 1);
+      mbar_init(acc_mid(b), 32 * EPI_WARPS);
+      mbar_init(acc_empty(b), 32 * EPI_WARPS);
+    }
     mbar_init(mma_done, 1);
     *abort_flag = 0;
     fence_mbar_init();
-    tma_prefetch_desc(&tm_x_off);
-    tma_prefetch_desc(&tm_x_on);
-    tma_prefetch_desc(&tm_w);
-    tma_prefetch_desc(&tm_u);
-    tma_prefetch_desc(&tm_b);
   }
   if (warp == 1) {
     tmem_alloc(smem_u32(tmem_slot), TMEM_COLS);
@@ -177,29 +205,49 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------------------ TMA producer
-      int issued = 0;
-      for (int kb = 0; kb < total_kb; ++kb) {
-        const int s = kb % STAGES;
-        const uint32_t ph = (kb / STAGES) & 1;
-        if (!mbar_wait_bounded(empty_bar(s), ph ^ 1, abort_flag, p.err, kDevTimeoutProducer)) break;
+      tma_prefetch_desc(&tm_x_off);
+      tma_prefetch_desc(&tm_x_on);
+      tma_prefetch_desc(&tm_w);
+      tma_prefetch_desc(&tm_u);
+      tma_prefetch_desc(&tm_b);
+      int it = 0;
+      bool ok = true;
+      auto load = [&](const CUtensorMap* ma, int xa, int ya, const CUtensorMap* mb, int xb,
+                      int yb) {
+        const int s = it % STAGES;
+        const uint32_t ph = (it / STAGES) & 1;
+        if (!mbar_wait_bounded(empty_bar(s), ph ^ 1, abort_flag, p.err, kDevTimeoutProducer)) {
+          ok = false;
+          return;
+        }
         mbar_arrive_expect_tx(full_bar(s), STAGE_BYTES);
         const uint32_t a_dst = smem_base + s * STAGE_BYTES;
-        const uint32_t b_dst = a_dst + A_TILE;
-        if (kb < p.kb_main) {
-          tma_load_2d(a_dst, tmx, kb * BK, m0, full_bar(s));
-          tma_load_2d(b_dst, &tm_w, kb * BK, n0, full_bar(s));
-        } else {
-          const int kl = kb - p.kb_main;
-          tma_load_2d(a_dst, &tm_u, kl * BK, m0, full_bar(s));
-          tma_load_2d(b_dst, &tm_b, kl * BK, n0, full_bar(s));
+        tma_load_2d(a_dst, ma, xa, ya, full_bar(s));
+        tma_load_2d(a_dst + A_TILE, mb, xb, yb, full_bar(s));
+        ++it;
+      };
+      Tile prev{0, 0, 0, 0};
+      for (int j = 0; j < n_local && ok; ++j) {
+        const Tile tl = decode(p, blockIdx.x + j * gridDim.x);
+        const CUtensorMap* tmx = (tl.stream == 1) ? &tm_x_on : &tm_x_off;
+        for (int kb = 0; kb < p.kb_main && ok; ++kb) {
+          load(tmx, kb * BK, tl.m0, &tm_w, kb * BK, tl.n0);
+          if (p.deferred && j > 0 && kb == defer_at)
+            for (int kl = 0; kl < prev.n_lora && ok; ++kl)
+              load(&tm_u, kl * BK, prev.m0, &tm_b, kl * BK, prev.n0);
         }
-        ++issued;
+        if (!p.deferred)
+          for (int kl = 0; kl < tl.n_lora && ok; ++kl)
+            load(&tm_u, kl * BK, tl.m0, &tm_b, kl * BK, tl.n0);
+        prev = tl;
       }
+      if (p.deferred && n_local > 0)
+        for (int kl = 0; kl < prev.n_lora && ok; ++kl)
+          load(&tm_u, kl * BK, prev.m0, &tm_b, kl * BK, prev.n0);
       // copies still in flight must land before the CTA's shared memory is released
-      const int first = issued > STAGES ? issued - STAGES : 0;
-      for (int kb = first; kb < issued; ++kb) {
+      for (int k = (it > STAGES ? it - STAGES : 0); k < it; ++k) {
         volatile int no_abort = 0;
-        mbar_wait_bounded(full_bar(kb % STAGES), (kb / STAGES) & 1, &no_abort, p.err,
+        mbar_wait_bounded(full_bar(k % STAGES), (k / STAGES) & 1, &no_abort, p.err,
                           kDevTimeoutDrain);
       }
     }
@@ -207,37 +255,55 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   } else if (warp == 1) {
     if (lane == 0) {
       // ------------------------------------------------------------ MMA issuer
+      int it = 0;
       bool ok = true;
-      for (int kb = 0; kb < total_kb && ok; ++kb) {
-        if (kb == p.kb_main && mid_drain) {
-          tc_commit(acc_full);  // y_off = x W^T is complete in TMEM
-          if (!mbar_wait_bounded(acc_empty, 0, abort_flag, p.err, kDevTimeoutMma)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-        }
-        const int s = kb % STAGES;
-        const uint32_t ph = (kb / STAGES) & 1;
+      // one ring item: nsub MMAs of K = 16 into the accumulator at `acc`
+      auto consume = [&](uint32_t acc, int nsub, bool first) {
+        const int s = it % STAGES;
+        const uint32_t ph = (it / STAGES) & 1;
         if (!mbar_wait_bounded(full_bar(s), ph, abort_flag, p.err, kDevTimeoutMma)) {
           ok = false;
-          break;
+          return;
         }
         tc_fence_after();
         const uint32_t a_base = smem_base + s * STAGE_BYTES;
         const uint32_t b_base = a_base + A_TILE;
-        int nsub = BK / 16;
-        if (kb >= p.kb_main) {
-          const int rem = p.r - (kb - p.kb_main) * BK;
-          nsub = min(BK / 16, (rem + 15) / 16);
-        }
-        for (int k = 0; k < nsub; ++k) {
-          tc_mma_bf16(tmem_base, smem_desc_sw128(a_base + k * 32), smem_desc_sw128(b_base + k * 32),
-                      IDESC, (kb > 0 || k > 0) ? 1u : 0u);
-        }
+        for (int k = 0; k < nsub; ++k)
+          tc_mma_bf16(acc, smem_desc_sw128(a_base + k * 32), smem_desc_sw128(b_base + k * 32),
+                      IDESC, (first && k == 0) ? 0u : 1u);
         tc_commit(empty_bar(s));
+        ++it;
+      };
+      auto lora_nsub = [&](int kl) { return min(BK / 16, (p.r - kl * BK + 15) / 16); };
+      auto lora_items = [&](int jj, int n_lora, bool wait_mid) {
+        const int b = jj & 1;
+        if (wait_mid) {
+          if (!mbar_wait_bounded(acc_mid(b), (jj >> 1) & 1, abort_flag, p.err, kDevTimeoutMma)) {
+            ok = false;
+            return;
+          }
+          tc_fence_after();
+        }
+        for (int kl = 0; kl < n_lora && ok; ++kl) consume(tmem_base + b * 256, lora_nsub(kl), false);
+        if (ok) tc_commit(acc_full(b));
+      };
+      Tile prev{0, 0, 0, 0};
+      for (int j = 0; j < n_local && ok; ++j) {
+        const Tile tl = decode(p, blockIdx.x + j * gridDim.x);
+        const int b = j & 1;
+        if (!mbar_wait_bounded(acc_empty(b), ((j >> 1) & 1) ^ 1, abort_flag, p.err, kDevTimeoutMma))
+          break;
+        tc_fence_after();
+        const uint32_t acc = tmem_base + b * 256;
+        for (int kb = 0; kb < p.kb_main && ok; ++kb) {
+          consume(acc, BK / 16, kb == 0);
+          if (kb == p.kb_main - 1 && ok && (p.deferred || tl.n_lora == 0)) tc_commit(acc_full(b));
+          if (p.deferred && j > 0 && kb == defer_at && ok) lora_items(j - 1, prev.n_lora, true);
+        }
+        if (!p.deferred && tl.n_lora > 0 && ok) lora_items(j, tl.n_lora, false);
+        prev = tl;
       }
-      if (ok) tc_commit(acc_full);
+      if (p.deferred && n_local > 0 && ok) lora_items(n_local - 1, prev.n_lora, true);
       // every issued MMA has finished before TMEM is released
       tc_commit(mma_done);
       volatile int no_abort = 0;
@@ -247,28 +313,45 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   } else {
     // -------------------------------------------------------------- epilogue
     const int q = warp & 3;
-    const int row = q * 32 + lane;
-    const int m = m0 + row;
-    const uint32_t tmem_row = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
-    uint32_t phase = 0;
-    bool ok = true;
-    if (mid_drain) {
-      ok = mbar_wait_bounded(acc_full, 0, abort_flag, p.err, kDevTimeoutEpilogue);
-      if (ok) {
+    const uint32_t staging = smem_u32(staging_base) + (warp - 2) * 2 * STAGING_BYTES;
+    uint32_t chunk_ctr = 0;
+    const CUtensorMap* y_off = p.has_off ? &tm_y_off : nullptr;
+    const CUtensorMap* y_on = p.has_on ? &tm_y_on : nullptr;
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_y_off);
+      tma_prefetch_desc(&tm_y_on);
+    }
+    for (int j = 0; j < n_local; ++j) {
+      const Tile tl = decode(p, blockIdx.x + j * gridDim.x);
+      const int b = j & 1;
+      const uint32_t acc = tmem_base + b * 256;
+      if (p.deferred) {
+        if (!mbar_wait_bounded(acc_full(b), 0, abort_flag, p.err, kDevTimeoutEpilogue)) break;
         tc_fence_after();
-        drain(tmem_row, m, p.M, n0, p, p.y_off, nullptr);
+        drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, y_off, nullptr);
         tc_fence_before();
-        mbar_arrive(acc_empty);
-        phase = 1;
+        mbar_arrive(acc_mid(b));
+        if (!mbar_wait_bounded(acc_full(b), 1, abort_flag, p.err, kDevTimeoutEpilogue)) break;
+        tc_fence_after();
+        drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, y_on, nullptr);
+      } else {
+        if (!mbar_wait_bounded(acc_full(b), (j >> 1) & 1, abort_flag, p.err, kDevTimeoutEpilogue))
+          break;
+        tc_fence_after();
+        if (p.shared_x)
+          drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, tl.n_lora > 0 ? nullptr : y_off, y_on);
+        else
+          drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, tl.stream == 1 ? y_on : y_off,
+                nullptr);
       }
+      tc_fence_before();
+      mbar_arrive(acc_empty(b));
     }
-    if (ok && mbar_wait_bounded(acc_full, phase, abort_flag, p.err, kDevTimeoutEpilogue)) {
-      tc_fence_after();
-      drain(tmem_row, m, p.M, n0, p, fin0, fin1);
-    }
-    tc_fence_before();
+    if (lane == 0) bulk_wait_all();
+    __syncwarp();
   }
 
+  tc_fence_before();
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
@@ -298,20 +381,34 @@ static EncodeTiledFn get_encode_fn() {
   return fn;
 }
 
-// 2-D bf16 tensor map over a row-major [rows, cols] matrix, box [box_rows, 64] with
-// 128-byte swizzle; out-of-bounds elements read as zero.
+// 2-D tensor map over a row-major [rows, cols] matrix with 128-byte swizzle and a box of
+// [box_rows, 128 bytes]; out-of-bounds loads read zero, out-of-bounds stores are dropped.
 static bool make_map(CUtensorMap* map, const void* base, int64_t rows, int64_t cols,
-                     int box_rows) {
+                     int box_rows, bool f32) {
   EncodeTiledFn enc = get_encode_fn();
   if (enc == nullptr) return false;
+  const int esize = f32 ? 4 : 2;
   cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
-  cuuint64_t strides[1] = {static_cast<cuuint64_t>(cols) * 2};
-  cuuint32_t box[2] = {static_cast<cuuint32_t>(tcgemm::BK), static_cast<cuuint32_t>(box_rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(cols) * esize};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(128 / esize), static_cast<cuuint32_t>(box_rows)};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
-                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  CUresult r = enc(map, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                   const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                   CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
+}
+
+static int sm_count() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  if (cached[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    cached[dev] = n;
+  }
+  return cached[dev];
 }
 
 int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream) {
@@ -323,18 +420,25 @@ int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream) {
       return -1;
     attr_set = true;
   }
-  CUtensorMap m_xoff, m_xon, m_w, m_u, m_b;
+  const int nsm = sm_count();
+  if (nsm <= 0) return -1;
+  CUtensorMap m_xoff, m_xon, m_w, m_u, m_b, m_yoff, m_yon;
   const bool lora = a.r > 0;
-  if (!make_map(&m_xoff, a.x_off, a.M, a.K, BM)) return -2;
-  if (!make_map(&m_xon, a.shared_x ? a.x_off : a.x_on, a.M, a.K, BM)) return -2;
-  if (!make_map(&m_w, a.W, a.N, a.K, BN)) return -2;
+  const bool f32 = a.out_f32 != 0;
+  if (!make_map(&m_xoff, a.x_off, a.M, a.K, BM, false)) return -2;
+  if (!make_map(&m_xon, a.shared_x ? a.x_off : a.x_on, a.M, a.K, BM, false)) return -2;
+  if (!make_map(&m_w, a.W, a.N, a.K, BN, false)) return -2;
   if (lora) {
-    if (!make_map(&m_u, a.u, a.M, a.r, BM)) return -2;
-    if (!make_map(&m_b, a.B, a.N, a.r, BN)) return -2;
+    if (!make_map(&m_u, a.u, a.M, a.r, BM, false)) return -2;
+    if (!make_map(&m_b, a.B, a.N, a.r, BN, false)) return -2;
   } else {
     m_u = m_xoff;
     m_b = m_w;
   }
+  const void* any_y = a.y_off ? a.y_off : a.y_on;
+  if (!make_map(&m_yoff, a.y_off ? a.y_off : any_y, a.M, a.N, 32, f32)) return -2;
+  if (!make_map(&m_yon, a.y_on ? a.y_on : any_y, a.M, a.N, 32, f32)) return -2;
+
   Params p;
   p.M = static_cast<int>(a.M);
   p.N = static_cast<int>(a.N);
@@ -343,15 +447,18 @@ int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream) {
   p.kb_lora = lora ? static_cast<int>((a.r + BK - 1) / BK) : 0;
   p.r = static_cast<int>(a.r);
   p.shared_x = a.shared_x ? 1 : 0;
+  p.has_off = a.y_off != nullptr;
+  p.has_on = a.y_on != nullptr;
+  p.deferred = (p.shared_x && lora && p.has_off && p.has_on) ? 1 : 0;
+  p.streams = a.shared_x ? 1 : 2;
   p.m_tiles = static_cast<int>((a.M + BM - 1) / BM);
   p.n_tiles = static_cast<int>((a.N + BN - 1) / BN);
-  p.y_off = a.y_off;
-  p.y_on = a.y_on;
+  p.total_tiles = p.m_tiles * p.n_tiles * p.streams;
   p.out_f32 = a.out_f32;
   p.err = a.err;
-  const int streams = a.shared_x ? 1 : 2;
-  const unsigned grid = static_cast<unsigned>(p.m_tiles) * p.n_tiles * streams;
-  dual_lora_gemm_kernel<<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(m_xoff, m_xon, m_w, m_u, m_b, p);
+  const unsigned grid = static_cast<unsigned>(p.total_tiles < nsm ? p.total_tiles : nsm);
+  dual_lora_gemm_kernel<<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(m_xoff, m_xon, m_w, m_u, m_b,
+                                                                   m_yoff, m_yon, p);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
 }
 
