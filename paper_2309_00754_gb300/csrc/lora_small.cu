@@ -1,8 +1,9 @@
-// Skinny LoRA kernels on the CUDA cores:
+// Skinny LoRA kernels:
 //  * lora_down: u = s * (x_on A^T), bf16 [M, r]; the rank-r down-projection of the
 //    LoRA update (§2 Stage 3: LoRA on all linear layers), with the scale folded in fp32
-//    before the bf16 rounding. It is the operand of the LoRA-up MMA of the tensor-core
-//    kernel and of the GEMV below.
+//    before the bf16 rounding. It is the operand of the LoRA-up MMA of the tcgen05
+//    kernel and of the GEMV below. (Uses mma.sync: a skinny product far too narrow for a
+//    128-row tcgen05 tile to stay busy.)
 //  * dual_lora_gemv: the dual-output linear for decode-shaped inputs (at most 16 token
 //    rows over both streams), y_off = x_off W^T, y_on = x_on W^T + u B^T. One warp owns two
 //    rows of W and streams them once with 128-bit loads; the token rows are re-read from
@@ -28,63 +29,92 @@ __device__ __forceinline__ float dot8(const float (&a)[8], const float (&b)[8]) 
 }
 
 // ---------------------------------------------------------------- lora_down
+//
+// u[M, r] = bf16(s * x A^T) as a skinny matrix product on the tensor cores (mma.sync
+// m16n8k16, bf16 in, fp32 accumulate): one CTA per 16 token rows and per 64 ranks; its 8
+// warps split K, load their fragments straight from global memory (each 32-byte row
+// segment is read whole by four lanes) and reduce the 8 partial tiles in shared memory.
 
-constexpr int kDownRows = 4;   // token rows per warp
-constexpr int kDownRJ = 16;    // LoRA ranks per CTA column (grid.y covers r)
+constexpr int kDownWarps = 8;
 
-__global__ void __launch_bounds__(256)
+__device__ __forceinline__ uint32_t ld_pair(const __nv_bfloat16* p, bool ok) {
+  return ok ? __ldg(reinterpret_cast<const uint32_t*>(p)) : 0u;
+}
+
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
+                                               uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+template <int NT>  // NT n-tiles of 8 ranks
+__global__ void __launch_bounds__(32 * kDownWarps)
     lora_down_kernel(const __nv_bfloat16* __restrict__ x, int M, int K,
                      const __nv_bfloat16* __restrict__ A, int r, float s,
                      __nv_bfloat16* __restrict__ u) {
+  __shared__ float red[kDownWarps][16][NT * 8 + 1];
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int row0 = (blockIdx.x * 8 + warp) * kDownRows;
-  const int j0 = blockIdx.y * kDownRJ;
-  if (row0 >= M) return;
-  float acc[kDownRows][kDownRJ];
-#pragma unroll
-  for (int i = 0; i < kDownRows; ++i)
-#pragma unroll
-    for (int j = 0; j < kDownRJ; ++j) acc[i][j] = 0.f;
+  const int g = lane >> 2, c = lane & 3;
+  const int row0 = blockIdx.x * 16;
+  const int n_base = blockIdx.y * NT * 8;
+  // this warp's K range, in whole k-steps of 16
+  const int ksteps = (K + 15) / 16;
+  const int per = (ksteps + kDownWarps - 1) / kDownWarps;
+  const int ks0 = warp * per;
+  const int ks1 = min(ksteps, ks0 + per);
 
-  for (int k = lane * 8; k < K; k += 256) {
-    float xv[kDownRows][8];
+  const bool r_lo = row0 + g < M, r_hi = row0 + g + 8 < M;
+  const __nv_bfloat16* x_lo = x + static_cast<size_t>(r_lo ? row0 + g : 0) * K;
+  const __nv_bfloat16* x_hi = x + static_cast<size_t>(r_hi ? row0 + g + 8 : 0) * K;
+  const __nv_bfloat16* a_row[NT];
+  bool a_ok[NT];
 #pragma unroll
-    for (int i = 0; i < kDownRows; ++i) {
-      if (row0 + i < M) {
-        unpack8(__ldg(reinterpret_cast<const uint4*>(x + static_cast<size_t>(row0 + i) * K + k)),
-                xv[i]);
-      } else {
+  for (int t = 0; t < NT; ++t) {
+    const int n = n_base + t * 8 + g;
+    a_ok[t] = n < r;
+    a_row[t] = A + static_cast<size_t>(a_ok[t] ? n : 0) * K;
+  }
+  float d[NT][4];
 #pragma unroll
-        for (int e = 0; e < 8; ++e) xv[i][e] = 0.f;
-      }
-    }
+  for (int t = 0; t < NT; ++t) d[t][0] = d[t][1] = d[t][2] = d[t][3] = 0.f;
+
+#pragma unroll 4
+  for (int ks = ks0; ks < ks1; ++ks) {
+    const int k0 = ks * 16 + 2 * c;
+    const int k1 = k0 + 8;
+    const bool v0 = k0 < K, v1 = k1 < K;
+    uint32_t a[4];
+    a[0] = ld_pair(x_lo + k0, r_lo && v0);
+    a[1] = ld_pair(x_hi + k0, r_hi && v0);
+    a[2] = ld_pair(x_lo + k1, r_lo && v1);
+    a[3] = ld_pair(x_hi + k1, r_hi && v1);
 #pragma unroll
-    for (int j = 0; j < kDownRJ; ++j) {
-      if (j0 + j < r) {
-        float av[8];
-        unpack8(__ldg(reinterpret_cast<const uint4*>(A + static_cast<size_t>(j0 + j) * K + k)), av);
-#pragma unroll
-        for (int i = 0; i < kDownRows; ++i) acc[i][j] += dot8(xv[i], av);
-      }
+    for (int t = 0; t < NT; ++t) {
+      const uint32_t b0 = ld_pair(a_row[t] + k0, a_ok[t] && v0);
+      const uint32_t b1 = ld_pair(a_row[t] + k1, a_ok[t] && v1);
+      mma_bf16_16816(d[t], a, b0, b1);
     }
   }
 #pragma unroll
-  for (int i = 0; i < kDownRows; ++i)
+  for (int t = 0; t < NT; ++t) {
+    red[warp][g][t * 8 + 2 * c] = d[t][0];
+    red[warp][g][t * 8 + 2 * c + 1] = d[t][1];
+    red[warp][g + 8][t * 8 + 2 * c] = d[t][2];
+    red[warp][g + 8][t * 8 + 2 * c + 1] = d[t][3];
+  }
+  __syncthreads();
+  for (int e = threadIdx.x; e < 16 * NT * 8; e += blockDim.x) {
+    const int rr = e / (NT * 8), cc = e % (NT * 8);
+    float v = 0.f;
 #pragma unroll
-    for (int j = 0; j < kDownRJ; ++j) {
-      float v = acc[i][j];
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-      acc[i][j] = v;
-    }
-#pragma unroll
-  for (int i = 0; i < kDownRows; ++i)
-#pragma unroll
-    for (int j = 0; j < kDownRJ; ++j) {
-      if (((i * kDownRJ + j) & 31) == lane && row0 + i < M && j0 + j < r)
-        u[static_cast<size_t>(row0 + i) * r + j0 + j] = __float2bfloat16_rn(s * acc[i][j]);
-    }
+    for (int w = 0; w < kDownWarps; ++w) v += red[w][rr][cc];
+    const int m = row0 + rr, n = n_base + cc;
+    if (m < M && n < r) u[static_cast<size_t>(m) * r + n] = __float2bfloat16_rn(s * v);
+  }
 }
 
 // ---------------------------------------------------------------- dual_lora_gemv
@@ -223,12 +253,21 @@ void launch_gemv_t(const GemmArgs& a, cudaStream_t stream) {
 int launch_lora_down(const void* x, int64_t M, int64_t K, const void* A, int64_t r, float s,
                      void* u, cudaStream_t stream) {
   if (M == 0 || r == 0) return 0;
-  dim3 grid(static_cast<unsigned>((M + 8 * kDownRows - 1) / (8 * kDownRows)),
-            static_cast<unsigned>((r + kDownRJ - 1) / kDownRJ));
-  lora_down_kernel<<<grid, 256, 0, stream>>>(
-      static_cast<const __nv_bfloat16*>(x), static_cast<int>(M), static_cast<int>(K),
-      static_cast<const __nv_bfloat16*>(A), static_cast<int>(r), s,
-      static_cast<__nv_bfloat16*>(u));
+  const dim3 block(32 * kDownWarps);
+  const auto* xp = static_cast<const __nv_bfloat16*>(x);
+  const auto* ap = static_cast<const __nv_bfloat16*>(A);
+  auto* up = static_cast<__nv_bfloat16*>(u);
+  const unsigned gx = static_cast<unsigned>((M + 15) / 16);
+  if (r <= 8) {
+    lora_down_kernel<1><<<dim3(gx, 1), block, 0, stream>>>(xp, static_cast<int>(M), static_cast<int>(K), ap, static_cast<int>(r), s, up);
+  } else if (r <= 16) {
+    lora_down_kernel<2><<<dim3(gx, 1), block, 0, stream>>>(xp, static_cast<int>(M), static_cast<int>(K), ap, static_cast<int>(r), s, up);
+  } else if (r <= 32) {
+    lora_down_kernel<4><<<dim3(gx, 1), block, 0, stream>>>(xp, static_cast<int>(M), static_cast<int>(K), ap, static_cast<int>(r), s, up);
+  } else {
+    lora_down_kernel<8><<<dim3(gx, static_cast<unsigned>((r + 63) / 64)), block, 0, stream>>>(
+        xp, static_cast<int>(M), static_cast<int>(K), ap, static_cast<int>(r), s, up);
+  }
   return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
 }
 
