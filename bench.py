@@ -4,6 +4,10 @@
 One step = one pass of the scoring path over one batch of synthetic input, inputs resident
 in HBM. Prints ONE JSON line (rank 0). Workloads:
 
+  hydra_scoring_llama7b (default) : the full J-Hydra scoring pass (hydra_score_llama) on a
+                    random-init Llama-7B, batch 4 x (256 prompt + 512 response) tokens,
+                    LoRA r=16 on q/v/gate/up/down, reward/value head 4096 -> 1.
+
   lm_head_scoring : final hidden states [4 x 512 x 4096] bf16 -> LoRA down (r=16) ->
                     dual-output LM head 4096 -> 32000 (fp32 logits, both streams, one pass
                     over W) -> sampled-token log-probs + KL reward (beta 0.1, score at the
@@ -113,6 +117,7 @@ class LmHeadScoring:
     """Final hidden states -> dual LM head -> log-probs + KL reward -> GAE."""
 
     name = "lm_head_scoring"
+    seed = 3
     S, L, d, V, r, s = 4, 512, 4096, 32000, 16, 2.0
     beta, gamma, lam = 0.1, 1.0, 0.95
     default_steps, default_warmup = 300, 10
@@ -245,8 +250,158 @@ class LmHeadScoring:
         return n
 
 
-WORKLOADS = {LmHeadScoring.name: LmHeadScoring}
-DEFAULT_WORKLOAD = LmHeadScoring.name
+class HydraScoringLlama7B:
+    """Full J-Hydra scoring pass on a random-init Llama-7B (32 layers, d 4096, 32 heads,
+    SwiGLU 11008, vocab 32000, bf16), LoRA r=16 on q/v/gate/up/down (s = 2), reward head
+    4096 -> 1 on the LoRA-off stream (values: same head on the LoRA-on stream); batch 4 x
+    (256 prompt + 512 response) tokens -> actor/ref log-probs, reward, GAE."""
+
+    name = "hydra_scoring_llama7b"
+    seed = 4
+    default_steps, default_warmup = 20, 3
+
+    def __init__(self, device, seed=4, reference=False):
+        import torch
+        from paper_2309_00754_gb300 import llama, synth
+        self.llama = llama
+        self.cfg = dict(llama.LLAMA7B)
+        c = self.cfg
+        self.S, self.P0, self.L = 4, c["prompt_len"], c["response_len"]
+        self.beta, self.gamma, self.lam = c["beta"], c["gamma"], c["lam"]
+        P = self.P0 + self.L
+        self.weights = llama.random_device_weights(c, seed, device)
+        self.ids = torch.from_numpy(synth.randint(seed * 1000 + 1, (self.S, P), 0, c["vocab"])).to(device)
+        self.lengths = torch.full((self.S,), self.L, dtype=torch.int32, device=device)
+        if not reference:  # the reference arm (fp64 oracle) never loads libhydra
+            from paper_2309_00754_gb300 import hydra as H
+            self.H = H
+            self.ws = torch.empty(H.score_llama_workspace_size(c, self.S), dtype=torch.uint8,
+                                  device=device)
+            self.out = llama.alloc_outputs(self.S, self.L, device)
+        self.units = int(self.S * self.L)
+        T, SL = self.S * P, self.S * self.L
+        d, F, V, r = c["d_model"], c["ffn"], c["vocab"], c["lora_rank"]
+        per_layer = (2 * (2 * T * d * 3 * d) + 2 * T * 2 * r * 3 * d      # qkv (+ LoRA-up)
+                     + 2 * (2 * T * d * d)                                 # o
+                     + 2 * (2 * T * d * 2 * F) + 2 * T * 2 * r * 2 * F     # gate/up
+                     + 2 * (2 * T * F * d) + 2 * T * r * d)                # down
+        self.gemm_flops = c["n_layers"] * per_layer + 2 * (2 * SL * d * V)
+        self.attn_flops = c["n_layers"] * 2 * self.S * c["n_heads"] * 2 * P * P * 128  # causal half
+        self.logp_bytes = SL * V * 4 * 2 + SL * 16
+        self.launches_per_step = None
+
+    def step(self, ev=None):
+        self.H.hydra_score_llama(self.cfg, self.weights, self.ids, self.lengths, self.ws, self.out)
+
+    def e2e_setup(self):
+        import torch
+        self.ids_host = self.ids.cpu().pin_memory()
+        self.len_host = self.lengths.cpu().pin_memory()
+        self.out_host = {k: torch.empty(v.shape, pin_memory=True) for k, v in self.out.items()}
+        self.h2d = self.ids_host.numel() * 4 + self.len_host.numel() * 4
+        self.d2h = sum(v.numel() * 4 for v in self.out_host.values())
+
+    def e2e_step(self):
+        self.ids.copy_(self.ids_host, non_blocking=True)
+        self.lengths.copy_(self.len_host, non_blocking=True)
+        self.step()
+        for k, v in self.out.items():
+            self.out_host[k].copy_(v, non_blocking=True)
+
+    def kernels(self, peaks, prof):
+        out = {}
+        for k, (ms, n) in prof.items():
+            if n:
+                out[k] = {"ms_total": ms, "launches": n, "ms_per_launch": ms / n}
+        g = prof["gemm"]
+        out["gemm"]["TFLOP/s"] = self.gemm_flops * (g[1] / self.launch_counts["gemm"]) / g[0] / 1e9
+        a = prof["attention"]
+        out["attention"]["TFLOP/s"] = self.attn_flops * (a[1] / self.launch_counts["attention"]) / a[0] / 1e9
+        lp = prof["logprobs"]
+        out["logprobs"]["GB/s"] = self.logp_bytes * lp[1] / lp[0] / 1e6
+        return out
+
+    def roofline(self, peaks, prof):
+        ms, n = prof["gemm"]
+        steps = n / self.launch_counts["gemm"]
+        achieved = self.gemm_flops * steps / ms / 1e9
+        peak = peaks["bf16_tflops_sustained"]
+        return {"kernel": "dual_lora_gemm_tcgen05 (all projections + LM head of the pass)",
+                "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": achieved / peak, "traffic": None,
+                "peak_kind": f"bf16 dense, {peaks['source']} sustained",
+                "per_launch_flop": self.gemm_flops / self.launch_counts["gemm"],
+                "per_launch_ms": ms / n}
+
+    def config(self):
+        return {"workload": "hydra_scoring_llama7b: random-init Llama-7B (32 layers, d 4096, 32 heads, "
+                            "SwiGLU 11008, vocab 32000, bf16), LoRA r=16 s=2 on q/v/gate/up/down, reward/"
+                            "value head 4096->1; batch 4 x (256 prompt + 512 response); logp/KL beta 0.1, "
+                            "GAE gamma 1 lambda 0.95",
+                "batch": self.S, "prompt_len": self.P0, "response_len": self.L,
+                "scored_tokens_per_step": self.units,
+                "processed_tokens_per_step": 2 * self.S * (self.P0 + self.L),
+                "l2": "inputs larger than L2 (13.5 GB of weights streamed per step)"}
+
+    # ---- CPU oracle on a bounded slice of the same workload
+    def oracle_sample(self, n_layers, prompt=32, resp=64):
+        import oracle as O
+        torch = __import__("torch")
+        c = self.cfg
+        d, F, r = c["d_model"], c["ffn"], c["lora_rank"]
+        W = self.weights
+
+        def f64(t):
+            return O.bf16_to_f64(t.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16))
+        w = {"wq": [], "wk": [], "wv": [], "wo": [], "wg": [], "wu": [], "wd": [], "norm1": [],
+             "norm2": [], "lora": {}}
+        lo = {k: ([], []) for k in ("wq", "wv", "wg", "wu", "wd")}
+        for l in range(n_layers):
+            qkv = f64(W["w_qkv"][l])
+            w["wq"].append(qkv[:d]); w["wk"].append(qkv[d:2 * d]); w["wv"].append(qkv[2 * d:])
+            w["wo"].append(f64(W["w_o"][l]))
+            gu = f64(W["w_gu"][l])
+            w["wg"].append(gu[:F]); w["wu"].append(gu[F:])
+            w["wd"].append(f64(W["w_down"][l]))
+            w["norm1"].append(f64(W["norm_attn"][l])); w["norm2"].append(f64(W["norm_ffn"][l]))
+            a, b = f64(W["a_qv"][l]), f64(W["b_qkv"][l])
+            lo["wq"][0].append(a[:r]); lo["wq"][1].append(b[:d, :r])
+            lo["wv"][0].append(a[r:]); lo["wv"][1].append(b[2 * d:, r:])
+            a, b = f64(W["a_gu"][l]), f64(W["b_gu"][l])
+            lo["wg"][0].append(a[:r]); lo["wg"][1].append(b[:F, :r])
+            lo["wu"][0].append(a[r:]); lo["wu"][1].append(b[F:, r:])
+            lo["wd"][0].append(f64(W["a_down"][l])); lo["wd"][1].append(f64(W["b_down"][l]))
+        w = {k: (np.stack(v) if v else np.zeros((0,))) for k, v in w.items() if k != "lora"}
+        w["lora"] = {k: (np.stack(a), np.stack(b)) for k, (a, b) in lo.items()}
+        for k in ("embed", "final_norm", "lm_head", "w_rm"):
+            w[k] = f64(W[k])
+        ids = self.ids[0, self.P0 - prompt:self.P0 + resp].cpu().numpy()
+        ocfg = {"d": d, "n_heads": c["n_heads"], "eps": c["rms_eps"], "lora_scale": c["lora_scale"],
+                "rope_theta": c["rope_theta"], "n_layers": n_layers}
+        return {"w": w, "ids": ids, "prompt": prompt, "resp": resp, "cfg": ocfg}
+
+    def oracle_time(self, smp, n_layers):
+        import oracle as O
+        t0 = time.perf_counter()
+        O.llama_score(smp["w"], smp["ids"], smp["prompt"], smp["cfg"], n_layers=n_layers,
+                      beta=self.beta, gamma=self.gamma, lam=self.lam)
+        return time.perf_counter() - t0
+
+    def oracle_throughput(self, steps=1):
+        """(tokens/s, description): the slice's pass time is t(0 layers) + 32 (t(1) - t(0))."""
+        smp = self.oracle_sample(1)
+        t_head = self.oracle_time(smp, 0)
+        t1 = [self.oracle_time(smp, 1) for _ in range(steps)]
+        n = self.cfg["n_layers"]
+        t_pass = [t_head + n * max(t - t_head, 0.0) for t in t1]
+        desc = (f"one sequence slice of {smp['prompt']} prompt + {smp['resp']} response tokens at full "
+                f"width through the fp64 oracle: embed + heads {t_head:.2f} s, one decoder layer "
+                f"{statistics.mean(t1) - t_head:.2f} s, pass time extrapolated to {n} layers")
+        return smp["resp"] * len(t_pass) / sum(t_pass), desc
+
+
+WORKLOADS = {LmHeadScoring.name: LmHeadScoring, HydraScoringLlama7B.name: HydraScoringLlama7B}
+DEFAULT_WORKLOAD = HydraScoringLlama7B.name
 
 
 # ----------------------------------------------------------------------------- helpers
@@ -270,6 +425,12 @@ def max_over_ranks(value, world, device=None):
     return float(t.item())
 
 
+def aggregate(units_per_rank_step, steps, world, ms_max):
+    """Whole-job throughput: every rank scores its own batch (weak scaling), so the job
+    processes units_per_rank_step * steps * world units in the max-over-ranks time."""
+    return units_per_rank_step * steps * world / (ms_max / 1e3)
+
+
 def barrier(world, device=None):
     if world > 1:
         import torch.distributed as dist
@@ -281,6 +442,11 @@ def barrier(world, device=None):
 
 def time_oracle(wl, target_s=12.0):
     """Oracle throughput on a bounded sample (rank 0, host cores)."""
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    if hasattr(wl, "oracle_throughput"):
+        value, desc = wl.oracle_throughput()
+        return {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                "sample": desc + "; BLAS threads = cores"}
     probe = wl.oracle_sample(8)
     t0 = time.perf_counter()
     wl.oracle_run(probe)
@@ -306,7 +472,23 @@ def run_reference(args, wl_cls):
     import torch
     if torch.cuda.is_available():
         torch.cuda.set_device(local)
-    wl = wl_cls("cuda" if torch.cuda.is_available() else "cpu")
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    if hasattr(wl_cls, "oracle_throughput"):
+        wl = wl_cls(dev, reference=True)
+        value, desc = wl.oracle_throughput(steps=args.steps)
+        t_step = wl.L / value
+        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_step * 1e3,
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+                "data": "synthetic", "impl": "reference", "config": wl.config(),
+                "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                                 "sample": desc},
+                "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}}
+        print(json.dumps(line), flush=True)
+        return 0
+    wl = wl_cls(dev)
     smp = wl.oracle_sample(16)
     for _ in range(args.warmup):
         wl.oracle_run(smp)
@@ -343,7 +525,7 @@ def run_ours(args, wl_cls):
     from paper_2309_00754_gb300 import hydra as H
     H.device_error(clear=True)
     peaks = load_peaks()
-    wl = wl_cls(device)
+    wl = wl_cls(device, seed=wl_cls.seed + 100 * rank)  # every rank scores its own batch
     steps = args.steps if args.steps is not None else wl.default_steps
     warmup = max(3, args.warmup if args.warmup is not None else wl.default_warmup)
 
@@ -353,9 +535,18 @@ def run_ours(args, wl_cls):
     if H.device_error(clear=True) != 0:
         raise RuntimeError("device error during warm-up")
 
+    driver = isinstance(wl, HydraScoringLlama7B)
     names = ("down", "gemm", "logp", "gae")
-    evs = [{n: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-            for n in names} for _ in range(steps)]
+    evs = [None] * steps
+    if driver:
+        # launch counts of one pass, then event timing of every launch of the timed steps
+        H.profile_enable(True)
+        wl.step()
+        wl.launch_counts = {k: n for k, (_, n) in H.profile_collect(reset=True).items()}
+        wl.launches_per_step = sum(wl.launch_counts.values())
+    else:
+        evs = [{n: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                for n in names} for _ in range(steps)]
     clocks = ClockSampler(local)
     barrier(world, device)
     torch.cuda.synchronize()
@@ -371,7 +562,11 @@ def run_ours(args, wl_cls):
     clk = clocks.stop()
     ms_total = start.elapsed_time(end)
     ms_total_max = max_over_ranks(ms_total, world, device)
-    per_kernel = {n: statistics.mean(e[n][0].elapsed_time(e[n][1]) for e in evs) for n in names}
+    if driver:
+        per_kernel = H.profile_collect(reset=True)
+        H.profile_enable(False)
+    else:
+        per_kernel = {n: statistics.mean(e[n][0].elapsed_time(e[n][1]) for e in evs) for n in names}
     if H.device_error(clear=True) != 0:
         raise RuntimeError("device error during the timed steps")
 
@@ -393,9 +588,8 @@ def run_ours(args, wl_cls):
     barrier(world, device)
     e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, device)
 
-    total_units = wl.units * steps * world
-    value = total_units / (ms_total_max / 1e3)
-    e2e_value = wl.units * e2e_steps * world / (e2e_ms / 1e3)
+    value = aggregate(wl.units, steps, world, ms_total_max)
+    e2e_value = aggregate(wl.units, e2e_steps, world, e2e_ms)
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": steps,
         "warmup": warmup, "ms_per_step": ms_total_max / steps, "higher_is_better": True,
@@ -430,7 +624,7 @@ def main(argv=None):
     wl_cls = WORKLOADS[args.workload]
     if args.impl == "reference":
         if args.steps is None:
-            args.steps = 20
+            args.steps = 3 if args.workload == HydraScoringLlama7B.name else 20
         if args.warmup is None:
             args.warmup = 3
         return run_reference(args, wl_cls)

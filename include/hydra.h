@@ -198,6 +198,135 @@ hydra_status ppo_gae(const float* rewards, const float* values, const int32_t* l
                      int64_t L, float gamma, float lam, float* advantages, float* returns,
                      void* stream);
 
+/* ===================================================================================
+ * Llama decoder pieces and the full scoring pass (the paper runs Llama 7b, §4; the pass
+ * follows the scoring steps of Algorithm 1, J-Hydra-PPO). The LoRA-off and LoRA-on streams
+ * are stacked row-wise: rows [0, T) are the off stream, rows [T, 2T) the on stream, where
+ * T = S * P for S sequences of P tokens. Residual stream fp32, matmul operands bf16.
+ * =================================================================================== */
+
+/* h[(c T + t), :] = table[ids[t], :] (bf16 -> fp32) for every copy c < copies.
+ * table bf16 [V, d], ids int32 [T] in [0, V) (out of range: NaN row + device error),
+ * h fp32 [copies * T, d]. d % 8 == 0. */
+hydra_status hydra_embed(const void* table, int64_t V, int64_t d, const int32_t* ids, int64_t T,
+                         int copies, float* h, void* stream);
+
+/* RMSNorm (Zhang & Sennrich 2019): y[i] = bf16(x[j] / sqrt(mean(x[j]^2) + eps) * w) with
+ * row gather j = (i / g_out) * g_in + off + i % g_out (g_out = g_in = rows, off = 0 for the
+ * identity). x fp32 [*, d], w bf16 [d], y bf16 [rows, d]. d % 8 == 0. */
+hydra_status hydra_rmsnorm(const float* x, const void* w, int64_t rows, int64_t d, float eps,
+                           int64_t g_out, int64_t g_in, int64_t off, void* y, void* stream);
+
+/* Rotary embedding (Su et al. 2021), rotate-half pairing, in place on the q block
+ * (columns [0, d)) and k block ([d, 2d)) of each row of qkv (bf16 [R, ld]): dims (i, i + Dh/2)
+ * of every head rotate by pos * theta^(-2i/Dh), pos = row % P. */
+hydra_status hydra_rope(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t head_dim, int64_t P,
+                        float theta, void* stream);
+
+/* Causal attention, out = softmax(q k^T / sqrt(Dh) + causal mask) v per head, for nseq
+ * sequences of P rows each: q, k, v are column blocks [0, d), [d, 2d), [2d, 3d) of qkv
+ * (bf16, row stride ld), out bf16 with row stride ld_out. head_dim must be 128. */
+hydra_status hydra_causal_attention(const void* qkv, int64_t nseq, int64_t P, int64_t ld,
+                                    int64_t n_heads, int64_t head_dim, void* out, int64_t ld_out,
+                                    void* stream);
+
+/* SwiGLU (Shazeer 2020): m = bf16(silu(g) * u), gu bf16 [R, 2F] = [gate | up], m [R, F]. */
+hydra_status hydra_swiglu(const void* gu, int64_t R, int64_t F, void* m, void* stream);
+
+/* h += float(y) over n elements (h fp32, y bf16, n % 8 == 0). */
+hydra_status hydra_residual_add(float* h, const void* y, int64_t n, void* stream);
+
+/* Scalar head (reward model / value head): out[i] = sum_k x[j, k] w[k] with the row gather
+ * of hydra_rmsnorm. x bf16, w bf16 [d], out fp32 [n]. */
+hydra_status hydra_head_dot(const void* x, int64_t d, const void* w, int64_t n, int64_t g_out,
+                            int64_t g_in, int64_t off, float* out, void* stream);
+
+typedef struct hydra_llama_config {
+  int64_t n_layers, d_model, n_heads, head_dim, ffn, vocab;
+  int64_t prompt_len;   /* P0: prompt tokens per sequence */
+  int64_t response_len; /* L: response slots per sequence (each sequence is P0 + L tokens) */
+  int64_t lora_rank;    /* r of every adapted linear (q, v, gate, up, down) */
+  float lora_scale, rms_eps, rope_theta;
+  float beta, gamma, lam; /* KL coefficient, GAE discount and lambda */
+} hydra_llama_config;
+
+/* One decoder layer, fused layouts (device pointers, bf16):
+ *   w_qkv [3d, d] = [Wq; Wk; Wv]        a_qv [2r, d] = [Aq; Av]
+ *   b_qkv [3d, 2r] = [[Bq, 0]; [0, 0]; [0, Bv]]   (LoRA on q and v only)
+ *   w_o [d, d] (no LoRA)
+ *   w_gu [2F, d] = [W_gate; W_up]       a_gu [2r, d] = [A_gate; A_up]
+ *   b_gu [2F, 2r] = [[B_gate, 0]; [0, B_up]]
+ *   w_down [d, F], a_down [r, F], b_down [d, r]
+ *   norm_attn, norm_ffn [d] */
+typedef struct hydra_llama_layer {
+  const void* w_qkv;
+  const void* a_qv;
+  const void* b_qkv;
+  const void* w_o;
+  const void* w_gu;
+  const void* a_gu;
+  const void* b_gu;
+  const void* w_down;
+  const void* a_down;
+  const void* b_down;
+  const void* norm_attn;
+  const void* norm_ffn;
+} hydra_llama_layer;
+
+typedef struct hydra_llama_weights {
+  const void* embed;               /* bf16 [V, d] */
+  const hydra_llama_layer* layers; /* HOST array of n_layers entries */
+  const void* final_norm;          /* bf16 [d] */
+  const void* lm_head;             /* bf16 [V, d] */
+  const void* w_rm;                /* bf16 [d]: reward-model head; also the value head */
+} hydra_llama_weights;
+
+/* Workspace bytes of hydra_score_llama for S sequences. */
+size_t hydra_score_llama_workspace_size(const hydra_llama_config* cfg, int64_t S);
+
+/*
+ * The full J-Hydra scoring pass (Algorithm 1: the LoRA-off model gives the reference
+ * log-probabilities and the reward; §3 Dynamic LoRA; J-Hydra uses one LoRA set for actor
+ * and critic) over S sequences of P0 prompt + L response tokens:
+ *   both streams through n_layers Llama blocks (q/v/gate/up/down carry LoRA, k/o/LM head
+ *   do not) -> final RMSNorm -> LM head on the rows predicting response tokens ->
+ *   logp_actor (LoRA on), logp_ref (LoRA off) -> score_s = w_rm . h_off[P0 + len_s - 1],
+ *   values_t = w_rm . h_on[P0 + t - 1] -> reward_t = -beta (la - lr) + [t = len-1] score
+ *   -> GAE advantages and returns.
+ * ids int32 [S, P0 + L]; lengths int32 [S] valid response tokens (0..L) or NULL (all L).
+ * Outputs fp32 [S, L] (0 at t >= len): logp_actor, logp_ref, reward, values, advantages,
+ * returns; score fp32 [S]. Requirements: head_dim == 128, d == n_heads * 128,
+ * ffn % 8 == 0, vocab % 8 == 0, r % 8 == 0, 8 <= r <= 128, P0 >= 1, L >= 1.
+ */
+hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_weights* w,
+                               const int32_t* ids, const int32_t* lengths, int64_t S,
+                               void* workspace, size_t workspace_bytes, float* logp_actor,
+                               float* logp_ref, float* reward, float* values, float* advantages,
+                               float* returns, float* score, void* stream);
+
+/* Kernel classes of the optional launch timing of hydra_score_llama. */
+enum {
+  HYDRA_PROF_GEMM = 0,        /* tcgen05 dual-output linear (or the small-M GEMV) */
+  HYDRA_PROF_LORA_DOWN = 1,   /* u = s x A^T */
+  HYDRA_PROF_ATTENTION = 2,   /* causal attention */
+  HYDRA_PROF_ELEMENTWISE = 3, /* embedding, RMSNorm, RoPE, SwiGLU, residual add */
+  HYDRA_PROF_LOGPROBS = 4,    /* log-softmax + gather + KL reward */
+  HYDRA_PROF_GAE = 5,         /* GAE scan */
+  HYDRA_PROF_HEADS = 6,       /* reward-model score and value head */
+  HYDRA_PROF_CLASSES = 7
+};
+
+/*
+ * Launch timing of hydra_score_llama. While enabled, every kernel launch of the pass is
+ * bracketed by CUDA events recorded on the call's stream (host-side overhead only; the
+ * events come from a library pool created on first use). hydra_profile_collect waits for
+ * the recorded events, writes the summed milliseconds and launch counts per class into
+ * ms[HYDRA_PROF_CLASSES] and launches[HYDRA_PROF_CLASSES] (host arrays), and with reset
+ * != 0 starts a new collection. This is measurement support, not part of the paper.
+ */
+hydra_status hydra_profile_enable(int on);
+hydra_status hydra_profile_collect(float* ms, int64_t* launches, int reset);
+
 #ifdef __cplusplus
 }
 #endif

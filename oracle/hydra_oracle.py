@@ -33,6 +33,8 @@ Readings where the paper is silent (the same readings the CUDA path implements):
 
 Parity pins for every function live in tests/test_oracle_pins.py (closed forms,
 invariants, brute force, library routines, hand-worked fixtures in tests/golden/).
+`set_storage_dither` (off by default) is a sensitivity probe used to derive the end-to-end
+tolerance of the multi-layer composition; it never changes the default results.
 The full 32-layer Llama composition (`llama_score`) is pinned only through its per-op
 pieces and small-size invariants: parity unpinned for the composition as a whole.
 """
@@ -60,8 +62,25 @@ def f64_to_bf16_bits(x) -> np.ndarray:
     return u.astype(np.uint16)
 
 
+_DITHER = {"eps": 0.0, "rng": None}
+
+
+def set_storage_dither(eps, seed=0):
+    """Sensitivity probe (off by default): with eps > 0 every value is multiplied by
+    (1 + eps * xi), xi = +-1 at random, before it is stored as bf16. A real fp32 kernel
+    reaches each stored value through an accumulation order that differs from the exact
+    fp64 sum by a relative amount of this size, so two dithered runs show how far equally
+    valid roundings of the same chain drift apart. eps = 0 restores the plain oracle."""
+    _DITHER["eps"] = float(eps)
+    _DITHER["rng"] = np.random.default_rng(seed) if eps > 0 else None
+
+
 def round_bf16(x) -> np.ndarray:
     """Value of x after storing it as bf16 (float64 result)."""
+    if _DITHER["eps"] > 0:
+        x = np.asarray(x, dtype=np.float64)
+        xi = _DITHER["rng"].integers(0, 2, size=x.shape) * 2.0 - 1.0
+        x = x * (1.0 + _DITHER["eps"] * xi)
     return bf16_to_f64(f64_to_bf16_bits(x))
 
 

@@ -14,7 +14,12 @@ __device__ int g_hydra_err = 0;
 constexpr int kMaxDevices = 64;
 int* g_err_ptr[kMaxDevices] = {nullptr};
 
-int* device_err_ptr() {
+}  // namespace
+
+namespace hydra {
+
+// Device address of the library's error word on the current device (resolved once).
+int* device_error_word() {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
   if (g_err_ptr[dev] == nullptr) {
@@ -24,6 +29,10 @@ int* device_err_ptr() {
   }
   return g_err_ptr[dev];
 }
+
+}  // namespace hydra
+
+namespace {
 
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
@@ -60,7 +69,7 @@ hydra_status lora_linear_impl(const void* x_off, const void* x_on, int64_t M, in
   if (algo == 2 && rows > hydra::kGemvMaxRows) return HYDRA_ERR_SHAPE;
   if (M == 0) return HYDRA_OK;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  int* err = device_err_ptr();
+  int* err = hydra::device_error_word();
   if (err == nullptr) return HYDRA_ERR_CUDA;
 
   const void* xo = shared_x ? x_off : x_on;
@@ -177,10 +186,10 @@ hydra_status hydra_token_logprobs_kl(const void* logits_actor, const void* logit
   if (logits_actor == nullptr || logits_ref == nullptr || ids == nullptr ||
       logp_actor == nullptr || logp_ref == nullptr || reward_tok == nullptr)
     return HYDRA_ERR_NULL;
-  int* err = device_err_ptr();
+  int* err = hydra::device_error_word();
   if (err == nullptr) return HYDRA_ERR_CUDA;
   return hydra::launch_token_logprobs_kl(logits_actor, logits_ref, logits_dtype == HYDRA_BF16, S, L,
-                                         V, ld, ids, lengths, seq_score, beta, logp_actor, logp_ref,
+                                         V, ld, ids, L, lengths, seq_score, beta, logp_actor, logp_ref,
                                          reward_tok, lse_actor, lse_ref, err,
                                          static_cast<cudaStream_t>(stream)) == 0
              ? HYDRA_OK
@@ -195,7 +204,7 @@ hydra_status ppo_gae(const float* rewards, const float* values, const int32_t* l
   if (S == 0 || L == 0) return HYDRA_OK;
   if (rewards == nullptr || values == nullptr || advantages == nullptr || returns == nullptr)
     return HYDRA_ERR_NULL;
-  int* err = device_err_ptr();
+  int* err = hydra::device_error_word();
   if (err == nullptr) return HYDRA_ERR_CUDA;
   return hydra::launch_gae(rewards, values, lengths, S, L, gamma, lam, advantages, returns, err,
                            static_cast<cudaStream_t>(stream)) == 0

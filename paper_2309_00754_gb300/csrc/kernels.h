@@ -25,16 +25,43 @@ struct GemmArgs {
   int* err;
 };
 
+// Device address of the library's error word on the current device (NULL on failure).
+int* device_error_word();
+
 int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream);
 int launch_dual_lora_gemv(const GemmArgs& a, cudaStream_t stream);
 int launch_lora_down(const void* x, int64_t M, int64_t K, const void* A, int64_t r, float s,
                      void* u, cudaStream_t stream);
+// ids of sequence s start at ids + s * ids_ld (ids_ld = L for a dense [S, L] array)
 int launch_token_logprobs_kl(const void* za, const void* zr, int bf16_logits, int64_t S, int64_t L,
-                             int64_t V, int64_t ld, const int32_t* ids, const int32_t* lengths,
+                             int64_t V, int64_t ld, const int32_t* ids, int64_t ids_ld,
+                             const int32_t* lengths,
                              const float* score, float beta, float* la, float* lr, float* rew,
                              float* lse_a, float* lse_r, int* err, cudaStream_t stream);
 int launch_gae(const float* r, const float* v, const int32_t* lengths, int64_t S, int64_t L,
                float gamma, float lam, float* adv, float* ret, int* err, cudaStream_t stream);
+
+// Row gather used by the per-row Llama kernels: output row i reads input row
+// (i / g_out) * g_in + off + i % g_out (g_out = g_in, off = 0 is the identity).
+struct RowMap {
+  long long g_out, g_in, off;
+};
+
+int launch_embed(const void* table, int64_t V, int64_t d, const int32_t* ids, int64_t T,
+                 int copies, float* h, int* err, cudaStream_t st);
+int launch_rmsnorm(const float* x, const void* w, int64_t rows, int64_t d, float eps,
+                   const RowMap& map, void* y, cudaStream_t st);
+int launch_rope(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t Dh, int64_t P, float theta,
+                cudaStream_t st);
+int launch_swiglu(const void* gu, int64_t R, int64_t F, void* m, cudaStream_t st);
+int launch_residual_add(float* h, const void* y, int64_t n, cudaStream_t st);
+int launch_head_dot(const void* x, int64_t d, const void* w, const RowMap& map, int64_t n,
+                    const int32_t* lengths, int64_t L, float* out, cudaStream_t st);
+int launch_seq_score(const float* h, const void* norm, const void* w, int64_t d, float eps,
+                     const int32_t* lengths, int64_t S, int64_t L, int64_t P, int64_t p0,
+                     float* score, cudaStream_t st);
+int launch_causal_attention(const void* qkv, int64_t nseq, int64_t P, int64_t ld, int64_t n_heads,
+                            int64_t head_dim, void* out, int64_t ld_out, cudaStream_t st);
 
 // Largest sequence length the shared-memory GAE scan accepts.
 constexpr int64_t kGaeMaxL = 16384;

@@ -71,7 +71,7 @@ struct Vec<__nv_bfloat16> {
 template <typename T, bool kVec>
 __global__ void __launch_bounds__(kThreads)
     logprobs_kl_kernel(const T* __restrict__ za, const T* __restrict__ zr, int L, int V,
-                       long long ld, const int32_t* __restrict__ ids,
+                       long long ld, const int32_t* __restrict__ ids, long long ids_ld,
                        const int32_t* __restrict__ lengths, const float* __restrict__ score,
                        float beta, float* __restrict__ la, float* __restrict__ lr,
                        float* __restrict__ rew, float* __restrict__ lse_a,
@@ -143,7 +143,7 @@ __global__ void __launch_bounds__(kThreads)
     }
     const float lsa = ma + logf(sa);
     const float lsr = mr + logf(sr);
-    const int id = ids[row];
+    const int id = ids[static_cast<long long>(s) * ids_ld + t];
     float va, vr, rw;
     if (id < 0 || id >= V) {
       record_error(err, kDevBadTokenId);
@@ -164,7 +164,7 @@ __global__ void __launch_bounds__(kThreads)
 
 template <typename T>
 int launch_t(const void* za, const void* zr, int64_t S, int64_t L, int64_t V, int64_t ld,
-             const int32_t* ids, const int32_t* lengths, const float* score, float beta, float* la,
+             const int32_t* ids, int64_t ids_ld, const int32_t* lengths, const float* score, float beta, float* la,
              float* lr, float* rew, float* lse_a, float* lse_r, int* err, cudaStream_t stream) {
   const T* a = static_cast<const T*>(za);
   const T* r = static_cast<const T*>(zr);
@@ -174,11 +174,11 @@ int launch_t(const void* za, const void* zr, int64_t S, int64_t L, int64_t V, in
   const unsigned grid = static_cast<unsigned>(S * L);
   if (vec)
     logprobs_kl_kernel<T, true><<<grid, kThreads, 0, stream>>>(
-        a, r, static_cast<int>(L), static_cast<int>(V), ld, ids, lengths, score, beta, la, lr, rew,
+        a, r, static_cast<int>(L), static_cast<int>(V), ld, ids, ids_ld, lengths, score, beta, la, lr, rew,
         lse_a, lse_r, err);
   else
     logprobs_kl_kernel<T, false><<<grid, kThreads, 0, stream>>>(
-        a, r, static_cast<int>(L), static_cast<int>(V), ld, ids, lengths, score, beta, la, lr, rew,
+        a, r, static_cast<int>(L), static_cast<int>(V), ld, ids, ids_ld, lengths, score, beta, la, lr, rew,
         lse_a, lse_r, err);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
 }
@@ -186,14 +186,15 @@ int launch_t(const void* za, const void* zr, int64_t S, int64_t L, int64_t V, in
 }  // namespace
 
 int launch_token_logprobs_kl(const void* za, const void* zr, int bf16_logits, int64_t S, int64_t L,
-                             int64_t V, int64_t ld, const int32_t* ids, const int32_t* lengths,
-                             const float* score, float beta, float* la, float* lr, float* rew,
-                             float* lse_a, float* lse_r, int* err, cudaStream_t stream) {
+                             int64_t V, int64_t ld, const int32_t* ids, int64_t ids_ld,
+                             const int32_t* lengths, const float* score, float beta, float* la,
+                             float* lr, float* rew, float* lse_a, float* lse_r, int* err,
+                             cudaStream_t stream) {
   if (S == 0 || L == 0) return 0;
   if (bf16_logits)
-    return launch_t<__nv_bfloat16>(za, zr, S, L, V, ld, ids, lengths, score, beta, la, lr, rew,
+    return launch_t<__nv_bfloat16>(za, zr, S, L, V, ld, ids, ids_ld, lengths, score, beta, la, lr, rew,
                                    lse_a, lse_r, err, stream);
-  return launch_t<float>(za, zr, S, L, V, ld, ids, lengths, score, beta, la, lr, rew, lse_a, lse_r,
+  return launch_t<float>(za, zr, S, L, V, ld, ids, ids_ld, lengths, score, beta, la, lr, rew, lse_a, lse_r,
                          err, stream);
 }
 

@@ -1,0 +1,350 @@
+// C-ABI of the Llama decoder pieces and the native host driver of the full J-Hydra scoring
+// pass (Algorithm 1 scoring steps; §3 Dynamic LoRA and J-Hydra-PPO: one frozen base, the
+// LoRA-off stream gives the reference policy and the reward model, the LoRA-on stream the
+// actor and the critic). Both streams' rows are stacked so every kernel covers both in one
+// launch and each projection's W tiles are fetched from HBM once.
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <mutex>
+#include <vector>
+
+#include "../../include/hydra.h"
+#include "kernels.h"
+
+namespace {
+
+// ---------------------------------------------------------------- kernel-class timing
+// When enabled, hydra_score_llama brackets every launch with CUDA events recorded on the
+// call's stream; hydra_profile_collect sums the elapsed times per kernel class. Events come
+// from a pool that grows on demand and is reused after each collect.
+struct Profiler {
+  bool on = false;
+  std::vector<cudaEvent_t> pool;
+  size_t used = 0;
+  std::vector<int> cls;  // class of event pair i (events 2i, 2i + 1)
+  std::mutex mu;
+} g_prof;
+
+cudaEvent_t prof_event() {
+  if (g_prof.used == g_prof.pool.size()) {
+    cudaEvent_t e;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    g_prof.pool.push_back(e);
+  }
+  return g_prof.pool[g_prof.used++];
+}
+
+struct ProfScope {
+  cudaStream_t st;
+  bool active;
+  ProfScope(int c, cudaStream_t s) : st(s), active(g_prof.on) {
+    if (!active) return;
+    cudaEvent_t e = prof_event();
+    if (e == nullptr) {
+      active = false;
+      return;
+    }
+    g_prof.cls.push_back(c);
+    cudaEventRecord(e, st);
+  }
+  ~ProfScope() {
+    if (!active) return;
+    cudaEvent_t e = prof_event();
+    if (e != nullptr) cudaEventRecord(e, st);
+  }
+};
+
+inline bool a16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+inline size_t up256(size_t v) { return (v + 255) / 256 * 256; }
+inline hydra_status rc(int r) { return r == 0 ? HYDRA_OK : HYDRA_ERR_CUDA; }
+
+// Workspace layout of the full pass, in bytes from the workspace base.
+struct PassLayout {
+  size_t h, a, qkv, attn, y, gu, m, u, fin, logits, sc, total;
+};
+
+PassLayout layout(const hydra_llama_config& c, int64_t S) {
+  const size_t P = static_cast<size_t>(c.prompt_len + c.response_len);
+  const size_t T = static_cast<size_t>(S) * P;
+  const size_t R = 2 * T;
+  const size_t d = static_cast<size_t>(c.d_model), F = static_cast<size_t>(c.ffn);
+  const size_t SL = static_cast<size_t>(S) * static_cast<size_t>(c.response_len);
+  PassLayout L;
+  size_t o = 0;
+  L.h = o;      o += up256(R * d * 4);
+  L.a = o;      o += up256(R * d * 2);
+  L.qkv = o;    o += up256(R * 3 * d * 2);
+  L.attn = o;   o += up256(R * d * 2);
+  L.y = o;      o += up256(R * d * 2);
+  L.gu = o;     o += up256(R * 2 * F * 2);
+  L.m = o;      o += up256(R * F * 2);
+  L.u = o;      o += up256(T * 2 * static_cast<size_t>(c.lora_rank) * 2);
+  L.fin = o;    o += up256(2 * SL * d * 2);
+  L.logits = o; o += up256(2 * SL * static_cast<size_t>(c.vocab) * 4);
+  L.sc = o;     o += up256(static_cast<size_t>(S) * 4);
+  L.total = o;
+  return L;
+}
+
+bool valid_config(const hydra_llama_config* c) {
+  if (c == nullptr) return false;
+  if (c->n_layers < 1 || c->head_dim != 128 || c->n_heads < 1) return false;
+  if (c->d_model != c->n_heads * c->head_dim) return false;
+  if (c->ffn < 8 || c->ffn % 8 != 0 || c->vocab < 8 || c->vocab % 8 != 0) return false;
+  if (c->lora_rank < 8 || c->lora_rank > 128 || c->lora_rank % 8 != 0) return false;
+  if (c->prompt_len < 1 || c->response_len < 1) return false;
+  if (c->response_len > hydra::kGaeMaxL) return false;
+  return true;
+}
+
+// stacked dual linear: rows [0, T) of x are the off stream, [T, 2T) the on stream
+int stacked_linear(const void* x, int64_t T, int64_t K, int64_t N, const void* W, const void* A,
+                   const void* B, int64_t r, float s, void* u, void* y, bool f32, int* err,
+                   cudaStream_t st) {
+  const size_t xs = static_cast<size_t>(T) * K * 2;
+  const size_t ys = static_cast<size_t>(T) * N * (f32 ? 4 : 2);
+  const void* x_off = x;
+  const void* x_on = static_cast<const uint8_t*>(x) + xs;
+  if (r > 0) {
+    ProfScope ps(HYDRA_PROF_LORA_DOWN, st);
+    const int e = hydra::launch_lora_down(x_on, T, K, A, r, s, u, st);
+    if (e != 0) return e;
+  }
+  ProfScope ps(HYDRA_PROF_GEMM, st);
+  hydra::GemmArgs g;
+  g.x_off = x_off;
+  g.x_on = x_on;
+  g.M = T;
+  g.K = K;
+  g.N = N;
+  g.W = W;
+  g.u = r > 0 ? u : nullptr;
+  g.B = r > 0 ? B : nullptr;
+  g.r = r;
+  g.shared_x = false;
+  g.y_off = y;
+  g.y_on = static_cast<uint8_t*>(y) + ys;
+  g.out_f32 = f32 ? 1 : 0;
+  g.err = err;
+  return (2 * T <= hydra::kGemvMaxRows) ? hydra::launch_dual_lora_gemv(g, st)
+                                        : hydra::launch_dual_lora_gemm_tc(g, st);
+}
+
+}  // namespace
+
+extern "C" {
+
+hydra_status hydra_embed(const void* table, int64_t V, int64_t d, const int32_t* ids, int64_t T,
+                         int copies, float* h, void* stream) {
+  if (table == nullptr || ids == nullptr || h == nullptr) return HYDRA_ERR_NULL;
+  if (V < 1 || d < 8 || T < 0 || copies < 1 || copies > 2) return HYDRA_ERR_SHAPE;
+  if (d % 8 != 0 || !a16(table) || !a16(h)) return HYDRA_ERR_ALIGN;
+  int* err = hydra::device_error_word();
+  if (err == nullptr) return HYDRA_ERR_CUDA;
+  return rc(hydra::launch_embed(table, V, d, ids, T, copies, h, err,
+                                static_cast<cudaStream_t>(stream)));
+}
+
+hydra_status hydra_rmsnorm(const float* x, const void* w, int64_t rows, int64_t d, float eps,
+                           int64_t g_out, int64_t g_in, int64_t off, void* y, void* stream) {
+  if (x == nullptr || w == nullptr || y == nullptr) return HYDRA_ERR_NULL;
+  if (rows < 0 || d < 8 || g_out < 1 || g_in < 0 || off < 0) return HYDRA_ERR_SHAPE;
+  if (d % 8 != 0 || !a16(x) || !a16(w) || !a16(y)) return HYDRA_ERR_ALIGN;
+  hydra::RowMap m{g_out, g_in, off};
+  return rc(hydra::launch_rmsnorm(x, w, rows, d, eps, m, y, static_cast<cudaStream_t>(stream)));
+}
+
+hydra_status hydra_rope(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t head_dim, int64_t P,
+                        float theta, void* stream) {
+  if (qkv == nullptr) return HYDRA_ERR_NULL;
+  if (R < 0 || P < 1 || head_dim < 2 || head_dim % 2 != 0 || d % head_dim != 0 || ld < 2 * d)
+    return HYDRA_ERR_SHAPE;
+  if (!(theta > 0.f)) return HYDRA_ERR_RANGE;
+  return rc(hydra::launch_rope(qkv, R, ld, d, head_dim, P, theta, static_cast<cudaStream_t>(stream)));
+}
+
+hydra_status hydra_causal_attention(const void* qkv, int64_t nseq, int64_t P, int64_t ld,
+                                    int64_t n_heads, int64_t head_dim, void* out, int64_t ld_out,
+                                    void* stream) {
+  if (qkv == nullptr || out == nullptr) return HYDRA_ERR_NULL;
+  if (head_dim != 128) return HYDRA_ERR_SHAPE;
+  if (nseq < 0 || P < 0 || n_heads < 1 || ld < 3 * n_heads * head_dim ||
+      ld_out < n_heads * head_dim)
+    return HYDRA_ERR_SHAPE;
+  if (ld % 8 != 0 || ld_out % 2 != 0 || !a16(qkv) || !a16(out)) return HYDRA_ERR_ALIGN;
+  return rc(hydra::launch_causal_attention(qkv, nseq, P, ld, n_heads, head_dim, out, ld_out,
+                                           static_cast<cudaStream_t>(stream)));
+}
+
+hydra_status hydra_swiglu(const void* gu, int64_t R, int64_t F, void* m, void* stream) {
+  if (gu == nullptr || m == nullptr) return HYDRA_ERR_NULL;
+  if (R < 0 || F < 8) return HYDRA_ERR_SHAPE;
+  if (F % 8 != 0 || !a16(gu) || !a16(m)) return HYDRA_ERR_ALIGN;
+  return rc(hydra::launch_swiglu(gu, R, F, m, static_cast<cudaStream_t>(stream)));
+}
+
+hydra_status hydra_residual_add(float* h, const void* y, int64_t n, void* stream) {
+  if (h == nullptr || y == nullptr) return HYDRA_ERR_NULL;
+  if (n < 0) return HYDRA_ERR_SHAPE;
+  if (n % 8 != 0 || !a16(h) || !a16(y)) return HYDRA_ERR_ALIGN;
+  return rc(hydra::launch_residual_add(h, y, n, static_cast<cudaStream_t>(stream)));
+}
+
+hydra_status hydra_head_dot(const void* x, int64_t d, const void* w, int64_t n, int64_t g_out,
+                            int64_t g_in, int64_t off, float* out, void* stream) {
+  if (x == nullptr || w == nullptr || out == nullptr) return HYDRA_ERR_NULL;
+  if (n < 0 || d < 8 || g_out < 1 || g_in < 0 || off < 0) return HYDRA_ERR_SHAPE;
+  if (d % 8 != 0 || !a16(x) || !a16(w)) return HYDRA_ERR_ALIGN;
+  hydra::RowMap m{g_out, g_in, off};
+  return rc(hydra::launch_head_dot(x, d, w, m, n, nullptr, 1, out,
+                                   static_cast<cudaStream_t>(stream)));
+}
+
+hydra_status hydra_profile_enable(int on) {
+  std::lock_guard<std::mutex> lock(g_prof.mu);
+  g_prof.on = on != 0;
+  return HYDRA_OK;
+}
+
+hydra_status hydra_profile_collect(float* ms, int64_t* launches, int reset) {
+  if (ms == nullptr || launches == nullptr) return HYDRA_ERR_NULL;
+  std::lock_guard<std::mutex> lock(g_prof.mu);
+  for (int c = 0; c < HYDRA_PROF_CLASSES; ++c) {
+    ms[c] = 0.f;
+    launches[c] = 0;
+  }
+  for (size_t i = 0; i < g_prof.cls.size(); ++i) {
+    if (2 * i + 1 >= g_prof.used) break;
+    cudaEvent_t a = g_prof.pool[2 * i], b = g_prof.pool[2 * i + 1];
+    if (cudaEventSynchronize(b) != cudaSuccess) return HYDRA_ERR_CUDA;
+    float t = 0.f;
+    if (cudaEventElapsedTime(&t, a, b) != cudaSuccess) return HYDRA_ERR_CUDA;
+    ms[g_prof.cls[i]] += t;
+    launches[g_prof.cls[i]] += 1;
+  }
+  if (reset) {
+    g_prof.cls.clear();
+    g_prof.used = 0;
+  }
+  return HYDRA_OK;
+}
+
+size_t hydra_score_llama_workspace_size(const hydra_llama_config* cfg, int64_t S) {
+  if (!valid_config(cfg) || S < 0) return 0;
+  return layout(*cfg, S).total;
+}
+
+hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_weights* w,
+                               const int32_t* ids, const int32_t* lengths, int64_t S,
+                               void* workspace, size_t workspace_bytes, float* logp_actor,
+                               float* logp_ref, float* reward, float* values, float* advantages,
+                               float* returns, float* score, void* stream) {
+  if (cfg == nullptr || w == nullptr) return HYDRA_ERR_NULL;
+  if (!valid_config(cfg)) return HYDRA_ERR_SHAPE;
+  if (S < 0) return HYDRA_ERR_SHAPE;
+  if (S == 0) return HYDRA_OK;
+  if (ids == nullptr || logp_actor == nullptr || logp_ref == nullptr || reward == nullptr ||
+      values == nullptr || advantages == nullptr || returns == nullptr || score == nullptr)
+    return HYDRA_ERR_NULL;
+  if (w->embed == nullptr || w->layers == nullptr || w->final_norm == nullptr ||
+      w->lm_head == nullptr || w->w_rm == nullptr)
+    return HYDRA_ERR_NULL;
+  const hydra_llama_config& c = *cfg;
+  for (int64_t l = 0; l < c.n_layers; ++l) {
+    const hydra_llama_layer& ly = w->layers[l];
+    const void* ptrs[] = {ly.w_qkv, ly.a_qv, ly.b_qkv, ly.w_o, ly.w_gu, ly.a_gu,
+                          ly.b_gu, ly.w_down, ly.a_down, ly.b_down, ly.norm_attn, ly.norm_ffn};
+    for (const void* p : ptrs) {
+      if (p == nullptr) return HYDRA_ERR_NULL;
+      if (!a16(p)) return HYDRA_ERR_ALIGN;
+    }
+  }
+  const PassLayout Lo = layout(c, S);
+  if (workspace == nullptr) return HYDRA_ERR_WORKSPACE;
+  if (!a16(workspace)) return HYDRA_ERR_ALIGN;
+  if (workspace_bytes < Lo.total) return HYDRA_ERR_WORKSPACE;
+  int* err = hydra::device_error_word();
+  if (err == nullptr) return HYDRA_ERR_CUDA;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  std::unique_lock<std::mutex> prof_lock(g_prof.mu, std::defer_lock);
+  if (g_prof.on) prof_lock.lock();
+
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  float* h = reinterpret_cast<float*>(ws + Lo.h);
+  void* a = ws + Lo.a;
+  void* qkv = ws + Lo.qkv;
+  void* attn = ws + Lo.attn;
+  void* y = ws + Lo.y;
+  void* gu = ws + Lo.gu;
+  void* m = ws + Lo.m;
+  void* u = ws + Lo.u;
+  void* fin = ws + Lo.fin;
+  float* logits = reinterpret_cast<float*>(ws + Lo.logits);
+  float* sc = reinterpret_cast<float*>(ws + Lo.sc);
+
+  const int64_t P = c.prompt_len + c.response_len;
+  const int64_t T = S * P;
+  const int64_t R = 2 * T;
+  const int64_t d = c.d_model, F = c.ffn, V = c.vocab, r = c.lora_rank, L = c.response_len;
+  const int64_t SL = S * L;
+  const float s = c.lora_scale;
+  const hydra::RowMap ident{R, R, 0};
+  int e = 0;
+#define HY_TRY(x)                     \
+  do {                                \
+    if ((e = (x)) != 0) return rc(e); \
+  } while (0)
+#define HY_PROF(cls, x)        \
+  do {                         \
+    ProfScope ps_(cls, st);    \
+    HY_TRY(x);                 \
+  } while (0)
+
+  HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_embed(w->embed, V, d, ids, T, 2, h, err, st));
+  for (int64_t l = 0; l < c.n_layers; ++l) {
+    const hydra_llama_layer& ly = w->layers[l];
+    // attention block
+    HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(h, ly.norm_attn, R, d, c.rms_eps, ident, a, st));
+    HY_TRY(stacked_linear(a, T, d, 3 * d, ly.w_qkv, ly.a_qv, ly.b_qkv, 2 * r, s, u, qkv, false,
+                          err, st));
+    HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rope(qkv, R, 3 * d, d, c.head_dim, P, c.rope_theta, st));
+    HY_PROF(HYDRA_PROF_ATTENTION,
+            hydra::launch_causal_attention(qkv, 2 * S, P, 3 * d, c.n_heads, c.head_dim, attn, d, st));
+    HY_TRY(stacked_linear(attn, T, d, d, ly.w_o, nullptr, nullptr, 0, s, u, y, false, err, st));
+    HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_residual_add(h, y, R * d, st));
+    // feed-forward block
+    HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(h, ly.norm_ffn, R, d, c.rms_eps, ident, a, st));
+    HY_TRY(stacked_linear(a, T, d, 2 * F, ly.w_gu, ly.a_gu, ly.b_gu, 2 * r, s, u, gu, false, err, st));
+    HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_swiglu(gu, R, F, m, st));
+    HY_TRY(stacked_linear(m, T, F, d, ly.w_down, ly.a_down, ly.b_down, r, s, u, y, false, err, st));
+    HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_residual_add(h, y, R * d, st));
+  }
+  // final norm on the rows that predict response tokens: row P0 - 1 + t of each sequence
+  const hydra::RowMap resp{L, P, c.prompt_len - 1};
+  HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(h, w->final_norm, 2 * SL, d, c.rms_eps, resp, fin, st));
+  HY_TRY(stacked_linear(fin, SL, d, V, w->lm_head, nullptr, nullptr, 0, s, u, logits, true, err, st));
+  // reward-model score on the LoRA-off stream at the last valid token; values on the
+  // LoRA-on stream (the same head: r_phi = LO(V))
+  HY_PROF(HYDRA_PROF_HEADS, hydra::launch_seq_score(h, w->final_norm, w->w_rm, d, c.rms_eps,
+                                                    lengths, S, L, P, c.prompt_len, sc, st));
+  const void* fin_on = static_cast<uint8_t*>(fin) + static_cast<size_t>(SL) * d * 2;
+  const hydra::RowMap dense{SL, SL, 0};
+  HY_PROF(HYDRA_PROF_HEADS, hydra::launch_head_dot(fin_on, d, w->w_rm, dense, SL, lengths, L, values, st));
+  const float* z_ref = logits;
+  const float* z_act = logits + static_cast<size_t>(SL) * V;
+  HY_PROF(HYDRA_PROF_LOGPROBS,
+          hydra::launch_token_logprobs_kl(z_act, z_ref, 0, S, L, V, V, ids + c.prompt_len, P,
+                                          lengths, sc, c.beta, logp_actor, logp_ref, reward,
+                                          nullptr, nullptr, err, st));
+  HY_PROF(HYDRA_PROF_GAE, hydra::launch_gae(reward, values, lengths, S, L, c.gamma, c.lam,
+                                            advantages, returns, err, st));
+  if (cudaMemcpyAsync(score, sc, static_cast<size_t>(S) * 4, cudaMemcpyDeviceToDevice, st) !=
+      cudaSuccess)
+    return HYDRA_ERR_CUDA;
+#undef HY_TRY
+#undef HY_PROF
+  return HYDRA_OK;
+}
+
+}  // extern "C"

@@ -44,6 +44,49 @@ _SIGNATURES = {
                                _vp, _vp]),
 }
 
+
+class LlamaConfigC(ctypes.Structure):
+    _fields_ = [("n_layers", _c_i64), ("d_model", _c_i64), ("n_heads", _c_i64),
+                ("head_dim", _c_i64), ("ffn", _c_i64), ("vocab", _c_i64),
+                ("prompt_len", _c_i64), ("response_len", _c_i64), ("lora_rank", _c_i64),
+                ("lora_scale", ctypes.c_float), ("rms_eps", ctypes.c_float),
+                ("rope_theta", ctypes.c_float), ("beta", ctypes.c_float),
+                ("gamma", ctypes.c_float), ("lam", ctypes.c_float)]
+
+
+class LlamaLayerC(ctypes.Structure):
+    _fields_ = [(n, _vp) for n in ("w_qkv", "a_qv", "b_qkv", "w_o", "w_gu", "a_gu", "b_gu",
+                                   "w_down", "a_down", "b_down", "norm_attn", "norm_ffn")]
+
+
+class LlamaWeightsC(ctypes.Structure):
+    _fields_ = [("embed", _vp), ("layers", ctypes.POINTER(LlamaLayerC)), ("final_norm", _vp),
+                ("lm_head", _vp), ("w_rm", _vp)]
+
+
+_SIGNATURES.update({
+    "hydra_embed": (ctypes.c_int, [_vp, _c_i64, _c_i64, _vp, _c_i64, ctypes.c_int, _vp, _vp]),
+    "hydra_rmsnorm": (ctypes.c_int, [_vp, _vp, _c_i64, _c_i64, ctypes.c_float, _c_i64, _c_i64,
+                                     _c_i64, _vp, _vp]),
+    "hydra_rope": (ctypes.c_int, [_vp, _c_i64, _c_i64, _c_i64, _c_i64, _c_i64, ctypes.c_float,
+                                  _vp]),
+    "hydra_causal_attention": (ctypes.c_int, [_vp, _c_i64, _c_i64, _c_i64, _c_i64, _c_i64, _vp,
+                                              _c_i64, _vp]),
+    "hydra_swiglu": (ctypes.c_int, [_vp, _c_i64, _c_i64, _vp, _vp]),
+    "hydra_residual_add": (ctypes.c_int, [_vp, _vp, _c_i64, _vp]),
+    "hydra_head_dot": (ctypes.c_int, [_vp, _c_i64, _vp, _c_i64, _c_i64, _c_i64, _c_i64, _vp,
+                                      _vp]),
+    "hydra_profile_enable": (ctypes.c_int, [ctypes.c_int]),
+    "hydra_profile_collect": (ctypes.c_int, [ctypes.POINTER(ctypes.c_float),
+                                             ctypes.POINTER(ctypes.c_int64), ctypes.c_int]),
+    "hydra_score_llama_workspace_size": (ctypes.c_size_t, [ctypes.POINTER(LlamaConfigC),
+                                                           _c_i64]),
+    "hydra_score_llama": (ctypes.c_int, [ctypes.POINTER(LlamaConfigC),
+                                         ctypes.POINTER(LlamaWeightsC), _vp, _vp, _c_i64, _vp,
+                                         ctypes.c_size_t, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                         _vp]),
+})
+
 _lib = None
 
 
@@ -211,3 +254,124 @@ def ppo_gae(rewards, values, lengths, gamma, lam, advantages, returns, stream=No
     S, L = rewards.shape
     _check("ppo_gae", load().ppo_gae(_p(rewards), _p(values), _p(lengths), S, L, float(gamma),
                                      float(lam), _p(advantages), _p(returns), _stream(stream)))
+
+
+# ----------------------------------------------------------------------------- Llama pieces
+
+
+def hydra_embed(table, ids, copies, h, stream=None):
+    _req(table, torch.bfloat16, "table")
+    _req(ids, torch.int32, "ids")
+    _req(h, torch.float32, "h")
+    V, d = table.shape
+    _check("hydra_embed", load().hydra_embed(_p(table), V, d, _p(ids), ids.numel(), int(copies),
+                                             _p(h), _stream(stream)))
+
+
+def hydra_rmsnorm(x, w, eps, y, rows=None, g_out=None, g_in=None, off=0, stream=None):
+    """y[i] = bf16(RMSNorm(x[j]) * w), j = (i // g_out) * g_in + off + i % g_out."""
+    _req(x, torch.float32, "x")
+    _req(w, torch.bfloat16, "w")
+    _req(y, torch.bfloat16, "y")
+    d = x.shape[-1]
+    rows = y.shape[0] if rows is None else rows
+    g_out = rows if g_out is None else g_out
+    g_in = g_out if g_in is None else g_in
+    _check("hydra_rmsnorm", load().hydra_rmsnorm(_p(x), _p(w), rows, d, float(eps), g_out, g_in,
+                                                 off, _p(y), _stream(stream)))
+
+
+def hydra_rope(qkv, d, head_dim, P, theta, stream=None):
+    _req(qkv, torch.bfloat16, "qkv")
+    R, ld = qkv.shape
+    _check("hydra_rope", load().hydra_rope(_p(qkv), R, ld, d, head_dim, P, float(theta),
+                                           _stream(stream)))
+
+
+def hydra_causal_attention(qkv, nseq, P, n_heads, head_dim, out, stream=None):
+    _req(qkv, torch.bfloat16, "qkv")
+    _req(out, torch.bfloat16, "out")
+    _check("hydra_causal_attention", load().hydra_causal_attention(
+        _p(qkv), nseq, P, qkv.shape[1], n_heads, head_dim, _p(out), out.shape[1],
+        _stream(stream)))
+
+
+def hydra_swiglu(gu, m, stream=None):
+    _req(gu, torch.bfloat16, "gu")
+    _req(m, torch.bfloat16, "m")
+    _check("hydra_swiglu", load().hydra_swiglu(_p(gu), gu.shape[0], m.shape[1], _p(m),
+                                               _stream(stream)))
+
+
+def hydra_residual_add(h, y, stream=None):
+    _req(h, torch.float32, "h")
+    _req(y, torch.bfloat16, "y")
+    _check("hydra_residual_add", load().hydra_residual_add(_p(h), _p(y), h.numel(),
+                                                           _stream(stream)))
+
+
+def hydra_head_dot(x, w, out, g_out=None, g_in=None, off=0, stream=None):
+    _req(x, torch.bfloat16, "x")
+    _req(w, torch.bfloat16, "w")
+    _req(out, torch.float32, "out")
+    n = out.numel()
+    g_out = n if g_out is None else g_out
+    g_in = g_out if g_in is None else g_in
+    _check("hydra_head_dot", load().hydra_head_dot(_p(x), x.shape[-1], _p(w), n, g_out, g_in, off,
+                                                   _p(out), _stream(stream)))
+
+
+def llama_config_c(cfg):
+    """hydra_llama_config from a dict with the keys of LlamaConfigC."""
+    return LlamaConfigC(**{k: cfg[k] for k, _ in LlamaConfigC._fields_})
+
+
+def score_llama_workspace_size(cfg, S):
+    c = llama_config_c(cfg)
+    return int(load().hydra_score_llama_workspace_size(ctypes.byref(c), S))
+
+
+def hydra_score_llama(cfg, weights, ids, lengths, workspace, outputs, stream=None):
+    """Full J-Hydra scoring pass. cfg: dict (LlamaConfigC keys); weights: dict of device
+    tensors in the fused layouts (see include/hydra.h: embed, final_norm, lm_head, w_rm and
+    per-layer lists w_qkv, a_qv, b_qkv, w_o, w_gu, a_gu, b_gu, w_down, a_down, b_down,
+    norm_attn, norm_ffn); ids int32 [S, P0 + L]; lengths int32 [S] or None; outputs: dict
+    with fp32 logp_actor, logp_ref, reward, values, advantages, returns [S, L], score [S]."""
+    c = llama_config_c(cfg)
+    n = cfg["n_layers"]
+    layers = (LlamaLayerC * n)()
+    for l in range(n):
+        for name, _ in LlamaLayerC._fields_:
+            t = weights[name][l]
+            _req(t, torch.bfloat16, name)
+            setattr(layers[l], name, t.data_ptr())
+    for name in ("embed", "final_norm", "lm_head", "w_rm"):
+        _req(weights[name], torch.bfloat16, name)
+    w = LlamaWeightsC(weights["embed"].data_ptr(), layers, weights["final_norm"].data_ptr(),
+                      weights["lm_head"].data_ptr(), weights["w_rm"].data_ptr())
+    _req(ids, torch.int32, "ids")
+    _req(lengths, torch.int32, "lengths")
+    names = ("logp_actor", "logp_ref", "reward", "values", "advantages", "returns", "score")
+    for k in names:
+        _req(outputs[k], torch.float32, k)
+    S = ids.shape[0]
+    ws_bytes = workspace.numel() * workspace.element_size()
+    _check("hydra_score_llama", load().hydra_score_llama(
+        ctypes.byref(c), ctypes.byref(w), _p(ids), _p(lengths), S, _p(workspace), ws_bytes,
+        *[_p(outputs[k]) for k in names], _stream(stream)))
+
+
+PROF_CLASSES = ("gemm", "lora_down", "attention", "elementwise", "logprobs", "gae", "heads")
+
+
+def profile_enable(on=True):
+    _check("hydra_profile_enable", load().hydra_profile_enable(int(bool(on))))
+
+
+def profile_collect(reset=True):
+    """{class: (ms, launches)} summed since the last reset."""
+    n = len(PROF_CLASSES)
+    ms = (ctypes.c_float * n)()
+    cnt = (ctypes.c_int64 * n)()
+    _check("hydra_profile_collect", load().hydra_profile_collect(ms, cnt, int(reset)))
+    return {k: (float(ms[i]), int(cnt[i])) for i, k in enumerate(PROF_CLASSES)}

@@ -7,8 +7,9 @@ their inputs from it without sharing any of the computation under test.
 Generator: SplitMix64 (Steele, Lea and Flood, "Fast splittable pseudorandom number
 generators", OOPSLA 2014) in counter form, i.e. draw i of stream `seed` is
 mix(seed_state + (i + 1) * 0x9E3779B97F4A7C15). Uniforms take the top 53 bits.
-Normals use the Box-Muller transform on two independent uniform streams. bf16 values
-are produced by rounding the fp32 value to nearest-even on the upper 16 bits.
+Normals use the Box-Muller transform in float32: each 64-bit draw gives two 32-bit
+uniforms (u1, u2) and two normals, r cos(2 pi u2) and r sin(2 pi u2), r = sqrt(-2 ln u1).
+bf16 values are produced by rounding the fp32 value to nearest-even on the upper 16 bits.
 
 Everything returned is numpy: bf16 tensors as uint16 bit patterns, fp32 as float32,
 integer ids/lengths as int32.
@@ -27,11 +28,14 @@ def _splitmix64(seed: int, start: int, n: int) -> np.ndarray:
     """Counter-based SplitMix64 outputs for indices start .. start+n-1 of stream `seed`."""
     with np.errstate(over="ignore"):
         base = np.uint64(seed & 0xFFFFFFFFFFFFFFFF) * _GOLDEN
-        idx = np.arange(start + 1, start + n + 1, dtype=np.uint64)
-        z = base + idx * _GOLDEN
-        z = (z ^ (z >> np.uint64(30))) * _M1
-        z = (z ^ (z >> np.uint64(27))) * _M2
-        z = z ^ (z >> np.uint64(31))
+        z = np.arange(start + 1, start + n + 1, dtype=np.uint64)
+        z *= _GOLDEN
+        z += base
+        z ^= z >> np.uint64(30)
+        z *= _M1
+        z ^= z >> np.uint64(27)
+        z *= _M2
+        z ^= z >> np.uint64(31)
     return z
 
 
@@ -46,10 +50,23 @@ def uniform(seed: int, n: int) -> np.ndarray:
 
 
 def normal(seed: int, n: int, std: float = 1.0) -> np.ndarray:
-    """n fp64 draws from N(0, std^2) by Box-Muller on two uniform streams."""
-    u1 = uniform(seed * 2 + 1, n)
-    u2 = uniform(seed * 2 + 2, n)
-    return std * np.sqrt(-2.0 * np.log(u1)) * np.cos(2.0 * np.pi * u2)
+    """n float32 draws from N(0, std^2) (Box-Muller, two normals per 64-bit draw)."""
+    out = np.empty(2 * ((n + 1) // 2), dtype=np.float32)
+    half = out.size // 2
+    scale = np.float32(1.0 / 4294967296.0)
+    for s in range(0, half, _CHUNK):
+        m = min(_CHUNK, half - s)
+        z = _splitmix64(seed, s, m)
+        u1 = ((z >> np.uint64(32)).astype(np.float32) + np.float32(0.5)) * scale
+        u2 = ((z & np.uint64(0xFFFFFFFF)).astype(np.float32) + np.float32(0.5)) * scale
+        np.log(u1, out=u1)
+        u1 *= np.float32(-2.0)
+        np.sqrt(u1, out=u1)
+        u1 *= np.float32(std)
+        u2 *= np.float32(2.0 * np.pi)
+        out[2 * s:2 * (s + m):2] = u1 * np.cos(u2)
+        out[2 * s + 1:2 * (s + m):2] = u1 * np.sin(u2)
+    return out[:n]
 
 
 def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:

@@ -1,0 +1,336 @@
+"""GPU parity of the Llama decoder pieces and of the full J-Hydra scoring pass
+(hydra_score_llama) against the fp64 oracle, through the C-ABI."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2309_00754_gb300 import build as Bld
+from paper_2309_00754_gb300 import hydra as H
+from paper_2309_00754_gb300 import llama, synth
+from tests.helpers import (TOL_GAE, TOL_LINEAR, TOL_LOGP, assert_abs, assert_rel, dev_bf16,
+                           dev_f32, dev_i32, f64, host_f64, max_abs_err)
+
+pytestmark = pytest.mark.gpu
+ONE_BF16 = np.uint16(0x3F80)
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    Bld.build()
+    H.load()
+    H.device_error(clear=True)
+    yield
+    assert H.device_error(clear=True) == 0
+
+
+# ------------------------------------------------------------------ pieces
+
+
+def test_embed_two_copies_exact():
+    V, d, T = 300, 256, 77
+    table = synth.normal_bf16(501, (V, d), 0.02)
+    ids = synth.randint(502, (T,), 0, V)
+    h = torch.full((2 * T, d), float("nan"), device="cuda")
+    H.hydra_embed(dev_bf16(table), dev_i32(ids), 2, h)
+    ref = f64(table)[ids]
+    got = host_f64(h)
+    assert np.array_equal(got[:T], ref) and np.array_equal(got[T:], ref)
+
+
+def test_rmsnorm_with_row_gather():
+    d, S, P, L, p0 = 512, 3, 40, 25, 9
+    x = synth.normal_f32(511, (2 * S * P, d), 1.5)
+    w = synth.normal_bf16(512, (d,), 1.0)
+    y = torch.empty(2 * S * L, d, dtype=torch.bfloat16, device="cuda")
+    H.hydra_rmsnorm(dev_f32(x), dev_bf16(w), 1e-6, y, g_out=L, g_in=P, off=p0 - 1)
+    rows = np.array([(i // L) * P + p0 - 1 + i % L for i in range(2 * S * L)])
+    ref = O.round_bf16(O.rmsnorm(x[rows].astype(np.float64), f64(w), 1e-6))
+    assert_rel(host_f64(y), ref, TOL_LINEAR, "rmsnorm")
+
+
+def test_rope_q_k_rotated_v_untouched():
+    H_, Dh, S, P = 3, 128, 2, 70
+    d = H_ * Dh
+    qkv_bits = synth.normal_bf16(521, (S * P, 3 * d), 1.0)
+    qkv = dev_bf16(qkv_bits)
+    H.hydra_rope(qkv, d, Dh, P, 10000.0)
+    got = host_f64(qkv)
+    x = f64(qkv_bits)
+    pos = np.arange(S * P) % P
+    for blk in range(2):
+        ref = O.round_bf16(O.rope(x[:, blk * d:(blk + 1) * d].reshape(-1, H_, Dh), pos, 10000.0))
+        assert_rel(got[:, blk * d:(blk + 1) * d], ref.reshape(-1, d), TOL_LINEAR, f"rope block {blk}")
+    assert np.array_equal(got[:, 2 * d:], x[:, 2 * d:])
+
+
+@pytest.mark.parametrize("nseq,P,H_", [(3, 100, 2), (1, 768, 1), (2, 64, 1), (1, 1, 2)])
+def test_causal_attention(nseq, P, H_):
+    Dh = 128
+    d = H_ * Dh
+    qkv_bits = synth.normal_bf16(531 + P, (nseq * P, 3 * d), 1.0)
+    out = torch.full((nseq * P, d), float("nan"), dtype=torch.bfloat16, device="cuda")
+    H.hydra_causal_attention(dev_bf16(qkv_bits), nseq, P, H_, Dh, out)
+    x = f64(qkv_bits)
+    got = host_f64(out)
+    for s in range(nseq):
+        blk = x[s * P:(s + 1) * P]
+        q = blk[:, :d].reshape(P, H_, Dh)
+        k = blk[:, d:2 * d].reshape(P, H_, Dh)
+        v = blk[:, 2 * d:].reshape(P, H_, Dh)
+        ref = O.causal_attention(q, k, v).reshape(P, d)
+        assert_rel(got[s * P:(s + 1) * P], ref, TOL_LINEAR, f"attention seq {s}")
+
+
+def test_swiglu_residual_head_dot():
+    R, F, d = 70, 520, 256
+    gu = synth.normal_bf16(541, (R, 2 * F), 2.0)
+    m = torch.empty(R, F, dtype=torch.bfloat16, device="cuda")
+    H.hydra_swiglu(dev_bf16(gu), m)
+    g = f64(gu)
+    assert_rel(host_f64(m), O.round_bf16(O.swiglu(g[:, :F], g[:, F:])), TOL_LINEAR, "swiglu")
+
+    h0 = synth.normal_f32(542, (R, d))
+    y = synth.normal_bf16(543, (R, d))
+    h = dev_f32(h0)
+    H.hydra_residual_add(h, dev_bf16(y))
+    assert_rel(host_f64(h), h0.astype(np.float64) + f64(y), 1e-6, "residual")
+
+    x = synth.normal_bf16(544, (R, d))
+    w = synth.normal_bf16(545, (d,), 0.02)
+    out = torch.empty(R, device="cuda")
+    H.hydra_head_dot(dev_bf16(x), dev_bf16(w), out)
+    assert_rel(host_f64(out), f64(x) @ f64(w), 1e-5, "head dot")
+
+
+# ------------------------------------------------------------------ the full pass
+
+
+def make_model(cfg, seed, zero_B=False, lora_std=0.02, emb_std=1.0):
+    nl, d, F, V, r = cfg["n_layers"], cfg["d_model"], cfg["ffn"], cfg["vocab"], cfg["lora_rank"]
+    g = lambda i: synth.tensor_seed(seed, i)  # noqa: E731
+    sep = {
+        "wq": synth.normal_bf16(g(1), (nl, d, d), 0.02),
+        "wk": synth.normal_bf16(g(2), (nl, d, d), 0.02),
+        "wv": synth.normal_bf16(g(3), (nl, d, d), 0.02),
+        "wo": synth.normal_bf16(g(4), (nl, d, d), 0.02),
+        "wg": synth.normal_bf16(g(5), (nl, F, d), 0.02),
+        "wu": synth.normal_bf16(g(6), (nl, F, d), 0.02),
+        "wd": synth.normal_bf16(g(7), (nl, d, F), 0.02),
+        "norm1": np.full((nl, d), ONE_BF16, dtype=np.uint16),
+        "norm2": np.full((nl, d), ONE_BF16, dtype=np.uint16),
+        "embed": synth.normal_bf16(g(8), (V, d), emb_std),
+        "final_norm": np.full((d,), ONE_BF16, dtype=np.uint16),
+        "lm_head": synth.normal_bf16(g(9), (V, d), 0.02),
+        "w_rm": synth.normal_bf16(g(10), (d,), 0.02),
+        "lora": {},
+    }
+    dims = {"wq": (d, d), "wv": (d, d), "wg": (F, d), "wu": (F, d), "wd": (d, F)}
+    for i, (name, (n_out, n_in)) in enumerate(dims.items()):
+        A = synth.normal_bf16(g(20 + i), (nl, r, n_in), lora_std)
+        Bm = (np.zeros((nl, n_out, r), dtype=np.uint16) if zero_B
+              else synth.normal_bf16(g(30 + i), (nl, n_out, r), lora_std))
+        sep["lora"][name] = (A, Bm)
+    w64 = {k: f64(v) for k, v in sep.items() if k != "lora"}
+    w64["lora"] = {k: (f64(a), f64(b)) for k, (a, b) in sep["lora"].items()}
+    return sep, w64
+
+
+def oracle_cfg(cfg):
+    return {"d": cfg["d_model"], "n_heads": cfg["n_heads"], "eps": cfg["rms_eps"],
+            "lora_scale": cfg["lora_scale"], "rope_theta": cfg["rope_theta"],
+            "n_layers": cfg["n_layers"]}
+
+
+def run_pass(cfg, sep, ids, lengths):
+    S = ids.shape[0]
+    w = llama.to_device(llama.fuse_separate(sep), "cuda")
+    ws = torch.empty(H.score_llama_workspace_size(cfg, S), dtype=torch.uint8, device="cuda")
+    out = llama.alloc_outputs(S, cfg["response_len"], "cuda")
+    H.hydra_score_llama(cfg, w, dev_i32(ids), None if lengths is None else dev_i32(lengths), ws, out)
+    torch.cuda.synchronize()
+    return {k: host_f64(v) for k, v in out.items()}
+
+
+# Relative size of the fp32-accumulation difference that a kernel's stored values carry
+# (measured: 0.23 % of the bf16 outputs of a K = 4096 tensor-core product differ by one ulp
+# from the exactly rounded fp64 result, i.e. about 1e-5 relative before rounding).
+DITHER_EPS = 1e-5
+
+
+def chain_spread(w64, ids_s, P0, cfg, n):
+    """How far two equally valid roundings of the bf16 chain drift apart: the oracle against
+    itself with every stored value perturbed by DITHER_EPS relative before rounding."""
+    kw = dict(seq_lengths=n, beta=cfg["beta"], gamma=cfg["gamma"], lam=cfg["lam"])
+    O.set_storage_dither(DITHER_EPS, seed=17)
+    try:
+        alt = O.llama_score(w64, ids_s, P0, oracle_cfg(cfg), **kw)
+    finally:
+        O.set_storage_dither(0.0)
+    return alt
+
+
+def check_pass(cfg, got, w64, ids, lengths, derive_tol=False):
+    """Compare a pass with the oracle. With derive_tol, each end-to-end tolerance is the
+    larger of the stated one and 3x the chain's own spread under DITHER_EPS (a wide, deep
+    bf16 chain amplifies one-ulp flips, so the stated per-kernel tolerances bound each
+    kernel, not a composition of many)."""
+    P0, L = cfg["prompt_len"], cfg["response_len"]
+    g_, lam, beta = cfg["gamma"], cfg["lam"], cfg["beta"]
+    S = ids.shape[0]
+    e_r = e_v = 0.0
+    for s in range(S):
+        n = L if lengths is None else int(lengths[s])
+        ref = O.llama_score(w64, ids[s], P0, oracle_cfg(cfg), seq_lengths=n, beta=beta,
+                            gamma=g_, lam=lam)
+        tol_lp, tol_lin = TOL_LOGP, TOL_LINEAR
+        if derive_tol:
+            alt = chain_spread(w64, ids[s], P0, cfg, n)
+            spread_lp = max(max_abs_err(alt["logp_actor"], ref["logp_actor"]),
+                            max_abs_err(alt["logp_ref"], ref["logp_ref"]))
+            spread_lin = max(max_abs_err(alt["values"], ref["values"]),
+                             abs(alt["score"] - ref["score"]))
+            tol_lp = max(TOL_LOGP, 3 * spread_lp)
+            tol_lin = max(TOL_LINEAR, 3 * spread_lin)
+            print(f"seq {s}: chain spread logp {spread_lp:.2e}, head {spread_lin:.2e} "
+                  f"-> tolerances {tol_lp:.2e}, {tol_lin:.2e}")
+        assert_abs(got["logp_actor"][s], ref["logp_actor"], tol_lp, f"logp_actor seq {s}")
+        assert_abs(got["logp_ref"][s], ref["logp_ref"], tol_lp, f"logp_ref seq {s}")
+        assert_rel(got["score"][s:s + 1], [ref["score"]], tol_lin, f"score seq {s}")
+        assert_rel(got["values"][s], ref["values"], tol_lin, f"values seq {s}")
+        # the KL part of the reward; the score enters at t = len - 1 on each side
+        kl_got = got["reward"][s].copy()
+        kl_ref = ref["reward"].copy()
+        if n > 0:
+            kl_got[n - 1] -= got["score"][s]
+            kl_ref[n - 1] -= ref["score"]
+        assert_abs(kl_got, kl_ref, tol_lp, f"KL reward seq {s}")
+        e_r = max(e_r, max_abs_err(got["reward"][s], ref["reward"]))
+        e_v = max(e_v, max_abs_err(got["values"][s], ref["values"]))
+        # GAE on the GPU's own rewards and values: the scan's tolerance
+        a1, r1 = O.gae(got["reward"][s:s + 1], got["values"][s:s + 1], [n], g_, lam)
+        assert_rel(got["advantages"][s:s + 1], a1, TOL_GAE, f"advantages seq {s}")
+        assert_rel(got["returns"][s:s + 1], r1, TOL_GAE, f"returns seq {s}")
+        # end to end: reward and value errors pass through sum_k (gamma lambda)^k
+        bound = (e_r + (1 + g_) * e_v) / (1 - g_ * lam) + TOL_GAE
+        assert_abs(got["advantages"][s], ref["advantages"], bound, f"advantages e2e seq {s}")
+
+
+SMALL = dict(n_layers=2, d_model=256, n_heads=2, head_dim=128, ffn=512, vocab=512,
+             prompt_len=16, response_len=40, lora_rank=8, lora_scale=2.0, rms_eps=1e-6,
+             rope_theta=10000.0, beta=0.1, gamma=1.0, lam=0.95)
+
+
+def test_score_llama_small_ragged():
+    cfg = dict(SMALL)
+    sep, w64 = make_model(cfg, 61)
+    S, P = 3, cfg["prompt_len"] + cfg["response_len"]
+    ids = synth.randint(611, (S, P), 0, cfg["vocab"])
+    lengths = np.array([40, 17, 1], dtype=np.int32)
+    got = run_pass(cfg, sep, ids, lengths)
+    check_pass(cfg, got, w64, ids, lengths)
+
+
+def test_score_llama_several_key_blocks_rank16():
+    cfg = dict(SMALL, n_layers=1, prompt_len=100, response_len=60, lora_rank=16, vocab=1024)
+    sep, w64 = make_model(cfg, 62)
+    ids = synth.randint(621, (2, 160), 0, cfg["vocab"])
+    got = run_pass(cfg, sep, ids, None)
+    check_pass(cfg, got, w64, ids, None)
+
+
+def test_score_llama_lora_off_streams_agree_bitwise():
+    # §3 Dynamic LoRA: with every B = 0 the LoRA-on stream is the LoRA-off stream, so the
+    # actor and reference log-probabilities agree exactly and the reward is the score alone
+    cfg = dict(SMALL)
+    sep, _ = make_model(cfg, 63, zero_B=True)
+    S, P = 2, cfg["prompt_len"] + cfg["response_len"]
+    ids = synth.randint(631, (S, P), 0, cfg["vocab"])
+    lengths = np.array([40, 33], dtype=np.int32)
+    got = run_pass(cfg, sep, ids, lengths)
+    assert np.array_equal(got["logp_actor"], got["logp_ref"])
+    expect = np.zeros_like(got["reward"])
+    for s in range(S):
+        expect[s, lengths[s] - 1] = got["score"][s]
+    assert np.array_equal(got["reward"], expect)
+
+
+def test_score_llama_full_width_one_layer():
+    """Llama-7B widths (d 4096, 32 heads, FFN 11008, vocab 32000, LoRA r 16) at the
+    benchmark's sequence shape (256 prompt + 512 response tokens), one decoder layer, one
+    sequence, compared in full with the oracle."""
+    cfg = dict(llama.LLAMA7B, n_layers=1)
+    sep, w64 = make_model(cfg, 64)
+    ids = synth.randint(641, (1, 768), 0, cfg["vocab"])
+    lengths = np.array([512], dtype=np.int32)
+    got = run_pass(cfg, sep, ids, lengths)
+    check_pass(cfg, got, w64, ids, lengths, derive_tol=True)
+
+
+# ------------------------------------------------------------------ full size, properties
+
+
+@pytest.fixture(scope="module")
+def llama7b():
+    """The benchmark's model and batch: random-init Llama-7B (32 layers), 4 x (256 + 512)."""
+    cfg = dict(llama.LLAMA7B)
+    w = llama.random_device_weights(cfg, 4, "cuda")
+    S, P = 4, cfg["prompt_len"] + cfg["response_len"]
+    ids = torch.from_numpy(synth.randint(4001, (S, P), 0, cfg["vocab"])).cuda()
+    ws = torch.empty(H.score_llama_workspace_size(cfg, S), dtype=torch.uint8, device="cuda")
+    yield cfg, w, ids, ws
+    del w, ws
+    torch.cuda.empty_cache()
+
+
+def _score(cfg, w, ids, lengths, ws):
+    out = llama.alloc_outputs(ids.shape[0], cfg["response_len"], "cuda")
+    H.hydra_score_llama(cfg, w, ids, lengths, ws, out)
+    torch.cuda.synchronize()
+    return {k: v.clone() for k, v in out.items()}
+
+
+def test_llama7b_deterministic_batch_permutation_and_causal(llama7b):
+    cfg, w, ids, ws = llama7b
+    L = cfg["response_len"]
+    lengths = torch.tensor([512, 300, 64, 1], dtype=torch.int32, device="cuda")
+    a = _score(cfg, w, ids, lengths, ws)
+    b = _score(cfg, w, ids, lengths, ws)
+    for k in a:
+        assert torch.equal(a[k], b[k]), f"{k} not deterministic"
+    for k in ("logp_actor", "logp_ref", "reward", "values", "advantages"):
+        assert torch.isfinite(a[k]).all()
+    # sequences are independent: a permuted batch gives the permuted outputs, bit for bit
+    perm = torch.tensor([2, 0, 3, 1], device="cuda")
+    c = _score(cfg, w, ids[perm].contiguous(), lengths[perm].contiguous(), ws)
+    for k in a:
+        assert torch.equal(c[k], a[k][perm]), f"{k} changes with the batch order"
+    # causal: changing sequence 0's last token moves nothing before it
+    ids2 = ids.clone()
+    ids2[0, -1] = (ids2[0, -1] + 1) % cfg["vocab"]
+    d = _score(cfg, w, ids2, lengths, ws)
+    for k in ("logp_actor", "logp_ref", "values"):
+        assert torch.equal(d[k][0, :L - 1], a[k][0, :L - 1])
+        assert torch.equal(d[k][1:], a[k][1:])
+    assert not torch.equal(d["logp_actor"][0, L - 1], a["logp_actor"][0, L - 1])
+    # GAE of the pass's own rewards and values (the scan's tolerance)
+    rw, vv = host_f64(a["reward"]), host_f64(a["values"])
+    adv, ret = O.gae(rw, vv, lengths.cpu().numpy(), cfg["gamma"], cfg["lam"])
+    assert_rel(host_f64(a["advantages"]), adv, TOL_GAE, "advantages")
+    assert_rel(host_f64(a["returns"]), ret, TOL_GAE, "returns")
+
+
+def test_llama7b_lora_off_streams_agree_bitwise(llama7b):
+    # §3 Dynamic LoRA at full size: zero every LoRA B and the two streams coincide
+    cfg, w, ids, ws = llama7b
+    wz = dict(w)
+    for k in ("b_qkv", "b_gu", "b_down"):
+        wz[k] = [torch.zeros_like(t) for t in w[k]]
+    lengths = torch.tensor([512, 512, 200, 7], dtype=torch.int32, device="cuda")
+    a = _score(cfg, wz, ids, lengths, ws)
+    assert torch.equal(a["logp_actor"], a["logp_ref"])
+    expect = torch.zeros_like(a["reward"])
+    for s in range(4):
+        expect[s, lengths[s] - 1] = a["score"][s]
+    assert torch.equal(a["reward"], expect)

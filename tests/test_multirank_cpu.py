@@ -1,0 +1,54 @@
+"""The benchmark's multi-rank host logic on CPU with the gloo backend (world size 2): the
+max-over-ranks timing reduction, the barrier and the weak-scaling aggregate. No GPU and no
+data-path collective are involved: ranks score independent batches."""
+import os
+import socket
+
+import pytest
+import torch
+import torch.distributed as dist
+import torch.multiprocessing as mp
+
+
+def _free_port():
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    port = s.getsockname()[1]
+    s.close()
+    return port
+
+
+def _worker(rank, world, port, q):
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    import bench
+    ms = [120.0, 150.0][rank]  # rank 1 is the slower one
+    bench.barrier(world)
+    ms_max = bench.max_over_ranks(ms, world)
+    value = bench.aggregate(2048, 10, world, ms_max)
+    q.put((rank, ms_max, value))
+    bench.barrier(world)
+    dist.destroy_process_group()
+
+
+def test_max_over_ranks_and_weak_scaling_aggregate():
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_worker, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    res = sorted(q.get(timeout=120) for _ in range(2))
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    for rank, ms_max, value in res:
+        assert ms_max == 150.0
+        assert value == pytest.approx(2048 * 10 * 2 / 0.150)
+
+
+def test_single_rank_is_identity():
+    import bench
+    assert bench.max_over_ranks(3.5, 1) == 3.5
+    assert bench.aggregate(100, 4, 1, 200.0) == pytest.approx(2000.0)

@@ -374,3 +374,17 @@ def test_llama_score_causal_and_lora_changes_actor_only():
     # turning LoRA on changes the actor stream but never the reference stream
     np.testing.assert_allclose(out["logp_ref"], ref0["logp_ref"], atol=0)
     assert np.max(np.abs(out["logp_actor"] - ref0["logp_actor"])) > 1e-6
+
+
+def test_storage_dither_is_off_by_default_and_bounded():
+    x = np.array([1.0, 1.0 + 2 ** -9 + 2 ** -20, 3.0, -0.3])
+    base = O.round_bf16(x)
+    O.set_storage_dither(1e-5, seed=1)
+    try:
+        d = O.round_bf16(x)
+        # a dither far below half an ulp moves a value only when it sits next to a tie
+        assert np.array_equal(d[[0, 2]], base[[0, 2]])
+        assert np.all(np.abs(d - base) <= 2 ** -7 * np.abs(base))
+    finally:
+        O.set_storage_dither(0.0)
+    assert np.array_equal(O.round_bf16(x), base)
