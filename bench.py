@@ -281,11 +281,17 @@ class HydraScoringLlama7B:
         self.units = int(self.S * self.L)
         T, SL = self.S * P, self.S * self.L
         d, F, V, r = c["d_model"], c["ffn"], c["vocab"], c["lora_rank"]
-        per_layer = (2 * (2 * T * d * 3 * d) + 2 * T * 2 * r * 3 * d      # qkv (+ LoRA-up)
-                     + 2 * (2 * T * d * d)                                 # o
-                     + 2 * (2 * T * d * 2 * F) + 2 * T * 2 * r * 2 * F     # gate/up
-                     + 2 * (2 * T * F * d) + 2 * T * r * d)                # down
-        self.gemm_flops = c["n_layers"] * per_layer + 2 * (2 * SL * d * V)
+        nl = c["n_layers"]
+        # algorithmic flops per pass of each projection class (both streams; LoRA-up on the
+        # on stream only)
+        self.class_flops = {
+            "gemm_qkv": nl * (2 * (2 * T * d * 3 * d) + 2 * T * 2 * r * 3 * d),
+            "gemm_o": nl * 2 * (2 * T * d * d),
+            "gemm_gu": nl * (2 * (2 * T * d * 2 * F) + 2 * T * 2 * r * 2 * F),
+            "gemm_down": nl * (2 * (2 * T * F * d) + 2 * T * r * d),
+            "gemm_lmhead": 2 * (2 * SL * d * V),
+        }
+        self.gemm_flops = sum(self.class_flops.values())
         self.attn_flops = c["n_layers"] * 2 * self.S * c["n_heads"] * 2 * P * P * 128  # causal half
         self.logp_bytes = SL * V * 4 * 2 + SL * 16
         self.launches_per_step = None
@@ -313,8 +319,9 @@ class HydraScoringLlama7B:
         for k, (ms, n) in prof.items():
             if n:
                 out[k] = {"ms_total": ms, "launches": n, "ms_per_launch": ms / n}
-        g = prof["gemm"]
-        out["gemm"]["TFLOP/s"] = self.gemm_flops * (g[1] / self.launch_counts["gemm"]) / g[0] / 1e9
+        for k, fl in self.class_flops.items():
+            ms, n = prof[k]
+            out[k]["TFLOP/s"] = fl * (n / self.launch_counts[k]) / ms / 1e9
         a = prof["attention"]
         out["attention"]["TFLOP/s"] = self.attn_flops * (a[1] / self.launch_counts["attention"]) / a[0] / 1e9
         lp = prof["logprobs"]
@@ -322,15 +329,16 @@ class HydraScoringLlama7B:
         return out
 
     def roofline(self, peaks, prof):
-        ms, n = prof["gemm"]
-        steps = n / self.launch_counts["gemm"]
+        ms = sum(prof[k][0] for k in self.class_flops)
+        n = sum(prof[k][1] for k in self.class_flops)
+        steps = n / sum(self.launch_counts[k] for k in self.class_flops)
         achieved = self.gemm_flops * steps / ms / 1e9
         peak = peaks["bf16_tflops_sustained"]
         return {"kernel": "dual_lora_gemm_tcgen05 (all projections + LM head of the pass)",
                 "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": achieved / peak, "traffic": None,
                 "peak_kind": f"bf16 dense, {peaks['source']} sustained",
-                "per_launch_flop": self.gemm_flops / self.launch_counts["gemm"],
+                "per_launch_flop": self.gemm_flops / sum(self.launch_counts[k] for k in self.class_flops),
                 "per_launch_ms": ms / n}
 
     def config(self):
@@ -360,16 +368,17 @@ class HydraScoringLlama7B:
             qkv = f64(W["w_qkv"][l])
             w["wq"].append(qkv[:d]); w["wk"].append(qkv[d:2 * d]); w["wv"].append(qkv[2 * d:])
             w["wo"].append(f64(W["w_o"][l]))
-            gu = f64(W["w_gu"][l])
-            w["wg"].append(gu[:F]); w["wu"].append(gu[F:])
+            g_, u_ = self.llama.deinterleave_gate_up(f64(W["w_gu"][l]))
+            w["wg"].append(g_); w["wu"].append(u_)
             w["wd"].append(f64(W["w_down"][l]))
             w["norm1"].append(f64(W["norm_attn"][l])); w["norm2"].append(f64(W["norm_ffn"][l]))
             a, b = f64(W["a_qv"][l]), f64(W["b_qkv"][l])
             lo["wq"][0].append(a[:r]); lo["wq"][1].append(b[:d, :r])
             lo["wv"][0].append(a[r:]); lo["wv"][1].append(b[2 * d:, r:])
-            a, b = f64(W["a_gu"][l]), f64(W["b_gu"][l])
-            lo["wg"][0].append(a[:r]); lo["wg"][1].append(b[:F, :r])
-            lo["wu"][0].append(a[r:]); lo["wu"][1].append(b[F:, r:])
+            a = f64(W["a_gu"][l])
+            bg, bu = self.llama.deinterleave_gate_up(f64(W["b_gu"][l]))
+            lo["wg"][0].append(a[:r]); lo["wg"][1].append(bg[:, :r])
+            lo["wu"][0].append(a[r:]); lo["wu"][1].append(bu[:, r:])
             lo["wd"][0].append(f64(W["a_down"][l])); lo["wd"][1].append(f64(W["b_down"][l]))
         w = {k: (np.stack(v) if v else np.zeros((0,))) for k, v in w.items() if k != "lora"}
         w["lora"] = {k: (np.stack(a), np.stack(b)) for k, (a, b) in lo.items()}

@@ -120,6 +120,32 @@ hydra_status hydra_dual_linear(const void* x_off, const void* x_on, int64_t M, i
                                int64_t N, const void* W, const void* u, const void* B, int64_t r,
                                void* y_off, void* y_on, int out_dtype, int algo, void* stream);
 
+/* Epilogues of hydra_dual_linear_ex. */
+enum {
+  HYDRA_EPI_STORE = 0,    /* y = result (bf16 or fp32), as hydra_dual_linear */
+  HYDRA_EPI_SWIGLU = 1,   /* gated FFN: see hydra_dual_linear_ex */
+  HYDRA_EPI_RESIDUAL = 2  /* residual stream update: see hydra_dual_linear_ex */
+};
+
+/*
+ * hydra_dual_linear on the tcgen05 kernel with a fused epilogue (Llama decoder blocks of the
+ * scoring pass; §4 uses Llama 7b):
+ *  HYDRA_EPI_STORE    as hydra_dual_linear (algo 1).
+ *  HYDRA_EPI_SWIGLU   W rows come in blocks of 128: block 2j holds gate rows, block 2j + 1 the
+ *                     up rows of the same 128 features (B rows likewise; N % 256 == 0).
+ *                     y_* are bf16 [M, N/2]: y[:, 128 j + i] = bf16(silu(g) * u) with
+ *                     g = bf16(gate row 256 j + i), u = bf16(up row 256 j + 128 + i),
+ *                     silu(g) = g / (1 + exp(-g)) (Shazeer 2020).
+ *  HYDRA_EPI_RESIDUAL y_* are fp32 [M, N] residual streams, updated in place:
+ *                     y += float(bf16(x W^T (+ u B^T))). Outputs of different calls may not
+ *                     overlap in flight; within one call every element is updated once.
+ * out_dtype applies to HYDRA_EPI_STORE only. Other arguments and errors as hydra_dual_linear.
+ */
+hydra_status hydra_dual_linear_ex(const void* x_off, const void* x_on, int64_t M, int64_t K,
+                                  int64_t N, const void* W, const void* u, const void* B,
+                                  int64_t r, void* y_off, void* y_on, int out_dtype, int epilogue,
+                                  void* stream);
+
 /*
  * hydra_lora_linear with the kernel family chosen by the caller:
  *   algo 0 = automatic (as hydra_lora_linear), 1 = tcgen05 tile kernel (any M),
@@ -219,7 +245,7 @@ hydra_status hydra_rmsnorm(const float* x, const void* w, int64_t rows, int64_t 
 
 /* Rotary embedding (Su et al. 2021), rotate-half pairing, in place on the q block
  * (columns [0, d)) and k block ([d, 2d)) of each row of qkv (bf16 [R, ld]): dims (i, i + Dh/2)
- * of every head rotate by pos * theta^(-2i/Dh), pos = row % P. */
+ * of every head rotate by pos * theta^(-2i/Dh), pos = row % P. head_dim % 4 == 0, ld even. */
 hydra_status hydra_rope(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t head_dim, int64_t P,
                         float theta, void* stream);
 
@@ -254,8 +280,11 @@ typedef struct hydra_llama_config {
  *   w_qkv [3d, d] = [Wq; Wk; Wv]        a_qv [2r, d] = [Aq; Av]
  *   b_qkv [3d, 2r] = [[Bq, 0]; [0, 0]; [0, Bv]]   (LoRA on q and v only)
  *   w_o [d, d] (no LoRA)
- *   w_gu [2F, d] = [W_gate; W_up]       a_gu [2r, d] = [A_gate; A_up]
- *   b_gu [2F, 2r] = [[B_gate, 0]; [0, B_up]]
+ *   w_gu [2F, d]: gate and up rows interleaved in blocks of 128 (block 2j = gate rows
+ *        128j..128j+127, block 2j+1 = up rows of the same features); F % 128 == 0
+ *   a_gu [2r, d] = [A_gate; A_up]
+ *   b_gu [2F, 2r]: rows interleaved like w_gu; gate rows [B_gate_row, 0], up rows
+ *        [0, B_up_row]
  *   w_down [d, F], a_down [r, F], b_down [d, r]
  *   norm_attn, norm_ffn [d] */
 typedef struct hydra_llama_layer {
@@ -296,7 +325,7 @@ size_t hydra_score_llama_workspace_size(const hydra_llama_config* cfg, int64_t S
  * ids int32 [S, P0 + L]; lengths int32 [S] valid response tokens (0..L) or NULL (all L).
  * Outputs fp32 [S, L] (0 at t >= len): logp_actor, logp_ref, reward, values, advantages,
  * returns; score fp32 [S]. Requirements: head_dim == 128, d == n_heads * 128,
- * ffn % 8 == 0, vocab % 8 == 0, r % 8 == 0, 8 <= r <= 128, P0 >= 1, L >= 1.
+ * ffn % 128 == 0, vocab % 8 == 0, r % 8 == 0, 8 <= r <= 128, P0 >= 1, L >= 1.
  */
 hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_weights* w,
                                const int32_t* ids, const int32_t* lengths, int64_t S,
@@ -306,14 +335,18 @@ hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_
 
 /* Kernel classes of the optional launch timing of hydra_score_llama. */
 enum {
-  HYDRA_PROF_GEMM = 0,        /* tcgen05 dual-output linear (or the small-M GEMV) */
-  HYDRA_PROF_LORA_DOWN = 1,   /* u = s x A^T */
-  HYDRA_PROF_ATTENTION = 2,   /* causal attention */
-  HYDRA_PROF_ELEMENTWISE = 3, /* embedding, RMSNorm, RoPE, SwiGLU, residual add */
-  HYDRA_PROF_LOGPROBS = 4,    /* log-softmax + gather + KL reward */
-  HYDRA_PROF_GAE = 5,         /* GAE scan */
-  HYDRA_PROF_HEADS = 6,       /* reward-model score and value head */
-  HYDRA_PROF_CLASSES = 7
+  HYDRA_PROF_GEMM_QKV = 0,    /* tcgen05 dual-output linears: fused q/k/v */
+  HYDRA_PROF_GEMM_O = 1,      /* o projection (+ residual add epilogue) */
+  HYDRA_PROF_GEMM_GU = 2,     /* fused gate/up (+ SwiGLU epilogue) */
+  HYDRA_PROF_GEMM_DOWN = 3,   /* down projection (+ residual add epilogue) */
+  HYDRA_PROF_GEMM_LMHEAD = 4, /* LM head, fp32 logits */
+  HYDRA_PROF_LORA_DOWN = 5,   /* u = s x A^T */
+  HYDRA_PROF_ATTENTION = 6,   /* causal attention */
+  HYDRA_PROF_ELEMENTWISE = 7, /* embedding, RMSNorm, RoPE */
+  HYDRA_PROF_LOGPROBS = 8,    /* log-softmax + gather + KL reward */
+  HYDRA_PROF_GAE = 9,         /* GAE scan */
+  HYDRA_PROF_HEADS = 10,      /* reward-model score and value head */
+  HYDRA_PROF_CLASSES = 11
 };
 
 /*

@@ -39,14 +39,18 @@ inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 
 inline size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
 // u_given: `workspace` already holds u = s x_on A^T (hydra_dual_linear); A is unused.
+// epi: tcgen05 epilogue (store / SwiGLU / residual add); non-store epilogues need algo 1.
 hydra_status lora_linear_impl(const void* x_off, const void* x_on, int64_t M, int64_t K,
                               int64_t N, const void* W, const void* A, const void* B, int64_t r,
                               float s, void* y_off, void* y_on, int out_dtype, void* workspace,
                               size_t workspace_bytes, int algo, void* stream,
-                              bool u_given = false) {
+                              bool u_given = false, int epi = HYDRA_EPI_STORE) {
   if (x_off == nullptr || W == nullptr) return HYDRA_ERR_NULL;
   if (y_off == nullptr && y_on == nullptr) return HYDRA_ERR_NULL;
   if (algo < 0 || algo > 2) return HYDRA_ERR_RANGE;
+  if (epi < HYDRA_EPI_STORE || epi > HYDRA_EPI_RESIDUAL) return HYDRA_ERR_RANGE;
+  if (epi != HYDRA_EPI_STORE && algo != 1) return HYDRA_ERR_RANGE;
+  if (epi == HYDRA_EPI_SWIGLU && N % 256 != 0) return HYDRA_ERR_SHAPE;
   if (out_dtype != HYDRA_BF16 && out_dtype != HYDRA_F32) return HYDRA_ERR_RANGE;
   if (M < 0 || K < 8 || N < 8 || M >= (1LL << 31) || K >= (1LL << 31) || N >= (1LL << 31))
     return HYDRA_ERR_SHAPE;
@@ -91,6 +95,7 @@ hydra_status lora_linear_impl(const void* x_off, const void* x_on, int64_t M, in
   g.y_on = y_on;
   g.out_f32 = out_dtype == HYDRA_F32 ? 1 : 0;
   g.err = err;
+  g.epi = epi;
   const bool use_gemv = (algo == 2) || (algo == 0 && rows <= hydra::kGemvMaxRows);
   const int rc = use_gemv ? hydra::launch_dual_lora_gemv(g, st) : hydra::launch_dual_lora_gemm_tc(g, st);
   return rc == 0 ? HYDRA_OK : HYDRA_ERR_CUDA;
@@ -171,6 +176,15 @@ hydra_status hydra_dual_linear(const void* x_off, const void* x_on, int64_t M, i
   return lora_linear_impl(x_off, x_on, M, K, N, W, nullptr, B, r, 1.0f, y_off, y_on, out_dtype,
                           const_cast<void*>(u), hydra_lora_linear_workspace_size(M, r), algo,
                           stream, true);
+}
+
+hydra_status hydra_dual_linear_ex(const void* x_off, const void* x_on, int64_t M, int64_t K,
+                                  int64_t N, const void* W, const void* u, const void* B,
+                                  int64_t r, void* y_off, void* y_on, int out_dtype, int epilogue,
+                                  void* stream) {
+  return lora_linear_impl(x_off, x_on, M, K, N, W, nullptr, B, r, 1.0f, y_off, y_on, out_dtype,
+                          const_cast<void*>(u), hydra_lora_linear_workspace_size(M, r), 1, stream,
+                          true, epilogue);
 }
 
 hydra_status hydra_token_logprobs_kl(const void* logits_actor, const void* logits_ref,

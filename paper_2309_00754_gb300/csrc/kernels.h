@@ -23,6 +23,7 @@ struct GemmArgs {
   void* y_on;         // [M, N] bf16 or fp32, may be NULL
   int out_f32;
   int* err;
+  int epi = 0;        // tcgen05 kernel epilogue: 0 store, 1 SwiGLU, 2 residual add (fp32)
 };
 
 // Device address of the library's error word on the current device (NULL on failure).

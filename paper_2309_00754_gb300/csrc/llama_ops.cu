@@ -87,27 +87,30 @@ __global__ void __launch_bounds__(128)
 
 // In place on the q and k blocks of each row of qkv ([R, ld] bf16; q at column 0, k at
 // column d). Rotate-half pairing: dims (i, i + Dh/2) of each head rotate by
-// pos * theta^(-2i/Dh), pos = row % P (position within its sequence).
-__global__ void rope_kernel(__nv_bfloat16* __restrict__ qkv, long long R, int ld, int d, int Dh,
-                            int P, float log2_theta) {
-  const long long row = blockIdx.x;
+// pos * theta^(-2i/Dh), pos = row % P (position within its sequence). One warp per row;
+// lane l owns the pair indices i = 2l, 2l + 1 (+ 64 l' for Dh > 128), computes their angles
+// once and applies them to every head of q and k with 4-byte (bf16 x 2) accesses.
+__global__ void __launch_bounds__(128)
+    rope_kernel(__nv_bfloat16* __restrict__ qkv, long long R, int ld, int d, int Dh, int P,
+                float log2_theta) {
+  const long long row = blockIdx.x * 4LL + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= R) return;
   const int half = Dh / 2;
   const float pos = static_cast<float>(row % P);
   __nv_bfloat16* base = qkv + static_cast<size_t>(row) * ld;
-  const int pairs = d / 2;  // per q or k block
-  for (int p = threadIdx.x; p < 2 * pairs; p += blockDim.x) {
-    const int which = p / pairs;  // 0 = q, 1 = k
-    const int pp = p - which * pairs;
-    const int head = pp / half;
-    const int i = pp - head * half;
-    const float inv_freq = exp2f(-(2.0f * i / Dh) * log2_theta);
-    float sn, cs;
-    sincosf(pos * inv_freq, &sn, &cs);
-    __nv_bfloat16* hp = base + which * d + head * Dh;
-    const float x1 = __bfloat162float(hp[i]);
-    const float x2 = __bfloat162float(hp[i + half]);
-    hp[i] = __float2bfloat16_rn(x1 * cs - x2 * sn);
-    hp[i + half] = __float2bfloat16_rn(x1 * sn + x2 * cs);
+  const int heads = d / Dh;
+  for (int i = 2 * lane; i < half; i += 64) {
+    float c0, s0, c1, s1;
+    sincosf(pos * exp2f(-(2.0f * i / Dh) * log2_theta), &s0, &c0);
+    sincosf(pos * exp2f(-(2.0f * (i + 1) / Dh) * log2_theta), &s1, &c1);
+    for (int hb = 0; hb < 2 * heads; ++hb) {  // q heads then k heads (k block starts at d)
+      uint32_t* p1 = reinterpret_cast<uint32_t*>(base + hb * Dh + i);
+      uint32_t* p2 = reinterpret_cast<uint32_t*>(base + hb * Dh + i + half);
+      const float2 x1 = unpack_bf16x2(*p1), x2 = unpack_bf16x2(*p2);
+      *p1 = pack_bf16x2(x1.x * c0 - x2.x * s0, x1.y * c1 - x2.y * s1);
+      *p2 = pack_bf16x2(x1.x * s0 + x2.x * c0, x1.y * s1 + x2.y * c1);
+    }
   }
 }
 
@@ -258,7 +261,7 @@ int launch_rmsnorm(const float* x, const void* w, int64_t rows, int64_t d, float
 int launch_rope(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t Dh, int64_t P, float theta,
                 cudaStream_t st) {
   if (R == 0) return 0;
-  rope_kernel<<<static_cast<unsigned>(R), 256, 0, st>>>(static_cast<__nv_bfloat16*>(qkv), R,
+  rope_kernel<<<static_cast<unsigned>((R + 3) / 4), 128, 0, st>>>(static_cast<__nv_bfloat16*>(qkv), R,
                                                         static_cast<int>(ld), static_cast<int>(d),
                                                         static_cast<int>(Dh), static_cast<int>(P),
                                                         log2f(theta));

@@ -45,8 +45,16 @@ constexpr int SMEM_BYTES =
     1024 + STAGES * STAGE_BYTES + EPI_WARPS * 2 * STAGING_BYTES + NUM_BARS * 8 + 16;
 constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN);
 
+// Epilogue modes (what a drained accumulator tile becomes):
+//  EPI_STORE    y = acc (bf16 or fp32)
+//  EPI_SWIGLU   columns [0, 128) of the tile are gate, [128, 256) up for the same 128
+//               features: y[:, n0/2 + j] = bf16(silu(bf16(gate_j)) * bf16(up_j))
+//  EPI_RESIDUAL y (fp32 residual stream) += float(bf16(acc)) by TMA reduce-add in L2
+enum { EPI_STORE = 0, EPI_SWIGLU = 1, EPI_RESIDUAL = 2 };
+
 struct Params {
   int M, N, K;
+  int epi;
   int kb_main;  // ceil(K / BK)
   int kb_lora;  // ceil(r / BK); 0 = no LoRA
   int r;
@@ -80,6 +88,17 @@ __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, uint32_t sr
                "r"(x), "r"(y), "r"(src)
                : "memory");
 }
+__device__ __forceinline__ void tma_reduce_add_2d(const CUtensorMap* map, uint32_t src, int x,
+                                                  int y) {
+  asm volatile(
+      "cp.reduce.async.bulk.tensor.2d.global.shared::cta.add.tile.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+          reinterpret_cast<uint64_t>(map)),
+      "r"(x), "r"(y), "r"(src)
+      : "memory");
+}
+__device__ __forceinline__ float bf16_round(float v) {
+  return __bfloat162float(__float2bfloat16_rn(v));
+}
 __device__ __forceinline__ void bulk_commit() {
   asm volatile("cp.async.bulk.commit_group;" ::: "memory");
 }
@@ -106,7 +125,9 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t
 __device__ __forceinline__ void drain(uint32_t tmem_acc, int q, int lane, uint32_t staging,
                                       uint32_t& chunk_ctr, const Params& p, int m0, int n0,
                                       const CUtensorMap* t0, const CUtensorMap* t1) {
-  const int nchunks = p.out_f32 ? BN / 32 : BN / 64;
+  // output chunks of 128 bytes per row: fp32 32 columns, bf16 64 columns, SwiGLU 64
+  // output columns from 128 accumulator columns
+  const int nchunks = p.epi == EPI_SWIGLU ? 2 : ((p.out_f32 || p.epi == EPI_RESIDUAL) ? BN / 32 : BN / 64);
   const uint32_t lane_taddr = tmem_acc + (static_cast<uint32_t>(q * 32) << 16);
   const int y = m0 + q * 32;
   for (int c = 0; c < nchunks; ++c) {
@@ -115,7 +136,30 @@ __device__ __forceinline__ void drain(uint32_t tmem_acc, int q, int lane, uint32
     __syncwarp();
     uint32_t w[32];
     int x;
-    if (p.out_f32) {
+    if (p.epi == EPI_SWIGLU) {
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        uint32_t g[32], u[32];
+        tc_ld_32x32b_x32(lane_taddr + c * 64 + h * 32, g);
+        tc_ld_32x32b_x32(lane_taddr + BN / 2 + c * 64 + h * 32, u);
+        tc_wait_ld();
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const float g0 = bf16_round(__uint_as_float(g[2 * i]));
+          const float g1 = bf16_round(__uint_as_float(g[2 * i + 1]));
+          const float u0 = bf16_round(__uint_as_float(u[2 * i]));
+          const float u1 = bf16_round(__uint_as_float(u[2 * i + 1]));
+          w[h * 16 + i] = pack_bf16x2(g0 / (1.0f + expf(-g0)) * u0, g1 / (1.0f + expf(-g1)) * u1);
+        }
+      }
+      x = n0 / 2 + c * 64;
+    } else if (p.epi == EPI_RESIDUAL) {
+      tc_ld_32x32b_x32(lane_taddr + c * 32, w);
+      tc_wait_ld();
+#pragma unroll
+      for (int i = 0; i < 32; ++i) w[i] = __float_as_uint(bf16_round(__uint_as_float(w[i])));
+      x = n0 + c * 32;
+    } else if (p.out_f32) {
       tc_ld_32x32b_x32(lane_taddr + c * 32, w);
       tc_wait_ld();
       x = n0 + c * 32;
@@ -139,9 +183,15 @@ __device__ __forceinline__ void drain(uint32_t tmem_acc, int q, int lane, uint32
     fence_async_smem();
     __syncwarp();
     if (lane == 0) {
-      if (x < p.N && y < p.M) {
-        if (t0) tma_store_2d(t0, buf, x, y);
-        if (t1) tma_store_2d(t1, buf, x, y);
+      const int n_out = p.epi == EPI_SWIGLU ? p.N / 2 : p.N;
+      if (x < n_out && y < p.M) {
+        if (p.epi == EPI_RESIDUAL) {
+          if (t0) tma_reduce_add_2d(t0, buf, x, y);
+          if (t1) tma_reduce_add_2d(t1, buf, x, y);
+        } else {
+          if (t0) tma_store_2d(t0, buf, x, y);
+          if (t1) tma_store_2d(t1, buf, x, y);
+        }
       }
       bulk_commit();
     }
@@ -436,13 +486,17 @@ int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream) {
     m_b = m_w;
   }
   const void* any_y = a.y_off ? a.y_off : a.y_on;
-  if (!make_map(&m_yoff, a.y_off ? a.y_off : any_y, a.M, a.N, 32, f32)) return -2;
-  if (!make_map(&m_yon, a.y_on ? a.y_on : any_y, a.M, a.N, 32, f32)) return -2;
+  // output tensor: SwiGLU writes bf16 [M, N/2]; the residual mode adds into fp32 [M, N]
+  const int64_t n_out = a.epi == tcgemm::EPI_SWIGLU ? a.N / 2 : a.N;
+  const bool out32 = a.epi == tcgemm::EPI_RESIDUAL ? true : (a.epi == tcgemm::EPI_SWIGLU ? false : f32);
+  if (!make_map(&m_yoff, a.y_off ? a.y_off : any_y, a.M, n_out, 32, out32)) return -2;
+  if (!make_map(&m_yon, a.y_on ? a.y_on : any_y, a.M, n_out, 32, out32)) return -2;
 
   Params p;
   p.M = static_cast<int>(a.M);
   p.N = static_cast<int>(a.N);
   p.K = static_cast<int>(a.K);
+  p.epi = a.epi;
   p.kb_main = static_cast<int>((a.K + BK - 1) / BK);
   p.kb_lora = lora ? static_cast<int>((a.r + BK - 1) / BK) : 0;
   p.r = static_cast<int>(a.r);

@@ -61,7 +61,7 @@ inline hydra_status rc(int r) { return r == 0 ? HYDRA_OK : HYDRA_ERR_CUDA; }
 
 // Workspace layout of the full pass, in bytes from the workspace base.
 struct PassLayout {
-  size_t h, a, qkv, attn, y, gu, m, u, fin, logits, sc, total;
+  size_t h, a, qkv, attn, m, u, fin, logits, sc, total;
 };
 
 PassLayout layout(const hydra_llama_config& c, int64_t S) {
@@ -76,8 +76,6 @@ PassLayout layout(const hydra_llama_config& c, int64_t S) {
   L.a = o;      o += up256(R * d * 2);
   L.qkv = o;    o += up256(R * 3 * d * 2);
   L.attn = o;   o += up256(R * d * 2);
-  L.y = o;      o += up256(R * d * 2);
-  L.gu = o;     o += up256(R * 2 * F * 2);
   L.m = o;      o += up256(R * F * 2);
   L.u = o;      o += up256(T * 2 * static_cast<size_t>(c.lora_rank) * 2);
   L.fin = o;    o += up256(2 * SL * d * 2);
@@ -91,7 +89,7 @@ bool valid_config(const hydra_llama_config* c) {
   if (c == nullptr) return false;
   if (c->n_layers < 1 || c->head_dim != 128 || c->n_heads < 1) return false;
   if (c->d_model != c->n_heads * c->head_dim) return false;
-  if (c->ffn < 8 || c->ffn % 8 != 0 || c->vocab < 8 || c->vocab % 8 != 0) return false;
+  if (c->ffn < 128 || c->ffn % 128 != 0 || c->vocab < 8 || c->vocab % 8 != 0) return false;
   if (c->lora_rank < 8 || c->lora_rank > 128 || c->lora_rank % 8 != 0) return false;
   if (c->prompt_len < 1 || c->response_len < 1) return false;
   if (c->response_len > hydra::kGaeMaxL) return false;
@@ -99,11 +97,15 @@ bool valid_config(const hydra_llama_config* c) {
 }
 
 // stacked dual linear: rows [0, T) of x are the off stream, [T, 2T) the on stream
-int stacked_linear(const void* x, int64_t T, int64_t K, int64_t N, const void* W, const void* A,
-                   const void* B, int64_t r, float s, void* u, void* y, bool f32, int* err,
-                   cudaStream_t st) {
+// epi: tcgen05 epilogue; y is [2T, N] (store), [2T, N/2] bf16 (SwiGLU) or the fp32 residual
+// stream [2T, N] (residual add)
+int stacked_linear(int prof_class, const void* x, int64_t T, int64_t K, int64_t N, const void* W,
+                   const void* A, const void* B, int64_t r, float s, void* u, void* y, bool f32,
+                   int* err, cudaStream_t st, int epi = HYDRA_EPI_STORE) {
   const size_t xs = static_cast<size_t>(T) * K * 2;
-  const size_t ys = static_cast<size_t>(T) * N * (f32 ? 4 : 2);
+  const size_t ys = epi == HYDRA_EPI_SWIGLU    ? static_cast<size_t>(T) * (N / 2) * 2
+                    : epi == HYDRA_EPI_RESIDUAL ? static_cast<size_t>(T) * N * 4
+                                                : static_cast<size_t>(T) * N * (f32 ? 4 : 2);
   const void* x_off = x;
   const void* x_on = static_cast<const uint8_t*>(x) + xs;
   if (r > 0) {
@@ -111,7 +113,7 @@ int stacked_linear(const void* x, int64_t T, int64_t K, int64_t N, const void* W
     const int e = hydra::launch_lora_down(x_on, T, K, A, r, s, u, st);
     if (e != 0) return e;
   }
-  ProfScope ps(HYDRA_PROF_GEMM, st);
+  ProfScope ps(prof_class, st);
   hydra::GemmArgs g;
   g.x_off = x_off;
   g.x_on = x_on;
@@ -127,8 +129,8 @@ int stacked_linear(const void* x, int64_t T, int64_t K, int64_t N, const void* W
   g.y_on = static_cast<uint8_t*>(y) + ys;
   g.out_f32 = f32 ? 1 : 0;
   g.err = err;
-  return (2 * T <= hydra::kGemvMaxRows) ? hydra::launch_dual_lora_gemv(g, st)
-                                        : hydra::launch_dual_lora_gemm_tc(g, st);
+  g.epi = epi;
+  return hydra::launch_dual_lora_gemm_tc(g, st);
 }
 
 }  // namespace
@@ -158,8 +160,9 @@ hydra_status hydra_rmsnorm(const float* x, const void* w, int64_t rows, int64_t 
 hydra_status hydra_rope(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t head_dim, int64_t P,
                         float theta, void* stream) {
   if (qkv == nullptr) return HYDRA_ERR_NULL;
-  if (R < 0 || P < 1 || head_dim < 2 || head_dim % 2 != 0 || d % head_dim != 0 || ld < 2 * d)
+  if (R < 0 || P < 1 || head_dim < 4 || head_dim % 4 != 0 || d % head_dim != 0 || ld < 2 * d)
     return HYDRA_ERR_SHAPE;
+  if (ld % 2 != 0 || (reinterpret_cast<uintptr_t>(qkv) & 3u) != 0) return HYDRA_ERR_ALIGN;
   if (!(theta > 0.f)) return HYDRA_ERR_RANGE;
   return rc(hydra::launch_rope(qkv, R, ld, d, head_dim, P, theta, static_cast<cudaStream_t>(stream)));
 }
@@ -275,8 +278,6 @@ hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_
   void* a = ws + Lo.a;
   void* qkv = ws + Lo.qkv;
   void* attn = ws + Lo.attn;
-  void* y = ws + Lo.y;
-  void* gu = ws + Lo.gu;
   void* m = ws + Lo.m;
   void* u = ws + Lo.u;
   void* fin = ws + Lo.fin;
@@ -306,24 +307,25 @@ hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_
     const hydra_llama_layer& ly = w->layers[l];
     // attention block
     HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(h, ly.norm_attn, R, d, c.rms_eps, ident, a, st));
-    HY_TRY(stacked_linear(a, T, d, 3 * d, ly.w_qkv, ly.a_qv, ly.b_qkv, 2 * r, s, u, qkv, false,
+    HY_TRY(stacked_linear(HYDRA_PROF_GEMM_QKV, a, T, d, 3 * d, ly.w_qkv, ly.a_qv, ly.b_qkv, 2 * r, s, u, qkv, false,
                           err, st));
     HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rope(qkv, R, 3 * d, d, c.head_dim, P, c.rope_theta, st));
     HY_PROF(HYDRA_PROF_ATTENTION,
             hydra::launch_causal_attention(qkv, 2 * S, P, 3 * d, c.n_heads, c.head_dim, attn, d, st));
-    HY_TRY(stacked_linear(attn, T, d, d, ly.w_o, nullptr, nullptr, 0, s, u, y, false, err, st));
-    HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_residual_add(h, y, R * d, st));
-    // feed-forward block
+    // o projection added straight into the residual stream (fused epilogue)
+    HY_TRY(stacked_linear(HYDRA_PROF_GEMM_O, attn, T, d, d, ly.w_o, nullptr, nullptr, 0, s, u, h, false, err, st,
+                          HYDRA_EPI_RESIDUAL));
+    // feed-forward block: gate/up with the SwiGLU fused into the epilogue, down added into h
     HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(h, ly.norm_ffn, R, d, c.rms_eps, ident, a, st));
-    HY_TRY(stacked_linear(a, T, d, 2 * F, ly.w_gu, ly.a_gu, ly.b_gu, 2 * r, s, u, gu, false, err, st));
-    HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_swiglu(gu, R, F, m, st));
-    HY_TRY(stacked_linear(m, T, F, d, ly.w_down, ly.a_down, ly.b_down, r, s, u, y, false, err, st));
-    HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_residual_add(h, y, R * d, st));
+    HY_TRY(stacked_linear(HYDRA_PROF_GEMM_GU, a, T, d, 2 * F, ly.w_gu, ly.a_gu, ly.b_gu, 2 * r, s, u, m, false, err, st,
+                          HYDRA_EPI_SWIGLU));
+    HY_TRY(stacked_linear(HYDRA_PROF_GEMM_DOWN, m, T, F, d, ly.w_down, ly.a_down, ly.b_down, r, s, u, h, false, err, st,
+                          HYDRA_EPI_RESIDUAL));
   }
   // final norm on the rows that predict response tokens: row P0 - 1 + t of each sequence
   const hydra::RowMap resp{L, P, c.prompt_len - 1};
   HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(h, w->final_norm, 2 * SL, d, c.rms_eps, resp, fin, st));
-  HY_TRY(stacked_linear(fin, SL, d, V, w->lm_head, nullptr, nullptr, 0, s, u, logits, true, err, st));
+  HY_TRY(stacked_linear(HYDRA_PROF_GEMM_LMHEAD, fin, SL, d, V, w->lm_head, nullptr, nullptr, 0, s, u, logits, true, err, st));
   // reward-model score on the LoRA-off stream at the last valid token; values on the
   // LoRA-on stream (the same head: r_phi = LO(V))
   HY_PROF(HYDRA_PROF_HEADS, hydra::launch_seq_score(h, w->final_norm, w->w_rm, d, c.rms_eps,

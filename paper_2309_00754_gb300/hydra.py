@@ -34,6 +34,8 @@ _SIGNATURES = {
                                               ctypes.c_size_t, ctypes.c_int, _vp]),
     "hydra_dual_linear": (ctypes.c_int, [_vp, _vp, _c_i64, _c_i64, _c_i64, _vp, _vp, _vp, _c_i64,
                                          _vp, _vp, ctypes.c_int, ctypes.c_int, _vp]),
+    "hydra_dual_linear_ex": (ctypes.c_int, [_vp, _vp, _c_i64, _c_i64, _c_i64, _vp, _vp, _vp,
+                                            _c_i64, _vp, _vp, ctypes.c_int, ctypes.c_int, _vp]),
     "hydra_lora_linear_noalloc": (ctypes.c_int, [_vp, _vp, _c_i64, _c_i64, _c_i64, _vp, _vp, _vp,
                                                  _c_i64, ctypes.c_float, _vp, _vp, ctypes.c_int,
                                                  _vp]),
@@ -220,6 +222,26 @@ def hydra_lora_linear_noalloc(x_off, x_on, W, A, B, s, y_off, y_on, stream=None)
         out_dtype, _stream(stream)))
 
 
+EPI_STORE, EPI_SWIGLU, EPI_RESIDUAL = 0, 1, 2
+
+
+def hydra_dual_linear_ex(x_off, x_on, W, u, B, y_off, y_on, epilogue, stream=None):
+    """tcgen05 dual linear with a fused epilogue (EPI_STORE, EPI_SWIGLU: bf16 [M, N/2] from
+    128-row-interleaved gate/up weights, EPI_RESIDUAL: fp32 [M, N] += bf16 result)."""
+    for t, n in ((x_off, "x_off"), (x_on, "x_on"), (W, "W"), (u, "u"), (B, "B")):
+        _req(t, torch.bfloat16, n)
+    out = y_off if y_off is not None else y_on
+    out_dtype = HYDRA_F32 if out.dtype == torch.float32 else HYDRA_BF16
+    for t, n in ((y_off, "y_off"), (y_on, "y_on")):
+        _req(t, out.dtype, n)
+    M, K = x_off.shape
+    N = W.shape[0]
+    r = 0 if u is None else u.shape[1]
+    _check("hydra_dual_linear_ex", load().hydra_dual_linear_ex(
+        _p(x_off), _p(x_on), M, K, N, _p(W), _p(u), _p(B), r, _p(y_off), _p(y_on), out_dtype,
+        int(epilogue), _stream(stream)))
+
+
 def hydra_token_logprobs_kl(logits_actor, logits_ref, ids, lengths, seq_score, beta, S, L,
                             logp_actor, logp_ref, reward_tok, lse_actor=None, lse_ref=None,
                             stream=None):
@@ -361,7 +383,9 @@ def hydra_score_llama(cfg, weights, ids, lengths, workspace, outputs, stream=Non
         *[_p(outputs[k]) for k in names], _stream(stream)))
 
 
-PROF_CLASSES = ("gemm", "lora_down", "attention", "elementwise", "logprobs", "gae", "heads")
+PROF_CLASSES = ("gemm_qkv", "gemm_o", "gemm_gu", "gemm_down", "gemm_lmhead", "lora_down",
+                "attention", "elementwise", "logprobs", "gae", "heads")
+GEMM_CLASSES = PROF_CLASSES[:5]
 
 
 def profile_enable(on=True):

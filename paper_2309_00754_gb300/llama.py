@@ -1,8 +1,10 @@
 """Llama-7B-shaped model weights in the layouts hydra_score_llama takes (include/hydra.h):
 q/k/v fused into w_qkv [3d, d] with LoRA a_qv [2r, d] / b_qkv [3d, 2r] block-structured so
-that q and v carry their own LoRA pair and k none; gate/up fused into w_gu [2F, d] with
-a_gu [2r, d] / b_gu [2F, 2r]; down with its own rank-r pair. This module only arranges
-tensors; all arithmetic runs in libhydra."""
+that q and v carry their own LoRA pair and k none; gate/up fused into w_gu [2F, d], their
+rows interleaved in blocks of 128 (gate block j, then up block j) so that one 256-column
+output tile holds matching gate and up features, with a_gu [2r, d] / b_gu [2F, 2r]; down
+with its own rank-r pair. This module only arranges tensors; all arithmetic runs in
+libhydra."""
 from __future__ import annotations
 
 import numpy as np
@@ -14,6 +16,27 @@ LLAMA7B = dict(n_layers=32, d_model=4096, n_heads=32, head_dim=128, ffn=11008, v
 
 LAYER_KEYS = ("w_qkv", "a_qv", "b_qkv", "w_o", "w_gu", "a_gu", "b_gu", "w_down", "a_down",
               "b_down", "norm_attn", "norm_ffn")
+
+
+def interleave_gate_up(gate, up, block=128):
+    """Rows [g_0..g_127, u_0..u_127, g_128.., u_128.., ...] from gate [F, *] and up [F, *]
+    (numpy or torch)."""
+    F = gate.shape[0]
+    assert F % block == 0 and up.shape[0] == F
+    nb = F // block
+    g = gate.reshape(nb, block, *gate.shape[1:])
+    u = up.reshape(nb, block, *up.shape[1:])
+    if isinstance(gate, np.ndarray):
+        return np.stack([g, u], axis=1).reshape(2 * F, *gate.shape[1:])
+    return torch.stack([g, u], dim=1).reshape(2 * F, *gate.shape[1:])
+
+
+def deinterleave_gate_up(gu, block=128):
+    """(gate, up) from rows interleaved by interleave_gate_up."""
+    F = gu.shape[0] // 2
+    nb = F // block
+    x = gu.reshape(nb, 2, block, *gu.shape[1:])
+    return x[:, 0].reshape(F, *gu.shape[1:]), x[:, 1].reshape(F, *gu.shape[1:])
 
 
 def random_device_weights(cfg, seed, device, std=0.02):
@@ -36,12 +59,13 @@ def random_device_weights(cfg, seed, device, std=0.02):
         b[2 * d:, r:] = rnd(d, r)
         w["b_qkv"].append(b)
         w["w_o"].append(rnd(d, d))
-        w["w_gu"].append(rnd(2 * F, d))
+        w["w_gu"].append(rnd(2 * F, d))  # random rows: any interleave is equally random
         w["a_gu"].append(rnd(2 * r, d))
-        b = torch.zeros(2 * F, 2 * r, dtype=bf, device=device)
-        b[:F, :r] = rnd(F, r)
-        b[F:, r:] = rnd(F, r)
-        w["b_gu"].append(b)
+        bg = torch.zeros(F, 2 * r, dtype=bf, device=device)
+        bu = torch.zeros(F, 2 * r, dtype=bf, device=device)
+        bg[:, :r] = rnd(F, r)
+        bu[:, r:] = rnd(F, r)
+        w["b_gu"].append(interleave_gate_up(bg, bu))
         w["w_down"].append(rnd(d, F))
         w["a_down"].append(rnd(r, F))
         w["b_down"].append(rnd(d, r))
@@ -73,12 +97,13 @@ def fuse_separate(sep):
         b[2 * d:, r:] = lo["wv"][1][l]
         out["b_qkv"].append(b)
         out["w_o"].append(sep["wo"][l])
-        out["w_gu"].append(np.concatenate([sep["wg"][l], sep["wu"][l]], 0))
+        out["w_gu"].append(interleave_gate_up(sep["wg"][l], sep["wu"][l]))
         out["a_gu"].append(np.concatenate([lo["wg"][0][l], lo["wu"][0][l]], 0))
-        b = np.zeros((2 * F, 2 * r), dtype=np.uint16)
-        b[:F, :r] = lo["wg"][1][l]
-        b[F:, r:] = lo["wu"][1][l]
-        out["b_gu"].append(b)
+        bg = np.zeros((F, 2 * r), dtype=np.uint16)
+        bu = np.zeros((F, 2 * r), dtype=np.uint16)
+        bg[:, :r] = lo["wg"][1][l]
+        bu[:, r:] = lo["wu"][1][l]
+        out["b_gu"].append(interleave_gate_up(bg, bu))
         out["w_down"].append(sep["wd"][l])
         out["a_down"].append(lo["wd"][0][l])
         out["b_down"].append(lo["wd"][1][l])

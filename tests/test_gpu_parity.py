@@ -267,3 +267,66 @@ def test_decode_gemv_sampled(M):
         ref_off, ref_on = O.dual_lora_linear(f64(x), f64(x), f64(W), f64(A), f64(Bm), 2.0)
         assert_rel(host_f64(y_off), ref_off, TOL_LINEAR, "y_off")
         assert_rel(host_f64(y_on), ref_on, TOL_LINEAR, "y_on")
+
+
+# ------------------------------------------------------------------ fused epilogues
+
+
+@pytest.mark.parametrize("shared", [True, False])
+def test_swiglu_epilogue(shared):
+    """Gate/up projection with the SwiGLU fused into the tcgen05 epilogue."""
+    from paper_2309_00754_gb300 import llama
+    M, K, F, r = 300, 512, 384, 16
+    x, x2, _, _, _ = _linear_problem(M, K, 8, 8, seed=41)
+    Wg = synth.normal_bf16(411, (F, K), 0.02)
+    Wu = synth.normal_bf16(412, (F, K), 0.02)
+    Bg = synth.normal_bf16(413, (F, r), 0.02)
+    Bu = synth.normal_bf16(414, (F, r), 0.02)
+    u = synth.normal_bf16(415, (M, 2 * r), 2.0)
+    zg = np.zeros((F, r), np.uint16)
+    Bcat_g = np.concatenate([Bg, zg], 1)
+    Bcat_u = np.concatenate([zg, Bu], 1)
+    W = llama.interleave_gate_up(Wg, Wu)
+    B = llama.interleave_gate_up(Bcat_g, Bcat_u)
+    xo = x if shared else x2
+    y_off = torch.full((M, F), float("nan"), dtype=torch.bfloat16, device="cuda")
+    y_on = torch.full((M, F), float("nan"), dtype=torch.bfloat16, device="cuda")
+    H.hydra_dual_linear_ex(dev_bf16(x), None if shared else dev_bf16(x2), dev_bf16(W),
+                           dev_bf16(u), dev_bf16(B), y_off, y_on, H.EPI_SWIGLU)
+    uu = f64(u)
+    g_off = O.round_bf16(f64(x) @ f64(Wg).T)
+    u_off = O.round_bf16(f64(x) @ f64(Wu).T)
+    g_on = O.round_bf16(f64(xo) @ f64(Wg).T + uu @ f64(Bcat_g).T)
+    u_on = O.round_bf16(f64(xo) @ f64(Wu).T + uu @ f64(Bcat_u).T)
+    assert_rel(host_f64(y_off), O.round_bf16(O.swiglu(g_off, u_off)), TOL_LINEAR, "swiglu off")
+    assert_rel(host_f64(y_on), O.round_bf16(O.swiglu(g_on, u_on)), TOL_LINEAR, "swiglu on")
+
+
+@pytest.mark.parametrize("shared", [True, False])
+def test_residual_epilogue(shared):
+    """Projection added into an fp32 residual stream by the tcgen05 epilogue."""
+    M, K, N, r = 260, 640, 520, 16
+    x, x2, W, _, B = _linear_problem(M, K, N, r, seed=42)
+    u = synth.normal_bf16(421, (M, r), 2.0)
+    h0 = synth.normal_f32(422, (2, M, N), 3.0)
+    h = dev_f32(h0)
+    xo = x if shared else x2
+    H.hydra_dual_linear_ex(dev_bf16(x), None if shared else dev_bf16(x2), dev_bf16(W),
+                           dev_bf16(u), dev_bf16(B), h[0], h[1], H.EPI_RESIDUAL)
+    y_off = O.round_bf16(f64(x) @ f64(W).T)
+    y_on = O.round_bf16(f64(xo) @ f64(W).T + f64(u) @ f64(B).T)
+    got = host_f64(h)
+    assert_rel(got[0], h0[0].astype(np.float64) + y_off, TOL_LINEAR, "residual off")
+    assert_rel(got[1], h0[1].astype(np.float64) + y_on, TOL_LINEAR, "residual on")
+
+
+def test_epilogue_argument_errors():
+    x = torch.zeros(16, 64, dtype=torch.bfloat16, device="cuda")
+    W = torch.zeros(200, 64, dtype=torch.bfloat16, device="cuda")
+    y = torch.zeros(16, 100, dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(H.HydraError) as e:  # SwiGLU needs N % 256 == 0
+        H.hydra_dual_linear_ex(x, None, W, None, None, y, None, H.EPI_SWIGLU)
+    assert e.value.status == 2
+    with pytest.raises(H.HydraError) as e:
+        H.hydra_dual_linear_ex(x, None, W, None, None, y, None, 7)
+    assert e.value.status == 4
