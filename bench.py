@@ -409,7 +409,124 @@ class HydraScoringLlama7B:
         return smp["resp"] * len(t_pass) / sum(t_pass), desc
 
 
-WORKLOADS = {LmHeadScoring.name: LmHeadScoring, HydraScoringLlama7B.name: HydraScoringLlama7B}
+class KernelSweep:
+    """Per-kernel measurements of the rows the full pass does not exercise at their own
+    shapes (one JSON line; value = the sweep's mean fraction of roofline):
+      projection sweep: M = 2048 tokens through q/k/v/o (4096 -> 4096), gate/up
+        (4096 -> 11008), down (11008 -> 4096), shared input, LoRA r in {8, 16, 64}, s = 2,
+        both outputs -> TFLOP/s (the tensor-core dual-output kernel);
+      decode: M in {1, 4, 8, 16} token rows through the distinct projection shapes
+        (4096 -> 4096, 4096 -> 11008, 11008 -> 4096) and the 4096 -> 32000 LM head, r = 16,
+        both outputs -> GB/s of W + x + u + y (the GEMV);
+    Kernels are replayed back to back from CUDA graphs, weights rotated through copies
+    larger than L2.
+      GAE: 65536 sequences x 512 tokens -> GB/s;
+      log-probs/KL: 2048 rows x 32000 fp32 logits x 2 heads -> GB/s."""
+
+    name = "kernel_sweep"
+    seed = 5
+    PROJ = (("q", 4096, 4096), ("k", 4096, 4096), ("v", 4096, 4096), ("o", 4096, 4096),
+            ("gate", 4096, 11008), ("up", 4096, 11008), ("down", 11008, 4096))
+
+    def __init__(self, device, seed=5, reference=False):
+        self.device = device
+
+    def run(self, peaks, reps=20):
+        import torch
+        from paper_2309_00754_gb300 import hydra as H
+        g = torch.Generator(device=self.device)
+        g.manual_seed(self.seed)
+        bf = torch.bfloat16
+        dev = self.device
+
+        def rnd(*shape, std=0.02):
+            return (std * torch.randn(*shape, device=dev, generator=g)).to(bf)
+
+        def graph_ms(launch, n):
+            """Mean time per launch of n back-to-back launches replayed from a CUDA graph
+            (no host gaps between kernels)."""
+            launch(0)  # first call outside capture (one-time kernel attribute set-up)
+            torch.cuda.synchronize()
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph):
+                for i in range(n):
+                    launch(i)
+            graph.replay()
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            graph.replay()
+            e1.record()
+            torch.cuda.synchronize()
+            return e0.elapsed_time(e1) / n
+
+        out = {"projection_sweep": {}, "decode": {}, "gae": {}, "logprobs": {}}
+        # ---- projection sweep (c2): W rotates through 3 copies per shape so consecutive
+        # launches do not find W in L2
+        M = 2048
+        x = torch.randn(M, 11008, device=dev, generator=g).to(bf)
+        fr = []
+        for r in (8, 16, 64):
+            for name, K, N in self.PROJ:
+                Ws = [rnd(N, K) for _ in range(3)]
+                B = rnd(N, r)
+                u = rnd(M, r, std=1.0)
+                xs = x[:, :K].contiguous()
+                y0 = torch.empty(M, N, dtype=bf, device=dev)
+                y1 = torch.empty(M, N, dtype=bf, device=dev)
+                ms = graph_ms(lambda i: H.hydra_dual_linear(xs, None, Ws[i % 3], u, B, y0, y1, algo=1), reps)
+                tf = (2.0 * M * K * N + 2.0 * M * r * N) / ms / 1e9
+                out["projection_sweep"][f"{name}_r{r}"] = {"ms": ms, "TFLOP/s": tf}
+                fr.append(tf / peaks["bf16_tflops"])
+                del Ws
+        sweep = out["projection_sweep"]
+        sweep["mean_TFLOP/s"] = statistics.mean(v["TFLOP/s"] for v in list(sweep.values()))
+        sweep["frac_of_measured_burst"] = statistics.mean(fr)
+        sweep["frac_of_2.25PF"] = sweep["mean_TFLOP/s"] / 2250.0
+        # ---- decode (c5): W rotates through enough copies that they exceed L2
+        shapes = list(self.PROJ[:1]) + list(self.PROJ[4:5]) + list(self.PROJ[6:]) + [("lm_head", 4096, 32000)]
+        gb = []
+        for n, K, N in shapes:
+            ncopy = max(2, -(-300_000_000 // (N * K * 2)))  # > 2 x L2 of weights
+            Wd = [rnd(N, K) for _ in range(ncopy)]
+            Bd = rnd(N, 16)
+            for Mt in (1, 4, 8, 16):
+                xd = torch.randn(Mt, K, device=dev, generator=g).to(bf)
+                ud = rnd(Mt, 16, std=1.0)
+                y0 = torch.empty(Mt, N, dtype=bf, device=dev)
+                y1 = torch.empty(Mt, N, dtype=bf, device=dev)
+                ms = graph_ms(lambda i: H.hydra_dual_linear(xd, None, Wd[i % ncopy], ud, Bd, y0, y1),
+                              max(reps, 2 * ncopy))
+                byts = 2.0 * (N * K + 16 * (K + N) + Mt * K + 2 * Mt * N)
+                out["decode"].setdefault(f"M{Mt}", {})[n] = {"ms": ms, "GB/s": byts / ms / 1e6}
+                gb.append(byts / ms / 1e6)
+            del Wd
+        out["decode"]["frac_of_measured_hbm_mean"] = statistics.mean(gb) / peaks["hbm_gbs"]
+        # ---- GAE at 65536 x 512
+        S, L = 65536, 512
+        rw = torch.randn(S, L, device=dev, generator=g)
+        vv = torch.randn(S, L, device=dev, generator=g)
+        ln = torch.randint(64, 513, (S,), device=dev, generator=g, dtype=torch.int32)
+        adv, ret = torch.empty_like(rw), torch.empty_like(rw)
+        ms = graph_ms(lambda i: H.ppo_gae(rw, vv, ln, 1.0, 0.95, adv, ret), reps)
+        valid = float(ln.sum().item())
+        byts = valid * 8 + S * L * 8 + S * 4  # read valid r, V; write all A, R
+        out["gae"] = {"ms": ms, "GB/s": byts / ms / 1e6, "frac_of_measured_hbm": byts / ms / 1e6 / peaks["hbm_gbs"]}
+        del rw, vv, adv, ret
+        # ---- log-probs/KL at 2048 x 32000 x 2 heads, all rows valid
+        T, V = 2048, 32000
+        za = torch.randn(T, V, device=dev, generator=g)
+        zr = torch.randn(T, V, device=dev, generator=g)
+        ids = torch.randint(0, V, (T,), device=dev, generator=g, dtype=torch.int32)
+        o3 = [torch.empty(T, device=dev) for _ in range(3)]
+        ms = graph_ms(lambda i: H.hydra_token_logprobs_kl(za, zr, ids, None, None, 0.1, 4, 512, *o3), reps)
+        byts = T * V * 4 * 2 + T * 16
+        out["logprobs"] = {"ms": ms, "GB/s": byts / ms / 1e6, "frac_of_measured_hbm": byts / ms / 1e6 / peaks["hbm_gbs"]}
+        return out
+
+
+WORKLOADS = {LmHeadScoring.name: LmHeadScoring, HydraScoringLlama7B.name: HydraScoringLlama7B,
+             KernelSweep.name: KernelSweep}
 DEFAULT_WORKLOAD = HydraScoringLlama7B.name
 
 
@@ -515,6 +632,23 @@ def run_reference(args, wl_cls):
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
                              "sample": "16 token rows of sequence 0 per step through the fp64 oracle"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_sweep(args):
+    import torch
+    torch.cuda.set_device(0)
+    import __graft_entry__
+    __graft_entry__.build()
+    peaks = load_peaks()
+    clocks = ClockSampler(0)
+    clocks.start()
+    res = KernelSweep(torch.device("cuda", 0)).run(peaks)
+    clk = clocks.stop()
+    line = {"metric": "per-kernel roofline fractions (projection sweep, decode GEMV, GAE, log-probs)",
+            "value": res["projection_sweep"]["frac_of_measured_burst"], "unit": "fraction",
+            "workload": KernelSweep.name, "results": res, "clocks": clk, "peaks": peaks}
     print(json.dumps(line), flush=True)
     return 0
 
@@ -631,6 +765,8 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args(argv)
     wl_cls = WORKLOADS[args.workload]
+    if wl_cls is KernelSweep:
+        return run_sweep(args)
     if args.impl == "reference":
         if args.steps is None:
             args.steps = 3 if args.workload == HydraScoringLlama7B.name else 20

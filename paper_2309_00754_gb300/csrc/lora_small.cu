@@ -5,28 +5,13 @@
 //    kernel and of the GEMV below. (Uses mma.sync: a skinny product far too narrow for a
 //    128-row tcgen05 tile to stay busy.)
 //  * dual_lora_gemv: the dual-output linear for decode-shaped inputs (at most 16 token
-//    rows over both streams), y_off = x_off W^T, y_on = x_on W^T + u B^T. One warp owns two
-//    rows of W and streams them once with 128-bit loads; the token rows are re-read from
-//    L1. Used where a 128-row tensor-core tile would be almost empty.
+//    rows over both streams), y_off = x_off W^T, y_on = x_on W^T + u B^T, streaming W once
+//    (see the kernel). Used where a 128-row tcgen05 tile would be almost empty.
 #include "common.cuh"
 #include "kernels.h"
 
 namespace hydra {
 namespace {
-
-__device__ __forceinline__ void unpack8(const uint4& v, float (&f)[8]) {
-  float2 a = unpack_bf16x2(v.x), b = unpack_bf16x2(v.y), c = unpack_bf16x2(v.z),
-         d = unpack_bf16x2(v.w);
-  f[0] = a.x; f[1] = a.y; f[2] = b.x; f[3] = b.y;
-  f[4] = c.x; f[5] = c.y; f[6] = d.x; f[7] = d.y;
-}
-
-__device__ __forceinline__ float dot8(const float (&a)[8], const float (&b)[8]) {
-  float s = a[0] * b[0];
-#pragma unroll
-  for (int i = 1; i < 8; ++i) s = fmaf(a[i], b[i], s);
-  return s;
-}
 
 // ---------------------------------------------------------------- lora_down
 //
@@ -118,129 +103,189 @@ __global__ void __launch_bounds__(32 * kDownWarps)
 }
 
 // ---------------------------------------------------------------- dual_lora_gemv
+//
+// Decode-shaped dual-output linear (at most 16 token rows over both streams). HBM-bound:
+// every byte of W is read once. One CTA per 16 rows of W; its 8 warps split K and stream
+// their [16 x 64] W and token-row slices into XOR-swizzled shared memory with cp.async
+// (3 stages per warp, 16-byte copies), then run mma.sync m16n8k16 with W as the 16-row
+// operand and the token rows as the 8-wide operand (both through ldmatrix), so the
+// arithmetic never limits the stream even at 16 rows. The 8 partial tiles are reduced in
+// shared memory, where each thread also adds the rank-r LoRA term of its (row, token).
 
-constexpr int kGemvNR = 2;  // W rows per warp
+constexpr int kGvWarps = 8;
+constexpr int kGvStages = 3;
+constexpr int kGvStageBytes = 2 * 16 * 128;  // 16 W rows + 16 token rows, 64 bf16 each
 
-template <int MT>
-__global__ void __launch_bounds__(256)
+__device__ __forceinline__ void gv_cp_async16(uint32_t dst, const void* src, bool ok) {
+  const int n = ok ? 16 : 0;
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(n)
+               : "memory");
+}
+__device__ __forceinline__ void gv_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void gv_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void gv_ldsm_x4(uint32_t addr, uint32_t (&a)[4]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(a[0]), "=r"(a[1]), "=r"(a[2]), "=r"(a[3])
+               : "r"(addr));
+}
+
+template <int NT>  // n-tiles of 8 token rows (1 or 2)
+__global__ void __launch_bounds__(32 * kGvWarps)
     dual_lora_gemv_kernel(const __nv_bfloat16* __restrict__ x_off,
                           const __nv_bfloat16* __restrict__ x_on, int M, int K, int N,
                           const __nv_bfloat16* __restrict__ W, const __nv_bfloat16* __restrict__ u,
                           const __nv_bfloat16* __restrict__ B, int r, void* y_off, void* y_on,
                           int out_f32, int shared_x) {
+  extern __shared__ __align__(1024) uint8_t smem[];
+  float* red = reinterpret_cast<float*>(smem + kGvWarps * kGvStages * kGvStageBytes);
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int n0 = (blockIdx.x * 8 + warp) * kGemvNR;
-  if (n0 >= N) return;
-  // token rows: [0, M) from x_off; in the stacked case rows [M, 2M) from x_on
-  const int rows = shared_x ? M : 2 * M;
-  float acc[MT][kGemvNR];
-#pragma unroll
-  for (int i = 0; i < MT; ++i)
-#pragma unroll
-    for (int q = 0; q < kGemvNR; ++q) acc[i][q] = 0.f;
+  const int g = lane >> 2, c = lane & 3;
+  const int n0 = blockIdx.x * 16;
+  const int tokens = shared_x ? M : 2 * M;  // token rows: x_off rows, then x_on rows
+  const uint32_t wsm = smem_u32(smem) + warp * kGvStages * kGvStageBytes;
 
-  for (int k = lane * 8; k < K; k += 256) {
-    float wv[kGemvNR][8];
+  // this warp's K range in chunks of 64
+  const int nchunk = (K + 63) / 64;
+  const int per = (nchunk + kGvWarps - 1) / kGvWarps;
+  const int c0 = warp * per;
+  const int c1 = min(nchunk, c0 + per);
+
+  // token row copied by this lane's slice of the x stage (rows lane >> 3 and 4 + lane >> 3...)
+  auto xrow = [&](int tk) {
+    return (tk < M) ? x_off + static_cast<size_t>(tk) * K : x_on + static_cast<size_t>(tk - M) * K;
+  };
+  auto issue = [&](int ch, int slot) {
+    const uint32_t base = wsm + slot * kGvStageBytes;
+    // W: 16 rows x 8 segments of 16 B, lane copies segments lane + 32 e
 #pragma unroll
-    for (int q = 0; q < kGemvNR; ++q) {
-      if (n0 + q < N) {
-        unpack8(__ldcs(reinterpret_cast<const uint4*>(W + static_cast<size_t>(n0 + q) * K + k)),
-                wv[q]);
-      } else {
-#pragma unroll
-        for (int e = 0; e < 8; ++e) wv[q][e] = 0.f;
-      }
+    for (int e = 0; e < 4; ++e) {
+      const int idx = lane + 32 * e;
+      const int row = idx >> 3, seg = idx & 7;
+      const int k = ch * 64 + seg * 8;
+      const bool ok = (n0 + row < N) && (k < K);
+      const __nv_bfloat16* src = W + static_cast<size_t>(ok ? n0 + row : 0) * K + (ok ? k : 0);
+      gv_cp_async16(base + row * 128 + ((seg ^ (row & 7)) << 4), src, ok);
     }
+    // token rows 0 .. 8 NT - 1 (missing rows and columns read as zero)
 #pragma unroll
-    for (int i = 0; i < MT; ++i) {
-      if (i < rows) {
-        const __nv_bfloat16* xr =
-            (i < M) ? x_off + static_cast<size_t>(i) * K : x_on + static_cast<size_t>(i - M) * K;
-        float xv[8];
-        unpack8(__ldg(reinterpret_cast<const uint4*>(xr + k)), xv);
-#pragma unroll
-        for (int q = 0; q < kGemvNR; ++q) acc[i][q] += dot8(xv, wv[q]);
-      }
+    for (int e = 0; e < NT * 2; ++e) {
+      const int idx = lane + 32 * e;
+      const int row = idx >> 3, seg = idx & 7;
+      const int k = ch * 64 + seg * 8;
+      const bool ok = (row < tokens) && (k < K);
+      const __nv_bfloat16* src = ok ? xrow(row) + k : W;
+      gv_cp_async16(base + 16 * 128 + row * 128 + ((seg ^ (row & 7)) << 4), src, ok);
     }
+  };
+  float d[NT][4];
+#pragma unroll
+  for (int t = 0; t < NT; ++t) d[t][0] = d[t][1] = d[t][2] = d[t][3] = 0.f;
+
+  // prologue: up to kGvStages - 1 chunks in flight
+#pragma unroll
+  for (int i = 0; i < kGvStages - 1; ++i) {
+    if (c0 + i < c1) issue(c0 + i, i);
+    gv_commit();
   }
+  for (int ch = c0; ch < c1; ++ch) {
+    const int i = ch - c0;
+    if (ch + kGvStages - 1 < c1) issue(ch + kGvStages - 1, (i + kGvStages - 1) % kGvStages);
+    gv_commit();
+    gv_wait<kGvStages - 1>();
+    __syncwarp();
+    const uint32_t st = wsm + (i % kGvStages) * kGvStageBytes;
 #pragma unroll
-  for (int i = 0; i < MT; ++i)
+    for (int kk = 0; kk < 4; ++kk) {
+      const int k0 = ch * 64 + kk * 16;
+      if (k0 >= K) break;
+      uint32_t a[4];
+      // matrices: rows (lane & 15), 16-byte segment 2 kk + (lane >> 4)
+      const int row = lane & 15;
+      gv_ldsm_x4(st + row * 128 + (((2 * kk + (lane >> 4)) ^ (row & 7)) << 4), a);
+      // B fragments of token rows t*8 .. t*8 + 7: matrices (rows lane & 7, segment 2 kk and
+      // 2 kk + 1) for n-tiles t = 0 (lanes 0-15) and t = 1 (lanes 16-31)
+      uint32_t b[4];
+      {
+        const int trow = (lane & 7) + ((lane >> 4) << 3);
+        const int seg = 2 * kk + ((lane >> 3) & 1);
+        gv_ldsm_x4(st + 16 * 128 + trow * 128 + ((seg ^ (trow & 7)) << 4), b);
+      }
 #pragma unroll
-    for (int q = 0; q < kGemvNR; ++q) {
-      float v = acc[i][q];
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-      acc[i][q] = v;
+      for (int t = 0; t < NT; ++t) mma_bf16_16816(d[t], a, b[2 * t], b[2 * t + 1]);
     }
+    __syncwarp();
+  }
+  gv_wait<0>();
 
-  // LoRA-up on the on-stream rows: lanes split the rank dimension
-  float lora[MT][kGemvNR];
+  // partial [16 rows x 8 NT tokens] of this warp -> shared memory
+  float* rw = red + warp * 16 * 16;
 #pragma unroll
-  for (int i = 0; i < MT; ++i)
+  for (int t = 0; t < NT; ++t) {
+    rw[g * 16 + t * 8 + 2 * c] = d[t][0];
+    rw[g * 16 + t * 8 + 2 * c + 1] = d[t][1];
+    rw[(g + 8) * 16 + t * 8 + 2 * c] = d[t][2];
+    rw[(g + 8) * 16 + t * 8 + 2 * c + 1] = d[t][3];
+  }
+  __syncthreads();
+  // one (row, token) output per thread: row fastest for coalesced stores
+  const int row = threadIdx.x & 15, tk = threadIdx.x >> 4;
+  const int n = n0 + row;
+  if (tk >= tokens || tk >= NT * 8 || n >= N) return;
+  float acc = 0.f;
 #pragma unroll
-    for (int q = 0; q < kGemvNR; ++q) lora[i][q] = 0.f;
-  if (u != nullptr) {
+  for (int w = 0; w < kGvWarps; ++w) acc += red[w * 256 + row * 16 + tk];
+  auto put = [&](void* y, int m, float v) {
+    if (y == nullptr) return;
+    const size_t o = static_cast<size_t>(m) * N + n;
+    if (out_f32)
+      reinterpret_cast<float*>(y)[o] = v;
+    else
+      reinterpret_cast<__nv_bfloat16*>(y)[o] = __float2bfloat16_rn(v);
+  };
+  auto lora = [&](int m) {
+    // rank-r dot product with 16-byte loads (r % 8 == 0)
+    float v = 0.f;
+    if (u != nullptr) {
+      const uint4* up = reinterpret_cast<const uint4*>(u + static_cast<size_t>(m) * r);
+      const uint4* bp = reinterpret_cast<const uint4*>(B + static_cast<size_t>(n) * r);
+      for (int j = 0; j < r / 8; ++j) {
+        const uint4 a4 = __ldg(up + j), b4 = __ldg(bp + j);
+        const uint32_t* ap = &a4.x;
+        const uint32_t* bq = &b4.x;
 #pragma unroll
-    for (int i = 0; i < MT; ++i) {
-      if (i < M) {
-#pragma unroll
-        for (int q = 0; q < kGemvNR; ++q) {
-          float v = 0.f;
-          if (n0 + q < N) {
-            for (int j = lane; j < r; j += 32)
-              v = fmaf(__bfloat162float(u[static_cast<size_t>(i) * r + j]),
-                       __bfloat162float(B[static_cast<size_t>(n0 + q) * r + j]), v);
-          }
-#pragma unroll
-          for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-          lora[i][q] = v;
+        for (int e = 0; e < 4; ++e) {
+          const float2 fa = unpack_bf16x2(ap[e]), fb = unpack_bf16x2(bq[e]);
+          v = fmaf(fa.x, fb.x, v);
+          v = fmaf(fa.y, fb.y, v);
         }
       }
     }
+    return v;
+  };
+  if (shared_x) {
+    put(y_off, tk, acc);
+    if (y_on != nullptr) put(y_on, tk, acc + lora(tk));
+  } else if (tk < M) {
+    put(y_off, tk, acc);
+  } else {
+    put(y_on, tk - M, acc + lora(tk - M));
   }
-
-#pragma unroll
-  for (int i = 0; i < MT; ++i)
-#pragma unroll
-    for (int q = 0; q < kGemvNR; ++q) {
-      if (((i * kGemvNR + q) & 31) != lane || i >= rows || n0 + q >= N) continue;
-      const int n = n0 + q;
-      // (output, token row, value) for this accumulator
-      void* dst0 = nullptr;
-      void* dst1 = nullptr;
-      int m;
-      float v0, v1 = 0.f;
-      if (shared_x) {
-        m = i;
-        dst0 = y_off;
-        v0 = acc[i][q];
-        dst1 = y_on;
-        v1 = acc[i][q] + lora[i][q];
-      } else if (i < M) {
-        m = i;
-        dst0 = y_off;
-        v0 = acc[i][q];
-      } else {
-        m = i - M;
-        dst0 = y_on;
-        v0 = acc[i][q] + lora[m][q];
-      }
-      const size_t o = static_cast<size_t>(m) * N + n;
-      if (out_f32) {
-        if (dst0) reinterpret_cast<float*>(dst0)[o] = v0;
-        if (dst1) reinterpret_cast<float*>(dst1)[o] = v1;
-      } else {
-        if (dst0) reinterpret_cast<__nv_bfloat16*>(dst0)[o] = __float2bfloat16_rn(v0);
-        if (dst1) reinterpret_cast<__nv_bfloat16*>(dst1)[o] = __float2bfloat16_rn(v1);
-      }
-    }
 }
 
-template <int MT>
+template <int NT>
 void launch_gemv_t(const GemmArgs& a, cudaStream_t stream) {
-  const unsigned grid = static_cast<unsigned>((a.N + 8 * kGemvNR - 1) / (8 * kGemvNR));
-  dual_lora_gemv_kernel<MT><<<grid, 256, 0, stream>>>(
+  constexpr int smem = kGvWarps * kGvStages * kGvStageBytes + kGvWarps * 16 * 16 * 4;
+  static bool attr = false;
+  if (!attr) {
+    cudaFuncSetAttribute(dual_lora_gemv_kernel<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    attr = true;
+  }
+  const unsigned grid = static_cast<unsigned>((a.N + 15) / 16);
+  dual_lora_gemv_kernel<NT><<<grid, 32 * kGvWarps, smem, stream>>>(
       static_cast<const __nv_bfloat16*>(a.x_off),
       static_cast<const __nv_bfloat16*>(a.shared_x ? a.x_off : a.x_on), static_cast<int>(a.M),
       static_cast<int>(a.K), static_cast<int>(a.N), static_cast<const __nv_bfloat16*>(a.W),
@@ -273,16 +318,10 @@ int launch_lora_down(const void* x, int64_t M, int64_t K, const void* A, int64_t
 
 int launch_dual_lora_gemv(const GemmArgs& a, cudaStream_t stream) {
   const int64_t rows = a.shared_x ? a.M : 2 * a.M;
-  if (rows <= 1)
+  if (rows <= 8)
     launch_gemv_t<1>(a, stream);
-  else if (rows <= 2)
-    launch_gemv_t<2>(a, stream);
-  else if (rows <= 4)
-    launch_gemv_t<4>(a, stream);
-  else if (rows <= 8)
-    launch_gemv_t<8>(a, stream);
   else
-    launch_gemv_t<16>(a, stream);
+    launch_gemv_t<2>(a, stream);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
 }
 

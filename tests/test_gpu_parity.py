@@ -36,7 +36,8 @@ def sample_rows(seed, M, n=64):
 
 
 @pytest.mark.parametrize("S,L,seed", [(4, 64, 1), (4, 512, 4), (64, 512, 5), (3, 37, 7),
-                                      (5, 1000, 8), (2, 1, 9), (7, 33, 10)])
+                                      (5, 1000, 8), (2, 1, 9), (7, 33, 10), (9, 128, 11),
+                                      (5, 384, 12), (3, 256, 13)])
 def test_gae_parity(S, L, seed):
     r = synth.normal_f32(synth.tensor_seed(seed, 1), (S, L))
     v = synth.normal_f32(synth.tensor_seed(seed, 2), (S, L))
