@@ -113,7 +113,7 @@ hydra_status hydra_lora_linear(const void* x_off, const void* x_on, int64_t M, i
  *     y_off = x_off W^T,   y_on = x_on W^T + u B^T
  *   u : bf16 [M, r] = s (x_on A^T) as written by hydra_lora_down; B : bf16 [N, r].
  *   r == 0 (u, B ignored) means no LoRA. algo: 0 automatic, 1 tcgen05 tile kernel,
- *   2 GEMV (at most 16 token rows over both streams).
+ *   2 GEMV (at most 16 token rows over both streams), 3 tcgen05 single-CTA tiles.
  * Same layout, alignment and error rules as hydra_lora_linear; no workspace.
  */
 hydra_status hydra_dual_linear(const void* x_off, const void* x_on, int64_t M, int64_t K,
@@ -148,9 +148,10 @@ hydra_status hydra_dual_linear_ex(const void* x_off, const void* x_on, int64_t M
 
 /*
  * hydra_lora_linear with the kernel family chosen by the caller:
- *   algo 0 = automatic (as hydra_lora_linear), 1 = tcgen05 tile kernel (any M),
- *   2 = GEMV kernel (requires at most 16 token rows over both streams).
- * Same arguments, results and errors otherwise; algo outside 0..2 is HYDRA_ERR_RANGE.
+ *   algo 0 = automatic (as hydra_lora_linear), 1 = tcgen05 tile kernel (any M; CTA pairs
+ *   with 256-row tiles when M > 128), 2 = GEMV kernel (requires at most 16 token rows over
+ *   both streams), 3 = tcgen05 tile kernel on single CTAs only (128-row tiles).
+ * Same arguments, results and errors otherwise; algo outside 0..3 is HYDRA_ERR_RANGE.
  */
 hydra_status hydra_lora_linear_algo(const void* x_off, const void* x_on, int64_t M, int64_t K,
                                     int64_t N, const void* W, const void* A, const void* B,

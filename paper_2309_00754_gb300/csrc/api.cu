@@ -47,9 +47,9 @@ hydra_status lora_linear_impl(const void* x_off, const void* x_on, int64_t M, in
                               bool u_given = false, int epi = HYDRA_EPI_STORE) {
   if (x_off == nullptr || W == nullptr) return HYDRA_ERR_NULL;
   if (y_off == nullptr && y_on == nullptr) return HYDRA_ERR_NULL;
-  if (algo < 0 || algo > 2) return HYDRA_ERR_RANGE;
+  if (algo < 0 || algo > 3) return HYDRA_ERR_RANGE;
   if (epi < HYDRA_EPI_STORE || epi > HYDRA_EPI_RESIDUAL) return HYDRA_ERR_RANGE;
-  if (epi != HYDRA_EPI_STORE && algo != 1) return HYDRA_ERR_RANGE;
+  if (epi != HYDRA_EPI_STORE && algo != 1 && algo != 3) return HYDRA_ERR_RANGE;
   if (epi == HYDRA_EPI_SWIGLU && N % 256 != 0) return HYDRA_ERR_SHAPE;
   if (out_dtype != HYDRA_BF16 && out_dtype != HYDRA_F32) return HYDRA_ERR_RANGE;
   if (M < 0 || K < 8 || N < 8 || M >= (1LL << 31) || K >= (1LL << 31) || N >= (1LL << 31))
@@ -96,6 +96,7 @@ hydra_status lora_linear_impl(const void* x_off, const void* x_on, int64_t M, in
   g.out_f32 = out_dtype == HYDRA_F32 ? 1 : 0;
   g.err = err;
   g.epi = epi;
+  g.single_cta = algo == 3;
   const bool use_gemv = (algo == 2) || (algo == 0 && rows <= hydra::kGemvMaxRows);
   const int rc = use_gemv ? hydra::launch_dual_lora_gemv(g, st) : hydra::launch_dual_lora_gemm_tc(g, st);
   return rc == 0 ? HYDRA_OK : HYDRA_ERR_CUDA;

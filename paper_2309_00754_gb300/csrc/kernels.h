@@ -24,6 +24,7 @@ struct GemmArgs {
   int out_f32;
   int* err;
   int epi = 0;        // tcgen05 kernel epilogue: 0 store, 1 SwiGLU, 2 residual add (fp32)
+  bool single_cta = false;  // tcgen05: never use the CTA-pair (cta_group::2) kernel
 };
 
 // Device address of the library's error word on the current device (NULL on failure).

@@ -409,6 +409,330 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   }
 }
 
+
+// ============================================================================================
+// Two-CTA variant (tcgen05 cta_group::2): a cluster of two CTAs on two SMs computes a
+// 256 x 256 tile with one M = 256 MMA stream issued by the leader CTA (cluster rank 0).
+// Each CTA holds its 128 rows of A and 128 of the 256 rows of B, so a pair moves half the
+// B bytes of two independent 128 x 256 tiles, and a 32 KiB stage allows a 6-deep ring per
+// SM. Each CTA's TMEM holds the accumulator rows of its own 128 output rows; each CTA's
+// epilogue drains them. Protocol: both CTAs' TMA loads complete on the leader's full
+// barrier (the leader posts the byte count of both); the leader's MMA commits arrive on
+// the empty / accumulator barriers of both CTAs (multicast); both CTAs' epilogue warps
+// arrive on the leader's accumulator-drained barriers.
+constexpr int STAGES2 = 6;
+constexpr int B_HALF = 128 * BK * 2;             // 16 KiB: this CTA's 128 rows of B
+constexpr int STAGE2_BYTES = A_TILE + B_HALF;     // 32 KiB
+constexpr int SMEM2_BYTES =
+    1024 + STAGES2 * STAGE2_BYTES + EPI_WARPS * 2 * STAGING_BYTES + (2 * STAGES2 + 7) * 8 + 16;
+constexpr uint32_t IDESC2 = idesc_bf16_f32(256, BN);
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// arrive on an mbarrier of a CTA of the cluster (shared::cluster address)
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_bar) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_bar)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ bool mbar_wait_cluster_bounded(uint32_t bar, uint32_t parity,
+                                                          volatile int* abort, int* err, int code) {
+  if (mbar_try_wait_cluster(bar, parity)) return true;
+  const long long t0 = clock64();
+  for (uint32_t i = 1;; ++i) {
+    if (mbar_try_wait_cluster(bar, parity)) return true;
+    if ((i & 255u) == 0u) {
+      if (*abort) return false;
+      if (clock64() - t0 > kWaitBudgetCycles) {
+        *abort = 1;
+        record_error(err, code);
+        return false;
+      }
+    }
+  }
+}
+// TMA load into this CTA's shared memory, completing on an mbarrier of either CTA of the pair
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map, int x, int y,
+                                                 uint32_t cluster_bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cta.global.tile.mbarrier::complete_tx::bytes.cta_group::2"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(cluster_bar)
+      : "memory");
+}
+__device__ __forceinline__ void tc_mma2_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                             uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// arrive on the barrier at this shared address in both CTAs once all prior MMAs are done
+__device__ __forceinline__ void tc_commit_pair(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(bar),
+      "h"(static_cast<uint16_t>(3))
+      : "memory");
+}
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
+    dual_lora_gemm_2cta_kernel(const __grid_constant__ CUtensorMap tm_x_off,
+                               const __grid_constant__ CUtensorMap tm_x_on,
+                               const __grid_constant__ CUtensorMap tm_w,
+                               const __grid_constant__ CUtensorMap tm_u,
+                               const __grid_constant__ CUtensorMap tm_b,
+                               const __grid_constant__ CUtensorMap tm_y_off,
+                               const __grid_constant__ CUtensorMap tm_y_on, const Params p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* staging_base = smem + STAGES2 * STAGE2_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(staging_base + EPI_WARPS * 2 * STAGING_BYTES);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES2 + 7);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_rank();
+  const bool leader = rank == 0;
+  const int cluster = static_cast<int>(blockIdx.x >> 1);
+  const int nclusters = static_cast<int>(gridDim.x >> 1);
+  const int n_local = (p.total_tiles - cluster + nclusters - 1) / nclusters;
+  const int defer_at = min(DEFER, p.kb_main) - 1;
+
+  const uint32_t smem_base = smem_u32(smem);
+  auto full_bar = [&](int s) { return smem_u32(&bars[s]); };
+  auto empty_bar = [&](int s) { return smem_u32(&bars[STAGES2 + s]); };
+  auto acc_full = [&](int b) { return smem_u32(&bars[2 * STAGES2 + b]); };
+  auto acc_mid = [&](int b) { return smem_u32(&bars[2 * STAGES2 + 2 + b]); };
+  auto acc_empty = [&](int b) { return smem_u32(&bars[2 * STAGES2 + 4 + b]); };
+  const uint32_t mma_done = smem_u32(&bars[2 * STAGES2 + 6]);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES2; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(acc_full(b), 1);
+      mbar_init(acc_mid(b), 2 * EPI_WARPS);
+      mbar_init(acc_empty(b), 2 * EPI_WARPS);
+    }
+    mbar_init(mma_done, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(tmem_slot)),
+                 "r"(TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // barriers of both CTAs are initialised before any remote signal
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  // tile -> (stream, 256-row block, column block); this CTA's rows are m0 + 128 rank
+  auto decode2 = [&](int t) {
+    Tile tl;
+    tl.stream = t % p.streams;
+    t /= p.streams;
+    tl.m0 = (t % p.m_tiles) * 256 + static_cast<int>(rank) * 128;
+    tl.n0 = (t / p.m_tiles) * BN;
+    const bool on = p.shared_x ? true : (tl.stream == 1);
+    tl.n_lora = (p.kb_lora > 0 && on && p.has_on) ? p.kb_lora : 0;
+    return tl;
+  };
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ TMA producer (both CTAs)
+      int it = 0;
+      bool ok = true;
+      const uint32_t leader_full0 = map_to_rank(full_bar(0), 0);
+      auto load = [&](const CUtensorMap* ma, int xa, int ya, const CUtensorMap* mb, int xb,
+                      int yb) {
+        const int s = it % STAGES2;
+        const uint32_t ph = (it / STAGES2) & 1;
+        if (!mbar_wait_bounded(empty_bar(s), ph ^ 1, abort_flag, p.err, kDevTimeoutProducer)) {
+          ok = false;
+          return;
+        }
+        if (leader) mbar_arrive_expect_tx(full_bar(s), 2 * STAGE2_BYTES);
+        const uint32_t bar = leader_full0 + s * 8;
+        const uint32_t a_dst = smem_base + s * STAGE2_BYTES;
+        tma_load_2d_pair(a_dst, ma, xa, ya, bar);
+        tma_load_2d_pair(a_dst + A_TILE, mb, xb, yb, bar);
+        ++it;
+      };
+      const int brow = static_cast<int>(rank) * 128;  // this CTA's half of the B rows
+      Tile prev{0, 0, 0, 0};
+      for (int j = 0; j < n_local && ok; ++j) {
+        const Tile tl = decode2(cluster + j * nclusters);
+        const CUtensorMap* tmx = (tl.stream == 1) ? &tm_x_on : &tm_x_off;
+        for (int kb = 0; kb < p.kb_main && ok; ++kb) {
+          load(tmx, kb * BK, tl.m0, &tm_w, kb * BK, tl.n0 + brow);
+          if (p.deferred && j > 0 && kb == defer_at)
+            for (int kl = 0; kl < prev.n_lora && ok; ++kl)
+              load(&tm_u, kl * BK, prev.m0, &tm_b, kl * BK, prev.n0 + brow);
+        }
+        if (!p.deferred)
+          for (int kl = 0; kl < tl.n_lora && ok; ++kl)
+            load(&tm_u, kl * BK, tl.m0, &tm_b, kl * BK, tl.n0 + brow);
+        prev = tl;
+      }
+      if (p.deferred && n_local > 0)
+        for (int kl = 0; kl < prev.n_lora && ok; ++kl)
+          load(&tm_u, kl * BK, prev.m0, &tm_b, kl * BK, prev.n0 + brow);
+      // this CTA's copies in flight must land before its shared memory is released: the
+      // stage's empty barrier (committed after the MMAs that read it) covers them
+      for (int k = (it > STAGES2 ? it - STAGES2 : 0); k < it; ++k) {
+        volatile int no_abort = 0;
+        mbar_wait_bounded(empty_bar(k % STAGES2), (k / STAGES2) & 1, &no_abort, p.err,
+                          kDevTimeoutDrain);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0 && leader) {
+      // ------------------------------------------------------------ MMA issuer (leader only)
+      int it = 0;
+      bool ok = true;
+      auto consume = [&](uint32_t acc, int nsub, bool first) {
+        const int s = it % STAGES2;
+        const uint32_t ph = (it / STAGES2) & 1;
+        if (!mbar_wait_bounded(full_bar(s), ph, abort_flag, p.err, kDevTimeoutMma)) {
+          ok = false;
+          return;
+        }
+        tc_fence_after();
+        const uint32_t a_base = smem_base + s * STAGE2_BYTES;
+        const uint32_t b_base = a_base + A_TILE;
+        for (int k = 0; k < nsub; ++k)
+          tc_mma2_bf16(acc, smem_desc_sw128(a_base + k * 32), smem_desc_sw128(b_base + k * 32),
+                       IDESC2, (first && k == 0) ? 0u : 1u);
+        tc_commit_pair(empty_bar(s));
+        ++it;
+      };
+      auto lora_nsub = [&](int kl) { return min(BK / 16, (p.r - kl * BK + 15) / 16); };
+      auto lora_items = [&](int jj, int n_lora, bool wait_mid) {
+        const int b = jj & 1;
+        if (wait_mid) {
+          if (!mbar_wait_cluster_bounded(acc_mid(b), (jj >> 1) & 1, abort_flag, p.err,
+                                         kDevTimeoutMma)) {
+            ok = false;
+            return;
+          }
+          tc_fence_after();
+        }
+        for (int kl = 0; kl < n_lora && ok; ++kl) consume(tmem_base + b * 256, lora_nsub(kl), false);
+        if (ok) tc_commit_pair(acc_full(b));
+      };
+      Tile prev{0, 0, 0, 0};
+      for (int j = 0; j < n_local && ok; ++j) {
+        const Tile tl = decode2(cluster + j * nclusters);
+        const int b = j & 1;
+        if (!mbar_wait_cluster_bounded(acc_empty(b), ((j >> 1) & 1) ^ 1, abort_flag, p.err,
+                                       kDevTimeoutMma))
+          break;
+        tc_fence_after();
+        const uint32_t acc = tmem_base + b * 256;
+        for (int kb = 0; kb < p.kb_main && ok; ++kb) {
+          consume(acc, BK / 16, kb == 0);
+          if (kb == p.kb_main - 1 && ok && (p.deferred || tl.n_lora == 0)) tc_commit_pair(acc_full(b));
+          if (p.deferred && j > 0 && kb == defer_at && ok) lora_items(j - 1, prev.n_lora, true);
+        }
+        if (!p.deferred && tl.n_lora > 0 && ok) lora_items(j, tl.n_lora, false);
+        prev = tl;
+      }
+      if (p.deferred && n_local > 0 && ok) lora_items(n_local - 1, prev.n_lora, true);
+      tc_commit_pair(mma_done);
+      volatile int no_abort = 0;
+      mbar_wait_bounded(mma_done, 0, &no_abort, p.err, kDevTimeoutDrain);
+    }
+    __syncwarp();
+  } else {
+    // -------------------------------------------------------------- epilogue (both CTAs)
+    const int q = warp & 3;
+    const uint32_t staging = smem_u32(staging_base) + (warp - 2) * 2 * STAGING_BYTES;
+    uint32_t chunk_ctr = 0;
+    const CUtensorMap* y_off = p.has_off ? &tm_y_off : nullptr;
+    const CUtensorMap* y_on = p.has_on ? &tm_y_on : nullptr;
+    const uint32_t leader_mid0 = map_to_rank(acc_mid(0), 0);
+    const uint32_t leader_empty0 = map_to_rank(acc_empty(0), 0);
+    auto signal = [&](uint32_t leader_bar0, int b) {
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(leader_bar0 + b * 8);
+    };
+    for (int j = 0; j < n_local; ++j) {
+      const Tile tl = decode2(cluster + j * nclusters);
+      const int b = j & 1;
+      const uint32_t acc = tmem_base + b * 256;
+      if (p.deferred) {
+        if (!mbar_wait_bounded(acc_full(b), 0, abort_flag, p.err, kDevTimeoutEpilogue)) break;
+        tc_fence_after();
+        drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, y_off, nullptr);
+        tc_fence_before();
+        signal(leader_mid0, b);
+        if (!mbar_wait_bounded(acc_full(b), 1, abort_flag, p.err, kDevTimeoutEpilogue)) break;
+        tc_fence_after();
+        drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, y_on, nullptr);
+      } else {
+        if (!mbar_wait_bounded(acc_full(b), (j >> 1) & 1, abort_flag, p.err, kDevTimeoutEpilogue))
+          break;
+        tc_fence_after();
+        if (p.shared_x)
+          drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, tl.n_lora > 0 ? nullptr : y_off, y_on);
+        else
+          drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, tl.stream == 1 ? y_on : y_off,
+                nullptr);
+      }
+      tc_fence_before();
+      signal(leader_empty0, b);
+    }
+    if (lane == 0) bulk_wait_all();
+    __syncwarp();
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // no CTA leaves while its peer may still touch its barriers or smem
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
+                 "r"(TMEM_COLS)
+                 : "memory");
+  }
+}
+
 }  // namespace tcgemm
 
 // ------------------------------------------------------------------ host side
@@ -468,19 +792,25 @@ int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream) {
     if (cudaFuncSetAttribute(dual_lora_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              SMEM_BYTES) != cudaSuccess)
       return -1;
+    if (cudaFuncSetAttribute(dual_lora_gemm_2cta_kernel,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM2_BYTES) != cudaSuccess)
+      return -1;
     attr_set = true;
   }
   const int nsm = sm_count();
   if (nsm <= 0) return -1;
+  // 256-row CTA pairs once every stream has more than one 128-row tile of work
+  const bool pair = a.M > BM && nsm >= 2 && !a.single_cta;
   CUtensorMap m_xoff, m_xon, m_w, m_u, m_b, m_yoff, m_yon;
   const bool lora = a.r > 0;
   const bool f32 = a.out_f32 != 0;
   if (!make_map(&m_xoff, a.x_off, a.M, a.K, BM, false)) return -2;
   if (!make_map(&m_xon, a.shared_x ? a.x_off : a.x_on, a.M, a.K, BM, false)) return -2;
-  if (!make_map(&m_w, a.W, a.N, a.K, BN, false)) return -2;
+  const int brows = pair ? 128 : BN;  // a CTA of a pair loads half of the tile's W rows
+  if (!make_map(&m_w, a.W, a.N, a.K, brows, false)) return -2;
   if (lora) {
     if (!make_map(&m_u, a.u, a.M, a.r, BM, false)) return -2;
-    if (!make_map(&m_b, a.B, a.N, a.r, BN, false)) return -2;
+    if (!make_map(&m_b, a.B, a.N, a.r, brows, false)) return -2;
   } else {
     m_u = m_xoff;
     m_b = m_w;
@@ -505,11 +835,19 @@ int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream) {
   p.has_on = a.y_on != nullptr;
   p.deferred = (p.shared_x && lora && p.has_off && p.has_on) ? 1 : 0;
   p.streams = a.shared_x ? 1 : 2;
-  p.m_tiles = static_cast<int>((a.M + BM - 1) / BM);
+  p.m_tiles = static_cast<int>(pair ? (a.M + 255) / 256 : (a.M + BM - 1) / BM);
   p.n_tiles = static_cast<int>((a.N + BN - 1) / BN);
   p.total_tiles = p.m_tiles * p.n_tiles * p.streams;
   p.out_f32 = a.out_f32;
   p.err = a.err;
+  if (pair) {
+    const int nclusters = nsm / 2;
+    const unsigned grid =
+        2u * static_cast<unsigned>(p.total_tiles < nclusters ? p.total_tiles : nclusters);
+    dual_lora_gemm_2cta_kernel<<<grid, NUM_THREADS, SMEM2_BYTES, stream>>>(
+        m_xoff, m_xon, m_w, m_u, m_b, m_yoff, m_yon, p);
+    return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
+  }
   const unsigned grid = static_cast<unsigned>(p.total_tiles < nsm ? p.total_tiles : nsm);
   dual_lora_gemm_kernel<<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(m_xoff, m_xon, m_w, m_u, m_b,
                                                                    m_yoff, m_yon, p);

@@ -64,7 +64,7 @@ def test_lora_linear_argument_errors(lib):
     assert _lin(lib, r=16, A=FAKE, B=FAKE, y_on=FAKE, ws=FAKE, wsb=100) == 7
     assert _lin(lib, x_off=FAKE + 8) == 3                       # misaligned pointer
     assert _lin(lib, dt=7) == 4
-    assert _lin(lib, algo=3) == 4
+    assert _lin(lib, algo=4) == 4
     assert _lin(lib, algo=2, M=9, x_on=FAKE * 2) == 2           # GEMV takes <= 16 rows
     assert _lin(lib, M=0) == 0                                  # empty: no launch
 

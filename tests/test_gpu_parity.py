@@ -158,14 +158,21 @@ def _run_linear(x_off, x_on, W, A, Bm, s, out=torch.bfloat16, algo=0, want=(True
 
 
 @pytest.mark.parametrize("M,K,N,r,shared,algo", [
-    (256, 512, 512, 8, True, 1),      # config-1 first linear
+    (256, 512, 512, 8, True, 1),      # config-1 first linear (CTA pairs)
+    (256, 512, 512, 8, True, 3),      # same on single CTAs
     (300, 328, 520, 16, True, 1),     # ragged M, K (OOB k-block), N tail
+    (300, 328, 520, 16, True, 3),
     (300, 328, 520, 16, False, 1),    # stacked streams
+    (300, 328, 520, 16, False, 3),
     (129, 64, 256, 64, True, 1),
     (130, 1024, 768, 72, False, 1),   # two LoRA k-blocks
+    (130, 1024, 768, 72, False, 3),
     (200, 512, 264, 128, True, 1),
+    (700, 1024, 1280, 16, True, 1),   # several tiles per CTA pair (persistent loop)
+    (700, 1024, 1280, 16, False, 1),
     (64, 256, 512, 0, True, 1),       # no LoRA
     (96, 256, 512, 0, False, 1),
+    (400, 256, 512, 0, False, 1),
     (1, 4096, 4096, 16, True, 2),     # decode GEMV shapes
     (4, 4096, 1032, 16, True, 2),
     (8, 1024, 520, 8, False, 2),
