@@ -421,6 +421,7 @@ class KernelSweep:
     Kernels are replayed back to back from CUDA graphs, weights rotated through copies
     larger than L2.
       GAE: 65536 sequences x 512 tokens -> GB/s;
+      causal attention: 8 sequences x 768 tokens x 32 heads of 128 -> TFLOP/s;
       log-probs/KL: 2048 rows x 32000 fp32 logits x 2 heads -> GB/s."""
 
     name = "kernel_sweep"
@@ -460,7 +461,7 @@ class KernelSweep:
             torch.cuda.synchronize()
             return e0.elapsed_time(e1) / n
 
-        out = {"projection_sweep": {}, "decode": {}, "gae": {}, "logprobs": {}}
+        out = {"projection_sweep": {}, "decode": {}, "gae": {}, "logprobs": {}, "attention": {}}
         # ---- projection sweep (c2): W rotates through 3 copies per shape so consecutive
         # launches do not find W in L2
         M = 2048
@@ -513,6 +514,15 @@ class KernelSweep:
         byts = valid * 8 + S * L * 8 + S * 4  # read valid r, V; write all A, R
         out["gae"] = {"ms": ms, "GB/s": byts / ms / 1e6, "frac_of_measured_hbm": byts / ms / 1e6 / peaks["hbm_gbs"]}
         del rw, vv, adv, ret
+        # ---- causal attention at the full pass's shape: 2 streams x 4 sequences x 768 tokens,
+        # 32 heads of 128
+        nseq, Pq, Hh = 8, 768, 32
+        qkv = torch.randn(nseq * Pq, 3 * Hh * 128, device=dev, generator=g).to(bf)
+        att = torch.empty(nseq * Pq, Hh * 128, dtype=bf, device=dev)
+        ms = graph_ms(lambda i: H.hydra_causal_attention(qkv, nseq, Pq, Hh, 128, att), reps)
+        fl = 4.0 * nseq * Hh * 128 * (Pq * (Pq + 1) / 2)  # q k^T and p v over the causal half
+        out["attention"] = {"ms": ms, "TFLOP/s": fl / ms / 1e9}
+        del qkv, att
         # ---- log-probs/KL at 2048 x 32000 x 2 heads, all rows valid
         T, V = 2048, 32000
         za = torch.randn(T, V, device=dev, generator=g)

@@ -17,13 +17,15 @@ namespace {
 //
 // u[M, r] = bf16(s * x A^T) as a skinny matrix product on the tensor cores (mma.sync
 // m16n8k16, bf16 in, fp32 accumulate): one CTA per 16 token rows and per 64 ranks; its 8
-// warps split K, load their fragments straight from global memory (each 32-byte row
-// segment is read whole by four lanes) and reduce the 8 partial tiles in shared memory.
+// warps split K and reduce their partial tiles in shared memory. The contraction over k
+// is order-free, so inside each 32-wide chunk of k both operands use the same
+// permutation of k: the fragment slots a lane feeds in the chunk's two k-steps are its
+// 8 consecutive elements [8c, 8c + 8), which arrive with one 16-byte load per row.
 
 constexpr int kDownWarps = 8;
 
-__device__ __forceinline__ uint32_t ld_pair(const __nv_bfloat16* p, bool ok) {
-  return ok ? __ldg(reinterpret_cast<const uint32_t*>(p)) : 0u;
+__device__ __forceinline__ uint4 ld16(const __nv_bfloat16* p, bool ok) {
+  return ok ? __ldg(reinterpret_cast<const uint4*>(p)) : make_uint4(0u, 0u, 0u, 0u);
 }
 
 __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
@@ -46,42 +48,42 @@ __global__ void __launch_bounds__(32 * kDownWarps)
   const int g = lane >> 2, c = lane & 3;
   const int row0 = blockIdx.x * 16;
   const int n_base = blockIdx.y * NT * 8;
-  // this warp's K range, in whole k-steps of 16
-  const int ksteps = (K + 15) / 16;
-  const int per = (ksteps + kDownWarps - 1) / kDownWarps;
-  const int ks0 = warp * per;
-  const int ks1 = min(ksteps, ks0 + per);
+  // this warp's K range, in chunks of 32
+  const int nchunk = (K + 31) / 32;
+  const int per = (nchunk + kDownWarps - 1) / kDownWarps;
+  const int ch0 = warp * per;
+  const int ch1 = min(nchunk, ch0 + per);
 
   const bool r_lo = row0 + g < M, r_hi = row0 + g + 8 < M;
-  const __nv_bfloat16* x_lo = x + static_cast<size_t>(r_lo ? row0 + g : 0) * K;
-  const __nv_bfloat16* x_hi = x + static_cast<size_t>(r_hi ? row0 + g + 8 : 0) * K;
+  const __nv_bfloat16* x_lo = x + static_cast<size_t>(r_lo ? row0 + g : 0) * K + 8 * c;
+  const __nv_bfloat16* x_hi = x + static_cast<size_t>(r_hi ? row0 + g + 8 : 0) * K + 8 * c;
   const __nv_bfloat16* a_row[NT];
   bool a_ok[NT];
 #pragma unroll
   for (int t = 0; t < NT; ++t) {
     const int n = n_base + t * 8 + g;
     a_ok[t] = n < r;
-    a_row[t] = A + static_cast<size_t>(a_ok[t] ? n : 0) * K;
+    a_row[t] = A + static_cast<size_t>(a_ok[t] ? n : 0) * K + 8 * c;
   }
   float d[NT][4];
 #pragma unroll
   for (int t = 0; t < NT; ++t) d[t][0] = d[t][1] = d[t][2] = d[t][3] = 0.f;
 
 #pragma unroll 4
-  for (int ks = ks0; ks < ks1; ++ks) {
-    const int k0 = ks * 16 + 2 * c;
-    const int k1 = k0 + 8;
-    const bool v0 = k0 < K, v1 = k1 < K;
-    uint32_t a[4];
-    a[0] = ld_pair(x_lo + k0, r_lo && v0);
-    a[1] = ld_pair(x_hi + k0, r_hi && v0);
-    a[2] = ld_pair(x_lo + k1, r_lo && v1);
-    a[3] = ld_pair(x_hi + k1, r_hi && v1);
+  for (int ch = ch0; ch < ch1; ++ch) {
+    const int k = ch * 32;
+    const bool kv = k + 8 * c < K;  // K % 8 == 0: a lane's 8 elements are all in or all out
+    const uint4 xl = ld16(x_lo + k, r_lo && kv);
+    const uint4 xh = ld16(x_hi + k, r_hi && kv);
+    uint4 bv[NT];
+#pragma unroll
+    for (int t = 0; t < NT; ++t) bv[t] = ld16(a_row[t] + k, a_ok[t] && kv);
+    const uint32_t a0[4] = {xl.x, xh.x, xl.y, xh.y};  // k-step 0: elements 8c .. 8c + 3
+    const uint32_t a1[4] = {xl.z, xh.z, xl.w, xh.w};  // k-step 1: elements 8c + 4 .. 8c + 7
 #pragma unroll
     for (int t = 0; t < NT; ++t) {
-      const uint32_t b0 = ld_pair(a_row[t] + k0, a_ok[t] && v0);
-      const uint32_t b1 = ld_pair(a_row[t] + k1, a_ok[t] && v1);
-      mma_bf16_16816(d[t], a, b0, b1);
+      mma_bf16_16816(d[t], a0, bv[t].x, bv[t].y);
+      mma_bf16_16816(d[t], a1, bv[t].z, bv[t].w);
     }
   }
 #pragma unroll
@@ -107,14 +109,20 @@ __global__ void __launch_bounds__(32 * kDownWarps)
 // Decode-shaped dual-output linear (at most 16 token rows over both streams). HBM-bound:
 // every byte of W is read once. One CTA per 16 rows of W; its 8 warps split K and stream
 // their [16 x 64] W and token-row slices into XOR-swizzled shared memory with cp.async
-// (3 stages per warp, 16-byte copies), then run mma.sync m16n8k16 with W as the 16-row
+// (3-4 stages per warp, 16-byte copies), then run mma.sync m16n8k16 with W as the 16-row
 // operand and the token rows as the 8-wide operand (both through ldmatrix), so the
 // arithmetic never limits the stream even at 16 rows. The 8 partial tiles are reduced in
 // shared memory, where each thread also adds the rank-r LoRA term of its (row, token).
 
 constexpr int kGvWarps = 8;
-constexpr int kGvStages = 3;
-constexpr int kGvStageBytes = 2 * 16 * 128;  // 16 W rows + 16 token rows, 64 bf16 each
+// per-warp ring: stage = 16 W rows + 8 NT token rows of 64 bf16; 4 stages for <= 8 token
+// rows, 3 for 16 (so that two CTAs fit an SM)
+template <int NT>
+struct Gv {
+  static constexpr int kStages = NT == 1 ? 4 : 3;
+  static constexpr int kStageBytes = (16 + 8 * NT) * 128;
+  static constexpr int kSmem = kGvWarps * kStages * kStageBytes + kGvWarps * 16 * 16 * 4;
+};
 
 __device__ __forceinline__ void gv_cp_async16(uint32_t dst, const void* src, bool ok) {
   const int n = ok ? 16 : 0;
@@ -140,6 +148,8 @@ __global__ void __launch_bounds__(32 * kGvWarps)
                           const __nv_bfloat16* __restrict__ B, int r, void* y_off, void* y_on,
                           int out_f32, int shared_x) {
   extern __shared__ __align__(1024) uint8_t smem[];
+  constexpr int kGvStages = Gv<NT>::kStages;
+  constexpr int kGvStageBytes = Gv<NT>::kStageBytes;
   float* red = reinterpret_cast<float*>(smem + kGvWarps * kGvStages * kGvStageBytes);
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -212,7 +222,14 @@ __global__ void __launch_bounds__(32 * kGvWarps)
       {
         const int trow = (lane & 7) + ((lane >> 4) << 3);
         const int seg = 2 * kk + ((lane >> 3) & 1);
-        gv_ldsm_x4(st + 16 * 128 + trow * 128 + ((seg ^ (trow & 7)) << 4), b);
+        const uint32_t addr = st + 16 * 128 + trow * 128 + ((seg ^ (trow & 7)) << 4);
+        if (NT == 2) {
+          gv_ldsm_x4(addr, b);
+        } else {  // token rows 0..7 only: two matrices, addresses from lanes 0-15
+          asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0,%1}, [%2];"
+                       : "=r"(b[0]), "=r"(b[1])
+                       : "r"(addr));
+        }
       }
 #pragma unroll
       for (int t = 0; t < NT; ++t) mma_bf16_16816(d[t], a, b[2 * t], b[2 * t + 1]);
@@ -278,7 +295,7 @@ __global__ void __launch_bounds__(32 * kGvWarps)
 
 template <int NT>
 void launch_gemv_t(const GemmArgs& a, cudaStream_t stream) {
-  constexpr int smem = kGvWarps * kGvStages * kGvStageBytes + kGvWarps * 16 * 16 * 4;
+  constexpr int smem = Gv<NT>::kSmem;
   static bool attr = false;
   if (!attr) {
     cudaFuncSetAttribute(dual_lora_gemv_kernel<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
