@@ -96,6 +96,25 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,
   }
 }
 
+// mbar_wait_bounded run by every lane of a warp; the result is warp-uniform (false if any
+// lane gave up). Roles that issue async work loop as whole warps and let one elected lane
+// issue: a loop run by a single lane of a diverged warp feeds the tensor pipe more slowly.
+__device__ __forceinline__ bool warp_wait_bounded(uint32_t bar, uint32_t parity,
+                                                  volatile int* abort, int* err, int code) {
+  return __all_sync(0xffffffffu, mbar_wait_bounded(bar, parity, abort, err, code));
+}
+
+// One lane of a converged warp (the lowest) returns true.
+__device__ __forceinline__ bool elect_one() {
+  uint32_t p;
+  asm volatile(
+      "{\n\t.reg .pred P;\n\t"
+      "elect.sync _|P, 0xffffffff;\n\t"
+      "selp.u32 %0, 1, 0, P;\n\t}"
+      : "=r"(p));
+  return p != 0;
+}
+
 // ---------------------------------------------------------------- TMA (tiled, 2-D)
 
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {

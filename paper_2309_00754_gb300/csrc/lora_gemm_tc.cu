@@ -253,113 +253,119 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const uint32_t tmem_base = *tmem_slot;
 
   if (warp == 0) {
-    if (lane == 0) {
-      // ------------------------------------------------------------ TMA producer
+    // ------------------------------------------------------------ TMA producer (whole warp)
+    if (elect_one()) {
       tma_prefetch_desc(&tm_x_off);
       tma_prefetch_desc(&tm_x_on);
       tma_prefetch_desc(&tm_w);
       tma_prefetch_desc(&tm_u);
       tma_prefetch_desc(&tm_b);
-      int it = 0;
-      bool ok = true;
-      auto load = [&](const CUtensorMap* ma, int xa, int ya, const CUtensorMap* mb, int xb,
-                      int yb) {
-        const int s = it % STAGES;
-        const uint32_t ph = (it / STAGES) & 1;
-        if (!mbar_wait_bounded(empty_bar(s), ph ^ 1, abort_flag, p.err, kDevTimeoutProducer)) {
-          ok = false;
-          return;
-        }
+    }
+    __syncwarp();
+    int it = 0;
+    bool ok = true;
+    auto load = [&](const CUtensorMap* ma, int xa, int ya, const CUtensorMap* mb, int xb, int yb) {
+      const int s = it % STAGES;
+      const uint32_t ph = (it / STAGES) & 1;
+      if (!warp_wait_bounded(empty_bar(s), ph ^ 1, abort_flag, p.err, kDevTimeoutProducer)) {
+        ok = false;
+        return;
+      }
+      if (elect_one()) {
         mbar_arrive_expect_tx(full_bar(s), STAGE_BYTES);
         const uint32_t a_dst = smem_base + s * STAGE_BYTES;
         tma_load_2d(a_dst, ma, xa, ya, full_bar(s));
         tma_load_2d(a_dst + A_TILE, mb, xb, yb, full_bar(s));
-        ++it;
-      };
-      Tile prev{0, 0, 0, 0};
-      for (int j = 0; j < n_local && ok; ++j) {
-        const Tile tl = decode(p, blockIdx.x + j * gridDim.x);
-        const CUtensorMap* tmx = (tl.stream == 1) ? &tm_x_on : &tm_x_off;
-        for (int kb = 0; kb < p.kb_main && ok; ++kb) {
-          load(tmx, kb * BK, tl.m0, &tm_w, kb * BK, tl.n0);
-          if (p.deferred && j > 0 && kb == defer_at)
-            for (int kl = 0; kl < prev.n_lora && ok; ++kl)
-              load(&tm_u, kl * BK, prev.m0, &tm_b, kl * BK, prev.n0);
-        }
-        if (!p.deferred)
-          for (int kl = 0; kl < tl.n_lora && ok; ++kl)
-            load(&tm_u, kl * BK, tl.m0, &tm_b, kl * BK, tl.n0);
-        prev = tl;
       }
-      if (p.deferred && n_local > 0)
-        for (int kl = 0; kl < prev.n_lora && ok; ++kl)
-          load(&tm_u, kl * BK, prev.m0, &tm_b, kl * BK, prev.n0);
-      // copies still in flight must land before the CTA's shared memory is released
-      for (int k = (it > STAGES ? it - STAGES : 0); k < it; ++k) {
-        volatile int no_abort = 0;
-        mbar_wait_bounded(full_bar(k % STAGES), (k / STAGES) & 1, &no_abort, p.err,
-                          kDevTimeoutDrain);
+      __syncwarp();
+      ++it;
+    };
+    Tile prev{0, 0, 0, 0};
+    for (int j = 0; j < n_local && ok; ++j) {
+      const Tile tl = decode(p, blockIdx.x + j * gridDim.x);
+      const CUtensorMap* tmx = (tl.stream == 1) ? &tm_x_on : &tm_x_off;
+      for (int kb = 0; kb < p.kb_main && ok; ++kb) {
+        load(tmx, kb * BK, tl.m0, &tm_w, kb * BK, tl.n0);
+        if (p.deferred && j > 0 && kb == defer_at)
+          for (int kl = 0; kl < prev.n_lora && ok; ++kl)
+            load(&tm_u, kl * BK, prev.m0, &tm_b, kl * BK, prev.n0);
       }
+      if (!p.deferred)
+        for (int kl = 0; kl < tl.n_lora && ok; ++kl)
+          load(&tm_u, kl * BK, tl.m0, &tm_b, kl * BK, tl.n0);
+      prev = tl;
     }
-    __syncwarp();
+    if (p.deferred && n_local > 0)
+      for (int kl = 0; kl < prev.n_lora && ok; ++kl)
+        load(&tm_u, kl * BK, prev.m0, &tm_b, kl * BK, prev.n0);
+    // copies still in flight must land before the CTA's shared memory is released
+    for (int k = (it > STAGES ? it - STAGES : 0); k < it; ++k) {
+      volatile int no_abort = 0;
+      warp_wait_bounded(full_bar(k % STAGES), (k / STAGES) & 1, &no_abort, p.err, kDevTimeoutDrain);
+    }
   } else if (warp == 1) {
-    if (lane == 0) {
-      // ------------------------------------------------------------ MMA issuer
-      int it = 0;
-      bool ok = true;
-      // one ring item: nsub MMAs of K = 16 into the accumulator at `acc`
-      auto consume = [&](uint32_t acc, int nsub, bool first) {
-        const int s = it % STAGES;
-        const uint32_t ph = (it / STAGES) & 1;
-        if (!mbar_wait_bounded(full_bar(s), ph, abort_flag, p.err, kDevTimeoutMma)) {
-          ok = false;
-          return;
-        }
-        tc_fence_after();
+    // ------------------------------------------------------------ MMA issuer (whole warp,
+    // one elected lane issues; the same lane issues every MMA and commit, so each commit
+    // covers all MMAs before it)
+    int it = 0;
+    bool ok = true;
+    // one ring item: nsub MMAs of K = 16 into the accumulator at `acc`; `then` (if non-zero)
+    // is an extra barrier to arrive on once these MMAs are done
+    auto consume = [&](uint32_t acc, int nsub, bool first, uint32_t then) {
+      const int s = it % STAGES;
+      const uint32_t ph = (it / STAGES) & 1;
+      if (!warp_wait_bounded(full_bar(s), ph, abort_flag, p.err, kDevTimeoutMma)) {
+        ok = false;
+        return;
+      }
+      tc_fence_after();
+      if (elect_one()) {
         const uint32_t a_base = smem_base + s * STAGE_BYTES;
         const uint32_t b_base = a_base + A_TILE;
         for (int k = 0; k < nsub; ++k)
           tc_mma_bf16(acc, smem_desc_sw128(a_base + k * 32), smem_desc_sw128(b_base + k * 32),
                       IDESC, (first && k == 0) ? 0u : 1u);
         tc_commit(empty_bar(s));
-        ++it;
-      };
-      auto lora_nsub = [&](int kl) { return min(BK / 16, (p.r - kl * BK + 15) / 16); };
-      auto lora_items = [&](int jj, int n_lora, bool wait_mid) {
-        const int b = jj & 1;
-        if (wait_mid) {
-          if (!mbar_wait_bounded(acc_mid(b), (jj >> 1) & 1, abort_flag, p.err, kDevTimeoutMma)) {
-            ok = false;
-            return;
-          }
-          tc_fence_after();
-        }
-        for (int kl = 0; kl < n_lora && ok; ++kl) consume(tmem_base + b * 256, lora_nsub(kl), false);
-        if (ok) tc_commit(acc_full(b));
-      };
-      Tile prev{0, 0, 0, 0};
-      for (int j = 0; j < n_local && ok; ++j) {
-        const Tile tl = decode(p, blockIdx.x + j * gridDim.x);
-        const int b = j & 1;
-        if (!mbar_wait_bounded(acc_empty(b), ((j >> 1) & 1) ^ 1, abort_flag, p.err, kDevTimeoutMma))
-          break;
-        tc_fence_after();
-        const uint32_t acc = tmem_base + b * 256;
-        for (int kb = 0; kb < p.kb_main && ok; ++kb) {
-          consume(acc, BK / 16, kb == 0);
-          if (kb == p.kb_main - 1 && ok && (p.deferred || tl.n_lora == 0)) tc_commit(acc_full(b));
-          if (p.deferred && j > 0 && kb == defer_at && ok) lora_items(j - 1, prev.n_lora, true);
-        }
-        if (!p.deferred && tl.n_lora > 0 && ok) lora_items(j, tl.n_lora, false);
-        prev = tl;
+        if (then) tc_commit(then);
       }
-      if (p.deferred && n_local > 0 && ok) lora_items(n_local - 1, prev.n_lora, true);
-      // every issued MMA has finished before TMEM is released
-      tc_commit(mma_done);
-      volatile int no_abort = 0;
-      mbar_wait_bounded(mma_done, 0, &no_abort, p.err, kDevTimeoutDrain);
+      __syncwarp();
+      ++it;
+    };
+    auto lora_nsub = [&](int kl) { return min(BK / 16, (p.r - kl * BK + 15) / 16); };
+    auto lora_items = [&](int jj, int n_lora, bool wait_mid) {
+      const int b = jj & 1;
+      if (wait_mid) {
+        if (!warp_wait_bounded(acc_mid(b), (jj >> 1) & 1, abort_flag, p.err, kDevTimeoutMma)) {
+          ok = false;
+          return;
+        }
+        tc_fence_after();
+      }
+      for (int kl = 0; kl < n_lora && ok; ++kl)
+        consume(tmem_base + b * 256, lora_nsub(kl), false, kl == n_lora - 1 ? acc_full(b) : 0u);
+    };
+    Tile prev{0, 0, 0, 0};
+    for (int j = 0; j < n_local && ok; ++j) {
+      const Tile tl = decode(p, blockIdx.x + j * gridDim.x);
+      const int b = j & 1;
+      if (!warp_wait_bounded(acc_empty(b), ((j >> 1) & 1) ^ 1, abort_flag, p.err, kDevTimeoutMma))
+        break;
+      tc_fence_after();
+      const uint32_t acc = tmem_base + b * 256;
+      for (int kb = 0; kb < p.kb_main && ok; ++kb) {
+        const bool last = kb == p.kb_main - 1 && (p.deferred || tl.n_lora == 0);
+        consume(acc, BK / 16, kb == 0, last ? acc_full(b) : 0u);
+        if (p.deferred && j > 0 && kb == defer_at && ok) lora_items(j - 1, prev.n_lora, true);
+      }
+      if (!p.deferred && tl.n_lora > 0 && ok) lora_items(j, tl.n_lora, false);
+      prev = tl;
     }
+    if (p.deferred && n_local > 0 && ok) lora_items(n_local - 1, prev.n_lora, true);
+    // every issued MMA has finished before TMEM is released
+    if (elect_one()) tc_commit(mma_done);
     __syncwarp();
+    volatile int no_abort = 0;
+    warp_wait_bounded(mma_done, 0, &no_abort, p.err, kDevTimeoutDrain);
   } else {
     // -------------------------------------------------------------- epilogue
     const int q = warp & 3;
@@ -473,6 +479,10 @@ __device__ __forceinline__ bool mbar_wait_cluster_bounded(uint32_t bar, uint32_t
     }
   }
 }
+__device__ __forceinline__ bool warp_wait_cluster_bounded(uint32_t bar, uint32_t parity,
+                                                          volatile int* abort, int* err, int code) {
+  return __all_sync(0xffffffffu, mbar_wait_cluster_bounded(bar, parity, abort, err, code));
+}
 // TMA load into this CTA's shared memory, completing on an mbarrier of either CTA of the pair
 __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map, int x, int y,
                                                  uint32_t cluster_bar) {
@@ -573,112 +583,117 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
   };
 
   if (warp == 0) {
-    if (lane == 0) {
-      // ------------------------------------------------------------ TMA producer (both CTAs)
-      int it = 0;
-      bool ok = true;
-      const uint32_t leader_full0 = map_to_rank(full_bar(0), 0);
-      auto load = [&](const CUtensorMap* ma, int xa, int ya, const CUtensorMap* mb, int xb,
-                      int yb) {
-        const int s = it % STAGES2;
-        const uint32_t ph = (it / STAGES2) & 1;
-        if (!mbar_wait_bounded(empty_bar(s), ph ^ 1, abort_flag, p.err, kDevTimeoutProducer)) {
-          ok = false;
-          return;
-        }
+    // ------------------------------------------------------------ TMA producer (both CTAs;
+    // whole warp, one elected lane issues)
+    int it = 0;
+    bool ok = true;
+    const uint32_t leader_full0 = map_to_rank(full_bar(0), 0);
+    auto load = [&](const CUtensorMap* ma, int xa, int ya, const CUtensorMap* mb, int xb, int yb) {
+      const int s = it % STAGES2;
+      const uint32_t ph = (it / STAGES2) & 1;
+      if (!warp_wait_bounded(empty_bar(s), ph ^ 1, abort_flag, p.err, kDevTimeoutProducer)) {
+        ok = false;
+        return;
+      }
+      if (elect_one()) {
         if (leader) mbar_arrive_expect_tx(full_bar(s), 2 * STAGE2_BYTES);
         const uint32_t bar = leader_full0 + s * 8;
         const uint32_t a_dst = smem_base + s * STAGE2_BYTES;
         tma_load_2d_pair(a_dst, ma, xa, ya, bar);
         tma_load_2d_pair(a_dst + A_TILE, mb, xb, yb, bar);
-        ++it;
-      };
-      const int brow = static_cast<int>(rank) * 128;  // this CTA's half of the B rows
-      Tile prev{0, 0, 0, 0};
-      for (int j = 0; j < n_local && ok; ++j) {
-        const Tile tl = decode2(cluster + j * nclusters);
-        const CUtensorMap* tmx = (tl.stream == 1) ? &tm_x_on : &tm_x_off;
-        for (int kb = 0; kb < p.kb_main && ok; ++kb) {
-          load(tmx, kb * BK, tl.m0, &tm_w, kb * BK, tl.n0 + brow);
-          if (p.deferred && j > 0 && kb == defer_at)
-            for (int kl = 0; kl < prev.n_lora && ok; ++kl)
-              load(&tm_u, kl * BK, prev.m0, &tm_b, kl * BK, prev.n0 + brow);
-        }
-        if (!p.deferred)
-          for (int kl = 0; kl < tl.n_lora && ok; ++kl)
-            load(&tm_u, kl * BK, tl.m0, &tm_b, kl * BK, tl.n0 + brow);
-        prev = tl;
       }
-      if (p.deferred && n_local > 0)
-        for (int kl = 0; kl < prev.n_lora && ok; ++kl)
-          load(&tm_u, kl * BK, prev.m0, &tm_b, kl * BK, prev.n0 + brow);
-      // this CTA's copies in flight must land before its shared memory is released: the
-      // stage's empty barrier (committed after the MMAs that read it) covers them
-      for (int k = (it > STAGES2 ? it - STAGES2 : 0); k < it; ++k) {
-        volatile int no_abort = 0;
-        mbar_wait_bounded(empty_bar(k % STAGES2), (k / STAGES2) & 1, &no_abort, p.err,
-                          kDevTimeoutDrain);
+      __syncwarp();
+      ++it;
+    };
+    const int brow = static_cast<int>(rank) * 128;  // this CTA's half of the B rows
+    Tile prev{0, 0, 0, 0};
+    for (int j = 0; j < n_local && ok; ++j) {
+      const Tile tl = decode2(cluster + j * nclusters);
+      const CUtensorMap* tmx = (tl.stream == 1) ? &tm_x_on : &tm_x_off;
+      for (int kb = 0; kb < p.kb_main && ok; ++kb) {
+        load(tmx, kb * BK, tl.m0, &tm_w, kb * BK, tl.n0 + brow);
+        if (p.deferred && j > 0 && kb == defer_at)
+          for (int kl = 0; kl < prev.n_lora && ok; ++kl)
+            load(&tm_u, kl * BK, prev.m0, &tm_b, kl * BK, prev.n0 + brow);
       }
+      if (!p.deferred)
+        for (int kl = 0; kl < tl.n_lora && ok; ++kl)
+          load(&tm_u, kl * BK, tl.m0, &tm_b, kl * BK, tl.n0 + brow);
+      prev = tl;
     }
-    __syncwarp();
+    if (p.deferred && n_local > 0)
+      for (int kl = 0; kl < prev.n_lora && ok; ++kl)
+        load(&tm_u, kl * BK, prev.m0, &tm_b, kl * BK, prev.n0 + brow);
+    // this CTA's copies in flight must land before its shared memory is released: the
+    // stage's empty barrier (committed after the MMAs that read it) covers them
+    for (int k = (it > STAGES2 ? it - STAGES2 : 0); k < it; ++k) {
+      volatile int no_abort = 0;
+      warp_wait_bounded(empty_bar(k % STAGES2), (k / STAGES2) & 1, &no_abort, p.err,
+                        kDevTimeoutDrain);
+    }
   } else if (warp == 1) {
-    if (lane == 0 && leader) {
-      // ------------------------------------------------------------ MMA issuer (leader only)
+    if (leader) {
+      // ---------------------------------------------------------- MMA issuer (leader CTA;
+      // whole warp, one elected lane issues every MMA and commit)
       int it = 0;
       bool ok = true;
-      auto consume = [&](uint32_t acc, int nsub, bool first) {
+      auto consume = [&](uint32_t acc, int nsub, bool first, uint32_t then) {
         const int s = it % STAGES2;
         const uint32_t ph = (it / STAGES2) & 1;
-        if (!mbar_wait_bounded(full_bar(s), ph, abort_flag, p.err, kDevTimeoutMma)) {
+        if (!warp_wait_bounded(full_bar(s), ph, abort_flag, p.err, kDevTimeoutMma)) {
           ok = false;
           return;
         }
         tc_fence_after();
-        const uint32_t a_base = smem_base + s * STAGE2_BYTES;
-        const uint32_t b_base = a_base + A_TILE;
-        for (int k = 0; k < nsub; ++k)
-          tc_mma2_bf16(acc, smem_desc_sw128(a_base + k * 32), smem_desc_sw128(b_base + k * 32),
-                       IDESC2, (first && k == 0) ? 0u : 1u);
-        tc_commit_pair(empty_bar(s));
+        if (elect_one()) {
+          const uint32_t a_base = smem_base + s * STAGE2_BYTES;
+          const uint32_t b_base = a_base + A_TILE;
+          for (int k = 0; k < nsub; ++k)
+            tc_mma2_bf16(acc, smem_desc_sw128(a_base + k * 32), smem_desc_sw128(b_base + k * 32),
+                         IDESC2, (first && k == 0) ? 0u : 1u);
+          tc_commit_pair(empty_bar(s));
+          if (then) tc_commit_pair(then);
+        }
+        __syncwarp();
         ++it;
       };
       auto lora_nsub = [&](int kl) { return min(BK / 16, (p.r - kl * BK + 15) / 16); };
       auto lora_items = [&](int jj, int n_lora, bool wait_mid) {
         const int b = jj & 1;
         if (wait_mid) {
-          if (!mbar_wait_cluster_bounded(acc_mid(b), (jj >> 1) & 1, abort_flag, p.err,
+          if (!warp_wait_cluster_bounded(acc_mid(b), (jj >> 1) & 1, abort_flag, p.err,
                                          kDevTimeoutMma)) {
             ok = false;
             return;
           }
           tc_fence_after();
         }
-        for (int kl = 0; kl < n_lora && ok; ++kl) consume(tmem_base + b * 256, lora_nsub(kl), false);
-        if (ok) tc_commit_pair(acc_full(b));
+        for (int kl = 0; kl < n_lora && ok; ++kl)
+          consume(tmem_base + b * 256, lora_nsub(kl), false, kl == n_lora - 1 ? acc_full(b) : 0u);
       };
       Tile prev{0, 0, 0, 0};
       for (int j = 0; j < n_local && ok; ++j) {
         const Tile tl = decode2(cluster + j * nclusters);
         const int b = j & 1;
-        if (!mbar_wait_cluster_bounded(acc_empty(b), ((j >> 1) & 1) ^ 1, abort_flag, p.err,
+        if (!warp_wait_cluster_bounded(acc_empty(b), ((j >> 1) & 1) ^ 1, abort_flag, p.err,
                                        kDevTimeoutMma))
           break;
         tc_fence_after();
         const uint32_t acc = tmem_base + b * 256;
         for (int kb = 0; kb < p.kb_main && ok; ++kb) {
-          consume(acc, BK / 16, kb == 0);
-          if (kb == p.kb_main - 1 && ok && (p.deferred || tl.n_lora == 0)) tc_commit_pair(acc_full(b));
+          const bool last = kb == p.kb_main - 1 && (p.deferred || tl.n_lora == 0);
+          consume(acc, BK / 16, kb == 0, last ? acc_full(b) : 0u);
           if (p.deferred && j > 0 && kb == defer_at && ok) lora_items(j - 1, prev.n_lora, true);
         }
         if (!p.deferred && tl.n_lora > 0 && ok) lora_items(j, tl.n_lora, false);
         prev = tl;
       }
       if (p.deferred && n_local > 0 && ok) lora_items(n_local - 1, prev.n_lora, true);
-      tc_commit_pair(mma_done);
+      if (elect_one()) tc_commit_pair(mma_done);
+      __syncwarp();
       volatile int no_abort = 0;
-      mbar_wait_bounded(mma_done, 0, &no_abort, p.err, kDevTimeoutDrain);
+      warp_wait_bounded(mma_done, 0, &no_abort, p.err, kDevTimeoutDrain);
     }
-    __syncwarp();
   } else {
     // -------------------------------------------------------------- epilogue (both CTAs)
     const int q = warp & 3;
