@@ -115,6 +115,25 @@ __device__ __forceinline__ bool elect_one() {
   return p != 0;
 }
 
+// ---------------------------------------------------------------- programmatic dependent launch
+//
+// A kernel launched with the programmatic-stream-serialisation attribute (launch_pdl) may
+// start while the preceding kernel of the stream is still running. pdl_wait() returns once
+// that kernel has completed and its writes are visible; a kernel reads nothing the
+// preceding work may write, and writes nothing, before it. pdl_launch_dependents() lets
+// the next such launch start early. Both are no-ops in a normal launch.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+// Bring [p, p + bytes) into L2 (p and bytes multiples of 16). L2 is the device's point of
+// coherence, so a prefetch issued before pdl_wait() never makes a later read stale.
+__device__ __forceinline__ void prefetch_l2_bulk(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(p)),
+               "r"(bytes)
+               : "memory");
+}
+
 // ---------------------------------------------------------------- TMA (tiled, 2-D)
 
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {

@@ -8,7 +8,28 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include <utility>
+
 namespace hydra {
+
+// Launch with programmatic stream serialisation: the kernel may begin while the preceding
+// kernel of the stream finishes, and must call pdl_wait() (common.cuh) before reading
+// anything that work may write or writing anything.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t stream, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 struct GemmArgs {
   const void* x_off;  // bf16 [M, K]

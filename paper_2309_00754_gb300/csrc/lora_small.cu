@@ -43,6 +43,8 @@ __global__ void __launch_bounds__(32 * kDownWarps)
                      const __nv_bfloat16* __restrict__ A, int r, float s,
                      __nv_bfloat16* __restrict__ u) {
   __shared__ float red[kDownWarps][16][NT * 8 + 1];
+  pdl_launch_dependents();
+  pdl_wait();  // x is written by the preceding kernel
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int g = lane >> 2, c = lane & 3;
@@ -163,6 +165,16 @@ __global__ void __launch_bounds__(32 * kGvWarps)
   const int per = (nchunk + kGvWarps - 1) / kGvWarps;
   const int c0 = warp * per;
   const int c1 = min(nchunk, c0 + per);
+
+  // W is frozen: the first chunks of this warp's [16 x K-range] slice stream into L2 while
+  // the preceding kernel finishes (programmatic dependent launch); x, u and y are touched
+  // only after pdl_wait(). Prefetching the whole slice instead evicts, on the large
+  // shapes, lines the running kernel has yet to read.
+  pdl_launch_dependents();
+  if (c0 < c1 && lane < 16 && n0 + lane < N)
+    prefetch_l2_bulk(W + static_cast<size_t>(n0 + lane) * K + c0 * 64,
+                     static_cast<uint32_t>(min(K, min(c1, c0 + kGvStages) * 64) - c0 * 64) * 2u);
+  pdl_wait();
 
   // token row copied by this lane's slice of the x stage (rows lane >> 3 and 4 + lane >> 3...)
   auto xrow = [&](int tk) {
@@ -302,7 +314,7 @@ void launch_gemv_t(const GemmArgs& a, cudaStream_t stream) {
     attr = true;
   }
   const unsigned grid = static_cast<unsigned>((a.N + 15) / 16);
-  dual_lora_gemv_kernel<NT><<<grid, 32 * kGvWarps, smem, stream>>>(
+  launch_pdl(dual_lora_gemv_kernel<NT>, dim3(grid), dim3(32 * kGvWarps), smem, stream,
       static_cast<const __nv_bfloat16*>(a.x_off),
       static_cast<const __nv_bfloat16*>(a.shared_x ? a.x_off : a.x_on), static_cast<int>(a.M),
       static_cast<int>(a.K), static_cast<int>(a.N), static_cast<const __nv_bfloat16*>(a.W),
@@ -320,16 +332,16 @@ int launch_lora_down(const void* x, int64_t M, int64_t K, const void* A, int64_t
   const auto* ap = static_cast<const __nv_bfloat16*>(A);
   auto* up = static_cast<__nv_bfloat16*>(u);
   const unsigned gx = static_cast<unsigned>((M + 15) / 16);
-  if (r <= 8) {
-    lora_down_kernel<1><<<dim3(gx, 1), block, 0, stream>>>(xp, static_cast<int>(M), static_cast<int>(K), ap, static_cast<int>(r), s, up);
-  } else if (r <= 16) {
-    lora_down_kernel<2><<<dim3(gx, 1), block, 0, stream>>>(xp, static_cast<int>(M), static_cast<int>(K), ap, static_cast<int>(r), s, up);
-  } else if (r <= 32) {
-    lora_down_kernel<4><<<dim3(gx, 1), block, 0, stream>>>(xp, static_cast<int>(M), static_cast<int>(K), ap, static_cast<int>(r), s, up);
-  } else {
-    lora_down_kernel<8><<<dim3(gx, static_cast<unsigned>((r + 63) / 64)), block, 0, stream>>>(
-        xp, static_cast<int>(M), static_cast<int>(K), ap, static_cast<int>(r), s, up);
-  }
+  const int Mi = static_cast<int>(M), Ki = static_cast<int>(K), ri = static_cast<int>(r);
+  if (r <= 8)
+    launch_pdl(lora_down_kernel<1>, dim3(gx, 1), block, 0, stream, xp, Mi, Ki, ap, ri, s, up);
+  else if (r <= 16)
+    launch_pdl(lora_down_kernel<2>, dim3(gx, 1), block, 0, stream, xp, Mi, Ki, ap, ri, s, up);
+  else if (r <= 32)
+    launch_pdl(lora_down_kernel<4>, dim3(gx, 1), block, 0, stream, xp, Mi, Ki, ap, ri, s, up);
+  else
+    launch_pdl(lora_down_kernel<8>, dim3(gx, static_cast<unsigned>((r + 63) / 64)), block, 0,
+               stream, xp, Mi, Ki, ap, ri, s, up);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
 }
 

@@ -177,6 +177,7 @@ def _run_linear(x_off, x_on, W, A, Bm, s, out=torch.bfloat16, algo=0, want=(True
     (4, 4096, 1032, 16, True, 2),
     (8, 1024, 520, 8, False, 2),
     (16, 512, 512, 64, True, 2),
+    (5, 1032, 1048, 16, False, 2),    # 10 token rows, K % 16 == 8 after two full chunks, N tail
     (3, 520, 72, 16, True, 0),
 ])
 def test_lora_linear_parity(M, K, N, r, shared, algo):
