@@ -252,7 +252,9 @@ hydra_status hydra_rope(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t hea
 
 /* Causal attention, out = softmax(q k^T / sqrt(Dh) + causal mask) v per head, for nseq
  * sequences of P rows each: q, k, v are column blocks [0, d), [d, 2d), [2d, 3d) of qkv
- * (bf16, row stride ld), out bf16 with row stride ld_out. head_dim must be 128. */
+ * (bf16, row stride ld), out bf16 with row stride ld_out. head_dim must be 128; ld and
+ * ld_out multiples of 8, qkv and out 16-byte aligned (else HYDRA_ERR_ALIGN). Runs on the
+ * tcgen05 tensor cores with the probabilities rounded to bf16 before the P V product. */
 hydra_status hydra_causal_attention(const void* qkv, int64_t nseq, int64_t P, int64_t ld,
                                     int64_t n_heads, int64_t head_dim, void* out, int64_t ld_out,
                                     void* stream);

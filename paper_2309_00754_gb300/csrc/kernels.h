@@ -4,6 +4,7 @@
 // failed.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
 #include <stdint.h>
@@ -52,6 +53,10 @@ struct GemmArgs {
 int* device_error_word();
 
 int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream);
+// TMA map over a row-major [rows, cols] bf16 (or fp32) matrix with row stride ld elements:
+// 128-byte swizzle, boxes of [box_rows x 128 bytes], zero fill out of bounds
+bool make_tma_map(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int64_t ld,
+                  int box_rows, bool f32);
 int launch_dual_lora_gemv(const GemmArgs& a, cudaStream_t stream);
 int launch_lora_down(const void* x, int64_t M, int64_t K, const void* A, int64_t r, float s,
                      void* u, cudaStream_t stream);

@@ -770,15 +770,16 @@ static EncodeTiledFn get_encode_fn() {
   return fn;
 }
 
-// 2-D tensor map over a row-major [rows, cols] matrix with 128-byte swizzle and a box of
-// [box_rows, 128 bytes]; out-of-bounds loads read zero, out-of-bounds stores are dropped.
-static bool make_map(CUtensorMap* map, const void* base, int64_t rows, int64_t cols,
-                     int box_rows, bool f32) {
+// 2-D tensor map over a row-major [rows, cols] matrix with row stride ld elements, 128-byte
+// swizzle and a box of [box_rows, 128 bytes]; out-of-bounds loads read zero, out-of-bounds
+// stores are dropped.
+bool make_tma_map(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int64_t ld,
+                  int box_rows, bool f32) {
   EncodeTiledFn enc = get_encode_fn();
   if (enc == nullptr) return false;
   const int esize = f32 ? 4 : 2;
   cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
-  cuuint64_t strides[1] = {static_cast<cuuint64_t>(cols) * esize};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * esize};
   cuuint32_t box[2] = {static_cast<cuuint32_t>(128 / esize), static_cast<cuuint32_t>(box_rows)};
   cuuint32_t estr[2] = {1, 1};
   CUresult r = enc(map, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
@@ -786,6 +787,11 @@ static bool make_map(CUtensorMap* map, const void* base, int64_t rows, int64_t c
                    CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
+}
+
+static bool make_map(CUtensorMap* map, const void* base, int64_t rows, int64_t cols,
+                     int box_rows, bool f32) {
+  return make_tma_map(map, base, rows, cols, cols, box_rows, f32);
 }
 
 static int sm_count() {

@@ -175,7 +175,7 @@ hydra_status hydra_causal_attention(const void* qkv, int64_t nseq, int64_t P, in
   if (nseq < 0 || P < 0 || n_heads < 1 || ld < 3 * n_heads * head_dim ||
       ld_out < n_heads * head_dim)
     return HYDRA_ERR_SHAPE;
-  if (ld % 8 != 0 || ld_out % 2 != 0 || !a16(qkv) || !a16(out)) return HYDRA_ERR_ALIGN;
+  if (ld % 8 != 0 || ld_out % 8 != 0 || !a16(qkv) || !a16(out)) return HYDRA_ERR_ALIGN;
   return rc(hydra::launch_causal_attention(qkv, nseq, P, ld, n_heads, head_dim, out, ld_out,
                                            static_cast<cudaStream_t>(stream)));
 }

@@ -65,11 +65,15 @@ def test_rope_q_k_rotated_v_untouched():
     assert np.array_equal(got[:, 2 * d:], x[:, 2 * d:])
 
 
-@pytest.mark.parametrize("nseq,P,H_", [(3, 100, 2), (1, 768, 1), (2, 64, 1), (1, 1, 2)])
-def test_causal_attention(nseq, P, H_):
+@pytest.mark.parametrize("nseq,P,H_,q_std", [(3, 100, 2, 1.0), (1, 768, 1, 1.0), (2, 64, 1, 1.0),
+                                             (1, 1, 2, 1.0), (2, 300, 2, 1.0),
+                                             (1, 640, 1, 8.0)])  # peaked rows: the running maximum moves
+def test_causal_attention(nseq, P, H_, q_std):
     Dh = 128
     d = H_ * Dh
     qkv_bits = synth.normal_bf16(531 + P, (nseq * P, 3 * d), 1.0)
+    if q_std != 1.0:
+        qkv_bits[:, :d] = synth.normal_bf16(532 + P, (nseq * P, d), q_std)
     out = torch.full((nseq * P, d), float("nan"), dtype=torch.bfloat16, device="cuda")
     H.hydra_causal_attention(dev_bf16(qkv_bits), nseq, P, H_, Dh, out)
     x = f64(qkv_bits)
