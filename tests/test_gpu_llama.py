@@ -67,7 +67,9 @@ def test_rope_q_k_rotated_v_untouched():
 
 @pytest.mark.parametrize("nseq,P,H_,q_std", [(3, 100, 2, 1.0), (1, 768, 1, 1.0), (2, 64, 1, 1.0),
                                              (1, 1, 2, 1.0), (2, 300, 2, 1.0),
-                                             (1, 640, 1, 8.0)])  # peaked rows: the running maximum moves
+                                             (1, 640, 1, 8.0),   # peaked rows: the running maximum moves
+                                             (5, 700, 8, 1.0),   # 240 tiles: CTAs take several
+                                             (3, 384, 4, 8.0)])
 def test_causal_attention(nseq, P, H_, q_std):
     Dh = 128
     d = H_ * Dh
