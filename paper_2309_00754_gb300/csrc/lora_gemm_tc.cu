@@ -64,6 +64,9 @@ struct Params {
   int m_tiles, n_tiles, total_tiles;
   int has_off, has_on;
   int out_f32;
+  int bn;          // tile width in output columns (multiple of 16; 256 for the single-CTA kernel)
+  void* y_off_ptr;  // the outputs as plain pointers, for columns past the last full store chunk
+  void* y_on_ptr;
   int* err;
 };
 
@@ -76,7 +79,7 @@ __device__ __forceinline__ Tile decode(const Params& p, int t) {
   tl.stream = t % p.streams;
   t /= p.streams;
   tl.m0 = (t % p.m_tiles) * BM;
-  tl.n0 = (t / p.m_tiles) * BN;
+  tl.n0 = (t / p.m_tiles) * p.bn;
   const bool on = p.shared_x ? true : (tl.stream == 1);
   tl.n_lora = (p.kb_lora > 0 && on && p.has_on) ? p.kb_lora : 0;
   return tl;
@@ -124,10 +127,14 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t
 // -> TMA store of a [32 rows x 128 B] box; two staging buffers alternate.
 __device__ __forceinline__ void drain(uint32_t tmem_acc, int q, int lane, uint32_t staging,
                                       uint32_t& chunk_ctr, const Params& p, int m0, int n0,
-                                      const CUtensorMap* t0, const CUtensorMap* t1) {
+                                      const CUtensorMap* t0, const CUtensorMap* t1, void* p0,
+                                      void* p1) {
   // output chunks of 128 bytes per row: fp32 32 columns, bf16 64 columns, SwiGLU 64
-  // output columns from 128 accumulator columns
-  const int nchunks = p.epi == EPI_SWIGLU ? 2 : ((p.out_f32 || p.epi == EPI_RESIDUAL) ? BN / 32 : BN / 64);
+  // output columns from 128 accumulator columns; a tile width that is not a whole number of
+  // chunks leaves a tail of tail_cols accumulator columns
+  const int chunk_cols = (p.out_f32 || p.epi == EPI_RESIDUAL) ? 32 : 64;
+  const int nchunks = p.epi == EPI_SWIGLU ? 2 : p.bn / chunk_cols;
+  const int tail_cols = p.epi == EPI_SWIGLU ? 0 : p.bn - nchunks * chunk_cols;
   const uint32_t lane_taddr = tmem_acc + (static_cast<uint32_t>(q * 32) << 16);
   const int y = m0 + q * 32;
   for (int c = 0; c < nchunks; ++c) {
@@ -196,6 +203,47 @@ __device__ __forceinline__ void drain(uint32_t tmem_acc, int q, int lane, uint32
       bulk_commit();
     }
     ++chunk_ctr;
+  }
+  // the tail (a multiple of 16 columns) goes straight from registers to global memory: thread
+  // `lane` owns output row y + lane; only this tile writes these columns
+  const int row = y + lane;
+  for (int c16 = 0; c16 < tail_cols; c16 += 16) {
+    uint32_t v[16];
+    tc_ld_32x32b_x16(lane_taddr + nchunks * chunk_cols + c16, v);
+    tc_wait_ld();
+    const int xc = n0 + nchunks * chunk_cols + c16;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int x = xc + 8 * h;
+      if (row >= p.M || x >= p.N) continue;  // N % 8 == 0: 8 columns are all in or all out
+      const size_t off = static_cast<size_t>(row) * p.N + x;
+#pragma unroll
+      for (int o = 0; o < 2; ++o) {
+        void* dst = o == 0 ? p0 : p1;
+        if (dst == nullptr) continue;
+        if (p.epi == EPI_RESIDUAL || p.out_f32) {
+          float4* d4 = reinterpret_cast<float4*>(static_cast<float*>(dst) + off);
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            float4 val = make_float4(__uint_as_float(v[8 * h + 4 * e]), __uint_as_float(v[8 * h + 4 * e + 1]),
+                                     __uint_as_float(v[8 * h + 4 * e + 2]), __uint_as_float(v[8 * h + 4 * e + 3]));
+            if (p.epi == EPI_RESIDUAL) {
+              const float4 old = d4[e];
+              val = make_float4(old.x + bf16_round(val.x), old.y + bf16_round(val.y),
+                                old.z + bf16_round(val.z), old.w + bf16_round(val.w));
+            }
+            d4[e] = val;
+          }
+        } else {
+          uint4 w4;
+          w4.x = pack_bf16x2(__uint_as_float(v[8 * h]), __uint_as_float(v[8 * h + 1]));
+          w4.y = pack_bf16x2(__uint_as_float(v[8 * h + 2]), __uint_as_float(v[8 * h + 3]));
+          w4.z = pack_bf16x2(__uint_as_float(v[8 * h + 4]), __uint_as_float(v[8 * h + 5]));
+          w4.w = pack_bf16x2(__uint_as_float(v[8 * h + 6]), __uint_as_float(v[8 * h + 7]));
+          *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(dst) + off) = w4;
+        }
+      }
+    }
   }
 }
 
@@ -373,6 +421,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     uint32_t chunk_ctr = 0;
     const CUtensorMap* y_off = p.has_off ? &tm_y_off : nullptr;
     const CUtensorMap* y_on = p.has_on ? &tm_y_on : nullptr;
+    void* py_off = p.has_off ? p.y_off_ptr : nullptr;
+    void* py_on = p.has_on ? p.y_on_ptr : nullptr;
     if (lane == 0) {
       tma_prefetch_desc(&tm_y_off);
       tma_prefetch_desc(&tm_y_on);
@@ -384,21 +434,22 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       if (p.deferred) {
         if (!mbar_wait_bounded(acc_full(b), 0, abort_flag, p.err, kDevTimeoutEpilogue)) break;
         tc_fence_after();
-        drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, y_off, nullptr);
+        drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, y_off, nullptr, py_off, nullptr);
         tc_fence_before();
         mbar_arrive(acc_mid(b));
         if (!mbar_wait_bounded(acc_full(b), 1, abort_flag, p.err, kDevTimeoutEpilogue)) break;
         tc_fence_after();
-        drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, y_on, nullptr);
+        drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, y_on, nullptr, py_on, nullptr);
       } else {
         if (!mbar_wait_bounded(acc_full(b), (j >> 1) & 1, abort_flag, p.err, kDevTimeoutEpilogue))
           break;
         tc_fence_after();
         if (p.shared_x)
-          drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, tl.n_lora > 0 ? nullptr : y_off, y_on);
+          drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, tl.n_lora > 0 ? nullptr : y_off, y_on,
+                tl.n_lora > 0 ? nullptr : py_off, py_on);
         else
           drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, tl.stream == 1 ? y_on : y_off,
-                nullptr);
+                nullptr, tl.stream == 1 ? py_on : py_off, nullptr);
       }
       tc_fence_before();
       mbar_arrive(acc_empty(b));
@@ -431,7 +482,6 @@ constexpr int B_HALF = 128 * BK * 2;             // 16 KiB: this CTA's 128 rows 
 constexpr int STAGE2_BYTES = A_TILE + B_HALF;     // 32 KiB
 constexpr int SMEM2_BYTES =
     1024 + STAGES2 * STAGE2_BYTES + EPI_WARPS * 2 * STAGING_BYTES + (2 * STAGES2 + 7) * 8 + 16;
-constexpr uint32_t IDESC2 = idesc_bf16_f32(256, BN);
 
 __device__ __forceinline__ uint32_t cluster_rank() {
   uint32_t r;
@@ -576,7 +626,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     tl.stream = t % p.streams;
     t /= p.streams;
     tl.m0 = (t % p.m_tiles) * 256 + static_cast<int>(rank) * 128;
-    tl.n0 = (t / p.m_tiles) * BN;
+    tl.n0 = (t / p.m_tiles) * p.bn;
     const bool on = p.shared_x ? true : (tl.stream == 1);
     tl.n_lora = (p.kb_lora > 0 && on && p.has_on) ? p.kb_lora : 0;
     return tl;
@@ -596,7 +646,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
         return;
       }
       if (elect_one()) {
-        if (leader) mbar_arrive_expect_tx(full_bar(s), 2 * STAGE2_BYTES);
+        if (leader) mbar_arrive_expect_tx(full_bar(s), 2 * (A_TILE + p.bn * 64));
         const uint32_t bar = leader_full0 + s * 8;
         const uint32_t a_dst = smem_base + s * STAGE2_BYTES;
         tma_load_2d_pair(a_dst, ma, xa, ya, bar);
@@ -605,7 +655,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       __syncwarp();
       ++it;
     };
-    const int brow = static_cast<int>(rank) * 128;  // this CTA's half of the B rows
+    const int brow = static_cast<int>(rank) * (p.bn / 2);  // this CTA's half of the B rows
     Tile prev{0, 0, 0, 0};
     for (int j = 0; j < n_local && ok; ++j) {
       const Tile tl = decode2(cluster + j * nclusters);
@@ -635,6 +685,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     if (leader) {
       // ---------------------------------------------------------- MMA issuer (leader CTA;
       // whole warp, one elected lane issues every MMA and commit)
+      const uint32_t idesc2 = idesc_bf16_f32(256, p.bn);
       int it = 0;
       bool ok = true;
       auto consume = [&](uint32_t acc, int nsub, bool first, uint32_t then) {
@@ -650,7 +701,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
           const uint32_t b_base = a_base + A_TILE;
           for (int k = 0; k < nsub; ++k)
             tc_mma2_bf16(acc, smem_desc_sw128(a_base + k * 32), smem_desc_sw128(b_base + k * 32),
-                         IDESC2, (first && k == 0) ? 0u : 1u);
+                         idesc2, (first && k == 0) ? 0u : 1u);
           tc_commit_pair(empty_bar(s));
           if (then) tc_commit_pair(then);
         }
@@ -701,6 +752,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     uint32_t chunk_ctr = 0;
     const CUtensorMap* y_off = p.has_off ? &tm_y_off : nullptr;
     const CUtensorMap* y_on = p.has_on ? &tm_y_on : nullptr;
+    void* py_off = p.has_off ? p.y_off_ptr : nullptr;
+    void* py_on = p.has_on ? p.y_on_ptr : nullptr;
     const uint32_t leader_mid0 = map_to_rank(acc_mid(0), 0);
     const uint32_t leader_empty0 = map_to_rank(acc_empty(0), 0);
     auto signal = [&](uint32_t leader_bar0, int b) {
@@ -714,21 +767,22 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       if (p.deferred) {
         if (!mbar_wait_bounded(acc_full(b), 0, abort_flag, p.err, kDevTimeoutEpilogue)) break;
         tc_fence_after();
-        drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, y_off, nullptr);
+        drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, y_off, nullptr, py_off, nullptr);
         tc_fence_before();
         signal(leader_mid0, b);
         if (!mbar_wait_bounded(acc_full(b), 1, abort_flag, p.err, kDevTimeoutEpilogue)) break;
         tc_fence_after();
-        drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, y_on, nullptr);
+        drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, y_on, nullptr, py_on, nullptr);
       } else {
         if (!mbar_wait_bounded(acc_full(b), (j >> 1) & 1, abort_flag, p.err, kDevTimeoutEpilogue))
           break;
         tc_fence_after();
         if (p.shared_x)
-          drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, tl.n_lora > 0 ? nullptr : y_off, y_on);
+          drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, tl.n_lora > 0 ? nullptr : y_off, y_on,
+                tl.n_lora > 0 ? nullptr : py_off, py_on);
         else
           drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, tl.stream == 1 ? y_on : y_off,
-                nullptr);
+                nullptr, tl.stream == 1 ? py_on : py_off, nullptr);
       }
       tc_fence_before();
       signal(leader_empty0, b);
@@ -806,6 +860,30 @@ static int sm_count() {
   return cached[dev];
 }
 
+// Tile width of the CTA-pair kernel: the candidate with the least waves x (width + 224)
+// over the clusters. A tile costs its columns plus a fixed share worth about 224 columns
+// (fitted on GB300: 6144 x 4096 x 12288 ran 6.8 % slower at 208 wide, 19 full waves, than at
+// 256, 15.2 waves). Narrower tiles pay off when they turn a nearly empty last wave into
+// full ones (4096 output columns at 3072 rows per stream: 256 wide gives 5.05 waves, 224
+// wide exactly 6; measured +8 %). The SwiGLU epilogue needs 256 (128 gate + 128 up).
+static int pick_tile_width(const GemmArgs& a, int nclusters) {
+  if (a.epi == tcgemm::EPI_SWIGLU || nclusters < 1) return 256;
+  const int64_t m_tiles = (a.M + 255) / 256;
+  const int64_t streams = a.shared_x ? 1 : 2;
+  int best = 256;
+  int64_t best_cost = INT64_MAX;
+  for (int bn : {256, 240, 224, 208, 192}) {
+    const int64_t tiles = m_tiles * streams * ((a.N + bn - 1) / bn);
+    const int64_t waves = (tiles + nclusters - 1) / nclusters;
+    const int64_t cost = waves * (bn + 224);
+    if (cost < best_cost) {
+      best = bn;
+      best_cost = cost;
+    }
+  }
+  return best;
+}
+
 int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream) {
   using namespace tcgemm;
   static bool attr_set = false;
@@ -822,12 +900,13 @@ int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream) {
   if (nsm <= 0) return -1;
   // 256-row CTA pairs once every stream has more than one 128-row tile of work
   const bool pair = a.M > BM && nsm >= 2 && !a.single_cta;
+  const int bn = pair ? pick_tile_width(a, nsm / 2) : BN;
   CUtensorMap m_xoff, m_xon, m_w, m_u, m_b, m_yoff, m_yon;
   const bool lora = a.r > 0;
   const bool f32 = a.out_f32 != 0;
   if (!make_map(&m_xoff, a.x_off, a.M, a.K, BM, false)) return -2;
   if (!make_map(&m_xon, a.shared_x ? a.x_off : a.x_on, a.M, a.K, BM, false)) return -2;
-  const int brows = pair ? 128 : BN;  // a CTA of a pair loads half of the tile's W rows
+  const int brows = pair ? bn / 2 : BN;  // a CTA of a pair loads half of the tile's W rows
   if (!make_map(&m_w, a.W, a.N, a.K, brows, false)) return -2;
   if (lora) {
     if (!make_map(&m_u, a.u, a.M, a.r, BM, false)) return -2;
@@ -857,9 +936,12 @@ int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream) {
   p.deferred = (p.shared_x && lora && p.has_off && p.has_on) ? 1 : 0;
   p.streams = a.shared_x ? 1 : 2;
   p.m_tiles = static_cast<int>(pair ? (a.M + 255) / 256 : (a.M + BM - 1) / BM);
-  p.n_tiles = static_cast<int>((a.N + BN - 1) / BN);
+  p.n_tiles = static_cast<int>((a.N + bn - 1) / bn);
   p.total_tiles = p.m_tiles * p.n_tiles * p.streams;
   p.out_f32 = a.out_f32;
+  p.bn = bn;
+  p.y_off_ptr = a.y_off;
+  p.y_on_ptr = a.y_on;
   p.err = a.err;
   if (pair) {
     const int nclusters = nsm / 2;

@@ -170,6 +170,9 @@ def _run_linear(x_off, x_on, W, A, Bm, s, out=torch.bfloat16, algo=0, want=(True
     (200, 512, 264, 128, True, 1),
     (700, 1024, 1280, 16, True, 1),   # several tiles per CTA pair (persistent loop)
     (700, 1024, 1280, 16, False, 1),
+    (300, 256, 4264, 16, False, 1),   # CTA-pair tile widths 240, 208, 224 on GB300: stores of
+    (300, 256, 3656, 16, False, 1),   # the columns past the last whole 64-column chunk
+    (300, 256, 3960, 16, False, 1),
     (64, 256, 512, 0, True, 1),       # no LoRA
     (96, 256, 512, 0, False, 1),
     (400, 256, 512, 0, False, 1),
@@ -311,10 +314,12 @@ def test_swiglu_epilogue(shared):
     assert_rel(host_f64(y_on), O.round_bf16(O.swiglu(g_on, u_on)), TOL_LINEAR, "swiglu on")
 
 
-@pytest.mark.parametrize("shared", [True, False])
-def test_residual_epilogue(shared):
-    """Projection added into an fp32 residual stream by the tcgen05 epilogue."""
-    M, K, N, r = 260, 640, 520, 16
+@pytest.mark.parametrize("shared,M,K,N", [(True, 260, 640, 520), (False, 260, 640, 520),
+                                           (False, 300, 256, 4264), (False, 300, 256, 3656)])
+def test_residual_epilogue(shared, M, K, N):
+    """Projection added into an fp32 residual stream by the tcgen05 epilogue (the last two
+    shapes take 240- and 208-column CTA-pair tiles on GB300: a 16-column tail per tile)."""
+    r = 16
     x, x2, W, _, B = _linear_problem(M, K, N, r, seed=42)
     u = synth.normal_bf16(421, (M, r), 2.0)
     h0 = synth.normal_f32(422, (2, M, N), 3.0)
@@ -327,6 +332,19 @@ def test_residual_epilogue(shared):
     got = host_f64(h)
     assert_rel(got[0], h0[0].astype(np.float64) + y_off, TOL_LINEAR, "residual off")
     assert_rel(got[1], h0[1].astype(np.float64) + y_on, TOL_LINEAR, "residual on")
+
+
+@pytest.mark.parametrize("N", [4264, 3656])
+def test_fp32_output_tile_tails(N):
+    """fp32 outputs with 240- / 208-column CTA-pair tiles (32-column store chunks + a 16-column
+    tail per tile)."""
+    M, K, r = 300, 256, 16
+    x, x2, W, A, Bm = _linear_problem(M, K, N, r, seed=43 + N)
+    y_off, y_on = _run_linear(dev_bf16(x), dev_bf16(x2), dev_bf16(W), dev_bf16(A), dev_bf16(Bm), 2.0,
+                              out=torch.float32, algo=1)
+    ref_off, ref_on = O.dual_lora_linear(f64(x), f64(x2), f64(W), f64(A), f64(Bm), 2.0, out_bf16=False)
+    assert_rel(host_f64(y_off), ref_off, 1e-4, "y_off fp32")
+    assert_rel(host_f64(y_on), ref_on, 1e-4, "y_on fp32")
 
 
 def test_epilogue_argument_errors():
