@@ -147,6 +147,37 @@ hydra_status hydra_dual_linear_ex(const void* x_off, const void* x_on, int64_t M
                                   void* stream);
 
 /*
+ * Rotation table of the rotary position embedding (RoFormer, rotate-half pairing, as used by
+ * hydra_rope): table[2 (pos * head_dim/2 + i) + {0, 1}] = (cos a, sin a) with
+ * a = pos * theta^(-2i/head_dim), evaluated in fp32 exactly as hydra_rope evaluates it, for
+ * pos in [0, P) and pair i in [0, head_dim/2). table: fp32 [P, head_dim/2, 2], 16-byte
+ * aligned, caller-owned. Errors: NULL table -> HYDRA_ERR_NULL; P < 0, odd or < 2 head_dim ->
+ * HYDRA_ERR_SHAPE; theta <= 0 -> HYDRA_ERR_RANGE; misaligned table -> HYDRA_ERR_ALIGN.
+ */
+hydra_status hydra_rope_table(int64_t P, int64_t head_dim, float theta, float* table,
+                              void* stream);
+
+/*
+ * hydra_dual_linear on the tcgen05 kernel with the rotary position embedding of the Llama
+ * attention fused into the epilogue, for the fused q/k/v projection: every output value is
+ * first rounded to bf16 (the value hydra_dual_linear would store); then on columns
+ * [0, rope_cols), in heads of head_dim = 128, the pairs (i, i + 64) of a head become
+ *     x_i cos(a) - x_{i+64} sin(a),   x_i sin(a) + x_{i+64} cos(a)
+ * with (cos a, sin a) = rope_table[row % P][i] (hydra_rope_table with this P and head_dim;
+ * rows of each stream are sequences of P tokens), each product and sum rounded as hydra_rope
+ * rounds them, so the result equals hydra_dual_linear followed by hydra_rope bit for bit.
+ * Columns from rope_cols on are stored as hydra_dual_linear would. bf16 outputs only.
+ * Errors: as hydra_dual_linear_ex; NULL rope_table -> HYDRA_ERR_NULL; misaligned
+ * rope_table -> HYDRA_ERR_ALIGN; head_dim != 128 -> HYDRA_ERR_RANGE; P < 1,
+ * rope_cols % 128 != 0 or rope_cols > N -> HYDRA_ERR_SHAPE.
+ */
+hydra_status hydra_dual_linear_rope(const void* x_off, const void* x_on, int64_t M, int64_t K,
+                                    int64_t N, const void* W, const void* u, const void* B,
+                                    int64_t r, void* y_off, void* y_on, int64_t P,
+                                    int64_t rope_cols, int64_t head_dim, const float* rope_table,
+                                    void* stream);
+
+/*
  * hydra_lora_linear with the kernel family chosen by the caller:
  *   algo 0 = automatic (as hydra_lora_linear), 1 = tcgen05 tile kernel (any M; CTA pairs
  *   with 256-row tiles when M > 128), 2 = GEMV kernel (requires at most 16 token rows over

@@ -38,17 +38,33 @@ inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 
 
 inline size_t round_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
+// Rotary epilogue arguments (hydra_dual_linear_rope).
+struct RopeArgs {
+  int64_t P, cols, head_dim;
+  const float* table;
+};
+constexpr int kEpiRope = 3;  // internal epilogue code of the rotary mode
+
 // u_given: `workspace` already holds u = s x_on A^T (hydra_dual_linear); A is unused.
-// epi: tcgen05 epilogue (store / SwiGLU / residual add); non-store epilogues need algo 1.
+// epi: tcgen05 epilogue (store / SwiGLU / residual add / rotary); non-store epilogues need
+// algo 1 or 3; rope carries the rotary arguments of epi == kEpiRope.
 hydra_status lora_linear_impl(const void* x_off, const void* x_on, int64_t M, int64_t K,
                               int64_t N, const void* W, const void* A, const void* B, int64_t r,
                               float s, void* y_off, void* y_on, int out_dtype, void* workspace,
                               size_t workspace_bytes, int algo, void* stream,
-                              bool u_given = false, int epi = HYDRA_EPI_STORE) {
+                              bool u_given = false, int epi = HYDRA_EPI_STORE,
+                              const RopeArgs* rope = nullptr) {
   if (x_off == nullptr || W == nullptr) return HYDRA_ERR_NULL;
   if (y_off == nullptr && y_on == nullptr) return HYDRA_ERR_NULL;
   if (algo < 0 || algo > 3) return HYDRA_ERR_RANGE;
-  if (epi < HYDRA_EPI_STORE || epi > HYDRA_EPI_RESIDUAL) return HYDRA_ERR_RANGE;
+  if (epi < HYDRA_EPI_STORE || epi > (rope != nullptr ? kEpiRope : HYDRA_EPI_RESIDUAL))
+    return HYDRA_ERR_RANGE;
+  if (epi == kEpiRope) {
+    if (rope->table == nullptr) return HYDRA_ERR_NULL;
+    if (!aligned16(rope->table)) return HYDRA_ERR_ALIGN;
+    if (out_dtype != HYDRA_BF16 || rope->head_dim != 128) return HYDRA_ERR_RANGE;
+    if (rope->P < 1 || rope->cols < 0 || rope->cols > N || rope->cols % 128 != 0) return HYDRA_ERR_SHAPE;
+  }
   if (epi != HYDRA_EPI_STORE && algo != 1 && algo != 3) return HYDRA_ERR_RANGE;
   if (epi == HYDRA_EPI_SWIGLU && N % 256 != 0) return HYDRA_ERR_SHAPE;
   if (out_dtype != HYDRA_BF16 && out_dtype != HYDRA_F32) return HYDRA_ERR_RANGE;
@@ -97,6 +113,11 @@ hydra_status lora_linear_impl(const void* x_off, const void* x_on, int64_t M, in
   g.err = err;
   g.epi = epi;
   g.single_cta = algo == 3;
+  if (epi == kEpiRope) {
+    g.rope_P = rope->P;
+    g.rope_cols = rope->cols;
+    g.rope_table = rope->table;
+  }
   const bool use_gemv = (algo == 2) || (algo == 0 && rows <= hydra::kGemvMaxRows);
   const int rc = use_gemv ? hydra::launch_dual_lora_gemv(g, st) : hydra::launch_dual_lora_gemm_tc(g, st);
   return rc == 0 ? HYDRA_OK : HYDRA_ERR_CUDA;
@@ -186,6 +207,28 @@ hydra_status hydra_dual_linear_ex(const void* x_off, const void* x_on, int64_t M
   return lora_linear_impl(x_off, x_on, M, K, N, W, nullptr, B, r, 1.0f, y_off, y_on, out_dtype,
                           const_cast<void*>(u), hydra_lora_linear_workspace_size(M, r), 1, stream,
                           true, epilogue);
+}
+
+hydra_status hydra_dual_linear_rope(const void* x_off, const void* x_on, int64_t M, int64_t K,
+                                    int64_t N, const void* W, const void* u, const void* B,
+                                    int64_t r, void* y_off, void* y_on, int64_t P,
+                                    int64_t rope_cols, int64_t head_dim, const float* rope_table,
+                                    void* stream) {
+  const RopeArgs rope{P, rope_cols, head_dim, rope_table};
+  return lora_linear_impl(x_off, x_on, M, K, N, W, nullptr, B, r, 1.0f, y_off, y_on, HYDRA_BF16,
+                          const_cast<void*>(u), hydra_lora_linear_workspace_size(M, r), 1, stream,
+                          true, kEpiRope, &rope);
+}
+
+hydra_status hydra_rope_table(int64_t P, int64_t head_dim, float theta, float* table,
+                              void* stream) {
+  if (table == nullptr) return HYDRA_ERR_NULL;
+  if (P < 0 || head_dim < 2 || head_dim % 2 != 0) return HYDRA_ERR_SHAPE;
+  if (!(theta > 0.f)) return HYDRA_ERR_RANGE;
+  if (!aligned16(table)) return HYDRA_ERR_ALIGN;
+  return hydra::launch_rope_table(P, head_dim, theta, table, static_cast<cudaStream_t>(stream)) == 0
+             ? HYDRA_OK
+             : HYDRA_ERR_CUDA;
 }
 
 hydra_status hydra_token_logprobs_kl(const void* logits_actor, const void* logits_ref,

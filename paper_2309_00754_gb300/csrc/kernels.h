@@ -45,8 +45,13 @@ struct GemmArgs {
   void* y_on;         // [M, N] bf16 or fp32, may be NULL
   int out_f32;
   int* err;
-  int epi = 0;        // tcgen05 kernel epilogue: 0 store, 1 SwiGLU, 2 residual add (fp32)
+  int epi = 0;        // tcgen05 kernel epilogue: 0 store, 1 SwiGLU, 2 residual add (fp32), 3 rotary
   bool single_cta = false;  // tcgen05: never use the CTA-pair (cta_group::2) kernel
+  // epi 3 (rotary): columns [0, rope_cols) rotate in heads of 128 at position row % rope_P,
+  // by the (cos, sin) pairs of rope_table [rope_P][64] (launch_rope_table)
+  int64_t rope_P = 1;
+  int64_t rope_cols = 0;
+  const void* rope_table = nullptr;
 };
 
 // Device address of the library's error word on the current device (NULL on failure).
@@ -79,6 +84,8 @@ int launch_embed(const void* table, int64_t V, int64_t d, const int32_t* ids, in
                  int copies, float* h, int* err, cudaStream_t st);
 int launch_rmsnorm(const float* x, const void* w, int64_t rows, int64_t d, float eps,
                    const RowMap& map, void* y, cudaStream_t st);
+// (cos, sin) float2 table [P][Dh / 2] of the rotary angles pos * theta^(-2i/Dh)
+int launch_rope_table(int64_t P, int64_t Dh, float theta, void* table, cudaStream_t st);
 int launch_rope(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t Dh, int64_t P, float theta,
                 cudaStream_t st);
 int launch_swiglu(const void* gu, int64_t R, int64_t F, void* m, cudaStream_t st);

@@ -108,9 +108,27 @@ __global__ void __launch_bounds__(128)
       uint32_t* p1 = reinterpret_cast<uint32_t*>(base + hb * Dh + i);
       uint32_t* p2 = reinterpret_cast<uint32_t*>(base + hb * Dh + i + half);
       const float2 x1 = unpack_bf16x2(*p1), x2 = unpack_bf16x2(*p2);
-      *p1 = pack_bf16x2(x1.x * c0 - x2.x * s0, x1.y * c1 - x2.y * s1);
-      *p2 = pack_bf16x2(x1.x * s0 + x2.x * c0, x1.y * s1 + x2.y * c1);
+      // explicit roundings (no contraction), so the rotary epilogue of the tcgen05 GEMM, which
+      // runs the same operations, gives the same bits
+      *p1 = pack_bf16x2(__fsub_rn(__fmul_rn(x1.x, c0), __fmul_rn(x2.x, s0)),
+                        __fsub_rn(__fmul_rn(x1.y, c1), __fmul_rn(x2.y, s1)));
+      *p2 = pack_bf16x2(__fadd_rn(__fmul_rn(x1.x, s0), __fmul_rn(x2.x, c0)),
+                        __fadd_rn(__fmul_rn(x1.y, s1), __fmul_rn(x2.y, c1)));
     }
+  }
+}
+
+// (cos a, sin a) for a = pos * theta^(-2i/Dh), pos in [0, P), pair i in [0, Dh/2): the rotation
+// table of the fused rotary GEMM epilogue, the same expression as rope_kernel evaluates
+__global__ void rope_table_kernel(long long n, int half, int Dh, float log2_theta,
+                                  float2* __restrict__ table) {
+  for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < n;
+       e += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const float pos = static_cast<float>(e / half);
+    const int i = static_cast<int>(e % half);
+    float c, s;
+    sincosf(pos * exp2f(-(2.0f * i / Dh) * log2_theta), &s, &c);
+    table[e] = make_float2(c, s);
   }
 }
 
@@ -265,6 +283,15 @@ int launch_rope(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t Dh, int64_t
                                                         static_cast<int>(ld), static_cast<int>(d),
                                                         static_cast<int>(Dh), static_cast<int>(P),
                                                         log2f(theta));
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
+}
+
+int launch_rope_table(int64_t P, int64_t Dh, float theta, void* table, cudaStream_t st) {
+  if (P == 0) return 0;
+  const long long n = P * (Dh / 2);
+  rope_table_kernel<<<grid_for(n, 256), 256, 0, st>>>(n, static_cast<int>(Dh / 2),
+                                                      static_cast<int>(Dh), log2f(theta),
+                                                      static_cast<float2*>(table));
   return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
 }
 

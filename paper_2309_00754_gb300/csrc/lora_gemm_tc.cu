@@ -50,7 +50,9 @@ constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN);
 //  EPI_SWIGLU   columns [0, 128) of the tile are gate, [128, 256) up for the same 128
 //               features: y[:, n0/2 + j] = bf16(silu(bf16(gate_j)) * bf16(up_j))
 //  EPI_RESIDUAL y (fp32 residual stream) += float(bf16(acc)) by TMA reduce-add in L2
-enum { EPI_STORE = 0, EPI_SWIGLU = 1, EPI_RESIDUAL = 2 };
+//  EPI_ROPE     y = bf16 rotary embedding of bf16(acc) on columns [0, rope_cols) (heads of
+//               128, rotate-half pairs (i, i + 64), position row % rope_P), bf16(acc) after
+enum { EPI_STORE = 0, EPI_SWIGLU = 1, EPI_RESIDUAL = 2, EPI_ROPE = 3 };
 
 struct Params {
   int M, N, K;
@@ -65,6 +67,8 @@ struct Params {
   int has_off, has_on;
   int out_f32;
   int bn;          // tile width in output columns (multiple of 16; 256 for the single-CTA kernel)
+  int rope_P, rope_cols;
+  const float2* rope_table;  // (cos, sin) [rope_P][64]
   void* y_off_ptr;  // the outputs as plain pointers, for columns past the last full store chunk
   void* y_on_ptr;
   int* err;
@@ -111,6 +115,9 @@ __device__ __forceinline__ void bulk_wait_read1() {
 __device__ __forceinline__ void bulk_wait_all() {
   asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
 }
+__device__ __forceinline__ void bulk_wait_all_read() {
+  asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
 __device__ __forceinline__ void fence_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
@@ -120,6 +127,73 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t
   asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c),
                "r"(d)
                : "memory");
+}
+
+// Rotary epilogue of one warp's 32 rows (thread `lane` owns row y + lane), one head of 128
+// columns at a time: the head's two halves x1 = [0, 64) and x2 = [64, 128) become
+// x1 cos - x2 sin and x1 sin + x2 cos with (cos, sin) of pair i at position pos from the
+// rotation table, on the bf16-rounded accumulator, each rounding explicit (the rotary kernel
+// runs the same operations on the same angles). Both halves are staged (one buffer each)
+// and stored as [32 x 64] boxes.
+__device__ __forceinline__ void drain_rope(uint32_t lane_taddr, int lane, uint32_t staging,
+                                           const Params& p, int y, int n0, const CUtensorMap* t0,
+                                           const CUtensorMap* t1) {
+  const int row = y + lane;
+  const float4* trow = reinterpret_cast<const float4*>(p.rope_table + (row % p.rope_P) * 64);
+  for (int h = 0; h < p.bn / 128; ++h) {
+    const int col0 = n0 + 128 * h;
+    const bool rot = col0 < p.rope_cols;
+    if (lane == 0) bulk_wait_all_read();  // both staging buffers are free
+    __syncwarp();
+#pragma unroll 1
+    for (int g = 0; g < 2; ++g) {
+      uint32_t x1[32], x2[32];
+      tc_ld_32x32b_x32(lane_taddr + 128 * h + 32 * g, x1);
+      tc_ld_32x32b_x32(lane_taddr + 128 * h + 64 + 32 * g, x2);
+      tc_wait_ld();
+      uint32_t o1[16], o2[16];
+#pragma unroll
+      for (int e = 0; e < 16; ++e) {
+        const float a0 = bf16_round(__uint_as_float(x1[2 * e]));
+        const float a1 = bf16_round(__uint_as_float(x1[2 * e + 1]));
+        const float b0 = bf16_round(__uint_as_float(x2[2 * e]));
+        const float b1 = bf16_round(__uint_as_float(x2[2 * e + 1]));
+        if (rot) {
+          const float4 cs = __ldg(trow + 16 * g + e);  // (cos, sin) of pairs 32 g + 2 e, + 1
+          const float c0 = cs.x, s0 = cs.y, c1 = cs.z, s1 = cs.w;
+          o1[e] = pack_bf16x2(__fsub_rn(__fmul_rn(a0, c0), __fmul_rn(b0, s0)),
+                              __fsub_rn(__fmul_rn(a1, c1), __fmul_rn(b1, s1)));
+          o2[e] = pack_bf16x2(__fadd_rn(__fmul_rn(a0, s0), __fmul_rn(b0, c0)),
+                              __fadd_rn(__fmul_rn(a1, s1), __fmul_rn(b1, c1)));
+        } else {
+          o1[e] = pack_bf16x2(a0, a1);
+          o2[e] = pack_bf16x2(b0, b1);
+        }
+      }
+      // half rows of the two [32 x 128 B] staging buffers (128-byte swizzle)
+      const uint32_t r1 = staging + lane * 128, r2 = staging + STAGING_BYTES + lane * 128;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int u = 4 * g + j;
+        st_shared_v4(r1 + ((u ^ (lane & 7)) << 4), o1[4 * j], o1[4 * j + 1], o1[4 * j + 2], o1[4 * j + 3]);
+        st_shared_v4(r2 + ((u ^ (lane & 7)) << 4), o2[4 * j], o2[4 * j + 1], o2[4 * j + 2], o2[4 * j + 3]);
+      }
+    }
+    fence_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      if (y < p.M) {
+        for (int half = 0; half < 2; ++half) {
+          const int x = col0 + 64 * half;
+          if (x >= p.N) continue;
+          const uint32_t buf = staging + half * STAGING_BYTES;
+          if (t0) tma_store_2d(t0, buf, x, y);
+          if (t1) tma_store_2d(t1, buf, x, y);
+        }
+      }
+      bulk_commit();
+    }
+  }
 }
 
 // Epilogue warp: drain the warp's 32 accumulator rows (TMEM lanes) of one tile to up to two
@@ -137,6 +211,10 @@ __device__ __forceinline__ void drain(uint32_t tmem_acc, int q, int lane, uint32
   const int tail_cols = p.epi == EPI_SWIGLU ? 0 : p.bn - nchunks * chunk_cols;
   const uint32_t lane_taddr = tmem_acc + (static_cast<uint32_t>(q * 32) << 16);
   const int y = m0 + q * 32;
+  if (p.epi == EPI_ROPE) {
+    drain_rope(lane_taddr, lane, staging, p, y, n0, t0, t1);
+    return;
+  }
   for (int c = 0; c < nchunks; ++c) {
     const uint32_t buf = staging + (chunk_ctr & 1u) * STAGING_BYTES;
     if (lane == 0) bulk_wait_read1();  // the store issued two chunks ago has read `buf`
@@ -867,7 +945,7 @@ static int sm_count() {
 // full ones (4096 output columns at 3072 rows per stream: 256 wide gives 5.05 waves, 224
 // wide exactly 6; measured +8 %). The SwiGLU epilogue needs 256 (128 gate + 128 up).
 static int pick_tile_width(const GemmArgs& a, int nclusters) {
-  if (a.epi == tcgemm::EPI_SWIGLU || nclusters < 1) return 256;
+  if (a.epi == tcgemm::EPI_SWIGLU || a.epi == tcgemm::EPI_ROPE || nclusters < 1) return 256;
   const int64_t m_tiles = (a.M + 255) / 256;
   const int64_t streams = a.shared_x ? 1 : 2;
   int best = 256;
@@ -940,6 +1018,9 @@ int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream) {
   p.total_tiles = p.m_tiles * p.n_tiles * p.streams;
   p.out_f32 = a.out_f32;
   p.bn = bn;
+  p.rope_P = static_cast<int>(a.rope_P < 1 ? 1 : a.rope_P);
+  p.rope_cols = static_cast<int>(a.rope_cols);
+  p.rope_table = static_cast<const float2*>(a.rope_table);
   p.y_off_ptr = a.y_off;
   p.y_on_ptr = a.y_on;
   p.err = a.err;

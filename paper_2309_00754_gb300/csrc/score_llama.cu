@@ -61,7 +61,7 @@ inline hydra_status rc(int r) { return r == 0 ? HYDRA_OK : HYDRA_ERR_CUDA; }
 
 // Workspace layout of the full pass, in bytes from the workspace base.
 struct PassLayout {
-  size_t h, a, qkv, attn, m, u, fin, logits, sc, total;
+  size_t h, a, qkv, attn, m, u, fin, logits, sc, rope, total;
 };
 
 PassLayout layout(const hydra_llama_config& c, int64_t S) {
@@ -81,6 +81,7 @@ PassLayout layout(const hydra_llama_config& c, int64_t S) {
   L.fin = o;    o += up256(2 * SL * d * 2);
   L.logits = o; o += up256(2 * SL * static_cast<size_t>(c.vocab) * 4);
   L.sc = o;     o += up256(static_cast<size_t>(S) * 4);
+  L.rope = o;   o += up256(P * static_cast<size_t>(c.head_dim / 2) * 8);
   L.total = o;
   return L;
 }
@@ -91,17 +92,23 @@ bool valid_config(const hydra_llama_config* c) {
   if (c->d_model != c->n_heads * c->head_dim) return false;
   if (c->ffn < 128 || c->ffn % 128 != 0 || c->vocab < 8 || c->vocab % 8 != 0) return false;
   if (c->lora_rank < 8 || c->lora_rank > 128 || c->lora_rank % 8 != 0) return false;
-  if (c->prompt_len < 1 || c->response_len < 1) return false;
+  if (c->prompt_len < 1 || c->response_len < 1 || !(c->rope_theta > 0.f)) return false;
   if (c->response_len > hydra::kGaeMaxL) return false;
   return true;
 }
 
 // stacked dual linear: rows [0, T) of x are the off stream, [T, 2T) the on stream
-// epi: tcgen05 epilogue; y is [2T, N] (store), [2T, N/2] bf16 (SwiGLU) or the fp32 residual
-// stream [2T, N] (residual add)
+// epi: tcgen05 epilogue; y is [2T, N] (store, rotary), [2T, N/2] bf16 (SwiGLU) or the fp32
+// residual stream [2T, N] (residual add); rope: rotary arguments of epi == kEpiRope
+constexpr int kEpiRope = 3;
+struct RopeCfg {
+  int64_t P, cols;
+  const void* table;  // (cos, sin) [P][head_dim / 2]
+};
 int stacked_linear(int prof_class, const void* x, int64_t T, int64_t K, int64_t N, const void* W,
                    const void* A, const void* B, int64_t r, float s, void* u, void* y, bool f32,
-                   int* err, cudaStream_t st, int epi = HYDRA_EPI_STORE) {
+                   int* err, cudaStream_t st, int epi = HYDRA_EPI_STORE,
+                   const RopeCfg* rope = nullptr) {
   const size_t xs = static_cast<size_t>(T) * K * 2;
   const size_t ys = epi == HYDRA_EPI_SWIGLU    ? static_cast<size_t>(T) * (N / 2) * 2
                     : epi == HYDRA_EPI_RESIDUAL ? static_cast<size_t>(T) * N * 4
@@ -130,6 +137,11 @@ int stacked_linear(int prof_class, const void* x, int64_t T, int64_t K, int64_t 
   g.out_f32 = f32 ? 1 : 0;
   g.err = err;
   g.epi = epi;
+  if (rope != nullptr) {
+    g.rope_P = rope->P;
+    g.rope_cols = rope->cols;
+    g.rope_table = rope->table;
+  }
   return hydra::launch_dual_lora_gemm_tc(g, st);
 }
 
@@ -283,6 +295,7 @@ hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_
   void* fin = ws + Lo.fin;
   float* logits = reinterpret_cast<float*>(ws + Lo.logits);
   float* sc = reinterpret_cast<float*>(ws + Lo.sc);
+  void* rope_table = ws + Lo.rope;
 
   const int64_t P = c.prompt_len + c.response_len;
   const int64_t T = S * P;
@@ -303,13 +316,16 @@ hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_
   } while (0)
 
   HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_embed(w->embed, V, d, ids, T, 2, h, err, st));
+  // rotation table of the positions 0..P-1, shared by every layer's q/k/v epilogue
+  HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rope_table(P, c.head_dim, c.rope_theta, rope_table, st));
   for (int64_t l = 0; l < c.n_layers; ++l) {
     const hydra_llama_layer& ly = w->layers[l];
     // attention block
     HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(h, ly.norm_attn, R, d, c.rms_eps, ident, a, st));
+    // q/k/v projection with the rotary embedding of q and k fused into the epilogue
+    const RopeCfg rope{P, 2 * d, rope_table};
     HY_TRY(stacked_linear(HYDRA_PROF_GEMM_QKV, a, T, d, 3 * d, ly.w_qkv, ly.a_qv, ly.b_qkv, 2 * r, s, u, qkv, false,
-                          err, st));
-    HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rope(qkv, R, 3 * d, d, c.head_dim, P, c.rope_theta, st));
+                          err, st, kEpiRope, &rope));
     HY_PROF(HYDRA_PROF_ATTENTION,
             hydra::launch_causal_attention(qkv, 2 * S, P, 3 * d, c.n_heads, c.head_dim, attn, d, st));
     // o projection added straight into the residual stream (fused epilogue)

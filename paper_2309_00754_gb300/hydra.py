@@ -36,6 +36,10 @@ _SIGNATURES = {
                                          _vp, _vp, ctypes.c_int, ctypes.c_int, _vp]),
     "hydra_dual_linear_ex": (ctypes.c_int, [_vp, _vp, _c_i64, _c_i64, _c_i64, _vp, _vp, _vp,
                                             _c_i64, _vp, _vp, ctypes.c_int, ctypes.c_int, _vp]),
+    "hydra_dual_linear_rope": (ctypes.c_int, [_vp, _vp, _c_i64, _c_i64, _c_i64, _vp, _vp, _vp,
+                                              _c_i64, _vp, _vp, _c_i64, _c_i64, _c_i64, _vp,
+                                              _vp]),
+    "hydra_rope_table": (ctypes.c_int, [_c_i64, _c_i64, ctypes.c_float, _vp, _vp]),
     "hydra_lora_linear_noalloc": (ctypes.c_int, [_vp, _vp, _c_i64, _c_i64, _c_i64, _vp, _vp, _vp,
                                                  _c_i64, ctypes.c_float, _vp, _vp, ctypes.c_int,
                                                  _vp]),
@@ -240,6 +244,30 @@ def hydra_dual_linear_ex(x_off, x_on, W, u, B, y_off, y_on, epilogue, stream=Non
     _check("hydra_dual_linear_ex", load().hydra_dual_linear_ex(
         _p(x_off), _p(x_on), M, K, N, _p(W), _p(u), _p(B), r, _p(y_off), _p(y_on), out_dtype,
         int(epilogue), _stream(stream)))
+
+
+def hydra_rope_table(P, head_dim, theta, table, stream=None):
+    """(cos, sin) of the rotary angles: table fp32 [P, head_dim // 2, 2]."""
+    _req(table, torch.float32, "table")
+    _check("hydra_rope_table", load().hydra_rope_table(int(P), int(head_dim), float(theta),
+                                                       _p(table), _stream(stream)))
+
+
+def hydra_dual_linear_rope(x_off, x_on, W, u, B, y_off, y_on, P, rope_cols, head_dim, table,
+                           stream=None):
+    """tcgen05 dual linear (bf16 outputs) with the rotary embedding of columns
+    [0, rope_cols) fused into the epilogue, angles from hydra_rope_table; equal to
+    hydra_dual_linear + hydra_rope."""
+    _req(table, torch.float32, "table")
+    for t, n in ((x_off, "x_off"), (x_on, "x_on"), (W, "W"), (u, "u"), (B, "B"),
+                 (y_off, "y_off"), (y_on, "y_on")):
+        _req(t, torch.bfloat16, n)
+    M, K = x_off.shape
+    N = W.shape[0]
+    r = 0 if u is None else u.shape[1]
+    _check("hydra_dual_linear_rope", load().hydra_dual_linear_rope(
+        _p(x_off), _p(x_on), M, K, N, _p(W), _p(u), _p(B), r, _p(y_off), _p(y_on), int(P),
+        int(rope_cols), int(head_dim), _p(table), _stream(stream)))
 
 
 def hydra_token_logprobs_kl(logits_actor, logits_ref, ids, lengths, seq_score, beta, S, L,

@@ -69,6 +69,29 @@ def test_lora_linear_argument_errors(lib):
     assert _lin(lib, M=0) == 0                                  # empty: no launch
 
 
+def test_rope_linear_argument_errors(lib):
+    f = lib.hydra_dual_linear_rope
+
+    def call(**kw):
+        a = dict(M=64, K=64, N=768, P=100, cols=512, hd=128, table=FAKE)
+        a.update(kw)
+        return f(FAKE, None, a["M"], a["K"], a["N"], FAKE, None, None, 0, FAKE, None, a["P"],
+                 a["cols"], a["hd"], a["table"], None)
+    assert call(hd=64) == 4          # heads of 128 only
+    assert call(table=None) == 1
+    assert call(table=FAKE + 8) == 3
+    assert call(cols=500) == 2       # whole heads
+    assert call(cols=896) == 2       # beyond N
+    assert call(P=0) == 2
+    assert call(M=0) == 0            # empty: no launch
+    t = lib.hydra_rope_table
+    assert t(100, 128, 1e4, None, None) == 1
+    assert t(100, 127, 1e4, FAKE, None) == 2
+    assert t(100, 128, 0.0, FAKE, None) == 4
+    assert t(100, 128, 1e4, FAKE + 4, None) == 3
+    assert t(0, 128, 1e4, FAKE, None) == 0
+
+
 def test_logprobs_and_gae_argument_errors(lib):
     f = lib.hydra_token_logprobs_kl
     assert f(FAKE, FAKE, 5, 1, 1, 10, 10, FAKE, None, None, 0.1, FAKE, FAKE, FAKE, None, None, None) == 4

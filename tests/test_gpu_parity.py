@@ -347,6 +347,42 @@ def test_fp32_output_tile_tails(N):
     assert_rel(host_f64(y_on), ref_on, 1e-4, "y_on fp32")
 
 
+@pytest.mark.parametrize("M,shared", [(300, False), (100, True), (700, False)])
+def test_rope_epilogue(M, shared):
+    """q/k/v projection with the rotary embedding fused into the tcgen05 epilogue: equal bit for
+    bit to the projection followed by hydra_rope, and to the oracle's rotation of the
+    bf16-rounded projection within the linear tolerance. M = 100 runs the single-CTA kernel."""
+    H_, Dh, K, r, P, theta = 3, 128, 256, 16, 150, 10000.0
+    d = H_ * Dh
+    N = 3 * d
+    x, x2, W, _, B = _linear_problem(M, K, N, r, seed=44 + M)
+    u = synth.normal_bf16(441 + M, (M, r), 2.0)
+    xs = [dev_bf16(t) for t in (x, x2, W, u, B)]
+    x_on = None if shared else xs[1]
+    ref = [torch.empty(M, N, dtype=torch.bfloat16, device="cuda") for _ in range(2)]
+    H.hydra_dual_linear(xs[0], x_on, xs[2], xs[3], xs[4], ref[0], ref[1], algo=1)
+    for t in ref:
+        H.hydra_rope(t, d, Dh, P, theta)
+    table = torch.empty(P, Dh // 2, 2, device="cuda")
+    H.hydra_rope_table(P, Dh, theta, table)
+    ang = np.arange(P)[:, None] * theta ** (-np.arange(Dh // 2) * 2.0 / Dh)[None, :]
+    tab = host_f64(table)
+    assert np.abs(tab[..., 0] - np.cos(ang)).max() < 1e-4 and np.abs(tab[..., 1] - np.sin(ang)).max() < 1e-4
+    got = [torch.full((M, N), float("nan"), dtype=torch.bfloat16, device="cuda") for _ in range(2)]
+    H.hydra_dual_linear_rope(xs[0], x_on, xs[2], xs[3], xs[4], got[0], got[1], P, 2 * d, Dh, table)
+    assert torch.equal(got[0], ref[0]) and torch.equal(got[1], ref[1])
+    xo = x if shared else x2
+    pos = np.arange(M) % P
+    for y_dev, inp, lora in ((got[0], x, False), (got[1], xo, True)):
+        lin = f64(inp) @ f64(W).T + (f64(u) @ f64(B).T if lora else 0.0)
+        lin = O.round_bf16(lin)
+        want = lin.copy()
+        for blk in range(2):
+            want[:, blk * d:(blk + 1) * d] = O.round_bf16(
+                O.rope(lin[:, blk * d:(blk + 1) * d].reshape(M, H_, Dh), pos, theta)).reshape(M, d)
+        assert_rel(host_f64(y_dev), want, TOL_LINEAR, "rotary epilogue")
+
+
 def test_epilogue_argument_errors():
     x = torch.zeros(16, 64, dtype=torch.bfloat16, device="cuda")
     W = torch.zeros(200, 64, dtype=torch.bfloat16, device="cuda")
