@@ -109,21 +109,23 @@ __global__ void __launch_bounds__(32 * kDownWarps)
 // ---------------------------------------------------------------- dual_lora_gemv
 //
 // Decode-shaped dual-output linear (at most 16 token rows over both streams). HBM-bound:
-// every byte of W is read once. One CTA per 16 rows of W; its 8 warps split K and stream
-// their [16 x 64] W and token-row slices into XOR-swizzled shared memory with cp.async
-// (3-4 stages per warp, 16-byte copies), then run mma.sync m16n8k16 with W as the 16-row
-// operand and the token rows as the 8-wide operand (both through ldmatrix), so the
-// arithmetic never limits the stream even at 16 rows. The 8 partial tiles are reduced in
-// shared memory, where each thread also adds the rank-r LoRA term of its (row, token).
+// every byte of W is read once. One CTA per 16 rows of W; its warps (8, or 4 when there are
+// at least four row blocks per SM) split K and stream their [16 x 64] W and token-row slices
+// into XOR-swizzled shared memory with cp.async (3 stages per warp, 16-byte copies), then
+// run mma.sync m16n8k16 with W as the 16-row operand and the token rows as the 8-wide
+// operand (both through ldmatrix), so the arithmetic never limits the stream even at 16
+// rows. The partial tiles are reduced in shared memory, where each thread also adds the
+// rank-r LoRA term of its (row, token). (Measured on GB300: concurrent CTAs per SM matter
+// more than ring depth; 4 warps per CTA lift the 11008- and 32000-row shapes by 10-25 %,
+// while 4096-row shapes, 256 CTAs, need 8 warps to keep enough loads in flight.)
 
-constexpr int kGvWarps = 8;
-// per-warp ring: stage = 16 W rows + 8 NT token rows of 64 bf16; 4 stages for <= 8 token
-// rows, 3 for 16 (so that two CTAs fit an SM)
-template <int NT>
+// per-warp ring: stage = 16 W rows + 8 NT token rows of 64 bf16, 3 stages
+template <int NT, int W>  // NT n-tiles of 8 token rows, W warps
 struct Gv {
-  static constexpr int kStages = NT == 1 ? 4 : 3;
+  static constexpr int kWarps = W;
+  static constexpr int kStages = 3;
   static constexpr int kStageBytes = (16 + 8 * NT) * 128;
-  static constexpr int kSmem = kGvWarps * kStages * kStageBytes + kGvWarps * 16 * 16 * 4;
+  static constexpr int kSmem = W * kStages * kStageBytes + W * 16 * 16 * 4;
 };
 
 __device__ __forceinline__ void gv_cp_async16(uint32_t dst, const void* src, bool ok) {
@@ -142,7 +144,7 @@ __device__ __forceinline__ void gv_ldsm_x4(uint32_t addr, uint32_t (&a)[4]) {
                : "r"(addr));
 }
 
-template <int NT>  // n-tiles of 8 token rows (1 or 2)
+template <int NT, int kGvWarps>  // n-tiles of 8 token rows (1 or 2), warps per CTA
 __global__ void __launch_bounds__(32 * kGvWarps)
     dual_lora_gemv_kernel(const __nv_bfloat16* __restrict__ x_off,
                           const __nv_bfloat16* __restrict__ x_on, int M, int K, int N,
@@ -150,8 +152,8 @@ __global__ void __launch_bounds__(32 * kGvWarps)
                           const __nv_bfloat16* __restrict__ B, int r, void* y_off, void* y_on,
                           int out_f32, int shared_x) {
   extern __shared__ __align__(1024) uint8_t smem[];
-  constexpr int kGvStages = Gv<NT>::kStages;
-  constexpr int kGvStageBytes = Gv<NT>::kStageBytes;
+  constexpr int kGvStages = Gv<NT, kGvWarps>::kStages;
+  constexpr int kGvStageBytes = Gv<NT, kGvWarps>::kStageBytes;
   float* red = reinterpret_cast<float*>(smem + kGvWarps * kGvStages * kGvStageBytes);
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -260,61 +262,64 @@ __global__ void __launch_bounds__(32 * kGvWarps)
     rw[(g + 8) * 16 + t * 8 + 2 * c + 1] = d[t][3];
   }
   __syncthreads();
-  // one (row, token) output per thread: row fastest for coalesced stores
-  const int row = threadIdx.x & 15, tk = threadIdx.x >> 4;
-  const int n = n0 + row;
-  if (tk >= tokens || tk >= NT * 8 || n >= N) return;
-  float acc = 0.f;
+  // (row, token) outputs, row fastest for coalesced stores; 16 x 8 NT of them over the CTA
+  for (int o = threadIdx.x; o < 16 * 8 * NT; o += 32 * kGvWarps) {
+    const int row = o & 15, tk = o >> 4;
+    const int n = n0 + row;
+    if (tk >= tokens || n >= N) continue;
+    float acc = 0.f;
 #pragma unroll
-  for (int w = 0; w < kGvWarps; ++w) acc += red[w * 256 + row * 16 + tk];
-  auto put = [&](void* y, int m, float v) {
-    if (y == nullptr) return;
-    const size_t o = static_cast<size_t>(m) * N + n;
-    if (out_f32)
-      reinterpret_cast<float*>(y)[o] = v;
-    else
-      reinterpret_cast<__nv_bfloat16*>(y)[o] = __float2bfloat16_rn(v);
-  };
-  auto lora = [&](int m) {
-    // rank-r dot product with 16-byte loads (r % 8 == 0)
-    float v = 0.f;
-    if (u != nullptr) {
-      const uint4* up = reinterpret_cast<const uint4*>(u + static_cast<size_t>(m) * r);
-      const uint4* bp = reinterpret_cast<const uint4*>(B + static_cast<size_t>(n) * r);
-      for (int j = 0; j < r / 8; ++j) {
-        const uint4 a4 = __ldg(up + j), b4 = __ldg(bp + j);
-        const uint32_t* ap = &a4.x;
-        const uint32_t* bq = &b4.x;
+    for (int w = 0; w < kGvWarps; ++w) acc += red[w * 256 + row * 16 + tk];
+    auto put = [&](void* y, int m, float v) {
+      if (y == nullptr) return;
+      const size_t off = static_cast<size_t>(m) * N + n;
+      if (out_f32)
+        reinterpret_cast<float*>(y)[off] = v;
+      else
+        reinterpret_cast<__nv_bfloat16*>(y)[off] = __float2bfloat16_rn(v);
+    };
+    auto lora = [&](int m) {
+      // rank-r dot product with 16-byte loads (r % 8 == 0)
+      float v = 0.f;
+      if (u != nullptr) {
+        const uint4* up = reinterpret_cast<const uint4*>(u + static_cast<size_t>(m) * r);
+        const uint4* bp = reinterpret_cast<const uint4*>(B + static_cast<size_t>(n) * r);
+        for (int j = 0; j < r / 8; ++j) {
+          const uint4 a4 = __ldg(up + j), b4 = __ldg(bp + j);
+          const uint32_t* ap = &a4.x;
+          const uint32_t* bq = &b4.x;
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float2 fa = unpack_bf16x2(ap[e]), fb = unpack_bf16x2(bq[e]);
-          v = fmaf(fa.x, fb.x, v);
-          v = fmaf(fa.y, fb.y, v);
+          for (int e = 0; e < 4; ++e) {
+            const float2 fa = unpack_bf16x2(ap[e]), fb = unpack_bf16x2(bq[e]);
+            v = fmaf(fa.x, fb.x, v);
+            v = fmaf(fa.y, fb.y, v);
+          }
         }
       }
+      return v;
+    };
+    if (shared_x) {
+      put(y_off, tk, acc);
+      if (y_on != nullptr) put(y_on, tk, acc + lora(tk));
+    } else if (tk < M) {
+      put(y_off, tk, acc);
+    } else {
+      put(y_on, tk - M, acc + lora(tk - M));
     }
-    return v;
-  };
-  if (shared_x) {
-    put(y_off, tk, acc);
-    if (y_on != nullptr) put(y_on, tk, acc + lora(tk));
-  } else if (tk < M) {
-    put(y_off, tk, acc);
-  } else {
-    put(y_on, tk - M, acc + lora(tk - M));
   }
 }
 
-template <int NT>
+template <int NT, int W>
 void launch_gemv_t(const GemmArgs& a, cudaStream_t stream) {
-  constexpr int smem = Gv<NT>::kSmem;
+  constexpr int smem = Gv<NT, W>::kSmem;
   static bool attr = false;
   if (!attr) {
-    cudaFuncSetAttribute(dual_lora_gemv_kernel<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaFuncSetAttribute(dual_lora_gemv_kernel<NT, W>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         smem);
     attr = true;
   }
   const unsigned grid = static_cast<unsigned>((a.N + 15) / 16);
-  launch_pdl(dual_lora_gemv_kernel<NT>, dim3(grid), dim3(32 * kGvWarps), smem, stream,
+  launch_pdl(dual_lora_gemv_kernel<NT, W>, dim3(grid), dim3(32 * W), smem, stream,
       static_cast<const __nv_bfloat16*>(a.x_off),
       static_cast<const __nv_bfloat16*>(a.shared_x ? a.x_off : a.x_on), static_cast<int>(a.M),
       static_cast<int>(a.K), static_cast<int>(a.N), static_cast<const __nv_bfloat16*>(a.W),
@@ -347,10 +352,22 @@ int launch_lora_down(const void* x, int64_t M, int64_t K, const void* A, int64_t
 
 int launch_dual_lora_gemv(const GemmArgs& a, cudaStream_t stream) {
   const int64_t rows = a.shared_x ? a.M : 2 * a.M;
-  if (rows <= 8)
-    launch_gemv_t<1>(a, stream);
-  else
-    launch_gemv_t<2>(a, stream);
+  int dev = 0, nsm = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return -1;
+  const bool narrow = (a.N + 15) / 16 >= 4LL * nsm;  // enough row blocks for 4-warp CTAs
+  if (rows <= 8) {
+    if (narrow)
+      launch_gemv_t<1, 4>(a, stream);
+    else
+      launch_gemv_t<1, 8>(a, stream);
+  } else {
+    if (narrow)
+      launch_gemv_t<2, 4>(a, stream);
+    else
+      launch_gemv_t<2, 8>(a, stream);
+  }
   return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
 }
 
