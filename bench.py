@@ -143,37 +143,28 @@ class LmHeadScoring:
         self.lengths = torch.from_numpy(self.lengths_np).to(device)
         self.score = torch.randn(S, device=device, generator=g)
         self.values = torch.randn(S, L, device=device, generator=g)
-        self.u = torch.empty(T, r, dtype=bf, device=device)
-        self.z_ref = torch.empty(T, V, device=device)
-        self.z_act = torch.empty(T, V, device=device)
+        # the fused LM head keeps per-tile log-softmax partials, never the logits
+        self.ws = torch.empty(H.lm_head_logprobs_workspace_size(S, L, V, r), dtype=torch.uint8,
+                              device=device)
         self.la, self.lr, self.rw = (torch.empty(T, device=device) for _ in range(3))
         self.adv = torch.empty(S, L, device=device)
         self.ret = torch.empty(S, L, device=device)
         self.units = int(self.lengths_np.sum())
-        self.launches_per_step = 4
-        # algorithmic work of each kernel per launch
+        self.launches_per_step = 4  # lora_down, GEMM with log-softmax epilogue, combine, GAE
+        self.event_names = ("gemm", "gae")  # CUDA-event pairs recorded by step()
+        # algorithmic work per step: the LM head's flops (both heads, LoRA-up on the actor)
         self.gemm_flops = 2.0 * T * d * V + 2.0 * T * r * V
-        valid_rows = self.units
-        self.logp_bytes = valid_rows * V * 4 * 2 + T * (4 + 4 * 3) + S * 8
         self.gae_bytes = S * L * 16 + S * 4
-        self.down_bytes = T * d * 2 + r * d * 2 + T * r * 2
 
     def step(self, ev=None):
         H = self.H
         if ev:
-            ev["down"][0].record()
-        H.hydra_lora_down(self.h, self.A, self.s, self.u)
-        if ev:
-            ev["down"][1].record()
             ev["gemm"][0].record()
-        H.hydra_dual_linear(self.h, None, self.W, self.u, self.B, self.z_ref, self.z_act)
+        H.hydra_lm_head_logprobs(self.h, None, self.W, self.A, self.B, self.s, self.ids,
+                                 self.lengths, self.score, self.beta, self.S, self.L, self.la,
+                                 self.lr, self.rw, self.ws)
         if ev:
             ev["gemm"][1].record()
-            ev["logp"][0].record()
-        H.hydra_token_logprobs_kl(self.z_act, self.z_ref, self.ids, self.lengths, self.score,
-                                  self.beta, self.S, self.L, self.la, self.lr, self.rw)
-        if ev:
-            ev["logp"][1].record()
             ev["gae"][0].record()
         H.ppo_gae(self.rw.view(self.S, self.L), self.values, self.lengths, self.gamma, self.lam,
                   self.adv, self.ret)
@@ -207,25 +198,27 @@ class LmHeadScoring:
     def kernels(self, peaks, ms):
         """Per-kernel achieved throughput from mean event times (ms per launch)."""
         return {
-            "dual_lora_gemm_tcgen05": {"ms": ms["gemm"], "TFLOP/s": self.gemm_flops / ms["gemm"] / 1e9},
-            "logsoftmax_gather_kl": {"ms": ms["logp"], "GB/s": self.logp_bytes / ms["logp"] / 1e6},
+            "lm_head_logprobs_fused": {"ms": ms["gemm"], "TFLOP/s": self.gemm_flops / ms["gemm"] / 1e9,
+                                       "covers": "lora_down + tcgen05 LM head with log-softmax "
+                                                 "epilogue + partial combine"},
             "gae_reverse_scan": {"ms": ms["gae"], "GB/s": self.gae_bytes / ms["gae"] / 1e6},
-            "lora_down": {"ms": ms["down"], "GB/s": self.down_bytes / ms["down"] / 1e6},
         }
 
     def roofline(self, peaks, ms):
         achieved = self.gemm_flops / ms["gemm"] / 1e9
         peak = peaks["bf16_tflops_sustained"]
-        return {"kernel": "dual_lora_gemm_tcgen05", "bound": "tensor", "achieved": achieved,
+        return {"kernel": "dual_lora_gemm_tcgen05 with the log-softmax epilogue (timed with its "
+                          "lora_down and combine)", "bound": "tensor", "achieved": achieved,
                 "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak, "traffic": None,
                 "peak_kind": f"bf16 dense, {peaks['source']} sustained"}
 
     def config(self):
         return {"workload": "lm_head_scoring: h[4x512x4096] -> dual LM head 4096->32000 (LoRA r=16, "
-                            "s=2, fp32 logits) -> logp/KL (beta 0.1) -> GAE (gamma 1, lambda 0.95)",
+                            "s=2) with the log-softmax reduced in the GEMM epilogue (no logits "
+                            "stored) -> logp/KL (beta 0.1) -> GAE (gamma 1, lambda 0.95)",
                 "batch": self.S, "response_len": self.L, "lengths": "U[64,512]",
                 "scored_tokens_per_step": self.units, "l2": "inputs larger than L2 "
-                "(W_lm 262 MB, logits 2 x 262 MB)"}
+                "(W_lm 262 MB)"}
 
     # ---- CPU oracle on a bounded sample of the same workload
     def oracle_sample(self, n_rows):
@@ -293,7 +286,8 @@ class HydraScoringLlama7B:
         }
         self.gemm_flops = sum(self.class_flops.values())
         self.attn_flops = c["n_layers"] * 2 * self.S * c["n_heads"] * 2 * P * P * 128  # causal half
-        self.logp_bytes = SL * V * 4 * 2 + SL * 16
+        # the log-probability class is the combine of the LM head's per-tile partials
+        self.logp_bytes = SL * (2 * ((V + 255) // 256) * 8 + 2 * 4 + 4 + 12)
         self.launches_per_step = None
 
     def step(self, ev=None):
@@ -689,7 +683,7 @@ def run_ours(args, wl_cls):
         raise RuntimeError("device error during warm-up")
 
     driver = isinstance(wl, HydraScoringLlama7B)
-    names = ("down", "gemm", "logp", "gae")
+    names = getattr(wl, "event_names", ())
     evs = [None] * steps
     if driver:
         # launch counts of one pass, then event timing of every launch of the timed steps

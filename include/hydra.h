@@ -242,6 +242,33 @@ hydra_status hydra_token_logprobs_kl(const void* logits_actor, const void* logit
                                      float* lse_ref, void* stream);
 
 /*
+ * The dual LM head and the log-probabilities in one pass, without materialising logits:
+ * equal to hydra_lora_linear(h_off, h_on, ..., W_lm, A, B, r, s, z_ref, z_actor, HYDRA_F32)
+ * followed by hydra_token_logprobs_kl(z_actor, z_ref, ...), up to the fp32 summation order.
+ * The tcgen05 GEMM's epilogue reduces each [row x 256-column] logit tile to a (max, sum exp)
+ * pair and keeps the sampled token's logit; a second kernel merges the pairs into lse.
+ * Arguments:
+ *   h_off, h_on : bf16 [S*L, d] final hidden states of the reference (LoRA off) and actor
+ *           (LoRA on) streams; h_on == h_off or NULL when they share the input.
+ *   W : bf16 [V, d] LM head. A [r, d], B [V, r], r, s : LoRA of the actor head (r == 0: none).
+ *   ids, lengths, seq_score, beta, logp_actor, logp_ref, reward_tok, lse_actor, lse_ref : as
+ *           hydra_token_logprobs_kl with ids dense [S*L].
+ *   workspace : hydra_lm_head_logprobs_workspace_size(S, L, V, r) bytes, 16-byte aligned
+ *           (per-tile partials, sampled-token logits and u).
+ * Errors: NULL required pointer -> HYDRA_ERR_NULL; d, V, r not multiples of 8 or a
+ * misaligned pointer -> HYDRA_ERR_ALIGN; d < 8, V < 8, r > 256, S*L >= 2^31 ->
+ * HYDRA_ERR_SHAPE; small workspace -> HYDRA_ERR_WORKSPACE. S*L == 0 is a no-op.
+ */
+size_t hydra_lm_head_logprobs_workspace_size(int64_t S, int64_t L, int64_t V, int64_t r);
+hydra_status hydra_lm_head_logprobs(const void* h_off, const void* h_on, int64_t S, int64_t L,
+                                    int64_t d, int64_t V, const void* W, const void* A,
+                                    const void* B, int64_t r, float s, const int32_t* ids,
+                                    const int32_t* lengths, const float* seq_score, float beta,
+                                    float* logp_actor, float* logp_ref, float* reward_tok,
+                                    float* lse_actor, float* lse_ref, void* workspace,
+                                    size_t workspace_bytes, void* stream);
+
+/*
  * Generalised advantage estimation over each sequence's valid tokens (§2: GAE uses
  * V(x, y) to build the advantage estimates and the critic regresses the returns;
  * Appendix B: gamma = 1.0, lambda = 0.95):
@@ -352,8 +379,9 @@ size_t hydra_score_llama_workspace_size(const hydra_llama_config* cfg, int64_t S
  * log-probabilities and the reward; §3 Dynamic LoRA; J-Hydra uses one LoRA set for actor
  * and critic) over S sequences of P0 prompt + L response tokens:
  *   both streams through n_layers Llama blocks (q/v/gate/up/down carry LoRA, k/o/LM head
- *   do not) -> final RMSNorm -> LM head on the rows predicting response tokens ->
- *   logp_actor (LoRA on), logp_ref (LoRA off) -> score_s = w_rm . h_off[P0 + len_s - 1],
+ *   do not) -> final RMSNorm -> LM head on the rows predicting response tokens, reduced
+ *   in its epilogue to log-softmax partials (as hydra_lm_head_logprobs; no logits are
+ *   stored) -> logp_actor (LoRA on), logp_ref (LoRA off) -> score_s = w_rm . h_off[P0 + len_s - 1],
  *   values_t = w_rm . h_on[P0 + t - 1] -> reward_t = -beta (la - lr) + [t = len-1] score
  *   -> GAE advantages and returns.
  * ids int32 [S, P0 + L]; lengths int32 [S] valid response tokens (0..L) or NULL (all L).
@@ -373,7 +401,7 @@ enum {
   HYDRA_PROF_GEMM_O = 1,      /* o projection (+ residual add epilogue) */
   HYDRA_PROF_GEMM_GU = 2,     /* fused gate/up (+ SwiGLU epilogue) */
   HYDRA_PROF_GEMM_DOWN = 3,   /* down projection (+ residual add epilogue) */
-  HYDRA_PROF_GEMM_LMHEAD = 4, /* LM head, fp32 logits */
+  HYDRA_PROF_GEMM_LMHEAD = 4, /* LM head with the log-softmax partials in its epilogue */
   HYDRA_PROF_LORA_DOWN = 5,   /* u = s x A^T */
   HYDRA_PROF_ATTENTION = 6,   /* causal attention */
   HYDRA_PROF_ELEMENTWISE = 7, /* embedding, RMSNorm, RoPE */

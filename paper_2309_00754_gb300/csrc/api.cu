@@ -220,6 +220,76 @@ hydra_status hydra_dual_linear_rope(const void* x_off, const void* x_on, int64_t
                           true, kEpiRope, &rope);
 }
 
+size_t hydra_lm_head_logprobs_workspace_size(int64_t S, int64_t L, int64_t V, int64_t r) {
+  if (S < 0 || L < 0 || V < 1 || r < 0) return 0;
+  const size_t rows = static_cast<size_t>(S) * static_cast<size_t>(L);
+  const size_t nt = static_cast<size_t>((V + 255) / 256);
+  return round_up(2 * rows * nt * 8, 256) + round_up(2 * rows * 4, 256) +
+         round_up(rows * static_cast<size_t>(r) * 2, 256);
+}
+
+hydra_status hydra_lm_head_logprobs(const void* h_off, const void* h_on, int64_t S, int64_t L,
+                                    int64_t d, int64_t V, const void* W, const void* A,
+                                    const void* B, int64_t r, float s, const int32_t* ids,
+                                    const int32_t* lengths, const float* seq_score, float beta,
+                                    float* logp_actor, float* logp_ref, float* reward_tok,
+                                    float* lse_actor, float* lse_ref, void* workspace,
+                                    size_t workspace_bytes, void* stream) {
+  if (h_off == nullptr || W == nullptr || ids == nullptr || logp_actor == nullptr ||
+      logp_ref == nullptr || reward_tok == nullptr || workspace == nullptr)
+    return HYDRA_ERR_NULL;
+  if (S < 0 || L < 0 || d < 8 || V < 8 || r < 0 || r > 256) return HYDRA_ERR_SHAPE;
+  if (S * L >= (1LL << 31) || d >= (1LL << 31) || V >= (1LL << 31)) return HYDRA_ERR_SHAPE;
+  if (d % 8 != 0 || V % 8 != 0 || r % 8 != 0) return HYDRA_ERR_ALIGN;
+  const bool shared_x = (h_on == nullptr || h_on == h_off);
+  if (r > 0 && (A == nullptr || B == nullptr)) return HYDRA_ERR_NULL;
+  if (!aligned16(h_off) || (!shared_x && !aligned16(h_on)) || !aligned16(W) ||
+      !aligned16(workspace) || (r > 0 && (!aligned16(A) || !aligned16(B))))
+    return HYDRA_ERR_ALIGN;
+  if (workspace_bytes < hydra_lm_head_logprobs_workspace_size(S, L, V, r)) return HYDRA_ERR_WORKSPACE;
+  const int64_t M = S * L;
+  if (M == 0) return HYDRA_OK;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int* err = hydra::device_error_word();
+  if (err == nullptr) return HYDRA_ERR_CUDA;
+  // workspace: partials of both heads, sampled-token logits of both heads, u
+  const size_t nt = static_cast<size_t>((V + 255) / 256);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  float2* part = reinterpret_cast<float2*>(ws);
+  float* tgt = reinterpret_cast<float*>(ws + round_up(2 * static_cast<size_t>(M) * nt * 8, 256));
+  void* u = ws + round_up(2 * static_cast<size_t>(M) * nt * 8, 256) +
+            round_up(2 * static_cast<size_t>(M) * 4, 256);
+  const void* xo = shared_x ? h_off : h_on;
+  if (r > 0 && hydra::launch_lora_down(xo, M, d, A, r, s, u, st) != 0) return HYDRA_ERR_CUDA;
+  hydra::GemmArgs g;
+  g.x_off = h_off;
+  g.x_on = xo;
+  g.M = M;
+  g.K = d;
+  g.N = V;
+  g.W = W;
+  g.u = r > 0 ? u : nullptr;
+  g.B = r > 0 ? B : nullptr;
+  g.r = r;
+  g.shared_x = shared_x;
+  g.y_off = part;                                  // reference head (LoRA off)
+  g.y_on = part + static_cast<size_t>(M) * nt;     // actor head (LoRA on)
+  g.out_f32 = 1;
+  g.err = err;
+  g.epi = 4;
+  g.lsm_target = tgt;
+  g.lsm_ids = ids;
+  g.lsm_L = L;
+  g.lsm_ids_ld = L;
+  g.lsm_ids_off = 0;
+  if (hydra::launch_dual_lora_gemm_tc(g, st) != 0) return HYDRA_ERR_CUDA;
+  return hydra::launch_lse_combine(part, part + static_cast<size_t>(M) * nt, static_cast<int64_t>(nt),
+                                   tgt, tgt + M, S, L, V, ids, L, lengths, seq_score, beta,
+                                   logp_actor, logp_ref, reward_tok, lse_actor, lse_ref, err, st) == 0
+             ? HYDRA_OK
+             : HYDRA_ERR_CUDA;
+}
+
 hydra_status hydra_rope_table(int64_t P, int64_t head_dim, float theta, float* table,
                               void* stream) {
   if (table == nullptr) return HYDRA_ERR_NULL;

@@ -45,13 +45,20 @@ struct GemmArgs {
   void* y_on;         // [M, N] bf16 or fp32, may be NULL
   int out_f32;
   int* err;
-  int epi = 0;        // tcgen05 kernel epilogue: 0 store, 1 SwiGLU, 2 residual add (fp32), 3 rotary
+  int epi = 0;        // tcgen05 epilogue: 0 store, 1 SwiGLU, 2 residual add (fp32), 3 rotary,
+                      // 4 log-softmax partials
   bool single_cta = false;  // tcgen05: never use the CTA-pair (cta_group::2) kernel
   // epi 3 (rotary): columns [0, rope_cols) rotate in heads of 128 at position row % rope_P,
   // by the (cos, sin) pairs of rope_table [rope_P][64] (launch_rope_table)
   int64_t rope_P = 1;
   int64_t rope_cols = 0;
   const void* rope_table = nullptr;
+  // epi 4 (log-softmax partials): y_off / y_on are float2 [M][ceil(N / 256)] partial
+  // (max, sum exp) arrays, lsm_target float [2][M] the sampled-token logits, and the token of
+  // row m is lsm_ids[(m / lsm_L) * lsm_ids_ld + lsm_ids_off + m % lsm_L]
+  float* lsm_target = nullptr;
+  const int32_t* lsm_ids = nullptr;
+  int64_t lsm_L = 1, lsm_ids_ld = 1, lsm_ids_off = 0;
 };
 
 // Device address of the library's error word on the current device (NULL on failure).
@@ -66,6 +73,14 @@ int launch_dual_lora_gemv(const GemmArgs& a, cudaStream_t stream);
 int launch_lora_down(const void* x, int64_t M, int64_t K, const void* A, int64_t r, float s,
                      void* u, cudaStream_t stream);
 // ids of sequence s start at ids + s * ids_ld (ids_ld = L for a dense [S, L] array)
+// merge the per-tile (max, sum exp) partials [rows][n_tiles] (float2) of the reference and
+// actor heads and their sampled-token logits [rows] into logp / reward (as
+// launch_token_logprobs_kl); ids of sequence s start at ids + s * ids_ld
+int launch_lse_combine(const void* part_ref, const void* part_act, int64_t n_tiles,
+                       const float* tgt_ref, const float* tgt_act, int64_t S, int64_t L, int64_t V,
+                       const int32_t* ids, int64_t ids_ld, const int32_t* lengths,
+                       const float* score, float beta, float* la, float* lr, float* rew,
+                       float* lse_a, float* lse_r, int* err, cudaStream_t stream);
 int launch_token_logprobs_kl(const void* za, const void* zr, int bf16_logits, int64_t S, int64_t L,
                              int64_t V, int64_t ld, const int32_t* ids, int64_t ids_ld,
                              const int32_t* lengths,

@@ -183,7 +183,86 @@ int launch_t(const void* za, const void* zr, int64_t S, int64_t L, int64_t V, in
   return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
 }
 
+// One warp per token row: merges the row's per-tile (max, sum exp) partials of both heads,
+// written by the log-softmax epilogue of the LM-head GEMM (the logits never reach memory),
+// into lse_h, and emits logp_h = z_h[id] - lse_h and the reward exactly as
+// logprobs_kl_kernel does. Head 0 (part0, tgt0) is the reference (LoRA off), head 1 the actor.
+__global__ void __launch_bounds__(256)
+    lse_combine_kernel(const float2* __restrict__ part0, const float2* __restrict__ part1,
+                       int n_tiles, const float* __restrict__ tgt0, const float* __restrict__ tgt1,
+                       long long rows, int L, int V, const int32_t* __restrict__ ids,
+                       long long ids_ld, const int32_t* __restrict__ lengths,
+                       const float* __restrict__ score, float beta, float* __restrict__ la,
+                       float* __restrict__ lr, float* __restrict__ rew, float* __restrict__ lse_a,
+                       float* __restrict__ lse_r, int* err) {
+  const long long row = blockIdx.x * 8LL + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  const int s = static_cast<int>(row / L);
+  const int t = static_cast<int>(row - static_cast<long long>(s) * L);
+  int n = lengths ? lengths[s] : L;
+  if (n < 0 || n > L) {
+    if (lane == 0) record_error(err, kDevBadLength);
+    n = n < 0 ? 0 : L;
+  }
+  if (t >= n) {
+    if (lane == 0) {
+      la[row] = 0.f;
+      lr[row] = 0.f;
+      rew[row] = 0.f;
+      if (lse_a) lse_a[row] = 0.f;
+      if (lse_r) lse_r[row] = 0.f;
+    }
+    return;
+  }
+  float ma = -FLT_MAX, sa = 0.f, mr = -FLT_MAX, sr = 0.f;
+  for (int k = lane; k < n_tiles; k += 32) {
+    const float2 pr = part0[row * n_tiles + k], pa = part1[row * n_tiles + k];
+    merge(mr, sr, pr.x, pr.y);
+    merge(ma, sa, pa.x, pa.y);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    merge(ma, sa, __shfl_xor_sync(0xffffffffu, ma, off), __shfl_xor_sync(0xffffffffu, sa, off));
+    merge(mr, sr, __shfl_xor_sync(0xffffffffu, mr, off), __shfl_xor_sync(0xffffffffu, sr, off));
+  }
+  if (lane == 0) {
+    const float lsa = ma + logf(sa);
+    const float lsr = mr + logf(sr);
+    const int id = ids[static_cast<long long>(s) * ids_ld + t];
+    float va, vr, rw;
+    if (id < 0 || id >= V) {
+      record_error(err, kDevBadTokenId);
+      va = vr = rw = __int_as_float(0x7fc00000);
+    } else {
+      va = tgt1[row] - lsa;
+      vr = tgt0[row] - lsr;
+      rw = -beta * (va - vr);
+      if (score != nullptr && t == n - 1) rw += score[s];
+    }
+    la[row] = va;
+    lr[row] = vr;
+    rew[row] = rw;
+    if (lse_a) lse_a[row] = lsa;
+    if (lse_r) lse_r[row] = lsr;
+  }
+}
+
 }  // namespace
+
+int launch_lse_combine(const void* part_ref, const void* part_act, int64_t n_tiles,
+                       const float* tgt_ref, const float* tgt_act, int64_t S, int64_t L, int64_t V,
+                       const int32_t* ids, int64_t ids_ld, const int32_t* lengths,
+                       const float* score, float beta, float* la, float* lr, float* rew,
+                       float* lse_a, float* lse_r, int* err, cudaStream_t stream) {
+  const int64_t rows = S * L;
+  if (rows == 0) return 0;
+  lse_combine_kernel<<<static_cast<unsigned>((rows + 7) / 8), 256, 0, stream>>>(
+      static_cast<const float2*>(part_ref), static_cast<const float2*>(part_act),
+      static_cast<int>(n_tiles), tgt_ref, tgt_act, rows, static_cast<int>(L), static_cast<int>(V),
+      ids, ids_ld, lengths, score, beta, la, lr, rew, lse_a, lse_r, err);
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
+}
 
 int launch_token_logprobs_kl(const void* za, const void* zr, int bf16_logits, int64_t S, int64_t L,
                              int64_t V, int64_t ld, const int32_t* ids, int64_t ids_ld,

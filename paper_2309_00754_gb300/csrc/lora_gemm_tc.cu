@@ -22,6 +22,8 @@
 //    on stream run the main loop followed directly by the LoRA k-blocks
 //    ([x_on | u] [W | B]^T) and produce y_on. Off and on tiles of one (m, n) block are
 //    adjacent in the schedule, so each W tile comes from HBM once and again from L2.
+#include <float.h>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -52,7 +54,10 @@ constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN);
 //  EPI_RESIDUAL y (fp32 residual stream) += float(bf16(acc)) by TMA reduce-add in L2
 //  EPI_ROPE     y = bf16 rotary embedding of bf16(acc) on columns [0, rope_cols) (heads of
 //               128, rotate-half pairs (i, i + 64), position row % rope_P), bf16(acc) after
-enum { EPI_STORE = 0, EPI_SWIGLU = 1, EPI_RESIDUAL = 2, EPI_ROPE = 3 };
+//  EPI_LOGSOFTMAX  nothing stored per column: per (row, 256-column tile) the fp32 logits'
+//               (max, sum exp(z - max)) go to a partials array [rows][n_tiles] (float2), and
+//               the logit of the row's sampled token to targets [rows] if it is in the tile
+enum { EPI_STORE = 0, EPI_SWIGLU = 1, EPI_RESIDUAL = 2, EPI_ROPE = 3, EPI_LOGSOFTMAX = 4 };
 
 struct Params {
   int M, N, K;
@@ -69,6 +74,12 @@ struct Params {
   int bn;          // tile width in output columns (multiple of 16; 256 for the single-CTA kernel)
   int rope_P, rope_cols;
   const float2* rope_table;  // (cos, sin) [rope_P][64]
+  // EPI_LOGSOFTMAX: y_off_ptr / y_on_ptr are the two streams' partials [M][n_tiles]; the
+  // streams' targets are lsm_target [2][M]; the token of row m is
+  // lsm_ids[(m / lsm_L) * lsm_ids_ld + lsm_ids_off + m % lsm_L]
+  float* lsm_target;
+  const int32_t* lsm_ids;
+  int lsm_L, lsm_ids_ld, lsm_ids_off;
   void* y_off_ptr;  // the outputs as plain pointers, for columns past the last full store chunk
   void* y_on_ptr;
   int* err;
@@ -196,6 +207,61 @@ __device__ __forceinline__ void drain_rope(uint32_t lane_taddr, int lane, uint32
   }
 }
 
+// Log-softmax epilogue of one warp's 32 rows (thread `lane` owns row y + lane): the row's
+// fp32 logits in this tile, [n0, n0 + bn) clipped at N, reduce to an online (max, sum of
+// exp) pair (the normaliser of Milakov & Gimelshein, as the log-probability kernel keeps
+// it) written to partials[row][n0 / bn] of each requested stream; the logit of the row's
+// token goes to that stream's target if the token falls in the tile. part0 / part1 are the
+// streams' partial arrays (NULL: not requested).
+__device__ __forceinline__ void drain_logsoftmax(uint32_t lane_taddr, int lane, const Params& p,
+                                                 int y, int n0, void* part0, void* part1) {
+  const int row = y + lane;
+  const bool live = row < p.M;
+  int id = -1;
+  if (live) {
+    const int s = row / p.lsm_L, t = row - s * p.lsm_L;
+    id = p.lsm_ids[static_cast<int64_t>(s) * p.lsm_ids_ld + p.lsm_ids_off + t];
+  }
+  float m = -FLT_MAX, sum = 0.f, z = 0.f;
+  bool hit = false;
+  for (int c = 0; c < p.bn / 32; ++c) {
+    uint32_t v[32];
+    tc_ld_32x32b_x32(lane_taddr + 32 * c, v);
+    tc_wait_ld();
+    const int col0 = n0 + 32 * c;
+    if (col0 >= p.N) break;  // uniform over the warp
+    const int nv = min(32, p.N - col0);
+    float mx = -FLT_MAX;
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      if (j < nv) mx = fmaxf(mx, __uint_as_float(v[j]));
+    if (mx > m) {
+      sum *= __expf(m - mx);
+      m = mx;
+    }
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      if (j < nv) sum += __expf(__uint_as_float(v[j]) - m);
+    if (id >= col0 && id < col0 + nv) {
+      // arithmetic select (exact: every other term is +0), so v stays in registers
+      const int k = id - col0;
+      float acc = 0.f;
+#pragma unroll
+      for (int j = 0; j < 32; ++j) acc += (k == j) ? __uint_as_float(v[j]) : 0.f;
+      z = acc;
+      hit = true;
+    }
+  }
+  if (!live) return;
+  const int64_t slot = static_cast<int64_t>(row) * p.n_tiles + n0 / p.bn;
+  for (int o = 0; o < 2; ++o) {
+    float2* part = static_cast<float2*>(o == 0 ? part0 : part1);
+    if (part == nullptr) continue;
+    part[slot] = make_float2(m, sum);
+    if (hit) p.lsm_target[(part == p.y_on_ptr ? p.M : 0) + row] = z;
+  }
+}
+
 // Epilogue warp: drain the warp's 32 accumulator rows (TMEM lanes) of one tile to up to two
 // outputs. Each 128-byte-wide column chunk goes registers -> 128B-swizzled staging buffer
 // -> TMA store of a [32 rows x 128 B] box; two staging buffers alternate.
@@ -213,6 +279,10 @@ __device__ __forceinline__ void drain(uint32_t tmem_acc, int q, int lane, uint32
   const int y = m0 + q * 32;
   if (p.epi == EPI_ROPE) {
     drain_rope(lane_taddr, lane, staging, p, y, n0, t0, t1);
+    return;
+  }
+  if (p.epi == EPI_LOGSOFTMAX) {
+    drain_logsoftmax(lane_taddr, lane, p, y, n0, p0, p1);
     return;
   }
   for (int c = 0; c < nchunks; ++c) {
@@ -945,7 +1015,9 @@ static int sm_count() {
 // full ones (4096 output columns at 3072 rows per stream: 256 wide gives 5.05 waves, 224
 // wide exactly 6; measured +8 %). The SwiGLU epilogue needs 256 (128 gate + 128 up).
 static int pick_tile_width(const GemmArgs& a, int nclusters) {
-  if (a.epi == tcgemm::EPI_SWIGLU || a.epi == tcgemm::EPI_ROPE || nclusters < 1) return 256;
+  if (a.epi == tcgemm::EPI_SWIGLU || a.epi == tcgemm::EPI_ROPE || a.epi == tcgemm::EPI_LOGSOFTMAX ||
+      nclusters < 1)
+    return 256;
   const int64_t m_tiles = (a.M + 255) / 256;
   const int64_t streams = a.shared_x ? 1 : 2;
   int best = 256;
@@ -997,8 +1069,13 @@ int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream) {
   // output tensor: SwiGLU writes bf16 [M, N/2]; the residual mode adds into fp32 [M, N]
   const int64_t n_out = a.epi == tcgemm::EPI_SWIGLU ? a.N / 2 : a.N;
   const bool out32 = a.epi == tcgemm::EPI_RESIDUAL ? true : (a.epi == tcgemm::EPI_SWIGLU ? false : f32);
-  if (!make_map(&m_yoff, a.y_off ? a.y_off : any_y, a.M, n_out, 32, out32)) return -2;
-  if (!make_map(&m_yon, a.y_on ? a.y_on : any_y, a.M, n_out, 32, out32)) return -2;
+  if (a.epi == tcgemm::EPI_LOGSOFTMAX) {  // no per-column outputs: the maps are never used
+    m_yoff = m_xoff;
+    m_yon = m_xoff;
+  } else {
+    if (!make_map(&m_yoff, a.y_off ? a.y_off : any_y, a.M, n_out, 32, out32)) return -2;
+    if (!make_map(&m_yon, a.y_on ? a.y_on : any_y, a.M, n_out, 32, out32)) return -2;
+  }
 
   Params p;
   p.M = static_cast<int>(a.M);
@@ -1021,6 +1098,11 @@ int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream) {
   p.rope_P = static_cast<int>(a.rope_P < 1 ? 1 : a.rope_P);
   p.rope_cols = static_cast<int>(a.rope_cols);
   p.rope_table = static_cast<const float2*>(a.rope_table);
+  p.lsm_target = a.lsm_target;
+  p.lsm_ids = a.lsm_ids;
+  p.lsm_L = static_cast<int>(a.lsm_L < 1 ? 1 : a.lsm_L);
+  p.lsm_ids_ld = static_cast<int>(a.lsm_ids_ld);
+  p.lsm_ids_off = static_cast<int>(a.lsm_ids_off);
   p.y_off_ptr = a.y_off;
   p.y_on_ptr = a.y_on;
   p.err = a.err;

@@ -61,7 +61,7 @@ inline hydra_status rc(int r) { return r == 0 ? HYDRA_OK : HYDRA_ERR_CUDA; }
 
 // Workspace layout of the full pass, in bytes from the workspace base.
 struct PassLayout {
-  size_t h, a, qkv, attn, m, u, fin, logits, sc, rope, total;
+  size_t h, a, qkv, attn, m, u, fin, part, tgt, sc, rope, total;
 };
 
 PassLayout layout(const hydra_llama_config& c, int64_t S) {
@@ -79,7 +79,10 @@ PassLayout layout(const hydra_llama_config& c, int64_t S) {
   L.m = o;      o += up256(R * F * 2);
   L.u = o;      o += up256(T * 2 * static_cast<size_t>(c.lora_rank) * 2);
   L.fin = o;    o += up256(2 * SL * d * 2);
-  L.logits = o; o += up256(2 * SL * static_cast<size_t>(c.vocab) * 4);
+  // LM head: per-(row, 256-column tile) log-softmax partials and sampled-token logits of both
+  // heads (the logits themselves never reach memory)
+  L.part = o;   o += up256(2 * SL * static_cast<size_t>((c.vocab + 255) / 256) * 8);
+  L.tgt = o;    o += up256(2 * SL * 4);
   L.sc = o;     o += up256(static_cast<size_t>(S) * 4);
   L.rope = o;   o += up256(P * static_cast<size_t>(c.head_dim / 2) * 8);
   L.total = o;
@@ -293,7 +296,8 @@ hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_
   void* m = ws + Lo.m;
   void* u = ws + Lo.u;
   void* fin = ws + Lo.fin;
-  float* logits = reinterpret_cast<float*>(ws + Lo.logits);
+  float2* part = reinterpret_cast<float2*>(ws + Lo.part);
+  float* tgt = reinterpret_cast<float*>(ws + Lo.tgt);
   float* sc = reinterpret_cast<float*>(ws + Lo.sc);
   void* rope_table = ws + Lo.rope;
 
@@ -341,7 +345,32 @@ hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_
   // final norm on the rows that predict response tokens: row P0 - 1 + t of each sequence
   const hydra::RowMap resp{L, P, c.prompt_len - 1};
   HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(h, w->final_norm, 2 * SL, d, c.rms_eps, resp, fin, st));
-  HY_TRY(stacked_linear(HYDRA_PROF_GEMM_LMHEAD, fin, SL, d, V, w->lm_head, nullptr, nullptr, 0, s, u, logits, true, err, st));
+  // LM head of both streams with the log-softmax reduced in the GEMM epilogue
+  const int64_t nt = (V + 255) / 256;
+  const int32_t* resp_ids = ids + c.prompt_len;  // token of response row s * L + t: ids[s * P + P0 + t]
+  {
+    ProfScope ps(HYDRA_PROF_GEMM_LMHEAD, st);
+    hydra::GemmArgs g;
+    g.x_off = fin;
+    g.x_on = static_cast<const uint8_t*>(fin) + static_cast<size_t>(SL) * d * 2;
+    g.M = SL;
+    g.K = d;
+    g.N = V;
+    g.W = w->lm_head;
+    g.r = 0;
+    g.shared_x = false;
+    g.y_off = part;                                // reference head (LoRA off)
+    g.y_on = part + static_cast<size_t>(SL) * nt;  // actor head (LoRA on)
+    g.out_f32 = 1;
+    g.err = err;
+    g.epi = 4;
+    g.lsm_target = tgt;
+    g.lsm_ids = resp_ids;
+    g.lsm_L = L;
+    g.lsm_ids_ld = P;
+    g.lsm_ids_off = 0;
+    HY_TRY(hydra::launch_dual_lora_gemm_tc(g, st));
+  }
   // reward-model score on the LoRA-off stream at the last valid token; values on the
   // LoRA-on stream (the same head: r_phi = LO(V))
   HY_PROF(HYDRA_PROF_HEADS, hydra::launch_seq_score(h, w->final_norm, w->w_rm, d, c.rms_eps,
@@ -349,12 +378,10 @@ hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_
   const void* fin_on = static_cast<uint8_t*>(fin) + static_cast<size_t>(SL) * d * 2;
   const hydra::RowMap dense{SL, SL, 0};
   HY_PROF(HYDRA_PROF_HEADS, hydra::launch_head_dot(fin_on, d, w->w_rm, dense, SL, lengths, L, values, st));
-  const float* z_ref = logits;
-  const float* z_act = logits + static_cast<size_t>(SL) * V;
   HY_PROF(HYDRA_PROF_LOGPROBS,
-          hydra::launch_token_logprobs_kl(z_act, z_ref, 0, S, L, V, V, ids + c.prompt_len, P,
-                                          lengths, sc, c.beta, logp_actor, logp_ref, reward,
-                                          nullptr, nullptr, err, st));
+          hydra::launch_lse_combine(part, part + static_cast<size_t>(SL) * nt, nt, tgt, tgt + SL, S, L, V,
+                                    resp_ids, P, lengths, sc, c.beta, logp_actor, logp_ref, reward,
+                                    nullptr, nullptr, err, st));
   HY_PROF(HYDRA_PROF_GAE, hydra::launch_gae(reward, values, lengths, S, L, c.gamma, c.lam,
                                             advantages, returns, err, st));
   if (cudaMemcpyAsync(score, sc, static_cast<size_t>(S) * 4, cudaMemcpyDeviceToDevice, st) !=

@@ -40,6 +40,11 @@ _SIGNATURES = {
                                               _c_i64, _vp, _vp, _c_i64, _c_i64, _c_i64, _vp,
                                               _vp]),
     "hydra_rope_table": (ctypes.c_int, [_c_i64, _c_i64, ctypes.c_float, _vp, _vp]),
+    "hydra_lm_head_logprobs_workspace_size": (ctypes.c_size_t, [_c_i64, _c_i64, _c_i64, _c_i64]),
+    "hydra_lm_head_logprobs": (ctypes.c_int, [_vp, _vp, _c_i64, _c_i64, _c_i64, _c_i64, _vp, _vp,
+                                              _vp, _c_i64, ctypes.c_float, _vp, _vp, _vp,
+                                              ctypes.c_float, _vp, _vp, _vp, _vp, _vp, _vp,
+                                              ctypes.c_size_t, _vp]),
     "hydra_lora_linear_noalloc": (ctypes.c_int, [_vp, _vp, _c_i64, _c_i64, _c_i64, _vp, _vp, _vp,
                                                  _c_i64, ctypes.c_float, _vp, _vp, ctypes.c_int,
                                                  _vp]),
@@ -268,6 +273,31 @@ def hydra_dual_linear_rope(x_off, x_on, W, u, B, y_off, y_on, P, rope_cols, head
     _check("hydra_dual_linear_rope", load().hydra_dual_linear_rope(
         _p(x_off), _p(x_on), M, K, N, _p(W), _p(u), _p(B), r, _p(y_off), _p(y_on), int(P),
         int(rope_cols), int(head_dim), _p(table), _stream(stream)))
+
+
+def lm_head_logprobs_workspace_size(S, L, V, r):
+    return int(load().hydra_lm_head_logprobs_workspace_size(S, L, V, r))
+
+
+def hydra_lm_head_logprobs(h_off, h_on, W, A, B, s, ids, lengths, seq_score, beta, S, L,
+                           logp_actor, logp_ref, reward_tok, workspace, lse_actor=None,
+                           lse_ref=None, stream=None):
+    """Dual LM head + log-probabilities/KL without materialised logits. h_*: bf16 [S*L, d]
+    (h_on None: shared input); W bf16 [V, d]; A/B the actor head's LoRA (None: none)."""
+    for t, n in ((h_off, "h_off"), (h_on, "h_on"), (W, "W"), (A, "A"), (B, "B")):
+        _req(t, torch.bfloat16, n)
+    _req(ids, torch.int32, "ids")
+    _req(lengths, torch.int32, "lengths")
+    for t, n in ((seq_score, "seq_score"), (logp_actor, "logp_actor"), (logp_ref, "logp_ref"),
+                 (reward_tok, "reward_tok"), (lse_actor, "lse_actor"), (lse_ref, "lse_ref")):
+        _req(t, torch.float32, n)
+    d = h_off.shape[1]
+    V = W.shape[0]
+    r = 0 if A is None else A.shape[0]
+    _check("hydra_lm_head_logprobs", load().hydra_lm_head_logprobs(
+        _p(h_off), _p(h_on), S, L, d, V, _p(W), _p(A), _p(B), r, float(s), _p(ids), _p(lengths),
+        _p(seq_score), float(beta), _p(logp_actor), _p(logp_ref), _p(reward_tok), _p(lse_actor),
+        _p(lse_ref), _p(workspace), workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
 def hydra_token_logprobs_kl(logits_actor, logits_ref, ids, lengths, seq_score, beta, S, L,
