@@ -120,6 +120,28 @@ hydra_status hydra_dual_linear(const void* x_off, const void* x_on, int64_t M, i
                                int64_t N, const void* W, const void* u, const void* B, int64_t r,
                                void* y_off, void* y_on, int out_dtype, int algo, void* stream);
 
+/*
+ * Hydra-PPO's three streams through one frozen weight (Algorithm 2: the critic LoRA gives
+ * the values, LoRA off the reward and reference log-probabilities, the actor LoRA the policy;
+ * §3 Stage 2: two LoRA sets on one base model):
+ *     y_off  = x_off  W^T
+ *     y_act  = x_act  W^T + u_a B_act^T,    u_a = s (x_act  A_act^T)  stored as bf16
+ *     y_crit = x_crit W^T + u_c B_crit^T,   u_c = s (x_crit A_crit^T) stored as bf16
+ * on the tcgen05 kernel with the three streams' tiles of one output block adjacent, so each W
+ * tile comes from HBM once and twice more from L2. Inputs may alias one another (the first
+ * layer of a pass); any output may be NULL (not all three), and a NULL output's LoRA set may
+ * be NULL. With A_crit = A_act, B_crit = B_act and x_crit = x_act, y_crit equals y_act bit
+ * for bit (J-Hydra's single LoRA set). Layouts, alignment and errors as hydra_lora_linear;
+ * workspace: hydra_lora_linear_tri_workspace_size(M, r) bytes (both u).
+ */
+size_t hydra_lora_linear_tri_workspace_size(int64_t M, int64_t r);
+hydra_status hydra_lora_linear_tri(const void* x_off, const void* x_act, const void* x_crit,
+                                   int64_t M, int64_t K, int64_t N, const void* W,
+                                   const void* A_act, const void* B_act, const void* A_crit,
+                                   const void* B_crit, int64_t r, float s, void* y_off,
+                                   void* y_act, void* y_crit, int out_dtype, void* workspace,
+                                   size_t workspace_bytes, void* stream);
+
 /* Epilogues of hydra_dual_linear_ex. */
 enum {
   HYDRA_EPI_STORE = 0,    /* y = result (bf16 or fp32), as hydra_dual_linear */

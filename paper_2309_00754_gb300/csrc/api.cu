@@ -220,6 +220,72 @@ hydra_status hydra_dual_linear_rope(const void* x_off, const void* x_on, int64_t
                           true, kEpiRope, &rope);
 }
 
+size_t hydra_lora_linear_tri_workspace_size(int64_t M, int64_t r) {
+  if (M <= 0 || r <= 0) return 0;
+  return 2 * round_up(static_cast<size_t>(M) * static_cast<size_t>(r) * 2, 256);
+}
+
+hydra_status hydra_lora_linear_tri(const void* x_off, const void* x_act, const void* x_crit,
+                                   int64_t M, int64_t K, int64_t N, const void* W,
+                                   const void* A_act, const void* B_act, const void* A_crit,
+                                   const void* B_crit, int64_t r, float s, void* y_off,
+                                   void* y_act, void* y_crit, int out_dtype, void* workspace,
+                                   size_t workspace_bytes, void* stream) {
+  if (x_off == nullptr || x_act == nullptr || x_crit == nullptr || W == nullptr)
+    return HYDRA_ERR_NULL;
+  if (y_off == nullptr && y_act == nullptr && y_crit == nullptr) return HYDRA_ERR_NULL;
+  if (out_dtype != HYDRA_BF16 && out_dtype != HYDRA_F32) return HYDRA_ERR_RANGE;
+  if (M < 0 || K < 8 || N < 8 || M >= (1LL << 31) || K >= (1LL << 31) || N >= (1LL << 31))
+    return HYDRA_ERR_SHAPE;
+  if (K % 8 != 0 || N % 8 != 0) return HYDRA_ERR_ALIGN;
+  if (r < 0 || r > 256) return HYDRA_ERR_SHAPE;
+  if (r > 0 && r % 8 != 0) return HYDRA_ERR_ALIGN;
+  if (!aligned16(x_off) || !aligned16(x_act) || !aligned16(x_crit) || !aligned16(W) ||
+      !aligned16(y_off) || !aligned16(y_act) || !aligned16(y_crit))
+    return HYDRA_ERR_ALIGN;
+  const bool lora_a = r > 0 && y_act != nullptr, lora_c = r > 0 && y_crit != nullptr;
+  if ((lora_a && (A_act == nullptr || B_act == nullptr)) ||
+      (lora_c && (A_crit == nullptr || B_crit == nullptr)))
+    return HYDRA_ERR_NULL;
+  if ((lora_a && (!aligned16(A_act) || !aligned16(B_act))) ||
+      (lora_c && (!aligned16(A_crit) || !aligned16(B_crit))))
+    return HYDRA_ERR_ALIGN;
+  if (lora_a || lora_c) {
+    if (workspace == nullptr) return HYDRA_ERR_WORKSPACE;
+    if (!aligned16(workspace)) return HYDRA_ERR_ALIGN;
+    if (workspace_bytes < hydra_lora_linear_tri_workspace_size(M, r)) return HYDRA_ERR_WORKSPACE;
+  }
+  if (M == 0) return HYDRA_OK;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int* err = hydra::device_error_word();
+  if (err == nullptr) return HYDRA_ERR_CUDA;
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  void* u_a = ws;
+  void* u_c = lora_a || lora_c ? ws + round_up(static_cast<size_t>(M) * r * 2, 256) : nullptr;
+  if (lora_a && hydra::launch_lora_down(x_act, M, K, A_act, r, s, u_a, st) != 0) return HYDRA_ERR_CUDA;
+  if (lora_c && hydra::launch_lora_down(x_crit, M, K, A_crit, r, s, u_c, st) != 0) return HYDRA_ERR_CUDA;
+  hydra::GemmArgs g;
+  g.x_off = x_off;
+  g.x_on = x_act;
+  g.x_crit = x_crit;
+  g.M = M;
+  g.K = K;
+  g.N = N;
+  g.W = W;
+  g.u = lora_a ? u_a : nullptr;
+  g.B = lora_a ? B_act : nullptr;
+  g.u_crit = lora_c ? u_c : nullptr;
+  g.B_crit = lora_c ? B_crit : nullptr;
+  g.r = (lora_a || lora_c) ? r : 0;
+  g.shared_x = false;
+  g.y_off = y_off;
+  g.y_on = y_act;
+  g.y_crit = y_crit;
+  g.out_f32 = out_dtype == HYDRA_F32 ? 1 : 0;
+  g.err = err;
+  return hydra::launch_dual_lora_gemm_tc(g, st) == 0 ? HYDRA_OK : HYDRA_ERR_CUDA;
+}
+
 size_t hydra_lm_head_logprobs_workspace_size(int64_t S, int64_t L, int64_t V, int64_t r) {
   if (S < 0 || L < 0 || V < 1 || r < 0) return 0;
   const size_t rows = static_cast<size_t>(S) * static_cast<size_t>(L);

@@ -45,6 +45,12 @@ struct GemmArgs {
   void* y_on;         // [M, N] bf16 or fp32, may be NULL
   int out_f32;
   int* err;
+  // third stream (Hydra-PPO critic): input, LoRA operands (same r as the on stream) and
+  // output; NULL x_crit means two streams
+  const void* x_crit = nullptr;
+  const void* u_crit = nullptr;
+  const void* B_crit = nullptr;
+  void* y_crit = nullptr;
   int epi = 0;        // tcgen05 epilogue: 0 store, 1 SwiGLU, 2 residual add (fp32), 3 rotary,
                       // 4 log-softmax partials
   bool single_cta = false;  // tcgen05: never use the CTA-pair (cta_group::2) kernel

@@ -69,7 +69,7 @@ struct Params {
   int deferred;   // shared input with LoRA and both outputs: y_off drain, then LoRA
   int streams;    // 1 (shared) or 2 (stacked)
   int m_tiles, n_tiles, total_tiles;
-  int has_off, has_on;
+  int has_off, has_on, has_crit;
   int out_f32;
   int bn;          // tile width in output columns (multiple of 16; 256 for the single-CTA kernel)
   int rope_P, rope_cols;
@@ -82,7 +82,18 @@ struct Params {
   int lsm_L, lsm_ids_ld, lsm_ids_off;
   void* y_off_ptr;  // the outputs as plain pointers, for columns past the last full store chunk
   void* y_on_ptr;
+  void* y_crit_ptr;
   int* err;
+};
+
+// The kernel's TMA descriptors: inputs of the off, on (actor) and critic streams, W, the
+// LoRA operands (u, B) of the on and critic streams, and the three streams' outputs.
+struct Maps {
+  CUtensorMap x[3];
+  CUtensorMap w;
+  CUtensorMap u[2];
+  CUtensorMap b[2];
+  CUtensorMap y[3];
 };
 
 struct Tile {
@@ -95,8 +106,10 @@ __device__ __forceinline__ Tile decode(const Params& p, int t) {
   t /= p.streams;
   tl.m0 = (t % p.m_tiles) * BM;
   tl.n0 = (t / p.m_tiles) * p.bn;
-  const bool on = p.shared_x ? true : (tl.stream == 1);
-  tl.n_lora = (p.kb_lora > 0 && on && p.has_on) ? p.kb_lora : 0;
+  // stream 0 is LoRA-off; stream 1 carries the on (actor) LoRA set, stream 2 the critic set
+  const bool lora = p.shared_x ? true : (tl.stream >= 1);
+  const bool wanted = tl.stream == 2 ? p.has_crit : p.has_on;
+  tl.n_lora = (p.kb_lora > 0 && lora && wanted) ? p.kb_lora : 0;
   return tl;
 }
 
@@ -396,13 +409,7 @@ __device__ __forceinline__ void drain(uint32_t tmem_acc, int q, int lane, uint32
 }
 
 __global__ void __launch_bounds__(NUM_THREADS, 1)
-    dual_lora_gemm_kernel(const __grid_constant__ CUtensorMap tm_x_off,
-                          const __grid_constant__ CUtensorMap tm_x_on,
-                          const __grid_constant__ CUtensorMap tm_w,
-                          const __grid_constant__ CUtensorMap tm_u,
-                          const __grid_constant__ CUtensorMap tm_b,
-                          const __grid_constant__ CUtensorMap tm_y_off,
-                          const __grid_constant__ CUtensorMap tm_y_on, const Params p) {
+    dual_lora_gemm_kernel(const __grid_constant__ Maps mp, const Params p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -451,11 +458,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer (whole warp)
     if (elect_one()) {
-      tma_prefetch_desc(&tm_x_off);
-      tma_prefetch_desc(&tm_x_on);
-      tma_prefetch_desc(&tm_w);
-      tma_prefetch_desc(&tm_u);
-      tma_prefetch_desc(&tm_b);
+      for (int i = 0; i < 3; ++i) tma_prefetch_desc(&mp.x[i]);
+      tma_prefetch_desc(&mp.w);
+      for (int i = 0; i < 2; ++i) {
+        tma_prefetch_desc(&mp.u[i]);
+        tma_prefetch_desc(&mp.b[i]);
+      }
     }
     __syncwarp();
     int it = 0;
@@ -479,21 +487,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     Tile prev{0, 0, 0, 0};
     for (int j = 0; j < n_local && ok; ++j) {
       const Tile tl = decode(p, blockIdx.x + j * gridDim.x);
-      const CUtensorMap* tmx = (tl.stream == 1) ? &tm_x_on : &tm_x_off;
+      const CUtensorMap* tmx = &mp.x[tl.stream];
       for (int kb = 0; kb < p.kb_main && ok; ++kb) {
-        load(tmx, kb * BK, tl.m0, &tm_w, kb * BK, tl.n0);
+        load(tmx, kb * BK, tl.m0, &mp.w, kb * BK, tl.n0);
         if (p.deferred && j > 0 && kb == defer_at)
           for (int kl = 0; kl < prev.n_lora && ok; ++kl)
-            load(&tm_u, kl * BK, prev.m0, &tm_b, kl * BK, prev.n0);
+            load(&mp.u[prev.stream == 2 ? 1 : 0], kl * BK, prev.m0, &mp.b[prev.stream == 2 ? 1 : 0], kl * BK, prev.n0);
       }
       if (!p.deferred)
         for (int kl = 0; kl < tl.n_lora && ok; ++kl)
-          load(&tm_u, kl * BK, tl.m0, &tm_b, kl * BK, tl.n0);
+          load(&mp.u[tl.stream == 2 ? 1 : 0], kl * BK, tl.m0, &mp.b[tl.stream == 2 ? 1 : 0], kl * BK, tl.n0);
       prev = tl;
     }
     if (p.deferred && n_local > 0)
       for (int kl = 0; kl < prev.n_lora && ok; ++kl)
-        load(&tm_u, kl * BK, prev.m0, &tm_b, kl * BK, prev.n0);
+        load(&mp.u[prev.stream == 2 ? 1 : 0], kl * BK, prev.m0, &mp.b[prev.stream == 2 ? 1 : 0], kl * BK, prev.n0);
     // copies still in flight must land before the CTA's shared memory is released
     for (int k = (it > STAGES ? it - STAGES : 0); k < it; ++k) {
       volatile int no_abort = 0;
@@ -567,13 +575,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const int q = warp & 3;
     const uint32_t staging = smem_u32(staging_base) + (warp - 2) * 2 * STAGING_BYTES;
     uint32_t chunk_ctr = 0;
-    const CUtensorMap* y_off = p.has_off ? &tm_y_off : nullptr;
-    const CUtensorMap* y_on = p.has_on ? &tm_y_on : nullptr;
+    const CUtensorMap* y_off = p.has_off ? &mp.y[0] : nullptr;
+    const CUtensorMap* y_on = p.has_on ? &mp.y[1] : nullptr;
+    const CUtensorMap* y_crit = p.has_crit ? &mp.y[2] : nullptr;
     void* py_off = p.has_off ? p.y_off_ptr : nullptr;
     void* py_on = p.has_on ? p.y_on_ptr : nullptr;
+    void* py_crit = p.has_crit ? p.y_crit_ptr : nullptr;
     if (lane == 0) {
-      tma_prefetch_desc(&tm_y_off);
-      tma_prefetch_desc(&tm_y_on);
+      for (int i = 0; i < 3; ++i) tma_prefetch_desc(&mp.y[i]);
     }
     for (int j = 0; j < n_local; ++j) {
       const Tile tl = decode(p, blockIdx.x + j * gridDim.x);
@@ -596,8 +605,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, tl.n_lora > 0 ? nullptr : y_off, y_on,
                 tl.n_lora > 0 ? nullptr : py_off, py_on);
         else
-          drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, tl.stream == 1 ? y_on : y_off,
-                nullptr, tl.stream == 1 ? py_on : py_off, nullptr);
+          drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0,
+                tl.stream == 0 ? y_off : (tl.stream == 1 ? y_on : y_crit), nullptr,
+                tl.stream == 0 ? py_off : (tl.stream == 1 ? py_on : py_crit), nullptr);
       }
       tc_fence_before();
       mbar_arrive(acc_empty(b));
@@ -709,13 +719,7 @@ __device__ __forceinline__ void tc_commit_pair(uint32_t bar) {
 }
 
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
-    dual_lora_gemm_2cta_kernel(const __grid_constant__ CUtensorMap tm_x_off,
-                               const __grid_constant__ CUtensorMap tm_x_on,
-                               const __grid_constant__ CUtensorMap tm_w,
-                               const __grid_constant__ CUtensorMap tm_u,
-                               const __grid_constant__ CUtensorMap tm_b,
-                               const __grid_constant__ CUtensorMap tm_y_off,
-                               const __grid_constant__ CUtensorMap tm_y_on, const Params p) {
+    dual_lora_gemm_2cta_kernel(const __grid_constant__ Maps mp, const Params p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -775,8 +779,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     t /= p.streams;
     tl.m0 = (t % p.m_tiles) * 256 + static_cast<int>(rank) * 128;
     tl.n0 = (t / p.m_tiles) * p.bn;
-    const bool on = p.shared_x ? true : (tl.stream == 1);
-    tl.n_lora = (p.kb_lora > 0 && on && p.has_on) ? p.kb_lora : 0;
+    const bool lora = p.shared_x ? true : (tl.stream >= 1);
+    const bool wanted = tl.stream == 2 ? p.has_crit : p.has_on;
+    tl.n_lora = (p.kb_lora > 0 && lora && wanted) ? p.kb_lora : 0;
     return tl;
   };
 
@@ -807,21 +812,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     Tile prev{0, 0, 0, 0};
     for (int j = 0; j < n_local && ok; ++j) {
       const Tile tl = decode2(cluster + j * nclusters);
-      const CUtensorMap* tmx = (tl.stream == 1) ? &tm_x_on : &tm_x_off;
+      const CUtensorMap* tmx = &mp.x[tl.stream];
       for (int kb = 0; kb < p.kb_main && ok; ++kb) {
-        load(tmx, kb * BK, tl.m0, &tm_w, kb * BK, tl.n0 + brow);
+        load(tmx, kb * BK, tl.m0, &mp.w, kb * BK, tl.n0 + brow);
         if (p.deferred && j > 0 && kb == defer_at)
           for (int kl = 0; kl < prev.n_lora && ok; ++kl)
-            load(&tm_u, kl * BK, prev.m0, &tm_b, kl * BK, prev.n0 + brow);
+            load(&mp.u[prev.stream == 2 ? 1 : 0], kl * BK, prev.m0, &mp.b[prev.stream == 2 ? 1 : 0], kl * BK, prev.n0 + brow);
       }
       if (!p.deferred)
         for (int kl = 0; kl < tl.n_lora && ok; ++kl)
-          load(&tm_u, kl * BK, tl.m0, &tm_b, kl * BK, tl.n0 + brow);
+          load(&mp.u[tl.stream == 2 ? 1 : 0], kl * BK, tl.m0, &mp.b[tl.stream == 2 ? 1 : 0], kl * BK, tl.n0 + brow);
       prev = tl;
     }
     if (p.deferred && n_local > 0)
       for (int kl = 0; kl < prev.n_lora && ok; ++kl)
-        load(&tm_u, kl * BK, prev.m0, &tm_b, kl * BK, prev.n0 + brow);
+        load(&mp.u[prev.stream == 2 ? 1 : 0], kl * BK, prev.m0, &mp.b[prev.stream == 2 ? 1 : 0], kl * BK, prev.n0 + brow);
     // this CTA's copies in flight must land before its shared memory is released: the
     // stage's empty barrier (committed after the MMAs that read it) covers them
     for (int k = (it > STAGES2 ? it - STAGES2 : 0); k < it; ++k) {
@@ -898,10 +903,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     const int q = warp & 3;
     const uint32_t staging = smem_u32(staging_base) + (warp - 2) * 2 * STAGING_BYTES;
     uint32_t chunk_ctr = 0;
-    const CUtensorMap* y_off = p.has_off ? &tm_y_off : nullptr;
-    const CUtensorMap* y_on = p.has_on ? &tm_y_on : nullptr;
+    const CUtensorMap* y_off = p.has_off ? &mp.y[0] : nullptr;
+    const CUtensorMap* y_on = p.has_on ? &mp.y[1] : nullptr;
+    const CUtensorMap* y_crit = p.has_crit ? &mp.y[2] : nullptr;
     void* py_off = p.has_off ? p.y_off_ptr : nullptr;
     void* py_on = p.has_on ? p.y_on_ptr : nullptr;
+    void* py_crit = p.has_crit ? p.y_crit_ptr : nullptr;
     const uint32_t leader_mid0 = map_to_rank(acc_mid(0), 0);
     const uint32_t leader_empty0 = map_to_rank(acc_empty(0), 0);
     auto signal = [&](uint32_t leader_bar0, int b) {
@@ -929,8 +936,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
           drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, tl.n_lora > 0 ? nullptr : y_off, y_on,
                 tl.n_lora > 0 ? nullptr : py_off, py_on);
         else
-          drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0, tl.stream == 1 ? y_on : y_off,
-                nullptr, tl.stream == 1 ? py_on : py_off, nullptr);
+          drain(acc, q, lane, staging, chunk_ctr, p, tl.m0, tl.n0,
+                tl.stream == 0 ? y_off : (tl.stream == 1 ? y_on : y_crit), nullptr,
+                tl.stream == 0 ? py_off : (tl.stream == 1 ? py_on : py_crit), nullptr);
       }
       tc_fence_before();
       signal(leader_empty0, b);
@@ -1019,7 +1027,7 @@ static int pick_tile_width(const GemmArgs& a, int nclusters) {
       nclusters < 1)
     return 256;
   const int64_t m_tiles = (a.M + 255) / 256;
-  const int64_t streams = a.shared_x ? 1 : 2;
+  const int64_t streams = a.shared_x ? 1 : (a.x_crit != nullptr ? 3 : 2);
   int best = 256;
   int64_t best_cost = INT64_MAX;
   for (int bn : {256, 240, 224, 208, 192}) {
@@ -1051,30 +1059,37 @@ int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream) {
   // 256-row CTA pairs once every stream has more than one 128-row tile of work
   const bool pair = a.M > BM && nsm >= 2 && !a.single_cta;
   const int bn = pair ? pick_tile_width(a, nsm / 2) : BN;
-  CUtensorMap m_xoff, m_xon, m_w, m_u, m_b, m_yoff, m_yon;
+  const bool tri = a.x_crit != nullptr && !a.shared_x;  // off, on and critic streams
+  Maps mp;
   const bool lora = a.r > 0;
   const bool f32 = a.out_f32 != 0;
-  if (!make_map(&m_xoff, a.x_off, a.M, a.K, BM, false)) return -2;
-  if (!make_map(&m_xon, a.shared_x ? a.x_off : a.x_on, a.M, a.K, BM, false)) return -2;
+  if (!make_map(&mp.x[0], a.x_off, a.M, a.K, BM, false)) return -2;
+  if (!make_map(&mp.x[1], a.shared_x ? a.x_off : a.x_on, a.M, a.K, BM, false)) return -2;
+  if (!make_map(&mp.x[2], tri ? a.x_crit : a.x_off, a.M, a.K, BM, false)) return -2;
   const int brows = pair ? bn / 2 : BN;  // a CTA of a pair loads half of the tile's W rows
-  if (!make_map(&m_w, a.W, a.N, a.K, brows, false)) return -2;
-  if (lora) {
-    if (!make_map(&m_u, a.u, a.M, a.r, BM, false)) return -2;
-    if (!make_map(&m_b, a.B, a.N, a.r, brows, false)) return -2;
-  } else {
-    m_u = m_xoff;
-    m_b = m_w;
+  if (!make_map(&mp.w, a.W, a.N, a.K, brows, false)) return -2;
+  for (int i = 0; i < 2; ++i) {
+    const void* u = i == 0 ? a.u : a.u_crit;
+    const void* B = i == 0 ? a.B : a.B_crit;
+    if (lora && u != nullptr && B != nullptr) {
+      if (!make_map(&mp.u[i], u, a.M, a.r, BM, false)) return -2;
+      if (!make_map(&mp.b[i], B, a.N, a.r, brows, false)) return -2;
+    } else {  // never read
+      mp.u[i] = mp.x[0];
+      mp.b[i] = mp.w;
+    }
   }
-  const void* any_y = a.y_off ? a.y_off : a.y_on;
+  const void* any_y = a.y_off ? a.y_off : (a.y_on ? a.y_on : a.y_crit);
   // output tensor: SwiGLU writes bf16 [M, N/2]; the residual mode adds into fp32 [M, N]
   const int64_t n_out = a.epi == tcgemm::EPI_SWIGLU ? a.N / 2 : a.N;
   const bool out32 = a.epi == tcgemm::EPI_RESIDUAL ? true : (a.epi == tcgemm::EPI_SWIGLU ? false : f32);
-  if (a.epi == tcgemm::EPI_LOGSOFTMAX) {  // no per-column outputs: the maps are never used
-    m_yoff = m_xoff;
-    m_yon = m_xoff;
-  } else {
-    if (!make_map(&m_yoff, a.y_off ? a.y_off : any_y, a.M, n_out, 32, out32)) return -2;
-    if (!make_map(&m_yon, a.y_on ? a.y_on : any_y, a.M, n_out, 32, out32)) return -2;
+  for (int i = 0; i < 3; ++i) {
+    void* y = i == 0 ? a.y_off : (i == 1 ? a.y_on : a.y_crit);
+    if (a.epi == tcgemm::EPI_LOGSOFTMAX) {  // no per-column outputs: the maps are never used
+      mp.y[i] = mp.x[0];
+    } else if (!make_map(&mp.y[i], y ? y : any_y, a.M, n_out, 32, out32)) {
+      return -2;
+    }
   }
 
   Params p;
@@ -1088,8 +1103,9 @@ int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream) {
   p.shared_x = a.shared_x ? 1 : 0;
   p.has_off = a.y_off != nullptr;
   p.has_on = a.y_on != nullptr;
+  p.has_crit = tri && a.y_crit != nullptr && (!lora || (a.u_crit != nullptr && a.B_crit != nullptr));
   p.deferred = (p.shared_x && lora && p.has_off && p.has_on) ? 1 : 0;
-  p.streams = a.shared_x ? 1 : 2;
+  p.streams = a.shared_x ? 1 : (tri ? 3 : 2);
   p.m_tiles = static_cast<int>(pair ? (a.M + 255) / 256 : (a.M + BM - 1) / BM);
   p.n_tiles = static_cast<int>((a.N + bn - 1) / bn);
   p.total_tiles = p.m_tiles * p.n_tiles * p.streams;
@@ -1105,18 +1121,17 @@ int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream) {
   p.lsm_ids_off = static_cast<int>(a.lsm_ids_off);
   p.y_off_ptr = a.y_off;
   p.y_on_ptr = a.y_on;
+  p.y_crit_ptr = a.y_crit;
   p.err = a.err;
   if (pair) {
     const int nclusters = nsm / 2;
     const unsigned grid =
         2u * static_cast<unsigned>(p.total_tiles < nclusters ? p.total_tiles : nclusters);
-    dual_lora_gemm_2cta_kernel<<<grid, NUM_THREADS, SMEM2_BYTES, stream>>>(
-        m_xoff, m_xon, m_w, m_u, m_b, m_yoff, m_yon, p);
+    dual_lora_gemm_2cta_kernel<<<grid, NUM_THREADS, SMEM2_BYTES, stream>>>(mp, p);
     return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
   }
   const unsigned grid = static_cast<unsigned>(p.total_tiles < nsm ? p.total_tiles : nsm);
-  dual_lora_gemm_kernel<<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(m_xoff, m_xon, m_w, m_u, m_b,
-                                                                   m_yoff, m_yon, p);
+  dual_lora_gemm_kernel<<<grid, NUM_THREADS, SMEM_BYTES, stream>>>(mp, p);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
 }
 

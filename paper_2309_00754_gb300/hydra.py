@@ -40,6 +40,10 @@ _SIGNATURES = {
                                               _c_i64, _vp, _vp, _c_i64, _c_i64, _c_i64, _vp,
                                               _vp]),
     "hydra_rope_table": (ctypes.c_int, [_c_i64, _c_i64, ctypes.c_float, _vp, _vp]),
+    "hydra_lora_linear_tri_workspace_size": (ctypes.c_size_t, [_c_i64, _c_i64]),
+    "hydra_lora_linear_tri": (ctypes.c_int, [_vp, _vp, _vp, _c_i64, _c_i64, _c_i64, _vp, _vp, _vp,
+                                             _vp, _vp, _c_i64, ctypes.c_float, _vp, _vp, _vp,
+                                             ctypes.c_int, _vp, ctypes.c_size_t, _vp]),
     "hydra_lm_head_logprobs_workspace_size": (ctypes.c_size_t, [_c_i64, _c_i64, _c_i64, _c_i64]),
     "hydra_lm_head_logprobs": (ctypes.c_int, [_vp, _vp, _c_i64, _c_i64, _c_i64, _c_i64, _vp, _vp,
                                               _vp, _c_i64, ctypes.c_float, _vp, _vp, _vp,
@@ -273,6 +277,31 @@ def hydra_dual_linear_rope(x_off, x_on, W, u, B, y_off, y_on, P, rope_cols, head
     _check("hydra_dual_linear_rope", load().hydra_dual_linear_rope(
         _p(x_off), _p(x_on), M, K, N, _p(W), _p(u), _p(B), r, _p(y_off), _p(y_on), int(P),
         int(rope_cols), int(head_dim), _p(table), _stream(stream)))
+
+
+def lora_linear_tri_workspace_size(M, r):
+    return int(load().hydra_lora_linear_tri_workspace_size(M, r))
+
+
+def hydra_lora_linear_tri(x_off, x_act, x_crit, W, A_act, B_act, A_crit, B_crit, s, y_off, y_act,
+                          y_crit, workspace=None, stream=None):
+    """Hydra-PPO's off / actor / critic streams through one W (two LoRA sets)."""
+    for t, n in ((x_off, "x_off"), (x_act, "x_act"), (x_crit, "x_crit"), (W, "W"),
+                 (A_act, "A_act"), (B_act, "B_act"), (A_crit, "A_crit"), (B_crit, "B_crit")):
+        _req(t, torch.bfloat16, n)
+    out = next(t for t in (y_off, y_act, y_crit) if t is not None)
+    out_dtype = HYDRA_F32 if out.dtype == torch.float32 else HYDRA_BF16
+    for t, n in ((y_off, "y_off"), (y_act, "y_act"), (y_crit, "y_crit")):
+        _req(t, out.dtype, n)
+    M, K = x_off.shape
+    N = W.shape[0]
+    A = A_act if A_act is not None else A_crit
+    r = 0 if A is None else A.shape[0]
+    wsb = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check("hydra_lora_linear_tri", load().hydra_lora_linear_tri(
+        _p(x_off), _p(x_act), _p(x_crit), M, K, N, _p(W), _p(A_act), _p(B_act), _p(A_crit),
+        _p(B_crit), r, float(s), _p(y_off), _p(y_act), _p(y_crit), out_dtype, _p(workspace), wsb,
+        _stream(stream)))
 
 
 def lm_head_logprobs_workspace_size(S, L, V, r):

@@ -383,6 +383,48 @@ def test_rope_epilogue(M, shared):
         assert_rel(host_f64(y_dev), want, TOL_LINEAR, "rotary epilogue")
 
 
+@pytest.mark.parametrize("M,K,N,r,out", [(300, 328, 520, 16, torch.bfloat16),
+                                        (100, 256, 264, 8, torch.bfloat16),   # single-CTA tiles
+                                        (700, 1024, 1280, 16, torch.bfloat16),  # several tiles per pair
+                                        (260, 384, 4264, 16, torch.float32)])   # 240-wide pair tiles
+def test_hydra_three_streams(M, K, N, r, out):
+    """Hydra-PPO's off / actor / critic streams (two LoRA sets) through one W, against the
+    oracle's dual-output linear of each LoRA set."""
+    x, x2, W, A, Bm = _linear_problem(M, K, N, r, seed=61 + M)
+    x3 = synth.normal_bf16(611 + M, (M, K), 1.0)
+    A2 = synth.normal_bf16(612 + M, (r, K), 0.02)
+    B2 = synth.normal_bf16(613 + M, (N, r), 0.02)
+    ys = [torch.full((M, N), float("nan"), dtype=out, device="cuda") for _ in range(3)]
+    ws = torch.empty(max(1, H.lora_linear_tri_workspace_size(M, r)), dtype=torch.uint8, device="cuda")
+    H.hydra_lora_linear_tri(dev_bf16(x), dev_bf16(x2), dev_bf16(x3), dev_bf16(W), dev_bf16(A),
+                            dev_bf16(Bm), dev_bf16(A2), dev_bf16(B2), 2.0, ys[0], ys[1], ys[2], ws)
+    bf = out == torch.bfloat16
+    tol = TOL_LINEAR if bf else 1e-4
+    ref_off, ref_act = O.dual_lora_linear(f64(x), f64(x2), f64(W), f64(A), f64(Bm), 2.0, out_bf16=bf)
+    _, ref_crit = O.dual_lora_linear(f64(x), f64(x3), f64(W), f64(A2), f64(B2), 2.0, out_bf16=bf)
+    assert_rel(host_f64(ys[0]), ref_off, tol, "y_off")
+    assert_rel(host_f64(ys[1]), ref_act, tol, "y_act")
+    assert_rel(host_f64(ys[2]), ref_crit, tol, "y_crit")
+
+
+def test_hydra_three_streams_reduce_to_two():
+    """One LoRA set for actor and critic on one input (J-Hydra): the critic output equals the
+    actor output and both equal the two-stream kernel's, bit for bit; an absent output is
+    skipped."""
+    M, K, N, r = 300, 512, 776, 16
+    x, x2, W, A, Bm = _linear_problem(M, K, N, r, seed=71)
+    d = [dev_bf16(t) for t in (x, x2, W, A, Bm)]
+    ys = [torch.empty(M, N, dtype=torch.bfloat16, device="cuda") for _ in range(3)]
+    ws = torch.empty(H.lora_linear_tri_workspace_size(M, r), dtype=torch.uint8, device="cuda")
+    H.hydra_lora_linear_tri(d[0], d[1], d[1], d[2], d[3], d[4], d[3], d[4], 2.0, ys[0], ys[1], ys[2], ws)
+    two = _run_linear(d[0], d[1], d[2], d[3], d[4], 2.0, algo=1)
+    assert torch.equal(ys[2], ys[1]) and torch.equal(ys[1], two[1]) and torch.equal(ys[0], two[0])
+    crit_only = torch.empty(M, N, dtype=torch.bfloat16, device="cuda")
+    H.hydra_lora_linear_tri(d[0], d[1], d[1], d[2], None, None, d[3], d[4], 2.0, None, None,
+                            crit_only, ws)
+    assert torch.equal(crit_only, ys[2])
+
+
 def test_epilogue_argument_errors():
     x = torch.zeros(16, 64, dtype=torch.bfloat16, device="cuda")
     W = torch.zeros(200, 64, dtype=torch.bfloat16, device="cuda")
