@@ -35,8 +35,10 @@ Parity pins for every function live in tests/test_oracle_pins.py (closed forms,
 invariants, brute force, library routines, hand-worked fixtures in tests/golden/).
 `set_storage_dither` (off by default) is a sensitivity probe used to derive the end-to-end
 tolerance of the multi-layer composition; it never changes the default results.
-The full 32-layer Llama composition (`llama_score`) is pinned only through its per-op
-pieces and small-size invariants: parity unpinned for the composition as a whole.
+The full 32-layer Llama composition (`llama_score`, and the three-stream Hydra-PPO pass
+`llama_score_hydra`) is pinned only through its per-op pieces and small-size invariants
+(LoRA off, causality, one LoRA set reducing Hydra-PPO to J-Hydra-PPO, a critic set that
+moves only the values): parity unpinned for the composition as a whole.
 """
 from __future__ import annotations
 
@@ -338,4 +340,76 @@ def llama_score(weights, ids, prompt_len, cfg, seq_lengths=None, beta=0.1, gamma
         "returns": ret[0],
         "h_off": f_off,
         "h_on": f_on,
+    }
+
+
+def llama_score_hydra(weights, lora_critic, ids, prompt_len, cfg, seq_lengths=None, beta=0.1,
+                      gamma=1.0, lam=0.95, n_layers=None):
+    """One sequence of the Hydra-PPO scoring pass (Alg. 2 scoring steps): three streams of
+    the same frozen base model (§3 Stage 2: two LoRA sets on one base; dynamic LoRA):
+      off    LoRA ignored: reference log-probabilities and the reward score,
+      actor  the actor's LoRA set weights["lora"]: the policy log-probabilities,
+      critic the critic's LoRA set lora_critic: the values through the reward head,
+             r_phi <- LO(V), so V_t = w_rm . h_critic[p_t - 1].
+    weights, ids, prompt_len, cfg as llama_score; lora_critic has the layout of
+    weights["lora"]. Returns llama_score's outputs with values from the critic stream and
+    the final normed hidden states h_off, h_act, h_crit. With lora_critic equal to the
+    actor's set this is J-Hydra-PPO and the outputs equal llama_score's."""
+    d = cfg["d"]
+    H = cfg["n_heads"]
+    Dh = d // H
+    eps = cfg["eps"]
+    s = cfg["lora_scale"]
+    T = len(ids)
+    P = prompt_len
+    L = T - P
+    n_layers = cfg["n_layers"] if n_layers is None else n_layers
+    pos = np.arange(T)
+    sets = [None, weights["lora"], lora_critic]
+
+    def lin1(name, l, a, lora):
+        # one stream of the dual-output linear: no LoRA, or this stream's LoRA set
+        W = weights[name][l]
+        ab = None if lora is None else lora.get(name)
+        if ab is None:
+            return dual_lora_linear(a, a, W, None, None, s)[0]
+        return dual_lora_linear(a, a, W, ab[0][l], ab[1][l], s)[1]
+
+    h = [weights["embed"][np.asarray(ids)] for _ in range(3)]
+    for l in range(n_layers):
+        for i, lora in enumerate(sets):
+            a = round_bf16(rmsnorm(h[i], weights["norm1"][l], eps))
+            q = lin1("wq", l, a, lora)
+            k = lin1("wk", l, a, lora)
+            v = lin1("wv", l, a, lora)
+            qi = round_bf16(rope(q.reshape(T, H, Dh), pos, cfg["rope_theta"]))
+            ki = round_bf16(rope(k.reshape(T, H, Dh), pos, cfg["rope_theta"]))
+            att = round_bf16(causal_attention(qi, ki, v.reshape(T, H, Dh)).reshape(T, d))
+            h[i] = h[i] + lin1("wo", l, att, lora)
+            a = round_bf16(rmsnorm(h[i], weights["norm2"][l], eps))
+            m = round_bf16(swiglu(lin1("wg", l, a, lora), lin1("wu", l, a, lora)))
+            h[i] = h[i] + lin1("wd", l, m, lora)
+
+    f = [round_bf16(rmsnorm(hi, weights["final_norm"], eps)) for hi in h]
+    rows = np.arange(P - 1, T - 1)                       # hidden row predicting token P+t
+    resp_ids = np.asarray(ids)[P:]
+    lr, _ = log_softmax_gather(f[0][rows] @ weights["lm_head"].T, resp_ids)
+    la, _ = log_softmax_gather(f[1][rows] @ weights["lm_head"].T, resp_ids)
+    n = L if seq_lengths is None else int(seq_lengths)
+    score = float(f[0][P - 1 + n] @ weights["w_rm"]) if n > 0 else 0.0
+    values = f[2][rows] @ weights["w_rm"]
+    reward = kl_penalised_reward(la[None], lr[None], [n], [score], beta)[0]
+    adv, ret = gae(reward[None], values[None], [n], gamma, lam)
+    valid = np.arange(L) < n
+    return {
+        "logp_actor": np.where(valid, la, 0.0),
+        "logp_ref": np.where(valid, lr, 0.0),
+        "reward": reward,
+        "values": np.where(valid, values, 0.0),
+        "score": score,
+        "advantages": adv[0],
+        "returns": ret[0],
+        "h_off": f[0],
+        "h_act": f[1],
+        "h_crit": f[2],
     }

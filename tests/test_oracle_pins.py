@@ -388,3 +388,35 @@ def test_storage_dither_is_off_by_default_and_bounded():
     finally:
         O.set_storage_dither(0.0)
     assert np.array_equal(O.round_bf16(x), base)
+
+
+def test_hydra_ppo_one_lora_set_is_j_hydra():
+    """Hydra-PPO with the critic's LoRA set equal to the actor's is J-Hydra-PPO (§3: J-Hydra
+    uses one LoRA set for actor and critic): every output equals llama_score's exactly."""
+    w, cfg = tiny_llama()
+    ids = np.random.default_rng(16).integers(0, 64, size=12)
+    j = O.llama_score(w, ids, 4, cfg, seq_lengths=6)
+    h = O.llama_score_hydra(w, w["lora"], ids, 4, cfg, seq_lengths=6)
+    for k in ("logp_actor", "logp_ref", "reward", "values", "advantages", "returns"):
+        assert np.array_equal(h[k], j[k]), k
+    assert h["score"] == j["score"]
+    assert np.array_equal(h["h_crit"], j["h_on"]) and np.array_equal(h["h_act"], j["h_on"])
+
+
+def test_hydra_ppo_critic_stream_is_separate():
+    """The critic's LoRA set moves only the values: with its B = 0 the critic stream is the
+    LoRA-off stream (values = w_rm . h_off rows); a different critic set leaves the actor and
+    reference log-probabilities, the score and the reward unchanged."""
+    w, cfg = tiny_llama()
+    w0, _ = tiny_llama(zero_B=True)
+    ids = np.random.default_rng(17).integers(0, 64, size=12)
+    off_crit = O.llama_score_hydra(w, w0["lora"], ids, 4, cfg)
+    assert np.array_equal(off_crit["h_crit"], off_crit["h_off"])
+    rows = np.arange(3, 11)
+    assert np.array_equal(off_crit["values"], off_crit["h_off"][rows] @ w["w_rm"])
+    other, _ = tiny_llama(seed=99)
+    alt = O.llama_score_hydra(w, other["lora"], ids, 4, cfg)
+    for k in ("logp_actor", "logp_ref", "reward"):
+        assert np.array_equal(alt[k], off_crit[k]), k
+    assert alt["score"] == off_crit["score"]
+    assert np.max(np.abs(alt["values"] - off_crit["values"])) > 1e-6
