@@ -393,6 +393,18 @@ typedef struct hydra_llama_weights {
   const void* w_rm;                /* bf16 [d]: reward-model head; also the value head */
 } hydra_llama_weights;
 
+/* One LoRA set of a decoder layer in the fused layouts of hydra_llama_layer (the critic's
+ * set of Hydra-PPO): a_qv [2r, d] / b_qkv [3d, 2r] (q and v adapted, k not), a_gu [2r, d] /
+ * b_gu [2F, 2r] (interleaved gate/up rows), a_down [r, F] / b_down [d, r]. */
+typedef struct hydra_llama_lora {
+  const void* a_qv;
+  const void* b_qkv;
+  const void* a_gu;
+  const void* b_gu;
+  const void* a_down;
+  const void* b_down;
+} hydra_llama_lora;
+
 /* Workspace bytes of hydra_score_llama for S sequences. */
 size_t hydra_score_llama_workspace_size(const hydra_llama_config* cfg, int64_t S);
 
@@ -416,6 +428,25 @@ hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_
                                void* workspace, size_t workspace_bytes, float* logp_actor,
                                float* logp_ref, float* reward, float* values, float* advantages,
                                float* returns, float* score, void* stream);
+
+/*
+ * The Hydra-PPO scoring pass (Algorithm 2; §3 Stage 2: two LoRA sets on one base model):
+ * as hydra_score_llama with three stacked streams through every layer, each W read once for
+ * all three (hydra_lora_linear_tri): LoRA off (reference log-probabilities, reward score),
+ * the actor's LoRA set w->layers (logp_actor) and the critic's LoRA set critic[l] (a HOST
+ * array of n_layers entries, same rank r), whose final hidden states give the values through
+ * the reward head (r_phi <- LO(V)): values_t = w_rm . h_critic[P0 + t - 1]. With critic equal
+ * to the actor's LoRA pointers the outputs equal hydra_score_llama's (J-Hydra-PPO).
+ * Workspace: hydra_score_llama_hydra_workspace_size(cfg, S); other arguments and errors as
+ * hydra_score_llama; NULL critic -> HYDRA_ERR_NULL.
+ */
+size_t hydra_score_llama_hydra_workspace_size(const hydra_llama_config* cfg, int64_t S);
+hydra_status hydra_score_llama_hydra(const hydra_llama_config* cfg, const hydra_llama_weights* w,
+                                     const hydra_llama_lora* critic, const int32_t* ids,
+                                     const int32_t* lengths, int64_t S, void* workspace,
+                                     size_t workspace_bytes, float* logp_actor, float* logp_ref,
+                                     float* reward, float* values, float* advantages,
+                                     float* returns, float* score, void* stream);
 
 /* Kernel classes of the optional launch timing of hydra_score_llama. */
 enum {

@@ -64,10 +64,11 @@ struct PassLayout {
   size_t h, a, qkv, attn, m, u, fin, part, tgt, sc, rope, total;
 };
 
-PassLayout layout(const hydra_llama_config& c, int64_t S) {
+// ns stacked streams: 2 (J-Hydra: off, on) or 3 (Hydra-PPO: off, actor, critic)
+PassLayout layout(const hydra_llama_config& c, int64_t S, int ns = 2) {
   const size_t P = static_cast<size_t>(c.prompt_len + c.response_len);
   const size_t T = static_cast<size_t>(S) * P;
-  const size_t R = 2 * T;
+  const size_t R = static_cast<size_t>(ns) * T;
   const size_t d = static_cast<size_t>(c.d_model), F = static_cast<size_t>(c.ffn);
   const size_t SL = static_cast<size_t>(S) * static_cast<size_t>(c.response_len);
   PassLayout L;
@@ -77,8 +78,8 @@ PassLayout layout(const hydra_llama_config& c, int64_t S) {
   L.qkv = o;    o += up256(R * 3 * d * 2);
   L.attn = o;   o += up256(R * d * 2);
   L.m = o;      o += up256(R * F * 2);
-  L.u = o;      o += up256(T * 2 * static_cast<size_t>(c.lora_rank) * 2);
-  L.fin = o;    o += up256(2 * SL * d * 2);
+  L.u = o;      o += up256((ns - 1) * T * 2 * static_cast<size_t>(c.lora_rank) * 2);
+  L.fin = o;    o += up256(static_cast<size_t>(ns) * SL * d * 2);
   // LM head: per-(row, 256-column tile) log-softmax partials and sampled-token logits of both
   // heads (the logits themselves never reach memory)
   L.part = o;   o += up256(2 * SL * static_cast<size_t>((c.vocab + 255) / 256) * 8);
@@ -100,9 +101,11 @@ bool valid_config(const hydra_llama_config* c) {
   return true;
 }
 
-// stacked dual linear: rows [0, T) of x are the off stream, [T, 2T) the on stream
-// epi: tcgen05 epilogue; y is [2T, N] (store, rotary), [2T, N/2] bf16 (SwiGLU) or the fp32
-// residual stream [2T, N] (residual add); rope: rotary arguments of epi == kEpiRope
+// stacked linear of ns streams: rows [0, T) of x are the off stream, [T, 2T) the on
+// (actor) stream and, when ns == 3, [2T, 3T) the critic stream with its own LoRA set
+// (A2, B2; u2 receives its down-projection)
+// epi: tcgen05 epilogue; y is [ns T, N] (store, rotary), [ns T, N/2] bf16 (SwiGLU) or the
+// fp32 residual stream [ns T, N] (residual add); rope: rotary arguments of epi == kEpiRope
 constexpr int kEpiRope = 3;
 struct RopeCfg {
   int64_t P, cols;
@@ -111,16 +114,19 @@ struct RopeCfg {
 int stacked_linear(int prof_class, const void* x, int64_t T, int64_t K, int64_t N, const void* W,
                    const void* A, const void* B, int64_t r, float s, void* u, void* y, bool f32,
                    int* err, cudaStream_t st, int epi = HYDRA_EPI_STORE,
-                   const RopeCfg* rope = nullptr) {
+                   const RopeCfg* rope = nullptr, int ns = 2, const void* A2 = nullptr,
+                   const void* B2 = nullptr, void* u2 = nullptr) {
   const size_t xs = static_cast<size_t>(T) * K * 2;
   const size_t ys = epi == HYDRA_EPI_SWIGLU    ? static_cast<size_t>(T) * (N / 2) * 2
                     : epi == HYDRA_EPI_RESIDUAL ? static_cast<size_t>(T) * N * 4
                                                 : static_cast<size_t>(T) * N * (f32 ? 4 : 2);
   const void* x_off = x;
   const void* x_on = static_cast<const uint8_t*>(x) + xs;
+  const void* x_crit = static_cast<const uint8_t*>(x) + 2 * xs;
   if (r > 0) {
     ProfScope ps(HYDRA_PROF_LORA_DOWN, st);
-    const int e = hydra::launch_lora_down(x_on, T, K, A, r, s, u, st);
+    int e = hydra::launch_lora_down(x_on, T, K, A, r, s, u, st);
+    if (e == 0 && ns == 3) e = hydra::launch_lora_down(x_crit, T, K, A2, r, s, u2, st);
     if (e != 0) return e;
   }
   ProfScope ps(prof_class, st);
@@ -137,6 +143,12 @@ int stacked_linear(int prof_class, const void* x, int64_t T, int64_t K, int64_t 
   g.shared_x = false;
   g.y_off = y;
   g.y_on = static_cast<uint8_t*>(y) + ys;
+  if (ns == 3) {
+    g.x_crit = x_crit;
+    g.u_crit = r > 0 ? u2 : nullptr;
+    g.B_crit = r > 0 ? B2 : nullptr;
+    g.y_crit = static_cast<uint8_t*>(y) + 2 * ys;
+  }
   g.out_f32 = f32 ? 1 : 0;
   g.err = err;
   g.epi = epi;
@@ -253,12 +265,16 @@ size_t hydra_score_llama_workspace_size(const hydra_llama_config* cfg, int64_t S
   return layout(*cfg, S).total;
 }
 
-hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_weights* w,
-                               const int32_t* ids, const int32_t* lengths, int64_t S,
-                               void* workspace, size_t workspace_bytes, float* logp_actor,
-                               float* logp_ref, float* reward, float* values, float* advantages,
-                               float* returns, float* score, void* stream) {
+// The scoring pass over ns = 2 (J-Hydra; critic == NULL) or 3 (Hydra-PPO: critic holds the
+// critic's LoRA set per layer) stacked streams.
+static hydra_status score_pass(const hydra_llama_config* cfg, const hydra_llama_weights* w,
+                               const hydra_llama_lora* critic, const int32_t* ids,
+                               const int32_t* lengths, int64_t S, void* workspace,
+                               size_t workspace_bytes, float* logp_actor, float* logp_ref,
+                               float* reward, float* values, float* advantages, float* returns,
+                               float* score, void* stream) {
   if (cfg == nullptr || w == nullptr) return HYDRA_ERR_NULL;
+  const int ns = critic != nullptr ? 3 : 2;
   if (!valid_config(cfg)) return HYDRA_ERR_SHAPE;
   if (S < 0) return HYDRA_ERR_SHAPE;
   if (S == 0) return HYDRA_OK;
@@ -277,8 +293,16 @@ hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_
       if (p == nullptr) return HYDRA_ERR_NULL;
       if (!a16(p)) return HYDRA_ERR_ALIGN;
     }
+    if (critic != nullptr) {
+      const hydra_llama_lora& cl = critic[l];
+      const void* cp[] = {cl.a_qv, cl.b_qkv, cl.a_gu, cl.b_gu, cl.a_down, cl.b_down};
+      for (const void* p : cp) {
+        if (p == nullptr) return HYDRA_ERR_NULL;
+        if (!a16(p)) return HYDRA_ERR_ALIGN;
+      }
+    }
   }
-  const PassLayout Lo = layout(c, S);
+  const PassLayout Lo = layout(c, S, ns);
   if (workspace == nullptr) return HYDRA_ERR_WORKSPACE;
   if (!a16(workspace)) return HYDRA_ERR_ALIGN;
   if (workspace_bytes < Lo.total) return HYDRA_ERR_WORKSPACE;
@@ -295,6 +319,8 @@ hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_
   void* attn = ws + Lo.attn;
   void* m = ws + Lo.m;
   void* u = ws + Lo.u;
+  void* u2 = static_cast<uint8_t*>(u) + static_cast<size_t>(S) * (c.prompt_len + c.response_len) *
+                                            2 * c.lora_rank * 2;  // critic stream's u
   void* fin = ws + Lo.fin;
   float2* part = reinterpret_cast<float2*>(ws + Lo.part);
   float* tgt = reinterpret_cast<float*>(ws + Lo.tgt);
@@ -303,7 +329,7 @@ hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_
 
   const int64_t P = c.prompt_len + c.response_len;
   const int64_t T = S * P;
-  const int64_t R = 2 * T;
+  const int64_t R = ns * T;
   const int64_t d = c.d_model, F = c.ffn, V = c.vocab, r = c.lora_rank, L = c.response_len;
   const int64_t SL = S * L;
   const float s = c.lora_scale;
@@ -319,32 +345,33 @@ hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_
     HY_TRY(x);                 \
   } while (0)
 
-  HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_embed(w->embed, V, d, ids, T, 2, h, err, st));
+  HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_embed(w->embed, V, d, ids, T, ns, h, err, st));
   // rotation table of the positions 0..P-1, shared by every layer's q/k/v epilogue
   HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rope_table(P, c.head_dim, c.rope_theta, rope_table, st));
   for (int64_t l = 0; l < c.n_layers; ++l) {
     const hydra_llama_layer& ly = w->layers[l];
+    const hydra_llama_lora* cl = critic != nullptr ? &critic[l] : nullptr;  // critic LoRA set
     // attention block
     HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(h, ly.norm_attn, R, d, c.rms_eps, ident, a, st));
     // q/k/v projection with the rotary embedding of q and k fused into the epilogue
     const RopeCfg rope{P, 2 * d, rope_table};
     HY_TRY(stacked_linear(HYDRA_PROF_GEMM_QKV, a, T, d, 3 * d, ly.w_qkv, ly.a_qv, ly.b_qkv, 2 * r, s, u, qkv, false,
-                          err, st, kEpiRope, &rope));
+                          err, st, kEpiRope, &rope, ns, cl ? cl->a_qv : nullptr, cl ? cl->b_qkv : nullptr, u2));
     HY_PROF(HYDRA_PROF_ATTENTION,
-            hydra::launch_causal_attention(qkv, 2 * S, P, 3 * d, c.n_heads, c.head_dim, attn, d, st));
+            hydra::launch_causal_attention(qkv, ns * S, P, 3 * d, c.n_heads, c.head_dim, attn, d, st));
     // o projection added straight into the residual stream (fused epilogue)
     HY_TRY(stacked_linear(HYDRA_PROF_GEMM_O, attn, T, d, d, ly.w_o, nullptr, nullptr, 0, s, u, h, false, err, st,
-                          HYDRA_EPI_RESIDUAL));
+                          HYDRA_EPI_RESIDUAL, nullptr, ns));
     // feed-forward block: gate/up with the SwiGLU fused into the epilogue, down added into h
     HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(h, ly.norm_ffn, R, d, c.rms_eps, ident, a, st));
     HY_TRY(stacked_linear(HYDRA_PROF_GEMM_GU, a, T, d, 2 * F, ly.w_gu, ly.a_gu, ly.b_gu, 2 * r, s, u, m, false, err, st,
-                          HYDRA_EPI_SWIGLU));
+                          HYDRA_EPI_SWIGLU, nullptr, ns, cl ? cl->a_gu : nullptr, cl ? cl->b_gu : nullptr, u2));
     HY_TRY(stacked_linear(HYDRA_PROF_GEMM_DOWN, m, T, F, d, ly.w_down, ly.a_down, ly.b_down, r, s, u, h, false, err, st,
-                          HYDRA_EPI_RESIDUAL));
+                          HYDRA_EPI_RESIDUAL, nullptr, ns, cl ? cl->a_down : nullptr, cl ? cl->b_down : nullptr, u2));
   }
   // final norm on the rows that predict response tokens: row P0 - 1 + t of each sequence
   const hydra::RowMap resp{L, P, c.prompt_len - 1};
-  HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(h, w->final_norm, 2 * SL, d, c.rms_eps, resp, fin, st));
+  HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(h, w->final_norm, ns * SL, d, c.rms_eps, resp, fin, st));
   // LM head of both streams with the log-softmax reduced in the GEMM epilogue
   const int64_t nt = (V + 255) / 256;
   const int32_t* resp_ids = ids + c.prompt_len;  // token of response row s * L + t: ids[s * P + P0 + t]
@@ -375,7 +402,8 @@ hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_
   // LoRA-on stream (the same head: r_phi = LO(V))
   HY_PROF(HYDRA_PROF_HEADS, hydra::launch_seq_score(h, w->final_norm, w->w_rm, d, c.rms_eps,
                                                     lengths, S, L, P, c.prompt_len, sc, st));
-  const void* fin_on = static_cast<uint8_t*>(fin) + static_cast<size_t>(SL) * d * 2;
+  // values from the last stream: the on stream (J-Hydra) or the critic stream (Hydra-PPO)
+  const void* fin_on = static_cast<uint8_t*>(fin) + static_cast<size_t>(ns - 1) * SL * d * 2;
   const hydra::RowMap dense{SL, SL, 0};
   HY_PROF(HYDRA_PROF_HEADS, hydra::launch_head_dot(fin_on, d, w->w_rm, dense, SL, lengths, L, values, st));
   HY_PROF(HYDRA_PROF_LOGPROBS,
@@ -390,6 +418,31 @@ hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_
 #undef HY_TRY
 #undef HY_PROF
   return HYDRA_OK;
+}
+
+hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_weights* w,
+                               const int32_t* ids, const int32_t* lengths, int64_t S,
+                               void* workspace, size_t workspace_bytes, float* logp_actor,
+                               float* logp_ref, float* reward, float* values, float* advantages,
+                               float* returns, float* score, void* stream) {
+  return score_pass(cfg, w, nullptr, ids, lengths, S, workspace, workspace_bytes, logp_actor,
+                    logp_ref, reward, values, advantages, returns, score, stream);
+}
+
+size_t hydra_score_llama_hydra_workspace_size(const hydra_llama_config* cfg, int64_t S) {
+  if (!valid_config(cfg) || S < 0) return 0;
+  return layout(*cfg, S, 3).total;
+}
+
+hydra_status hydra_score_llama_hydra(const hydra_llama_config* cfg, const hydra_llama_weights* w,
+                                     const hydra_llama_lora* critic, const int32_t* ids,
+                                     const int32_t* lengths, int64_t S, void* workspace,
+                                     size_t workspace_bytes, float* logp_actor, float* logp_ref,
+                                     float* reward, float* values, float* advantages,
+                                     float* returns, float* score, void* stream) {
+  if (critic == nullptr) return HYDRA_ERR_NULL;
+  return score_pass(cfg, w, critic, ids, lengths, S, workspace, workspace_bytes, logp_actor,
+                    logp_ref, reward, values, advantages, returns, score, stream);
 }
 
 }  // extern "C"

@@ -74,6 +74,10 @@ class LlamaLayerC(ctypes.Structure):
                                    "w_down", "a_down", "b_down", "norm_attn", "norm_ffn")]
 
 
+class LlamaLoraC(ctypes.Structure):
+    _fields_ = [(n, _vp) for n in ("a_qv", "b_qkv", "a_gu", "b_gu", "a_down", "b_down")]
+
+
 class LlamaWeightsC(ctypes.Structure):
     _fields_ = [("embed", _vp), ("layers", ctypes.POINTER(LlamaLayerC)), ("final_norm", _vp),
                 ("lm_head", _vp), ("w_rm", _vp)]
@@ -100,6 +104,13 @@ _SIGNATURES.update({
                                          ctypes.POINTER(LlamaWeightsC), _vp, _vp, _c_i64, _vp,
                                          ctypes.c_size_t, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
                                          _vp]),
+    "hydra_score_llama_hydra_workspace_size": (ctypes.c_size_t, [ctypes.POINTER(LlamaConfigC),
+                                                                 _c_i64]),
+    "hydra_score_llama_hydra": (ctypes.c_int, [ctypes.POINTER(LlamaConfigC),
+                                               ctypes.POINTER(LlamaWeightsC),
+                                               ctypes.POINTER(LlamaLoraC), _vp, _vp, _c_i64,
+                                               _vp, ctypes.c_size_t, _vp, _vp, _vp, _vp, _vp,
+                                               _vp, _vp, _vp]),
 })
 
 _lib = None
@@ -438,6 +449,50 @@ def llama_config_c(cfg):
 def score_llama_workspace_size(cfg, S):
     c = llama_config_c(cfg)
     return int(load().hydra_score_llama_workspace_size(ctypes.byref(c), S))
+
+
+def score_llama_hydra_workspace_size(cfg, S):
+    c = llama_config_c(cfg)
+    return int(load().hydra_score_llama_hydra_workspace_size(ctypes.byref(c), S))
+
+
+def _weights_c(cfg, weights):
+    n = cfg["n_layers"]
+    layers = (LlamaLayerC * n)()
+    for l in range(n):
+        for name, _ in LlamaLayerC._fields_:
+            t = weights[name][l]
+            _req(t, torch.bfloat16, name)
+            setattr(layers[l], name, t.data_ptr())
+    for name in ("embed", "final_norm", "lm_head", "w_rm"):
+        _req(weights[name], torch.bfloat16, name)
+    w = LlamaWeightsC(weights["embed"].data_ptr(), layers, weights["final_norm"].data_ptr(),
+                      weights["lm_head"].data_ptr(), weights["w_rm"].data_ptr())
+    return w, layers
+
+
+def hydra_score_llama_hydra(cfg, weights, critic, ids, lengths, workspace, outputs, stream=None):
+    """Hydra-PPO scoring pass: as hydra_score_llama with the critic's LoRA set critic (dict of
+    per-layer lists a_qv, b_qkv, a_gu, b_gu, a_down, b_down in the fused layouts) as a third
+    stream whose final hidden states give the values."""
+    c = llama_config_c(cfg)
+    w, _layers = _weights_c(cfg, weights)
+    n = cfg["n_layers"]
+    crit = (LlamaLoraC * n)()
+    for l in range(n):
+        for name, _ in LlamaLoraC._fields_:
+            t = critic[name][l]
+            _req(t, torch.bfloat16, name)
+            setattr(crit[l], name, t.data_ptr())
+    _req(ids, torch.int32, "ids")
+    _req(lengths, torch.int32, "lengths")
+    names = ("logp_actor", "logp_ref", "reward", "values", "advantages", "returns", "score")
+    for k in names:
+        _req(outputs[k], torch.float32, k)
+    ws_bytes = workspace.numel() * workspace.element_size()
+    _check("hydra_score_llama_hydra", load().hydra_score_llama_hydra(
+        ctypes.byref(c), ctypes.byref(w), crit, _p(ids), _p(lengths), ids.shape[0], _p(workspace),
+        ws_bytes, *[_p(outputs[k]) for k in names], _stream(stream)))
 
 
 def hydra_score_llama(cfg, weights, ids, lengths, workspace, outputs, stream=None):

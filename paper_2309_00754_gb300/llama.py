@@ -114,6 +114,38 @@ def fuse_separate(sep):
     return out
 
 
+LORA_KEYS = ("a_qv", "b_qkv", "a_gu", "b_gu", "a_down", "b_down")
+
+
+def fuse_lora(lora, d, F):
+    """One LoRA set in the fused layouts of hydra_llama_lora (numpy bf16 bit patterns): lora =
+    {name: (A [nl, r, in], B [nl, out, r])} for name in wq, wv, wg, wu, wd."""
+    nl = lora["wq"][0].shape[0]
+    r = lora["wq"][0].shape[1]
+    out = {k: [] for k in LORA_KEYS}
+    for l in range(nl):
+        out["a_qv"].append(np.concatenate([lora["wq"][0][l], lora["wv"][0][l]], 0))
+        b = np.zeros((3 * d, 2 * r), dtype=np.uint16)
+        b[:d, :r] = lora["wq"][1][l]
+        b[2 * d:, r:] = lora["wv"][1][l]
+        out["b_qkv"].append(b)
+        out["a_gu"].append(np.concatenate([lora["wg"][0][l], lora["wu"][0][l]], 0))
+        bg = np.zeros((F, 2 * r), dtype=np.uint16)
+        bu = np.zeros((F, 2 * r), dtype=np.uint16)
+        bg[:, :r] = lora["wg"][1][l]
+        bu[:, r:] = lora["wu"][1][l]
+        out["b_gu"].append(interleave_gate_up(bg, bu))
+        out["a_down"].append(lora["wd"][0][l])
+        out["b_down"].append(lora["wd"][1][l])
+    return out
+
+
+def lora_to_device(fused, device):
+    def dev(a):
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).to(device)
+    return {k: [dev(a) for a in fused[k]] for k in LORA_KEYS}
+
+
 def to_device(fused, device):
     def dev(a):
         return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).to(device)

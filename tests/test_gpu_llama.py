@@ -340,3 +340,66 @@ def test_llama7b_lora_off_streams_agree_bitwise(llama7b):
     for s in range(4):
         expect[s, lengths[s] - 1] = a["score"][s]
     assert torch.equal(a["reward"], expect)
+
+
+# ------------------------------------------------------------------ Hydra-PPO (three streams)
+
+
+def _critic_set(cfg, seed):
+    """A second LoRA set (the critic's): separate numpy bf16 bits and fp64 values."""
+    sep2, w2 = make_model(cfg, seed)
+    return sep2["lora"], w2["lora"]
+
+
+def run_hydra_pass(cfg, sep, crit_sep, ids, lengths):
+    S = ids.shape[0]
+    w = llama.to_device(llama.fuse_separate(sep), "cuda")
+    crit = llama.lora_to_device(llama.fuse_lora(crit_sep, cfg["d_model"], cfg["ffn"]), "cuda")
+    ws = torch.empty(H.score_llama_hydra_workspace_size(cfg, S), dtype=torch.uint8, device="cuda")
+    out = llama.alloc_outputs(S, cfg["response_len"], "cuda")
+    H.hydra_score_llama_hydra(cfg, w, crit, dev_i32(ids),
+                              None if lengths is None else dev_i32(lengths), ws, out)
+    torch.cuda.synchronize()
+    return {k: host_f64(v) for k, v in out.items()}
+
+
+def test_score_llama_hydra_small_ragged():
+    """Hydra-PPO's three-stream pass (critic LoRA set separate from the actor's) against the
+    oracle's three-stream pass, sequence by sequence."""
+    cfg = dict(SMALL)
+    sep, w64 = make_model(cfg, 65)
+    crit_sep, crit64 = _critic_set(cfg, 66)
+    S, P = 3, cfg["prompt_len"] + cfg["response_len"]
+    ids = synth.randint(651, (S, P), 0, cfg["vocab"])
+    lengths = np.array([40, 23, 2], dtype=np.int32)
+    got = run_hydra_pass(cfg, sep, crit_sep, ids, lengths)
+    P0, L, g_, lam, beta = cfg["prompt_len"], cfg["response_len"], cfg["gamma"], cfg["lam"], cfg["beta"]
+    for s in range(S):
+        n = int(lengths[s])
+        ref = O.llama_score_hydra(w64, crit64, ids[s], P0, oracle_cfg(cfg), seq_lengths=n,
+                                  beta=beta, gamma=g_, lam=lam)
+        assert_abs(got["logp_actor"][s], ref["logp_actor"], TOL_LOGP, f"logp_actor seq {s}")
+        assert_abs(got["logp_ref"][s], ref["logp_ref"], TOL_LOGP, f"logp_ref seq {s}")
+        assert_rel(got["score"][s:s + 1], [ref["score"]], TOL_LINEAR, f"score seq {s}")
+        assert_rel(got["values"][s], ref["values"], TOL_LINEAR, f"values seq {s}")
+        a1, r1 = O.gae(got["reward"][s:s + 1], got["values"][s:s + 1], [n], g_, lam)
+        assert_rel(got["advantages"][s:s + 1], a1, TOL_GAE, f"advantages seq {s}")
+    # the critic set moves the values: they differ from the J-Hydra pass's on-stream values
+    jh = run_pass(cfg, sep, ids, lengths)
+    assert np.array_equal(got["logp_actor"], jh["logp_actor"])
+    assert np.array_equal(got["logp_ref"], jh["logp_ref"])
+    assert np.max(np.abs(got["values"] - jh["values"])) > 1e-4
+
+
+def test_score_llama_hydra_one_lora_set_is_j_hydra():
+    """With the critic's LoRA set equal to the actor's, the three-stream pass returns the
+    J-Hydra pass's outputs bit for bit."""
+    cfg = dict(SMALL)
+    sep, _ = make_model(cfg, 67)
+    S, P = 2, cfg["prompt_len"] + cfg["response_len"]
+    ids = synth.randint(671, (S, P), 0, cfg["vocab"])
+    lengths = np.array([40, 31], dtype=np.int32)
+    got = run_hydra_pass(cfg, sep, sep["lora"], ids, lengths)
+    jh = run_pass(cfg, sep, ids, lengths)
+    for k in got:
+        assert np.array_equal(got[k], jh[k]), k
