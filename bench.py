@@ -403,6 +403,58 @@ class HydraScoringLlama7B:
         return smp["resp"] * len(t_pass) / sum(t_pass), desc
 
 
+class HydraPPOScoringLlama7B(HydraScoringLlama7B):
+    """Hydra-PPO scoring pass (Algorithm 2): the same model and batch as hydra_scoring_llama7b
+    with a second, random LoRA set for the critic, so three streams (LoRA off, actor, critic)
+    run through every layer; values come from the critic stream."""
+
+    name = "hydra_ppo_scoring_llama7b"
+    seed = 5
+
+    def __init__(self, device, seed=5, reference=False):
+        super().__init__(device, seed=seed, reference=reference)
+        c = self.cfg
+        self.critic = self.llama.random_device_lora(c, seed + 1000, device)
+        if not reference:
+            import torch
+            self.ws = torch.empty(self.H.score_llama_hydra_workspace_size(c, self.S),
+                                  dtype=torch.uint8, device=device)
+        P = self.P0 + self.L
+        T, SL = self.S * P, self.S * self.L
+        d, F, V, r, nl = c["d_model"], c["ffn"], c["vocab"], c["lora_rank"], c["n_layers"]
+        # three streams; the LoRA-up runs on the actor and critic streams
+        self.class_flops = {
+            "gemm_qkv": nl * (3 * (2 * T * d * 3 * d) + 2 * (2 * T * 2 * r * 3 * d)),
+            "gemm_o": nl * 3 * (2 * T * d * d),
+            "gemm_gu": nl * (3 * (2 * T * d * 2 * F) + 2 * (2 * T * 2 * r * 2 * F)),
+            "gemm_down": nl * (3 * (2 * T * F * d) + 2 * (2 * T * r * d)),
+            "gemm_lmhead": 2 * (2 * SL * d * V),
+        }
+        self.gemm_flops = sum(self.class_flops.values())
+        self.attn_flops = nl * 3 * self.S * c["n_heads"] * 2 * P * P * 128  # causal half
+
+    def step(self, ev=None):
+        self.H.hydra_score_llama_hydra(self.cfg, self.weights, self.critic, self.ids, self.lengths,
+                                       self.ws, self.out)
+
+    def config(self):
+        cfg = super().config()
+        cfg["workload"] = ("hydra_ppo_scoring_llama7b: random-init Llama-7B (32 layers, d 4096, 32 "
+                           "heads, SwiGLU 11008, vocab 32000, bf16), two LoRA sets r=16 s=2 (actor, "
+                           "critic) on q/v/gate/up/down, reward/value head 4096->1; three streams; batch "
+                           "4 x (256 prompt + 512 response); logp/KL beta 0.1, GAE gamma 1 lambda 0.95")
+        cfg["processed_tokens_per_step"] = 3 * self.S * (self.P0 + self.L)
+        return cfg
+
+    def oracle_time(self, smp, n_layers):
+        import oracle as O
+        t0 = time.perf_counter()
+        # the critic stream costs the same whichever set it carries: the actor's set stands in
+        O.llama_score_hydra(smp["w"], smp["w"]["lora"], smp["ids"], smp["prompt"], smp["cfg"],
+                            n_layers=n_layers, beta=self.beta, gamma=self.gamma, lam=self.lam)
+        return time.perf_counter() - t0
+
+
 class KernelSweep:
     """Per-kernel measurements of the rows the full pass does not exercise at their own
     shapes (one JSON line; value = the sweep's mean fraction of roofline):
@@ -530,6 +582,7 @@ class KernelSweep:
 
 
 WORKLOADS = {LmHeadScoring.name: LmHeadScoring, HydraScoringLlama7B.name: HydraScoringLlama7B,
+             HydraPPOScoringLlama7B.name: HydraPPOScoringLlama7B,
              KernelSweep.name: KernelSweep}
 DEFAULT_WORKLOAD = HydraScoringLlama7B.name
 

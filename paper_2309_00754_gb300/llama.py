@@ -78,6 +78,35 @@ def random_device_weights(cfg, seed, device, std=0.02):
     return w
 
 
+def random_device_lora(cfg, seed, device, std=0.02):
+    """A second random LoRA set (the Hydra-PPO critic's) in the fused layouts of
+    hydra_llama_lora, drawn on the device (benchmark data)."""
+    g = torch.Generator(device=device)
+    g.manual_seed(seed)
+    d, F, r, n = cfg["d_model"], cfg["ffn"], cfg["lora_rank"], cfg["n_layers"]
+    bf = torch.bfloat16
+
+    def rnd(*shape):
+        return (std * torch.randn(*shape, device=device, generator=g)).to(bf)
+
+    out = {k: [] for k in LORA_KEYS}
+    for _ in range(n):
+        out["a_qv"].append(rnd(2 * r, d))
+        b = torch.zeros(3 * d, 2 * r, dtype=bf, device=device)
+        b[:d, :r] = rnd(d, r)
+        b[2 * d:, r:] = rnd(d, r)
+        out["b_qkv"].append(b)
+        out["a_gu"].append(rnd(2 * r, d))
+        bg = torch.zeros(F, 2 * r, dtype=bf, device=device)
+        bu = torch.zeros(F, 2 * r, dtype=bf, device=device)
+        bg[:, :r] = rnd(F, r)
+        bu[:, r:] = rnd(F, r)
+        out["b_gu"].append(interleave_gate_up(bg, bu))
+        out["a_down"].append(rnd(r, F))
+        out["b_down"].append(rnd(d, r))
+    return out
+
+
 def fuse_separate(sep):
     """Fused numpy layouts (bf16 bit patterns, uint16) from separate per-projection arrays:
     sep has wq, wk, wv, wo [nl, d, d], wg, wu [nl, F, d], wd [nl, d, F], norm1, norm2
