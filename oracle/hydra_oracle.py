@@ -30,6 +30,10 @@ Readings where the paper is silent (the same readings the CUDA path implements):
   * Per-token KL penalty uses the sampled-token estimate logp_actor - logp_ref; the
     sequence score is added at the last valid token t = len - 1.
   * GAE: the value after the last valid token is 0 (terminal); positions >= len are 0.
+  * PPO update side: the paper gives no clip range; eps = 0.2 (the PPO paper's default) is
+    an argument. Losses are means over the valid tokens of the batch; the surrogate is
+    negated so both losses are minimised. Advantage whitening (optional, off by default)
+    uses the population variance over valid tokens with 1e-8 under the square root.
 
 Parity pins for every function live in tests/test_oracle_pins.py (closed forms,
 invariants, brute force, library routines, hand-worked fixtures in tests/golden/).
@@ -413,3 +417,61 @@ def llama_score_hydra(weights, lora_critic, ids, prompt_len, cfg, seq_lengths=No
         "h_act": f[1],
         "h_crit": f[2],
     }
+
+
+# ---------------------------------------------------------------------------
+# Update side of PPO (§2 Stage 3: ratio r(theta), clipped surrogate L^CLIP, squared-error
+# value loss on the returns; Alg. 1/2 "optimize surrogate L")
+# ---------------------------------------------------------------------------
+
+
+def ppo_loss(logp_new, logp_old, adv, returns, values, lengths, clip_eps=0.2, whiten=False):
+    """PPO losses over the valid tokens t < len_s of [S, L] arrays:
+      r_t       = exp(logp_new_t - logp_old_t)                         (probability ratio)
+      A_t       = adv_t, or (adv_t - mean) / sqrt(var + 1e-8) over valid tokens if whiten
+      s_t       = min(r_t A_t, clip(r_t, 1 - eps, 1 + eps) A_t)
+      loss_clip = -(1/n) sum_t s_t                                     (maximise L^CLIP)
+      loss_value = (1/n) sum_t (values_t - returns_t)^2
+    Returns dict with loss_clip, loss_value, clip_frac (share of valid tokens with
+    |r - 1| > eps), approx_kl ((1/n) sum (logp_old - logp_new)), adv_mean, adv_std (of the
+    raw advantages), grad_logp = d loss_clip / d logp_new and grad_values =
+    d loss_value / d values (0 at invalid tokens). A_t is treated as a constant."""
+    ln = np.asarray(logp_new, dtype=np.float64)
+    lo = np.asarray(logp_old, dtype=np.float64)
+    a = np.asarray(adv, dtype=np.float64)
+    R = np.asarray(returns, dtype=np.float64)
+    V = np.asarray(values, dtype=np.float64)
+    S, L = ln.shape
+    valid = np.arange(L)[None, :] < np.asarray(lengths, dtype=np.int64)[:, None]
+    n = int(valid.sum())
+    grad_logp = np.zeros((S, L))
+    grad_v = np.zeros((S, L))
+    if n == 0:
+        return {"loss_clip": 0.0, "loss_value": 0.0, "clip_frac": 0.0, "approx_kl": 0.0,
+                "adv_mean": 0.0, "adv_std": 0.0, "grad_logp": grad_logp, "grad_values": grad_v}
+    mean = float(a[valid].sum() / n)
+    var = float(((a[valid] - mean) ** 2).sum() / n)
+    A = (a - mean) / np.sqrt(var + 1e-8) if whiten else a
+    total_s = 0.0
+    total_v = 0.0
+    clipped = 0
+    kl = 0.0
+    for s in range(S):
+        for t in range(L):
+            if not valid[s, t]:
+                continue
+            r = float(np.exp(ln[s, t] - lo[s, t]))
+            rc = min(max(r, 1.0 - clip_eps), 1.0 + clip_eps)
+            unclipped, clip_term = r * A[s, t], rc * A[s, t]
+            total_s += min(unclipped, clip_term)
+            # the unclipped term is the active one (ties included): d(r A)/d logp = r A
+            if unclipped <= clip_term:
+                grad_logp[s, t] = -r * A[s, t] / n
+            if abs(r - 1.0) > clip_eps:
+                clipped += 1
+            kl += lo[s, t] - ln[s, t]
+            total_v += (V[s, t] - R[s, t]) ** 2
+            grad_v[s, t] = 2.0 * (V[s, t] - R[s, t]) / n
+    return {"loss_clip": -total_s / n, "loss_value": total_v / n, "clip_frac": clipped / n,
+            "approx_kl": kl / n, "adv_mean": mean, "adv_std": float(np.sqrt(var)),
+            "grad_logp": grad_logp, "grad_values": grad_v}

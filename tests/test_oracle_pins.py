@@ -420,3 +420,74 @@ def test_hydra_ppo_critic_stream_is_separate():
         assert np.array_equal(alt[k], off_crit[k]), k
     assert alt["score"] == off_crit["score"]
     assert np.max(np.abs(alt["values"] - off_crit["values"])) > 1e-6
+
+
+# ------------------------------------------------------------------ PPO update-side losses
+
+
+def test_ppo_loss_hand_example():
+    # eps = 0.2; ratios 0.5, 1.0, 1.5 (logp_new - logp_old = log r), advantages +1, -2, +1
+    lo = np.zeros((1, 3))
+    ln = np.log(np.array([[0.5, 1.0, 1.5]]))
+    A = np.array([[1.0, -2.0, 1.0]])
+    R = np.array([[1.0, 2.0, 3.0]])
+    V = np.array([[1.5, 2.0, 1.0]])
+    out = O.ppo_loss(ln, lo, A, R, V, [3], clip_eps=0.2)
+    # s = min(0.5, 0.8) = 0.5; min(-2, -2) = -2; min(1.5, 1.2) = 1.2
+    assert abs(out["loss_clip"] - (-(0.5 - 2.0 + 1.2) / 3)) < 1e-15
+    assert abs(out["loss_value"] - (0.25 + 0.0 + 4.0) / 3) < 1e-15
+    assert out["clip_frac"] == 2 / 3
+    np.testing.assert_allclose(out["grad_logp"], [[-0.5 / 3, 2.0 / 3, 0.0]], atol=1e-15)
+    np.testing.assert_allclose(out["grad_values"], [[1.0 / 3, 0.0, -4.0 / 3]], atol=1e-15)
+
+
+def _ppo_problem(seed, S=3, L=11):
+    rng = np.random.default_rng(seed)
+    lo = rng.normal(-2.0, 0.5, (S, L))
+    ln = lo + rng.normal(0.0, 0.3, (S, L))
+    A = rng.normal(0.0, 1.5, (S, L))
+    R = rng.normal(0.0, 1.0, (S, L))
+    V = rng.normal(0.0, 1.0, (S, L))
+    lengths = np.array([L, 5, 0][:S])
+    return ln, lo, A, R, V, lengths
+
+
+@pytest.mark.parametrize("whiten", [False, True])
+def test_ppo_loss_gradients_match_finite_differences(whiten):
+    ln, lo, A, R, V, lengths = _ppo_problem(21)
+    out = O.ppo_loss(ln, lo, A, R, V, lengths, whiten=whiten)
+    h = 1e-6
+    for s, t in [(0, 0), (0, 7), (1, 3), (1, 6), (2, 1)]:
+        lp, lm = ln.copy(), ln.copy()
+        lp[s, t] += h
+        lm[s, t] -= h
+        fd = (O.ppo_loss(lp, lo, A, R, V, lengths, whiten=whiten)["loss_clip"] -
+              O.ppo_loss(lm, lo, A, R, V, lengths, whiten=whiten)["loss_clip"]) / (2 * h)
+        assert abs(fd - out["grad_logp"][s, t]) < 1e-7, (s, t)
+        vp, vm = V.copy(), V.copy()
+        vp[s, t] += h
+        vm[s, t] -= h
+        fd = (O.ppo_loss(ln, lo, A, R, vp, lengths)["loss_value"] -
+              O.ppo_loss(ln, lo, A, R, vm, lengths)["loss_value"]) / (2 * h)
+        assert abs(fd - out["grad_values"][s, t]) < 1e-7, (s, t)
+
+
+def test_ppo_loss_special_cases():
+    ln, lo, A, R, V, lengths = _ppo_problem(22)
+    valid = np.arange(11)[None, :] < lengths[:, None]
+    # policy unchanged: ratio 1, L^CLIP is the mean advantage, nothing clipped, KL 0
+    same = O.ppo_loss(lo, lo, A, R, V, lengths)
+    assert abs(same["loss_clip"] + A[valid].mean()) < 1e-12
+    assert same["clip_frac"] == 0.0 and same["approx_kl"] == 0.0
+    # whitened advantages have mean 0 and variance 1 over the valid tokens
+    w = O.ppo_loss(lo, lo, A, R, V, lengths, whiten=True)
+    assert abs(w["loss_clip"]) < 1e-12
+    assert abs(w["adv_mean"] - A[valid].mean()) < 1e-12 and abs(w["adv_std"] - A[valid].std()) < 1e-12
+    # a huge ratio with positive advantage is clipped: no gradient
+    big = lo.copy()
+    big[0, 0] += 5.0
+    g = O.ppo_loss(big, lo, np.abs(A), R, V, lengths)
+    assert g["grad_logp"][0, 0] == 0.0
+    # no valid tokens
+    z = O.ppo_loss(ln, lo, A, R, V, [0, 0, 0])
+    assert z["loss_clip"] == 0.0 and not z["grad_logp"].any()
