@@ -425,53 +425,52 @@ def llama_score_hydra(weights, lora_critic, ids, prompt_len, cfg, seq_lengths=No
 # ---------------------------------------------------------------------------
 
 
-def ppo_loss(logp_new, logp_old, adv, returns, values, lengths, clip_eps=0.2, whiten=False):
+def ppo_loss(logp_new, logp_old, adv, returns, values, lengths, clip_eps=0.2, whiten=False,
+             moments=None):
     """PPO losses over the valid tokens t < len_s of [S, L] arrays:
       r_t       = exp(logp_new_t - logp_old_t)                         (probability ratio)
-      A_t       = adv_t, or (adv_t - mean) / sqrt(var + 1e-8) over valid tokens if whiten
+      A_t       = adv_t, or (adv_t - mean) / sqrt(M2 / n + 1e-8) if whiten
       s_t       = min(r_t A_t, clip(r_t, 1 - eps, 1 + eps) A_t)
       loss_clip = -(1/n) sum_t s_t                                     (maximise L^CLIP)
       loss_value = (1/n) sum_t (values_t - returns_t)^2
+    (n, mean, M2) are the count, mean and summed squared deviation of the valid advantages,
+    or the given `moments` (e.g. those of a larger batch this one is a shard of; n then
+    also normalises the losses).
     Returns dict with loss_clip, loss_value, clip_frac (share of valid tokens with
-    |r - 1| > eps), approx_kl ((1/n) sum (logp_old - logp_new)), adv_mean, adv_std (of the
-    raw advantages), grad_logp = d loss_clip / d logp_new and grad_values =
-    d loss_value / d values (0 at invalid tokens). A_t is treated as a constant."""
+    |r - 1| > eps, over n), approx_kl ((1/n) sum (logp_old - logp_new)), adv_mean, adv_std
+    (mean and population std of the raw advantages: from `moments` when given, else of
+    this batch), n, grad_logp = d loss_clip / d logp_new and grad_values =
+    d loss_value / d values (0 at invalid tokens). A_t is treated as a constant; where the
+    two surrogate terms tie, the unclipped one carries the gradient."""
     ln = np.asarray(logp_new, dtype=np.float64)
     lo = np.asarray(logp_old, dtype=np.float64)
     a = np.asarray(adv, dtype=np.float64)
     R = np.asarray(returns, dtype=np.float64)
     V = np.asarray(values, dtype=np.float64)
     S, L = ln.shape
-    valid = np.arange(L)[None, :] < np.asarray(lengths, dtype=np.int64)[:, None]
-    n = int(valid.sum())
-    grad_logp = np.zeros((S, L))
-    grad_v = np.zeros((S, L))
-    if n == 0:
-        return {"loss_clip": 0.0, "loss_value": 0.0, "clip_frac": 0.0, "approx_kl": 0.0,
-                "adv_mean": 0.0, "adv_std": 0.0, "grad_logp": grad_logp, "grad_values": grad_v}
-    mean = float(a[valid].sum() / n)
-    var = float(((a[valid] - mean) ** 2).sum() / n)
+    valid = np.arange(L)[None, :] < np.asarray(lengths, dtype=np.int64).reshape(S, 1)
+    if moments is None:
+        n = float(valid.sum())
+        mean = float(a[valid].sum() / n) if n > 0 else 0.0
+        m2 = float(((a[valid] - mean) ** 2).sum())
+    else:
+        n, mean, m2 = (float(v) for v in moments)
+    var = m2 / n if n > 0 else 0.0
+    inv_n = 1.0 / n if n > 0 else 0.0
     A = (a - mean) / np.sqrt(var + 1e-8) if whiten else a
-    total_s = 0.0
-    total_v = 0.0
-    clipped = 0
-    kl = 0.0
-    for s in range(S):
-        for t in range(L):
-            if not valid[s, t]:
-                continue
-            r = float(np.exp(ln[s, t] - lo[s, t]))
-            rc = min(max(r, 1.0 - clip_eps), 1.0 + clip_eps)
-            unclipped, clip_term = r * A[s, t], rc * A[s, t]
-            total_s += min(unclipped, clip_term)
-            # the unclipped term is the active one (ties included): d(r A)/d logp = r A
-            if unclipped <= clip_term:
-                grad_logp[s, t] = -r * A[s, t] / n
-            if abs(r - 1.0) > clip_eps:
-                clipped += 1
-            kl += lo[s, t] - ln[s, t]
-            total_v += (V[s, t] - R[s, t]) ** 2
-            grad_v[s, t] = 2.0 * (V[s, t] - R[s, t]) / n
-    return {"loss_clip": -total_s / n, "loss_value": total_v / n, "clip_frac": clipped / n,
-            "approx_kl": kl / n, "adv_mean": mean, "adv_std": float(np.sqrt(var)),
-            "grad_logp": grad_logp, "grad_values": grad_v}
+    r = np.exp(ln - lo)
+    rc = np.clip(r, 1.0 - clip_eps, 1.0 + clip_eps)
+    unclipped, clip_term = r * A, rc * A
+    surr = np.minimum(unclipped, clip_term)
+    dv = V - R
+    return {
+        "loss_clip": -float(surr[valid].sum()) * inv_n,
+        "loss_value": float((dv[valid] ** 2).sum()) * inv_n,
+        "clip_frac": float((valid & (np.abs(r - 1.0) > clip_eps)).sum()) * inv_n,
+        "approx_kl": float((lo - ln)[valid].sum()) * inv_n,
+        "adv_mean": mean,
+        "adv_std": float(np.sqrt(var)),
+        "n": n,
+        "grad_logp": np.where(valid & (unclipped <= clip_term), -unclipped * inv_n, 0.0),
+        "grad_values": np.where(valid, 2.0 * dv * inv_n, 0.0),
+    }

@@ -491,3 +491,19 @@ def test_ppo_loss_special_cases():
     # no valid tokens
     z = O.ppo_loss(ln, lo, A, R, V, [0, 0, 0])
     assert z["loss_clip"] == 0.0 and not z["grad_logp"].any()
+
+
+def test_ppo_loss_shards_with_merged_moments_add_up():
+    # a batch split into two shards, each normalised by the whole batch's moments: the
+    # shards' losses add up to the whole batch's and their gradients are the whole's rows
+    ln, lo, A, R, V, lengths = _ppo_problem(23, S=3, L=11)
+    for whiten in (False, True):
+        full = O.ppo_loss(ln, lo, A, R, V, lengths, whiten=whiten)
+        valid = np.arange(11)[None, :] < lengths[:, None]
+        mom = (valid.sum(), A[valid].mean(), ((A[valid] - A[valid].mean()) ** 2).sum())
+        p0 = O.ppo_loss(ln[:1], lo[:1], A[:1], R[:1], V[:1], lengths[:1], whiten=whiten, moments=mom)
+        p1 = O.ppo_loss(ln[1:], lo[1:], A[1:], R[1:], V[1:], lengths[1:], whiten=whiten, moments=mom)
+        for k in ("loss_clip", "loss_value", "clip_frac", "approx_kl"):
+            assert abs(p0[k] + p1[k] - full[k]) < 1e-12, k
+        np.testing.assert_allclose(np.vstack([p0["grad_logp"], p1["grad_logp"]]), full["grad_logp"],
+                                   atol=1e-15)
