@@ -467,6 +467,7 @@ class KernelSweep:
     Kernels are replayed back to back from CUDA graphs, weights rotated through copies
     larger than L2.
       GAE: 65536 sequences x 512 tokens -> GB/s;
+      PPO losses (clipped surrogate, value loss, gradients, whitening): the same batch -> GB/s;
       causal attention: 8 sequences x 768 tokens x 32 heads of 128 -> TFLOP/s;
       log-probs/KL: 2048 rows x 32000 fp32 logits x 2 heads -> GB/s."""
 
@@ -478,7 +479,9 @@ class KernelSweep:
     def __init__(self, device, seed=5, reference=False):
         self.device = device
 
-    def run(self, peaks, reps=20):
+    PARTS = ("projection_sweep", "decode", "gae", "ppo_loss", "attention", "logprobs")
+
+    def run(self, peaks, reps=20, parts=PARTS):
         import torch
         from paper_2309_00754_gb300 import hydra as H
         g = torch.Generator(device=self.device)
@@ -507,77 +510,103 @@ class KernelSweep:
             torch.cuda.synchronize()
             return e0.elapsed_time(e1) / n
 
-        out = {"projection_sweep": {}, "decode": {}, "gae": {}, "logprobs": {}, "attention": {}}
+        out = {k: {} for k in parts}
         # ---- projection sweep (c2): W rotates through 3 copies per shape so consecutive
         # launches do not find W in L2
-        M = 2048
-        x = torch.randn(M, 11008, device=dev, generator=g).to(bf)
-        fr = []
-        for r in (8, 16, 64):
-            for name, K, N in self.PROJ:
-                Ws = [rnd(N, K) for _ in range(3)]
-                B = rnd(N, r)
-                u = rnd(M, r, std=1.0)
-                xs = x[:, :K].contiguous()
-                y0 = torch.empty(M, N, dtype=bf, device=dev)
-                y1 = torch.empty(M, N, dtype=bf, device=dev)
-                ms = graph_ms(lambda i: H.hydra_dual_linear(xs, None, Ws[i % 3], u, B, y0, y1, algo=1), reps)
-                tf = (2.0 * M * K * N + 2.0 * M * r * N) / ms / 1e9
-                out["projection_sweep"][f"{name}_r{r}"] = {"ms": ms, "TFLOP/s": tf}
-                fr.append(tf / peaks["bf16_tflops"])
-                del Ws
-        sweep = out["projection_sweep"]
-        sweep["mean_TFLOP/s"] = statistics.mean(v["TFLOP/s"] for v in list(sweep.values()))
-        sweep["frac_of_measured_burst"] = statistics.mean(fr)
-        sweep["frac_of_2.25PF"] = sweep["mean_TFLOP/s"] / 2250.0
+        if "projection_sweep" in parts:
+            M = 2048
+            x = torch.randn(M, 11008, device=dev, generator=g).to(bf)
+            fr = []
+            for r in (8, 16, 64):
+                for name, K, N in self.PROJ:
+                    Ws = [rnd(N, K) for _ in range(3)]
+                    B = rnd(N, r)
+                    u = rnd(M, r, std=1.0)
+                    xs = x[:, :K].contiguous()
+                    y0 = torch.empty(M, N, dtype=bf, device=dev)
+                    y1 = torch.empty(M, N, dtype=bf, device=dev)
+                    ms = graph_ms(lambda i: H.hydra_dual_linear(xs, None, Ws[i % 3], u, B, y0, y1, algo=1), reps)
+                    tf = (2.0 * M * K * N + 2.0 * M * r * N) / ms / 1e9
+                    out["projection_sweep"][f"{name}_r{r}"] = {"ms": ms, "TFLOP/s": tf}
+                    fr.append(tf / peaks["bf16_tflops"])
+                    del Ws
+            sweep = out["projection_sweep"]
+            sweep["mean_TFLOP/s"] = statistics.mean(v["TFLOP/s"] for v in list(sweep.values()))
+            sweep["frac_of_measured_burst"] = statistics.mean(fr)
+            sweep["frac_of_2.25PF"] = sweep["mean_TFLOP/s"] / 2250.0
         # ---- decode (c5): W rotates through enough copies that they exceed L2
-        shapes = list(self.PROJ[:1]) + list(self.PROJ[4:5]) + list(self.PROJ[6:]) + [("lm_head", 4096, 32000)]
-        gb = []
-        for n, K, N in shapes:
-            ncopy = max(2, -(-300_000_000 // (N * K * 2)))  # > 2 x L2 of weights
-            Wd = [rnd(N, K) for _ in range(ncopy)]
-            Bd = rnd(N, 16)
-            for Mt in (1, 4, 8, 16):
-                xd = torch.randn(Mt, K, device=dev, generator=g).to(bf)
-                ud = rnd(Mt, 16, std=1.0)
-                y0 = torch.empty(Mt, N, dtype=bf, device=dev)
-                y1 = torch.empty(Mt, N, dtype=bf, device=dev)
-                ms = graph_ms(lambda i: H.hydra_dual_linear(xd, None, Wd[i % ncopy], ud, Bd, y0, y1),
-                              max(reps, 2 * ncopy))
-                byts = 2.0 * (N * K + 16 * (K + N) + Mt * K + 2 * Mt * N)
-                out["decode"].setdefault(f"M{Mt}", {})[n] = {"ms": ms, "GB/s": byts / ms / 1e6}
-                gb.append(byts / ms / 1e6)
-            del Wd
-        out["decode"]["frac_of_measured_hbm_mean"] = statistics.mean(gb) / peaks["hbm_gbs"]
+        if "decode" in parts:
+            shapes = list(self.PROJ[:1]) + list(self.PROJ[4:5]) + list(self.PROJ[6:]) + [("lm_head", 4096, 32000)]
+            gb = []
+            for n, K, N in shapes:
+                ncopy = max(2, -(-300_000_000 // (N * K * 2)))  # > 2 x L2 of weights
+                Wd = [rnd(N, K) for _ in range(ncopy)]
+                Bd = rnd(N, 16)
+                for Mt in (1, 4, 8, 16):
+                    xd = torch.randn(Mt, K, device=dev, generator=g).to(bf)
+                    ud = rnd(Mt, 16, std=1.0)
+                    y0 = torch.empty(Mt, N, dtype=bf, device=dev)
+                    y1 = torch.empty(Mt, N, dtype=bf, device=dev)
+                    ms = graph_ms(lambda i: H.hydra_dual_linear(xd, None, Wd[i % ncopy], ud, Bd, y0, y1),
+                                  max(reps, 2 * ncopy))
+                    byts = 2.0 * (N * K + 16 * (K + N) + Mt * K + 2 * Mt * N)
+                    out["decode"].setdefault(f"M{Mt}", {})[n] = {"ms": ms, "GB/s": byts / ms / 1e6}
+                    gb.append(byts / ms / 1e6)
+                del Wd
+            out["decode"]["frac_of_measured_hbm_mean"] = statistics.mean(gb) / peaks["hbm_gbs"]
         # ---- GAE at 65536 x 512
-        S, L = 65536, 512
-        rw = torch.randn(S, L, device=dev, generator=g)
-        vv = torch.randn(S, L, device=dev, generator=g)
-        ln = torch.randint(64, 513, (S,), device=dev, generator=g, dtype=torch.int32)
-        adv, ret = torch.empty_like(rw), torch.empty_like(rw)
-        ms = graph_ms(lambda i: H.ppo_gae(rw, vv, ln, 1.0, 0.95, adv, ret), reps)
-        valid = float(ln.sum().item())
-        byts = valid * 8 + S * L * 8 + S * 4  # read valid r, V; write all A, R
-        out["gae"] = {"ms": ms, "GB/s": byts / ms / 1e6, "frac_of_measured_hbm": byts / ms / 1e6 / peaks["hbm_gbs"]}
-        del rw, vv, adv, ret
+        if "gae" in parts or "ppo_loss" in parts:
+            S, L = 65536, 512
+            rw = torch.randn(S, L, device=dev, generator=g)
+            vv = torch.randn(S, L, device=dev, generator=g)
+            ln = torch.randint(64, 513, (S,), device=dev, generator=g, dtype=torch.int32)
+            adv, ret = torch.empty_like(rw), torch.empty_like(rw)
+            H.ppo_gae(rw, vv, ln, 1.0, 0.95, adv, ret)
+            valid = float(ln.sum().item())
+        if "gae" in parts:
+            ms = graph_ms(lambda i: H.ppo_gae(rw, vv, ln, 1.0, 0.95, adv, ret), reps)
+            byts = valid * 8 + S * L * 8 + S * 4  # read valid r, V; write all A, R
+            out["gae"] = {"ms": ms, "GB/s": byts / ms / 1e6, "frac_of_measured_hbm": byts / ms / 1e6 / peaks["hbm_gbs"]}
+        # ---- PPO losses at 65536 x 512, whitened: the moments pass reads the valid
+        # advantages, the loss pass reads five fp32 inputs at valid tokens and writes both
+        # gradient arrays in full
+        if "ppo_loss" in parts:
+            lo = -torch.randn(S, L, device=dev, generator=g).abs() * 2.0 - 0.05
+            lnew = lo + 0.15 * torch.randn(S, L, device=dev, generator=g)
+            gl, gv = torch.empty_like(lo), torch.empty_like(lo)
+            st = torch.zeros(7, dtype=torch.float64, device=dev)
+            ws = torch.empty(H.ppo_workspace_size(), dtype=torch.uint8, device=dev)
+            ms = graph_ms(lambda i: H.hydra_ppo_loss(lnew, lo, rw, vv, ret, ln, 0.2, True, gl, gv, st, ws), reps)
+            byts = valid * 24 + S * L * 8 + S * 8
+            out["ppo_loss"] = {"ms": ms, "GB/s": byts / ms / 1e6, "frac_of_measured_hbm": byts / ms / 1e6 / peaks["hbm_gbs"],
+                               "whiten": True}
+            ms = graph_ms(lambda i: H.hydra_ppo_loss(lnew, lo, rw, vv, ret, ln, 0.2, False, gl, gv, st, ws), reps)
+            byts = valid * 20 + S * L * 8 + S * 8
+            out["ppo_loss"]["unwhitened"] = {"ms": ms, "GB/s": byts / ms / 1e6,
+                                             "frac_of_measured_hbm": byts / ms / 1e6 / peaks["hbm_gbs"]}
+            del lo, lnew, gl, gv
+        if "gae" in parts or "ppo_loss" in parts:
+            del rw, vv, adv, ret
         # ---- causal attention at the full pass's shape: 2 streams x 4 sequences x 768 tokens,
         # 32 heads of 128
-        nseq, Pq, Hh = 8, 768, 32
-        qkv = torch.randn(nseq * Pq, 3 * Hh * 128, device=dev, generator=g).to(bf)
-        att = torch.empty(nseq * Pq, Hh * 128, dtype=bf, device=dev)
-        ms = graph_ms(lambda i: H.hydra_causal_attention(qkv, nseq, Pq, Hh, 128, att), reps)
-        fl = 4.0 * nseq * Hh * 128 * (Pq * (Pq + 1) / 2)  # q k^T and p v over the causal half
-        out["attention"] = {"ms": ms, "TFLOP/s": fl / ms / 1e9}
-        del qkv, att
+        if "attention" in parts:
+            nseq, Pq, Hh = 8, 768, 32
+            qkv = torch.randn(nseq * Pq, 3 * Hh * 128, device=dev, generator=g).to(bf)
+            att = torch.empty(nseq * Pq, Hh * 128, dtype=bf, device=dev)
+            ms = graph_ms(lambda i: H.hydra_causal_attention(qkv, nseq, Pq, Hh, 128, att), reps)
+            fl = 4.0 * nseq * Hh * 128 * (Pq * (Pq + 1) / 2)  # q k^T and p v over the causal half
+            out["attention"] = {"ms": ms, "TFLOP/s": fl / ms / 1e9}
+            del qkv, att
         # ---- log-probs/KL at 2048 x 32000 x 2 heads, all rows valid
-        T, V = 2048, 32000
-        za = torch.randn(T, V, device=dev, generator=g)
-        zr = torch.randn(T, V, device=dev, generator=g)
-        ids = torch.randint(0, V, (T,), device=dev, generator=g, dtype=torch.int32)
-        o3 = [torch.empty(T, device=dev) for _ in range(3)]
-        ms = graph_ms(lambda i: H.hydra_token_logprobs_kl(za, zr, ids, None, None, 0.1, 4, 512, *o3), reps)
-        byts = T * V * 4 * 2 + T * 16
-        out["logprobs"] = {"ms": ms, "GB/s": byts / ms / 1e6, "frac_of_measured_hbm": byts / ms / 1e6 / peaks["hbm_gbs"]}
+        if "logprobs" in parts:
+            T, V = 2048, 32000
+            za = torch.randn(T, V, device=dev, generator=g)
+            zr = torch.randn(T, V, device=dev, generator=g)
+            ids = torch.randint(0, V, (T,), device=dev, generator=g, dtype=torch.int32)
+            o3 = [torch.empty(T, device=dev) for _ in range(3)]
+            ms = graph_ms(lambda i: H.hydra_token_logprobs_kl(za, zr, ids, None, None, 0.1, 4, 512, *o3), reps)
+            byts = T * V * 4 * 2 + T * 16
+            out["logprobs"] = {"ms": ms, "GB/s": byts / ms / 1e6, "frac_of_measured_hbm": byts / ms / 1e6 / peaks["hbm_gbs"]}
         return out
 
 
@@ -701,10 +730,14 @@ def run_sweep(args):
     peaks = load_peaks()
     clocks = ClockSampler(0)
     clocks.start()
-    res = KernelSweep(torch.device("cuda", 0)).run(peaks)
+    parts = tuple(args.parts.split(",")) if args.parts else KernelSweep.PARTS
+    bad = [p for p in parts if p not in KernelSweep.PARTS]
+    if bad:
+        raise SystemExit(f"unknown --parts {bad}; choose from {','.join(KernelSweep.PARTS)}")
+    res = KernelSweep(torch.device("cuda", 0)).run(peaks, parts=parts)
     clk = clocks.stop()
-    line = {"metric": "per-kernel roofline fractions (projection sweep, decode GEMV, GAE, log-probs)",
-            "value": res["projection_sweep"]["frac_of_measured_burst"], "unit": "fraction",
+    line = {"metric": "per-kernel roofline fractions (projection sweep, decode GEMV, GAE, PPO losses, log-probs)",
+            "value": res.get("projection_sweep", {}).get("frac_of_measured_burst"), "unit": "fraction",
             "workload": KernelSweep.name, "results": res, "clocks": clk, "peaks": peaks}
     print(json.dumps(line), flush=True)
     return 0
@@ -820,6 +853,8 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default=DEFAULT_WORKLOAD)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--parts", default=None,
+                    help="kernel_sweep only: comma-separated subset of " + ",".join(KernelSweep.PARTS))
     args = ap.parse_args(argv)
     wl_cls = WORKLOADS[args.workload]
     if wl_cls is KernelSweep:

@@ -305,6 +305,66 @@ hydra_status ppo_gae(const float* rewards, const float* values, const int32_t* l
                      int64_t L, float gamma, float lam, float* advantages, float* returns,
                      void* stream);
 
+/*
+ * Update side of PPO over a scored batch (§2 "Stage 3: PPO": probability ratio r(theta),
+ * clipped surrogate L^CLIP, squared-error value loss on the returns; Algorithms 1 and 2
+ * optimise this surrogate after scoring). Per valid token t < len_s:
+ *     r_t = exp(logp_new_t - logp_old_t)
+ *     A_t = advantages_t, or with whiten = 1: (advantages_t - mean) / sqrt(M2 / n + 1e-8),
+ *           (n, mean, M2) the count, mean and sum of squared deviations of the valid
+ *           advantages (population variance M2 / n)
+ *     s_t = min(r_t A_t, clip(r_t, 1 - clip_eps, 1 + clip_eps) A_t)
+ * Outputs (all n-normalised; n from the moments):
+ *     grad_logp   fp32 [S, L]: d loss_clip / d logp_new = -r_t A_t / n where r_t A_t is the
+ *                 smaller term (ties included), else 0; 0 at t >= len_s
+ *     grad_values fp32 [S, L]: d loss_value / d values = 2 (values_t - returns_t) / n; 0 at
+ *                 t >= len_s
+ *     stats fp64 [7], device: [0] loss_clip = -(1/n) sum s_t, [1] loss_value = (1/n) sum
+ *                 (values_t - returns_t)^2, [2] share of valid tokens with |r_t - 1| >
+ *                 clip_eps, [3] approx KL (1/n) sum (logp_old_t - logp_new_t), [4] mean and
+ *                 [5] population standard deviation of the raw advantages, [6] n.
+ * The paper gives no clip range; clip_eps = 0.2 is the usual choice. A_t is a constant of
+ * the loss (no gradient flows into the advantages).
+ * Inputs logp_new, logp_old, advantages, returns, values: fp32 [S, L] row-major (row stride
+ * L), device; lengths int32 [S] in 0..L, or NULL for all L (out of range: clamped, device
+ * error 0x202). adv_moments: NULL, or device fp64 [3] = (n, mean, M2) to use instead of
+ * this batch's own (e.g. merged over data-parallel replicas); n then also normalises the
+ * losses and gradients, so replicas' losses add up to the global mean.
+ * Reductions: compensated (Kahan) fp32 within a thread, fp32 trees across threads and
+ * blocks, in a fixed order: results are bitwise reproducible for a given device and
+ * accurate to a few fp32 ulps of the sums of magnitudes; the fp64 outputs carry those
+ * values. exp overflows to inf for logp_new - logp_old
+ * > 88.
+ * workspace: device, 16-byte aligned, >= hydra_ppo_workspace_size() bytes, caller-owned;
+ * no initial contents required; calls sharing a workspace must be stream-ordered.
+ * Errors: NULL stats, or (S * L > 0) a NULL array -> HYDRA_ERR_NULL; S, L < 0 or S * L >= 2^31 ->
+ * HYDRA_ERR_SHAPE; clip_eps outside [0, 1) or whiten not 0/1 -> HYDRA_ERR_RANGE; small or
+ * misaligned workspace -> HYDRA_ERR_WORKSPACE. S * L == 0 writes stats of an empty batch
+ * (all 0). Outputs must not alias inputs.
+ */
+size_t hydra_ppo_workspace_size(void);
+hydra_status hydra_ppo_loss(const float* logp_new, const float* logp_old, const float* advantages,
+                            const float* returns, const float* values, const int32_t* lengths,
+                            int64_t S, int64_t L, float clip_eps, int whiten,
+                            const double* adv_moments, float* grad_logp, float* grad_values,
+                            double* stats, void* workspace, size_t workspace_bytes, void* stream);
+
+/* (n, mean, M2) of the valid advantages of an [S, L] batch (the moments hydra_ppo_loss
+ * whitens with), written to device fp64 [3] moments. Replicas merge their triples with the
+ * pairwise update of Chan, Golub and LeVeque (1979) and pass the result to hydra_ppo_loss
+ * as adv_moments. Arguments, workspace and errors as hydra_ppo_loss. */
+hydra_status hydra_ppo_adv_moments(const float* advantages, const int32_t* lengths, int64_t S,
+                                   int64_t L, double* moments, void* workspace,
+                                   size_t workspace_bytes, void* stream);
+
+/* Host-side merge of k moment triples (host fp64 [k][3] of (n, mean, M2), e.g. one per
+ * data-parallel replica, gathered in rank order) into one host fp64 [3] triple, by the
+ * pairwise update of Chan, Golub and LeVeque (1979) applied left to right:
+ *     n = na + nb,  mean = mean_a + d nb / n,  M2 = M2a + M2b + d^2 na nb / n,
+ * d = mean_b - mean_a. No device work. Errors: k < 0 -> HYDRA_ERR_SHAPE; NULL out (or NULL
+ * moments with k > 0) -> HYDRA_ERR_NULL; a negative or NaN n or M2 -> HYDRA_ERR_RANGE. */
+hydra_status hydra_ppo_merge_moments(const double* moments, int64_t k, double* out);
+
 /* ===================================================================================
  * Llama decoder pieces and the full scoring pass (the paper runs Llama 7b, §4; the pass
  * follows the scoring steps of Algorithm 1, J-Hydra-PPO). The LoRA-off and LoRA-on streams

@@ -406,4 +406,72 @@ hydra_status ppo_gae(const float* rewards, const float* values, const int32_t* l
              : HYDRA_ERR_CUDA;
 }
 
+static bool ppo_shape_ok(int64_t S, int64_t L) {
+  return S >= 0 && L >= 0 && S < (1LL << 31) && L < (1LL << 31) && S * L < (1LL << 31);
+}
+
+size_t hydra_ppo_workspace_size(void) { return hydra::ppo_loss_workspace_bytes(); }
+
+hydra_status hydra_ppo_adv_moments(const float* advantages, const int32_t* lengths, int64_t S,
+                                   int64_t L, double* moments, void* workspace,
+                                   size_t workspace_bytes, void* stream) {
+  if (!ppo_shape_ok(S, L)) return HYDRA_ERR_SHAPE;
+  if (moments == nullptr || (S * L > 0 && advantages == nullptr)) return HYDRA_ERR_NULL;
+  if (workspace == nullptr || workspace_bytes < hydra::ppo_loss_workspace_bytes() ||
+      reinterpret_cast<uintptr_t>(workspace) % 16 != 0)
+    return HYDRA_ERR_WORKSPACE;
+  int* err = hydra::device_error_word();
+  if (err == nullptr) return HYDRA_ERR_CUDA;
+  return hydra::launch_ppo_adv_moments(advantages, lengths, S, L, moments, workspace, err,
+                                       static_cast<cudaStream_t>(stream)) == 0
+             ? HYDRA_OK
+             : HYDRA_ERR_CUDA;
+}
+
+hydra_status hydra_ppo_loss(const float* logp_new, const float* logp_old, const float* advantages,
+                            const float* returns, const float* values, const int32_t* lengths,
+                            int64_t S, int64_t L, float clip_eps, int whiten,
+                            const double* adv_moments, float* grad_logp, float* grad_values,
+                            double* stats, void* workspace, size_t workspace_bytes,
+                            void* stream) {
+  if (!ppo_shape_ok(S, L)) return HYDRA_ERR_SHAPE;
+  if (!(clip_eps >= 0.f && clip_eps < 1.f) || (whiten != 0 && whiten != 1)) return HYDRA_ERR_RANGE;
+  if (stats == nullptr) return HYDRA_ERR_NULL;
+  if (S * L > 0 && (logp_new == nullptr || logp_old == nullptr || advantages == nullptr ||
+                    returns == nullptr || values == nullptr || grad_logp == nullptr ||
+                    grad_values == nullptr))
+    return HYDRA_ERR_NULL;
+  if (workspace == nullptr || workspace_bytes < hydra::ppo_loss_workspace_bytes() ||
+      reinterpret_cast<uintptr_t>(workspace) % 16 != 0)
+    return HYDRA_ERR_WORKSPACE;
+  int* err = hydra::device_error_word();
+  if (err == nullptr) return HYDRA_ERR_CUDA;
+  return hydra::launch_ppo_loss(logp_new, logp_old, advantages, returns, values, lengths, S, L,
+                                clip_eps, whiten != 0, adv_moments, grad_logp, grad_values, stats,
+                                workspace, err, static_cast<cudaStream_t>(stream)) == 0
+             ? HYDRA_OK
+             : HYDRA_ERR_CUDA;
+}
+
+hydra_status hydra_ppo_merge_moments(const double* moments, int64_t k, double* out) {
+  if (k < 0) return HYDRA_ERR_SHAPE;
+  if (out == nullptr || (k > 0 && moments == nullptr)) return HYDRA_ERR_NULL;
+  double n = 0.0, mean = 0.0, m2 = 0.0;
+  for (int64_t i = 0; i < k; ++i) {
+    const double nb = moments[3 * i], mb = moments[3 * i + 1], m2b = moments[3 * i + 2];
+    if (!(nb >= 0.0) || !(m2b >= 0.0)) return HYDRA_ERR_RANGE;
+    const double nn = n + nb;
+    if (nn == 0.0) continue;
+    const double d = mb - mean;
+    const double f = nb / nn;
+    mean += d * f;
+    m2 += m2b + d * d * n * f;
+    n = nn;
+  }
+  out[0] = n;
+  out[1] = mean;
+  out[2] = m2;
+  return HYDRA_OK;
+}
+
 }  // extern "C"

@@ -95,6 +95,19 @@ int launch_token_logprobs_kl(const void* za, const void* zr, int bf16_logits, in
 int launch_gae(const float* r, const float* v, const int32_t* lengths, int64_t S, int64_t L,
                float gamma, float lam, float* adv, float* ret, int* err, cudaStream_t stream);
 
+// PPO update-side losses (ppo_loss.cu). ext_moments (device [n, mean, M2]) or NULL.
+size_t ppo_loss_workspace_bytes();
+int launch_ppo_adv_moments(const float* adv, const int32_t* lengths, int64_t S, int64_t L,
+                           double* out, void* ws, int* err, cudaStream_t st);
+int launch_ppo_loss(const float* logp_new, const float* logp_old, const float* adv,
+                    const float* ret, const float* val, const int32_t* lengths, int64_t S,
+                    int64_t L, float eps, bool whiten, const double* ext_moments,
+                    float* grad_logp, float* grad_val, double* stats, void* ws, int* err,
+                    cudaStream_t st);
+// Blocks of the two PPO passes (one fp64 partial per block lives in the workspace).
+constexpr int kPpoMaxMomentBlocks = 1024;
+constexpr int kPpoMaxLossBlocks = 1024;
+
 // Row gather used by the per-row Llama kernels: output row i reads input row
 // (i / g_out) * g_in + off + i % g_out (g_out = g_in, off = 0 is the identity).
 struct RowMap {

@@ -57,6 +57,12 @@ _SIGNATURES = {
                                                _vp, _vp, _vp, _vp]),
     "ppo_gae": (ctypes.c_int, [_vp, _vp, _vp, _c_i64, _c_i64, ctypes.c_float, ctypes.c_float, _vp,
                                _vp, _vp]),
+    "hydra_ppo_workspace_size": (ctypes.c_size_t, []),
+    "hydra_ppo_loss": (ctypes.c_int, [_vp, _vp, _vp, _vp, _vp, _vp, _c_i64, _c_i64, ctypes.c_float,
+                                      ctypes.c_int, _vp, _vp, _vp, _vp, _vp, ctypes.c_size_t, _vp]),
+    "hydra_ppo_adv_moments": (ctypes.c_int, [_vp, _vp, _c_i64, _c_i64, _vp, _vp, ctypes.c_size_t,
+                                             _vp]),
+    "hydra_ppo_merge_moments": (ctypes.c_int, [_vp, _c_i64, _vp]),
 }
 
 
@@ -374,6 +380,70 @@ def ppo_gae(rewards, values, lengths, gamma, lam, advantages, returns, stream=No
     S, L = rewards.shape
     _check("ppo_gae", load().ppo_gae(_p(rewards), _p(values), _p(lengths), S, L, float(gamma),
                                      float(lam), _p(advantages), _p(returns), _stream(stream)))
+
+
+PPO_STATS = ("loss_clip", "loss_value", "clip_frac", "approx_kl", "adv_mean", "adv_std", "n")
+
+
+def ppo_workspace_size():
+    return int(load().hydra_ppo_workspace_size())
+
+
+def hydra_ppo_loss(logp_new, logp_old, advantages, returns, values, lengths, clip_eps, whiten,
+                   grad_logp, grad_values, stats, workspace, adv_moments=None, stream=None):
+    """Clipped surrogate, value loss and their gradients over [S, L] fp32 tensors; stats is a
+    device fp64 [7] tensor (order PPO_STATS); adv_moments an optional device fp64 [3]."""
+    for t, n in ((logp_new, "logp_new"), (logp_old, "logp_old"), (advantages, "advantages"),
+                 (returns, "returns"), (values, "values"), (grad_logp, "grad_logp"),
+                 (grad_values, "grad_values")):
+        _req(t, torch.float32, n)
+    _req(lengths, torch.int32, "lengths")
+    _req(stats, torch.float64, "stats")
+    _req(adv_moments, torch.float64, "adv_moments")
+    S, L = logp_new.shape
+    _check("hydra_ppo_loss", load().hydra_ppo_loss(
+        _p(logp_new), _p(logp_old), _p(advantages), _p(returns), _p(values), _p(lengths), S, L,
+        float(clip_eps), int(bool(whiten)), _p(adv_moments), _p(grad_logp), _p(grad_values),
+        _p(stats), _p(workspace), workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def hydra_ppo_adv_moments(advantages, lengths, moments, workspace, stream=None):
+    """(n, mean, M2) of the valid advantages into the device fp64 [3] tensor moments."""
+    _req(advantages, torch.float32, "advantages")
+    _req(lengths, torch.int32, "lengths")
+    _req(moments, torch.float64, "moments")
+    S, L = advantages.shape
+    _check("hydra_ppo_adv_moments", load().hydra_ppo_adv_moments(
+        _p(advantages), _p(lengths), S, L, _p(moments), _p(workspace),
+        workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def ppo_merge_moments(triples):
+    """Merge host (n, mean, M2) triples (a [k, 3] fp64 CPU tensor, rank order) in the library."""
+    t = torch.as_tensor(triples, dtype=torch.float64).contiguous().reshape(-1, 3)
+    out = torch.zeros(3, dtype=torch.float64)
+    _check("hydra_ppo_merge_moments", load().hydra_ppo_merge_moments(
+        t.data_ptr() if t.numel() else None, t.shape[0], out.data_ptr()))
+    return out
+
+
+def all_reduce_adv_moments(moments, group=None):
+    """Replace each rank's (n, mean, M2) by the merge over all ranks (all_gather of three
+    doubles, merged in rank order on the host, so every rank gets the same bits)."""
+    import torch.distributed as dist
+    host = moments.detach().to("cpu", torch.float64).reshape(3)
+    world = dist.get_world_size(group)
+    parts = [torch.zeros(3, dtype=torch.float64) for _ in range(world)]
+    if dist.get_backend(group) == "nccl":
+        dev = moments.device
+        gathered = [torch.zeros(3, dtype=torch.float64, device=dev) for _ in range(world)]
+        dist.all_gather(gathered, host.to(dev), group=group)
+        parts = [g.cpu() for g in gathered]
+    else:
+        dist.all_gather(parts, host, group=group)
+    merged = ppo_merge_moments(torch.stack(parts))
+    moments.copy_(merged.to(moments.device))
+    return moments
 
 
 # ----------------------------------------------------------------------------- Llama pieces

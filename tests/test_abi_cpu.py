@@ -108,3 +108,44 @@ def test_logprobs_and_gae_argument_errors(lib):
     assert lib.hydra_lora_down(FAKE, 4, 8, FAKE, 4, 1.0, FAKE, None) == 3
     code = ctypes.c_int32(0)
     assert lib.hydra_device_error(None, 0) == 1
+
+
+def test_ppo_loss_argument_errors(lib):
+    ws = H.ppo_workspace_size()
+    assert ws >= 16 * 512 + 32 * 1024
+    f = lib.hydra_ppo_loss
+    args = lambda S=4, L=8, eps=0.2, wh=0, stats=FAKE, a=FAKE, wsb=ws, wsp=FAKE: f(
+        a, FAKE, FAKE, FAKE, FAKE, None, S, L, eps, wh, None, FAKE, FAKE, stats, wsp, wsb, None)
+    assert args(S=-1) == 2
+    assert args(S=1 << 16, L=1 << 15) == 2  # S * L >= 2^31
+    assert args(eps=-0.1) == 4 and args(eps=1.0) == 4 and args(eps=float("nan")) == 4
+    assert args(wh=2) == 4
+    assert args(stats=None) == 1
+    assert args(a=None) == 1
+    assert args(wsb=ws - 8) == 7 and args(wsp=None) == 7 and args(wsp=FAKE + 8) == 7
+    m = lib.hydra_ppo_adv_moments
+    assert m(FAKE, None, -1, 4, FAKE, FAKE, ws, None) == 2
+    assert m(FAKE, None, 2, 4, None, FAKE, ws, None) == 1
+    assert m(FAKE, None, 2, 4, FAKE, FAKE, 16, None) == 7
+
+
+def test_ppo_merge_moments_matches_whole_batch(lib):
+    """The host merge of per-shard (n, mean, M2) triples equals the moments of the whole
+    batch (numpy mean and population variance), whatever the split, including empty shards."""
+    import numpy as np
+    import torch
+    rng = np.random.default_rng(7)
+    x = rng.normal(3.0, 2.0, 1000)
+    for cuts in ([0, 1000], [0, 1, 999, 1000], [0, 300, 300, 700, 1000], [0, 0, 1000]):
+        tri = []
+        for a, b in zip(cuts[:-1], cuts[1:]):
+            s = x[a:b]
+            m = s.mean() if len(s) else 0.0
+            tri.append([len(s), m, ((s - m) ** 2).sum()])
+        out = H.ppo_merge_moments(torch.tensor(tri, dtype=torch.float64)).numpy()
+        assert out[0] == 1000
+        assert abs(out[1] - x.mean()) < 1e-13
+        assert abs(out[2] / 1000 - x.var()) < 1e-12
+    assert H.ppo_merge_moments(torch.zeros(0, 3, dtype=torch.float64)).tolist() == [0.0, 0.0, 0.0]
+    with pytest.raises(H.HydraError):
+        H.ppo_merge_moments(torch.tensor([[-1.0, 0.0, 0.0]], dtype=torch.float64))
