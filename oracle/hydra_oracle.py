@@ -30,6 +30,8 @@ Readings where the paper is silent (the same readings the CUDA path implements):
   * Per-token KL penalty uses the sampled-token estimate logp_actor - logp_ref; the
     sequence score is added at the last valid token t = len - 1.
   * GAE: the value after the last valid token is 0 (terminal); positions >= len are 0.
+  * Sampling: the paper does not say how tokens are drawn; temperature 1 sampling from the
+    actor's softmax by the Gumbel-max trick, with the noise passed in (greedy without it).
   * PPO update side: the paper gives no clip range; eps = 0.2 (the PPO paper's default) is
     an argument. Losses are means over the valid tokens of the batch; the surrogate is
     negated so both losses are minimised. Advantage whitening (optional, off by default)
@@ -43,6 +45,11 @@ The full 32-layer Llama composition (`llama_score`, and the three-stream Hydra-P
 `llama_score_hydra`) is pinned only through its per-op pieces and small-size invariants
 (LoRA off, causality, one LoRA set reducing Hydra-PPO to J-Hydra-PPO, a critic set that
 moves only the values): parity unpinned for the composition as a whole.
+Generation (`llama_generate`, Alg. 1 and 2 "generate sequence ... for T steps") recomputes
+the whole stack at every step, with no cache, and draws each token by the Gumbel-max trick
+from noise that is an input (`gumbel_argmax`, pinned by the empirical distribution of its
+draws). It is pinned by its equality with `llama_score` on the finished sequence, so it
+inherits that composition's "parity unpinned".
 """
 from __future__ import annotations
 
@@ -257,31 +264,16 @@ def swiglu(g, u):
     return silu(g) * u
 
 
-def llama_score(weights, ids, prompt_len, cfg, seq_lengths=None, beta=0.1, gamma=1.0,
-                lam=0.95, n_layers=None):
-    """One sequence of the full J-Hydra scoring pass (Alg. 1 scoring steps), both streams.
-
-    weights: dict of float64 arrays (exact bf16 values):
-      embed [V, d]; per layer l: wq, wk, wv, wo [d, d]; wg, wu [F, d]; wd [d, F];
-      norm1, norm2 [d]; lora[name] = (A [r, in], B [out, r]) for name in q, v, g, u, d;
-      final_norm [d]; lm_head [V, d]; w_rm [d].
-    ids: [T] token ids (prompt then response); prompt_len P; response tokens are P..T-1.
-    Returns dict with logp_actor, logp_ref, reward, values, score, advantages, returns
-    (arrays of length T-P for the response) and the final normed hidden states.
-
-    Streams: "off" = LoRA ignored (reference policy and reward model, §3 Dynamic LoRA);
-    "on" = actor/critic with the single J-Hydra LoRA set (§3 J-Hydra-PPO).
-    Values: V_t = w_rm . h_on[p_t - 1]; score = w_rm . h_off[T - 1] (reward-model head on
-    the LoRA-off stream, critic = same head with LoRA on).
-    """
+def llama_final_hidden(weights, ids, cfg, n_layers=None):
+    """Final normed hidden states (bf16 values) of both streams at every position of one
+    sequence: the decoder stack of the J-Hydra model (LoRA off / on, §3 Dynamic LoRA), as
+    used by llama_score; row p is the state after token p, which predicts token p + 1."""
     d = cfg["d"]
     H = cfg["n_heads"]
     Dh = d // H
     eps = cfg["eps"]
     s = cfg["lora_scale"]
     T = len(ids)
-    P = prompt_len
-    L = T - P
     n_layers = cfg["n_layers"] if n_layers is None else n_layers
     pos = np.arange(T)
 
@@ -322,6 +314,30 @@ def llama_score(weights, ids, prompt_len, cfg, seq_lengths=None, beta=0.1, gamma
 
     f_off = round_bf16(rmsnorm(h_off, weights["final_norm"], eps))
     f_on = round_bf16(rmsnorm(h_on, weights["final_norm"], eps))
+    return f_off, f_on
+
+
+def llama_score(weights, ids, prompt_len, cfg, seq_lengths=None, beta=0.1, gamma=1.0,
+                lam=0.95, n_layers=None):
+    """One sequence of the full J-Hydra scoring pass (Alg. 1 scoring steps), both streams.
+
+    weights: dict of float64 arrays (exact bf16 values):
+      embed [V, d]; per layer l: wq, wk, wv, wo [d, d]; wg, wu [F, d]; wd [d, F];
+      norm1, norm2 [d]; lora[name] = (A [r, in], B [out, r]) for name in q, v, g, u, d;
+      final_norm [d]; lm_head [V, d]; w_rm [d].
+    ids: [T] token ids (prompt then response); prompt_len P; response tokens are P..T-1.
+    Returns dict with logp_actor, logp_ref, reward, values, score, advantages, returns
+    (arrays of length T-P for the response) and the final normed hidden states.
+
+    Streams: "off" = LoRA ignored (reference policy and reward model, §3 Dynamic LoRA);
+    "on" = actor/critic with the single J-Hydra LoRA set (§3 J-Hydra-PPO).
+    Values: V_t = w_rm . h_on[p_t - 1]; score = w_rm . h_off[T - 1] (reward-model head on
+    the LoRA-off stream, critic = same head with LoRA on).
+    """
+    P = prompt_len
+    T = len(ids)
+    L = T - P
+    f_off, f_on = llama_final_hidden(weights, ids, cfg, n_layers)
     rows = np.arange(P - 1, T - 1)                       # hidden row predicting token P+t
     z_ref = f_off[rows] @ weights["lm_head"].T
     z_act = f_on[rows] @ weights["lm_head"].T
@@ -474,3 +490,52 @@ def ppo_loss(logp_new, logp_old, adv, returns, values, lengths, clip_eps=0.2, wh
         "grad_logp": np.where(valid & (unclipped <= clip_term), -unclipped * inv_n, 0.0),
         "grad_values": np.where(valid, 2.0 * dv * inv_n, 0.0),
     }
+
+
+# ---------------------------------------------------------------------------
+# Generation with the actor (Alg. 1 and 2: "generate sequence using the policy for T steps";
+# J-Hydra-PPO retains the critic head's values while generating)
+# ---------------------------------------------------------------------------
+
+
+def gumbel_argmax(z, g=None):
+    """One draw from softmax(z) by the Gumbel-max trick (Gumbel 1954; Maddison, Tarlow and
+    Minka 2014): argmax_k (z_k + g_k) with g_k i.i.d. standard Gumbel (-log(-log U)). The
+    noise is an input; g None is the greedy argmax. Ties go to the lowest index."""
+    z = np.asarray(z, dtype=np.float64)
+    return int(np.argmax(z if g is None else z + np.asarray(g, dtype=np.float64)))
+
+
+def llama_generate(weights, prompt_ids, n_steps, cfg, gumbel=None, n_layers=None):
+    """Autoregressive generation of n_steps tokens after the prompt with the LoRA-on actor,
+    recording under both streams the log-probability of each drawn token and the J-Hydra
+    value of the state it is drawn from. No cache: step t runs the whole decoder stack over
+    the prompt and the t tokens drawn so far (the plain definition of a causal model's
+    next-token distribution) and reads the last position p = P0 + t - 1:
+      z_on = lm_head f_on[p], z_off = lm_head f_off[p]
+      token_t      = argmax_k (z_on[k] + gumbel[t, k])   (greedy when gumbel is None)
+      logp_actor_t = log_softmax(z_on)[token_t],  logp_ref_t = log_softmax(z_off)[token_t]
+      value_t      = w_rm . f_on[p]
+    score = w_rm . f_off at the last drawn token (one more pass over the whole sequence).
+    These are llama_score's logp_actor, logp_ref, values and score on the generated
+    sequence. gumbel: [n_steps, V] or None. Returns a dict of tokens (int array),
+    logp_actor, logp_ref, values (length n_steps) and score."""
+    ids = [int(t) for t in prompt_ids]
+    P = len(ids)
+    out = {k: np.zeros(n_steps) for k in ("logp_actor", "logp_ref", "values")}
+    tokens = np.zeros(n_steps, dtype=np.int64)
+    for t in range(n_steps):
+        f_off, f_on = llama_final_hidden(weights, ids, cfg, n_layers)
+        z_on = f_on[-1] @ weights["lm_head"].T
+        z_off = f_off[-1] @ weights["lm_head"].T
+        tok = gumbel_argmax(z_on, None if gumbel is None else gumbel[t])
+        out["logp_actor"][t] = z_on[tok] - logsumexp_rows(z_on[None])[0]
+        out["logp_ref"][t] = z_off[tok] - logsumexp_rows(z_off[None])[0]
+        out["values"][t] = float(f_on[-1] @ weights["w_rm"])
+        tokens[t] = tok
+        ids.append(tok)
+    f_off, _ = llama_final_hidden(weights, ids, cfg, n_layers)
+    out["score"] = float(f_off[-1] @ weights["w_rm"])
+    out["tokens"] = tokens
+    out["prompt_len"] = P
+    return out

@@ -507,3 +507,53 @@ def test_ppo_loss_shards_with_merged_moments_add_up():
             assert abs(p0[k] + p1[k] - full[k]) < 1e-12, k
         np.testing.assert_allclose(np.vstack([p0["grad_logp"], p1["grad_logp"]]), full["grad_logp"],
                                    atol=1e-15)
+
+
+# ------------------------------------------------------------------ generation
+
+
+def test_gumbel_argmax_draws_follow_softmax():
+    """The Gumbel-max trick: argmax(z + g), g standard Gumbel, is a draw from softmax(z).
+    200k draws with numpy's own Gumbel noise: every empirical frequency within 5 sigma."""
+    z = np.array([1.5, -0.5, 0.0, 2.2, -3.0])
+    p = scipy.special.softmax(z)
+    rng = np.random.default_rng(5)
+    N = 200_000
+    g = -np.log(-np.log(rng.random((N, z.size))))
+    counts = np.bincount(np.argmax(z + g, axis=1), minlength=z.size)
+    draws = np.array([O.gumbel_argmax(z, g[i]) for i in range(2000)])
+    assert np.array_equal(draws, np.argmax(z + g[:2000], axis=1))
+    sigma = np.sqrt(N * p * (1 - p))
+    assert np.all(np.abs(counts - N * p) < 5 * sigma), (counts, N * p)
+    assert O.gumbel_argmax(z) == 3
+    assert O.gumbel_argmax(np.array([1.0, 3.0, 3.0])) == 1  # ties: lowest index
+
+
+@pytest.mark.parametrize("noise", [False, True])
+def test_generate_is_the_scoring_pass_on_its_own_sequence(noise):
+    """Each step's distribution is that of the last position of a full causal pass: the
+    recorded log-probs, values and score equal llama_score's on the finished sequence, and
+    every token is the argmax of that position's actor logits plus the step's noise."""
+    w, cfg = tiny_llama(seed=21)
+    rng = np.random.default_rng(22)
+    prompt = rng.integers(0, 64, size=5)
+    n = 7
+    g = -np.log(-np.log(rng.random((n, 64)))) if noise else None
+    gen = O.llama_generate(w, prompt, n, cfg, gumbel=g)
+    seq = np.concatenate([prompt, gen["tokens"]])
+    ref = O.llama_score(w, seq, 5, cfg)
+    for k in ("logp_actor", "logp_ref", "values"):
+        np.testing.assert_allclose(gen[k], ref[k], rtol=0, atol=1e-12)
+    assert abs(gen["score"] - ref["score"]) < 1e-12
+    z_on = ref["h_on"][4:4 + n] @ w["lm_head"].T
+    expect = np.argmax(z_on + (0.0 if g is None else g), axis=1)
+    assert np.array_equal(gen["tokens"], expect)
+    # log-probabilities are normalised distributions' entries
+    assert np.all(gen["logp_actor"] <= 0) and np.all(gen["logp_ref"] <= 0)
+
+
+def test_generate_lora_off_streams_agree():
+    w, cfg = tiny_llama(seed=23, zero_B=True)
+    prompt = np.random.default_rng(24).integers(0, 64, size=3)
+    gen = O.llama_generate(w, prompt, 4, cfg)
+    np.testing.assert_array_equal(gen["logp_actor"], gen["logp_ref"])
