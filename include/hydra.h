@@ -465,6 +465,43 @@ typedef struct hydra_llama_lora {
   const void* b_down;
 } hydra_llama_lora;
 
+/* Workspace bytes of hydra_generate_llama for S sequences (0 for an unsupported
+ * configuration or S outside 1..8). */
+size_t hydra_generate_llama_workspace_size(const hydra_llama_config* cfg, int64_t S);
+
+/*
+ * Generation with the actor (Algorithms 1 and 2: "generate sequence using the policy for T
+ * steps"; J-Hydra-PPO retains the critic head's values while generating), KV-cached, with
+ * the LoRA-off stream decoded beside the actor so that each drawn token also gets its
+ * reference log-probability (one read of W serves both streams' rows).
+ * For each of S sequences of P0 = cfg->prompt_len prompt tokens and steps t < n_steps:
+ *   z_on, z_off = LM head of the final normed hidden state at position P0 + t - 1 of the
+ *                 LoRA-on and LoRA-off streams (fp32 logits)
+ *   tokens[s, t]     = argmax_k (z_on[k] + gumbel[t, s, k])   (greedy argmax if gumbel is
+ *                      NULL; ties to the lowest k). With standard Gumbel noise this is a
+ *                      draw from softmax(z_on) (Gumbel-max); the noise is the caller's.
+ *   logp_actor[s, t] = log_softmax(z_on)[token],  logp_ref[s, t] = log_softmax(z_off)[token]
+ *   values[s, t]     = w_rm . h_on at position P0 + t - 1 (J-Hydra: r_phi = LO(V))
+ *   score[s]         = w_rm . h_off at position P0 + n_steps - 1 (the reward model on the
+ *                      state after the last drawn token; one more decode pass), if score
+ *                      is not NULL.
+ * These equal hydra_score_llama's logp_actor, logp_ref, values and score on the finished
+ * sequence (prompt + tokens). Weights as hydra_score_llama (fused layouts).
+ * prompt_ids int32 [S, P0]; gumbel fp32 [n_steps, S, V] or NULL; outputs int32 / fp32
+ * [S, n_steps] and fp32 [S]; all device. Requirements: as hydra_score_llama, plus
+ * 1 <= S <= 8, 1 <= n_steps <= cfg->response_len (the cache holds P0 + response_len
+ * positions; its scores fit shared memory for P0 + response_len up to about 50,000).
+ * workspace: device, 16-byte aligned, >= hydra_generate_llama_workspace_size(cfg, S).
+ * Errors: NULL pointer -> HYDRA_ERR_NULL; configuration or sizes outside the above ->
+ * HYDRA_ERR_SHAPE; misaligned weight or workspace -> HYDRA_ERR_ALIGN; small workspace ->
+ * HYDRA_ERR_WORKSPACE; token id out of range -> device error 0x201.
+ */
+hydra_status hydra_generate_llama(const hydra_llama_config* cfg, const hydra_llama_weights* w,
+                                  const int32_t* prompt_ids, int64_t S, int64_t n_steps,
+                                  const float* gumbel, void* workspace, size_t workspace_bytes,
+                                  int32_t* tokens, float* logp_actor, float* logp_ref,
+                                  float* values, float* score, void* stream);
+
 /* Workspace bytes of hydra_score_llama for S sequences. */
 size_t hydra_score_llama_workspace_size(const hydra_llama_config* cfg, int64_t S);
 

@@ -108,6 +108,40 @@ int launch_ppo_loss(const float* logp_new, const float* logp_old, const float* a
 constexpr int kPpoMaxMomentBlocks = 1024;
 constexpr int kPpoMaxLossBlocks = 1024;
 
+// The full pass's stacked linear over ns row-stacked streams (score_llama.cu): rows [0, T)
+// of x are the LoRA-off stream, [T, 2T) the LoRA-on stream (LoRA set A, B; u receives its
+// down-projection) and, for ns == 3, [2T, 3T) a third stream with the set A2, B2 (u2). epi:
+// HYDRA_EPI_* or kStackEpiRope with rope's arguments; y as the tcgen05 GEMM's epilogue
+// writes it. prof_class: the HYDRA_PROF_* class its launches are timed under.
+constexpr int kStackEpiRope = 3;
+struct StackRope {
+  int64_t P, cols;
+  const void* table;  // (cos, sin) [P][head_dim / 2]
+};
+int stacked_linear(int prof_class, const void* x, int64_t T, int64_t K, int64_t N, const void* W,
+                   const void* A, const void* B, int64_t r, float s, void* u, void* y, bool f32,
+                   int* err, cudaStream_t st, int epi = 0, const StackRope* rope = nullptr,
+                   int ns = 2, const void* A2 = nullptr, const void* B2 = nullptr,
+                   void* u2 = nullptr);
+
+// Generation loop kernels (decode.cu). Cache per layer: K then V, each [R][H][Pmax][128]
+// bf16; step: device counter of the current draw (the new token sits at P0 + step - 1).
+int launch_kv_store_prefill(const void* qkv, int64_t R, int64_t P0, int64_t ld, int64_t d,
+                            int64_t H, int64_t Pmax, void* ck, void* cv, cudaStream_t st);
+int launch_decode_rope_append(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t H,
+                              const void* table, int64_t P0, const int* step, int64_t Pmax,
+                              void* ck, void* cv, cudaStream_t st);
+size_t decode_attention_smem(int64_t Pmax);
+int launch_decode_attention(const void* qkv, int64_t R, int64_t ld, int64_t H, const void* ck,
+                            const void* cv, int64_t P0, const int* step, int64_t Pmax, void* out,
+                            int64_t ld_out, cudaStream_t st);
+int launch_swiglu_blocked(const void* gu, int64_t R, int64_t F, void* m, cudaStream_t st);
+int launch_sample_tokens(const float* logits, int64_t S, int64_t V, const float* gumbel,
+                         const void* fin, int64_t d, const void* w_rm, const int* step,
+                         int64_t n_steps, int32_t* tokens, float* logp_a, float* logp_r,
+                         float* values, int32_t* cur_ids, cudaStream_t st);
+int launch_step_advance(int* step, cudaStream_t st);
+
 // Row gather used by the per-row Llama kernels: output row i reads input row
 // (i / g_out) * g_in + off + i % g_out (g_out = g_in, off = 0 is the identity).
 struct RowMap {

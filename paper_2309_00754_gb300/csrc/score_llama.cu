@@ -105,17 +105,12 @@ bool valid_config(const hydra_llama_config* c) {
 // (actor) stream and, when ns == 3, [2T, 3T) the critic stream with its own LoRA set
 // (A2, B2; u2 receives its down-projection)
 // epi: tcgen05 epilogue; y is [ns T, N] (store, rotary), [ns T, N/2] bf16 (SwiGLU) or the
-// fp32 residual stream [ns T, N] (residual add); rope: rotary arguments of epi == kEpiRope
-constexpr int kEpiRope = 3;
-struct RopeCfg {
-  int64_t P, cols;
-  const void* table;  // (cos, sin) [P][head_dim / 2]
-};
-int stacked_linear(int prof_class, const void* x, int64_t T, int64_t K, int64_t N, const void* W,
-                   const void* A, const void* B, int64_t r, float s, void* u, void* y, bool f32,
-                   int* err, cudaStream_t st, int epi = HYDRA_EPI_STORE,
-                   const RopeCfg* rope = nullptr, int ns = 2, const void* A2 = nullptr,
-                   const void* B2 = nullptr, void* u2 = nullptr) {
+// fp32 residual stream [ns T, N] (residual add); rope: rotary arguments of epi == kStackEpiRope
+int stacked_linear_impl(int prof_class, const void* x, int64_t T, int64_t K, int64_t N,
+                        const void* W, const void* A, const void* B, int64_t r, float s, void* u,
+                        void* y, bool f32, int* err, cudaStream_t st, int epi,
+                        const hydra::StackRope* rope, int ns, const void* A2, const void* B2,
+                        void* u2) {
   const size_t xs = static_cast<size_t>(T) * K * 2;
   const size_t ys = epi == HYDRA_EPI_SWIGLU    ? static_cast<size_t>(T) * (N / 2) * 2
                     : epi == HYDRA_EPI_RESIDUAL ? static_cast<size_t>(T) * N * 4
@@ -161,6 +156,16 @@ int stacked_linear(int prof_class, const void* x, int64_t T, int64_t K, int64_t 
 }
 
 }  // namespace
+
+namespace hydra {
+int stacked_linear(int prof_class, const void* x, int64_t T, int64_t K, int64_t N, const void* W,
+                   const void* A, const void* B, int64_t r, float s, void* u, void* y, bool f32,
+                   int* err, cudaStream_t st, int epi, const StackRope* rope, int ns,
+                   const void* A2, const void* B2, void* u2) {
+  return stacked_linear_impl(prof_class, x, T, K, N, W, A, B, r, s, u, y, f32, err, st, epi, rope,
+                             ns, A2, B2, u2);
+}
+}  // namespace hydra
 
 extern "C" {
 
@@ -354,19 +359,19 @@ static hydra_status score_pass(const hydra_llama_config* cfg, const hydra_llama_
     // attention block
     HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(h, ly.norm_attn, R, d, c.rms_eps, ident, a, st));
     // q/k/v projection with the rotary embedding of q and k fused into the epilogue
-    const RopeCfg rope{P, 2 * d, rope_table};
-    HY_TRY(stacked_linear(HYDRA_PROF_GEMM_QKV, a, T, d, 3 * d, ly.w_qkv, ly.a_qv, ly.b_qkv, 2 * r, s, u, qkv, false,
-                          err, st, kEpiRope, &rope, ns, cl ? cl->a_qv : nullptr, cl ? cl->b_qkv : nullptr, u2));
+    const hydra::StackRope rope{P, 2 * d, rope_table};
+    HY_TRY(hydra::stacked_linear(HYDRA_PROF_GEMM_QKV, a, T, d, 3 * d, ly.w_qkv, ly.a_qv, ly.b_qkv, 2 * r, s, u, qkv, false,
+                          err, st, hydra::kStackEpiRope, &rope, ns, cl ? cl->a_qv : nullptr, cl ? cl->b_qkv : nullptr, u2));
     HY_PROF(HYDRA_PROF_ATTENTION,
             hydra::launch_causal_attention(qkv, ns * S, P, 3 * d, c.n_heads, c.head_dim, attn, d, st));
     // o projection added straight into the residual stream (fused epilogue)
-    HY_TRY(stacked_linear(HYDRA_PROF_GEMM_O, attn, T, d, d, ly.w_o, nullptr, nullptr, 0, s, u, h, false, err, st,
+    HY_TRY(hydra::stacked_linear(HYDRA_PROF_GEMM_O, attn, T, d, d, ly.w_o, nullptr, nullptr, 0, s, u, h, false, err, st,
                           HYDRA_EPI_RESIDUAL, nullptr, ns));
     // feed-forward block: gate/up with the SwiGLU fused into the epilogue, down added into h
     HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(h, ly.norm_ffn, R, d, c.rms_eps, ident, a, st));
-    HY_TRY(stacked_linear(HYDRA_PROF_GEMM_GU, a, T, d, 2 * F, ly.w_gu, ly.a_gu, ly.b_gu, 2 * r, s, u, m, false, err, st,
+    HY_TRY(hydra::stacked_linear(HYDRA_PROF_GEMM_GU, a, T, d, 2 * F, ly.w_gu, ly.a_gu, ly.b_gu, 2 * r, s, u, m, false, err, st,
                           HYDRA_EPI_SWIGLU, nullptr, ns, cl ? cl->a_gu : nullptr, cl ? cl->b_gu : nullptr, u2));
-    HY_TRY(stacked_linear(HYDRA_PROF_GEMM_DOWN, m, T, F, d, ly.w_down, ly.a_down, ly.b_down, r, s, u, h, false, err, st,
+    HY_TRY(hydra::stacked_linear(HYDRA_PROF_GEMM_DOWN, m, T, F, d, ly.w_down, ly.a_down, ly.b_down, r, s, u, h, false, err, st,
                           HYDRA_EPI_RESIDUAL, nullptr, ns, cl ? cl->a_down : nullptr, cl ? cl->b_down : nullptr, u2));
   }
   // final norm on the rows that predict response tokens: row P0 - 1 + t of each sequence

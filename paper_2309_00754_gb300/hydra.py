@@ -104,6 +104,12 @@ _SIGNATURES.update({
     "hydra_profile_enable": (ctypes.c_int, [ctypes.c_int]),
     "hydra_profile_collect": (ctypes.c_int, [ctypes.POINTER(ctypes.c_float),
                                              ctypes.POINTER(ctypes.c_int64), ctypes.c_int]),
+    "hydra_generate_llama_workspace_size": (ctypes.c_size_t, [ctypes.POINTER(LlamaConfigC),
+                                                              _c_i64]),
+    "hydra_generate_llama": (ctypes.c_int, [ctypes.POINTER(LlamaConfigC),
+                                            ctypes.POINTER(LlamaWeightsC), _vp, _c_i64, _c_i64,
+                                            _vp, _vp, ctypes.c_size_t, _vp, _vp, _vp, _vp, _vp,
+                                            _vp]),
     "hydra_score_llama_workspace_size": (ctypes.c_size_t, [ctypes.POINTER(LlamaConfigC),
                                                            _c_i64]),
     "hydra_score_llama": (ctypes.c_int, [ctypes.POINTER(LlamaConfigC),
@@ -593,6 +599,33 @@ def hydra_score_llama(cfg, weights, ids, lengths, workspace, outputs, stream=Non
     _check("hydra_score_llama", load().hydra_score_llama(
         ctypes.byref(c), ctypes.byref(w), _p(ids), _p(lengths), S, _p(workspace), ws_bytes,
         *[_p(outputs[k]) for k in names], _stream(stream)))
+
+
+def generate_llama_workspace_size(cfg, S):
+    c = llama_config_c(cfg)
+    return int(load().hydra_generate_llama_workspace_size(ctypes.byref(c), S))
+
+
+def hydra_generate_llama(cfg, weights, prompt_ids, n_steps, gumbel, workspace, outputs,
+                         stream=None):
+    """KV-cached generation with the actor plus the LoRA-off stream. prompt_ids int32
+    [S, P0]; gumbel fp32 [n_steps, S, V] or None (greedy); outputs: dict with int32 tokens
+    and fp32 logp_actor, logp_ref, values [S, n_steps], and fp32 score [S] or None."""
+    c = llama_config_c(cfg)
+    w, _layers = _weights_c(cfg, weights)
+    _req(prompt_ids, torch.int32, "prompt_ids")
+    _req(gumbel, torch.float32, "gumbel")
+    _req(outputs["tokens"], torch.int32, "tokens")
+    for k in ("logp_actor", "logp_ref", "values"):
+        _req(outputs[k], torch.float32, k)
+    _req(outputs.get("score"), torch.float32, "score")
+    S = prompt_ids.shape[0]
+    ws_bytes = workspace.numel() * workspace.element_size()
+    _check("hydra_generate_llama", load().hydra_generate_llama(
+        ctypes.byref(c), ctypes.byref(w), _p(prompt_ids), S, int(n_steps), _p(gumbel),
+        _p(workspace), ws_bytes, _p(outputs["tokens"]), _p(outputs["logp_actor"]),
+        _p(outputs["logp_ref"]), _p(outputs["values"]), _p(outputs.get("score")),
+        _stream(stream)))
 
 
 PROF_CLASSES = ("gemm_qkv", "gemm_o", "gemm_gu", "gemm_down", "gemm_lmhead", "lora_down",

@@ -1,0 +1,177 @@
+"""GPU parity of the KV-cached generation loop (hydra_generate_llama) against the fp64
+oracle, through the C-ABI.
+
+Which token is drawn depends on floating point where two candidates' logits-plus-noise
+nearly tie, so the drawn sequence is not compared with the oracle's own draws. Instead:
+- the oracle scores the GPU's finished sequence (prompt + drawn tokens; llama_score, the
+  definition each step must equal), and the recorded log-probabilities, values and score
+  must match it within the scoring pass's tolerances;
+- every drawn token must be a valid draw: its oracle logit plus the step's noise is within
+  TOL_DRAW of the maximum over the vocabulary.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2309_00754_gb300 import build as Bld
+from paper_2309_00754_gb300 import hydra as H
+from paper_2309_00754_gb300 import llama, synth
+from tests.helpers import TOL_LINEAR, TOL_LOGP, assert_abs, assert_rel, dev_i32, max_abs_err
+from tests.test_gpu_llama import SMALL, chain_spread, make_model, oracle_cfg
+
+pytestmark = pytest.mark.gpu
+
+# A drawn token's logit may sit below the oracle's maximum by the logit error of the bf16
+# chain: one-ulp differences (2^-8 relative) in the final hidden state, summed over d
+# products with LM-head weights of std 0.02, give about 0.02 * 2^-8 * sqrt(d) < 1e-3 at
+# d = 4096; TOL_DRAW leaves a factor of 10.
+TOL_DRAW = 1e-2
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    Bld.build()
+    H.load()
+    H.device_error(clear=True)
+    yield
+    assert H.device_error(clear=True) == 0
+
+
+def gumbel_noise(seed, n_steps, S, V):
+    u = synth.uniform(seed, n_steps * S * V)
+    return (-np.log(-np.log(u))).astype(np.float32).reshape(n_steps, S, V)
+
+
+def run_generate(cfg, sep, prompt, n_steps, noise, with_score=True):
+    S = prompt.shape[0]
+    w = llama.to_device(llama.fuse_separate(sep), "cuda")
+    ws = torch.empty(H.generate_llama_workspace_size(cfg, S), dtype=torch.uint8, device="cuda")
+    out = {"tokens": torch.full((S, n_steps), -1, dtype=torch.int32, device="cuda")}
+    for k in ("logp_actor", "logp_ref", "values"):
+        out[k] = torch.full((S, n_steps), float("nan"), device="cuda")
+    out["score"] = torch.full((S,), float("nan"), device="cuda") if with_score else None
+    g = None if noise is None else torch.from_numpy(noise).cuda()
+    H.hydra_generate_llama(cfg, w, dev_i32(prompt), n_steps, g, ws, out)
+    torch.cuda.synchronize()
+    assert H.device_error(clear=True) == 0
+    return {k: (None if v is None else v.cpu().numpy()) for k, v in out.items()}
+
+
+def check_generation(cfg, got, w64, prompt, noise, derive_tol=False):
+    P0 = cfg["prompt_len"]
+    S, n = got["tokens"].shape
+    V = cfg["vocab"]
+    for s in range(S):
+        tok = got["tokens"][s].astype(np.int64)
+        assert np.all((tok >= 0) & (tok < V))
+        seq = np.concatenate([prompt[s], tok])
+        ref = O.llama_score(w64, seq, P0, oracle_cfg(cfg), beta=cfg["beta"], gamma=cfg["gamma"],
+                            lam=cfg["lam"])
+        tol_lp, tol_lin = TOL_LOGP, TOL_LINEAR
+        if derive_tol:
+            alt = chain_spread(w64, seq, P0, cfg, n)
+            tol_lp = max(TOL_LOGP, 3 * max(max_abs_err(alt["logp_actor"], ref["logp_actor"]),
+                                           max_abs_err(alt["logp_ref"], ref["logp_ref"])))
+            tol_lin = max(TOL_LINEAR, 3 * max(max_abs_err(alt["values"], ref["values"]),
+                                              abs(alt["score"] - ref["score"])))
+        assert_abs(got["logp_actor"][s], ref["logp_actor"], tol_lp, f"logp_actor seq {s}")
+        assert_abs(got["logp_ref"][s], ref["logp_ref"], tol_lp, f"logp_ref seq {s}")
+        assert_rel(got["values"][s], ref["values"], tol_lin, f"values seq {s}")
+        if got["score"] is not None:
+            assert_rel(got["score"][s:s + 1], [ref["score"]], tol_lin, f"score seq {s}")
+        # every token is a valid draw from the oracle's logits at its step
+        z = ref["h_on"][P0 - 1:P0 - 1 + n] @ w64["lm_head"].T
+        key = z + (0.0 if noise is None else noise[:, s, :].astype(np.float64))
+        gap = key.max(axis=1) - key[np.arange(n), tok]
+        assert np.all(gap <= TOL_DRAW), f"seq {s}: drawn tokens {np.nonzero(gap > TOL_DRAW)[0]}"
+
+
+@pytest.mark.parametrize("sampled", [False, True])
+def test_generate_small(sampled):
+    cfg = dict(SMALL)
+    sep, w64 = make_model(cfg, 71)
+    S, n = 3, 12
+    prompt = synth.randint(711, (S, cfg["prompt_len"]), 0, cfg["vocab"])
+    noise = gumbel_noise(712, n, S, cfg["vocab"]) if sampled else None
+    got = run_generate(cfg, sep, prompt, n, noise)
+    check_generation(cfg, got, w64, prompt, noise)
+
+
+def test_generate_fills_the_cache():
+    """n_steps = response_len: the last draw attends over every cached position, and the
+    score pass writes the last one."""
+    cfg = dict(SMALL, prompt_len=5, response_len=20)
+    sep, w64 = make_model(cfg, 72)
+    prompt = synth.randint(721, (2, 5), 0, cfg["vocab"])
+    noise = gumbel_noise(722, 20, 2, cfg["vocab"])
+    got = run_generate(cfg, sep, prompt, 20, noise)
+    check_generation(cfg, got, w64, prompt, noise)
+
+
+def test_generate_eight_sequences_one_prompt_token():
+    """The largest batch (8 sequences: 16 GEMV rows) and a one-token prompt."""
+    cfg = dict(SMALL, prompt_len=1, response_len=6)
+    sep, w64 = make_model(cfg, 73)
+    prompt = synth.randint(731, (8, 1), 0, cfg["vocab"])
+    noise = gumbel_noise(732, 6, 8, cfg["vocab"])
+    got = run_generate(cfg, sep, prompt, 6, noise, with_score=False)
+    check_generation(cfg, got, w64, prompt, noise)
+
+
+def test_generate_lora_off_streams_agree_bitwise():
+    cfg = dict(SMALL)
+    sep, _ = make_model(cfg, 74, zero_B=True)
+    prompt = synth.randint(741, (2, cfg["prompt_len"]), 0, cfg["vocab"])
+    got = run_generate(cfg, sep, prompt, 8, gumbel_noise(742, 8, 2, cfg["vocab"]))
+    assert np.array_equal(got["logp_actor"], got["logp_ref"])
+
+
+def test_generate_matches_gpu_scoring_pass():
+    """The decode path (GEMV, cache) and the scoring pass (tcgen05 GEMM, full attention) on
+    the same finished sequence agree within the scoring tolerances."""
+    cfg = dict(SMALL)
+    sep, _ = make_model(cfg, 75)
+    S, n = 2, cfg["response_len"]
+    prompt = synth.randint(751, (S, cfg["prompt_len"]), 0, cfg["vocab"])
+    got = run_generate(cfg, sep, prompt, n, gumbel_noise(752, n, S, cfg["vocab"]))
+    ids = np.concatenate([prompt, got["tokens"]], axis=1).astype(np.int32)
+    w = llama.to_device(llama.fuse_separate(sep), "cuda")
+    ws = torch.empty(H.score_llama_workspace_size(cfg, S), dtype=torch.uint8, device="cuda")
+    out = llama.alloc_outputs(S, n, "cuda")
+    H.hydra_score_llama(cfg, w, dev_i32(ids), None, ws, out)
+    torch.cuda.synchronize()
+    sc = {k: v.cpu().numpy() for k, v in out.items()}
+    assert_abs(got["logp_actor"], sc["logp_actor"], TOL_LOGP, "logp_actor")
+    assert_abs(got["logp_ref"], sc["logp_ref"], TOL_LOGP, "logp_ref")
+    assert_rel(got["values"], sc["values"], TOL_LINEAR, "values")
+    assert_rel(got["score"], sc["score"], TOL_LINEAR, "score")
+
+
+def test_generate_full_width_one_layer():
+    """Llama-7B widths (d 4096, 32 heads, FFN 11008, vocab 32000, LoRA r 16), one decoder
+    layer, 2 sequences of 24 prompt tokens, 6 draws; tolerances derived from the chain."""
+    cfg = dict(llama.LLAMA7B, n_layers=1, prompt_len=24, response_len=6)
+    sep, w64 = make_model(cfg, 76)
+    prompt = synth.randint(761, (2, 24), 0, cfg["vocab"])
+    noise = gumbel_noise(762, 6, 2, cfg["vocab"])
+    got = run_generate(cfg, sep, prompt, 6, noise)
+    check_generation(cfg, got, w64, prompt, noise, derive_tol=True)
+
+
+def test_generate_argument_errors():
+    cfg = dict(SMALL)
+    sep, _ = make_model(cfg, 77)
+    w = llama.to_device(llama.fuse_separate(sep), "cuda")
+    ws = torch.empty(H.generate_llama_workspace_size(cfg, 2), dtype=torch.uint8, device="cuda")
+    prompt = dev_i32(synth.randint(771, (2, cfg["prompt_len"]), 0, cfg["vocab"]))
+    out = {"tokens": torch.zeros((2, 4), dtype=torch.int32, device="cuda"), "score": None}
+    for k in ("logp_actor", "logp_ref", "values"):
+        out[k] = torch.zeros((2, 4), device="cuda")
+    with pytest.raises(H.HydraError):  # more steps than the cache holds
+        H.hydra_generate_llama(cfg, w, prompt, cfg["response_len"] + 1, None, ws, out)
+    with pytest.raises(H.HydraError):  # workspace for fewer sequences
+        H.hydra_generate_llama(cfg, w, dev_i32(np.zeros((3, cfg["prompt_len"]), np.int32)), 4,
+                               None, ws, out)
+    assert H.generate_llama_workspace_size(cfg, 9) == 0
