@@ -455,6 +455,153 @@ class HydraPPOScoringLlama7B(HydraScoringLlama7B):
         return time.perf_counter() - t0
 
 
+class HydraGenerateLlama7B(HydraScoringLlama7B):
+    """KV-cached generation (Algorithms 1 and 2: the actor generates each sequence for T
+    steps, J-Hydra keeps the values) on the same random-init Llama-7B: 4 sequences of 256
+    prompt tokens, 64 draws each from the actor's softmax (Gumbel-max, noise drawn on the
+    device), the LoRA-off stream decoded beside the actor (reference log-probs of every
+    draw), values and the final reward score. One step = one hydra_generate_llama call:
+    prefill of both streams plus 64 decode steps of 8 rows (2 streams x 4 sequences)."""
+
+    name = "hydra_generate_llama7b"
+    seed = 6
+    default_steps, default_warmup = 5, 3
+    profiled = False
+    event_names = ("gen",)
+    metric = ("generated tokens/s (actor draws with logp_actor, logp_ref, values; both streams "
+              "decoded) on 1 GB300; decode step vs HBM roofline")
+    n_steps = 64
+
+    def __init__(self, device, seed=6, reference=False):
+        super().__init__(device, seed=seed, reference=reference)
+        import torch
+        c = self.cfg
+        S, V = self.S, c["vocab"]
+        self.prompt = self.ids[:, :self.P0].contiguous()
+        g = torch.Generator(device=device)
+        g.manual_seed(seed * 1000 + 7)
+        u = torch.rand(self.n_steps, S, V, device=device, generator=g).clamp_(1e-12, 1.0 - 1e-7)
+        self.gumbel = -torch.log(-torch.log(u))
+        del u
+        if not reference:
+            self.ws = torch.empty(self.H.generate_llama_workspace_size(c, S), dtype=torch.uint8,
+                                  device=device)
+            self.gen_out = {"tokens": torch.empty(S, self.n_steps, dtype=torch.int32, device=device),
+                            "score": torch.empty(S, device=device)}
+            for k in ("logp_actor", "logp_ref", "values"):
+                self.gen_out[k] = torch.empty(S, self.n_steps, device=device)
+        self.units = S * self.n_steps
+        d, F, r, nl, H = c["d_model"], c["ffn"], c["lora_rank"], c["n_layers"], c["n_heads"]
+        R = 2 * S
+        # algorithmic bytes of one decode step: every weight once (bf16), the LoRA factors, the
+        # cached keys and values up to the mean position, the new keys and values, the logits
+        w_layer = (3 * d * d + d * d + 2 * F * d + d * F + 2 * d) * 2
+        lora_layer = (2 * r * d + 3 * d * 2 * r + 2 * r * d + 2 * F * 2 * r + r * F + d * r) * 2
+        mean_pos = self.P0 + self.n_steps / 2
+        kv_layer = R * mean_pos * 2 * d * 2 + R * 2 * d * 2
+        self.step_bytes = nl * (w_layer + lora_layer + kv_layer) + V * d * 2 + R * V * 4 * 2
+        per_layer = 14
+        decode = 1 + per_layer * nl + 1 + 3
+        prefill = 2 + 11 * nl + 1 + 3
+        self.launches_per_step = prefill + (self.n_steps - 1) * decode + (1 + per_layer * nl + 2)
+
+    def _call(self, n_steps, out=None):
+        o = out or self.gen_out
+        if n_steps != self.n_steps:
+            o = {k: (v[:, :n_steps].contiguous() if v.dim() == 2 else v) for k, v in o.items()}
+        self.H.hydra_generate_llama(self.cfg, self.weights, self.prompt, n_steps, self.gumbel[:n_steps],
+                                    self.ws, o)
+
+    def step(self, ev=None):
+        if ev is not None:
+            ev["gen"][0].record()
+        self._call(self.n_steps)
+        if ev is not None:
+            ev["gen"][1].record()
+
+    def e2e_setup(self):
+        import torch
+        self.prompt_host = self.prompt.cpu().pin_memory()
+        self.gumbel_host = self.gumbel.cpu().pin_memory()
+        self.out_host = {k: torch.empty(v.shape, dtype=v.dtype, pin_memory=True)
+                         for k, v in self.gen_out.items()}
+        self.h2d = self.prompt_host.numel() * 4 + self.gumbel_host.numel() * 4
+        self.d2h = sum(v.numel() * 4 for v in self.out_host.values())
+
+    def e2e_step(self):
+        self.prompt.copy_(self.prompt_host, non_blocking=True)
+        self.gumbel.copy_(self.gumbel_host, non_blocking=True)
+        self._call(self.n_steps)
+        for k, v in self.gen_out.items():
+            self.out_host[k].copy_(v, non_blocking=True)
+
+    def _decode_step_ms(self, reps=3):
+        """Decode step time from two call lengths: (T(n) - T(1)) / (n - 1), CUDA events."""
+        import torch
+
+        def timed(n):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            for _ in range(reps):
+                self._call(n)
+            e1.record()
+            torch.cuda.synchronize()
+            return e0.elapsed_time(e1) / reps
+        t1 = timed(1)
+        tn = timed(self.n_steps)
+        return (tn - t1) / (self.n_steps - 1), t1
+
+    def kernels(self, peaks, ms):
+        step_ms, t1 = self._decode_step_ms()
+        self._step_ms = step_ms
+        return {"generate_call": {"ms": ms["gen"]},
+                "prefill_plus_first_draw": {"ms": t1},
+                "decode_step": {"ms": step_ms, "GB/s": self.step_bytes / step_ms / 1e6,
+                                "bytes": self.step_bytes}}
+
+    def roofline(self, peaks, ms):
+        step_ms = getattr(self, "_step_ms", None)
+        if step_ms is None:
+            step_ms, _ = self._decode_step_ms()
+        achieved = self.step_bytes / step_ms / 1e6
+        peak = peaks["hbm_gbs"]
+        return {"kernel": "decode step (dual-output GEMV for every projection and the LM head, "
+                          "decode attention over the cache, elementwise): 8 rows",
+                "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": achieved / peak, "traffic": None,
+                "peak_kind": f"HBM copy, {peaks['source']}",
+                "per_step_bytes": self.step_bytes, "per_step_ms": step_ms}
+
+    def config(self):
+        return {"workload": "hydra_generate_llama7b: random-init Llama-7B (32 layers, d 4096, 32 heads, "
+                            "SwiGLU 11008, vocab 32000, bf16), LoRA r=16 s=2 on q/v/gate/up/down; 4 "
+                            f"sequences x 256 prompt tokens, {self.n_steps} Gumbel-max draws each; LoRA-off stream "
+                            "decoded beside the actor; values and final score",
+                "batch": self.S, "prompt_len": self.P0, "draws": self.n_steps,
+                "generated_tokens_per_step": self.units,
+                "l2": "inputs larger than L2 (13.5 GB of weights read per decode step)"}
+
+    def oracle_time(self, smp, n_layers):
+        import oracle as O
+        t0 = time.perf_counter()
+        O.llama_generate(smp["w"], smp["ids"][:smp["prompt"]], 2, smp["cfg"], n_layers=n_layers)
+        return time.perf_counter() - t0
+
+    def oracle_throughput(self, steps=1):
+        """(tokens/s, description): 2 draws after a 32-token prompt, per-draw time t(0 layers)
+        + 32 (t(1) - t(0)), the oracle recomputing the whole prefix at each draw."""
+        smp = self.oracle_sample(1)
+        t_head = self.oracle_time(smp, 0)
+        t1 = [self.oracle_time(smp, 1) for _ in range(steps)]
+        n = self.cfg["n_layers"]
+        t_gen = [t_head + n * max(t - t_head, 0.0) for t in t1]
+        desc = (f"one sequence, {smp['prompt']} prompt tokens, 2 draws (plus the score pass) at full "
+                f"width through the fp64 oracle, which recomputes the prefix at every draw: embed + "
+                f"heads {t_head:.2f} s, one decoder layer {statistics.mean(t1) - t_head:.2f} s, time "
+                f"extrapolated to {n} layers")
+        return 2 * len(t_gen) / sum(t_gen), desc
+
+
 class KernelSweep:
     """Per-kernel measurements of the rows the full pass does not exercise at their own
     shapes (one JSON line; value = the sweep's mean fraction of roofline):
@@ -612,6 +759,7 @@ class KernelSweep:
 
 WORKLOADS = {LmHeadScoring.name: LmHeadScoring, HydraScoringLlama7B.name: HydraScoringLlama7B,
              HydraPPOScoringLlama7B.name: HydraPPOScoringLlama7B,
+             HydraGenerateLlama7B.name: HydraGenerateLlama7B,
              KernelSweep.name: KernelSweep}
 DEFAULT_WORKLOAD = HydraScoringLlama7B.name
 
@@ -678,6 +826,8 @@ def time_oracle(wl, target_s=12.0):
 
 
 def run_reference(args, wl_cls):
+    if getattr(args, "gen_steps", None) and hasattr(wl_cls, "n_steps"):
+        wl_cls.n_steps = args.gen_steps
     rank, world, local = dist_env()
     if rank != 0:
         return 0
@@ -689,8 +839,8 @@ def run_reference(args, wl_cls):
     if hasattr(wl_cls, "oracle_throughput"):
         wl = wl_cls(dev, reference=True)
         value, desc = wl.oracle_throughput(steps=args.steps)
-        t_step = wl.L / value
-        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        t_step = wl.units / value
+        line = {"metric": getattr(wl, "metric", METRIC), "value": value, "unit": UNIT, "n_gpus": args.gpus,
                 "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_step * 1e3,
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
                 "data": "synthetic", "impl": "reference", "config": wl.config(),
@@ -745,6 +895,8 @@ def run_sweep(args):
 
 def run_ours(args, wl_cls):
     import torch
+    if getattr(args, "gen_steps", None) and hasattr(wl_cls, "n_steps"):
+        wl_cls.n_steps = args.gen_steps
     rank, world, local = dist_env()
     if world > 1:
         import torch.distributed as dist
@@ -768,7 +920,7 @@ def run_ours(args, wl_cls):
     if H.device_error(clear=True) != 0:
         raise RuntimeError("device error during warm-up")
 
-    driver = isinstance(wl, HydraScoringLlama7B)
+    driver = isinstance(wl, HydraScoringLlama7B) and getattr(wl, "profiled", True)
     names = getattr(wl, "event_names", ())
     evs = [None] * steps
     if driver:
@@ -823,8 +975,9 @@ def run_ours(args, wl_cls):
 
     value = aggregate(wl.units, steps, world, ms_total_max)
     e2e_value = aggregate(wl.units, e2e_steps, world, e2e_ms)
+    metric = getattr(wl, "metric", METRIC)
     line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": steps,
+        "metric": metric, "value": value, "unit": UNIT, "n_gpus": world, "steps": steps,
         "warmup": warmup, "ms_per_step": ms_total_max / steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": dict(wl.config(), parallelism=f"replicas{world}" if world > 1 else "single"),
@@ -853,6 +1006,8 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default=DEFAULT_WORKLOAD)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--gen-steps", type=int, default=None,
+                    help="hydra_generate_llama7b only: draws per call (default 64)")
     ap.add_argument("--parts", default=None,
                     help="kernel_sweep only: comma-separated subset of " + ",".join(KernelSweep.PARTS))
     args = ap.parse_args(argv)

@@ -11,6 +11,8 @@
 // The step counter lives in device memory, so one captured step replays for every position.
 // Cache layout per layer: K [R][H][Pmax][Dh] then V [R][H][Pmax][Dh], bf16, row i = stream
 // * S + sequence.
+#include <utility>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -36,45 +38,41 @@ __global__ void kv_store_prefill_kernel(const __nv_bfloat16* __restrict__ qkv, i
   }
 }
 
-// One block per stacked row: q rotated in place, k rotated into the cache, v copied. The same
-// explicit roundings as the prefill's rotary (no contraction), from the same table.
+// One block per (head, row): q rotated in place, k rotated into the cache, v copied. The
+// same explicit roundings as the prefill's rotary (no contraction), from the same table.
 __global__ void decode_rope_append_kernel(__nv_bfloat16* __restrict__ qkv, int ld, int d, int H,
                                           const float2* __restrict__ table, int P0,
                                           const int* __restrict__ step, int Pmax,
                                           __nv_bfloat16* __restrict__ ck,
                                           __nv_bfloat16* __restrict__ cv) {
-  const int i = blockIdx.x;
+  pdl_wait();
+  pdl_launch_dependents();
+  const int h = blockIdx.x, i = blockIdx.y;
   const int pos = P0 + *step - 1;
   if (pos < 0 || pos >= Pmax) return;  // the host keeps every step inside the cache
-  __nv_bfloat16* row = qkv + static_cast<size_t>(i) * ld;
-  const float2* tb = table + static_cast<size_t>(pos) * (kDh / 2);
   constexpr int half = kDh / 2;
-  for (int e = threadIdx.x; e < 2 * H * half; e += blockDim.x) {
-    const int blk = e / (H * half);  // 0: q, 1: k
-    const int r = e - blk * H * half;
-    const int h = r / half, j = r % half;
-    __nv_bfloat16* x = row + blk * d + h * kDh;
-    const float x1 = __bfloat162float(x[j]), x2 = __bfloat162float(x[j + half]);
-    const float c = tb[j].x, s = tb[j].y;
-    const __nv_bfloat16 o1 = __float2bfloat16_rn(__fsub_rn(__fmul_rn(x1, c), __fmul_rn(x2, s)));
-    const __nv_bfloat16 o2 = __float2bfloat16_rn(__fadd_rn(__fmul_rn(x1, s), __fmul_rn(x2, c)));
-    if (blk == 0) {
-      x[j] = o1;
-      x[j + half] = o2;
-    } else {
-      __nv_bfloat16* dst = ck + ((static_cast<size_t>(i) * H + h) * Pmax + pos) * kDh;
-      dst[j] = o1;
-      dst[j + half] = o2;
-    }
+  __nv_bfloat16* row = qkv + static_cast<size_t>(i) * ld;
+  const size_t slot = ((static_cast<size_t>(i) * H + h) * Pmax + pos) * kDh;
+  const int j = threadIdx.x & (half - 1);
+  const int blk = threadIdx.x / half;  // 0: q, 1: k (128 threads)
+  const float2 cs = table[static_cast<size_t>(pos) * half + j];
+  __nv_bfloat16* x = row + blk * d + h * kDh;
+  const float x1 = __bfloat162float(x[j]), x2 = __bfloat162float(x[j + half]);
+  const __nv_bfloat16 o1 = __float2bfloat16_rn(__fsub_rn(__fmul_rn(x1, cs.x), __fmul_rn(x2, cs.y)));
+  const __nv_bfloat16 o2 = __float2bfloat16_rn(__fadd_rn(__fmul_rn(x1, cs.y), __fmul_rn(x2, cs.x)));
+  if (blk == 0) {
+    x[j] = o1;
+    x[j + half] = o2;
+  } else {
+    ck[slot + j] = o1;
+    ck[slot + j + half] = o2;
   }
-  for (int e = threadIdx.x * 8; e < d; e += blockDim.x * 8) {
-    const int h = e / kDh, j = e % kDh;
-    *reinterpret_cast<uint4*>(cv + ((static_cast<size_t>(i) * H + h) * Pmax + pos) * kDh + j) =
-        *reinterpret_cast<const uint4*>(row + 2 * d + e);
-  }
+  if (threadIdx.x < kDh / 8)
+    *reinterpret_cast<uint4*>(cv + slot + 8 * threadIdx.x) =
+        *reinterpret_cast<const uint4*>(row + 2 * d + h * kDh + 8 * threadIdx.x);
 }
 
-constexpr int kAttnThreads = 128;
+constexpr int kAttnThreads = 256;
 constexpr int kAttnWarps = kAttnThreads / 32;
 
 __device__ __forceinline__ float block_max(float v, float* red) {
@@ -112,6 +110,8 @@ __global__ void __launch_bounds__(kAttnThreads)
                             __nv_bfloat16* __restrict__ out, int ld_out) {
   extern __shared__ float sc[];  // [Pmax] scores, then [kAttnWarps][kDh] partial outputs
   __shared__ float red[kAttnWarps];
+  pdl_wait();
+  pdl_launch_dependents();
   const int h = blockIdx.x, i = blockIdx.y;
   const int npos = min(P0 + *step, Pmax);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -131,27 +131,40 @@ __global__ void __launch_bounds__(kAttnThreads)
       qf[2 * k + 1] = f.y * scale;
     }
   }
-  // warp-uniform trip count: all 32 lanes reach the shuffles
-  for (int base = warp * 4; base < npos; base += 4 * kAttnWarps) {
-    const int p = base + g;
-    uint4 a = make_uint4(0u, 0u, 0u, 0u), b = a;
-    if (p < npos) {
-      const __nv_bfloat16* kr = K + static_cast<size_t>(p) * kDh + 16 * sub;
-      a = __ldcs(reinterpret_cast<const uint4*>(kr));
-      b = __ldcs(reinterpret_cast<const uint4*>(kr + 8));
+  // warp-uniform trip count: all 32 lanes reach the shuffles. Each 8-lane group takes two
+  // keys per iteration, both loaded before either is reduced.
+  constexpr int kKeysPerIter = 2 * 4 * kAttnWarps;
+  for (int base = warp * 4; base < npos; base += kKeysPerIter) {
+    const int p0 = base + g, p1 = base + 4 * kAttnWarps + g;
+    uint4 a0 = make_uint4(0u, 0u, 0u, 0u), b0 = a0, a1 = a0, b1 = a0;
+    if (p0 < npos) {
+      const __nv_bfloat16* kr = K + static_cast<size_t>(p0) * kDh + 16 * sub;
+      a0 = __ldcs(reinterpret_cast<const uint4*>(kr));
+      b0 = __ldcs(reinterpret_cast<const uint4*>(kr + 8));
     }
-    const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
-    float acc = 0.f;
+    if (p1 < npos) {
+      const __nv_bfloat16* kr = K + static_cast<size_t>(p1) * kDh + 16 * sub;
+      a1 = __ldcs(reinterpret_cast<const uint4*>(kr));
+      b1 = __ldcs(reinterpret_cast<const uint4*>(kr + 8));
+    }
+    const uint32_t w0[8] = {a0.x, a0.y, a0.z, a0.w, b0.x, b0.y, b0.z, b0.w};
+    const uint32_t w1[8] = {a1.x, a1.y, a1.z, a1.w, b1.x, b1.y, b1.z, b1.w};
+    float acc0 = 0.f, acc1 = 0.f;
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
-      const float2 f = unpack_bf16x2(w[k]);
-      acc = fmaf(qf[2 * k], f.x, acc);
-      acc = fmaf(qf[2 * k + 1], f.y, acc);
+      const float2 f0 = unpack_bf16x2(w0[k]), f1 = unpack_bf16x2(w1[k]);
+      acc0 = fmaf(qf[2 * k], f0.x, acc0);
+      acc0 = fmaf(qf[2 * k + 1], f0.y, acc0);
+      acc1 = fmaf(qf[2 * k], f1.x, acc1);
+      acc1 = fmaf(qf[2 * k + 1], f1.y, acc1);
     }
-    acc += __shfl_xor_sync(0xffffffffu, acc, 1);
-    acc += __shfl_xor_sync(0xffffffffu, acc, 2);
-    acc += __shfl_xor_sync(0xffffffffu, acc, 4);
-    if (sub == 0 && p < npos) sc[p] = acc;
+#pragma unroll
+    for (int o = 1; o < 8; o <<= 1) {
+      acc0 += __shfl_xor_sync(0xffffffffu, acc0, o);
+      acc1 += __shfl_xor_sync(0xffffffffu, acc1, o);
+    }
+    if (sub == 0 && p0 < npos) sc[p0] = acc0;
+    if (sub == 0 && p1 < npos) sc[p1] = acc1;
   }
   __syncthreads();
   float m = -INFINITY;
@@ -165,7 +178,7 @@ __global__ void __launch_bounds__(kAttnThreads)
   }
   l = block_sum(l, red);  // ends with a barrier: every weight is in shared memory
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll 4
+#pragma unroll 8
   for (int p = warp; p < npos; p += kAttnWarps) {
     const float wgt = sc[p];
     const uint2 v = __ldcs(reinterpret_cast<const uint2*>(Vc + static_cast<size_t>(p) * kDh + 4 * lane));
@@ -213,6 +226,186 @@ __global__ void swiglu_blocked_kernel(const __nv_bfloat16* __restrict__ gu, long
     }
     *reinterpret_cast<uint4*>(m + static_cast<size_t>(row) * F + c) = o;
   }
+}
+
+// ---------------------------------------------------------------- fused row kernels
+// Thread-block clusters of kCl CTAs share one row: each CTA owns a 1/kCl slice of the columns,
+// partial sums meet through distributed shared memory (mapa + ld.shared::cluster) and are
+// added in CTA-rank order, so the result does not depend on timing.
+constexpr int kCl = 8;
+constexpr int kRowThreads = 256;
+constexpr int kRowWarps = kRowThreads / 32;
+constexpr int kMaxR2 = 256;  // LoRA ranks of one fused down-projection (2 r for q/v, gate/up)
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
+                   : "memory");
+}
+
+// a float in CTA `rank`'s shared memory at the address of `local` in this CTA
+__device__ __forceinline__ float ld_cluster_f32(const float* local, uint32_t rank) {
+  uint32_t raddr;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(raddr) : "r"(smem_u32(local)), "r"(rank));
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(raddr) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ float row_block_sum(float v, float* red) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+  __syncthreads();
+  float t = 0.f;
+#pragma unroll
+  for (int w = 0; w < kRowWarps; ++w) t += red[w];
+  return t;
+}
+
+// Partial LoRA down-projection of this CTA's slice: up[j] = sum_e xs[e] A[j][c0 + e] for
+// j < r2 (warps take j in turn, lanes 4 columns at a time); then rank 0 adds the kCl
+// partials in rank order and writes u = bf16(s * sum). xs holds the slice's bf16 values.
+__device__ __forceinline__ void lora_slice(const float* xs, int n, int c0, int K,
+                                           const __nv_bfloat16* __restrict__ A, int r2, float s,
+                                           float* up, __nv_bfloat16* __restrict__ u_row,
+                                           uint32_t rank) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int j = warp; j < r2; j += kRowWarps) {
+    const __nv_bfloat16* aj = A + static_cast<size_t>(j) * K + c0;
+    float acc = 0.f;
+    for (int e = 4 * lane; e < n; e += 128) {
+      const uint2 q = *reinterpret_cast<const uint2*>(aj + e);
+      const float2 a01 = unpack_bf16x2(q.x), a23 = unpack_bf16x2(q.y);
+      acc = fmaf(xs[e], a01.x, acc);
+      acc = fmaf(xs[e + 1], a01.y, acc);
+      acc = fmaf(xs[e + 2], a23.x, acc);
+      acc = fmaf(xs[e + 3], a23.y, acc);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (lane == 0) up[j] = acc;
+  }
+  cluster_sync_all();
+  if (rank == 0) {
+    for (int j = threadIdx.x; j < r2; j += kRowThreads) {
+      float t = 0.f;
+      for (uint32_t q = 0; q < kCl; ++q) t += ld_cluster_f32(up + j, q);
+      u_row[j] = __float2bfloat16_rn(s * t);
+    }
+  }
+}
+
+// Cluster (kCl, 1, 1) per row of h [R, d]: h += y (RESID), a = bf16(rmsnorm(h) w) and, for the
+// LoRA-on rows i >= S, u[i - S] = bf16(s a A^T) (A [r2, d]; none if A is NULL). The residual
+// add, the norm and the LoRA down-projection of the next projection in one launch.
+template <bool RESID>
+__global__ void __launch_bounds__(kRowThreads)
+    row_norm_lora_kernel(float* __restrict__ h, const __nv_bfloat16* __restrict__ y,
+                         const __nv_bfloat16* __restrict__ w, int d, float eps,
+                         __nv_bfloat16* __restrict__ a, int S, const __nv_bfloat16* __restrict__ A,
+                         int r2, float s, __nv_bfloat16* __restrict__ u) {
+  extern __shared__ float xs[];  // this CTA's slice of the row
+  __shared__ float red[kRowWarps];
+  __shared__ float part;
+  __shared__ float up[kMaxR2];
+  pdl_wait();
+  pdl_launch_dependents();
+  const uint32_t rank = cluster_rank();
+  const int row = blockIdx.y;
+  const int n = d / kCl, c0 = static_cast<int>(rank) * n;
+  float* hr = h + static_cast<size_t>(row) * d + c0;
+  float ss = 0.f;
+  for (int e = 4 * threadIdx.x; e < n; e += 4 * kRowThreads) {
+    float4 v = *reinterpret_cast<const float4*>(hr + e);
+    if (RESID) {
+      const uint2 q = *reinterpret_cast<const uint2*>(y + static_cast<size_t>(row) * d + c0 + e);
+      const float2 y01 = unpack_bf16x2(q.x), y23 = unpack_bf16x2(q.y);
+      v.x += y01.x;
+      v.y += y01.y;
+      v.z += y23.x;
+      v.w += y23.y;
+      *reinterpret_cast<float4*>(hr + e) = v;
+    }
+    xs[e] = v.x;
+    xs[e + 1] = v.y;
+    xs[e + 2] = v.z;
+    xs[e + 3] = v.w;
+    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+  }
+  ss = row_block_sum(ss, red);
+  if (threadIdx.x == 0) part = ss;
+  cluster_sync_all();
+  float tot = 0.f;
+  for (uint32_t q = 0; q < kCl; ++q) tot += ld_cluster_f32(&part, q);
+  const float inv = rsqrtf(tot / static_cast<float>(d) + eps);
+  __nv_bfloat16* ar = a + static_cast<size_t>(row) * d + c0;
+  for (int e = 4 * threadIdx.x; e < n; e += 4 * kRowThreads) {
+    const uint2 wq = __ldg(reinterpret_cast<const uint2*>(w + c0 + e));
+    const float2 w01 = unpack_bf16x2(wq.x), w23 = unpack_bf16x2(wq.y);
+    const uint32_t o0 = pack_bf16x2(xs[e] * inv * w01.x, xs[e + 1] * inv * w01.y);
+    const uint32_t o1 = pack_bf16x2(xs[e + 2] * inv * w23.x, xs[e + 3] * inv * w23.y);
+    *reinterpret_cast<uint2*>(ar + e) = make_uint2(o0, o1);
+    const float2 b01 = unpack_bf16x2(o0), b23 = unpack_bf16x2(o1);
+    xs[e] = b01.x;
+    xs[e + 1] = b01.y;
+    xs[e + 2] = b23.x;
+    xs[e + 3] = b23.y;
+  }
+  __syncthreads();
+  if (A != nullptr && row >= S)
+    lora_slice(xs, n, c0, d, A, r2, s, up, u + static_cast<size_t>(row - S) * r2, rank);
+  else
+    cluster_sync_all();  // the same cluster barriers on every path
+  cluster_sync_all();    // rank 0's remote reads finish before any CTA leaves
+}
+
+// Cluster (kCl, 1, 1) per row of gu [R, 2F] (gate/up interleaved in blocks of 128):
+// m = bf16(silu(gate) up) [R, F] and, for the LoRA-on rows, u[i - S] = bf16(s m A^T)
+// (A [r, F]): SwiGLU and the down projection's LoRA down-projection in one launch.
+__global__ void __launch_bounds__(kRowThreads)
+    swiglu_lora_kernel(const __nv_bfloat16* __restrict__ gu, int F, __nv_bfloat16* __restrict__ m,
+                       int S, const __nv_bfloat16* __restrict__ A, int r, float s,
+                       __nv_bfloat16* __restrict__ u) {
+  extern __shared__ float xs[];
+  __shared__ float up[kMaxR2];
+  pdl_wait();
+  pdl_launch_dependents();
+  const uint32_t rank = cluster_rank();
+  const int row = blockIdx.y;
+  const int n = F / kCl, c0 = static_cast<int>(rank) * n;
+  const __nv_bfloat16* g = gu + static_cast<size_t>(row) * 2 * F;
+  __nv_bfloat16* mr = m + static_cast<size_t>(row) * F + c0;
+  for (int e = 4 * threadIdx.x; e < n; e += 4 * kRowThreads) {
+    const int f = c0 + e;  // 4 features inside one block of 128
+    const int b = f / 128, j = f % 128;
+    const uint2 gq = *reinterpret_cast<const uint2*>(g + 256 * b + j);
+    const uint2 uq = *reinterpret_cast<const uint2*>(g + 256 * b + 128 + j);
+    const float2 g01 = unpack_bf16x2(gq.x), g23 = unpack_bf16x2(gq.y);
+    const float2 u01 = unpack_bf16x2(uq.x), u23 = unpack_bf16x2(uq.y);
+    const uint32_t o0 = pack_bf16x2(g01.x / (1.0f + expf(-g01.x)) * u01.x,
+                                    g01.y / (1.0f + expf(-g01.y)) * u01.y);
+    const uint32_t o1 = pack_bf16x2(g23.x / (1.0f + expf(-g23.x)) * u23.x,
+                                    g23.y / (1.0f + expf(-g23.y)) * u23.y);
+    *reinterpret_cast<uint2*>(mr + e) = make_uint2(o0, o1);
+    const float2 b01 = unpack_bf16x2(o0), b23 = unpack_bf16x2(o1);
+    xs[e] = b01.x;
+    xs[e + 1] = b01.y;
+    xs[e + 2] = b23.x;
+    xs[e + 3] = b23.y;
+  }
+  __syncthreads();
+  if (A != nullptr && row >= S)
+    lora_slice(xs, n, c0, F, A, r, s, up, u + static_cast<size_t>(row - S) * r, rank);
+  else
+    cluster_sync_all();
+  cluster_sync_all();
 }
 
 constexpr int kSampleThreads = 512;
@@ -319,11 +512,14 @@ int launch_decode_rope_append(void* qkv, int64_t R, int64_t ld, int64_t d, int64
                               const void* table, int64_t P0, const int* step, int64_t Pmax,
                               void* ck, void* cv, cudaStream_t st) {
   if (R == 0) return 0;
-  decode_rope_append_kernel<<<static_cast<unsigned>(R), 256, 0, st>>>(
-      static_cast<__nv_bfloat16*>(qkv), static_cast<int>(ld), static_cast<int>(d),
-      static_cast<int>(H), static_cast<const float2*>(table), static_cast<int>(P0), step,
-      static_cast<int>(Pmax), static_cast<__nv_bfloat16*>(ck), static_cast<__nv_bfloat16*>(cv));
-  return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
+  const cudaError_t e = launch_pdl(decode_rope_append_kernel,
+                                   dim3(static_cast<unsigned>(H), static_cast<unsigned>(R)),
+                                   dim3(kDh), 0, st, static_cast<__nv_bfloat16*>(qkv),
+                                   static_cast<int>(ld), static_cast<int>(d), static_cast<int>(H),
+                                   static_cast<const float2*>(table), static_cast<int>(P0), step,
+                                   static_cast<int>(Pmax), static_cast<__nv_bfloat16*>(ck),
+                                   static_cast<__nv_bfloat16*>(cv));
+  return e == cudaSuccess ? 0 : -3;
 }
 
 size_t decode_attention_smem(int64_t Pmax) {
@@ -342,13 +538,14 @@ int launch_decode_attention(const void* qkv, int64_t R, int64_t ld, int64_t H, c
       return -1;
     attr = smem;
   }
-  decode_attention_kernel<<<dim3(static_cast<unsigned>(H), static_cast<unsigned>(R)), kAttnThreads,
-                            smem, st>>>(
-      static_cast<const __nv_bfloat16*>(qkv), static_cast<int>(ld), static_cast<int>(H),
-      static_cast<const __nv_bfloat16*>(ck), static_cast<const __nv_bfloat16*>(cv),
-      static_cast<int>(P0), step, static_cast<int>(Pmax), 1.0f / sqrtf(static_cast<float>(kDh)),
-      static_cast<__nv_bfloat16*>(out), static_cast<int>(ld_out));
-  return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
+  const cudaError_t e = launch_pdl(
+      decode_attention_kernel, dim3(static_cast<unsigned>(H), static_cast<unsigned>(R)),
+      dim3(kAttnThreads), smem, st, static_cast<const __nv_bfloat16*>(qkv), static_cast<int>(ld),
+      static_cast<int>(H), static_cast<const __nv_bfloat16*>(ck),
+      static_cast<const __nv_bfloat16*>(cv), static_cast<int>(P0), step, static_cast<int>(Pmax),
+      1.0f / sqrtf(static_cast<float>(kDh)), static_cast<__nv_bfloat16*>(out),
+      static_cast<int>(ld_out));
+  return e == cudaSuccess ? 0 : -3;
 }
 
 int launch_swiglu_blocked(const void* gu, int64_t R, int64_t F, void* m, cudaStream_t st) {
@@ -369,6 +566,63 @@ int launch_sample_tokens(const float* logits, int64_t S, int64_t V, const float*
       static_cast<const __nv_bfloat16*>(w_rm), step, static_cast<int>(n_steps), tokens, logp_a,
       logp_r, values, cur_ids);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
+}
+
+// cudaLaunchKernelEx with a (kCl, 1, 1) cluster and programmatic dependent launch
+template <typename... KArgs, typename... Args>
+static cudaError_t launch_cluster(void (*kernel)(KArgs...), dim3 grid, size_t smem,
+                                  cudaStream_t st, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(kRowThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = kCl;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+int launch_row_norm_lora(float* h, const void* y, const void* w, int64_t R, int64_t d, float eps,
+                         void* a, int64_t S, const void* A, int64_t r2, float s, void* u,
+                         cudaStream_t st) {
+  if (R == 0) return 0;
+  if (d % (4 * kCl) != 0 || r2 > kMaxR2) return -1;
+  const size_t smem = static_cast<size_t>(d / kCl) * 4;
+  const dim3 grid(kCl, static_cast<unsigned>(R));
+  cudaError_t e;
+  if (y != nullptr)
+    e = launch_cluster(row_norm_lora_kernel<true>, grid, smem, st, h,
+                       static_cast<const __nv_bfloat16*>(y), static_cast<const __nv_bfloat16*>(w),
+                       static_cast<int>(d), eps, static_cast<__nv_bfloat16*>(a), static_cast<int>(S),
+                       static_cast<const __nv_bfloat16*>(A), static_cast<int>(r2), s,
+                       static_cast<__nv_bfloat16*>(u));
+  else
+    e = launch_cluster(row_norm_lora_kernel<false>, grid, smem, st, h,
+                       static_cast<const __nv_bfloat16*>(nullptr), static_cast<const __nv_bfloat16*>(w),
+                       static_cast<int>(d), eps, static_cast<__nv_bfloat16*>(a), static_cast<int>(S),
+                       static_cast<const __nv_bfloat16*>(A), static_cast<int>(r2), s,
+                       static_cast<__nv_bfloat16*>(u));
+  return e == cudaSuccess ? 0 : -3;
+}
+
+int launch_swiglu_lora(const void* gu, int64_t R, int64_t F, void* m, int64_t S, const void* A,
+                       int64_t r, float s, void* u, cudaStream_t st) {
+  if (R == 0) return 0;
+  if (F % (4 * kCl) != 0 || r > kMaxR2) return -1;
+  const size_t smem = static_cast<size_t>(F / kCl) * 4;
+  const cudaError_t e = launch_cluster(
+      swiglu_lora_kernel, dim3(kCl, static_cast<unsigned>(R)), smem, st,
+      static_cast<const __nv_bfloat16*>(gu), static_cast<int>(F), static_cast<__nv_bfloat16*>(m),
+      static_cast<int>(S), static_cast<const __nv_bfloat16*>(A), static_cast<int>(r), s,
+      static_cast<__nv_bfloat16*>(u));
+  return e == cudaSuccess ? 0 : -3;
 }
 
 int launch_step_advance(int* step, cudaStream_t st) {

@@ -7,10 +7,10 @@
 // Prefill: the prompt of both streams through the tcgen05 layer loop of the scoring pass
 // (rotary, SwiGLU and residual epilogues), with each layer's rotated keys and values copied
 // into the cache. Decode step (R = 2 S rows: off rows then on rows): embed the last drawn
-// token, per layer RMSNorm -> q/k/v GEMV (LoRA on q, v) -> rotary + cache append ->
-// attention over the cache -> o GEMV + residual -> RMSNorm -> gate/up GEMV (LoRA) ->
-// SwiGLU -> down GEMV (LoRA) + residual; then the final RMSNorm, the LM-head GEMV (fp32
-// logits) and the draw.
+// token, per layer [residual + RMSNorm + q/v LoRA down] -> q/k/v GEMV -> rotary + cache
+// append -> attention over the cache -> o GEMV -> [residual + RMSNorm + gate/up LoRA down]
+// -> gate/up GEMV -> [SwiGLU + down LoRA down] -> down GEMV; then [residual + final RMSNorm],
+// the LM-head GEMV (fp32 logits) and the draw. Brackets are thread-block-cluster kernels.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -77,16 +77,14 @@ bool gen_config_ok(const hydra_llama_config* c) {
   return true;
 }
 
-// y = [x_off; x_on] W^T (+ u B^T on the on rows, u = s x_on A^T) for S rows per stream,
-// through the dual-output GEMV; y [2 S, N] bf16 or fp32 (off rows first).
-int gemv_linear(const void* x, int64_t S, int64_t K, int64_t N, const void* W, const void* A,
-                const void* B, int64_t r, float s, void* u, void* y, bool f32, int* err,
-                cudaStream_t st) {
-  const void* x_on = static_cast<const uint8_t*>(x) + static_cast<size_t>(S) * K * 2;
-  if (r > 0 && hydra::launch_lora_down(x_on, S, K, A, r, s, u, st) != 0) return -3;
+// y = [x_off; x_on] W^T (+ u B^T on the on rows; u [S, r] = s x_on A^T, already computed by
+// the fused row kernel that produced x) for S rows per stream, through the dual-output GEMV;
+// y [2 S, N] bf16 or fp32 (off rows first).
+int gemv_linear(const void* x, int64_t S, int64_t K, int64_t N, const void* W, const void* B,
+                int64_t r, const void* u, void* y, bool f32, int* err, cudaStream_t st) {
   hydra::GemmArgs g;
   g.x_off = x;
-  g.x_on = x_on;
+  g.x_on = static_cast<const uint8_t*>(x) + static_cast<size_t>(S) * K * 2;
   g.M = S;
   g.K = K;
   g.N = N;
@@ -205,15 +203,18 @@ hydra_status hydra_generate_llama(const hydra_llama_config* cfg, const hydra_lla
   HY_TRY(hydra::launch_rmsnorm(h, w->final_norm, R, d, c.rms_eps, last, find, st));
 
   // one decode pass of the last drawn token (cur) at position P0 + step - 1, ending in the
-  // final-normed rows find
-  const hydra::RowMap dense{R, R, 0};
+  // final-normed rows find. Nine launches per layer: the residual add, the RMSNorm and the
+  // next projection's LoRA down-projection share one cluster kernel, as do the SwiGLU and
+  // the down projection's LoRA down-projection.
   auto decode_layers = [&]() -> int {
     int x = hydra::launch_embed(w->embed, V, d, cur, S, 2, hd, err, st);
+    const void* resid = nullptr;  // the previous layer's down projection, added into h
     for (int64_t l = 0; l < c.n_layers && x == 0; ++l) {
       const hydra_llama_layer& ly = w->layers[l];
-      if ((x = hydra::launch_rmsnorm(hd, ly.norm_attn, R, d, c.rms_eps, dense, ad, st)) != 0) break;
-      if ((x = gemv_linear(ad, S, d, 3 * d, ly.w_qkv, ly.a_qv, ly.b_qkv, 2 * r, s, ud, qkvd, false,
-                           err, st)) != 0)
+      if ((x = hydra::launch_row_norm_lora(hd, resid, ly.norm_attn, R, d, c.rms_eps, ad, S, ly.a_qv,
+                                           2 * r, s, ud, st)) != 0)
+        break;
+      if ((x = gemv_linear(ad, S, d, 3 * d, ly.w_qkv, ly.b_qkv, 2 * r, ud, qkvd, false, err, st)) != 0)
         break;
       if ((x = hydra::launch_decode_rope_append(qkvd, R, 3 * d, d, H, rope_table, P0, step, Pmax,
                                                 kcache(l), vcache(l), st)) != 0)
@@ -221,26 +222,24 @@ hydra_status hydra_generate_llama(const hydra_llama_config* cfg, const hydra_lla
       if ((x = hydra::launch_decode_attention(qkvd, R, 3 * d, H, kcache(l), vcache(l), P0, step,
                                               Pmax, attnd, d, st)) != 0)
         break;
-      if ((x = gemv_linear(attnd, S, d, d, ly.w_o, nullptr, nullptr, 0, s, ud, yd, false, err,
-                           st)) != 0)
+      if ((x = gemv_linear(attnd, S, d, d, ly.w_o, nullptr, 0, ud, yd, false, err, st)) != 0) break;
+      if ((x = hydra::launch_row_norm_lora(hd, yd, ly.norm_ffn, R, d, c.rms_eps, ad, S, ly.a_gu,
+                                           2 * r, s, ud, st)) != 0)
         break;
-      if ((x = hydra::launch_residual_add(hd, yd, R * d, st)) != 0) break;
-      if ((x = hydra::launch_rmsnorm(hd, ly.norm_ffn, R, d, c.rms_eps, dense, ad, st)) != 0) break;
-      if ((x = gemv_linear(ad, S, d, 2 * F, ly.w_gu, ly.a_gu, ly.b_gu, 2 * r, s, ud, gud, false,
-                           err, st)) != 0)
+      if ((x = gemv_linear(ad, S, d, 2 * F, ly.w_gu, ly.b_gu, 2 * r, ud, gud, false, err, st)) != 0)
         break;
-      if ((x = hydra::launch_swiglu_blocked(gud, R, F, md, st)) != 0) break;
-      if ((x = gemv_linear(md, S, F, d, ly.w_down, ly.a_down, ly.b_down, r, s, ud, yd, false, err,
-                           st)) != 0)
-        break;
-      x = hydra::launch_residual_add(hd, yd, R * d, st);
+      if ((x = hydra::launch_swiglu_lora(gud, R, F, md, S, ly.a_down, r, s, ud, st)) != 0) break;
+      if ((x = gemv_linear(md, S, F, d, ly.w_down, ly.b_down, r, ud, yd, false, err, st)) != 0) break;
+      resid = yd;
     }
-    if (x == 0) x = hydra::launch_rmsnorm(hd, w->final_norm, R, d, c.rms_eps, dense, find, st);
+    if (x == 0)
+      x = hydra::launch_row_norm_lora(hd, resid, w->final_norm, R, d, c.rms_eps, find, S, nullptr, 0,
+                                      s, nullptr, st);
     return x;
   };
   // the LM head on both streams' final rows and the draw of step *step
   auto draw = [&]() -> int {
-    int x = gemv_linear(find, S, d, V, w->lm_head, nullptr, nullptr, 0, s, ud, logits, true, err, st);
+    int x = gemv_linear(find, S, d, V, w->lm_head, nullptr, 0, nullptr, logits, true, err, st);
     if (x == 0)
       x = hydra::launch_sample_tokens(logits, S, V, gumbel, find, d, w->w_rm, step, n_steps, tokens,
                                       logp_actor, logp_ref, values, cur, st);
@@ -256,6 +255,7 @@ hydra_status hydra_generate_llama(const hydra_llama_config* cfg, const hydra_lla
   if (score != nullptr) {
     // the reward model (LoRA off) on the state after the last drawn token
     HY_TRY(decode_layers());
+    const hydra::RowMap dense{R, R, 0};
     HY_TRY(hydra::launch_head_dot(find, d, w->w_rm, dense, S, nullptr, 1, score, st));
   }
 #undef HY_TRY

@@ -141,6 +141,14 @@ int launch_sample_tokens(const float* logits, int64_t S, int64_t V, const float*
                          int64_t n_steps, int32_t* tokens, float* logp_a, float* logp_r,
                          float* values, int32_t* cur_ids, cudaStream_t st);
 int launch_step_advance(int* step, cudaStream_t st);
+// Thread-block-cluster row kernels of the decode step (8 CTAs per row): h += y (y may be
+// NULL), a = bf16(rmsnorm(h) w) and, for rows i >= S, u[i - S] = bf16(s a A^T) (A [r2, d] or
+// NULL); and m = SwiGLU(gu) (gate/up interleaved by 128) with u[i - S] = bf16(s m A^T).
+int launch_row_norm_lora(float* h, const void* y, const void* w, int64_t R, int64_t d, float eps,
+                         void* a, int64_t S, const void* A, int64_t r2, float s, void* u,
+                         cudaStream_t st);
+int launch_swiglu_lora(const void* gu, int64_t R, int64_t F, void* m, int64_t S, const void* A,
+                       int64_t r, float s, void* u, cudaStream_t st);
 
 // Row gather used by the per-row Llama kernels: output row i reads input row
 // (i / g_out) * g_in + off + i % g_out (g_out = g_in, off = 0 is the identity).
