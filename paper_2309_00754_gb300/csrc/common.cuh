@@ -128,6 +128,28 @@ __device__ __forceinline__ void pdl_launch_dependents() {
 }
 // Bring [p, p + bytes) into L2 (p and bytes multiples of 16). L2 is the device's point of
 // coherence, so a prefetch issued before pdl_wait() never makes a later read stale.
+// Thread-block clusters: this CTA's rank, a barrier over every thread of every CTA of the
+// cluster (release/acquire: shared-memory writes before it are visible to remote reads after
+// it), and a read of another CTA's shared memory at the address of `local` in this CTA.
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
+                   : "memory");
+}
+
+__device__ __forceinline__ float ld_cluster_f32(const float* local, uint32_t rank) {
+  uint32_t raddr;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(raddr) : "r"(smem_u32(local)), "r"(rank));
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(raddr) : "memory");
+  return v;
+}
+
 __device__ __forceinline__ void prefetch_l2_bulk(const void* p, uint32_t bytes) {
   asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(p)),
                "r"(bytes)

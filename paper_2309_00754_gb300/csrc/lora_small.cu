@@ -7,6 +7,9 @@
 //  * dual_lora_gemv: the dual-output linear for decode-shaped inputs (at most 16 token
 //    rows over both streams), y_off = x_off W^T, y_on = x_on W^T + u B^T, streaming W once
 //    (see the kernel). Used where a 128-row tcgen05 tile would be almost empty.
+#include <algorithm>
+#include <utility>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -16,11 +19,15 @@ namespace {
 // ---------------------------------------------------------------- lora_down
 //
 // u[M, r] = bf16(s * x A^T) as a skinny matrix product on the tensor cores (mma.sync
-// m16n8k16, bf16 in, fp32 accumulate): one CTA per 16 token rows and per 64 ranks; its 8
-// warps split K and reduce their partial tiles in shared memory. The contraction over k
-// is order-free, so inside each 32-wide chunk of k both operands use the same
-// permutation of k: the fragment slots a lane feeds in the chunk's two k-steps are its
-// 8 consecutive elements [8c, 8c + 8), which arrive with one 16-byte load per row.
+// m16n8k16, bf16 in, fp32 accumulate). A thread-block cluster of ck CTAs takes 16 token rows
+// and up to 64 ranks and splits K: each CTA's 8 warps split its slice again and reduce their
+// partial tiles in shared memory, and CTA rank 0 adds the ck tiles through distributed
+// shared memory in rank order (deterministic, no global scratch). The split puts enough
+// loads in flight: with one CTA per 16 rows, 2048 rows gave 128 CTAs, 12 % of the warp slots,
+// and the kernel waited on memory latency at 14 % of DRAM bandwidth. The contraction over k
+// is order-free, so inside each 32-wide chunk of k both operands use the same permutation of
+// k: the fragment slots a lane feeds in the chunk's two k-steps are its 8 consecutive
+// elements [8c, 8c + 8), which arrive with one 16-byte load per row.
 
 constexpr int kDownWarps = 8;
 
@@ -41,20 +48,25 @@ template <int NT>  // NT n-tiles of 8 ranks
 __global__ void __launch_bounds__(32 * kDownWarps)
     lora_down_kernel(const __nv_bfloat16* __restrict__ x, int M, int K,
                      const __nv_bfloat16* __restrict__ A, int r, float s,
-                     __nv_bfloat16* __restrict__ u) {
+                     __nv_bfloat16* __restrict__ u, int ck) {
   __shared__ float red[kDownWarps][16][NT * 8 + 1];
+  __shared__ float tile[16][NT * 8];  // this CTA's sum over its warps
   pdl_launch_dependents();
   pdl_wait();  // x is written by the preceding kernel
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int g = lane >> 2, c = lane & 3;
-  const int row0 = blockIdx.x * 16;
+  const uint32_t rank = ck > 1 ? cluster_rank() : 0u;
+  const int row0 = (blockIdx.x / ck) * 16;
   const int n_base = blockIdx.y * NT * 8;
-  // this warp's K range, in chunks of 32
+  // this CTA's K slice, then this warp's part of it, in chunks of 32
   const int nchunk = (K + 31) / 32;
-  const int per = (nchunk + kDownWarps - 1) / kDownWarps;
-  const int ch0 = warp * per;
-  const int ch1 = min(nchunk, ch0 + per);
+  const int per_cta = (nchunk + ck - 1) / ck;
+  const int cta0 = static_cast<int>(rank) * per_cta;
+  const int cta1 = min(nchunk, cta0 + per_cta);
+  const int per = (max(cta1 - cta0, 0) + kDownWarps - 1) / kDownWarps;
+  const int ch0 = cta0 + warp * per;
+  const int ch1 = min(cta1, ch0 + per);
 
   const bool r_lo = row0 + g < M, r_hi = row0 + g + 8 < M;
   const __nv_bfloat16* x_lo = x + static_cast<size_t>(r_lo ? row0 + g : 0) * K + 8 * c;
@@ -101,9 +113,42 @@ __global__ void __launch_bounds__(32 * kDownWarps)
     float v = 0.f;
 #pragma unroll
     for (int w = 0; w < kDownWarps; ++w) v += red[w][rr][cc];
-    const int m = row0 + rr, n = n_base + cc;
-    if (m < M && n < r) u[static_cast<size_t>(m) * r + n] = __float2bfloat16_rn(s * v);
+    tile[rr][cc] = v;
   }
+  if (ck > 1) cluster_sync_all();  // every CTA's tile is complete and visible
+  else __syncthreads();
+  if (rank == 0) {
+    for (int e = threadIdx.x; e < 16 * NT * 8; e += blockDim.x) {
+      const int rr = e / (NT * 8), cc = e % (NT * 8);
+      float v = tile[rr][cc];
+      for (int q = 1; q < ck; ++q) v += ld_cluster_f32(&tile[rr][cc], static_cast<uint32_t>(q));
+      const int m = row0 + rr, n = n_base + cc;
+      if (m < M && n < r) u[static_cast<size_t>(m) * r + n] = __float2bfloat16_rn(s * v);
+    }
+  }
+  if (ck > 1) cluster_sync_all();  // rank 0's remote reads end before any CTA exits
+}
+
+// cudaLaunchKernelEx with a (ck, 1, 1) cluster (none when ck == 1) and programmatic
+// dependent launch
+template <typename... KArgs, typename... Args>
+cudaError_t launch_down(void (*kernel)(KArgs...), dim3 grid, int ck, cudaStream_t st,
+                        Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(32 * kDownWarps);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = static_cast<unsigned>(ck);
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = ck > 1 ? 2 : 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
 
 // ---------------------------------------------------------------- dual_lora_gemv
@@ -332,22 +377,38 @@ void launch_gemv_t(const GemmArgs& a, cudaStream_t stream) {
 int launch_lora_down(const void* x, int64_t M, int64_t K, const void* A, int64_t r, float s,
                      void* u, cudaStream_t stream) {
   if (M == 0 || r == 0) return 0;
-  const dim3 block(32 * kDownWarps);
+  static int nsm = 0;
+  if (nsm == 0) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return -1;
+  }
   const auto* xp = static_cast<const __nv_bfloat16*>(x);
   const auto* ap = static_cast<const __nv_bfloat16*>(A);
   auto* up = static_cast<__nv_bfloat16*>(u);
-  const unsigned gx = static_cast<unsigned>((M + 15) / 16);
+  const int64_t tiles = (M + 15) / 16;
+  const int64_t ny = r <= 32 ? 1 : (r + 63) / 64;
+  // K split over a cluster: about 4 CTAs per SM (2 above 16 ranks, where each CTA already
+  // reads more of A than of x), each warp with at least 4 chunks of 32 (one unrolled batch of
+  // loads)
+  const int64_t target = (r > 16 ? 2LL : 4LL) * nsm;
+  int64_t ck = (target + tiles * ny - 1) / (tiles * ny);
+  ck = std::min<int64_t>(ck, std::max<int64_t>(1, K / (32 * 4 * kDownWarps)));
+  ck = std::max<int64_t>(1, std::min<int64_t>(8, ck));
+  const dim3 grid(static_cast<unsigned>(tiles * ck), static_cast<unsigned>(ny));
   const int Mi = static_cast<int>(M), Ki = static_cast<int>(K), ri = static_cast<int>(r);
+  const int cki = static_cast<int>(ck);
+  cudaError_t e;
   if (r <= 8)
-    launch_pdl(lora_down_kernel<1>, dim3(gx, 1), block, 0, stream, xp, Mi, Ki, ap, ri, s, up);
+    e = launch_down(lora_down_kernel<1>, grid, cki, stream, xp, Mi, Ki, ap, ri, s, up, cki);
   else if (r <= 16)
-    launch_pdl(lora_down_kernel<2>, dim3(gx, 1), block, 0, stream, xp, Mi, Ki, ap, ri, s, up);
+    e = launch_down(lora_down_kernel<2>, grid, cki, stream, xp, Mi, Ki, ap, ri, s, up, cki);
   else if (r <= 32)
-    launch_pdl(lora_down_kernel<4>, dim3(gx, 1), block, 0, stream, xp, Mi, Ki, ap, ri, s, up);
+    e = launch_down(lora_down_kernel<4>, grid, cki, stream, xp, Mi, Ki, ap, ri, s, up, cki);
   else
-    launch_pdl(lora_down_kernel<8>, dim3(gx, static_cast<unsigned>((r + 63) / 64)), block, 0,
-               stream, xp, Mi, Ki, ap, ri, s, up);
-  return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
+    e = launch_down(lora_down_kernel<8>, grid, cki, stream, xp, Mi, Ki, ap, ri, s, up, cki);
+  return e == cudaSuccess ? 0 : -3;
 }
 
 int launch_dual_lora_gemv(const GemmArgs& a, cudaStream_t stream) {
