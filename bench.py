@@ -500,7 +500,10 @@ class HydraGenerateLlama7B(HydraScoringLlama7B):
         mean_pos = self.P0 + self.n_steps / 2
         kv_layer = R * mean_pos * 2 * d * 2 + R * 2 * d * 2
         self.step_bytes = nl * (w_layer + lora_layer + kv_layer) + V * d * 2 + R * V * 4 * 2
-        per_layer = 14
+        # launches of one call: prefill (rotary table, embed, 11 per layer, final norm, draw of
+        # 3), each further draw (embed, 9 per layer, final norm, 3), the score pass (embed, 9
+        # per layer, final norm, head)
+        per_layer = 9
         decode = 1 + per_layer * nl + 1 + 3
         prefill = 2 + 11 * nl + 1 + 3
         self.launches_per_step = prefill + (self.n_steps - 1) * decode + (1 + per_layer * nl + 2)

@@ -3,8 +3,9 @@
 // step runs the R = 2 S stacked rows of the LoRA-off and LoRA-on streams of S sequences; the
 // projections are the dual-output GEMV, the rest is here:
 //   kv_store_prefill   the prompt's rotated keys and its values into the cache
-//   decode_rope_append rotary embedding of the new token's q and k, k and v appended
-//   decode_attention   one query row per (row, head) against the cached positions 0..pos
+//   decode_attention   rotary embedding of the new token's q and k, its k and v appended to
+//                      the cache, then one query row per (head, row) against the cached
+//                      positions 0..pos
 //   swiglu_blocked     SwiGLU on gate/up columns interleaved in blocks of 128
 //   sample_tokens      per sequence: log-softmax of both heads, the Gumbel-max draw from the
 //                      actor's logits, both log-probabilities of the drawn token, the value
@@ -38,40 +39,6 @@ __global__ void kv_store_prefill_kernel(const __nv_bfloat16* __restrict__ qkv, i
   }
 }
 
-// One block per (head, row): q rotated in place, k rotated into the cache, v copied. The
-// same explicit roundings as the prefill's rotary (no contraction), from the same table.
-__global__ void decode_rope_append_kernel(__nv_bfloat16* __restrict__ qkv, int ld, int d, int H,
-                                          const float2* __restrict__ table, int P0,
-                                          const int* __restrict__ step, int Pmax,
-                                          __nv_bfloat16* __restrict__ ck,
-                                          __nv_bfloat16* __restrict__ cv) {
-  pdl_wait();
-  pdl_launch_dependents();
-  const int h = blockIdx.x, i = blockIdx.y;
-  const int pos = P0 + *step - 1;
-  if (pos < 0 || pos >= Pmax) return;  // the host keeps every step inside the cache
-  constexpr int half = kDh / 2;
-  __nv_bfloat16* row = qkv + static_cast<size_t>(i) * ld;
-  const size_t slot = ((static_cast<size_t>(i) * H + h) * Pmax + pos) * kDh;
-  const int j = threadIdx.x & (half - 1);
-  const int blk = threadIdx.x / half;  // 0: q, 1: k (128 threads)
-  const float2 cs = table[static_cast<size_t>(pos) * half + j];
-  __nv_bfloat16* x = row + blk * d + h * kDh;
-  const float x1 = __bfloat162float(x[j]), x2 = __bfloat162float(x[j + half]);
-  const __nv_bfloat16 o1 = __float2bfloat16_rn(__fsub_rn(__fmul_rn(x1, cs.x), __fmul_rn(x2, cs.y)));
-  const __nv_bfloat16 o2 = __float2bfloat16_rn(__fadd_rn(__fmul_rn(x1, cs.y), __fmul_rn(x2, cs.x)));
-  if (blk == 0) {
-    x[j] = o1;
-    x[j + half] = o2;
-  } else {
-    ck[slot + j] = o1;
-    ck[slot + j + half] = o2;
-  }
-  if (threadIdx.x < kDh / 8)
-    *reinterpret_cast<uint4*>(cv + slot + 8 * threadIdx.x) =
-        *reinterpret_cast<const uint4*>(row + 2 * d + h * kDh + 8 * threadIdx.x);
-}
-
 constexpr int kAttnThreads = 256;
 constexpr int kAttnWarps = kAttnThreads / 32;
 
@@ -99,30 +66,56 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
   return v;
 }
 
-// One block per (head, row): scores of the npos = pos + 1 cached keys into shared memory
+// One block per (head, row): the new token's rotary and cache append for this head, then the
+// scores of the npos = pos + 1 cached keys into shared memory
 // (groups of 8 lanes per key, 32 bytes each, reduced by shuffles), the softmax over them,
 // then the weighted sum of the values (lane = 4 output dimensions, warps split positions).
 __global__ void __launch_bounds__(kAttnThreads)
-    decode_attention_kernel(const __nv_bfloat16* __restrict__ qkv, int ld, int H,
-                            const __nv_bfloat16* __restrict__ ck,
-                            const __nv_bfloat16* __restrict__ cv, int P0,
+    decode_attention_kernel(const __nv_bfloat16* __restrict__ qkv, int ld, int d, int H,
+                            const float2* __restrict__ table, __nv_bfloat16* __restrict__ ck,
+                            __nv_bfloat16* __restrict__ cv, int P0,
                             const int* __restrict__ step, int Pmax, float scale,
                             __nv_bfloat16* __restrict__ out, int ld_out) {
   extern __shared__ float sc[];  // [Pmax] scores, then [kAttnWarps][kDh] partial outputs
   __shared__ float red[kAttnWarps];
+  __shared__ __align__(16) __nv_bfloat16 qs[kDh];  // this head's rotated query
   pdl_wait();
   pdl_launch_dependents();
   const int h = blockIdx.x, i = blockIdx.y;
-  const int npos = min(P0 + *step, Pmax);
+  const int pos = P0 + *step - 1;
+  if (pos < 0 || pos >= Pmax) return;  // the host keeps every step inside the cache
+  const int npos = pos + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const __nv_bfloat16* K = ck + (static_cast<size_t>(i) * H + h) * Pmax * kDh;
-  const __nv_bfloat16* Vc = cv + (static_cast<size_t>(i) * H + h) * Pmax * kDh;
+  __nv_bfloat16* K = ck + (static_cast<size_t>(i) * H + h) * Pmax * kDh;
+  __nv_bfloat16* Vc = cv + (static_cast<size_t>(i) * H + h) * Pmax * kDh;
+  {
+    // the new token: rotary embedding of this head's q (into shared memory) and k (into the
+    // cache at pos), and its v copied into the cache; the same explicit roundings as the
+    // prefill's rotary, from the same table
+    constexpr int half = kDh / 2;
+    const __nv_bfloat16* row = qkv + static_cast<size_t>(i) * ld;
+    if (threadIdx.x < 2 * half) {
+      const int j = threadIdx.x & (half - 1), blk = threadIdx.x / half;  // 0: q, 1: k
+      const float2 cs = table[static_cast<size_t>(pos) * half + j];
+      const __nv_bfloat16* x = row + blk * d + h * kDh;
+      const float x1 = __bfloat162float(x[j]), x2 = __bfloat162float(x[j + half]);
+      const __nv_bfloat16 o1 = __float2bfloat16_rn(__fsub_rn(__fmul_rn(x1, cs.x), __fmul_rn(x2, cs.y)));
+      const __nv_bfloat16 o2 = __float2bfloat16_rn(__fadd_rn(__fmul_rn(x1, cs.y), __fmul_rn(x2, cs.x)));
+      __nv_bfloat16* dst = blk == 0 ? qs : K + static_cast<size_t>(pos) * kDh;
+      dst[j] = o1;
+      dst[j + half] = o2;
+    } else if (threadIdx.x < 2 * half + kDh / 8) {
+      const int e = 8 * (threadIdx.x - 2 * half);
+      *reinterpret_cast<uint4*>(Vc + static_cast<size_t>(pos) * kDh + e) =
+          *reinterpret_cast<const uint4*>(row + 2 * d + h * kDh + e);
+    }
+  }
+  __syncthreads();  // q in shared memory, the new k and v visible to the whole block
   const int g = lane >> 3, sub = lane & 7;
   float qf[16];
   {
-    const __nv_bfloat16* q = qkv + static_cast<size_t>(i) * ld + h * kDh + 16 * sub;
-    const uint4 a = *reinterpret_cast<const uint4*>(q);
-    const uint4 b = *reinterpret_cast<const uint4*>(q + 8);
+    const uint4 a = *reinterpret_cast<const uint4*>(qs + 16 * sub);
+    const uint4 b = *reinterpret_cast<const uint4*>(qs + 16 * sub + 8);
     const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
@@ -249,16 +242,40 @@ __device__ __forceinline__ float row_block_sum(float v, float* red) {
   return t;
 }
 
+// The LoRA factor A is frozen: a CTA copies its slice A[0:r2][c0:c0+n] into shared memory
+// with cp.async before it waits on the preceding kernel, so the copy overlaps that kernel's
+// tail. Slices above kMaxAPrefetch bytes are read from global memory instead.
+constexpr int kMaxAPrefetch = 64 * 1024;
+
+__device__ __forceinline__ void prefetch_a_slice(const __nv_bfloat16* __restrict__ A, int K,
+                                                 int c0, int n, int r2, __nv_bfloat16* As) {
+  const int per_row = n / 8;  // 16-byte pieces per row (n % 8 == 0)
+  for (int c = threadIdx.x; c < r2 * per_row; c += kRowThreads) {
+    const int j = c / per_row, e = (c - j * per_row) * 8;
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(As + j * n + e)),
+                 "l"(A + static_cast<size_t>(j) * K + c0 + e)
+                 : "memory");
+  }
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+
+__device__ __forceinline__ void wait_a_slice() {
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
+  __syncthreads();
+}
+
 // Partial LoRA down-projection of this CTA's slice: up[j] = sum_e xs[e] A[j][c0 + e] for
 // j < r2 (warps take j in turn, lanes 4 columns at a time); then rank 0 adds the kCl
-// partials in rank order and writes u = bf16(s * sum). xs holds the slice's bf16 values.
+// partials in rank order and writes u = bf16(s * sum). xs holds the slice's bf16 values; As,
+// if not NULL, the prefetched slice of A ([r2][n]).
 __device__ __forceinline__ void lora_slice(const float* xs, int n, int c0, int K,
-                                           const __nv_bfloat16* __restrict__ A, int r2, float s,
-                                           float* up, __nv_bfloat16* __restrict__ u_row,
-                                           uint32_t rank) {
+                                           const __nv_bfloat16* __restrict__ A,
+                                           const __nv_bfloat16* As, int r2, float s, float* up,
+                                           __nv_bfloat16* __restrict__ u_row, uint32_t rank) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int j = warp; j < r2; j += kRowWarps) {
-    const __nv_bfloat16* aj = A + static_cast<size_t>(j) * K + c0;
+    // the slice from shared memory when it was prefetched, else from global memory
+    const __nv_bfloat16* aj = As ? As + static_cast<size_t>(j) * n : A + static_cast<size_t>(j) * K + c0;
     float acc = 0.f;
     for (int e = 4 * lane; e < n; e += 128) {
       const uint2 q = *reinterpret_cast<const uint2*>(aj + e);
@@ -291,15 +308,19 @@ __global__ void __launch_bounds__(kRowThreads)
                          const __nv_bfloat16* __restrict__ w, int d, float eps,
                          __nv_bfloat16* __restrict__ a, int S, const __nv_bfloat16* __restrict__ A,
                          int r2, float s, __nv_bfloat16* __restrict__ u) {
-  extern __shared__ float xs[];  // this CTA's slice of the row
+  extern __shared__ float xs[];  // this CTA's slice of the row, then the prefetched A slice
   __shared__ float red[kRowWarps];
   __shared__ float part;
   __shared__ float up[kMaxR2];
-  pdl_wait();
-  pdl_launch_dependents();
   const uint32_t rank = cluster_rank();
   const int row = blockIdx.y;
   const int n = d / kCl, c0 = static_cast<int>(rank) * n;
+  const bool lora = A != nullptr && row >= S;
+  __nv_bfloat16* As = (lora && r2 * n * 2 <= kMaxAPrefetch) ? reinterpret_cast<__nv_bfloat16*>(xs + n)
+                                                             : nullptr;
+  if (As) prefetch_a_slice(A, d, c0, n, r2, As);
+  pdl_wait();
+  pdl_launch_dependents();
   float* hr = h + static_cast<size_t>(row) * d + c0;
   float ss = 0.f;
   for (int e = 4 * threadIdx.x; e < n; e += 4 * kRowThreads) {
@@ -338,9 +359,10 @@ __global__ void __launch_bounds__(kRowThreads)
     xs[e + 2] = b23.x;
     xs[e + 3] = b23.y;
   }
-  __syncthreads();
-  if (A != nullptr && row >= S)
-    lora_slice(xs, n, c0, d, A, r2, s, up, u + static_cast<size_t>(row - S) * r2, rank);
+  if (As) wait_a_slice();
+  else __syncthreads();
+  if (lora)
+    lora_slice(xs, n, c0, d, A, As, r2, s, up, u + static_cast<size_t>(row - S) * r2, rank);
   else
     cluster_sync_all();  // the same cluster barriers on every path
   cluster_sync_all();    // rank 0's remote reads finish before any CTA leaves
@@ -353,13 +375,17 @@ __global__ void __launch_bounds__(kRowThreads)
     swiglu_lora_kernel(const __nv_bfloat16* __restrict__ gu, int F, __nv_bfloat16* __restrict__ m,
                        int S, const __nv_bfloat16* __restrict__ A, int r, float s,
                        __nv_bfloat16* __restrict__ u) {
-  extern __shared__ float xs[];
+  extern __shared__ float xs[];  // this CTA's slice of m, then the prefetched A slice
   __shared__ float up[kMaxR2];
-  pdl_wait();
-  pdl_launch_dependents();
   const uint32_t rank = cluster_rank();
   const int row = blockIdx.y;
   const int n = F / kCl, c0 = static_cast<int>(rank) * n;
+  const bool lora = A != nullptr && row >= S;
+  __nv_bfloat16* As = (lora && r * n * 2 <= kMaxAPrefetch) ? reinterpret_cast<__nv_bfloat16*>(xs + n)
+                                                            : nullptr;
+  if (As) prefetch_a_slice(A, F, c0, n, r, As);
+  pdl_wait();
+  pdl_launch_dependents();
   const __nv_bfloat16* g = gu + static_cast<size_t>(row) * 2 * F;
   __nv_bfloat16* mr = m + static_cast<size_t>(row) * F + c0;
   for (int e = 4 * threadIdx.x; e < n; e += 4 * kRowThreads) {
@@ -380,9 +406,10 @@ __global__ void __launch_bounds__(kRowThreads)
     xs[e + 2] = b23.x;
     xs[e + 3] = b23.y;
   }
-  __syncthreads();
-  if (A != nullptr && row >= S)
-    lora_slice(xs, n, c0, F, A, r, s, up, u + static_cast<size_t>(row - S) * r, rank);
+  if (As) wait_a_slice();
+  else __syncthreads();
+  if (lora)
+    lora_slice(xs, n, c0, F, A, As, r, s, up, u + static_cast<size_t>(row - S) * r, rank);
   else
     cluster_sync_all();
   cluster_sync_all();
@@ -488,27 +515,13 @@ int launch_kv_store_prefill(const void* qkv, int64_t R, int64_t P0, int64_t ld, 
   return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
 }
 
-int launch_decode_rope_append(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t H,
-                              const void* table, int64_t P0, const int* step, int64_t Pmax,
-                              void* ck, void* cv, cudaStream_t st) {
-  if (R == 0) return 0;
-  const cudaError_t e = launch_pdl(decode_rope_append_kernel,
-                                   dim3(static_cast<unsigned>(H), static_cast<unsigned>(R)),
-                                   dim3(kDh), 0, st, static_cast<__nv_bfloat16*>(qkv),
-                                   static_cast<int>(ld), static_cast<int>(d), static_cast<int>(H),
-                                   static_cast<const float2*>(table), static_cast<int>(P0), step,
-                                   static_cast<int>(Pmax), static_cast<__nv_bfloat16*>(ck),
-                                   static_cast<__nv_bfloat16*>(cv));
-  return e == cudaSuccess ? 0 : -3;
-}
-
 size_t decode_attention_smem(int64_t Pmax) {
   return static_cast<size_t>(Pmax) * 4 + static_cast<size_t>(kAttnWarps) * kDh * 4;
 }
 
-int launch_decode_attention(const void* qkv, int64_t R, int64_t ld, int64_t H, const void* ck,
-                            const void* cv, int64_t P0, const int* step, int64_t Pmax, void* out,
-                            int64_t ld_out, cudaStream_t st) {
+int launch_decode_attention(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t H,
+                            const void* table, void* ck, void* cv, int64_t P0, const int* step,
+                            int64_t Pmax, void* out, int64_t ld_out, cudaStream_t st) {
   if (R == 0) return 0;
   const size_t smem = decode_attention_smem(Pmax);
   static size_t attr = 0;
@@ -521,8 +534,9 @@ int launch_decode_attention(const void* qkv, int64_t R, int64_t ld, int64_t H, c
   const cudaError_t e = launch_pdl(
       decode_attention_kernel, dim3(static_cast<unsigned>(H), static_cast<unsigned>(R)),
       dim3(kAttnThreads), smem, st, static_cast<const __nv_bfloat16*>(qkv), static_cast<int>(ld),
-      static_cast<int>(H), static_cast<const __nv_bfloat16*>(ck),
-      static_cast<const __nv_bfloat16*>(cv), static_cast<int>(P0), step, static_cast<int>(Pmax),
+      static_cast<int>(d), static_cast<int>(H), static_cast<const float2*>(table),
+      static_cast<__nv_bfloat16*>(ck), static_cast<__nv_bfloat16*>(cv), static_cast<int>(P0),
+      step, static_cast<int>(Pmax),
       1.0f / sqrtf(static_cast<float>(kDh)), static_cast<__nv_bfloat16*>(out),
       static_cast<int>(ld_out));
   return e == cudaSuccess ? 0 : -3;
@@ -546,6 +560,17 @@ int launch_sample_tokens(const float* logits, int64_t S, int64_t V, const float*
       static_cast<const __nv_bfloat16*>(w_rm), step, static_cast<int>(n_steps), tokens, logp_a,
       logp_r, values, cur_ids);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
+}
+
+// Raise a kernel's dynamic shared-memory limit when a launch needs more than the default
+// (once per kernel and size: `done` remembers the largest limit set).
+static int set_smem_limit(const void* kernel, size_t bytes, size_t& done) {
+  if (bytes <= 48 * 1024 || bytes <= done) return 0;
+  if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(bytes)) != cudaSuccess)
+    return -1;
+  done = bytes;
+  return 0;
 }
 
 // cudaLaunchKernelEx with a (kCl, 1, 1) cluster and programmatic dependent launch
@@ -573,8 +598,15 @@ int launch_row_norm_lora(float* h, const void* y, const void* w, int64_t R, int6
                          void* a, int64_t S, const void* A, int64_t r2, float s, void* u,
                          cudaStream_t st) {
   if (R == 0) return 0;
-  if (d % (4 * kCl) != 0 || r2 > kMaxR2) return -1;
-  const size_t smem = static_cast<size_t>(d / kCl) * 4;
+  if (d % (8 * kCl) != 0 || r2 > kMaxR2) return -1;
+  const size_t n = static_cast<size_t>(d / kCl);
+  const size_t a_bytes = n * 2 * static_cast<size_t>(r2);
+  const size_t smem = n * 4 + (A != nullptr && a_bytes <= kMaxAPrefetch ? a_bytes : 0);
+  static size_t done_resid = 0, done_plain = 0;
+  if (set_smem_limit(y != nullptr ? reinterpret_cast<const void*>(row_norm_lora_kernel<true>)
+                                  : reinterpret_cast<const void*>(row_norm_lora_kernel<false>),
+                     smem, y != nullptr ? done_resid : done_plain) != 0)
+    return -1;
   const dim3 grid(kCl, static_cast<unsigned>(R));
   cudaError_t e;
   if (y != nullptr)
@@ -595,8 +627,12 @@ int launch_row_norm_lora(float* h, const void* y, const void* w, int64_t R, int6
 int launch_swiglu_lora(const void* gu, int64_t R, int64_t F, void* m, int64_t S, const void* A,
                        int64_t r, float s, void* u, cudaStream_t st) {
   if (R == 0) return 0;
-  if (F % (4 * kCl) != 0 || r > kMaxR2) return -1;
-  const size_t smem = static_cast<size_t>(F / kCl) * 4;
+  if (F % (8 * kCl) != 0 || r > kMaxR2) return -1;
+  const size_t n = static_cast<size_t>(F / kCl);
+  const size_t a_bytes = n * 2 * static_cast<size_t>(r);
+  const size_t smem = n * 4 + (A != nullptr && a_bytes <= kMaxAPrefetch ? a_bytes : 0);
+  static size_t done = 0;
+  if (set_smem_limit(reinterpret_cast<const void*>(swiglu_lora_kernel), smem, done) != 0) return -1;
   const cudaError_t e = launch_cluster(
       swiglu_lora_kernel, dim3(kCl, static_cast<unsigned>(R)), smem, st,
       static_cast<const __nv_bfloat16*>(gu), static_cast<int>(F), static_cast<__nv_bfloat16*>(m),

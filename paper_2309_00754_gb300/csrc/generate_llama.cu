@@ -7,10 +7,11 @@
 // Prefill: the prompt of both streams through the tcgen05 layer loop of the scoring pass
 // (rotary, SwiGLU and residual epilogues), with each layer's rotated keys and values copied
 // into the cache. Decode step (R = 2 S rows: off rows then on rows): embed the last drawn
-// token, per layer [residual + RMSNorm + q/v LoRA down] -> q/k/v GEMV -> rotary + cache
-// append -> attention over the cache -> o GEMV -> [residual + RMSNorm + gate/up LoRA down]
+// token, per layer [residual + RMSNorm + q/v LoRA down] -> q/k/v GEMV -> [rotary + cache
+// append + attention over the cache] -> o GEMV -> [residual + RMSNorm + gate/up LoRA down]
 // -> gate/up GEMV -> [SwiGLU + down LoRA down] -> down GEMV; then [residual + final RMSNorm],
-// the LM-head GEMV (fp32 logits) and the draw. Brackets are thread-block-cluster kernels.
+// the LM-head GEMV (fp32 logits) and the draw. The norm brackets are thread-block-cluster
+// kernels.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -203,7 +204,7 @@ hydra_status hydra_generate_llama(const hydra_llama_config* cfg, const hydra_lla
   HY_TRY(hydra::launch_rmsnorm(h, w->final_norm, R, d, c.rms_eps, last, find, st));
 
   // one decode pass of the last drawn token (cur) at position P0 + step - 1, ending in the
-  // final-normed rows find. Nine launches per layer: the residual add, the RMSNorm and the
+  // final-normed rows find. Eight launches per layer: the residual add, the RMSNorm and the
   // next projection's LoRA down-projection share one cluster kernel, as do the SwiGLU and
   // the down projection's LoRA down-projection.
   auto decode_layers = [&]() -> int {
@@ -216,11 +217,8 @@ hydra_status hydra_generate_llama(const hydra_llama_config* cfg, const hydra_lla
         break;
       if ((x = gemv_linear(ad, S, d, 3 * d, ly.w_qkv, ly.b_qkv, 2 * r, ud, qkvd, false, err, st)) != 0)
         break;
-      if ((x = hydra::launch_decode_rope_append(qkvd, R, 3 * d, d, H, rope_table, P0, step, Pmax,
-                                                kcache(l), vcache(l), st)) != 0)
-        break;
-      if ((x = hydra::launch_decode_attention(qkvd, R, 3 * d, H, kcache(l), vcache(l), P0, step,
-                                              Pmax, attnd, d, st)) != 0)
+      if ((x = hydra::launch_decode_attention(qkvd, R, 3 * d, d, H, rope_table, kcache(l),
+                                              vcache(l), P0, step, Pmax, attnd, d, st)) != 0)
         break;
       if ((x = gemv_linear(attnd, S, d, d, ly.w_o, nullptr, 0, ud, yd, false, err, st)) != 0) break;
       if ((x = hydra::launch_row_norm_lora(hd, yd, ly.norm_ffn, R, d, c.rms_eps, ad, S, ly.a_gu,

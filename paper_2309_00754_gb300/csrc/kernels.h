@@ -128,13 +128,12 @@ int stacked_linear(int prof_class, const void* x, int64_t T, int64_t K, int64_t 
 // bf16; step: device counter of the current draw (the new token sits at P0 + step - 1).
 int launch_kv_store_prefill(const void* qkv, int64_t R, int64_t P0, int64_t ld, int64_t d,
                             int64_t H, int64_t Pmax, void* ck, void* cv, cudaStream_t st);
-int launch_decode_rope_append(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t H,
-                              const void* table, int64_t P0, const int* step, int64_t Pmax,
-                              void* ck, void* cv, cudaStream_t st);
 size_t decode_attention_smem(int64_t Pmax);
-int launch_decode_attention(const void* qkv, int64_t R, int64_t ld, int64_t H, const void* ck,
-                            const void* cv, int64_t P0, const int* step, int64_t Pmax, void* out,
-                            int64_t ld_out, cudaStream_t st);
+// rotary of the new token's q and k (table [Pmax][64] (cos, sin)), its k and v appended to
+// the cache at P0 + step - 1, then attention of q over the cached positions
+int launch_decode_attention(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t H,
+                            const void* table, void* ck, void* cv, int64_t P0, const int* step,
+                            int64_t Pmax, void* out, int64_t ld_out, cudaStream_t st);
 int launch_swiglu_blocked(const void* gu, int64_t R, int64_t F, void* m, cudaStream_t st);
 int launch_sample_tokens(const float* logits, int64_t S, int64_t V, const float* gumbel,
                          const void* fin, int64_t d, const void* w_rm, const int* step,
