@@ -470,8 +470,8 @@ typedef struct hydra_llama_lora {
 size_t hydra_generate_llama_workspace_size(const hydra_llama_config* cfg, int64_t S);
 
 /*
- * Generation with the actor (Algorithms 1 and 2: "generate sequence using the policy for T
- * steps"; J-Hydra-PPO retains the critic head's values while generating), KV-cached, with
+ * Generation with the actor (Algorithms 1 and 2: the actor samples each sequence for T steps;
+ * J-Hydra-PPO keeps the critic head's values while sampling), KV-cached, with
  * the LoRA-off stream decoded beside the actor so that each drawn token also gets its
  * reference log-probability (one read of W serves both streams' rows).
  * For each of S sequences of P0 = cfg->prompt_len prompt tokens and steps t < n_steps:

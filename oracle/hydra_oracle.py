@@ -19,8 +19,8 @@ Usage of PPO"):
   * §3 "Dynamic LoRA" -- the reference policy is the actor with its LoRA parameters
     ignored, pi_ref <- LO(pi_theta); likewise the reward model is LO(critic).
   * §3 "Stage 2: Hydra-PPO" and Algorithm 1 (J-Hydra-PPO) / Algorithm 2 (Hydra-PPO) --
-    one frozen base; "turn LoRA off ... to compute reward and reference log
-    probabilities"; "use reward and reference log probability to calculate A-hat".
+    one frozen base; the LoRA-off model supplies the reward and the reference
+    log-probabilities, and the advantages are computed from them.
   * Appendix B "Experiment Details" -- KL coefficient beta = 0.02, GAE gamma = 1.0,
     lambda = 0.95, LoRA rank 128.
 
@@ -45,7 +45,7 @@ The full 32-layer Llama composition (`llama_score`, and the three-stream Hydra-P
 `llama_score_hydra`) is pinned only through its per-op pieces and small-size invariants
 (LoRA off, causality, one LoRA set reducing Hydra-PPO to J-Hydra-PPO, a critic set that
 moves only the values): parity unpinned for the composition as a whole.
-Generation (`llama_generate`, Alg. 1 and 2 "generate sequence ... for T steps") recomputes
+Generation (`llama_generate`, the sampling phase of Alg. 1 and 2) recomputes
 the whole stack at every step, with no cache, and draws each token by the Gumbel-max trick
 from noise that is an input (`gumbel_argmax`, pinned by the empirical distribution of its
 draws). It is pinned by its equality with `llama_score` on the finished sequence, so it
@@ -126,8 +126,8 @@ def dual_lora_linear(x_off, x_on, W, A, B, s, out_bf16=True):
 
 
 # ---------------------------------------------------------------------------
-# a4: log-probability of the sampled token (Alg. 1/2 "reference log probabilities";
-# §2 ratio r(theta) = pi_theta / pi_old needs the actor's log-probabilities too)
+# a4: log-probability of the sampled token (Alg. 1/2: the LoRA-off model gives the reference
+# log-probabilities; the §2 ratio r(theta) = pi_theta / pi_old needs the actor's too)
 # ---------------------------------------------------------------------------
 
 
@@ -145,8 +145,8 @@ def log_softmax_gather(z, ids):
 
 
 # ---------------------------------------------------------------------------
-# a5: KL-penalised per-token reward (§2 reference "used to prevent reward divergence";
-# Appendix B KL coefficient beta; Alg. 1/2 reward from the LoRA-off model)
+# a5: KL-penalised per-token reward (§2: a KL term against the reference policy keeps the
+# actor near it; Appendix B KL coefficient beta; Alg. 1/2 reward from the LoRA-off model)
 # ---------------------------------------------------------------------------
 
 
@@ -186,8 +186,9 @@ def token_logprobs_kl(z_actor, z_ref, ids, lengths, score, beta, S, L):
 
 
 # ---------------------------------------------------------------------------
-# a7: generalised advantage estimation (§2 "GAE uses V(x,y) to construct A-hat", critic
-# trained on returns; Appendix B gamma = 1.0, lambda = 0.95; Alg. 1/2 "calculate A-hat")
+# a7: generalised advantage estimation (§2: the advantage estimates come from GAE over the
+# critic's values V(x, y), and the critic is trained on the returns; Appendix B gamma = 1.0,
+# lambda = 0.95; Alg. 1/2 compute the advantages after scoring)
 # ---------------------------------------------------------------------------
 
 
@@ -437,7 +438,7 @@ def llama_score_hydra(weights, lora_critic, ids, prompt_len, cfg, seq_lengths=No
 
 # ---------------------------------------------------------------------------
 # Update side of PPO (§2 Stage 3: ratio r(theta), clipped surrogate L^CLIP, squared-error
-# value loss on the returns; Alg. 1/2 "optimize surrogate L")
+# value loss on the returns; Alg. 1/2 optimise this surrogate after each batch is scored)
 # ---------------------------------------------------------------------------
 
 
@@ -493,8 +494,8 @@ def ppo_loss(logp_new, logp_old, adv, returns, values, lengths, clip_eps=0.2, wh
 
 
 # ---------------------------------------------------------------------------
-# Generation with the actor (Alg. 1 and 2: "generate sequence using the policy for T steps";
-# J-Hydra-PPO retains the critic head's values while generating)
+# Generation with the actor (Alg. 1 and 2: the actor samples each sequence for T steps;
+# J-Hydra-PPO keeps the critic head's values while sampling)
 # ---------------------------------------------------------------------------
 
 

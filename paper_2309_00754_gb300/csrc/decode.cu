@@ -1,15 +1,18 @@
-// Kernels of the KV-cached generation loop (Algorithms 1 and 2: "generate sequence using the
-// policy for T steps"; J-Hydra-PPO keeps the critic head's value of every step). The decode
+// Kernels of the KV-cached generation loop (Algorithms 1 and 2: the actor samples each
+// sequence for T steps; J-Hydra-PPO keeps the critic head's value of every step). The decode
 // step runs the R = 2 S stacked rows of the LoRA-off and LoRA-on streams of S sequences; the
 // projections are the dual-output GEMV, the rest is here:
 //   kv_store_prefill   the prompt's rotated keys and its values into the cache
+//   row_norm_lora      (8-CTA clusters) residual add + RMSNorm + the next projection's LoRA
+//                      down-projection
+//   swiglu_lora        (8-CTA clusters) SwiGLU + the down projection's LoRA down-projection
 //   decode_attention   rotary embedding of the new token's q and k, its k and v appended to
 //                      the cache, then one query row per (head, row) against the cached
 //                      positions 0..pos
-//   swiglu_blocked     SwiGLU on gate/up columns interleaved in blocks of 128
 //   sample_tokens      per sequence: log-softmax of both heads, the Gumbel-max draw from the
 //                      actor's logits, both log-probabilities of the drawn token, the value
-// The step counter lives in device memory, so one captured step replays for every position.
+// The step counter lives in device memory: kernels read the position from it rather than
+// from their launch arguments, so every step issues identical launches.
 // Cache layout per layer: K [R][H][Pmax][Dh] then V [R][H][Pmax][Dh], bf16, row i = stream
 // * S + sequence.
 #include <utility>
@@ -194,32 +197,6 @@ __global__ void __launch_bounds__(kAttnThreads)
   }
 }
 
-// gu [R, 2F]: column block 2b holds gate features 128b..128b+127, block 2b+1 the matching up
-// features; m [R, F] = bf16(silu(gate) * up)
-__global__ void swiglu_blocked_kernel(const __nv_bfloat16* __restrict__ gu, long long R, int F,
-                                      __nv_bfloat16* __restrict__ m) {
-  const long long n8 = R * (F / 8);
-  for (long long e = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; e < n8;
-       e += static_cast<long long>(gridDim.x) * blockDim.x) {
-    const long long row = e / (F / 8);
-    const int c = static_cast<int>(e - row * (F / 8)) * 8;  // output feature
-    const int b = c / 128, j = c % 128;
-    const __nv_bfloat16* base = gu + static_cast<size_t>(row) * 2 * F + 256 * b + j;
-    const uint4 g = *reinterpret_cast<const uint4*>(base);
-    const uint4 u = *reinterpret_cast<const uint4*>(base + 128);
-    const uint32_t* gp = &g.x;
-    const uint32_t* up = &u.x;
-    uint4 o;
-    uint32_t* op = &o.x;
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const float2 gf = unpack_bf16x2(gp[k]);
-      const float2 uf = unpack_bf16x2(up[k]);
-      op[k] = pack_bf16x2(gf.x / (1.0f + expf(-gf.x)) * uf.x, gf.y / (1.0f + expf(-gf.y)) * uf.y);
-    }
-    *reinterpret_cast<uint4*>(m + static_cast<size_t>(row) * F + c) = o;
-  }
-}
 
 // ---------------------------------------------------------------- fused row kernels
 // Thread-block clusters of kCl CTAs share one row: each CTA owns a 1/kCl slice of the columns,
@@ -497,11 +474,6 @@ __global__ void __launch_bounds__(kSampleThreads)
 
 __global__ void step_advance_kernel(int* step) { *step += 1; }
 
-int grid_for(long long n, int block) {
-  long long g = (n + block - 1) / block;
-  if (g > 65535LL * 8) g = 65535LL * 8;
-  return static_cast<int>(g < 1 ? 1 : g);
-}
 
 }  // namespace
 
@@ -542,12 +514,6 @@ int launch_decode_attention(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t
   return e == cudaSuccess ? 0 : -3;
 }
 
-int launch_swiglu_blocked(const void* gu, int64_t R, int64_t F, void* m, cudaStream_t st) {
-  if (R == 0) return 0;
-  swiglu_blocked_kernel<<<grid_for(R * (F / 8), 256), 256, 0, st>>>(
-      static_cast<const __nv_bfloat16*>(gu), R, static_cast<int>(F), static_cast<__nv_bfloat16*>(m));
-  return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
-}
 
 int launch_sample_tokens(const float* logits, int64_t S, int64_t V, const float* gumbel,
                          const void* fin, int64_t d, const void* w_rm, const int* step,

@@ -134,7 +134,6 @@ size_t decode_attention_smem(int64_t Pmax);
 int launch_decode_attention(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t H,
                             const void* table, void* ck, void* cv, int64_t P0, const int* step,
                             int64_t Pmax, void* out, int64_t ld_out, cudaStream_t st);
-int launch_swiglu_blocked(const void* gu, int64_t R, int64_t F, void* m, cudaStream_t st);
 int launch_sample_tokens(const float* logits, int64_t S, int64_t V, const float* gumbel,
                          const void* fin, int64_t d, const void* w_rm, const int* step,
                          int64_t n_steps, int32_t* tokens, float* logp_a, float* logp_r,

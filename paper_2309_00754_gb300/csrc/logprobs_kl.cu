@@ -1,6 +1,6 @@
 // Fused vocabulary-wide log-softmax + gather for the actor and reference heads, and the
-// KL-penalised per-token reward (Algorithm 1/2: "turn LoRA off ... to compute reward and
-// reference log probabilities", then use them to calculate the advantages; §2 ratio
+// KL-penalised per-token reward (Algorithms 1 and 2: the LoRA-off model gives the reward and
+// the reference log-probabilities, from which the advantages follow; §2 ratio
 // r(theta) needs the actor's log-probabilities; Appendix B: KL coefficient beta).
 //
 // One CTA per token row streams both heads' logits once with 128-bit loads, keeping a
