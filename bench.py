@@ -605,6 +605,139 @@ class HydraGenerateLlama7B(HydraScoringLlama7B):
         return 2 * len(t_gen) / sum(t_gen), desc
 
 
+class HydraPPOIterationLlama7B(HydraGenerateLlama7B):
+    """One Hydra-PPO iteration's data path (Algorithm 2 without back-propagation) on the
+    random-init Llama-7B: the actor generates 64 tokens after each of 4 prompts of 256
+    (hydra_generate_llama, LoRA-off stream beside it), the drawn sequences go through the
+    three-stream scoring pass with a second LoRA set for the critic (reference log-probs,
+    reward, critic values, KL reward, GAE; hydra_score_llama_hydra), and the PPO losses and
+    their gradients follow, with the generation's log-probs as the old policy and advantage
+    whitening (hydra_ppo_loss). Both passes use the same weights, so the PPO ratio must be 1
+    up to the two paths' numerics: the reported approx_kl and clip fraction check the
+    KV-cached decode against the scoring pass at full size."""
+
+    name = "hydra_ppo_iteration_llama7b"
+    seed = 7
+    default_steps, default_warmup = 3, 3
+    event_names = ("gen", "score", "ppo")
+    metric = ("experience tokens/s (Hydra-PPO iteration without back-propagation: generation, "
+              "three-stream scoring, GAE, PPO losses) on 1 GB300; decode step vs HBM roofline")
+    n_steps = 64
+
+    def __init__(self, device, seed=7, reference=False):
+        super().__init__(device, seed=seed, reference=reference)
+        import torch
+        c = self.cfg
+        c["response_len"] = self.n_steps  # scoring covers exactly the drawn tokens
+        S, n, P0 = self.S, self.n_steps, self.P0
+        self.critic = self.llama.random_device_lora(c, seed + 1000, device)
+        self.ids_buf = torch.empty(S, P0 + n, dtype=torch.int32, device=device)
+        self.ids_buf[:, :P0].copy_(self.prompt)
+        self.lengths = torch.full((S,), n, dtype=torch.int32, device=device)
+        if not reference:
+            H = self.H
+            self.ws = torch.empty(H.generate_llama_workspace_size(c, S), dtype=torch.uint8,
+                                  device=device)
+            self.ws_score = torch.empty(H.score_llama_hydra_workspace_size(c, S),
+                                        dtype=torch.uint8, device=device)
+            self.score_out = self.llama.alloc_outputs(S, n, device)
+            self.grad_logp = torch.empty(S, n, device=device)
+            self.grad_values = torch.empty(S, n, device=device)
+            self.stats = torch.zeros(7, dtype=torch.float64, device=device)
+            self.ws_ppo = torch.empty(H.ppo_workspace_size(), dtype=torch.uint8, device=device)
+        self.units = S * n
+
+    def step(self, ev=None):
+        def rec(k, i):
+            if ev is not None:
+                ev[k][i].record()
+        rec("gen", 0)
+        self._call(self.n_steps)
+        rec("gen", 1)
+        self.ids_buf[:, self.P0:].copy_(self.gen_out["tokens"])
+        rec("score", 0)
+        self.H.hydra_score_llama_hydra(self.cfg, self.weights, self.critic, self.ids_buf,
+                                       self.lengths, self.ws_score, self.score_out)
+        rec("score", 1)
+        rec("ppo", 0)
+        o = self.score_out
+        self.H.hydra_ppo_loss(o["logp_actor"], self.gen_out["logp_actor"], o["advantages"],
+                              o["returns"], o["values"], self.lengths, 0.2, True, self.grad_logp,
+                              self.grad_values, self.stats, self.ws_ppo)
+        rec("ppo", 1)
+
+    def e2e_setup(self):
+        import torch
+        self.prompt_host = self.prompt.cpu().pin_memory()
+        self.gumbel_host = self.gumbel.cpu().pin_memory()
+        self.stats_host = torch.empty(7, dtype=torch.float64, pin_memory=True)
+        self.tokens_host = torch.empty(self.S, self.n_steps, dtype=torch.int32, pin_memory=True)
+        self.h2d = self.prompt_host.numel() * 4 + self.gumbel_host.numel() * 4
+        self.d2h = self.stats_host.numel() * 8 + self.tokens_host.numel() * 4
+
+    def e2e_step(self):
+        self.prompt.copy_(self.prompt_host, non_blocking=True)
+        self.ids_buf[:, :self.P0].copy_(self.prompt)
+        self.gumbel.copy_(self.gumbel_host, non_blocking=True)
+        self.step()
+        self.stats_host.copy_(self.stats, non_blocking=True)
+        self.tokens_host.copy_(self.gen_out["tokens"], non_blocking=True)
+
+    def kernels(self, peaks, ms):
+        import torch
+        out = super().kernels(peaks, {"gen": ms["gen"]})
+        out["scoring_hydra_ppo"] = {"ms": ms["score"]}
+        out["ppo_loss"] = {"ms": ms["ppo"]}
+        st = self.stats.cpu().tolist()
+        out["ppo_stats_of_last_iteration"] = dict(zip(self.H.PPO_STATS, st))
+        # decode path against the scoring pass on the same tokens and weights
+        d = (self.score_out["logp_actor"] - self.gen_out["logp_actor"]).abs()
+        dr = (self.score_out["logp_ref"] - self.gen_out["logp_ref"]).abs()
+        out["decode_vs_scoring_max_abs_dlogp"] = {"actor": float(d.max()), "ref": float(dr.max())}
+        # launches of the scoring pass, counted by the library's launch timing
+        self.H.profile_enable(True)
+        self.H.hydra_score_llama_hydra(self.cfg, self.weights, self.critic, self.ids_buf,
+                                       self.lengths, self.ws_score, self.score_out)
+        torch.cuda.synchronize()
+        n_score = sum(n for _, n in self.H.profile_collect(reset=True).values())
+        self.H.profile_enable(False)
+        self.launches_per_step += n_score + 4  # + the PPO moments, coef, loss, finalize
+        return out
+
+    def config(self):
+        return {"workload": "hydra_ppo_iteration_llama7b: random-init Llama-7B (32 layers, d 4096, 32 "
+                            "heads, SwiGLU 11008, vocab 32000, bf16), actor and critic LoRA sets r=16 "
+                            f"s=2; 4 sequences x 256 prompt tokens, {self.n_steps} Gumbel-max draws, "
+                            "three-stream scoring (reference, actor, critic), KL reward beta 0.1, GAE "
+                            "gamma 1 lambda 0.95, PPO losses clip 0.2 with whitening",
+                "batch": self.S, "prompt_len": self.P0, "draws": self.n_steps,
+                "experience_tokens_per_step": self.units,
+                "l2": "inputs larger than L2 (13.5 GB of weights read per decode step)"}
+
+    def oracle_time(self, smp, n_layers):
+        import oracle as O
+        t0 = time.perf_counter()
+        gen = O.llama_generate(smp["w"], smp["ids"][:smp["prompt"]], 2, smp["cfg"], n_layers=n_layers)
+        seq = np.concatenate([smp["ids"][:smp["prompt"]], gen["tokens"]])
+        sc = O.llama_score_hydra(smp["w"], smp["w"]["lora"], seq, smp["prompt"], smp["cfg"],
+                                 n_layers=n_layers, beta=self.beta, gamma=self.gamma, lam=self.lam)
+        O.ppo_loss(sc["logp_actor"][None], gen["logp_actor"][None], sc["advantages"][None],
+                   sc["returns"][None], sc["values"][None], [2], whiten=True)
+        return time.perf_counter() - t0
+
+    def oracle_throughput(self, steps=1):
+        smp = self.oracle_sample(1)
+        t_head = self.oracle_time(smp, 0)
+        t1 = [self.oracle_time(smp, 1) for _ in range(steps)]
+        n = self.cfg["n_layers"]
+        t_it = [t_head + n * max(t - t_head, 0.0) for t in t1]
+        desc = (f"one sequence, {smp['prompt']} prompt tokens, 2 draws, three-stream scoring of the "
+                f"result and the PPO losses at full width through the fp64 oracle: embed + heads "
+                f"{t_head:.2f} s, one decoder layer {statistics.mean(t1) - t_head:.2f} s, time "
+                f"extrapolated to {n} layers")
+        return 2 * len(t_it) / sum(t_it), desc
+
+
 class KernelSweep:
     """Per-kernel measurements of the rows the full pass does not exercise at their own
     shapes (one JSON line; value = the sweep's mean fraction of roofline):
@@ -763,6 +896,7 @@ class KernelSweep:
 WORKLOADS = {LmHeadScoring.name: LmHeadScoring, HydraScoringLlama7B.name: HydraScoringLlama7B,
              HydraPPOScoringLlama7B.name: HydraPPOScoringLlama7B,
              HydraGenerateLlama7B.name: HydraGenerateLlama7B,
+             HydraPPOIterationLlama7B.name: HydraPPOIterationLlama7B,
              KernelSweep.name: KernelSweep}
 DEFAULT_WORKLOAD = HydraScoringLlama7B.name
 
