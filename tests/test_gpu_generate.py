@@ -175,3 +175,59 @@ def test_generate_argument_errors():
         H.hydra_generate_llama(cfg, w, dev_i32(np.zeros((3, cfg["prompt_len"]), np.int32)), 4,
                                None, ws, out)
     assert H.generate_llama_workspace_size(cfg, 9) == 0
+
+
+def test_generate_llama7b_full_size_agrees_with_scoring_pass():
+    """The benchmark's shape: random-init Llama-7B (32 layers), 4 sequences of 256 prompt
+    tokens, 16 draws. Properties at full size:
+    - two runs give the same tokens and the same bits;
+    - the GPU scoring pass of the same finished sequences, a different path (tcgen05 GEMMs,
+      flash attention with bf16 probabilities, full-sequence norms), agrees with the decode
+      path's log-probabilities and values.
+
+    The two paths round at the same bf16 storage points but accumulate in different orders.
+    One-ulp flips in a small share of each layer's stored values then compound over 32
+    layers; at one full-width layer the oracle's own dither spread is 1.9e-2 in log-prob.
+    Measured: mean |d logp| 0.04, max 0.16. The bounds allow that drift with room to spare
+    and still catch real faults, which show up as O(1) differences or NaN:
+    - mean |d logp| <= 0.1;
+    - max |d logp| <= 0.5;
+    - every PPO ratio exp(d logp) of the first epoch inside [0.5, 2]."""
+    cfg = dict(llama.LLAMA7B, response_len=16)
+    w = llama.random_device_weights(cfg, 8, "cuda")
+    S, n, P0 = 4, 16, cfg["prompt_len"]
+    prompt = torch.from_numpy(synth.randint(8001, (S, P0), 0, cfg["vocab"])).cuda()
+    g = torch.Generator(device="cuda").manual_seed(8002)
+    u = torch.rand(n, S, cfg["vocab"], device="cuda", generator=g).clamp_(1e-12, 1 - 1e-7)
+    noise = -torch.log(-torch.log(u))
+    ws = torch.empty(H.generate_llama_workspace_size(cfg, S), dtype=torch.uint8, device="cuda")
+
+    def gen():
+        out = {"tokens": torch.empty((S, n), dtype=torch.int32, device="cuda"),
+               "score": torch.empty(S, device="cuda")}
+        for k in ("logp_actor", "logp_ref", "values"):
+            out[k] = torch.empty((S, n), device="cuda")
+        H.hydra_generate_llama(cfg, w, prompt, n, noise, ws, out)
+        torch.cuda.synchronize()
+        return out
+
+    a, b = gen(), gen()
+    assert H.device_error(clear=True) == 0
+    for k in a:
+        assert torch.equal(a[k], b[k]), k
+    assert torch.isfinite(a["logp_actor"]).all() and torch.isfinite(a["values"]).all()
+    ids = torch.cat([prompt, a["tokens"]], dim=1).contiguous()
+    ws2 = torch.empty(H.score_llama_workspace_size(cfg, S), dtype=torch.uint8, device="cuda")
+    sc = llama.alloc_outputs(S, n, "cuda")
+    H.hydra_score_llama(cfg, w, ids, None, ws2, sc)
+    torch.cuda.synchronize()
+    for k in ("logp_actor", "logp_ref"):
+        dl = (sc[k] - a[k]).abs()
+        print(f"{k}: mean |d| {dl.mean().item():.3e}, max {dl.max().item():.3e}")
+        assert dl.mean().item() <= 0.1 and dl.max().item() <= 0.5, k
+    ratio = torch.exp(sc["logp_actor"] - a["logp_actor"])
+    assert ((ratio >= 0.5) & (ratio <= 2.0)).all()
+    dv = (sc["values"] - a["values"]).abs()
+    assert dv.max().item() <= 0.5 * max(1.0, a["values"].abs().max().item())
+    del w, ws, ws2
+    torch.cuda.empty_cache()
