@@ -271,6 +271,66 @@ __global__ void __launch_bounds__(kPpoThreads, 3)
   pdl_launch_dependents();
 }
 
+// Pass 1, float4 rows (L % 4 == 0, aligned): one warp per row, two rows in flight per warp;
+// lane l loads tokens [4 l + 128 k, + 4) of a row's valid prefix, k < 4 at a time, and the
+// next pair's lengths are fetched before the current pair is added. A row's tokens past its
+// length are never read.
+__global__ void __launch_bounds__(kPpoThreads)
+    ppo_moments_rows_kernel(const float* __restrict__ adv, const int32_t* __restrict__ lengths,
+                            int S, int L, MomPart* __restrict__ part, int* err) {
+  __shared__ float sh[2][kPpoWarps];
+  __shared__ int shk[kPpoWarps];
+  pdl_wait();
+  const int lane = threadIdx.x & 31;
+  const int gw = blockIdx.x * kPpoWarps + (threadIdx.x >> 5);
+  const int nw = gridDim.x * kPpoWarps;
+  const float c = S > 0 ? __ldg(adv) : 0.f;
+  int n = 0;
+  Kahan s1, s2;
+  auto len_of = [&](int s) { return s < S ? (lengths ? __ldg(lengths + s) : L) : 0; };
+  int nlA = len_of(gw), nlB = len_of(gw + nw);
+  for (int s0 = gw; s0 < S; s0 += 2 * nw) {
+    const int sA = s0, sB = s0 + nw;
+    const int lenA = clamp_length(nlA, L, lane == 0 ? err : nullptr);
+    const int lenB = sB < S ? clamp_length(nlB, L, lane == 0 ? err : nullptr) : 0;
+    nlA = len_of(s0 + 2 * nw);
+    nlB = len_of(s0 + 3 * nw);
+    const float* ra = adv + static_cast<size_t>(sA) * L;
+    const float* rb = adv + static_cast<size_t>(sB < S ? sB : sA) * L;
+    const int lmax = max(lenA, lenB);
+    for (int base = 0; base < lmax; base += 512) {
+      float va[4][4], vb[4][4];
+      int ka[4], kb[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int t0 = base + 128 * k + 4 * lane;
+        ka[k] = min(max(lenA - t0, 0), 4);
+        kb[k] = min(max(lenB - t0, 0), 4);
+        if (ka[k] > 0) get_keep<4>(ra + t0, va[k]);
+        if (kb[k] > 0) get_keep<4>(rb + t0, vb[k]);
+      }
+      float b1 = 0.f, b2 = 0.f;
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const float da = j < ka[k] ? va[k][j] - c : 0.f;
+          const float db = j < kb[k] ? vb[k][j] - c : 0.f;
+          b1 += da + db;
+          b2 += da * da + db * db;
+        }
+#pragma unroll
+      for (int k = 0; k < 4; ++k) n += ka[k] + kb[k];
+      s1.add(b1);
+      s2.add(b2);
+    }
+  }
+  float v[2] = {s1.s, s2.s};
+  block_sums<2>(v, n, sh, shk);
+  if (threadIdx.x == 0) part[blockIdx.x] = MomPart{n, v[0], v[1], 0.f};
+  pdl_launch_dependents();
+}
+
 // Merge the moments partials (or take the caller's fp64 [n, mean, M2]) into the fp64
 // moments and the fp32 coefficients (mean, 1 / sqrt(var + 1e-8), 1 / n) of the loss pass.
 // Every thread loads its few partials at once (compensated fp32), then a fixed block tree.
@@ -565,11 +625,16 @@ int launch_moments_coef(const float* adv, const int32_t* lengths, int S, int L, 
   if (ext == nullptr) {
     const bool v4 = vec4_ok(L, {adv});
     cudaError_t e;
-    if (v4) {
-      G = one_wave(ppo_moments_kernel<4>, with_adv ? static_cast<long long>(S) * (L / 4) : S,
+    if (v4 && with_adv) {
+      // a warp per row pair: S / 2 warps of work
+      G = one_wave(ppo_moments_rows_kernel, (static_cast<long long>(S) + 1) / 2 * 32,
                    kPpoMaxMomentBlocks);
+      e = launch_pdl(ppo_moments_rows_kernel, dim3(G), dim3(kPpoThreads), 0, st, adv, lengths, S,
+                     L, w.mom, err);
+    } else if (v4) {
+      G = one_wave(ppo_moments_kernel<4>, S, kPpoMaxMomentBlocks);
       e = launch_pdl(ppo_moments_kernel<4>, dim3(G), dim3(kPpoThreads), 0, st, adv, lengths, S,
-                     L, with_adv ? 1 : 0, w.mom, err);
+                     L, 0, w.mom, err);
     } else {
       G = one_wave(ppo_moments_kernel<1>, with_adv ? static_cast<long long>(S) * L : S,
                    kPpoMaxMomentBlocks);
