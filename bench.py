@@ -259,7 +259,7 @@ class HydraScoringLlama7B:
         self.llama = llama
         self.cfg = dict(llama.LLAMA7B)
         c = self.cfg
-        self.S, self.P0, self.L = 4, c["prompt_len"], c["response_len"]
+        self.S, self.P0, self.L = getattr(self, "batch", 4), c["prompt_len"], c["response_len"]
         self.beta, self.gamma, self.lam = c["beta"], c["gamma"], c["lam"]
         P = self.P0 + self.L
         self.weights = llama.random_device_weights(c, seed, device)
@@ -471,6 +471,7 @@ class HydraGenerateLlama7B(HydraScoringLlama7B):
     metric = ("generated tokens/s (actor draws with logp_actor, logp_ref, values; both streams "
               "decoded) on 1 GB300; decode step vs HBM roofline")
     n_steps = 64
+    batch = 4
 
     def __init__(self, device, seed=6, reference=False):
         super().__init__(device, seed=seed, reference=reference)
@@ -568,8 +569,9 @@ class HydraGenerateLlama7B(HydraScoringLlama7B):
             step_ms, _ = self._decode_step_ms()
         achieved = self.step_bytes / step_ms / 1e6
         peak = peaks["hbm_gbs"]
-        return {"kernel": "decode step (dual-output GEMV for every projection and the LM head, "
-                          "decode attention over the cache, elementwise): 8 rows",
+        return {"kernel": "decode step (dual-output GEMV, or the tcgen05 GEMM above 16 rows, for every "
+                          f"projection and the LM head; decode attention over the cache; fused norms): "
+                          f"{2 * self.S} rows",
                 "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak, "traffic": None,
                 "peak_kind": f"HBM copy, {peaks['source']}",
@@ -577,7 +579,7 @@ class HydraGenerateLlama7B(HydraScoringLlama7B):
 
     def config(self):
         return {"workload": "hydra_generate_llama7b: random-init Llama-7B (32 layers, d 4096, 32 heads, "
-                            "SwiGLU 11008, vocab 32000, bf16), LoRA r=16 s=2 on q/v/gate/up/down; 4 "
+                            f"SwiGLU 11008, vocab 32000, bf16), LoRA r=16 s=2 on q/v/gate/up/down; {self.S} "
                             f"sequences x 256 prompt tokens, {self.n_steps} Gumbel-max draws each; LoRA-off stream "
                             "decoded beside the actor; values and final score",
                 "batch": self.S, "prompt_len": self.P0, "draws": self.n_steps,
@@ -965,6 +967,8 @@ def time_oracle(wl, target_s=12.0):
 def run_reference(args, wl_cls):
     if getattr(args, "gen_steps", None) and hasattr(wl_cls, "n_steps"):
         wl_cls.n_steps = args.gen_steps
+    if getattr(args, "gen_batch", None) and hasattr(wl_cls, "n_steps"):
+        wl_cls.batch = args.gen_batch
     rank, world, local = dist_env()
     if rank != 0:
         return 0
@@ -1034,6 +1038,8 @@ def run_ours(args, wl_cls):
     import torch
     if getattr(args, "gen_steps", None) and hasattr(wl_cls, "n_steps"):
         wl_cls.n_steps = args.gen_steps
+    if getattr(args, "gen_batch", None) and hasattr(wl_cls, "n_steps"):
+        wl_cls.batch = args.gen_batch
     rank, world, local = dist_env()
     if world > 1:
         import torch.distributed as dist
@@ -1144,7 +1150,9 @@ def main(argv=None):
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default=DEFAULT_WORKLOAD)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--gen-steps", type=int, default=None,
-                    help="hydra_generate_llama7b only: draws per call (default 64)")
+                    help="generation workloads only: draws per call (default 64)")
+    ap.add_argument("--gen-batch", type=int, default=None,
+                    help="generation workloads only: sequences per call (default 4, at most 64)")
     ap.add_argument("--parts", default=None,
                     help="kernel_sweep only: comma-separated subset of " + ",".join(KernelSweep.PARTS))
     args = ap.parse_args(argv)

@@ -466,7 +466,7 @@ typedef struct hydra_llama_lora {
 } hydra_llama_lora;
 
 /* Workspace bytes of hydra_generate_llama for S sequences (0 for an unsupported
- * configuration or S outside 1..8). */
+ * configuration or S outside 1..64). */
 size_t hydra_generate_llama_workspace_size(const hydra_llama_config* cfg, int64_t S);
 
 /*
@@ -489,7 +489,7 @@ size_t hydra_generate_llama_workspace_size(const hydra_llama_config* cfg, int64_
  * sequence (prompt + tokens). Weights as hydra_score_llama (fused layouts).
  * prompt_ids int32 [S, P0]; gumbel fp32 [n_steps, S, V] or NULL; outputs int32 / fp32
  * [S, n_steps] and fp32 [S]; all device. Requirements: as hydra_score_llama, plus
- * 1 <= S <= 8, 1 <= n_steps <= cfg->response_len (the cache holds P0 + response_len
+ * 1 <= S <= 64, 1 <= n_steps <= cfg->response_len (the cache holds P0 + response_len
  * positions; its scores fit shared memory for P0 + response_len up to about 50,000).
  * workspace: device, 16-byte aligned, >= hydra_generate_llama_workspace_size(cfg, S).
  * Errors: NULL pointer -> HYDRA_ERR_NULL; configuration or sizes outside the above ->

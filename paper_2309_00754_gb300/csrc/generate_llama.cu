@@ -24,7 +24,10 @@ inline bool a16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) =
 inline size_t up256(size_t v) { return (v + 255) / 256 * 256; }
 inline hydra_status rc(int r) { return r == 0 ? HYDRA_OK : HYDRA_ERR_CUDA; }
 
-constexpr int64_t kMaxGenSeqs = hydra::kGemvMaxRows / 2;  // both streams' rows in one GEMV
+// Up to 8 sequences both streams' rows fit one dual GEMV (16 rows); larger batches (up to 64
+// sequences, 128 rows per stream-pair tile) run the decode projections on the tcgen05 GEMM,
+// which also reads each W tile once.
+constexpr int64_t kMaxGenSeqs = 64;
 
 struct GenLayout {
   size_t h, a, qkv, attn, m, u;                                       // prefill, 2 S P0 rows
@@ -79,8 +82,8 @@ bool gen_config_ok(const hydra_llama_config* c) {
 }
 
 // y = [x_off; x_on] W^T (+ u B^T on the on rows; u [S, r] = s x_on A^T, already computed by
-// the fused row kernel that produced x) for S rows per stream, through the dual-output GEMV;
-// y [2 S, N] bf16 or fp32 (off rows first).
+// the fused row kernel that produced x) for S rows per stream: the dual-output GEMV for up to
+// 16 rows, the tcgen05 GEMM beyond; y [2 S, N] bf16 or fp32 (off rows first).
 int gemv_linear(const void* x, int64_t S, int64_t K, int64_t N, const void* W, const void* B,
                 int64_t r, const void* u, void* y, bool f32, int* err, cudaStream_t st) {
   hydra::GemmArgs g;
@@ -98,7 +101,8 @@ int gemv_linear(const void* x, int64_t S, int64_t K, int64_t N, const void* W, c
   g.y_on = static_cast<uint8_t*>(y) + static_cast<size_t>(S) * N * (f32 ? 4 : 2);
   g.out_f32 = f32 ? 1 : 0;
   g.err = err;
-  return hydra::launch_dual_lora_gemv(g, st);
+  return 2 * S <= hydra::kGemvMaxRows ? hydra::launch_dual_lora_gemv(g, st)
+                                       : hydra::launch_dual_lora_gemm_tc(g, st);
 }
 
 }  // namespace

@@ -120,6 +120,18 @@ def test_generate_eight_sequences_one_prompt_token():
     check_generation(cfg, got, w64, prompt, noise)
 
 
+@pytest.mark.parametrize("S", [12, 64])
+def test_generate_large_batches_use_the_tcgen05_gemm(S):
+    """More than 8 sequences: both streams' rows no longer fit one dual GEMV (16 rows), so the
+    decode projections run on the tcgen05 GEMM; 64 sequences (128 rows) is the limit."""
+    cfg = dict(SMALL, prompt_len=6, response_len=5)
+    sep, w64 = make_model(cfg, 78)
+    prompt = synth.randint(781 + S, (S, 6), 0, cfg["vocab"])
+    noise = gumbel_noise(782 + S, 5, S, cfg["vocab"])
+    got = run_generate(cfg, sep, prompt, 5, noise)
+    check_generation(cfg, got, w64, prompt, noise)
+
+
 def test_generate_lora_off_streams_agree_bitwise():
     cfg = dict(SMALL)
     sep, _ = make_model(cfg, 74, zero_B=True)
@@ -174,7 +186,7 @@ def test_generate_argument_errors():
     with pytest.raises(H.HydraError):  # workspace for fewer sequences
         H.hydra_generate_llama(cfg, w, dev_i32(np.zeros((3, cfg["prompt_len"]), np.int32)), 4,
                                None, ws, out)
-    assert H.generate_llama_workspace_size(cfg, 9) == 0
+    assert H.generate_llama_workspace_size(cfg, 65) == 0
 
 
 def test_generate_llama7b_full_size_agrees_with_scoring_pass():
