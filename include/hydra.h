@@ -121,6 +121,34 @@ hydra_status hydra_dual_linear(const void* x_off, const void* x_on, int64_t M, i
                                void* y_off, void* y_on, int out_dtype, int algo, void* stream);
 
 /*
+ * The decode-step form of hydra_dual_linear (§3 Dynamic LoRA: one frozen W serves both
+ * streams): the two streams' token rows stacked in one matrix x = [x_off; x_on], at most
+ * 128 rows, and
+ *     y[i] = x[i] W^T                          for every row i in [0, M)
+ *     y[i] = x[i] W^T + u[i - u_row0] B^T      for i in [u_row0, u_row0 + u_rows)
+ * on a tcgen05 kernel that splits K over a thread-block cluster, so that a weight read
+ * once, by only a few output tiles, still streams through most of the device's SMs.
+ *   x : bf16 [M, K], 0 <= M <= 128 (M == 0 is a no-op).   W : bf16 [N, K].
+ *   y : [M, N] of out_dtype (HYDRA_BF16: the fp32 sum rounded once; HYDRA_F32).
+ *   u : bf16 [u_rows, r] (s x_on A^T, as hydra_lora_down writes it); B : bf16 [N, r].
+ *       r == 0 means no LoRA (u, B, u_row0, u_rows ignored); otherwise 8 <= r <= 256,
+ *       r % 8 == 0, u_rows >= 1, u_row0 >= 0 and u_row0 + u_rows <= M.
+ *   tile_n  : output tile width, a multiple of 16 up to 256; 0 = chosen by the library.
+ *   split_k : CTAs of a cluster splitting K, 1..8 and at most ceil(K / 64); 0 = chosen.
+ *       The partial sums are added in a fixed order, so a given (tile_n, split_k) gives
+ *       the same bits on every call; different choices associate the fp32 sums
+ *       differently.
+ * Requirements: K % 8 == 0, N % 16 == 0, all pointers 16-byte aligned, K, N < 2^31.
+ * Errors: HYDRA_ERR_NULL (x, W or y NULL; u or B NULL with r > 0), HYDRA_ERR_SHAPE (M, N,
+ * r, u_row0 or u_rows out of range), HYDRA_ERR_ALIGN (misaligned pointer, K % 8 != 0,
+ * r % 8 != 0), HYDRA_ERR_RANGE (out_dtype, tile_n or split_k), HYDRA_ERR_CUDA (launch).
+ */
+hydra_status hydra_skinny_linear(const void* x, int64_t M, int64_t K, int64_t N, const void* W,
+                                 const void* u, int64_t u_row0, int64_t u_rows, const void* B,
+                                 int64_t r, void* y, int out_dtype, int tile_n, int split_k,
+                                 void* stream);
+
+/*
  * Hydra-PPO's three streams through one frozen weight (Algorithm 2: the critic LoRA gives
  * the values, LoRA off the reward and reference log-probabilities, the actor LoRA the policy;
  * §3 Stage 2: two LoRA sets on one base model):

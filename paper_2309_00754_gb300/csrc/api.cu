@@ -200,6 +200,48 @@ hydra_status hydra_dual_linear(const void* x_off, const void* x_on, int64_t M, i
                           stream, true);
 }
 
+hydra_status hydra_skinny_linear(const void* x, int64_t M, int64_t K, int64_t N, const void* W,
+                                 const void* u, int64_t u_row0, int64_t u_rows, const void* B,
+                                 int64_t r, void* y, int out_dtype, int tile_n, int split_k,
+                                 void* stream) {
+  if (x == nullptr || W == nullptr || y == nullptr) return HYDRA_ERR_NULL;
+  if (out_dtype != HYDRA_BF16 && out_dtype != HYDRA_F32) return HYDRA_ERR_RANGE;
+  if (M < 0 || M > 128 || K < 8 || N < 16 || K >= (1LL << 31) || N >= (1LL << 31) || N % 16 != 0)
+    return HYDRA_ERR_SHAPE;
+  if (K % 8 != 0) return HYDRA_ERR_ALIGN;
+  if (r < 0 || r > 256) return HYDRA_ERR_SHAPE;
+  if (r > 0) {
+    if (u == nullptr || B == nullptr) return HYDRA_ERR_NULL;
+    if (r % 8 != 0) return HYDRA_ERR_ALIGN;
+    if (u_rows < 1 || u_row0 < 0 || u_row0 + u_rows > M) return HYDRA_ERR_SHAPE;
+    if (!aligned16(u) || !aligned16(B)) return HYDRA_ERR_ALIGN;
+  }
+  if (!aligned16(x) || !aligned16(W) || !aligned16(y)) return HYDRA_ERR_ALIGN;
+  if (tile_n < 0 || tile_n > 256 || tile_n % 16 != 0) return HYDRA_ERR_RANGE;
+  if (split_k < 0 || split_k > 8 || split_k > (K + 63) / 64) return HYDRA_ERR_RANGE;
+  if (M == 0) return HYDRA_OK;
+  int* err = hydra::device_error_word();
+  if (err == nullptr) return HYDRA_ERR_CUDA;
+  hydra::SkinnyArgs a;
+  a.x = x;
+  a.M = M;
+  a.K = K;
+  a.N = N;
+  a.W = W;
+  a.u = r > 0 ? u : nullptr;
+  a.u_row0 = r > 0 ? u_row0 : 0;
+  a.u_rows = r > 0 ? u_rows : 0;
+  a.B = r > 0 ? B : nullptr;
+  a.r = r;
+  a.y = y;
+  a.out_f32 = out_dtype == HYDRA_F32 ? 1 : 0;
+  a.bn = tile_n;
+  a.ks = split_k;
+  a.err = err;
+  return hydra::launch_skinny_gemm_tc(a, static_cast<cudaStream_t>(stream)) == 0 ? HYDRA_OK
+                                                                                : HYDRA_ERR_CUDA;
+}
+
 hydra_status hydra_dual_linear_ex(const void* x_off, const void* x_on, int64_t M, int64_t K,
                                   int64_t N, const void* W, const void* u, const void* B,
                                   int64_t r, void* y_off, void* y_on, int out_dtype, int epilogue,

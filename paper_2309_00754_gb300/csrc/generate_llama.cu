@@ -83,9 +83,29 @@ bool gen_config_ok(const hydra_llama_config* c) {
 
 // y = [x_off; x_on] W^T (+ u B^T on the on rows; u [S, r] = s x_on A^T, already computed by
 // the fused row kernel that produced x) for S rows per stream: the dual-output GEMV for up to
-// 16 rows, the tcgen05 GEMM beyond; y [2 S, N] bf16 or fp32 (off rows first).
-int gemv_linear(const void* x, int64_t S, int64_t K, int64_t N, const void* W, const void* B,
-                int64_t r, const void* u, void* y, bool f32, int* err, cudaStream_t st) {
+// 16 rows, beyond that the split-K tcgen05 kernel over both streams' rows in one tile (the
+// CTA-tile GEMM when N is not a multiple of 16); y [2 S, N] bf16 or fp32 (off rows first).
+int decode_linear(const void* x, int64_t S, int64_t K, int64_t N, const void* W, const void* B,
+                  int64_t r, const void* u, void* y, bool f32, int* err, cudaStream_t st) {
+  if (2 * S > hydra::kGemvMaxRows && hydra::skinny_gemm_supported(2 * S, K, N, r)) {
+    hydra::SkinnyArgs a;
+    a.x = x;
+    a.M = 2 * S;
+    a.K = K;
+    a.N = N;
+    a.W = W;
+    a.u = r > 0 ? u : nullptr;
+    a.u_row0 = r > 0 ? S : 0;
+    a.u_rows = r > 0 ? S : 0;
+    a.B = r > 0 ? B : nullptr;
+    a.r = r;
+    a.y = y;
+    a.out_f32 = f32 ? 1 : 0;
+    a.bn = 0;
+    a.ks = 0;
+    a.err = err;
+    return hydra::launch_skinny_gemm_tc(a, st);
+  }
   hydra::GemmArgs g;
   g.x_off = x;
   g.x_on = static_cast<const uint8_t*>(x) + static_cast<size_t>(S) * K * 2;
@@ -219,19 +239,19 @@ hydra_status hydra_generate_llama(const hydra_llama_config* cfg, const hydra_lla
       if ((x = hydra::launch_row_norm_lora(hd, resid, ly.norm_attn, R, d, c.rms_eps, ad, S, ly.a_qv,
                                            2 * r, s, ud, st)) != 0)
         break;
-      if ((x = gemv_linear(ad, S, d, 3 * d, ly.w_qkv, ly.b_qkv, 2 * r, ud, qkvd, false, err, st)) != 0)
+      if ((x = decode_linear(ad, S, d, 3 * d, ly.w_qkv, ly.b_qkv, 2 * r, ud, qkvd, false, err, st)) != 0)
         break;
       if ((x = hydra::launch_decode_attention(qkvd, R, 3 * d, d, H, rope_table, kcache(l),
                                               vcache(l), P0, step, Pmax, attnd, d, st)) != 0)
         break;
-      if ((x = gemv_linear(attnd, S, d, d, ly.w_o, nullptr, 0, ud, yd, false, err, st)) != 0) break;
+      if ((x = decode_linear(attnd, S, d, d, ly.w_o, nullptr, 0, ud, yd, false, err, st)) != 0) break;
       if ((x = hydra::launch_row_norm_lora(hd, yd, ly.norm_ffn, R, d, c.rms_eps, ad, S, ly.a_gu,
                                            2 * r, s, ud, st)) != 0)
         break;
-      if ((x = gemv_linear(ad, S, d, 2 * F, ly.w_gu, ly.b_gu, 2 * r, ud, gud, false, err, st)) != 0)
+      if ((x = decode_linear(ad, S, d, 2 * F, ly.w_gu, ly.b_gu, 2 * r, ud, gud, false, err, st)) != 0)
         break;
       if ((x = hydra::launch_swiglu_lora(gud, R, F, md, S, ly.a_down, r, s, ud, st)) != 0) break;
-      if ((x = gemv_linear(md, S, F, d, ly.w_down, ly.b_down, r, ud, yd, false, err, st)) != 0) break;
+      if ((x = decode_linear(md, S, F, d, ly.w_down, ly.b_down, r, ud, yd, false, err, st)) != 0) break;
       resid = yd;
     }
     if (x == 0)
@@ -241,7 +261,7 @@ hydra_status hydra_generate_llama(const hydra_llama_config* cfg, const hydra_lla
   };
   // the LM head on both streams' final rows and the draw of step *step
   auto draw = [&]() -> int {
-    int x = gemv_linear(find, S, d, V, w->lm_head, nullptr, 0, nullptr, logits, true, err, st);
+    int x = decode_linear(find, S, d, V, w->lm_head, nullptr, 0, nullptr, logits, true, err, st);
     if (x == 0)
       x = hydra::launch_sample_tokens(logits, S, V, gumbel, find, d, w->w_rm, step, n_steps, tokens,
                                       logp_actor, logp_ref, values, cur, st);

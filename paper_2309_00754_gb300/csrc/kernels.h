@@ -76,6 +76,25 @@ int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream);
 bool make_tma_map(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int64_t ld,
                   int box_rows, bool f32);
 int launch_dual_lora_gemv(const GemmArgs& a, cudaStream_t stream);
+
+// Skinny linear (gemm_skinny.cu): y = x W^T for all M <= 128 rows of x, plus u B^T on rows
+// [u_row0, u_row0 + u_rows) (u [u_rows, r]). K is split over a cluster of ks CTAs; bn / ks
+// of 0 pick them by the kernel's cost model. Needs K % 8 == 0, N % 16 == 0, r % 8 == 0.
+struct SkinnyArgs {
+  const void* x;  // bf16 [M, K]
+  int64_t M, K, N;
+  const void* W;  // bf16 [N, K]
+  const void* u;  // bf16 [u_rows, r] (NULL when r == 0)
+  int64_t u_row0, u_rows;
+  const void* B;  // bf16 [N, r]
+  int64_t r;
+  void* y;        // [M, N], bf16 or fp32 (out_f32)
+  int out_f32;
+  int bn, ks;     // 0 = chosen by the cost model
+  int* err;
+};
+bool skinny_gemm_supported(int64_t M, int64_t K, int64_t N, int64_t r);
+int launch_skinny_gemm_tc(const SkinnyArgs& a, cudaStream_t stream);
 int launch_lora_down(const void* x, int64_t M, int64_t K, const void* A, int64_t r, float s,
                      void* u, cudaStream_t stream);
 // ids of sequence s start at ids + s * ids_ld (ids_ld = L for a dense [S, L] array)

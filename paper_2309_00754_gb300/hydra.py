@@ -32,6 +32,9 @@ _SIGNATURES = {
     "hydra_lora_linear_algo": (ctypes.c_int, [_vp, _vp, _c_i64, _c_i64, _c_i64, _vp, _vp, _vp,
                                               _c_i64, ctypes.c_float, _vp, _vp, ctypes.c_int, _vp,
                                               ctypes.c_size_t, ctypes.c_int, _vp]),
+    "hydra_skinny_linear": (ctypes.c_int, [_vp, _c_i64, _c_i64, _c_i64, _vp, _vp, _c_i64, _c_i64,
+                                           _vp, _c_i64, _vp, ctypes.c_int, ctypes.c_int,
+                                           ctypes.c_int, _vp]),
     "hydra_dual_linear": (ctypes.c_int, [_vp, _vp, _c_i64, _c_i64, _c_i64, _vp, _vp, _vp, _c_i64,
                                          _vp, _vp, ctypes.c_int, ctypes.c_int, _vp]),
     "hydra_dual_linear_ex": (ctypes.c_int, [_vp, _vp, _c_i64, _c_i64, _c_i64, _vp, _vp, _vp,
@@ -239,6 +242,23 @@ def hydra_dual_linear(x_off, x_on, W, u, B, y_off, y_on, algo=0, stream=None):
     _check("hydra_dual_linear", load().hydra_dual_linear(
         _p(x_off), _p(x_on), M, K, N, _p(W), _p(u), _p(B), r, _p(y_off), _p(y_on), out_dtype,
         int(algo), _stream(stream)))
+
+
+def hydra_skinny_linear(x, W, y, u=None, B=None, u_row0=0, tile_n=0, split_k=0, stream=None):
+    """Decode-step linear over both streams' rows stacked in x (at most 128): y = x W^T, plus
+    u B^T on rows [u_row0, u_row0 + len(u)) (u None: no LoRA). tile_n / split_k 0: chosen by
+    the library."""
+    for t, n in ((x, "x"), (W, "W"), (u, "u"), (B, "B")):
+        _req(t, torch.bfloat16, n)
+    out_dtype = HYDRA_F32 if y.dtype == torch.float32 else HYDRA_BF16
+    _req(y, y.dtype, "y")
+    M, K = x.shape
+    N = W.shape[0]
+    r = 0 if u is None else u.shape[1]
+    u_rows = 0 if u is None else u.shape[0]
+    _check("hydra_skinny_linear", load().hydra_skinny_linear(
+        _p(x), M, K, N, _p(W), _p(u), int(u_row0), u_rows, _p(B), r, _p(y), out_dtype,
+        int(tile_n), int(split_k), _stream(stream)))
 
 
 def hydra_lora_linear_noalloc(x_off, x_on, W, A, B, s, y_off, y_on, stream=None):

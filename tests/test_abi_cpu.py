@@ -69,6 +69,39 @@ def test_lora_linear_argument_errors(lib):
     assert _lin(lib, M=0) == 0                                  # empty: no launch
 
 
+def _skinny(lib, **kw):
+    a = dict(x=FAKE, M=128, K=4096, N=4096, W=FAKE, u=None, u_row0=0, u_rows=0, B=None, r=0,
+             y=FAKE, dt=0, tile_n=0, split_k=0)
+    a.update(kw)
+    return lib.hydra_skinny_linear(a["x"], a["M"], a["K"], a["N"], a["W"], a["u"], a["u_row0"],
+                                   a["u_rows"], a["B"], a["r"], a["y"], a["dt"], a["tile_n"],
+                                   a["split_k"], None)
+
+
+def test_skinny_linear_argument_errors(lib):
+    lora = dict(u=FAKE, B=FAKE, r=16, u_row0=64, u_rows=64)
+    assert _skinny(lib, x=None) == 1
+    assert _skinny(lib, W=None) == 1
+    assert _skinny(lib, y=None) == 1
+    assert _skinny(lib, r=16, u_row0=64, u_rows=64) == 1        # LoRA without u and B
+    assert _skinny(lib, M=129) == 2                             # one tile of at most 128 rows
+    assert _skinny(lib, M=-1) == 2
+    assert _skinny(lib, N=4104) == 2                            # N % 16
+    assert _skinny(lib, K=4100) == 3                            # K % 8
+    assert _skinny(lib, **dict(lora, r=12)) == 3
+    assert _skinny(lib, **dict(lora, r=264)) == 2
+    assert _skinny(lib, **dict(lora, u_row0=100, u_rows=64)) == 2  # LoRA rows past M
+    assert _skinny(lib, **dict(lora, u_rows=0)) == 2
+    assert _skinny(lib, **dict(lora, u_row0=-1)) == 2
+    assert _skinny(lib, x=FAKE + 8) == 3
+    assert _skinny(lib, dt=7) == 4
+    assert _skinny(lib, tile_n=24) == 4                         # multiple of 16
+    assert _skinny(lib, tile_n=272) == 4
+    assert _skinny(lib, split_k=9) == 4
+    assert _skinny(lib, K=128, split_k=3) == 4                  # more CTAs than k-blocks
+    assert _skinny(lib, M=0) == 0                               # empty: no launch
+
+
 def test_rope_linear_argument_errors(lib):
     f = lib.hydra_dual_linear_rope
 
