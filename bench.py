@@ -764,7 +764,8 @@ class KernelSweep:
     def __init__(self, device, seed=5, reference=False):
         self.device = device
 
-    PARTS = ("projection_sweep", "decode", "gae", "ppo_loss", "attention", "logprobs")
+    PARTS = ("projection_sweep", "decode", "decode_batch", "gae", "ppo_loss", "attention",
+             "logprobs")
 
     def run(self, peaks, reps=20, parts=PARTS):
         import torch
@@ -839,6 +840,29 @@ class KernelSweep:
                     gb.append(byts / ms / 1e6)
                 del Wd
             out["decode"]["frac_of_measured_hbm_mean"] = statistics.mean(gb) / peaks["hbm_gbs"]
+        # ---- decode at 12 and 64 sequences: both streams' rows (24, 128) through the split-K
+        # linear with the library's tile / cluster choice; W rotates through copies beyond L2
+        if "decode_batch" in parts:
+            shapes = (("qkv", 4096, 12288, 32), ("o", 4096, 4096, 0), ("gate_up", 4096, 22016, 32),
+                      ("down", 11008, 4096, 16), ("lm_head", 4096, 32000, 0))
+            gb = []
+            for Mt in (24, 128):
+                S = Mt // 2
+                for n, K, N, r in shapes:
+                    ncopy = max(2, -(-300_000_000 // (N * K * 2)))
+                    Wd = [rnd(N, K) for _ in range(ncopy)]
+                    Bd = rnd(N, r) if r else None
+                    xd = torch.randn(Mt, K, device=dev, generator=g).to(bf)
+                    ud = rnd(S, r, std=1.0) if r else None
+                    yd = torch.empty(Mt, N, dtype=torch.float32 if n == "lm_head" else bf, device=dev)
+                    ms = graph_ms(lambda i: H.hydra_skinny_linear(xd, Wd[i % ncopy], yd, u=ud, B=Bd,
+                                                                  u_row0=S),
+                                  max(reps, 2 * ncopy))
+                    byts = 2.0 * (N * (K + r) + S * r + Mt * K) + yd.element_size() * Mt * N
+                    out["decode_batch"].setdefault(f"M{Mt}", {})[n] = {"ms": ms, "GB/s": byts / ms / 1e6}
+                    gb.append(byts / ms / 1e6)
+                    del Wd
+            out["decode_batch"]["frac_of_measured_hbm_mean"] = statistics.mean(gb) / peaks["hbm_gbs"]
         # ---- GAE at 65536 x 512
         if "gae" in parts or "ppo_loss" in parts:
             S, L = 65536, 512

@@ -120,10 +120,12 @@ def test_generate_eight_sequences_one_prompt_token():
     check_generation(cfg, got, w64, prompt, noise)
 
 
-@pytest.mark.parametrize("S", [12, 64])
+@pytest.mark.parametrize("S", [9, 12, 49, 64])
 def test_generate_large_batches_use_the_tcgen05_gemm(S):
     """More than 8 sequences: both streams' rows no longer fit one dual GEMV (16 rows), so the
-    decode projections run on the tcgen05 GEMM; 64 sequences (128 rows) is the limit."""
+    decode projections run on the split-K tcgen05 linear; above 96 rows the fused RMSNorm kernel takes
+    groups of rows (49 sequences put LoRA-off and LoRA-on rows in one group and end on a
+    partial group); 64 sequences (128 rows) is the limit."""
     cfg = dict(SMALL, prompt_len=6, response_len=5)
     sep, w64 = make_model(cfg, 78)
     prompt = synth.randint(781 + S, (S, 6), 0, cfg["vocab"])
@@ -132,11 +134,12 @@ def test_generate_large_batches_use_the_tcgen05_gemm(S):
     check_generation(cfg, got, w64, prompt, noise)
 
 
-def test_generate_lora_off_streams_agree_bitwise():
+@pytest.mark.parametrize("S", [2, 21, 49])
+def test_generate_lora_off_streams_agree_bitwise(S):
     cfg = dict(SMALL)
     sep, _ = make_model(cfg, 74, zero_B=True)
-    prompt = synth.randint(741, (2, cfg["prompt_len"]), 0, cfg["vocab"])
-    got = run_generate(cfg, sep, prompt, 8, gumbel_noise(742, 8, 2, cfg["vocab"]))
+    prompt = synth.randint(741, (S, cfg["prompt_len"]), 0, cfg["vocab"])
+    got = run_generate(cfg, sep, prompt, 8, gumbel_noise(742, 8, S, cfg["vocab"]))
     assert np.array_equal(got["logp_actor"], got["logp_ref"])
 
 
