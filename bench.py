@@ -863,6 +863,24 @@ class KernelSweep:
                     gb.append(byts / ms / 1e6)
                     del Wd
             out["decode_batch"]["frac_of_measured_hbm_mean"] = statistics.mean(gb) / peaks["hbm_gbs"]
+            # launch cost: 128 rows x N 4096 with 128-column tiles, K of 1 to 64 k-blocks per
+            # CTA, without a cluster and with 4 CTAs splitting K
+            Wd = [rnd(4096, 4096) for _ in range(9)]
+            xd = torch.randn(128, 4096, device=dev, generator=g).to(bf)
+            yd = torch.empty(128, 4096, dtype=bf, device=dev)
+            cost = {}
+            for K in (64, 256, 1024, 4096):
+                for ks in (1, 4):
+                    if ks > K // 64:
+                        continue
+                    xk = xd[:, :K].contiguous()
+                    Wk = [w[:, :K].contiguous() for w in Wd]
+                    ms = graph_ms(lambda i: H.hydra_skinny_linear(xk, Wk[i % 9], yd, tile_n=128,
+                                                                  split_k=ks), max(reps, 18))
+                    cost[f"K{K}_split{ks}"] = {"us": ms * 1000.0}
+                    del Wk
+            out["decode_batch"]["launch_cost_N4096_M128_tile128"] = cost
+            del Wd
         # ---- GAE at 65536 x 512
         if "gae" in parts or "ppo_loss" in parts:
             S, L = 65536, 512
