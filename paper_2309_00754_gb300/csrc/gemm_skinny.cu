@@ -145,6 +145,20 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       }
     }
     __syncwarp();
+    // Programmatic dependent launch: W and B are frozen, so the weight halves of the first
+    // ring's worth of items load before the wait on the preceding kernel (which writes x and
+    // u); a stage's barrier completes only once its x half, loaded after the wait, lands too.
+    const int pre = min(items, p.stages);
+    if (elect_one()) {
+      for (int i = 0; i < pre; ++i) {
+        mbar_arrive_expect_tx(full_bar(i), p.stage_bytes);
+        const uint32_t b_dst = smem_base + i * p.stage_bytes + A_TILE;
+        if (i < n_main) tma_load_2d(b_dst, &tm_w, (kb0 + i) * BK, n0, full_bar(i));
+        else tma_load_2d(b_dst, &tm_b, (i - n_main) * BK, n0, full_bar(i));
+      }
+    }
+    __syncwarp();
+    pdl_wait();
     int it = 0;
     for (; it < items; ++it) {
       const int s = it % p.stages;
@@ -152,16 +166,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                              kDevTimeoutProducer))
         break;
       if (elect_one()) {
-        mbar_arrive_expect_tx(full_bar(s), p.stage_bytes);
+        if (it >= pre) mbar_arrive_expect_tx(full_bar(s), p.stage_bytes);
         const uint32_t a_dst = smem_base + s * p.stage_bytes;
         if (it < n_main) {
           const int k = (kb0 + it) * BK;
           tma_load_2d(a_dst, &tm_x, k, 0, full_bar(s));
-          tma_load_2d(a_dst + A_TILE, &tm_w, k, n0, full_bar(s));
+          if (it >= pre) tma_load_2d(a_dst + A_TILE, &tm_w, k, n0, full_bar(s));
         } else {
           const int k = (it - n_main) * BK;
           tma_load_2d(a_dst, &tm_u, k, -p.u_row0, full_bar(s));  // rows above u_row0: zeros
-          tma_load_2d(a_dst + A_TILE, &tm_b, k, n0, full_bar(s));
+          if (it >= pre) tma_load_2d(a_dst + A_TILE, &tm_b, k, n0, full_bar(s));
         }
       }
       __syncwarp();
@@ -458,13 +472,15 @@ int launch_skinny_gemm_tc(const SkinnyArgs& a, cudaStream_t st) {
   cfg.blockDim = dim3(NUM_THREADS);
   cfg.dynamicSmemBytes = smem_bytes(c.bn, c.stages);
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = static_cast<unsigned>(c.ks);
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, skinny_gemm_kernel, mx, mw, mu, mb, p) == cudaSuccess ? 0 : -3;
 }
 
