@@ -82,12 +82,20 @@ bool gen_config_ok(const hydra_llama_config* c) {
 }
 
 // y = [x_off; x_on] W^T (+ u B^T on the on rows; u [S, r] = s x_on A^T, already computed by
-// the fused row kernel that produced x) for S rows per stream: the dual-output GEMV for up to
-// 16 rows, beyond that the split-K tcgen05 kernel over both streams' rows in one tile (the
-// CTA-tile GEMM when N is not a multiple of 16); y [2 S, N] bf16 or fp32 (off rows first).
+// the fused row kernel that produced x) for S rows per stream; y [2 S, N] bf16 or fp32 (off
+// rows first). Kernel by rows and width, as measured on GB300 (7B decode step, both streams):
+//  * up to 8 rows: the dual-output GEMV (4 sequences: 3.73 ms per step against 3.97 ms with
+//    the split-K kernel on the wide projections);
+//  * 9 to 16 rows: the split-K tcgen05 kernel for outputs of 8192 columns and more, the GEMV
+//    for the narrower ones (8 sequences: 3.93 ms, against 4.48 ms all-GEMV and 4.13 ms
+//    all-split-K);
+//  * above 16 rows: the split-K kernel over both streams' rows in one tile (the CTA-tile GEMM
+//    when N is not a multiple of 16).
 int decode_linear(const void* x, int64_t S, int64_t K, int64_t N, const void* W, const void* B,
                   int64_t r, const void* u, void* y, bool f32, int* err, cudaStream_t st) {
-  if (2 * S > hydra::kGemvMaxRows && hydra::skinny_gemm_supported(2 * S, K, N, r)) {
+  const int64_t rows = 2 * S;
+  const bool split_k = rows > hydra::kGemvMaxRows || (rows > 8 && N >= 8192);
+  if (split_k && hydra::skinny_gemm_supported(rows, K, N, r)) {
     hydra::SkinnyArgs a;
     a.x = x;
     a.M = 2 * S;

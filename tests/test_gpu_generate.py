@@ -120,6 +120,17 @@ def test_generate_eight_sequences_one_prompt_token():
     check_generation(cfg, got, w64, prompt, noise)
 
 
+def test_generate_eight_sequences_wide_head():
+    """16 rows with an output of 8192 columns: the LM head runs on the split-K tcgen05 linear
+    while the narrower projections stay on the GEMV."""
+    cfg = dict(SMALL, vocab=8192, prompt_len=4, response_len=5)
+    sep, w64 = make_model(cfg, 79)
+    prompt = synth.randint(791, (8, 4), 0, cfg["vocab"])
+    noise = gumbel_noise(792, 5, 8, cfg["vocab"])
+    got = run_generate(cfg, sep, prompt, 5, noise)
+    check_generation(cfg, got, w64, prompt, noise)
+
+
 @pytest.mark.parametrize("S", [9, 12, 49, 64])
 def test_generate_large_batches_use_the_tcgen05_gemm(S):
     """More than 8 sequences: both streams' rows no longer fit one dual GEMV (16 rows), so the
