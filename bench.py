@@ -8,6 +8,9 @@ in HBM. Prints ONE JSON line (rank 0). Workloads:
                     random-init Llama-7B, batch 4 x (256 prompt + 512 response) tokens,
                     LoRA r=16 on q/v/gate/up/down, reward/value head 4096 -> 1.
 
+  hydra_scoring_llama7b_400_400 : the same pass at the paper's sequence shape (Appendix B:
+                    batch 4 x (400 prompt + 400 response)), for context.
+
   lm_head_scoring : final hidden states [4 x 512 x 4096] bf16 -> LoRA down (r=16) ->
                     dual-output LM head 4096 -> 32000 (fp32 logits, both streams, one pass
                     over W) -> sampled-token log-probs + KL reward (beta 0.1, score at the
@@ -259,6 +262,8 @@ class HydraScoringLlama7B:
         self.llama = llama
         self.cfg = dict(llama.LLAMA7B)
         c = self.cfg
+        if getattr(self, "shape", None):  # (prompt, response) of a variant workload
+            c["prompt_len"], c["response_len"] = self.shape
         self.S, self.P0, self.L = getattr(self, "batch", 4), c["prompt_len"], c["response_len"]
         self.beta, self.gamma, self.lam = c["beta"], c["gamma"], c["lam"]
         P = self.P0 + self.L
@@ -336,10 +341,10 @@ class HydraScoringLlama7B:
                 "per_launch_ms": ms / n}
 
     def config(self):
-        return {"workload": "hydra_scoring_llama7b: random-init Llama-7B (32 layers, d 4096, 32 heads, "
+        return {"workload": f"{self.name}: random-init Llama-7B (32 layers, d 4096, 32 heads, "
                             "SwiGLU 11008, vocab 32000, bf16), LoRA r=16 s=2 on q/v/gate/up/down, reward/"
-                            "value head 4096->1; batch 4 x (256 prompt + 512 response); logp/KL beta 0.1, "
-                            "GAE gamma 1 lambda 0.95",
+                            f"value head 4096->1; batch {self.S} x ({self.P0} prompt + {self.L} response); "
+                            "logp/KL beta 0.1, GAE gamma 1 lambda 0.95",
                 "batch": self.S, "prompt_len": self.P0, "response_len": self.L,
                 "scored_tokens_per_step": self.units,
                 "processed_tokens_per_step": 2 * self.S * (self.P0 + self.L),
@@ -390,9 +395,10 @@ class HydraScoringLlama7B:
                       beta=self.beta, gamma=self.gamma, lam=self.lam)
         return time.perf_counter() - t0
 
-    def oracle_throughput(self, steps=1):
-        """(tokens/s, description): the slice's pass time is t(0 layers) + 32 (t(1) - t(0))."""
-        smp = self.oracle_sample(1)
+    def oracle_throughput(self, steps=1, single_thread=False):
+        """(tokens/s, description): the slice's pass time is t(0 layers) + 32 (t(1) - t(0)); a
+        quarter-size slice on one BLAS thread."""
+        smp = self.oracle_sample(1, prompt=16, resp=32) if single_thread else self.oracle_sample(1)
         t_head = self.oracle_time(smp, 0)
         t1 = [self.oracle_time(smp, 1) for _ in range(steps)]
         n = self.cfg["n_layers"]
@@ -401,6 +407,14 @@ class HydraScoringLlama7B:
                 f"width through the fp64 oracle: embed + heads {t_head:.2f} s, one decoder layer "
                 f"{statistics.mean(t1) - t_head:.2f} s, pass time extrapolated to {n} layers")
         return smp["resp"] * len(t_pass) / sum(t_pass), desc
+
+
+class HydraScoringLlama7BPaperShape(HydraScoringLlama7B):
+    """The full J-Hydra scoring pass at the paper's sequence shape (Appendix B: batch 4,
+    400-token prompts, 400-token completions), for context beside the 256 + 512 workload."""
+
+    name = "hydra_scoring_llama7b_400_400"
+    shape = (400, 400)
 
 
 class HydraPPOScoringLlama7B(HydraScoringLlama7B):
@@ -592,7 +606,7 @@ class HydraGenerateLlama7B(HydraScoringLlama7B):
         O.llama_generate(smp["w"], smp["ids"][:smp["prompt"]], 2, smp["cfg"], n_layers=n_layers)
         return time.perf_counter() - t0
 
-    def oracle_throughput(self, steps=1):
+    def oracle_throughput(self, steps=1, single_thread=False):
         """(tokens/s, description): 2 draws after a 32-token prompt, per-draw time t(0 layers)
         + 32 (t(1) - t(0)), the oracle recomputing the whole prefix at each draw."""
         smp = self.oracle_sample(1)
@@ -727,7 +741,7 @@ class HydraPPOIterationLlama7B(HydraGenerateLlama7B):
                    sc["returns"][None], sc["values"][None], [2], whiten=True)
         return time.perf_counter() - t0
 
-    def oracle_throughput(self, steps=1):
+    def oracle_throughput(self, steps=1, single_thread=False):
         smp = self.oracle_sample(1)
         t_head = self.oracle_time(smp, 0)
         t1 = [self.oracle_time(smp, 1) for _ in range(steps)]
@@ -938,6 +952,7 @@ class KernelSweep:
 
 
 WORKLOADS = {LmHeadScoring.name: LmHeadScoring, HydraScoringLlama7B.name: HydraScoringLlama7B,
+             HydraScoringLlama7BPaperShape.name: HydraScoringLlama7BPaperShape,
              HydraPPOScoringLlama7B.name: HydraPPOScoringLlama7B,
              HydraGenerateLlama7B.name: HydraGenerateLlama7B,
              HydraPPOIterationLlama7B.name: HydraPPOIterationLlama7B,
@@ -981,13 +996,60 @@ def barrier(world, device=None):
             dist.barrier()
 
 
+_BLAS_THREAD_FNS = (("scipy_openblas_set_num_threads64_", "scipy_openblas_get_num_threads64_"),
+                    ("scipy_openblas_set_num_threads", "scipy_openblas_get_num_threads"),
+                    ("openblas_set_num_threads64_", "openblas_get_num_threads64_"),
+                    ("openblas_set_num_threads", "openblas_get_num_threads"))
+
+
+def blas_thread_control():
+    """(get, set) for the thread count of the OpenBLAS that numpy loaded, or None: the library
+    is found among this process's mapped files and driven through its exported setter."""
+    import ctypes
+    np.ones(2) @ np.ones(2)  # the BLAS is mapped once used
+    try:
+        with open("/proc/self/maps") as f:
+            paths = {ln.split()[-1] for ln in f if len(ln.split()) >= 6 and "openblas" in ln.lower()}
+    except OSError:
+        return None
+    for path in sorted(paths):
+        try:
+            lib = ctypes.CDLL(path)
+        except OSError:
+            continue
+        for set_name, get_name in _BLAS_THREAD_FNS:
+            if hasattr(lib, set_name) and hasattr(lib, get_name):
+                setter, getter = getattr(lib, set_name), getattr(lib, get_name)
+                setter.argtypes = [ctypes.c_int]
+                getter.restype = ctypes.c_int
+                return getter, setter
+    return None
+
+
+def single_thread_oracle(wl):
+    """The oracle's throughput with BLAS on one thread (a smaller slice than the all-core leg)."""
+    ctl = blas_thread_control()
+    if ctl is None or not hasattr(wl, "oracle_throughput"):
+        return None, "no OpenBLAS thread control found" if ctl is None else "not measured for this workload"
+    get, set_ = ctl
+    prev = get()
+    try:
+        set_(1)
+        value, desc = wl.oracle_throughput(single_thread=True)
+    finally:
+        set_(prev)
+    return value, desc + "; BLAS threads = 1"
+
+
 def time_oracle(wl, target_s=12.0):
-    """Oracle throughput on a bounded sample (rank 0, host cores)."""
+    """Oracle throughput on a bounded sample (rank 0, host cores), then on one thread."""
     cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
     if hasattr(wl, "oracle_throughput"):
         value, desc = wl.oracle_throughput()
+        st_value, st_desc = single_thread_oracle(wl)
         return {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
-                "sample": desc + "; BLAS threads = cores"}
+                "sample": desc + "; BLAS threads = cores",
+                "single_thread": {"value": st_value, "unit": UNIT, "cores": 1, "sample": st_desc}}
     probe = wl.oracle_sample(8)
     t0 = time.perf_counter()
     wl.oracle_run(probe)

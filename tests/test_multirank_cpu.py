@@ -98,3 +98,19 @@ def test_all_reduce_adv_moments_gloo():
     assert n == ref["n"]
     assert abs(mean - ref["adv_mean"]) < 1e-13
     assert abs(np.sqrt(m2 / n) - ref["adv_std"]) < 1e-13
+
+
+def test_blas_thread_control_sets_and_restores():
+    # the CPU baseline's single-thread leg drives numpy's OpenBLAS through its own setter
+    import bench
+    ctl = bench.blas_thread_control()
+    if ctl is None:
+        pytest.skip("numpy is not linked against an OpenBLAS with a thread setter here")
+    get, set_ = ctl
+    prev = get()
+    try:
+        set_(1)
+        assert get() == 1
+    finally:
+        set_(prev)
+    assert get() == prev
