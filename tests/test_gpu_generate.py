@@ -131,12 +131,24 @@ def test_generate_eight_sequences_wide_head():
     check_generation(cfg, got, w64, prompt, noise)
 
 
+def test_generate_vocab_not_multiple_of_16():
+    """A vocabulary of 520 (a multiple of 8, not of 16) at 9 sequences: the decode LM head
+    falls back to the CTA-tile tcgen05 GEMM while the other projections take the split-K
+    linear."""
+    cfg = dict(SMALL, vocab=520, prompt_len=4, response_len=4)
+    sep, w64 = make_model(cfg, 80)
+    prompt = synth.randint(801, (9, 4), 0, cfg["vocab"])
+    noise = gumbel_noise(802, 4, 9, cfg["vocab"])
+    got = run_generate(cfg, sep, prompt, 4, noise)
+    check_generation(cfg, got, w64, prompt, noise)
+
+
 @pytest.mark.parametrize("S", [9, 12, 49, 64])
 def test_generate_large_batches_use_the_tcgen05_gemm(S):
     """More than 8 sequences: both streams' rows no longer fit one dual GEMV (16 rows), so the
-    decode projections run on the split-K tcgen05 linear; above 96 rows the fused RMSNorm kernel takes
-    groups of rows (49 sequences put LoRA-off and LoRA-on rows in one group and end on a
-    partial group); 64 sequences (128 rows) is the limit."""
+    decode projections run on the split-K tcgen05 linear; above 96 rows the fused RMSNorm
+    kernel takes groups of rows (49 sequences put LoRA-off and LoRA-on rows in one group and
+    end on a partial group); 64 sequences (128 rows) is the limit."""
     cfg = dict(SMALL, prompt_len=6, response_len=5)
     sep, w64 = make_model(cfg, 78)
     prompt = synth.randint(781 + S, (S, 6), 0, cfg["vocab"])

@@ -70,6 +70,9 @@ def _run(x, W, u, Bm, u_row0, out=torch.bfloat16, tile_n=0, split_k=0):
     (50, 2048, 1024, 72, 128, 6),   # two LoRA k-blocks; ranks 4 and 5 own no columns
     (40, 1024, 1040, 16, 256, 1),   # single CTA per tile
     (64, 4096, 12288, 32, 0, 0),    # decode qkv shape
+    (64, 4096, 22016, 32, 0, 0),    # decode gate/up shape
+    (64, 11008, 4096, 16, 0, 0),    # decode down shape
+    (12, 11008, 4096, 16, 0, 0),    # down shape at 12 sequences
 ])
 def test_skinny_linear_parity(S, K, N, r, tile_n, split_k):
     x, W, A, Bm = _problem(2 * S, K, N, r, seed=S + K + N + r)
@@ -99,6 +102,15 @@ def test_skinny_linear_fp32_out(split_k):
     y = _run(dev_bf16(x), dev_bf16(W), dev_bf16(O.f64_to_bf16_bits(u)), dev_bf16(Bm), S,
              out=torch.float32, split_k=split_k)
     assert_rel(host_f64(y), ref, 1e-4, "y fp32")
+
+
+def test_skinny_linear_lm_head_shape_fp32():
+    # the decode LM head: 4096 -> 32000 with fp32 logits for both streams' 128 rows
+    S, K, N = 64, 4096, 32000
+    x, W, A, Bm = _problem(2 * S, K, N, 0, seed=17)
+    ref, _ = _reference(x, W, A, Bm, S, S, out_bf16=False)
+    y = _run(dev_bf16(x), dev_bf16(W), None, None, 0, out=torch.float32)
+    assert_rel(host_f64(y), ref, 1e-4, "logits")
 
 
 def test_skinny_linear_deterministic_and_lora_off_bitwise():
