@@ -315,17 +315,16 @@ size_t smem_bytes(int bn, int stages) {
 }
 
 // Clusters of ks CTAs with this shared-memory size that fit on the device at once.
-int active_clusters(int ks, size_t smem) {
+int active_clusters(int dev, int ks, size_t smem) {
   static std::mutex mu;
   static std::vector<std::pair<long long, int>> cache;
-  const long long key = static_cast<long long>(ks) << 32 | static_cast<long long>(smem);
+  const long long key = static_cast<long long>(dev) << 48 | static_cast<long long>(ks) << 32 |
+                        static_cast<long long>(smem);
   std::lock_guard<std::mutex> lock(mu);
   for (auto& e : cache)
     if (e.first == key) return e.second;
-  int dev = 0, nsm = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess ||
-      cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-    return 0;
+  int nsm = 0;
+  if (cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
   int n = nsm / ks;
   if (ks > 1) {
     cudaLaunchConfig_t cfg = {};
@@ -359,7 +358,7 @@ int active_clusters(int ks, size_t smem) {
 //  * a cluster adds about 1 us of barriers plus the exchange: ks - 1 partial slices of
 //    M x (bn / ks) fp32 read through distributed shared memory at about 120 GB/s.
 // Clusters beyond what fits on the device at once run in further waves.
-Choice choose(int64_t M, int64_t K, int64_t N, int64_t r) {
+Choice choose(int dev, int64_t M, int64_t K, int64_t N, int64_t r) {
   const int64_t kb = (K + skinny::BK - 1) / skinny::BK;
   const double t_hbm = 2.0 * static_cast<double>(N) * static_cast<double>(K + r) / 6.5e6;
   Choice best{256, 1, stages_for(256)};
@@ -371,7 +370,7 @@ Choice choose(int64_t M, int64_t K, int64_t N, int64_t r) {
       if (ks > kb) break;
       const int cw = ((bn / ks) + 15) / 16 * 16;
       if (ks > 1 && static_cast<int64_t>(cw) * (ks - 1) >= bn) continue;  // a rank with no columns
-      const int fit = active_clusters(ks, smem_bytes(bn, stages));
+      const int fit = active_clusters(dev, ks, smem_bytes(bn, stages));
       if (fit < 1) continue;
       const double waves = static_cast<double>((tiles + fit - 1) / fit);
       const double kb_cta = static_cast<double>((kb + ks - 1) / ks);
@@ -389,8 +388,9 @@ Choice choose(int64_t M, int64_t K, int64_t N, int64_t r) {
   return best;
 }
 
-Choice cached_choice(int64_t M, int64_t K, int64_t N, int64_t r) {
+Choice cached_choice(int dev, int64_t M, int64_t K, int64_t N, int64_t r) {
   struct Entry {
+    int dev;
     int64_t M, K, N, r;
     Choice c;
   };
@@ -399,11 +399,11 @@ Choice cached_choice(int64_t M, int64_t K, int64_t N, int64_t r) {
   {
     std::lock_guard<std::mutex> lock(mu);
     for (auto& e : cache)
-      if (e.M == M && e.K == K && e.N == N && e.r == r) return e.c;
+      if (e.dev == dev && e.M == M && e.K == K && e.N == N && e.r == r) return e.c;
   }
-  const Choice c = choose(M, K, N, r);
+  const Choice c = choose(dev, M, K, N, r);
   std::lock_guard<std::mutex> lock(mu);
-  if (cache.size() < 256) cache.push_back(Entry{M, K, N, r, c});
+  if (cache.size() < 256) cache.push_back(Entry{dev, M, K, N, r, c});
   return c;
 }
 
@@ -420,14 +420,17 @@ int launch_skinny_gemm_tc(const SkinnyArgs& a, cudaStream_t st) {
   if (a.r > 0 && (a.u == nullptr || a.B == nullptr || a.u_rows < 1 || a.u_row0 < 0 ||
                   a.u_row0 + a.u_rows > a.M))
     return -4;
-  static bool attr_set = false;
-  if (!attr_set) {
+  // the shared-memory limit is a per-device function attribute: set once per device
+  static bool attr_set[64] = {false};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return -1;
+  if (!attr_set[dev]) {
     if (cudaFuncSetAttribute(skinny_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              kSmemMax) != cudaSuccess)
       return -1;
-    attr_set = true;
+    attr_set[dev] = true;
   }
-  Choice c = cached_choice(a.M, a.K, a.N, a.r);
+  Choice c = cached_choice(dev, a.M, a.K, a.N, a.r);
   if (a.bn > 0) {  // explicit tile width / cluster size (sweeps and tests)
     if (a.bn % 16 != 0 || a.bn > kMaxBN) return -4;
     c.bn = a.bn;
