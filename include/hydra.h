@@ -67,6 +67,16 @@ int hydra_abi_version(void);
 hydra_status hydra_device_error(int32_t* code_out, int clear);
 
 /*
+ * Self-test of the in-kernel failure detection: one CTA waits on an mbarrier that nothing
+ * ever signals, through the same bounded wait every kernel of the library uses. The wait
+ * expires after about 2e9 SM clock cycles (about 1 s), the kernel records 0x105 in the
+ * device error word and returns; nothing traps and the context stays usable. Asynchronous
+ * on `stream` (a cudaStream_t, NULL = default); read the code with hydra_device_error.
+ * Returns HYDRA_OK, or HYDRA_ERR_CUDA when the launch fails.
+ */
+hydra_status hydra_selftest_wait_timeout(void* stream);
+
+/*
  * LoRA down-projection (§2 Stage 3: LoRA on all linear layers; the update is
  * y = x W + s (x A) B): u = s * (x_on A^T), rounded to bf16.
  *   x_on : bf16 [M, K]       A : bf16 [r, K] (the paper's K x r matrix A, transposed)

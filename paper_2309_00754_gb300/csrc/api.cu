@@ -4,6 +4,7 @@
 #include <stdint.h>
 
 #include "../../include/hydra.h"
+#include "common.cuh"
 #include "kernels.h"
 
 namespace {
@@ -123,6 +124,22 @@ hydra_status lora_linear_impl(const void* x_off, const void* x_on, int64_t M, in
   return rc == 0 ? HYDRA_OK : HYDRA_ERR_CUDA;
 }
 
+// One warp waits on an mbarrier that nothing ever arrives on, through the bounded wait that
+// every kernel of the library uses: the wait expires after kWaitBudgetCycles, records
+// kDevTimeoutSelftest in the device error word and the kernel returns.
+__global__ void bounded_wait_selftest_kernel(int* err) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    hydra::mbar_init(hydra::smem_u32(&bar), 1);
+    abort_flag = 0;
+    hydra::fence_mbar_init();
+  }
+  __syncthreads();
+  hydra::warp_wait_bounded(hydra::smem_u32(&bar), 0, reinterpret_cast<volatile int*>(&abort_flag),
+                           err, hydra::kDevTimeoutSelftest);
+}
+
 }  // namespace
 
 extern "C" {
@@ -143,6 +160,13 @@ const char* hydra_status_string(int status) {
 }
 
 int hydra_abi_version(void) { return 1; }
+
+hydra_status hydra_selftest_wait_timeout(void* stream) {
+  int* err = hydra::device_error_word();
+  if (err == nullptr) return HYDRA_ERR_CUDA;
+  bounded_wait_selftest_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(err);
+  return cudaPeekAtLastError() == cudaSuccess ? HYDRA_OK : HYDRA_ERR_CUDA;
+}
 
 hydra_status hydra_device_error(int32_t* code_out, int clear) {
   if (code_out == nullptr) return HYDRA_ERR_NULL;

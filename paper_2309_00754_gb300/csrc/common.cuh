@@ -18,6 +18,7 @@ enum DeviceError : int {
   kDevTimeoutMma = 0x102,
   kDevTimeoutEpilogue = 0x103,
   kDevTimeoutDrain = 0x104,
+  kDevTimeoutSelftest = 0x105,  // hydra_selftest_wait_timeout: the expected expiry
   kDevBadTokenId = 0x201,
   kDevBadLength = 0x202,
 };

@@ -32,6 +32,7 @@ _SIGNATURES = {
     "hydra_lora_linear_algo": (ctypes.c_int, [_vp, _vp, _c_i64, _c_i64, _c_i64, _vp, _vp, _vp,
                                               _c_i64, ctypes.c_float, _vp, _vp, ctypes.c_int, _vp,
                                               ctypes.c_size_t, ctypes.c_int, _vp]),
+    "hydra_selftest_wait_timeout": (ctypes.c_int, [_vp]),
     "hydra_skinny_linear": (ctypes.c_int, [_vp, _c_i64, _c_i64, _c_i64, _vp, _vp, _c_i64, _c_i64,
                                            _vp, _c_i64, _vp, ctypes.c_int, ctypes.c_int,
                                            ctypes.c_int, _vp]),
@@ -194,6 +195,11 @@ def device_error(clear: bool = True) -> int:
     code = ctypes.c_int32(0)
     _check("hydra_device_error", load().hydra_device_error(ctypes.byref(code), int(clear)))
     return code.value
+
+
+def selftest_wait_timeout(stream=None):
+    """Launch the bounded-wait self-test: about 1 s later the device error word holds 0x105."""
+    _check("hydra_selftest_wait_timeout", load().hydra_selftest_wait_timeout(_stream(stream)))
 
 
 def lora_linear_workspace_size(M: int, r: int) -> int:
