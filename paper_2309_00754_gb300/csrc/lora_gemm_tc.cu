@@ -69,6 +69,8 @@ struct Params {
   int deferred;   // shared input with LoRA and both outputs: y_off drain, then LoRA
   int streams;    // 1 (shared) or 2 (stacked)
   int m_tiles, n_tiles, total_tiles;
+  int m_group;  // CTA-pair kernel: 0 = m fastest over all of M; else groups of m_group
+                // m-tiles, m fastest inside a group, then n, then the next group
   int has_off, has_on, has_crit;
   int out_f32;
   int bn;          // tile width in output columns (multiple of 16; 256 for the single-CTA kernel)
@@ -700,8 +702,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     Tile tl;
     tl.stream = t % p.streams;
     t /= p.streams;
-    tl.m0 = (t % p.m_tiles) * 256 + static_cast<int>(rank) * 128;
-    tl.n0 = (t / p.m_tiles) * p.bn;
+    int mi, ni;
+    if (p.m_group > 0) {
+      const int per_group = p.m_group * p.n_tiles;
+      const int grp = t / per_group, r = t - grp * per_group;
+      const int gm = min(p.m_group, p.m_tiles - grp * p.m_group);  // the last group may be short
+      mi = grp * p.m_group + r % gm;
+      ni = r / gm;
+    } else {
+      mi = t % p.m_tiles;
+      ni = t / p.m_tiles;
+    }
+    tl.m0 = mi * 256 + static_cast<int>(rank) * 128;
+    tl.n0 = ni * p.bn;
     const bool lora = p.shared_x ? true : (tl.stream >= 1);
     const bool wanted = tl.stream == 2 ? p.has_crit : p.has_on;
     tl.n_lora = (p.kb_lora > 0 && lora && wanted) ? p.kb_lora : 0;
@@ -1032,6 +1045,21 @@ int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream) {
   p.m_tiles = static_cast<int>(pair ? (a.M + 255) / 256 : (a.M + BM - 1) / BM);
   p.n_tiles = static_cast<int>((a.N + bn - 1) / bn);
   p.total_tiles = p.m_tiles * p.n_tiles * p.streams;
+  // Tile order of the CTA-pair kernel. Over all of M, the tiles in flight at once (one per
+  // pair) cover every m-tile of a few n-columns: x stays in L2 if it fits, else it is read
+  // again for each column (a 3072 x 11008 down-projection input of both streams, 135 MB,
+  // measured 1026 MB of DRAM reads per launch). Beyond half of L2, m-tiles go in groups
+  // whose inputs total about 48 MB, and W is read once per group instead.
+  p.m_group = 0;
+  if (pair) {
+    const int64_t x_bytes = static_cast<int64_t>(p.streams) * a.M * a.K * 2;
+    const int64_t mtile_bytes = static_cast<int64_t>(p.streams) * 256 * a.K * 2;
+    if (x_bytes > (int64_t{64} << 20) && p.m_tiles > 1) {
+      const int64_t g = (int64_t{48} << 20) / mtile_bytes;
+      p.m_group = static_cast<int>(g < 1 ? 1 : (g > p.m_tiles ? p.m_tiles : g));
+      if (p.m_group >= p.m_tiles) p.m_group = 0;
+    }
+  }
   p.out_f32 = a.out_f32;
   p.bn = bn;
   p.rope_P = static_cast<int>(a.rope_P < 1 ? 1 : a.rope_P);
