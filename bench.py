@@ -255,6 +255,10 @@ class HydraScoringLlama7B:
     name = "hydra_scoring_llama7b"
     seed = 4
     default_steps, default_warmup = 20, 3
+    # DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) per GEMM launch, averaged over
+    # the 129 GEMM launches of one pass of this workload (batch 4, two streams) in a one-pass
+    # ncu capture of the current kernel; no figure for other shapes or stream counts
+    gemm_dram_bytes_per_launch = 520.6e6
 
     def __init__(self, device, seed=4, reference=False):
         import torch
@@ -327,6 +331,12 @@ class HydraScoringLlama7B:
         out["logprobs"]["GB/s"] = self.logp_bytes * lp[1] / lp[0] / 1e6
         return out
 
+    def traffic_per_launch(self):
+        """The captured DRAM bytes per GEMM launch, for the exact workload they were taken on."""
+        if type(self) is HydraScoringLlama7B and self.S == 4 and not getattr(self, "shape", None):
+            return self.gemm_dram_bytes_per_launch
+        return None
+
     def roofline(self, peaks, prof):
         ms = sum(prof[k][0] for k in self.class_flops)
         n = sum(prof[k][1] for k in self.class_flops)
@@ -335,7 +345,7 @@ class HydraScoringLlama7B:
         peak = peaks["bf16_tflops_sustained"]
         return {"kernel": "dual_lora_gemm_tcgen05 (all projections + LM head of the pass)",
                 "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                "frac": achieved / peak, "traffic": None,
+                "frac": achieved / peak, "traffic": self.traffic_per_launch(),
                 "peak_kind": f"bf16 dense, {peaks['source']} sustained",
                 "per_launch_flop": self.gemm_flops / sum(self.launch_counts[k] for k in self.class_flops),
                 "per_launch_ms": ms / n}
