@@ -77,6 +77,10 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
 // scores of the npos = pos + 1 cached keys into shared memory
 // (groups of 8 lanes per key, 32 bytes each, reduced by shuffles), the softmax over them,
 // then the weighted sum of the values (lane = 4 output dimensions, warps split positions).
+// kPrefetch: the key loads of the next iteration are issued before this one's are reduced,
+// for small batches (latency-bound); without it, each iteration loads its own keys (large
+// batches, bound by HBM bandwidth, measured faster that way).
+template <bool kPrefetch>
 __global__ void __launch_bounds__(kAttnThreads)
     decode_attention_kernel(const __nv_bfloat16* __restrict__ qkv, int ld, int d, int H,
                             const float2* __restrict__ table, __nv_bfloat16* __restrict__ ck,
@@ -132,20 +136,35 @@ __global__ void __launch_bounds__(kAttnThreads)
     }
   }
   // warp-uniform trip count: all 32 lanes reach the shuffles. Each 8-lane group takes two
-  // keys per iteration, both loaded before either is reduced.
+  // keys per iteration, both loaded before either is reduced (with kPrefetch, the next
+  // iteration's keys are loaded before this one's are reduced).
   constexpr int kKeysPerIter = 2 * 4 * kAttnWarps;
+  auto load_keys = [&](int base, uint4 (&kk)[4]) {
+    const int q0 = base + g, q1 = base + 4 * kAttnWarps + g;
+    kk[0] = kk[1] = kk[2] = kk[3] = make_uint4(0u, 0u, 0u, 0u);
+    if (q0 < npos) {
+      const __nv_bfloat16* kr = K + static_cast<size_t>(q0) * kDh + 16 * sub;
+      kk[0] = __ldcs(reinterpret_cast<const uint4*>(kr));
+      kk[1] = __ldcs(reinterpret_cast<const uint4*>(kr + 8));
+    }
+    if (q1 < npos) {
+      const __nv_bfloat16* kr = K + static_cast<size_t>(q1) * kDh + 16 * sub;
+      kk[2] = __ldcs(reinterpret_cast<const uint4*>(kr));
+      kk[3] = __ldcs(reinterpret_cast<const uint4*>(kr + 8));
+    }
+  };
+  uint4 cur[4], nxt[4];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) nxt[e] = make_uint4(0u, 0u, 0u, 0u);
+  if (kPrefetch) load_keys(warp * 4, cur);
   for (int base = warp * 4; base < npos; base += kKeysPerIter) {
     const int p0 = base + g, p1 = base + 4 * kAttnWarps + g;
-    uint4 a0 = make_uint4(0u, 0u, 0u, 0u), b0 = a0, a1 = a0, b1 = a0;
-    if (p0 < npos) {
-      const __nv_bfloat16* kr = K + static_cast<size_t>(p0) * kDh + 16 * sub;
-      a0 = __ldcs(reinterpret_cast<const uint4*>(kr));
-      b0 = __ldcs(reinterpret_cast<const uint4*>(kr + 8));
-    }
-    if (p1 < npos) {
-      const __nv_bfloat16* kr = K + static_cast<size_t>(p1) * kDh + 16 * sub;
-      a1 = __ldcs(reinterpret_cast<const uint4*>(kr));
-      b1 = __ldcs(reinterpret_cast<const uint4*>(kr + 8));
+    if (!kPrefetch) load_keys(base, cur);
+    else if (base + kKeysPerIter < npos) load_keys(base + kKeysPerIter, nxt);  // warp-uniform
+    const uint4 a0 = cur[0], b0 = cur[1], a1 = cur[2], b1 = cur[3];
+    if (kPrefetch) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) cur[e] = nxt[e];
     }
     const uint32_t w0[8] = {a0.x, a0.y, a0.z, a0.w, b0.x, b0.y, b0.z, b0.w};
     const uint32_t w1[8] = {a1.x, a1.y, a1.z, a1.w, b1.x, b1.y, b1.z, b1.w};
@@ -661,15 +680,19 @@ int launch_decode_attention(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t
                             int64_t Pmax, void* out, int64_t ld_out, cudaStream_t st) {
   if (R == 0) return 0;
   const size_t smem = decode_attention_smem(Pmax);
-  static size_t attr = 0;
-  if (smem > 48 * 1024 && smem > attr) {
-    if (cudaFuncSetAttribute(decode_attention_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  // pipelined key loads up to 16 rows (4 sequences: decode step 3.755 -> 3.617 ms); above, one
+  // iteration's loads at a time (64 sequences: 7.26 ms against 7.37-7.44 pipelined)
+  const bool prefetch = R <= kGemvMaxRows;
+  auto kernel = prefetch ? decode_attention_kernel<true> : decode_attention_kernel<false>;
+  static size_t attr[2] = {0, 0};
+  if (smem > 48 * 1024 && smem > attr[prefetch]) {
+    if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(smem)) != cudaSuccess)
       return -1;
-    attr = smem;
+    attr[prefetch] = smem;
   }
   const cudaError_t e = launch_pdl(
-      decode_attention_kernel, dim3(static_cast<unsigned>(H), static_cast<unsigned>(R)),
+      kernel, dim3(static_cast<unsigned>(H), static_cast<unsigned>(R)),
       dim3(kAttnThreads), smem, st, static_cast<const __nv_bfloat16*>(qkv), static_cast<int>(ld),
       static_cast<int>(d), static_cast<int>(H), static_cast<const float2*>(table),
       static_cast<__nv_bfloat16*>(ck), static_cast<__nv_bfloat16*>(cv), static_cast<int>(P0),
