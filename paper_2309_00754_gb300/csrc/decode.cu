@@ -681,7 +681,8 @@ int launch_decode_attention(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t
   if (R == 0) return 0;
   const size_t smem = decode_attention_smem(Pmax);
   // pipelined key loads up to 16 rows (4 sequences: decode step 3.755 -> 3.617 ms); above, one
-  // iteration's loads at a time (64 sequences: 7.26 ms against 7.37-7.44 pipelined)
+  // iteration's loads at a time (pipelined was slower at 12, 32 and 64 sequences: 4.38 against
+  // 4.18 ms, 5.62 against 5.58 ms, 7.37-7.44 against 7.26 ms)
   const bool prefetch = R <= kGemvMaxRows;
   auto kernel = prefetch ? decode_attention_kernel<true> : decode_attention_kernel<false>;
   static size_t attr[2] = {0, 0};
