@@ -180,6 +180,15 @@ def _stream(stream):
     return s.cuda_stream
 
 
+def _out_dtype(t, name="output"):
+    """HYDRA_BF16 or HYDRA_F32 for an output tensor; any other dtype is refused."""
+    if t.dtype == torch.float32:
+        return HYDRA_F32
+    if t.dtype == torch.bfloat16:
+        return HYDRA_BF16
+    raise ValueError(f"{name} must be torch.bfloat16 or torch.float32, got {t.dtype}")
+
+
 def _req(t, dtype, name):
     if t is None:
         return
@@ -222,7 +231,7 @@ def hydra_lora_linear(x_off, x_on, W, A, B, s, y_off, y_on, workspace=None, algo
     for t, n in ((x_off, "x_off"), (x_on, "x_on"), (W, "W"), (A, "A"), (B, "B")):
         _req(t, torch.bfloat16, n)
     out = y_off if y_off is not None else y_on
-    out_dtype = HYDRA_F32 if out.dtype == torch.float32 else HYDRA_BF16
+    out_dtype = _out_dtype(out)
     for t, n in ((y_off, "y_off"), (y_on, "y_on")):
         _req(t, out.dtype, n)
     M, K = x_off.shape
@@ -239,7 +248,7 @@ def hydra_dual_linear(x_off, x_on, W, u, B, y_off, y_on, algo=0, stream=None):
     for t, n in ((x_off, "x_off"), (x_on, "x_on"), (W, "W"), (u, "u"), (B, "B")):
         _req(t, torch.bfloat16, n)
     out = y_off if y_off is not None else y_on
-    out_dtype = HYDRA_F32 if out.dtype == torch.float32 else HYDRA_BF16
+    out_dtype = _out_dtype(out)
     for t, n in ((y_off, "y_off"), (y_on, "y_on")):
         _req(t, out.dtype, n)
     M, K = x_off.shape
@@ -256,7 +265,7 @@ def hydra_skinny_linear(x, W, y, u=None, B=None, u_row0=0, tile_n=0, split_k=0, 
     the library."""
     for t, n in ((x, "x"), (W, "W"), (u, "u"), (B, "B")):
         _req(t, torch.bfloat16, n)
-    out_dtype = HYDRA_F32 if y.dtype == torch.float32 else HYDRA_BF16
+    out_dtype = _out_dtype(y)
     _req(y, y.dtype, "y")
     M, K = x.shape
     N = W.shape[0]
@@ -273,7 +282,7 @@ def hydra_lora_linear_noalloc(x_off, x_on, W, A, B, s, y_off, y_on, stream=None)
     for t, n in ((x_off, "x_off"), (x_on, "x_on"), (W, "W"), (A, "A"), (B, "B")):
         _req(t, torch.bfloat16, n)
     out = y_off if y_off is not None else y_on
-    out_dtype = HYDRA_F32 if out.dtype == torch.float32 else HYDRA_BF16
+    out_dtype = _out_dtype(out)
     for t, n in ((y_off, "y_off"), (y_on, "y_on")):
         _req(t, out.dtype, n)
     M, K = x_off.shape
@@ -293,7 +302,7 @@ def hydra_dual_linear_ex(x_off, x_on, W, u, B, y_off, y_on, epilogue, stream=Non
     for t, n in ((x_off, "x_off"), (x_on, "x_on"), (W, "W"), (u, "u"), (B, "B")):
         _req(t, torch.bfloat16, n)
     out = y_off if y_off is not None else y_on
-    out_dtype = HYDRA_F32 if out.dtype == torch.float32 else HYDRA_BF16
+    out_dtype = _out_dtype(out)
     for t, n in ((y_off, "y_off"), (y_on, "y_on")):
         _req(t, out.dtype, n)
     M, K = x_off.shape
@@ -339,7 +348,7 @@ def hydra_lora_linear_tri(x_off, x_act, x_crit, W, A_act, B_act, A_crit, B_crit,
                  (A_act, "A_act"), (B_act, "B_act"), (A_crit, "A_crit"), (B_crit, "B_crit")):
         _req(t, torch.bfloat16, n)
     out = next(t for t in (y_off, y_act, y_crit) if t is not None)
-    out_dtype = HYDRA_F32 if out.dtype == torch.float32 else HYDRA_BF16
+    out_dtype = _out_dtype(out)
     for t, n in ((y_off, "y_off"), (y_act, "y_act"), (y_crit, "y_crit")):
         _req(t, out.dtype, n)
     M, K = x_off.shape

@@ -182,3 +182,11 @@ def test_ppo_merge_moments_matches_whole_batch(lib):
     assert H.ppo_merge_moments(torch.zeros(0, 3, dtype=torch.float64)).tolist() == [0.0, 0.0, 0.0]
     with pytest.raises(H.HydraError):
         H.ppo_merge_moments(torch.tensor([[-1.0, 0.0, 0.0]], dtype=torch.float64))
+
+
+def test_binding_refuses_other_output_dtypes():
+    import torch
+    assert H._out_dtype(torch.empty(1, dtype=torch.float32)) == H.HYDRA_F32
+    assert H._out_dtype(torch.empty(1, dtype=torch.bfloat16)) == H.HYDRA_BF16
+    with pytest.raises(ValueError):
+        H._out_dtype(torch.empty(1, dtype=torch.float16))
