@@ -41,15 +41,18 @@ Parity pins for every function live in tests/test_oracle_pins.py (closed forms,
 invariants, brute force, library routines, hand-worked fixtures in tests/golden/).
 `set_storage_dither` (off by default) is a sensitivity probe used to derive the end-to-end
 tolerance of the multi-layer composition; it never changes the default results.
-The full 32-layer Llama composition (`llama_score`, and the three-stream Hydra-PPO pass
-`llama_score_hydra`) is pinned only through its per-op pieces and small-size invariants
-(LoRA off, causality, one LoRA set reducing Hydra-PPO to J-Hydra-PPO, a critic set that
-moves only the values): parity unpinned for the composition as a whole.
+The Llama composition (`llama_final_hidden`, under `llama_score` and the three-stream
+Hydra-PPO pass `llama_score_hydra`) is pinned, with the bf16 storage rounding switched off,
+against the same architecture built from PyTorch library operations in fp64 (F.linear,
+F.rms_norm, causal F.scaled_dot_product_attention, F.silu, rotary as a complex rotation);
+and through its per-op pieces and invariants (LoRA off, causality, one LoRA set reducing
+Hydra-PPO to J-Hydra-PPO, a critic set that moves only the values). Where it rounds to bf16
+(the tensors the GPU stores as bf16) is a reading, not pinned by that comparison.
 Generation (`llama_generate`, the sampling phase of Alg. 1 and 2) recomputes
 the whole stack at every step, with no cache, and draws each token by the Gumbel-max trick
 from noise that is an input (`gumbel_argmax`, pinned by the empirical distribution of its
-draws). It is pinned by its equality with `llama_score` on the finished sequence, so it
-inherits that composition's "parity unpinned".
+draws). It is pinned by its equality with `llama_score` on the finished sequence, and
+through it by the library forward above.
 """
 from __future__ import annotations
 

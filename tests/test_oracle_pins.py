@@ -557,3 +557,64 @@ def test_generate_lora_off_streams_agree():
     prompt = np.random.default_rng(24).integers(0, 64, size=3)
     gen = O.llama_generate(w, prompt, 4, cfg)
     np.testing.assert_array_equal(gen["logp_actor"], gen["logp_ref"])
+
+
+def _torch_final_hidden(w, ids, cfg):
+    """The decoder stack written with PyTorch library operations in fp64: F.linear,
+    F.rms_norm, the causal F.scaled_dot_product_attention, F.silu, and the rotary
+    embedding as a complex rotation of the pairs (i, i + D/2). LoRA on wq/wv/wg/wu/wd of the
+    LoRA-on stream only."""
+    import torch
+    import torch.nn.functional as F
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a, dtype=np.float64))  # noqa: E731
+    d, H, eps, s = cfg["d"], cfg["n_heads"], cfg["eps"], cfg["lora_scale"]
+    Dh, T = d // H, len(ids)
+    inv = cfg["rope_theta"] ** (-torch.arange(Dh // 2, dtype=torch.float64) * 2.0 / Dh)
+    ang = torch.arange(T, dtype=torch.float64)[:, None] * inv[None, :]
+    rot = torch.polar(torch.ones_like(ang), ang)[:, None, :]  # [T, 1, Dh/2]
+
+    def rope(x):
+        z = torch.complex(x[..., :Dh // 2], x[..., Dh // 2:]) * rot
+        return torch.cat([z.real, z.imag], dim=-1)
+
+    def lin(x, name, l, on):
+        y = F.linear(x, t(w[name][l]))
+        if on and name in w["lora"]:
+            A, B = w["lora"][name]
+            y = y + s * F.linear(F.linear(x, t(A[l])), t(B[l]))
+        return y
+
+    outs = []
+    for on in (False, True):
+        h = t(w["embed"])[torch.as_tensor(np.asarray(ids))]
+        for l in range(cfg["n_layers"]):
+            a = F.rms_norm(h, (d,), weight=t(w["norm1"][l]), eps=eps)
+            q = rope(lin(a, "wq", l, on).view(T, H, Dh)).transpose(0, 1)
+            k = rope(lin(a, "wk", l, on).view(T, H, Dh)).transpose(0, 1)
+            v = lin(a, "wv", l, on).view(T, H, Dh).transpose(0, 1)
+            att = F.scaled_dot_product_attention(q, k, v, is_causal=True).transpose(0, 1).reshape(T, d)
+            h = h + lin(att, "wo", l, on)
+            a = F.rms_norm(h, (d,), weight=t(w["norm2"][l]), eps=eps)
+            h = h + lin(F.silu(lin(a, "wg", l, on)) * lin(a, "wu", l, on), "wd", l, on)
+        outs.append(F.rms_norm(h, (d,), weight=t(w["final_norm"]), eps=eps).numpy())
+    return outs
+
+
+def test_llama_composition_matches_a_library_forward(monkeypatch):
+    """The whole decoder stack (embedding, RMSNorm, rotary q/k, causal attention, residuals,
+    SwiGLU, LoRA on the on stream, final norm) against the same architecture built from
+    PyTorch's library operations. The bf16 storage rounding is switched off in the oracle
+    for this comparison, so both sides are exact fp64 compositions."""
+    pytest.importorskip("torch")
+    w, cfg = tiny_llama(seed=31, n_layers=3, d=32, H=4, F=48, V=64, r=4)
+    rng = np.random.default_rng(32)
+    w["norm1"] = 0.5 + rng.random(w["norm1"].shape)
+    w["norm2"] = 0.5 + rng.random(w["norm2"].shape)
+    w["final_norm"] = 0.5 + rng.random(w["final_norm"].shape)
+    ids = rng.integers(0, 64, size=13)
+    ref_off, ref_on = _torch_final_hidden(w, ids, cfg)
+    monkeypatch.setattr(O.hydra_oracle, "round_bf16", lambda x: np.asarray(x, dtype=np.float64))
+    f_off, f_on = O.llama_final_hidden(w, ids, cfg)
+    np.testing.assert_allclose(f_off, ref_off, rtol=1e-9, atol=1e-10)
+    np.testing.assert_allclose(f_on, ref_on, rtol=1e-9, atol=1e-10)
+    assert not np.allclose(f_off, f_on)  # the LoRA term reaches the on stream
