@@ -618,3 +618,23 @@ def test_llama_composition_matches_a_library_forward(monkeypatch):
     np.testing.assert_allclose(f_off, ref_off, rtol=1e-9, atol=1e-10)
     np.testing.assert_allclose(f_on, ref_on, rtol=1e-9, atol=1e-10)
     assert not np.allclose(f_off, f_on)  # the LoRA term reaches the on stream
+
+
+def test_hydra_three_stream_composition_matches_a_library_forward(monkeypatch):
+    """The three-stream stack of the Hydra-PPO oracle (LoRA off, the actor's set, the critic's
+    set) against the library forward of each stream, bf16 storage rounding switched off."""
+    pytest.importorskip("torch")
+    w, cfg = tiny_llama(seed=41, n_layers=2, d=32, H=4, F=48, V=64, r=4)
+    wc, _ = tiny_llama(seed=42, n_layers=2, d=32, H=4, F=48, V=64, r=4)
+    rng = np.random.default_rng(43)
+    w["norm1"] = 0.5 + rng.random(w["norm1"].shape)
+    w["norm2"] = 0.5 + rng.random(w["norm2"].shape)
+    w["final_norm"] = 0.5 + rng.random(w["final_norm"].shape)
+    ids = rng.integers(0, 64, size=11)
+    ref_off, ref_act = _torch_final_hidden(w, ids, cfg)
+    _, ref_crit = _torch_final_hidden(dict(w, lora=wc["lora"]), ids, cfg)
+    monkeypatch.setattr(O.hydra_oracle, "round_bf16", lambda x: np.asarray(x, dtype=np.float64))
+    out = O.llama_score_hydra(w, wc["lora"], ids, 4, cfg)
+    np.testing.assert_allclose(out["h_off"], ref_off, rtol=1e-9, atol=1e-10)
+    np.testing.assert_allclose(out["h_act"], ref_act, rtol=1e-9, atol=1e-10)
+    np.testing.assert_allclose(out["h_crit"], ref_crit, rtol=1e-9, atol=1e-10)
