@@ -52,9 +52,33 @@ def load_peaks():
         with open(p) as f:
             d = json.load(f)
         return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
-                "bf16_tflops_sustained": d["bf16_tflops_sustained"], "source": "measured"}
+                "bf16_tflops_sustained": d["bf16_tflops_sustained"], "source": "measured",
+                "sustained_sm_mhz": d.get("clocks_under_load", {}).get("sm_mhz_median")}
     return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
-            "source": "fallback"}
+            "source": "fallback", "sustained_sm_mhz": None}
+
+
+# nominal dense peaks of one GB300 (datasheet), reported beside the measured denominators
+NOMINAL = {"TFLOP/s": 2250.0, "GB/s": 7900.0}
+
+
+def annotate_roofline(roof, peaks, clk):
+    """Secondary fractions beside the measured-peak one: against the nominal dense peak, and
+    (tensor-bound, sustained peak) with both sides normalised by their median SM clock, since
+    the measured sustained peak ran at a lower clock than the pass may."""
+    if not roof or roof.get("achieved") is None:
+        return roof
+    nominal = NOMINAL.get(roof.get("unit"))
+    if nominal:
+        roof["frac_of_nominal"] = roof["achieved"] / nominal
+        roof["nominal_peak"] = nominal
+    mhz, peak_mhz = (clk or {}).get("sm_mhz"), peaks.get("sustained_sm_mhz")
+    if (roof.get("bound") == "tensor" and "sustained" in roof.get("peak_kind", "") and mhz
+            and peak_mhz):
+        roof["frac_clock_normalised"] = (roof["achieved"] / mhz) / (roof["peak"] / peak_mhz)
+        roof["clock_note"] = (f"pass median {mhz:.0f} MHz, measured sustained peak taken at "
+                              f"median {peak_mhz:.0f} MHz")
+    return roof
 
 
 # ----------------------------------------------------------------------------- clocks
@@ -348,7 +372,10 @@ class HydraScoringLlama7B:
                 "frac": achieved / peak, "traffic": self.traffic_per_launch(),
                 "peak_kind": f"bf16 dense, {peaks['source']} sustained",
                 "per_launch_flop": self.gemm_flops / sum(self.launch_counts[k] for k in self.class_flops),
-                "per_launch_ms": ms / n}
+                "per_launch_ms": ms / n,
+                "timing": "CUDA events around every launch on the library's stream, over a second "
+                          "run of the same steps right after the timed region",
+                "profiled_ms_per_step": getattr(self, "profiled_ms_per_step", None)}
 
     def config(self):
         return {"workload": f"{self.name}: random-init Llama-7B (32 layers, d 4096, 32 heads, "
@@ -405,12 +432,15 @@ class HydraScoringLlama7B:
                       beta=self.beta, gamma=self.gamma, lam=self.lam)
         return time.perf_counter() - t0
 
-    def oracle_throughput(self, steps=1, single_thread=False):
+    def oracle_throughput(self, steps=1, single_thread=False, warmup=0):
         """(tokens/s, description): the slice's pass time is t(0 layers) + 32 (t(1) - t(0)); a
         quarter-size slice on one BLAS thread."""
         smp = self.oracle_sample(1, prompt=16, resp=32) if single_thread else self.oracle_sample(1)
+        for _ in range(warmup):
+            self.oracle_time(smp, 1)
         t_head = self.oracle_time(smp, 0)
         t1 = [self.oracle_time(smp, 1) for _ in range(steps)]
+        self.oracle_timed = {"head_s": t_head, "sample_s": t1}
         n = self.cfg["n_layers"]
         t_pass = [t_head + n * max(t - t_head, 0.0) for t in t1]
         desc = (f"one sequence slice of {smp['prompt']} prompt + {smp['resp']} response tokens at full "
@@ -616,12 +646,15 @@ class HydraGenerateLlama7B(HydraScoringLlama7B):
         O.llama_generate(smp["w"], smp["ids"][:smp["prompt"]], 2, smp["cfg"], n_layers=n_layers)
         return time.perf_counter() - t0
 
-    def oracle_throughput(self, steps=1, single_thread=False):
+    def oracle_throughput(self, steps=1, single_thread=False, warmup=0):
         """(tokens/s, description): 2 draws after a 32-token prompt, per-draw time t(0 layers)
         + 32 (t(1) - t(0)), the oracle recomputing the whole prefix at each draw."""
         smp = self.oracle_sample(1)
+        for _ in range(warmup):
+            self.oracle_time(smp, 1)
         t_head = self.oracle_time(smp, 0)
         t1 = [self.oracle_time(smp, 1) for _ in range(steps)]
+        self.oracle_timed = {"head_s": t_head, "sample_s": t1}
         n = self.cfg["n_layers"]
         t_gen = [t_head + n * max(t - t_head, 0.0) for t in t1]
         desc = (f"one sequence, {smp['prompt']} prompt tokens, 2 draws (plus the score pass) at full "
@@ -751,10 +784,13 @@ class HydraPPOIterationLlama7B(HydraGenerateLlama7B):
                    sc["returns"][None], sc["values"][None], [2], whiten=True)
         return time.perf_counter() - t0
 
-    def oracle_throughput(self, steps=1, single_thread=False):
+    def oracle_throughput(self, steps=1, single_thread=False, warmup=0):
         smp = self.oracle_sample(1)
+        for _ in range(warmup):
+            self.oracle_time(smp, 1)
         t_head = self.oracle_time(smp, 0)
         t1 = [self.oracle_time(smp, 1) for _ in range(steps)]
+        self.oracle_timed = {"head_s": t_head, "sample_s": t1}
         n = self.cfg["n_layers"]
         t_it = [t_head + n * max(t - t_head, 0.0) for t in t1]
         desc = (f"one sequence, {smp['prompt']} prompt tokens, 2 draws, three-stream scoring of the "
@@ -1093,12 +1129,22 @@ def run_reference(args, wl_cls):
     cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
     if hasattr(wl_cls, "oracle_throughput"):
         wl = wl_cls(dev, reference=True)
-        value, desc = wl.oracle_throughput(steps=args.steps)
-        t_step = wl.units / value
+        value, desc = wl.oracle_throughput(steps=args.steps, warmup=args.warmup)
+        timed = wl.oracle_timed
+        # a step here is one timed oracle sample (the slice through embed, one decoder layer
+        # and the heads); value is that sample extrapolated to the full pass, stated apart
+        sample_ms = 1e3 * statistics.mean(timed["sample_s"])
         line = {"metric": getattr(wl, "metric", METRIC), "value": value, "unit": UNIT, "n_gpus": args.gpus,
-                "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_step * 1e3,
+                "steps": len(timed["sample_s"]), "warmup": args.warmup, "ms_per_step": sample_ms,
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
                 "data": "synthetic", "impl": "reference", "config": wl.config(),
+                "extrapolated_from": {
+                    "step": "one oracle sample: the slice through embed, one decoder layer and "
+                            "the heads", "sample_ms": [1e3 * t for t in timed["sample_s"]],
+                    "head_only_ms": 1e3 * timed["head_s"],
+                    "full_pass_ms_extrapolated": 1e3 * wl.units / value,
+                    "rule": "t(head) + n_layers x (t(sample) - t(head)), per full step of "
+                            f"{wl.units} units"},
                 "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
                                  "sample": desc},
                 "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
@@ -1181,11 +1227,13 @@ def run_ours(args, wl_cls):
     names = getattr(wl, "event_names", ())
     evs = [None] * steps
     if driver:
-        # launch counts of one pass, then event timing of every launch of the timed steps
+        # launch counts of one pass (per-launch events on); the timed steps run without them
         H.profile_enable(True)
         wl.step()
         wl.launch_counts = {k: n for k, (_, n) in H.profile_collect(reset=True).items()}
         wl.launches_per_step = sum(wl.launch_counts.values())
+        H.profile_enable(False)
+        torch.cuda.synchronize()
     else:
         evs = [{n: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                 for n in names} for _ in range(steps)]
@@ -1205,8 +1253,20 @@ def run_ours(args, wl_cls):
     ms_total = start.elapsed_time(end)
     ms_total_max = max_over_ranks(ms_total, world, device)
     if driver:
+        # per-kernel breakdown: the same K steps again, every launch bracketed by CUDA events
+        # on the library's stream (kept out of the timed region above)
+        H.profile_enable(True)
+        torch.cuda.synchronize()
+        p0 = torch.cuda.Event(enable_timing=True)
+        p1 = torch.cuda.Event(enable_timing=True)
+        p0.record()
+        for i in range(steps):
+            wl.step()
+        p1.record()
+        torch.cuda.synchronize()
         per_kernel = H.profile_collect(reset=True)
         H.profile_enable(False)
+        wl.profiled_ms_per_step = p0.elapsed_time(p1) / steps
     else:
         per_kernel = {n: statistics.mean(e[n][0].elapsed_time(e[n][1]) for e in evs) for n in names}
     if H.device_error(clear=True) != 0:
@@ -1238,7 +1298,7 @@ def run_ours(args, wl_cls):
         "warmup": warmup, "ms_per_step": ms_total_max / steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": dict(wl.config(), parallelism=f"replicas{world}" if world > 1 else "single"),
-        "roofline": wl.roofline(peaks, per_kernel),
+        "roofline": annotate_roofline(wl.roofline(peaks, per_kernel), peaks, clk),
         "kernels": wl.kernels(peaks, per_kernel),
         "clocks": clk,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": wl.h2d,

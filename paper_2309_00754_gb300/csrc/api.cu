@@ -3,6 +3,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <mutex>
+
 #include "../../include/hydra.h"
 #include "common.cuh"
 #include "kernels.h"
@@ -14,6 +16,7 @@ __device__ int g_hydra_err = 0;
 
 constexpr int kMaxDevices = 64;
 int* g_err_ptr[kMaxDevices] = {nullptr};
+std::mutex g_err_ptr_mutex;  // guards the first fill of g_err_ptr from concurrent host threads
 
 }  // namespace
 
@@ -23,6 +26,7 @@ namespace hydra {
 int* device_error_word() {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  std::lock_guard<std::mutex> lock(g_err_ptr_mutex);
   if (g_err_ptr[dev] == nullptr) {
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_hydra_err) != cudaSuccess) return nullptr;

@@ -4,8 +4,10 @@ pool, or a latency-critical caller that cannot afford cudaMalloc/cudaFree). It k
 LoRA down-projection u in the library's static device array instead of a workspace.
 
 The test calls it through the C-ABI twice in a row (the two calls share that array) and
-checks both results against the workspace entry point. The file name makes pytest collect
-it last, so a run that stops at the first failure has already run every other test."""
+checks both results against the workspace entry point. Both entry points run the same
+kernels on the same u, so the outputs must agree bit for bit. The file name makes pytest
+collect it last, so a run that stops at the first failure has already run every other
+test."""
 import numpy as np
 import pytest
 import torch
@@ -13,7 +15,7 @@ import torch
 from paper_2309_00754_gb300 import build as Bld
 from paper_2309_00754_gb300 import hydra as H
 from paper_2309_00754_gb300 import synth
-from tests.helpers import TOL_LINEAR, assert_rel, dev_bf16, host_f64
+from tests.helpers import dev_bf16, host_f64
 
 pytestmark = pytest.mark.gpu
 
@@ -57,9 +59,31 @@ def test_noalloc_matches_workspace_entry_point_on_two_calls():
         ref_off, ref_on = _outputs(M, N)
         ws = torch.empty(H.lora_linear_workspace_size(M, r), dtype=torch.uint8, device="cuda")
         H.hydra_lora_linear(x, x_on, W, A, B, 2.0, ref_off, ref_on, ws)
-        assert_rel(host_f64(y_off), host_f64(ref_off), TOL_LINEAR, "y_off")
-        assert_rel(host_f64(y_on), host_f64(ref_on), TOL_LINEAR, "y_on")
+        assert torch.equal(y_off, ref_off), "y_off differs from the workspace entry point"
+        assert torch.equal(y_on, ref_on), "y_on differs from the workspace entry point"
         assert np.all(np.isfinite(host_f64(y_on)))
+
+
+def test_noalloc_without_lora_matches_and_allocates_nothing():
+    # r = 0: no u at all, the plain dual linear; then a warm call with LoRA must leave the
+    # device's free memory where it was (the array was reserved when the library loaded)
+    M, K, N = 96, 512, 264
+    x, x_on, W, A, B = _problem(M, K, N, 16, 7300, False)
+    y_off, y_on = _outputs(M, N)
+    H.hydra_lora_linear_noalloc(x, x_on, W, None, None, 2.0, y_off, y_on)
+    ref_off, ref_on = _outputs(M, N)
+    H.hydra_lora_linear(x, x_on, W, None, None, 2.0, ref_off, ref_on, None)
+    torch.cuda.synchronize()
+    assert torch.equal(y_off, ref_off) and torch.equal(y_on, ref_on)
+
+    H.hydra_lora_linear_noalloc(x, x_on, W, A, B, 2.0, y_off, y_on)  # warm: set-up done
+    torch.cuda.synchronize()
+    free_before, _ = torch.cuda.mem_get_info()
+    for _ in range(3):
+        H.hydra_lora_linear_noalloc(x, x_on, W, A, B, 2.0, y_off, y_on)
+    torch.cuda.synchronize()
+    free_after, _ = torch.cuda.mem_get_info()
+    assert free_after == free_before, f"free device memory moved by {free_before - free_after} B"
 
 
 def test_noalloc_rejects_u_beyond_the_static_array():
