@@ -199,8 +199,10 @@ def check_pass(cfg, got, w64, ids, lengths, derive_tol=False):
                              abs(alt["score"] - ref["score"]))
             tol_lp = max(TOL_LOGP, 3 * spread_lp)
             tol_lin = max(TOL_LINEAR, 3 * spread_lin)
-            print(f"seq {s}: chain spread logp {spread_lp:.2e}, head {spread_lin:.2e} "
-                  f"-> tolerances {tol_lp:.2e}, {tol_lin:.2e}")
+            mean_lp = lambda a, b: float(np.mean(np.abs(np.asarray(a)[:n] - np.asarray(b)[:n])))  # noqa: E731
+            print(f"seq {s}: chain spread logp {spread_lp:.2e} (mean {mean_lp(alt['logp_actor'], ref['logp_actor']):.2e}), "
+                  f"head {spread_lin:.2e} -> tolerances {tol_lp:.2e}, {tol_lin:.2e}; GPU mean logp "
+                  f"error {mean_lp(got['logp_actor'][s], ref['logp_actor']):.2e}")
             print(f"seq {s}: GPU error logp actor {max_abs_err(got['logp_actor'][s], ref['logp_actor']):.2e}"
                   f", ref {max_abs_err(got['logp_ref'][s], ref['logp_ref']):.2e}, values "
                   f"{max_abs_err(got['values'][s], ref['values']):.2e}, score "
