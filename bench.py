@@ -814,7 +814,8 @@ class KernelSweep:
       GAE: 65536 sequences x 512 tokens -> GB/s;
       PPO losses (clipped surrogate, value loss, gradients, whitening): the same batch -> GB/s;
       causal attention: 8 sequences x 768 tokens x 32 heads of 128 -> TFLOP/s;
-      log-probs/KL: 2048 rows x 32000 fp32 logits x 2 heads -> GB/s."""
+      log-probs/KL: 2048 rows x 32000 fp32 logits x 2 heads -> GB/s;
+      LoRA down-projection: the full pass's and the LM head's shapes -> GB/s."""
 
     name = "kernel_sweep"
     seed = 5
@@ -825,7 +826,7 @@ class KernelSweep:
         self.device = device
 
     PARTS = ("projection_sweep", "decode", "decode_batch", "gae", "ppo_loss", "attention",
-             "logprobs")
+             "logprobs", "lora_down")
 
     def run(self, peaks, reps=20, parts=PARTS):
         import torch
@@ -994,6 +995,21 @@ class KernelSweep:
             ms = graph_ms(lambda i: H.hydra_token_logprobs_kl(za, zr, ids, None, None, 0.1, 4, 512, *o3), reps)
             byts = T * V * 4 * 2 + T * 16
             out["logprobs"] = {"ms": ms, "GB/s": byts / ms / 1e6, "frac_of_measured_hbm": byts / ms / 1e6 / peaks["hbm_gbs"]}
+        # ---- LoRA down-projection at the full pass's shapes (3072 on-stream rows: q/v and
+        # gate/up at K 4096 with 2 x 16 ranks, down at K 11008 with 16) and the LM-head
+        # workload's (2048 x 4096, r 16); x rotates through copies beyond L2
+        if "lora_down" in parts:
+            for n, Mt, K, r in (("qv_gu", 3072, 4096, 32), ("down", 3072, 11008, 16),
+                                ("lm_head", 2048, 4096, 16)):
+                ncopy = max(2, -(-300_000_000 // (Mt * K * 2)))
+                xs = [torch.randn(Mt, K, device=dev, generator=g).to(bf) for _ in range(ncopy)]
+                A = rnd(r, K)
+                u = torch.empty(Mt, r, dtype=bf, device=dev)
+                ms = graph_ms(lambda i: H.hydra_lora_down(xs[i % ncopy], A, 2.0, u), max(reps, 2 * ncopy))
+                byts = 2.0 * (Mt * K + r * K + Mt * r)
+                out["lora_down"][n] = {"ms": ms, "GB/s": byts / ms / 1e6,
+                                       "frac_of_measured_hbm": byts / ms / 1e6 / peaks["hbm_gbs"]}
+                del xs
         return out
 
 

@@ -151,6 +151,249 @@ cudaError_t launch_down(void (*kernel)(KArgs...), dim3 grid, int ck, cudaStream_
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
 
+// ---------------------------------------------------------------- lora_down, streaming form
+//
+// For 64 token rows and more, x is streamed once from HBM by TMA. A thread-block cluster of
+// ck CTAs (1, 2, 4 or 8) takes a block of 64 rows and up to 64 ranks and splits K into ck
+// contiguous ranges of 64-wide k-blocks. In each CTA one producer warp moves [64 rows x 64 k]
+// tiles of x and [8 NT ranks x 64 k] tiles of A through a 6-stage ring (128-byte swizzle);
+// each of four consumer warps takes one 16-wide k-step of every stage over all 64 rows
+// (ldmatrix, then mma.sync m16n8k16 with fp32 accumulation), so every byte staged in shared
+// memory is read once and the arithmetic never holds the stream back. The warps' partial
+// [64 x 8 NT] tiles are summed in shared memory in warp order; CTA q finishes rows
+// [q 64 / ck, (q + 1) 64 / ck) of the block: every CTA pushes its sums of those rows into
+// q's receive buffer with stores to distributed shared memory, one cluster barrier makes them
+// visible, and q adds the ck slices in rank order, so the result does not depend on timing
+// (a pull through remote loads cost about 2 us more per launch: each remote load waits a
+// full round trip). All CTAs of a launch fit on the GPU at once (2-4 per SM), so every load
+// of x is issued at the start and the launch costs about one pass over x at HBM speed plus
+// the reduction.
+namespace lds {
+
+constexpr int kBM = 64;          // token rows per CTA
+constexpr int kConsumers = 4;    // consumer warps; warp kConsumers is the producer
+constexpr int kThreads = 32 * (kConsumers + 1);
+constexpr int kXTile = kBM * 128;  // [64 rows x 64 bf16], 8 KiB
+
+template <int NT>  // NT n-tiles of 8 ranks (1, 2, 4 or 8)
+struct Cfg {
+  // ring depth: as deep as still lets three CTAs share an SM (two at 64 ranks)
+  static constexpr int kStages = NT <= 2 ? 6 : 5;
+  static constexpr int kATile = 8 * NT * 128;
+  static constexpr int kStage = kXTile + kATile;  // a multiple of 1024: tiles stay aligned
+  static constexpr int kRing = kStages * kStage;
+  static constexpr int kLd = 8 * NT + 4;          // fp32 row stride of the partial tiles
+  static constexpr int kPart = kBM * kLd * 4;
+  static_assert(kConsumers * kPart <= kRing, "partial tiles reuse the ring");
+  // receive buffer [ck][64 / ck][8 NT] fp32: the cluster's sums of this CTA's rows; outside
+  // the ring, since other CTAs may write it while this one still streams
+  static constexpr int kRecvOff = kRing;
+  static constexpr int kBarOff = kRecvOff + kBM * 8 * NT * 4;
+  static constexpr int kSmem = 1024 + kBarOff + 2 * kStages * 8 + 16;
+};
+
+__device__ __forceinline__ void st_cluster_v4(const float* local, uint32_t rank, float4 v) {
+  uint32_t raddr;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(raddr) : "r"(smem_u32(local)), "r"(rank));
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(raddr), "f"(v.x), "f"(v.y),
+               "f"(v.z), "f"(v.w)
+               : "memory");
+}
+
+__device__ __forceinline__ void store_u4(__nv_bfloat16* u, int r, int m, int nn, float s, float4 v) {
+  uint2 o;
+  o.x = pack_bf16x2(s * v.x, s * v.y);
+  o.y = pack_bf16x2(s * v.z, s * v.w);
+  *reinterpret_cast<uint2*>(u + static_cast<size_t>(m) * r + nn) = o;
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t (&a)[4]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(a[0]), "=r"(a[1]), "=r"(a[2]), "=r"(a[3])
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x2(uint32_t addr, uint32_t (&a)[2]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0,%1}, [%2];"
+               : "=r"(a[0]), "=r"(a[1])
+               : "r"(addr));
+}
+// byte offset of 16-byte chunk `chunk` of row `row` in a 128-byte-swizzled tile
+__device__ __forceinline__ uint32_t sw128(int row, int chunk) {
+  return static_cast<uint32_t>(row * 128 + ((chunk ^ (row & 7)) << 4));
+}
+
+template <int NT>
+__global__ void __launch_bounds__(kThreads)
+    lora_down_stream_kernel(const __grid_constant__ CUtensorMap tm_x,
+                            const __grid_constant__ CUtensorMap tm_a, int M, int K, int r, float s,
+                            __nv_bfloat16* __restrict__ u, int ck, int* err) {
+  using C = Cfg<NT>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::kBarOff);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(bars + 2 * C::kStages);
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t sbase = smem_u32(smem);
+  auto full = [&](int i) { return smem_u32(&bars[i]); };
+  auto empty = [&](int i) { return smem_u32(&bars[C::kStages + i]); };
+
+  const uint32_t rank = ck > 1 ? cluster_rank() : 0u;
+  const int row0 = static_cast<int>(blockIdx.x / ck) * kBM;
+  const int n_base = static_cast<int>(blockIdx.y) * 64;
+  const int nkb = (K + 63) / 64;
+  const int kb0 = static_cast<int>((static_cast<int64_t>(nkb) * rank) / ck);
+  const int kb1 = static_cast<int>((static_cast<int64_t>(nkb) * (rank + 1)) / ck);
+  const int n = kb1 - kb0;  // this CTA's k-blocks (may be 0)
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < C::kStages; ++i) {
+      mbar_init(full(i), 1);
+      mbar_init(empty(i), kConsumers);
+    }
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  // first half of a cluster barrier: its wait, before the first store to another CTA's shared
+  // memory, ensures every CTA of the cluster has started
+  if (ck > 1) asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+  pdl_launch_dependents();
+  pdl_wait();  // x is written by the preceding kernel, which may also still read u
+
+  float d[4][NT][4];
+#pragma unroll
+  for (int mt = 0; mt < 4; ++mt)
+#pragma unroll
+    for (int t = 0; t < NT; ++t) d[mt][t][0] = d[mt][t][1] = d[mt][t][2] = d[mt][t][3] = 0.f;
+
+  if (warp == kConsumers) {
+    // ---------------------------------------------------------------- producer
+    if (elect_one()) {
+      tma_prefetch_desc(&tm_x);
+      tma_prefetch_desc(&tm_a);
+    }
+    __syncwarp();
+    int i = 0;
+    for (; i < n; ++i) {
+      const int st = i % C::kStages;
+      if (i >= C::kStages && !warp_wait_bounded(empty(st), ((i / C::kStages) - 1) & 1, abort_flag, err,
+                                             kDevTimeoutProducer))
+        break;
+      if (elect_one()) {
+        const uint32_t dst = sbase + st * C::kStage;
+        const int k = (kb0 + i) * 64;
+        mbar_arrive_expect_tx(full(st), C::kStage);
+        tma_load_2d(dst, &tm_x, k, row0, full(st));
+        tma_load_2d(dst + kXTile, &tm_a, k, n_base, full(st));
+      }
+      __syncwarp();
+    }
+    // copies in flight land before the shared memory is reused or released
+    volatile int no_abort = 0;
+    for (int g = (i > C::kStages ? i - C::kStages : 0); g < i; ++g)
+      warp_wait_bounded(full(g % C::kStages), (g / C::kStages) & 1, &no_abort, err, kDevTimeoutDrain);
+  } else {
+    // ---------------------------------------------------------------- consumers
+    for (int i = 0; i < n; ++i) {
+      const int st = i % C::kStages;
+      if (!warp_wait_bounded(full(st), (i / C::kStages) & 1, abort_flag, err, kDevTimeoutEpilogue))
+        break;
+      const uint32_t xs = sbase + st * C::kStage;
+      const uint32_t as = xs + kXTile;
+      uint32_t a[4][4];
+#pragma unroll
+      for (int mt = 0; mt < 4; ++mt) {
+        const int row = mt * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+        ldsm_x4(xs + sw128(row, 2 * warp + (lane >> 4)), a[mt]);
+      }
+      if constexpr (NT == 1) {
+        uint32_t b[2];
+        const int nrow = lane & 7;
+        ldsm_x2(as + sw128(nrow, 2 * warp + ((lane >> 3) & 1)), b);
+#pragma unroll
+        for (int mt = 0; mt < 4; ++mt) mma_bf16_16816(d[mt][0], a[mt], b[0], b[1]);
+      } else {
+#pragma unroll
+        for (int tp = 0; tp < NT / 2; ++tp) {
+          uint32_t b[4];
+          const int nrow = 8 * (2 * tp + (lane >> 4)) + (lane & 7);
+          ldsm_x4(as + sw128(nrow, 2 * warp + ((lane >> 3) & 1)), b);
+#pragma unroll
+          for (int mt = 0; mt < 4; ++mt) {
+            mma_bf16_16816(d[mt][2 * tp], a[mt], b[0], b[1]);
+            mma_bf16_16816(d[mt][2 * tp + 1], a[mt], b[2], b[3]);
+          }
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(empty(st));
+    }
+  }
+  __syncthreads();  // every stage is consumed and no copy is in flight: the ring is free
+
+  // partial tiles of the consumer warps, summed in warp order
+  float* part = reinterpret_cast<float*>(smem);
+  float* recv = reinterpret_cast<float*>(smem + C::kRecvOff);
+  if (warp < kConsumers) {
+    float* pw = part + warp * (kBM * C::kLd);
+    const int g = lane >> 2, c = lane & 3;
+#pragma unroll
+    for (int mt = 0; mt < 4; ++mt)
+#pragma unroll
+      for (int t = 0; t < NT; ++t) {
+        *reinterpret_cast<float2*>(pw + (mt * 16 + g) * C::kLd + t * 8 + 2 * c) =
+            make_float2(d[mt][t][0], d[mt][t][1]);
+        *reinterpret_cast<float2*>(pw + (mt * 16 + g + 8) * C::kLd + t * 8 + 2 * c) =
+            make_float2(d[mt][t][2], d[mt][t][3]);
+      }
+  }
+  __syncthreads();
+  if (ck > 1) asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
+  const int rows_per = kBM / ck;
+  constexpr int kQ = 2 * NT;  // float4 groups per row
+  for (int e = threadIdx.x; e < kBM * kQ; e += kThreads) {
+    const int rr = e / kQ, cc = (e % kQ) * 4;
+    float4 v = *reinterpret_cast<const float4*>(part + rr * C::kLd + cc);
+#pragma unroll
+    for (int w = 1; w < kConsumers; ++w) {
+      const float4 p = *reinterpret_cast<const float4*>(part + w * (kBM * C::kLd) + rr * C::kLd + cc);
+      v.x += p.x;
+      v.y += p.y;
+      v.z += p.z;
+      v.w += p.w;
+    }
+    if (ck > 1) {
+      // row rr is finished by rank rr / rows_per, into its slot for this rank
+      const int dst = rr / rows_per, lr = rr % rows_per;
+      st_cluster_v4(recv + ((static_cast<int>(rank) * rows_per + lr) * 8 * NT + cc),
+                    static_cast<uint32_t>(dst), v);
+    } else {
+      const int m = row0 + rr, nn = n_base + cc;
+      if (m < M && nn < r) store_u4(u, r, m, nn, s, v);
+    }
+  }
+  if (ck > 1) {
+    cluster_sync_all();  // every CTA's pushes have landed and are visible
+    for (int e = threadIdx.x; e < rows_per * kQ; e += kThreads) {
+      const int lr = e / kQ, cc = (e % kQ) * 4;
+      float4 v = *reinterpret_cast<const float4*>(recv + lr * 8 * NT + cc);
+      for (int q = 1; q < ck; ++q) {
+        const float4 p = *reinterpret_cast<const float4*>(recv + ((q * rows_per + lr) * 8 * NT + cc));
+        v.x += p.x;
+        v.y += p.y;
+        v.z += p.z;
+        v.w += p.w;
+      }
+      const int m = row0 + static_cast<int>(rank) * rows_per + lr, nn = n_base + cc;
+      if (m < M && nn < r) store_u4(u, r, m, nn, s, v);
+    }
+  }
+}
+
+}  // namespace lds
+
 // ---------------------------------------------------------------- dual_lora_gemv
 //
 // Decode-shaped dual-output linear (at most 16 token rows over both streams). HBM-bound:
@@ -372,6 +615,52 @@ void launch_gemv_t(const GemmArgs& a, cudaStream_t stream) {
       static_cast<int>(a.r), a.y_off, a.y_on, a.out_f32, a.shared_x ? 1 : 0);
 }
 
+// Streaming lora_down: clusters of ck CTAs (a power of two up to 8) along K, ck as large as
+// still lets every CTA of the launch be resident at once, and at least one k-block per CTA.
+template <int NT>
+int launch_lora_down_stream(const void* x, int64_t M, int64_t K, const void* A, int64_t r,
+                            float s, void* u, int nsm, cudaStream_t stream) {
+  using C = lds::Cfg<NT>;
+  static bool attr = false;
+  if (!attr) {
+    if (cudaFuncSetAttribute(lds::lora_down_stream_kernel<NT>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmem) != cudaSuccess)
+      return -1;
+    attr = true;
+  }
+  int* err = device_error_word();
+  if (err == nullptr) return -1;
+  CUtensorMap mx, ma;
+  if (!make_tma_map(&mx, x, M, K, K, lds::kBM, false)) return -2;
+  if (!make_tma_map(&ma, A, r, K, K, 8 * NT, false)) return -2;
+  const int64_t rb = (M + lds::kBM - 1) / lds::kBM;
+  const int64_t ny = (r + 63) / 64;
+  const int64_t per_sm = std::max<int64_t>(1, (227 * 1024) / C::kSmem);
+  const int64_t fit = std::max<int64_t>(1, per_sm * nsm / (rb * ny));
+  const int64_t nkb = (K + 63) / 64;
+  int ck = 1;
+  while (ck < 8 && 2 * ck <= fit && 2 * ck <= nkb) ck *= 2;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(rb * ck), static_cast<unsigned>(ny));
+  cfg.blockDim = dim3(lds::kThreads);
+  cfg.dynamicSmemBytes = C::kSmem;
+  cfg.stream = stream;
+  cudaLaunchAttribute at[2];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  at[1].id = cudaLaunchAttributeClusterDimension;
+  at[1].val.clusterDim.x = static_cast<unsigned>(ck);
+  at[1].val.clusterDim.y = 1;
+  at[1].val.clusterDim.z = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = ck > 1 ? 2 : 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, lds::lora_down_stream_kernel<NT>, mx, ma,
+                                           static_cast<int>(M), static_cast<int>(K),
+                                           static_cast<int>(r), s, static_cast<__nv_bfloat16*>(u),
+                                           ck, err);
+  return e == cudaSuccess ? 0 : -3;
+}
+
 }  // namespace
 
 int launch_lora_down(const void* x, int64_t M, int64_t K, const void* A, int64_t r, float s,
@@ -387,6 +676,12 @@ int launch_lora_down(const void* x, int64_t M, int64_t K, const void* A, int64_t
   const auto* xp = static_cast<const __nv_bfloat16*>(x);
   const auto* ap = static_cast<const __nv_bfloat16*>(A);
   auto* up = static_cast<__nv_bfloat16*>(u);
+  if (M >= lds::kBM && K >= 64) {
+    if (r <= 8) return launch_lora_down_stream<1>(x, M, K, A, r, s, u, nsm, stream);
+    if (r <= 16) return launch_lora_down_stream<2>(x, M, K, A, r, s, u, nsm, stream);
+    if (r <= 32) return launch_lora_down_stream<4>(x, M, K, A, r, s, u, nsm, stream);
+    return launch_lora_down_stream<8>(x, M, K, A, r, s, u, nsm, stream);
+  }
   const int64_t tiles = (M + 15) / 16;
   const int64_t ny = r <= 32 ? 1 : (r + 63) / 64;
   // K split over a cluster: about 4 CTAs per SM (2 above 16 ranks, where each CTA already

@@ -68,8 +68,13 @@ def test_rope_q_k_rotated_v_untouched():
 @pytest.mark.parametrize("nseq,P,H_,q_std", [(3, 100, 2, 1.0), (1, 768, 1, 1.0), (2, 64, 1, 1.0),
                                              (1, 1, 2, 1.0), (2, 300, 2, 1.0),
                                              (1, 640, 1, 8.0),   # peaked rows: the running maximum moves
-                                             (5, 700, 8, 1.0),   # 240 tiles: CTAs take several
-                                             (3, 384, 4, 8.0)])
+                                             (5, 700, 8, 1.0),   # 120 two-tile units
+                                             (3, 384, 4, 8.0),
+                                             (8, 1000, 6, 1.0),  # 192 units: CTAs take two
+                                             (16, 300, 12, 1.0),  # odd tile count: 384 units,
+                                                                  # half without a second tile
+                                             (4, 129, 3, 8.0),   # second tile of one row
+                                             (6, 128, 2, 1.0)])  # one tile per sequence
 def test_causal_attention(nseq, P, H_, q_std):
     Dh = 128
     d = H_ * Dh

@@ -245,13 +245,28 @@ def test_gemv_and_tensor_core_kernel_agree():
         assert_rel(host_f64(u), host_f64(v), TOL_LINEAR, "gemv vs tcgen05")
 
 
-def test_lora_down_parity():
-    M, K, r = 300, 4096, 64
-    x, _, _, A, _ = _linear_problem(M, K, 8, r, seed=26)
-    u = torch.empty(M, r, dtype=torch.bfloat16, device="cuda")
+@pytest.mark.parametrize("M,K,r", [
+    (300, 4096, 64),     # streamed form, ragged last row block
+    (3072, 4096, 32),    # q/v and gate/up of the full pass (clusters of 8 along K)
+    (3072, 11008, 16),   # down projection of the full pass: 172 k-blocks, ragged split
+    (2048, 4096, 16),    # LM head of the log-softmax workload
+    (64, 1000, 8),       # one row block, K not a multiple of 64
+    (65, 128, 24),       # two k-blocks only, rank 24 (three n-tiles of a 32-wide tile)
+    (777, 4160, 136),    # three rank tiles of 64, the last partial
+    (130, 72, 40),       # K just above one k-block
+    (40, 4096, 16),      # below 64 rows: the register-fed form
+    (16, 11008, 32),     # decode-sized
+    (200, 48, 16),       # K below one k-block: the register-fed form
+])
+def test_lora_down_parity(M, K, r):
+    x, _, _, A, _ = _linear_problem(M, K, 8, r, seed=26 + M + K + r)
+    u = torch.full((M, r), float("nan"), dtype=torch.bfloat16, device="cuda")
     H.hydra_lora_down(dev_bf16(x), dev_bf16(A), 2.0, u)
     ref = O.lora_down(f64(x), f64(A), 2.0)
     assert_rel(host_f64(u), ref, TOL_LINEAR, "u")
+    u2 = torch.empty_like(u)
+    H.hydra_lora_down(dev_bf16(x), dev_bf16(A), 2.0, u2)
+    assert torch.equal(u, u2), "lora_down is not deterministic"
 
 
 # ------------------------------------------------------------------ full-size workloads
