@@ -4,25 +4,27 @@
 // q, k, v are the column blocks [0, d), [d, 2d), [2d, 3d) of the fused projection output
 // (row stride ld); o is written to columns [h Dh, (h + 1) Dh) of out.
 //
-// Persistent CTAs (one per SM) take tiles of 128 queries of one (sequence, head), longest
-// first; key/value blocks of 128 rows; flash attention with an online softmax. The rings
-// run on across tiles, so the next tile's loads and first Q K^T overlap this tile's tail:
-//  * warp 0 moves Q per tile and the K / V blocks through 3-stage rings with TMA (128-byte
-//    swizzle, [128 rows x 64] boxes); a K stage is released as soon as its Q K^T is done;
-//  * warp 1 owns TMEM and issues tcgen05.mma from one elected lane: S_j = Q K_j^T into the
-//    fp32 S accumulator, which the softmax copies to registers at once, so Q K_{j+1}^T runs
-//    while the softmax works on S_j; then O += P_j V_j into one of two O accumulators (one
-//    per tile in flight), with P read from TMEM and V as an MN-major shared-memory operand;
-//  * warps 2..5 are the softmax: thread i owns query row i (TMEM lane i), so row maxima and
-//    sums need no shuffles. P_j is computed in registers (overlapping P_{j-1} V_{j-1}) and
-//    stored to TMEM as bf16 pairs, so it costs no shared-memory bandwidth: the operand
-//    traffic left in shared memory (K and V in, Q K^T and P V operand reads) is what bounds
-//    a block. The running maximum is a reference value that moves
-//    only when a row's maximum grows by more than 2^8 (then the thread rescales its O row in
-//    TMEM); O and the row sum l share the reference, so O / l is exact either way and every
-//    p stays at most 2^8;
-//  * warps 6..9 are the epilogue: once a tile's last P V is done they normalise its O rows
-//    by the row sums the softmax left in shared memory and store them.
+// Persistent CTAs (one per SM) take units of two adjacent query tiles of 128 rows of one
+// (sequence, head), longest first; key/value blocks of 128 rows; flash attention with an
+// online softmax. Each K / V block staged in shared memory feeds both tiles, so a block costs
+// half the fill traffic per unit of MMA work that one tile per CTA would, and the two tiles
+// take turns on the tensor pipe: while one tile's softmax works, the other tile's products run.
+//  * warp 0 moves Q_a, Q_b per unit and the K / V blocks through one 3-stage ring with TMA
+//    (128-byte swizzle, [128 rows x 64] boxes), in the order the tiles first use them
+//    (K_0, V_0, K_1, V_1, ...); the ring runs on across units, and the next unit's first
+//    blocks are prefetched into L2 a few blocks before a unit ends. Warp 1 owns TMEM (S_a,
+//    S_b, O_a, O_b: 4 x 128 fp32 columns);
+//  * warps 4..7 (tile a) and 8..11 (tile b) each run their tile: thread i owns query row i
+//    (TMEM lane i), so row maxima and sums need no shuffles, and the group's first warp issues
+//    the tile's tcgen05.mma from one elected lane: per key block j, S_x = Q_x K_j^T, then,
+//    once the softmax has written P_x as bf16 pairs over the first 64 columns of S_x,
+//    O_x += P_x V_j (P_x is the A operand, read from TMEM, so it costs no shared-memory
+//    bandwidth) and S_x = Q_x K_{j+1}^T after that P V has finished reading P_x. A finished
+//    tile is normalised into a staging buffer and stored with TMA (one 128-byte line per row
+//    of a box rather than 16-byte pieces of 128 rows), while the tile's next unit runs. The running
+//    maximum is a reference value that moves only when a row's maximum grows by more than
+//    2^8 (then the thread rescales its O row in TMEM); O and the row sum l share the
+//    reference, so O / l is exact either way and every p stays at most 2^8.
 // The probabilities enter P V as bf16 (8 mantissa bits, relative error at most 2^-9); the row
 // sum l accumulates them in fp32.
 #include <float.h>
@@ -34,24 +36,28 @@ namespace hydra {
 namespace attn_tc {
 
 constexpr int kDh = 128;
-constexpr int kBQ = 128;                    // queries per CTA (MMA M, TMEM lanes)
+constexpr int kBQ = 128;                    // queries per tile (MMA M, TMEM lanes)
 constexpr int kBK = 128;                    // keys per block
-constexpr int kThreads = 320;               // producer, MMA, 4 softmax, 4 epilogue warps
+constexpr int kThreads = 384;               // warpgroup 0: TMA producer (warp 0), TMEM owner
+                                            // (warp 1); warpgroups 1, 2: tiles a, b
+// Registers per thread after setmaxnreg: 384 threads x 168 at launch = 128 x 56 + 256 x 224
+constexpr uint32_t kRegsLight = 56;
+constexpr uint32_t kRegsTile = 224;
+static_assert(128 * kRegsLight + 256 * kRegsTile <= kThreads * 168, "register split");
 constexpr int kTile = 128 * 64 * 2;         // [128 rows x 64 bf16] swizzled tile: 16 KiB
 constexpr int kMat = 2 * kTile;             // [128 x 128] bf16 operand: 32 KiB
-constexpr int kOffQ = 0;
-constexpr int kKStages = 3;                 // K ring: K_{j+3} loads once Q K_j^T is done
-constexpr int kVStages = 3;                 // V ring: V_{j+3} loads once P_j V_j is done
-constexpr int kOffK = kOffQ + kMat;
-constexpr int kOffV = kOffK + kKStages * kMat;
-constexpr int kOffL = kOffV + kVStages * kMat;  // final row sums of two tiles: 2 x 128 fp32
-constexpr int kOffBar = kOffL + 2 * kBQ * 4;
-constexpr int kNumBars = 25;
+constexpr int kOffQ = 0;                    // Q_a, Q_b
+constexpr int kStages = 3;                  // one ring for K and V blocks: K_0, V_0, K_1, ...
+constexpr int kOffKV = kOffQ + 2 * kMat;
+constexpr int kOffOut = kOffKV + kStages * kMat;  // output staging: one tile per tile
+constexpr int kOffBar = kOffOut + 2 * kMat;
+constexpr int kNumBars = 4 + 2 * kStages + 4;
 constexpr int kSmem = 1024 + kOffBar + kNumBars * 8 + 16;
+static_assert(kSmem <= 232448, "shared memory per CTA");
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColS = 0;               // S: 128 fp32 columns
-constexpr uint32_t kColP = 128;             // P: 128 bf16 = 64 columns
-constexpr uint32_t kColO = 256;             // O0, O1: 128 fp32 columns each
+constexpr uint32_t kColS = 0;               // S_a, S_b: 128 fp32 columns each; P_x (bf16
+                                            // pairs) overwrites the first 64 columns of S_x
+constexpr uint32_t kColO = 256;             // O_a, O_b: 128 fp32 columns each
 
 // instruction descriptors (kind::f16, bf16 A/B, fp32 D): S = Q K^T (both K-major) and
 // O += P V with V MN-major (bit 16)
@@ -69,6 +75,73 @@ __device__ __forceinline__ uint64_t smem_desc_sw128_mn(uint32_t addr, uint32_t m
   d |= static_cast<uint64_t>(1024u >> 4) << 32;
   d |= static_cast<uint64_t>(1u) << 46;
   d |= static_cast<uint64_t>(2u) << 61;
+  return d;
+}
+
+// Bring the box at (x, y) of a tensor map into L2 (no shared-memory destination).
+__device__ __forceinline__ void tma_prefetch_l2_2d(const CUtensorMap* map, int x, int y) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y)
+               : "memory");
+}
+
+// Store the box at (x, y, z) of a 3-D tensor map from shared memory at src (TMA; elements
+// outside the tensor are not written).
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, uint32_t src, int x, int y,
+                                             int z) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(
+          reinterpret_cast<uint64_t>(map)),
+      "r"(x), "r"(y), "r"(z), "r"(src)
+      : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// the shared-memory source of every committed bulk store has been read
+__device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+// every committed bulk store has completed
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// barrier over the 128 threads of one warpgroup (named barrier id 1 + x)
+__device__ __forceinline__ void wg_sync(int x) {
+  asm volatile("bar.sync %0, 128;" ::"r"(1 + x) : "memory");
+}
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
+                                             uint32_t e) {
+  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c),
+               "r"(e)
+               : "memory");
+}
+
+// Packed fp32 pairs (sm_100 and later execute add / fma on two fp32 lanes per instruction)
+// and a three-input maximum, for the softmax's elementwise steps. (Moving part of the
+// exponentials to the FMA pipe with a cubic was measured slower at every fraction tried.)
+__device__ __forceinline__ uint64_t f2_pack(float a, float b) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t v, float& a, float& b) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
   return d;
 }
 
@@ -133,99 +206,72 @@ __device__ __forceinline__ void tc_mma_ts_bf16(uint32_t d_tmem, uint32_t a_tmem,
 }
 
 
-// This CTA's work: tiles t = blockIdx.x + i * gridDim.x (i = 0, 1, ...) of the ordering
-// t -> (query block qb, head, sequence) with the largest qb (most key blocks) first, so the
-// static round-robin assignment stays balanced; each tile runs key blocks j = 0..qb.
-struct BlockCursor {
-  int nqb, heads, nseq, ntiles, stride;
-  int t, i, j;        // tile, this CTA's tile number, key block
-  int qb, head, seq;  // decoded tile
-  __device__ void init(int nqb_, int heads_, int nseq_, int first, int step) {
-    nqb = nqb_;
-    heads = heads_;
-    nseq = nseq_;
-    ntiles = nqb * heads * nseq;
-    stride = step;
-    t = first;
-    i = 0;
-    j = 0;
-    decode();
+// This CTA's work: units t = blockIdx.x + i * gridDim.x (i = 0, 1, ...) of the ordering
+// t -> (query-block pair p, head, sequence) with the largest p (most key blocks) first, so the
+// static round-robin assignment stays balanced. Unit (p, head, seq) holds the two query tiles
+// qa = 2p and qb = 2p + 1 (qb only when it exists): tile a runs key blocks 0..qa, tile b
+// 0..qb, and every key block the two share is loaded once for both.
+struct UnitCursor {
+  int t;               // unit
+  int p, head, seq;    // decoded unit
+  int na, nb, nblk;    // key blocks of tile a, of tile b (0: no tile b), of the unit
+  // the loop-invariant sizes are recomputed from the kernel arguments (constant bank) rather
+  // than kept in registers: the producer and MMA warps run with few registers
+  __device__ static int units(int P, int heads, int nseq) {
+    return (((P + kBQ - 1) / kBQ + 1) / 2) * heads * nseq;
   }
-  __device__ void decode() {
-    if (t >= ntiles) return;
+  __device__ void decode(int P, int heads, int nseq) {
+    const int nqb = (P + kBQ - 1) / kBQ;
     const int hs = heads * nseq;
-    qb = nqb - 1 - t / hs;
+    p = (nqb + 1) / 2 - 1 - t / hs;
     const int r = t % hs;
     head = r % heads;
     seq = r / heads;
-  }
-  __device__ bool valid() const { return t < ntiles; }
-  __device__ bool last() const { return j == qb; }
-  __device__ void next() {
-    if (++j > qb) {
-      j = 0;
-      ++i;
-      t += stride;
-      decode();
-    }
+    na = 2 * p + 1;
+    nb = (2 * p + 1 < nqb) ? 2 * p + 2 : 0;
+    nblk = nb > 0 ? nb : na;
   }
 };
 
 __global__ void __launch_bounds__(kThreads, 1)
-    causal_attention_tc_kernel(const __grid_constant__ CUtensorMap tm_qkv, int P, int d,
-                               int n_heads, int nseq, float scale_log2,
-                               __nv_bfloat16* __restrict__ out, int ld_out, int* err) {
+    causal_attention_tc_kernel(const __grid_constant__ CUtensorMap tm_qkv,
+                               const __grid_constant__ CUtensorMap tm_out, int P, int d,
+                               int n_heads, int nseq, float scale_log2, int* err) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  float* l_sm = reinterpret_cast<float*>(smem + kOffL);  // [2][kBQ]
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kOffBar);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + kNumBars);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int nqb = (P + kBQ - 1) / kBQ;
+  const int nunits = UnitCursor::units(P, n_heads, nseq);
 
   const uint32_t sbase = smem_u32(smem);
-  const uint32_t sQ = sbase + kOffQ, sK = sbase + kOffK, sV = sbase + kOffV;
+  auto sQ = [&](int x) { return sbase + kOffQ + x * kMat; };
+  auto sKV = [&](int st) { return sbase + kOffKV + st * kMat; };
   auto bar = [&](int i) { return smem_u32(&bars[i]); };
-  const uint32_t q_full = bar(0);
-  const uint32_t q_empty = bar(1);
-  auto k_full = [&](int i) { return bar(2 + i); };
-  auto k_empty = [&](int i) { return bar(5 + i); };
-  auto v_full = [&](int i) { return bar(8 + i); };
-  auto v_empty = [&](int i) { return bar(11 + i); };
-  const uint32_t s_full = bar(14);
-  const uint32_t s_free = bar(15);
-  const uint32_t p_full = bar(16);
-  const uint32_t pv_done = bar(17);
-  auto o_full = [&](int b) { return bar(18 + b); };
-  auto o_free = [&](int b) { return bar(20 + b); };
-  auto l_full = [&](int b) { return bar(22 + b); };
-  const uint32_t mma_done = bar(24);
+  auto q_full = [&](int x) { return bar(0 + x); };
+  auto q_empty = [&](int x) { return bar(2 + x); };
+  auto kv_full = [&](int st) { return bar(4 + st); };
+  auto kv_empty = [&](int st) { return bar(4 + kStages + st); };
+  auto s_full = [&](int x) { return bar(4 + 2 * kStages + x); };
+  auto pv_done = [&](int x) { return bar(6 + 2 * kStages + x); };
 
   if (threadIdx.x == 0) {
-    mbar_init(q_full, 1);
-    mbar_init(q_empty, 1);
-    for (int i = 0; i < kKStages; ++i) {
-      mbar_init(k_full(i), 1);
-      mbar_init(k_empty(i), 1);
+    for (int x = 0; x < 2; ++x) {
+      mbar_init(q_full(x), 1);
+      mbar_init(q_empty(x), 1);
+      mbar_init(s_full(x), 1);
+      mbar_init(pv_done(x), 1);
     }
-    for (int i = 0; i < kVStages; ++i) {
-      mbar_init(v_full(i), 1);
-      mbar_init(v_empty(i), 1);
+    // a K or V block is released by each of the two tiles (a block only one tile uses is
+    // released twice by that tile)
+    for (int i = 0; i < kStages; ++i) {
+      mbar_init(kv_full(i), 1);
+      mbar_init(kv_empty(i), 2);
     }
-    mbar_init(s_full, 1);
-    mbar_init(s_free, 4);
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(o_full(b), 1);
-      mbar_init(o_free(b), 4);
-      mbar_init(l_full(b), 4);
-    }
-    mbar_init(p_full, 4);
-    mbar_init(pv_done, 1);
-    mbar_init(mma_done, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -238,292 +284,318 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  if (warp == 0) {
-    // ---------------------------------------------------------------- TMA producer
-    if (elect_one()) tma_prefetch_desc(&tm_qkv);
-    __syncwarp();
-    // K runs one block ahead of V in issue order: K_{g+1} waits only for an earlier Q K^T,
-    // which finishes before the P V that V_g waits for. A tile's Q loads with its first K
-    // block, once the previous tile's last Q K^T is done.
-    BlockCursor kc, vc;
-    kc.init(nqb, n_heads, nseq, blockIdx.x, gridDim.x);
-    vc = kc;
-    int gk = 0, gv = 0, nq = 0;  // K blocks, V blocks, Q tiles issued
-    auto load_k = [&]() {
-      if (kc.j == 0) {
-        if (kc.i >= 1 &&
-            !warp_wait_bounded(q_empty, (kc.i - 1) & 1, abort_flag, err, kDevTimeoutProducer))
+  if (warp < 4) {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsLight));
+    if (warp == 0) {
+      // -------------------------------------------------------------- TMA producer
+      // Per unit: Q_a, K_0, Q_b, V_0, K_1, V_1, ..., the order in which the tiles first need
+      // them; the ring runs on across units
+      if (elect_one()) {
+        tma_prefetch_desc(&tm_qkv);
+        tma_prefetch_desc(&tm_out);
+      }
+      __syncwarp();
+      UnitCursor c;
+      int pos = 0, nq[2] = {0, 0};  // ring positions filled, Q tiles loaded per tile
+      bool ok = true;
+      auto load_q = [&](int x) {
+        if (nq[x] >= 1 && !warp_wait_bounded(q_empty(x), (nq[x] - 1) & 1, abort_flag, err,
+                                             kDevTimeoutProducer))
           return false;
         if (elect_one()) {
-          const int y = kc.seq * P + kc.qb * kBQ;
-          mbar_arrive_expect_tx(q_full, kMat);
-          tma_load_2d(sQ, &tm_qkv, kc.head * kDh, y, q_full);
-          tma_load_2d(sQ + kTile, &tm_qkv, kc.head * kDh + 64, y, q_full);
+          const int y = c.seq * P + (2 * c.p + x) * kBQ;
+          mbar_arrive_expect_tx(q_full(x), kMat);
+          tma_load_2d(sQ(x), &tm_qkv, c.head * kDh, y, q_full(x));
+          tma_load_2d(sQ(x) + kTile, &tm_qkv, c.head * kDh + 64, y, q_full(x));
         }
         __syncwarp();
-        ++nq;
-      }
-      const int st = gk % kKStages;
-      if (gk >= kKStages && !warp_wait_bounded(k_empty(st), (gk / kKStages - 1) & 1, abort_flag,
-                                               err, kDevTimeoutProducer))
-        return false;
-      if (elect_one()) {
-        const int y = kc.seq * P + kc.j * kBK;
-        mbar_arrive_expect_tx(k_full(st), kMat);
-        tma_load_2d(sK + st * kMat, &tm_qkv, d + kc.head * kDh, y, k_full(st));
-        tma_load_2d(sK + st * kMat + kTile, &tm_qkv, d + kc.head * kDh + 64, y, k_full(st));
-      }
-      __syncwarp();
-      ++gk;
-      kc.next();
-      return true;
-    };
-    auto load_v = [&]() {
-      const int st = gv % kVStages;
-      if (gv >= kVStages && !warp_wait_bounded(v_empty(st), (gv / kVStages - 1) & 1, abort_flag,
-                                               err, kDevTimeoutProducer))
-        return false;
-      if (elect_one()) {
-        const int y = vc.seq * P + vc.j * kBK;
-        mbar_arrive_expect_tx(v_full(st), kMat);
-        tma_load_2d(sV + st * kMat, &tm_qkv, 2 * d + vc.head * kDh, y, v_full(st));
-        tma_load_2d(sV + st * kMat + kTile, &tm_qkv, 2 * d + vc.head * kDh + 64, y, v_full(st));
-      }
-      __syncwarp();
-      ++gv;
-      vc.next();
-      return true;
-    };
-    // at a tile boundary V_g goes first: the next tile's Q waits for this tile's last Q K^T
-    bool ok = kc.valid() ? load_k() : false;
-    while (ok && vc.valid()) {
-      if (kc.valid() && kc.j != 0) {
-        if (!load_k() || !load_v()) break;
-      } else {
-        if (!load_v() || (kc.valid() && !load_k())) break;
-      }
-    }
-    // copies in flight land before the CTA's shared memory is released
-    volatile int no_abort = 0;
-    if (nq > 0) warp_wait_bounded(q_full, (nq - 1) & 1, &no_abort, err, kDevTimeoutDrain);
-    for (int g = (gk > kKStages ? gk - kKStages : 0); g < gk; ++g)
-      warp_wait_bounded(k_full(g % kKStages), (g / kKStages) & 1, &no_abort, err, kDevTimeoutDrain);
-    for (int g = (gv > kVStages ? gv - kVStages : 0); g < gv; ++g)
-      warp_wait_bounded(v_full(g % kVStages), (g / kVStages) & 1, &no_abort, err, kDevTimeoutDrain);
-  } else if (warp == 1) {
-    // ---------------------------------------------------------------- MMA issuer
-    // S_g = Q K_g^T for the next key block is issued before P_g V_g, so it overlaps the
-    // softmax of block g. O of a tile accumulates in O[tile & 1].
-    BlockCursor sc, pc;
-    sc.init(nqb, n_heads, nseq, blockIdx.x, gridDim.x);
-    pc = sc;
-    int gs = 0, gp = 0;  // S and P V products issued
-    auto issue_s = [&]() {
-      const int st = gs % kKStages;
-      if (sc.j == 0 && !warp_wait_bounded(q_full, sc.i & 1, abort_flag, err, kDevTimeoutMma))
-        return false;
-      if (!warp_wait_bounded(k_full(st), (gs / kKStages) & 1, abort_flag, err, kDevTimeoutMma))
-        return false;
-      // the softmax has copied S_{gs-1} to registers
-      if (gs >= 1 && !warp_wait_bounded(s_free, (gs - 1) & 1, abort_flag, err, kDevTimeoutMma))
-        return false;
-      tc_fence_after();
-      if (elect_one()) {
-        const uint32_t kb = sK + st * kMat;
-#pragma unroll
-        for (int k = 0; k < kDh / 16; ++k) {
-          const uint32_t off = (k >> 2) * kTile + (k & 3) * 32;
-          tc_mma_bf16(tmem + kColS, smem_desc_sw128(sQ + off), smem_desc_sw128(kb + off),
-                      kIdescQK, k > 0 ? 1u : 0u);
+        ++nq[x];
+        return true;
+      };
+      // K (kv = 1) or V (kv = 2) of key block j
+      auto load_kv = [&](int kv, int j) {
+        const int st = pos % kStages;
+        if (pos >= kStages && !warp_wait_bounded(kv_empty(st), (pos / kStages - 1) & 1,
+                                                 abort_flag, err, kDevTimeoutProducer))
+          return false;
+        if (elect_one()) {
+          const int y = c.seq * P + j * kBK;
+          const int x0 = kv * d + c.head * kDh;
+          mbar_arrive_expect_tx(kv_full(st), kMat);
+          tma_load_2d(sKV(st), &tm_qkv, x0, y, kv_full(st));
+          tma_load_2d(sKV(st) + kTile, &tm_qkv, x0 + 64, y, kv_full(st));
         }
-        tc_commit(s_full);
-        tc_commit(k_empty(st));
-        if (sc.last()) tc_commit(q_empty);
-      }
-      __syncwarp();
-      ++gs;
-      sc.next();
-      return true;
-    };
-    auto issue_pv = [&]() {
-      const int st = gp % kVStages, ob = pc.i & 1;
-      // O[ob] is free once the epilogue has read the tile two back
-      if (pc.j == 0 && pc.i >= 2 &&
-          !warp_wait_bounded(o_free(ob), ((pc.i - 2) >> 1) & 1, abort_flag, err, kDevTimeoutMma))
-        return false;
-      if (!warp_wait_bounded(p_full, gp & 1, abort_flag, err, kDevTimeoutMma) ||
-          !warp_wait_bounded(v_full(st), (gp / kVStages) & 1, abort_flag, err, kDevTimeoutMma))
-        return false;
-      tc_fence_after();
-      if (elect_one()) {
-        const uint32_t vb = sV + st * kMat;
-#pragma unroll
-        for (int k = 0; k < kBK / 16; ++k) {
-          // A: P keys [16k, 16k + 16) from TMEM (8 columns); B: V rows [16k, 16k + 16)
-          // (MN-major)
-          tc_mma_ts_bf16(tmem + kColO + ob * kDh, tmem + kColP + 8 * k,
-                         smem_desc_sw128_mn(vb + k * 2048, kTile), kIdescPV,
-                         (pc.j > 0 || k > 0) ? 1u : 0u);
-        }
-        tc_commit(pv_done);
-        tc_commit(v_empty(st));
-        if (pc.last()) tc_commit(o_full(ob));
-      }
-      __syncwarp();
-      ++gp;
-      pc.next();
-      return true;
-    };
-    // across a tile boundary P V goes first, so that the tile's last block does not wait for
-    // the next tile's Q
-    bool ok = sc.valid() ? issue_s() : false;
-    while (ok && pc.valid()) {
-      if (sc.valid() && sc.j != 0) {
-        if (!issue_s() || !issue_pv()) break;
-      } else {
-        if (!issue_pv() || (sc.valid() && !issue_s())) break;
-      }
-    }
-    // every issued MMA has finished before TMEM is released
-    if (elect_one()) tc_commit(mma_done);
-    __syncwarp();
-    volatile int no_abort = 0;
-    warp_wait_bounded(mma_done, 0, &no_abort, err, kDevTimeoutDrain);
-  } else if (warp < 6) {
-    // ---------------------------------------------------------------- softmax (warps 2..5)
-    const int q4 = warp & 3;                  // this warp may access TMEM lanes [32 q4, +32)
-    const int row = q4 * 32 + lane;           // query row of the tile = TMEM lane
-    const uint32_t t_lane = tmem + (static_cast<uint32_t>(q4 * 32) << 16);
-    BlockCursor c;
-    c.init(nqb, n_heads, nseq, blockIdx.x, gridDim.x);
-    float m_ref = -FLT_MAX;                   // reference maximum, log2 domain
-    float l = 0.f;                            // row sum of the probabilities
-    int g = 0;
-    while (c.valid()) {
-      const int ob = c.i & 1, j = c.j;
-      if (!warp_wait_bounded(s_full, g & 1, abort_flag, err, kDevTimeoutEpilogue)) break;
-      tc_fence_after();
-      float s[kBK];
-      tc_ld_x64(t_lane + kColS, *reinterpret_cast<float(*)[64]>(s));
-      tc_ld_x64(t_lane + kColS + 64, *reinterpret_cast<float(*)[64]>(s + 64));
-      tc_wait_ld();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(s_free);  // S_g is in registers: Q K_{g+1}^T may overwrite it
-      // maximum raw score over the visible keys (on the diagonal block, the tile's last, key
-      // c is visible to row `row` iff c <= row), eight chains; the scale (> 0) comes after
-      if (c.last()) {
-#pragma unroll
-        for (int k = 1; k < kBK; ++k)
-          if (k > row) s[k] = -INFINITY;
-      }
-      float pm[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) pm[i] = s[i];
-#pragma unroll
-      for (int k = 8; k < kBK; ++k) pm[k & 7] = fmaxf(pm[k & 7], s[k]);
-      const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
-                             fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7]))) *
-                       scale_log2;
-      bool rescale = false;
-      float corr = 1.f;
-      if (j == 0) {
-        m_ref = mx;
-        l = 0.f;
-      } else if (mx > m_ref + 8.f) {
-        corr = ex2(m_ref - mx);
-        m_ref = mx;
-        rescale = true;
-      }
-      // P_g = 2^(scale s - m_ref) in registers (bf16 pairs) before any wait
-      float ps[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) ps[i] = 0.f;
-      uint32_t w[kBK / 2];
-#pragma unroll
-      for (int i = 0; i < kBK / 2; ++i) {
-        const float p0 = ex2(fmaf(s[2 * i], scale_log2, -m_ref));
-        const float p1 = ex2(fmaf(s[2 * i + 1], scale_log2, -m_ref));
-        ps[(2 * i) & 7] += p0;
-        ps[(2 * i + 1) & 7] += p1;
-        w[i] = pack_bf16x2(p0, p1);
-      }
-      l = l * corr + (((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7])));
-      // P_{g-1} V_{g-1} has finished: P in TMEM may be overwritten and O is stable
-      if (g > 0 &&
-          !warp_wait_bounded(pv_done, (g - 1) & 1, abort_flag, err, kDevTimeoutEpilogue))
-        break;
-      tc_fence_after();
-      if (__any_sync(0xffffffffu, rescale)) {
-        const uint32_t t_o = t_lane + kColO + ob * kDh;
-#pragma unroll 1
-        for (int h = 0; h < 4; ++h) {
-          uint32_t o[32];
-          tc_ld_32x32b_x32(t_o + 32 * h, o);
-          tc_wait_ld();
-#pragma unroll
-          for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * corr);
-          tc_st_x32(t_o + 32 * h, o);
-        }
-        tc_wait_st();
-      }
-      tc_st_x32(t_lane + kColP, *reinterpret_cast<uint32_t(*)[32]>(w));
-      tc_st_x32(t_lane + kColP + 32, *reinterpret_cast<uint32_t(*)[32]>(w + 32));
-      tc_wait_st();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(p_full);
-      if (c.last()) {
-        // hand the row sum to the epilogue; its copy of the tile two back has been read
-        if (c.i >= 2 &&
-            !warp_wait_bounded(o_free(ob), ((c.i - 2) >> 1) & 1, abort_flag, err,
-                               kDevTimeoutEpilogue))
-          break;
-        l_sm[ob * kBQ + row] = l;
         __syncwarp();
-        if (lane == 0) mbar_arrive(l_full(ob));
+        ++pos;
+        return true;
+      };
+      // L2 prefetch of the next unit's Q tiles and first two K / V blocks, a few blocks before
+      // this unit ends: every CTA reaches a unit boundary at about the same time, and the
+      // loads there would otherwise queue behind each other in DRAM
+      auto prefetch_next = [&]() {
+        UnitCursor nx;
+        nx.t = c.t + gridDim.x;
+        if (nx.t >= nunits || !elect_one()) return;
+        nx.decode(P, n_heads, nseq);
+        const int y0 = nx.seq * P;
+        for (int x = 0; x < (nx.nb > 0 ? 2 : 1); ++x)
+          for (int h = 0; h < 2; ++h)
+            tma_prefetch_l2_2d(&tm_qkv, nx.head * kDh + 64 * h, y0 + (2 * nx.p + x) * kBQ);
+        for (int j = 0; j < (nx.nblk < 2 ? nx.nblk : 2); ++j)
+          for (int kv = 1; kv <= 2; ++kv)
+            for (int h = 0; h < 2; ++h)
+              tma_prefetch_l2_2d(&tm_qkv, kv * d + nx.head * kDh + 64 * h, y0 + j * kBK);
+      };
+      for (c.t = blockIdx.x; ok && c.t < nunits; c.t += gridDim.x) {
+        c.decode(P, n_heads, nseq);
+        const int jpf = c.nblk > 3 ? c.nblk - 3 : 0;  // prefetch after this block's loads
+        ok = load_q(0) && load_kv(1, 0);
+        if (ok && c.nb > 0) ok = load_q(1);
+        if (ok) ok = load_kv(2, 0);
+        if (ok && jpf == 0) prefetch_next();
+        __syncwarp();
+        for (int j = 1; ok && j < c.nblk; ++j) {
+          ok = load_kv(1, j) && load_kv(2, j);
+          if (ok && j == jpf) prefetch_next();
+          __syncwarp();
+        }
       }
-      ++g;
-      c.next();
+      // copies in flight land before the CTA's shared memory is released
+      volatile int no_abort = 0;
+      for (int x = 0; x < 2; ++x)
+        if (nq[x] > 0)
+          warp_wait_bounded(q_full(x), (nq[x] - 1) & 1, &no_abort, err, kDevTimeoutDrain);
+      for (int g = (pos > kStages ? pos - kStages : 0); g < pos; ++g)
+        warp_wait_bounded(kv_full(g % kStages), (g / kStages) & 1, &no_abort, err,
+                          kDevTimeoutDrain);
     }
   } else {
-    // ---------------------------------------------------------------- epilogue (warps 6..9)
-    const int q4 = warp & 3;
-    const int row = q4 * 32 + lane;
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegsTile));
+    // -------------------------------------------------------------- tiles (warps 4..11)
+    // Warps 4..7 own tile a, warps 8..11 tile b; thread i of a group owns query row i (TMEM
+    // lane i). Each group runs its tile's softmax and issues the tile's products itself:
+    // once P_x is in TMEM, one of its warps issues P_x V_j and then Q_x K_{j+1}^T (after that
+    // P V has finished reading P_x, which the next S overwrites), so no other warp sits on
+    // the path from a finished P to the tensor pipe. The two groups' products interleave on
+    // the pipe: one tile's softmax overlaps the other tile's products.
+    const int x = warp < 8 ? 0 : 1;
+    const int q4 = warp & 3;                  // this warp may access TMEM lanes [32 q4, +32)
+    const int row = q4 * 32 + lane;           // query row of the tile = TMEM lane
+    // the warp that issues the tile's products: sub-partition 1 for tile a, 2 for tile b, so
+    // that neither shares a scheduler with the other issuer or with the TMA producer (warp 0)
+    const bool issuer = (q4 == 1 + x);
     const uint32_t t_lane = tmem + (static_cast<uint32_t>(q4 * 32) << 16);
-    BlockCursor c;
-    c.init(nqb, n_heads, nseq, blockIdx.x, gridDim.x);
-    for (; c.valid(); c.t += c.stride, ++c.i, c.decode()) {
-      const int ob = c.i & 1;
-      if (!warp_wait_bounded(o_full(ob), (c.i >> 1) & 1, abort_flag, err, kDevTimeoutEpilogue) ||
-          !warp_wait_bounded(l_full(ob), (c.i >> 1) & 1, abort_flag, err, kDevTimeoutEpilogue))
-        break;
+    const uint32_t t_s = t_lane + kColS + x * 128;
+    const uint32_t t_o = t_lane + kColO + x * kDh;
+    const uint32_t s_stage = sbase + kOffOut + x * kMat;  // this tile's output staging
+    int gs = 0, gpv = 0, nqu = 0;             // S consumed, P V issued, units begun (Q tiles)
+    int kbase = 0;                            // ring block index of the unit's key block 0
+    bool s0_issued = false;                   // this unit's first Q K^T was issued already
+    bool ok = true;
+    // Q_x K^T of the block at ring position kpos (issuer warp); rel: releases of its stage
+    auto issue_s = [&](bool first, int kpos, int rel, bool last_s) {
+      if (first && !warp_wait_bounded(q_full(x), nqu & 1, abort_flag, err, kDevTimeoutMma))
+        return false;
+      const int st = kpos % kStages;
+      if (!warp_wait_bounded(kv_full(st), (kpos / kStages) & 1, abort_flag, err, kDevTimeoutMma))
+        return false;
+      if (gpv >= 1 &&
+          !warp_wait_bounded(pv_done(x), (gpv - 1) & 1, abort_flag, err, kDevTimeoutMma))
+        return false;
       tc_fence_after();
-      const float inv = 1.f / l_sm[ob * kBQ + row];
-      const int q = c.qb * kBQ + row;
-      __nv_bfloat16* orow = out + static_cast<size_t>(c.seq * P + q) * ld_out + c.head * kDh;
-#pragma unroll 1
-      for (int h = 0; h < 4; ++h) {
-        uint32_t o[32];
-        tc_ld_32x32b_x32(t_lane + kColO + ob * kDh + 32 * h, o);
-        tc_wait_ld();
-        if (q < P) {
+      if (elect_one()) {
+        // descriptors of the tile bases; a k-step adds its byte offset / 16 to the address
+        // field (every shared address here is below 2^18, so the field cannot carry over)
+        const uint64_t dq = smem_desc_sw128(sQ(x));
+        const uint64_t dk = smem_desc_sw128(sKV(st));
 #pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            auto f = [&](int e) { return __uint_as_float(o[8 * i + e]) * inv; };
-            uint4 v;
-            v.x = pack_bf16x2(f(0), f(1));
-            v.y = pack_bf16x2(f(2), f(3));
-            v.z = pack_bf16x2(f(4), f(5));
-            v.w = pack_bf16x2(f(6), f(7));
-            *reinterpret_cast<uint4*>(orow + 32 * h + 8 * i) = v;
+        for (int k = 0; k < kDh / 16; ++k) {
+          const uint32_t off = ((k >> 2) * kTile + (k & 3) * 32) >> 4;
+          tc_mma_bf16(tmem + kColS + x * 128, dq + off, dk + off, kIdescQK, k > 0 ? 1u : 0u);
+        }
+        tc_commit(s_full(x));
+        for (int i = 0; i < rel; ++i) tc_commit(kv_empty(st));
+        if (last_s) tc_commit(q_empty(x));
+      }
+      __syncwarp();
+      if (first) ++nqu;
+      return true;
+    };
+    // P_x V of the block at ring position vpos (issuer warp)
+    auto issue_pv = [&](bool first, int vpos, int rel) {
+      const int st = vpos % kStages;
+      if (!warp_wait_bounded(kv_full(st), (vpos / kStages) & 1, abort_flag, err, kDevTimeoutMma))
+        return false;
+      tc_fence_after();
+      if (elect_one()) {
+        const uint64_t dv = smem_desc_sw128_mn(sKV(st), kTile);
+#pragma unroll
+        for (int k = 0; k < kBK / 16; ++k)
+          tc_mma_ts_bf16(tmem + kColO + x * kDh, tmem + kColS + x * 128 + 8 * k,
+                         dv + ((k * 2048) >> 4), kIdescPV, (!first || k > 0) ? 1u : 0u);
+        tc_commit(pv_done(x));
+        for (int i = 0; i < rel; ++i) tc_commit(kv_empty(st));
+      }
+      __syncwarp();
+      ++gpv;
+      return true;
+    };
+    float m_ref = -FLT_MAX;                   // reference maximum, log2 domain
+    float l = 0.f;                            // row sum of the probabilities
+    UnitCursor c;
+    for (c.t = blockIdx.x; ok && c.t < nunits; c.t += gridDim.x) {
+      c.decode(P, n_heads, nseq);
+      const int n = x == 0 ? c.na : c.nb;     // this tile's key blocks (0: no tile b)
+      const int on = x == 0 ? c.nb : c.na;    // the other tile's
+      const int J = c.nblk;
+      if (n == 0) {
+        kbase += J;
+        s0_issued = false;
+        continue;
+      }
+      // ring positions: K_j at 2 (kbase + j), V_j right after it
+      if (!s0_issued && issuer) ok = issue_s(true, 2 * kbase, on > 0 ? 1 : 2, n == 1);
+      for (int j = 0; ok && j < n; ++j) {
+        if (!warp_wait_bounded(s_full(x), gs & 1, abort_flag, err, kDevTimeoutEpilogue)) {
+          ok = false;
+          break;
+        }
+        ++gs;
+        tc_fence_after();
+        float sv[kBK];
+        tc_ld_x64(t_s, *reinterpret_cast<float(*)[64]>(sv));
+        tc_ld_x64(t_s + 64, *reinterpret_cast<float(*)[64]>(sv + 64));
+        tc_wait_ld();
+        // the diagonal block (the tile's last): key c is visible to row `row` iff c <= row
+        const bool diag = (j == n - 1);
+        if (diag) {
+#pragma unroll
+          for (int k = 1; k < kBK; ++k)
+            if (k > row) sv[k] = -INFINITY;
+        }
+        float pm[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) pm[i] = -FLT_MAX;
+#pragma unroll
+        for (int i = 0; i < kBK / 2; ++i) pm[i & 7] = max3(pm[i & 7], sv[2 * i], sv[2 * i + 1]);
+        const float mx = max3(max3(pm[0], pm[1], pm[2]), max3(pm[3], pm[4], pm[5]),
+                              fmaxf(pm[6], pm[7])) *
+                         scale_log2;
+        bool rescale = false;
+        float corr = 1.f;
+        if (j == 0) {
+          m_ref = mx;
+          l = 0.f;
+        } else if (mx > m_ref + 8.f) {
+          corr = ex2(m_ref - mx);
+          m_ref = mx;
+          rescale = true;
+        }
+        // P = 2^(scale s - m_ref) as bf16 pairs over the first 64 columns of S_x; the argument
+        // and the row sum in packed pairs
+        const uint64_t sc2 = f2_pack(scale_log2, scale_log2), nm2 = f2_pack(-m_ref, -m_ref);
+        uint64_t acc[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) acc[i] = f2_pack(0.f, 0.f);
+        uint32_t w[kBK / 2];
+#pragma unroll
+        for (int i = 0; i < kBK / 2; ++i) {
+          float a0, a1;
+          f2_unpack(f2_fma(f2_pack(sv[2 * i], sv[2 * i + 1]), sc2, nm2), a0, a1);
+          const float p0 = ex2(a0), p1 = ex2(a1);
+          acc[i & 3] = f2_add(acc[i & 3], f2_pack(p0, p1));
+          w[i] = pack_bf16x2(p0, p1);
+        }
+        float ps[8];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) f2_unpack(acc[i], ps[2 * i], ps[2 * i + 1]);
+        l = l * corr + (((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7])));
+        // O_x holds the sum through the previous block (that P V finished before this S was
+        // issued): rescale the row when the reference moved
+        if (__any_sync(0xffffffffu, rescale)) {
+#pragma unroll 1
+          for (int h = 0; h < 4; ++h) {
+            uint32_t o[32];
+            tc_ld_32x32b_x32(t_o + 32 * h, o);
+            tc_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * corr);
+            tc_st_x32(t_o + 32 * h, o);
+            tc_wait_st();
+          }
+        }
+        tc_st_x32(t_s, *reinterpret_cast<uint32_t(*)[32]>(w));
+        tc_st_x32(t_s + 32, *reinterpret_cast<uint32_t(*)[32]>(w + 32));
+        tc_wait_st();
+        tc_fence_before();
+        wg_sync(x);  // P_x of the whole tile is in TMEM
+        if (issuer) {
+          ok = issue_pv(j == 0, 2 * (kbase + j) + 1, j < on ? 1 : 2);
+          if (ok && j + 1 < n) {
+            ok = issue_s(false, 2 * (kbase + j + 1), j + 1 < on ? 1 : 2, j + 1 == n - 1);
+          } else if (ok) {
+            // the next unit's first Q_x K^T, if it has tile x: its stage meanwhile fills
+            UnitCursor nx;
+            nx.t = c.t + gridDim.x;
+            s0_issued = false;
+            if (nx.t < nunits) {
+              nx.decode(P, n_heads, nseq);
+              const int nn = x == 0 ? nx.na : nx.nb, non = x == 0 ? nx.nb : nx.na;
+              if (nn > 0) {
+                ok = issue_s(true, 2 * (kbase + J), non > 0 ? 1 : 2, nn == 1);
+                s0_issued = true;
+              }
+            }
           }
         }
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(o_free(ob));
+      if (!ok) break;
+      // the finished tile (its last P V, the gs-th, is done): O_x / l as bf16 rows, staged in
+      // shared memory as two 128-byte-swizzled TMA boxes of 64 columns and stored with TMA;
+      // the staging buffer is reused only once the stores of the previous unit have read it
+      if (issuer) {
+        if (elect_one()) bulk_wait_read();
+        __syncwarp();
+      }
+      if (!warp_wait_bounded(pv_done(x), (gs - 1) & 1, abort_flag, err, kDevTimeoutEpilogue)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      {
+        uint32_t o[4][32];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) tc_ld_32x32b_x32(t_o + 32 * q, o[q]);
+        tc_wait_ld();
+        const float inv = 1.f / l;
+        wg_sync(x);  // the previous unit's stores have read the staging buffer
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const uint32_t box = s_stage + (q >> 1) * kTile + row * 128;
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            auto f = [&](int e) { return __uint_as_float(o[q][8 * i + e]) * inv; };
+            const int chunk = 4 * (q & 1) + i;
+            st_shared_v4(box + ((chunk ^ (row & 7)) << 4), pack_bf16x2(f(0), f(1)),
+                         pack_bf16x2(f(2), f(3)), pack_bf16x2(f(4), f(5)), pack_bf16x2(f(6), f(7)));
+          }
+        }
+      }
+      fence_proxy_async_smem();
+      wg_sync(x);
+      if (issuer) {
+        if (elect_one()) {
+          for (int h = 0; h < 2; ++h)
+            tma_store_3d(&tm_out, s_stage + h * kTile, c.head * kDh + 64 * h, (2 * c.p + x) * kBQ,
+                         c.seq);
+          bulk_commit();
+        }
+        __syncwarp();
+      }
+      kbase += J;
     }
+    if (issuer && elect_one()) bulk_wait_all();
+    __syncwarp();
   }
 
   tc_fence_before();
@@ -555,15 +627,16 @@ int launch_causal_attention(const void* qkv, int64_t nseq, int64_t P, int64_t ld
   int* err = device_error_word();
   if (err == nullptr) return -1;
   const int64_t d = n_heads * head_dim;
-  CUtensorMap map;
+  CUtensorMap map, map_out;
   if (!make_tma_map(&map, qkv, nseq * P, 3 * d, ld, 128, false)) return -2;
-  const int64_t ntiles = ((P + kBQ - 1) / kBQ) * n_heads * nseq;
-  const unsigned grid = static_cast<unsigned>(ntiles < nsm ? ntiles : nsm);
+  // output as nseq planes of [P, d]: a tile's rows past its sequence are not stored
+  if (!make_tma_map_3d(&map_out, out, d, P, nseq, ld_out, P * ld_out, kBQ)) return -2;
+  const int64_t nunits = ((P + 2 * kBQ - 1) / (2 * kBQ)) * n_heads * nseq;
+  const unsigned grid = static_cast<unsigned>(nunits < nsm ? nunits : nsm);
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(head_dim));
   causal_attention_tc_kernel<<<grid, kThreads, kSmem, st>>>(
-      map, static_cast<int>(P), static_cast<int>(d), static_cast<int>(n_heads),
-      static_cast<int>(nseq), scale_log2, static_cast<__nv_bfloat16*>(out),
-      static_cast<int>(ld_out), err);
+      map, map_out, static_cast<int>(P), static_cast<int>(d), static_cast<int>(n_heads),
+      static_cast<int>(nseq), scale_log2, err);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
 }
 

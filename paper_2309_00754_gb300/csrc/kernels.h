@@ -75,6 +75,11 @@ int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream);
 // 128-byte swizzle, boxes of [box_rows x 128 bytes], zero fill out of bounds
 bool make_tma_map(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int64_t ld,
                   int box_rows, bool f32);
+// TMA map over bf16 planes of [rows, cols] (row stride ld, plane stride plane_stride elements):
+// 128-byte swizzle, boxes of [box_rows x 64] in one plane; out-of-range elements are not
+// written by a store
+bool make_tma_map_3d(CUtensorMap* map, const void* base, int64_t cols, int64_t rows,
+                     int64_t planes, int64_t ld, int64_t plane_stride, int box_rows);
 int launch_dual_lora_gemv(const GemmArgs& a, cudaStream_t stream);
 
 // Skinny linear (gemm_skinny.cu): y = x W^T for all M <= 128 rows of x, plus u B^T on rows

@@ -935,6 +935,21 @@ bool make_tma_map(CUtensorMap* map, const void* base, int64_t rows, int64_t cols
   return r == CUDA_SUCCESS;
 }
 
+bool make_tma_map_3d(CUtensorMap* map, const void* base, int64_t cols, int64_t rows,
+                     int64_t planes, int64_t ld, int64_t plane_stride, int box_rows) {
+  EncodeTiledFn enc = get_encode_fn();
+  if (enc == nullptr) return false;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows),
+                        static_cast<cuuint64_t>(planes)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(ld) * 2, static_cast<cuuint64_t>(plane_stride) * 2};
+  cuuint32_t box[3] = {64, static_cast<cuuint32_t>(box_rows), 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
+                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 static bool make_map(CUtensorMap* map, const void* base, int64_t rows, int64_t cols,
                      int box_rows, bool f32) {
   return make_tma_map(map, base, rows, cols, cols, box_rows, f32);
