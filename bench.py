@@ -280,9 +280,10 @@ class HydraScoringLlama7B:
     seed = 4
     default_steps, default_warmup = 20, 3
     # DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) per GEMM launch, averaged over
-    # the 129 GEMM launches of one pass of this workload (batch 4, two streams) in a one-pass
-    # ncu capture of the current kernel; no figure for other shapes or stream counts
-    gemm_dram_bytes_per_launch = 520.6e6
+    # the 129 GEMM launches of one pass of this workload (batch 4, two streams): an ncu capture
+    # of one full-width decoder layer (its four GEMMs) and the LM head, scaled to 32 identical
+    # layers; no figure for other shapes or stream counts
+    gemm_dram_bytes_per_launch = 518.2e6
 
     def __init__(self, device, seed=4, reference=False):
         import torch
@@ -290,6 +291,8 @@ class HydraScoringLlama7B:
         self.llama = llama
         self.cfg = dict(llama.LLAMA7B)
         c = self.cfg
+        if getattr(self, "layers", None):  # fewer decoder layers: small profiling captures only
+            c["n_layers"] = self.layers
         if getattr(self, "shape", None):  # (prompt, response) of a variant workload
             c["prompt_len"], c["response_len"] = self.shape
         self.S, self.P0, self.L = getattr(self, "batch", 4), c["prompt_len"], c["response_len"]
@@ -357,7 +360,8 @@ class HydraScoringLlama7B:
 
     def traffic_per_launch(self):
         """The captured DRAM bytes per GEMM launch, for the exact workload they were taken on."""
-        if type(self) is HydraScoringLlama7B and self.S == 4 and not getattr(self, "shape", None):
+        if (type(self) is HydraScoringLlama7B and self.S == 4 and not getattr(self, "shape", None)
+                and self.cfg["n_layers"] == 32):
             return self.gemm_dram_bytes_per_launch
         return None
 
@@ -378,7 +382,7 @@ class HydraScoringLlama7B:
                 "profiled_ms_per_step": getattr(self, "profiled_ms_per_step", None)}
 
     def config(self):
-        return {"workload": f"{self.name}: random-init Llama-7B (32 layers, d 4096, 32 heads, "
+        return {"workload": f"{self.name}: random-init Llama-7B ({self.cfg['n_layers']} layers, d 4096, 32 heads, "
                             "SwiGLU 11008, vocab 32000, bf16), LoRA r=16 s=2 on q/v/gate/up/down, reward/"
                             f"value head 4096->1; batch {self.S} x ({self.P0} prompt + {self.L} response); "
                             "logp/KL beta 0.1, GAE gamma 1 lambda 0.95",
@@ -839,9 +843,19 @@ class KernelSweep:
         def rnd(*shape, std=0.02):
             return (std * torch.randn(*shape, device=dev, generator=g)).to(bf)
 
-        def graph_ms(launch, n):
+        def graph_ms(launch, n, tag=None):
             """Mean time per launch of n back-to-back launches replayed from a CUDA graph
-            (no host gaps between kernels)."""
+            (no host gaps between kernels). tag names an NVTX range around the measurement
+            (for profiler filters: the first launch inside it runs outside any graph)."""
+            if tag:
+                torch.cuda.nvtx.range_push(tag)
+            try:
+                return _graph_ms(launch, n)
+            finally:
+                if tag:
+                    torch.cuda.nvtx.range_pop()
+
+        def _graph_ms(launch, n):
             launch(0)  # first call outside capture (one-time kernel attribute set-up)
             torch.cuda.synchronize()
             graph = torch.cuda.CUDAGraph()
@@ -872,7 +886,8 @@ class KernelSweep:
                     xs = x[:, :K].contiguous()
                     y0 = torch.empty(M, N, dtype=bf, device=dev)
                     y1 = torch.empty(M, N, dtype=bf, device=dev)
-                    ms = graph_ms(lambda i: H.hydra_dual_linear(xs, None, Ws[i % 3], u, B, y0, y1, algo=1), reps)
+                    ms = graph_ms(lambda i: H.hydra_dual_linear(xs, None, Ws[i % 3], u, B, y0, y1, algo=1), reps,
+                                  tag=f"sweep:proj:{name}_r{r}")
                     tf = (2.0 * M * K * N + 2.0 * M * r * N) / ms / 1e9
                     out["projection_sweep"][f"{name}_r{r}"] = {"ms": ms, "TFLOP/s": tf}
                     fr.append(tf / peaks["bf16_tflops"])
@@ -895,7 +910,7 @@ class KernelSweep:
                     y0 = torch.empty(Mt, N, dtype=bf, device=dev)
                     y1 = torch.empty(Mt, N, dtype=bf, device=dev)
                     ms = graph_ms(lambda i: H.hydra_dual_linear(xd, None, Wd[i % ncopy], ud, Bd, y0, y1),
-                                  max(reps, 2 * ncopy))
+                                  max(reps, 2 * ncopy), tag=f"sweep:decode:{n}:M{Mt}")
                     byts = 2.0 * (N * K + 16 * (K + N) + Mt * K + 2 * Mt * N)
                     out["decode"].setdefault(f"M{Mt}", {})[n] = {"ms": ms, "GB/s": byts / ms / 1e6}
                     gb.append(byts / ms / 1e6)
@@ -952,7 +967,7 @@ class KernelSweep:
             H.ppo_gae(rw, vv, ln, 1.0, 0.95, adv, ret)
             valid = float(ln.sum().item())
         if "gae" in parts:
-            ms = graph_ms(lambda i: H.ppo_gae(rw, vv, ln, 1.0, 0.95, adv, ret), reps)
+            ms = graph_ms(lambda i: H.ppo_gae(rw, vv, ln, 1.0, 0.95, adv, ret), reps, tag="sweep:gae")
             byts = valid * 8 + S * L * 8 + S * 4  # read valid r, V; write all A, R
             out["gae"] = {"ms": ms, "GB/s": byts / ms / 1e6, "frac_of_measured_hbm": byts / ms / 1e6 / peaks["hbm_gbs"]}
         # ---- PPO losses at 65536 x 512, whitened: the moments pass reads the valid
@@ -981,7 +996,8 @@ class KernelSweep:
             nseq, Pq, Hh = 8, 768, 32
             qkv = torch.randn(nseq * Pq, 3 * Hh * 128, device=dev, generator=g).to(bf)
             att = torch.empty(nseq * Pq, Hh * 128, dtype=bf, device=dev)
-            ms = graph_ms(lambda i: H.hydra_causal_attention(qkv, nseq, Pq, Hh, 128, att), reps)
+            ms = graph_ms(lambda i: H.hydra_causal_attention(qkv, nseq, Pq, Hh, 128, att), reps,
+                          tag="sweep:attention")
             fl = 4.0 * nseq * Hh * 128 * (Pq * (Pq + 1) / 2)  # q k^T and p v over the causal half
             out["attention"] = {"ms": ms, "TFLOP/s": fl / ms / 1e9}
             del qkv, att
@@ -992,7 +1008,8 @@ class KernelSweep:
             zr = torch.randn(T, V, device=dev, generator=g)
             ids = torch.randint(0, V, (T,), device=dev, generator=g, dtype=torch.int32)
             o3 = [torch.empty(T, device=dev) for _ in range(3)]
-            ms = graph_ms(lambda i: H.hydra_token_logprobs_kl(za, zr, ids, None, None, 0.1, 4, 512, *o3), reps)
+            ms = graph_ms(lambda i: H.hydra_token_logprobs_kl(za, zr, ids, None, None, 0.1, 4, 512, *o3), reps,
+                          tag="sweep:logprobs")
             byts = T * V * 4 * 2 + T * 16
             out["logprobs"] = {"ms": ms, "GB/s": byts / ms / 1e6, "frac_of_measured_hbm": byts / ms / 1e6 / peaks["hbm_gbs"]}
         # ---- LoRA down-projection at the full pass's shapes (3072 on-stream rows: q/v and
@@ -1005,7 +1022,8 @@ class KernelSweep:
                 xs = [torch.randn(Mt, K, device=dev, generator=g).to(bf) for _ in range(ncopy)]
                 A = rnd(r, K)
                 u = torch.empty(Mt, r, dtype=bf, device=dev)
-                ms = graph_ms(lambda i: H.hydra_lora_down(xs[i % ncopy], A, 2.0, u), max(reps, 2 * ncopy))
+                ms = graph_ms(lambda i: H.hydra_lora_down(xs[i % ncopy], A, 2.0, u), max(reps, 2 * ncopy),
+                              tag=f"sweep:lora_down:{n}")
                 byts = 2.0 * (Mt * K + r * K + Mt * r)
                 out["lora_down"][n] = {"ms": ms, "GB/s": byts / ms / 1e6,
                                        "frac_of_measured_hbm": byts / ms / 1e6 / peaks["hbm_gbs"]}
@@ -1339,6 +1357,9 @@ def main(argv=None):
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default=DEFAULT_WORKLOAD)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", type=int, default=None,
+                    help="scoring workloads only: decoder layers (default 32); fewer layers make "
+                         "a small case for multi-pass profiler captures, never a bench value")
     ap.add_argument("--gen-steps", type=int, default=None,
                     help="generation workloads only: draws per call (default 64)")
     ap.add_argument("--gen-batch", type=int, default=None,
@@ -1347,6 +1368,10 @@ def main(argv=None):
                     help="kernel_sweep only: comma-separated subset of " + ",".join(KernelSweep.PARTS))
     args = ap.parse_args(argv)
     wl_cls = WORKLOADS[args.workload]
+    if args.layers is not None:
+        if not issubclass(wl_cls, HydraScoringLlama7B):
+            raise SystemExit("--layers applies to the scoring workloads only")
+        wl_cls.layers = args.layers
     if wl_cls is KernelSweep:
         return run_sweep(args)
     if args.impl == "reference":
