@@ -41,7 +41,7 @@ Parity pins for every function live in tests/test_oracle_pins.py (closed forms,
 invariants, brute force, library routines, hand-worked fixtures in tests/golden/).
 `set_storage_dither` (off by default) is a sensitivity probe used to derive the end-to-end
 tolerance of the multi-layer composition; it never changes the default results.
-The Llama composition (`llama_final_hidden`, under `llama_score` and the three-stream
+The Llama composition (`llama_final_hidden` over `llama_layer`, under `llama_score` and the three-stream
 Hydra-PPO pass `llama_score_hydra`) is pinned, with the bf16 storage rounding switched off,
 against the same architecture built from PyTorch library operations in fp64 (F.linear,
 F.rms_norm, causal F.scaled_dot_product_attention, F.silu, rotary as a complex rotation);
@@ -268,54 +268,60 @@ def swiglu(g, u):
     return silu(g) * u
 
 
-def llama_final_hidden(weights, ids, cfg, n_layers=None):
-    """Final normed hidden states (bf16 values) of both streams at every position of one
-    sequence: the decoder stack of the J-Hydra model (LoRA off / on, §3 Dynamic LoRA), as
-    used by llama_score; row p is the state after token p, which predicts token p + 1."""
+def llama_layer(weights, l, h_off, h_on, cfg):
+    """Decoder layer l of both streams (LoRA off / on, §3 Dynamic LoRA) on the residual
+    streams h_off, h_on [T, d] of one sequence (positions 0..T-1): pre-norm attention with
+    the rotary embedding, then the pre-norm SwiGLU feed-forward, each added into the residual
+    stream. Returns the new (h_off, h_on)."""
     d = cfg["d"]
     H = cfg["n_heads"]
     Dh = d // H
     eps = cfg["eps"]
     s = cfg["lora_scale"]
-    T = len(ids)
-    n_layers = cfg["n_layers"] if n_layers is None else n_layers
+    T = h_off.shape[0]
     pos = np.arange(T)
 
-    h_off = weights["embed"][np.asarray(ids)]
-    h_on = h_off.copy()
-
-    def lin(name, l, a_off, a_on):
+    def lin(name, a_off, a_on):
         W = weights[name][l]
         ab = weights["lora"].get(name)
         if ab is None:
             return dual_lora_linear(a_off, a_on, W, None, None, s)
         return dual_lora_linear(a_off, a_on, W, ab[0][l], ab[1][l], s)
 
-    for l in range(n_layers):
-        a_off = round_bf16(rmsnorm(h_off, weights["norm1"][l], eps))
-        a_on = round_bf16(rmsnorm(h_on, weights["norm1"][l], eps))
-        q = lin("wq", l, a_off, a_on)
-        k = lin("wk", l, a_off, a_on)
-        v = lin("wv", l, a_off, a_on)
-        att = []
-        for i in range(2):
-            qi = round_bf16(rope(q[i].reshape(T, H, Dh), pos, cfg["rope_theta"]))
-            ki = round_bf16(rope(k[i].reshape(T, H, Dh), pos, cfg["rope_theta"]))
-            vi = v[i].reshape(T, H, Dh)
-            att.append(round_bf16(causal_attention(qi, ki, vi).reshape(T, d)))
-        o = lin("wo", l, att[0], att[1])
-        h_off = h_off + o[0]
-        h_on = h_on + o[1]
-        a_off = round_bf16(rmsnorm(h_off, weights["norm2"][l], eps))
-        a_on = round_bf16(rmsnorm(h_on, weights["norm2"][l], eps))
-        g = lin("wg", l, a_off, a_on)
-        u = lin("wu", l, a_off, a_on)
-        m_off = round_bf16(swiglu(g[0], u[0]))
-        m_on = round_bf16(swiglu(g[1], u[1]))
-        dn = lin("wd", l, m_off, m_on)
-        h_off = h_off + dn[0]
-        h_on = h_on + dn[1]
+    a_off = round_bf16(rmsnorm(h_off, weights["norm1"][l], eps))
+    a_on = round_bf16(rmsnorm(h_on, weights["norm1"][l], eps))
+    q = lin("wq", a_off, a_on)
+    k = lin("wk", a_off, a_on)
+    v = lin("wv", a_off, a_on)
+    att = []
+    for i in range(2):
+        qi = round_bf16(rope(q[i].reshape(T, H, Dh), pos, cfg["rope_theta"]))
+        ki = round_bf16(rope(k[i].reshape(T, H, Dh), pos, cfg["rope_theta"]))
+        vi = v[i].reshape(T, H, Dh)
+        att.append(round_bf16(causal_attention(qi, ki, vi).reshape(T, d)))
+    o = lin("wo", att[0], att[1])
+    h_off = h_off + o[0]
+    h_on = h_on + o[1]
+    a_off = round_bf16(rmsnorm(h_off, weights["norm2"][l], eps))
+    a_on = round_bf16(rmsnorm(h_on, weights["norm2"][l], eps))
+    g = lin("wg", a_off, a_on)
+    u = lin("wu", a_off, a_on)
+    m_off = round_bf16(swiglu(g[0], u[0]))
+    m_on = round_bf16(swiglu(g[1], u[1]))
+    dn = lin("wd", m_off, m_on)
+    return h_off + dn[0], h_on + dn[1]
 
+
+def llama_final_hidden(weights, ids, cfg, n_layers=None):
+    """Final normed hidden states (bf16 values) of both streams at every position of one
+    sequence: the decoder stack of the J-Hydra model (LoRA off / on, §3 Dynamic LoRA), as
+    used by llama_score; row p is the state after token p, which predicts token p + 1."""
+    eps = cfg["eps"]
+    n_layers = cfg["n_layers"] if n_layers is None else n_layers
+    h_off = weights["embed"][np.asarray(ids)]
+    h_on = h_off.copy()
+    for l in range(n_layers):
+        h_off, h_on = llama_layer(weights, l, h_off, h_on, cfg)
     f_off = round_bf16(rmsnorm(h_off, weights["final_norm"], eps))
     f_on = round_bf16(rmsnorm(h_on, weights["final_norm"], eps))
     return f_off, f_on

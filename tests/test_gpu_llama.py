@@ -94,6 +94,27 @@ def test_causal_attention(nseq, P, H_, q_std):
         assert_rel(got[s * P:(s + 1) * P], ref, TOL_LINEAR, f"attention seq {s}")
 
 
+def test_causal_attention_strided_rows():
+    """Row strides above 3d (qkv) and d (output): only the heads' columns of the output are
+    written, each sequence's rows stay its own (the output is stored by sequence planes, so a
+    partial last query tile writes nothing into the next sequence)."""
+    nseq, P, H_, Dh = 3, 200, 2, 128
+    d = H_ * Dh
+    qkv_bits = synth.normal_bf16(537, (nseq * P, 3 * d + 64), 1.0)
+    out = torch.full((nseq * P, d + 64), float("nan"), dtype=torch.bfloat16, device="cuda")
+    H.hydra_causal_attention(dev_bf16(qkv_bits), nseq, P, H_, Dh, out)
+    x = f64(qkv_bits)
+    got = host_f64(out)
+    assert np.isnan(got[:, d:]).all(), "columns past the heads were written"
+    for s in range(nseq):
+        blk = x[s * P:(s + 1) * P]
+        q = blk[:, :d].reshape(P, H_, Dh)
+        k = blk[:, d:2 * d].reshape(P, H_, Dh)
+        v = blk[:, 2 * d:3 * d].reshape(P, H_, Dh)
+        ref = O.causal_attention(q, k, v).reshape(P, d)
+        assert_rel(got[s * P:(s + 1) * P, :d], ref, TOL_LINEAR, f"attention seq {s}")
+
+
 def test_swiglu_residual_head_dot():
     R, F, d = 70, 520, 256
     gu = synth.normal_bf16(541, (R, 2 * F), 2.0)
@@ -363,6 +384,136 @@ def test_score_llama7b_32_layers_against_oracle():
     torch.cuda.synchronize()
     got = {k: host_f64(v) for k, v in out.items()}
     check_pass(cfg, got, oracle_view(w, cfg), ids, lengths, derive_tol=True)
+    del w, ws
+    torch.cuda.empty_cache()
+
+
+def test_score_llama7b_every_kernel_of_every_layer_against_oracle():
+    """Every kernel of each of the 32 decoder layers of the benchmark's model at full width
+    (Llama-7B shapes, LoRA r 16, the benchmark's generator and seed), on one sequence of 256
+    prompt + 512 response tokens, against the oracle's step given the GPU's own input to that
+    kernel, within the stated tolerance for linear outputs (2e-2 max(1, |ref|); the o and down
+    projections are checked on what their epilogue added into the fp32 residual stream, the
+    rotary outputs relative to the norm of each rotated pair, the SwiGLU output after the
+    propagated one-ulp differences of its two unstored bf16 inputs). The
+    layers run through the library's per-op entry points (the kernels
+    and arguments hydra_score_llama launches), and the residual stream they leave after layer
+    32 equals, bit for bit, the one the full pass leaves in its workspace (whose first bytes
+    hold the fp32 residual stream): every kernel launch of the pass's decoder stack is checked
+    at its own full size, without the drift that a chain of bf16 stages accumulates (steps of
+    Algorithm 1's scoring pass; §3 Dynamic LoRA: both streams)."""
+    cfg = dict(llama.LLAMA7B)
+    nl, d, F, r, nh = cfg["n_layers"], cfg["d_model"], cfg["ffn"], cfg["lora_rank"], cfg["n_heads"]
+    P0, L = cfg["prompt_len"], cfg["response_len"]
+    P, S = P0 + L, 1
+    T = S * P
+    s, eps, Dh = cfg["lora_scale"], cfg["rms_eps"], cfg["head_dim"]
+    w = llama.random_device_weights(cfg, 4, "cuda")
+    ids = torch.from_numpy(synth.randint(4201, (S, P), 0, cfg["vocab"])).cuda()
+    bf = torch.bfloat16
+    # the pass itself
+    ws = torch.empty(H.score_llama_workspace_size(cfg, S), dtype=torch.uint8, device="cuda")
+    out = llama.alloc_outputs(S, L, "cuda")
+    H.hydra_score_llama(cfg, w, ids, None, ws, out)
+    torch.cuda.synchronize()
+    h_pass = ws[:2 * T * d * 4].view(torch.float32).view(2 * T, d).clone()
+    # the same layers through the per-op entry points
+    h = torch.empty(2 * T, d, device="cuda")
+    H.hydra_embed(w["embed"], ids.view(-1), 2, h)
+    table = torch.empty(P, Dh // 2, 2, device="cuda")
+    H.hydra_rope_table(P, Dh, cfg["rope_theta"], table)
+    a = torch.empty(2 * T, d, dtype=bf, device="cuda")
+    qkv = torch.empty(2 * T, 3 * d, dtype=bf, device="cuda")
+    attn = torch.empty(2 * T, d, dtype=bf, device="cuda")
+    m = torch.empty(2 * T, F, dtype=bf, device="cuda")
+    u2 = torch.empty(T, 2 * r, dtype=bf, device="cuda")
+    u1 = torch.empty(T, r, dtype=bf, device="cuda")
+    view = oracle_view(w, cfg)
+    pos = np.arange(P)
+    worst = {}
+
+    def check(name, got, ref, scale=None, extra=None):
+        # relative to max(1, |ref|), or to a given scale, after an allowed extra difference
+        sc = np.maximum(1.0, np.abs(ref) if scale is None else scale)
+        diff = np.abs(got - ref) if extra is None else np.maximum(np.abs(got - ref) - extra, 0.0)
+        e = float(np.max(diff / sc))
+        worst[name] = max(worst.get(name, 0.0), e)
+        assert np.all(np.isfinite(got)), f"{name}, layer {l}: non-finite output"
+        assert e <= TOL_LINEAR, f"{name}, layer {l}: max |err| / scale = {e:.3e} > {TOL_LINEAR:.0e}"
+
+    def pair_norm(x):
+        # rotary outputs: relative to the norm of each rotated pair (dims i, i + Dh/2 of a
+        # head), which the rotation preserves; a one-ulp difference of the linear output
+        # before the rotation is relative to that norm, not to the smaller rotated component
+        y = x.reshape(T, nh, 2, Dh // 2)
+        n = np.sqrt(y[:, :, 0] ** 2 + y[:, :, 1] ** 2)
+        return np.concatenate([n, n], axis=-1).reshape(T, nh * Dh)
+
+    for l in range(nl):
+        lw = view["wq"][l]  # noqa: F841  (widens layer l's weights once)
+        lo = view["lora"]
+        h_in = host_f64(h)
+        H.hydra_rmsnorm(h, w["norm_attn"][l], eps, a)
+        H.hydra_lora_down(a[T:], w["a_qv"][l], s, u2)
+        H.hydra_dual_linear_rope(a[:T], a[T:], w["w_qkv"][l], u2, w["b_qkv"][l], qkv[:T], qkv[T:],
+                                 P, 2 * d, Dh, table)
+        H.hydra_causal_attention(qkv, 2 * S, P, nh, Dh, attn)
+        a1, g_u2, g_qkv, g_attn = host_f64(a), host_f64(u2), host_f64(qkv), host_f64(attn)
+        H.hydra_dual_linear_ex(attn[:T], attn[T:], w["w_o"][l], None, None, h[:T], h[T:],
+                               H.EPI_RESIDUAL)
+        h_mid = host_f64(h)
+        H.hydra_rmsnorm(h, w["norm_ffn"][l], eps, a)
+        H.hydra_lora_down(a[T:], w["a_gu"][l], s, u2)
+        H.hydra_dual_linear_ex(a[:T], a[T:], w["w_gu"][l], u2, w["b_gu"][l], m[:T], m[T:],
+                               H.EPI_SWIGLU)
+        H.hydra_lora_down(m[T:], w["a_down"][l], s, u1)
+        H.hydra_dual_linear_ex(m[:T], m[T:], w["w_down"][l], u1, w["b_down"][l], h[:T], h[T:],
+                               H.EPI_RESIDUAL)
+        a2, g_ugu, g_m, g_ud, h_out = host_f64(a), host_f64(u2), host_f64(m), host_f64(u1), host_f64(h)
+
+        # attention block, each kernel from its own GPU input
+        check("rmsnorm (attention)", a1, O.round_bf16(O.rmsnorm(h_in, view["norm1"][l], eps)))
+        A_q, A_v = lo["wq"][0][l], lo["wv"][0][l]
+        check("lora_down q/v", g_u2, O.lora_down(a1[T:], np.concatenate([A_q, A_v]), s))
+        q = O.dual_lora_linear(a1[:T], a1[T:], view["wq"][l], A_q, lo["wq"][1][l], s)
+        k = O.dual_lora_linear(a1[:T], a1[T:], view["wk"][l], None, None, s)
+        v = O.dual_lora_linear(a1[:T], a1[T:], view["wv"][l], A_v, lo["wv"][1][l], s)
+        for i in range(2):
+            rows = slice(i * T, (i + 1) * T)
+            rq = O.round_bf16(O.rope(q[i].reshape(T, nh, Dh), pos, cfg["rope_theta"])).reshape(T, d)
+            rk = O.round_bf16(O.rope(k[i].reshape(T, nh, Dh), pos, cfg["rope_theta"])).reshape(T, d)
+            check("q/k/v linear + rotary, q", g_qkv[rows, :d], rq, pair_norm(rq))
+            check("q/k/v linear + rotary, k", g_qkv[rows, d:2 * d], rk, pair_norm(rk))
+            check("q/k/v linear, v", g_qkv[rows, 2 * d:], v[i])
+            qq = g_qkv[rows, :d].reshape(T, nh, Dh)
+            kk = g_qkv[rows, d:2 * d].reshape(T, nh, Dh)
+            vv = g_qkv[rows, 2 * d:].reshape(T, nh, Dh)
+            check("causal attention", g_attn[rows], O.round_bf16(O.causal_attention(qq, kk, vv)).reshape(T, d))
+        o = O.dual_lora_linear(g_attn[:T], g_attn[T:], view["wo"][l], None, None, s)
+        # the linear output (what the residual epilogue added), against the stated tolerance
+        check("o linear (added into the residual stream)", h_mid - h_in, np.concatenate(o))
+        # feed-forward block
+        check("rmsnorm (feed-forward)", a2, O.round_bf16(O.rmsnorm(h_mid, view["norm2"][l], eps)))
+        A_g, A_u = lo["wg"][0][l], lo["wu"][0][l]
+        check("lora_down gate/up", g_ugu, O.lora_down(a2[T:], np.concatenate([A_g, A_u]), s))
+        g_ = O.dual_lora_linear(a2[:T], a2[T:], view["wg"][l], A_g, lo["wg"][1][l], s)
+        u_ = O.dual_lora_linear(a2[:T], a2[T:], view["wu"][l], A_u, lo["wu"][1][l], s)
+        # the fused epilogue rounds gate and up to bf16 (as the oracle does) without storing
+        # them: a one-ulp difference of either, which a different fp32 summation order may
+        # give, reaches the SwiGLU output as |silu'(g) u| ulp(g) + |silu(g)| ulp(u)
+        gg, uu = np.concatenate(g_), np.concatenate(u_)
+        sig = 1.0 / (1.0 + np.exp(-gg))
+        dsilu = sig * (1.0 + gg * (1.0 - sig))
+        ulp = lambda x: np.exp2(np.floor(np.log2(np.maximum(np.abs(x), 1e-30))) - 7)  # noqa: E731
+        check("gate/up linear + SwiGLU", g_m,
+              np.concatenate([O.round_bf16(O.swiglu(g_[i], u_[i])) for i in range(2)]),
+              extra=np.abs(dsilu * uu) * ulp(gg) + np.abs(gg * sig) * ulp(uu))
+        check("lora_down down", g_ud, O.lora_down(g_m[T:], lo["wd"][0][l], s))
+        dn = O.dual_lora_linear(g_m[:T], g_m[T:], view["wd"][l], lo["wd"][0][l], lo["wd"][1][l], s)
+        check("down linear (added into the residual stream)", h_out - h_mid, np.concatenate(dn))
+    assert torch.equal(h, h_pass), "the per-op composition differs from the pass"
+    print("worst relative error per kernel over 32 layers (stated 2e-2): " +
+          ", ".join(f"{k} {v:.1e}" for k, v in worst.items()))
     del w, ws
     torch.cuda.empty_cache()
 
