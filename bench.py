@@ -270,6 +270,18 @@ class LmHeadScoring:
         return n
 
 
+def oracle_layer_times(timer, smp, steps, warmup):
+    """(t_head, [t_1 ...]): times of the oracle slice with no decoder layer (median of three)
+    and with one decoder layer (`steps` samples). Both depths run once untimed first, so that
+    neither carries the first call's thread start-up and page faults (a cold first call had
+    made the head look slower than head + layer)."""
+    timer(smp, 0)
+    for _ in range(max(warmup, 1)):
+        timer(smp, 1)
+    t_head = statistics.median(timer(smp, 0) for _ in range(3))
+    return t_head, [timer(smp, 1) for _ in range(steps)]
+
+
 class HydraScoringLlama7B:
     """Full J-Hydra scoring pass on a random-init Llama-7B (32 layers, d 4096, 32 heads,
     SwiGLU 11008, vocab 32000, bf16), LoRA r=16 on q/v/gate/up/down (s = 2), reward head
@@ -440,10 +452,7 @@ class HydraScoringLlama7B:
         """(tokens/s, description): the slice's pass time is t(0 layers) + 32 (t(1) - t(0)); a
         quarter-size slice on one BLAS thread."""
         smp = self.oracle_sample(1, prompt=16, resp=32) if single_thread else self.oracle_sample(1)
-        for _ in range(warmup):
-            self.oracle_time(smp, 1)
-        t_head = self.oracle_time(smp, 0)
-        t1 = [self.oracle_time(smp, 1) for _ in range(steps)]
+        t_head, t1 = oracle_layer_times(self.oracle_time, smp, steps, warmup)
         self.oracle_timed = {"head_s": t_head, "sample_s": t1}
         n = self.cfg["n_layers"]
         t_pass = [t_head + n * max(t - t_head, 0.0) for t in t1]
@@ -654,10 +663,7 @@ class HydraGenerateLlama7B(HydraScoringLlama7B):
         """(tokens/s, description): 2 draws after a 32-token prompt, per-draw time t(0 layers)
         + 32 (t(1) - t(0)), the oracle recomputing the whole prefix at each draw."""
         smp = self.oracle_sample(1)
-        for _ in range(warmup):
-            self.oracle_time(smp, 1)
-        t_head = self.oracle_time(smp, 0)
-        t1 = [self.oracle_time(smp, 1) for _ in range(steps)]
+        t_head, t1 = oracle_layer_times(self.oracle_time, smp, steps, warmup)
         self.oracle_timed = {"head_s": t_head, "sample_s": t1}
         n = self.cfg["n_layers"]
         t_gen = [t_head + n * max(t - t_head, 0.0) for t in t1]
@@ -790,10 +796,7 @@ class HydraPPOIterationLlama7B(HydraGenerateLlama7B):
 
     def oracle_throughput(self, steps=1, single_thread=False, warmup=0):
         smp = self.oracle_sample(1)
-        for _ in range(warmup):
-            self.oracle_time(smp, 1)
-        t_head = self.oracle_time(smp, 0)
-        t1 = [self.oracle_time(smp, 1) for _ in range(steps)]
+        t_head, t1 = oracle_layer_times(self.oracle_time, smp, steps, warmup)
         self.oracle_timed = {"head_s": t_head, "sample_s": t1}
         n = self.cfg["n_layers"]
         t_it = [t_head + n * max(t - t_head, 0.0) for t in t1]

@@ -12,14 +12,17 @@
 //  * warp 0 moves Q_a, Q_b per unit and the K / V blocks through one 3-stage ring with TMA
 //    (128-byte swizzle, [128 rows x 64] boxes), in the order the tiles first use them
 //    (K_0, V_0, K_1, V_1, ...); the ring runs on across units, and the next unit's first
-//    blocks are prefetched into L2 a few blocks before a unit ends. Warp 1 owns TMEM (S_a,
+//    blocks are prefetched into L2 a few blocks before a unit ends (in the longest-first unit
+//    order; see UnitCursor). Warp 1 owns TMEM (S_a,
 //    S_b, O_a, O_b: 4 x 128 fp32 columns);
 //  * warps 4..7 (tile a) and 8..11 (tile b) each run their tile: thread i owns query row i
 //    (TMEM lane i), so row maxima and sums need no shuffles, and the group's first warp issues
 //    the tile's tcgen05.mma from one elected lane: per key block j, S_x = Q_x K_j^T, then,
 //    once the softmax has written P_x as bf16 pairs over the first 64 columns of S_x,
 //    O_x += P_x V_j (P_x is the A operand, read from TMEM, so it costs no shared-memory
-//    bandwidth) and S_x = Q_x K_{j+1}^T after that P V has finished reading P_x. A finished
+//    bandwidth) and S_x = Q_x K_{j+1}^T right behind it: the tcgen05.mma operations one
+//    thread issues execute in issue order, so the next S, which overwrites the columns of
+//    P_x, cannot overtake the P V products that read them. A finished
 //    tile is normalised into a staging buffer and stored with TMA (one 128-byte line per row
 //    of a box rather than 16-byte pieces of 128 rows), while the tile's next unit runs. The running
 //    maximum is a reference value that moves only when a row's maximum grows by more than
@@ -28,6 +31,9 @@
 // The probabilities enter P V as bf16 (8 mantissa bits, relative error at most 2^-9); the row
 // sum l accumulates them in fp32.
 #include <float.h>
+
+#include <algorithm>
+#include <vector>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -206,27 +212,41 @@ __device__ __forceinline__ void tc_mma_ts_bf16(uint32_t d_tmem, uint32_t a_tmem,
 }
 
 
-// This CTA's work: units t = blockIdx.x + i * gridDim.x (i = 0, 1, ...) of the ordering
-// t -> (query-block pair p, head, sequence) with the largest p (most key blocks) first, so the
-// static round-robin assignment stays balanced. Unit (p, head, seq) holds the two query tiles
-// qa = 2p and qb = 2p + 1 (qb only when it exists): tile a runs key blocks 0..qa, tile b
-// 0..qb, and every key block the two share is loaded once for both.
+// This CTA's work: units t = blockIdx.x + i * gridDim.x (i = 0, 1, ...). Unit (p, head, seq)
+// holds the two query tiles qa = 2p and qb = 2p + 1 (qb only when it exists): tile a runs key
+// blocks 0..qa, tile b 0..qb, and every key block the two share is loaded once for both. Two
+// orders of the units t:
+//  * longest first: t -> (p, head, seq) with the largest p (most key blocks) first;
+//  * grouped: the units of one (head, sequence) consecutive, longest first within it, so
+//    that they run at the same time on neighbouring CTAs and read the key / value blocks
+//    they share from DRAM once (the longest-first order runs them waves apart, when the
+//    blocks have left L2).
+// The launcher takes the grouped order unless it raises the busiest CTA's load (in key
+// blocks) of the static round-robin assignment by more than 5 % over the longest-first order.
 struct UnitCursor {
   int t;               // unit
   int p, head, seq;    // decoded unit
   int na, nb, nblk;    // key blocks of tile a, of tile b (0: no tile b), of the unit
   // the loop-invariant sizes are recomputed from the kernel arguments (constant bank) rather
   // than kept in registers: the producer and MMA warps run with few registers
-  __device__ static int units(int P, int heads, int nseq) {
+  __host__ __device__ static int units(int P, int heads, int nseq) {
     return (((P + kBQ - 1) / kBQ + 1) / 2) * heads * nseq;
   }
-  __device__ void decode(int P, int heads, int nseq) {
+  __host__ __device__ void decode(int P, int heads, int nseq, int grouped) {
     const int nqb = (P + kBQ - 1) / kBQ;
-    const int hs = heads * nseq;
-    p = (nqb + 1) / 2 - 1 - t / hs;
-    const int r = t % hs;
-    head = r % heads;
-    seq = r / heads;
+    const int npairs = (nqb + 1) / 2;
+    if (grouped) {
+      const int g = t / npairs;
+      p = npairs - 1 - t % npairs;
+      head = g % heads;
+      seq = g / heads;
+    } else {
+      const int hs = heads * nseq;
+      p = npairs - 1 - t / hs;
+      const int r = t % hs;
+      head = r % heads;
+      seq = r / heads;
+    }
     na = 2 * p + 1;
     nb = (2 * p + 1 < nqb) ? 2 * p + 2 : 0;
     nblk = nb > 0 ? nb : na;
@@ -236,7 +256,7 @@ struct UnitCursor {
 __global__ void __launch_bounds__(kThreads, 1)
     causal_attention_tc_kernel(const __grid_constant__ CUtensorMap tm_qkv,
                                const __grid_constant__ CUtensorMap tm_out, int P, int d,
-                               int n_heads, int nseq, float scale_log2, int* err) {
+                               int n_heads, int nseq, int grouped, float scale_log2, int* err) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -295,7 +315,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tma_prefetch_desc(&tm_out);
       }
       __syncwarp();
-      UnitCursor c;
+      UnitCursor c = {};
       int pos = 0, nq[2] = {0, 0};  // ring positions filled, Q tiles loaded per tile
       bool ok = true;
       auto load_q = [&](int x) {
@@ -336,7 +356,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         UnitCursor nx;
         nx.t = c.t + gridDim.x;
         if (nx.t >= nunits || !elect_one()) return;
-        nx.decode(P, n_heads, nseq);
+        nx.decode(P, n_heads, nseq, grouped);
         const int y0 = nx.seq * P;
         for (int x = 0; x < (nx.nb > 0 ? 2 : 1); ++x)
           for (int h = 0; h < 2; ++h)
@@ -347,8 +367,10 @@ __global__ void __launch_bounds__(kThreads, 1)
               tma_prefetch_l2_2d(&tm_qkv, kv * d + nx.head * kDh + 64 * h, y0 + j * kBK);
       };
       for (c.t = blockIdx.x; ok && c.t < nunits; c.t += gridDim.x) {
-        c.decode(P, n_heads, nseq);
-        const int jpf = c.nblk > 3 ? c.nblk - 3 : 0;  // prefetch after this block's loads
+        c.decode(P, n_heads, nseq, grouped);
+        // prefetch after this block's loads (longest-first order only: with the grouped
+        // order the next unit's blocks are mostly in L2 already, and the prefetch measured slower)
+        const int jpf = grouped ? -1 : (c.nblk > 3 ? c.nblk - 3 : 0);
         ok = load_q(0) && load_kv(1, 0);
         if (ok && c.nb > 0) ok = load_q(1);
         if (ok) ok = load_kv(2, 0);
@@ -374,8 +396,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     // -------------------------------------------------------------- tiles (warps 4..11)
     // Warps 4..7 own tile a, warps 8..11 tile b; thread i of a group owns query row i (TMEM
     // lane i). Each group runs its tile's softmax and issues the tile's products itself:
-    // once P_x is in TMEM, one of its warps issues P_x V_j and then Q_x K_{j+1}^T (after that
-    // P V has finished reading P_x, which the next S overwrites), so no other warp sits on
+    // once P_x is in TMEM, one of its warps issues P_x V_j and then Q_x K_{j+1}^T (in issue
+    // order behind the P V products that read P_x, which the next S overwrites), so no other
+    // warp sits on
     // the path from a finished P to the tensor pipe. The two groups' products interleave on
     // the pipe: one tile's softmax overlaps the other tile's products.
     const int x = warp < 8 ? 0 : 1;
@@ -388,7 +411,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t t_s = t_lane + kColS + x * 128;
     const uint32_t t_o = t_lane + kColO + x * kDh;
     const uint32_t s_stage = sbase + kOffOut + x * kMat;  // this tile's output staging
-    int gs = 0, gpv = 0, nqu = 0;             // S consumed, P V issued, units begun (Q tiles)
+    int gs = 0, nqu = 0;                      // S consumed, units begun (Q tiles)
     int kbase = 0;                            // ring block index of the unit's key block 0
     bool s0_issued = false;                   // this unit's first Q K^T was issued already
     bool ok = true;
@@ -398,9 +421,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         return false;
       const int st = kpos % kStages;
       if (!warp_wait_bounded(kv_full(st), (kpos / kStages) & 1, abort_flag, err, kDevTimeoutMma))
-        return false;
-      if (gpv >= 1 &&
-          !warp_wait_bounded(pv_done(x), (gpv - 1) & 1, abort_flag, err, kDevTimeoutMma))
         return false;
       tc_fence_after();
       if (elect_one()) {
@@ -437,14 +457,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int i = 0; i < rel; ++i) tc_commit(kv_empty(st));
       }
       __syncwarp();
-      ++gpv;
       return true;
     };
     float m_ref = -FLT_MAX;                   // reference maximum, log2 domain
     float l = 0.f;                            // row sum of the probabilities
     UnitCursor c;
     for (c.t = blockIdx.x; ok && c.t < nunits; c.t += gridDim.x) {
-      c.decode(P, n_heads, nseq);
+      c.decode(P, n_heads, nseq, grouped);
       const int n = x == 0 ? c.na : c.nb;     // this tile's key blocks (0: no tile b)
       const int on = x == 0 ? c.nb : c.na;    // the other tile's
       const int J = c.nblk;
@@ -539,7 +558,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             nx.t = c.t + gridDim.x;
             s0_issued = false;
             if (nx.t < nunits) {
-              nx.decode(P, n_heads, nseq);
+              nx.decode(P, n_heads, nseq, grouped);
               const int nn = x == 0 ? nx.na : nx.nb, non = x == 0 ? nx.nb : nx.na;
               if (nn > 0) {
                 ok = issue_s(true, 2 * (kbase + J), non > 0 ? 1 : 2, nn == 1);
@@ -550,7 +569,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       if (!ok) break;
-      // the finished tile (its last P V, the gs-th, is done): O_x / l as bf16 rows, staged in
+      // the finished tile (its last P V, the gs-th, is done; the parity wait cannot alias an
+      // older phase: the tile's last S completed after every earlier product of the issuing
+      // thread, so only this P V can be outstanding): O_x / l as bf16 rows, staged in
       // shared memory as two 128-byte-swizzled TMA boxes of 64 columns and stored with TMA;
       // the staging buffer is reused only once the stores of the previous unit have read it
       if (issuer) {
@@ -633,10 +654,34 @@ int launch_causal_attention(const void* qkv, int64_t nseq, int64_t P, int64_t ld
   if (!make_tma_map_3d(&map_out, out, d, P, nseq, ld_out, P * ld_out, kBQ)) return -2;
   const int64_t nunits = ((P + 2 * kBQ - 1) / (2 * kBQ)) * n_heads * nseq;
   const unsigned grid = static_cast<unsigned>(nunits < nsm ? nunits : nsm);
+  // unit order: grouped unless it loads the busiest CTA of the static round-robin assignment
+  // with more than 5 % more key blocks than the longest-first order does (its shared reads
+  // measured worth that much: 8 x 768 x 32 heads, equal loads, 64 -> 58 us; 16 x 768 x 32
+  // heads, 46 against 44 blocks, 119 -> 102 us; 16 x 300 x 12 heads, 9 against 8, slower).
+  // The choice for the last shape is kept.
+  struct OrderChoice {
+    int64_t nseq, P, heads;
+    unsigned grid;
+    int grouped;
+  };
+  static thread_local OrderChoice last = {-1, -1, -1, 0, 0};
+  if (last.nseq != nseq || last.P != P || last.heads != n_heads || last.grid != grid) {
+    auto busiest = [&](int grouped) {
+      std::vector<int64_t> load(grid, 0);
+      UnitCursor c;
+      for (int64_t t = 0; t < nunits; ++t) {
+        c.t = static_cast<int>(t);
+        c.decode(static_cast<int>(P), static_cast<int>(n_heads), static_cast<int>(nseq), grouped);
+        load[t % grid] += c.nblk;
+      }
+      return *std::max_element(load.begin(), load.end());
+    };
+    last = {nseq, P, n_heads, grid, busiest(1) * 20 <= busiest(0) * 21 ? 1 : 0};
+  }
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(head_dim));
   causal_attention_tc_kernel<<<grid, kThreads, kSmem, st>>>(
       map, map_out, static_cast<int>(P), static_cast<int>(d), static_cast<int>(n_heads),
-      static_cast<int>(nseq), scale_log2, err);
+      static_cast<int>(nseq), last.grouped, scale_log2, err);
   return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
 }
 
