@@ -106,6 +106,16 @@ class ClockSampler:
                 stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
         except OSError:
             self.proc = None
+        # the timed region opens only once nvidia-smi has written its first sample: its
+        # start-up (NVML initialisation) was seen to stall the GPU work submitted meanwhile
+        t0 = time.time()
+        while self.proc is not None and time.time() - t0 < 10.0:
+            if self.proc.poll() is not None:
+                break
+            with open(self.path) as f:
+                if f.readline():
+                    break
+            time.sleep(0.05)
         time.sleep(0.15)
 
     def stop(self):
@@ -295,7 +305,7 @@ class HydraScoringLlama7B:
     # the 129 GEMM launches of one pass of this workload (batch 4, two streams): an ncu capture
     # of one full-width decoder layer (its four GEMMs) and the LM head, scaled to 32 identical
     # layers; no figure for other shapes or stream counts
-    gemm_dram_bytes_per_launch = 518.2e6
+    gemm_dram_bytes_per_launch = 496.7e6
 
     def __init__(self, device, seed=4, reference=False):
         import torch

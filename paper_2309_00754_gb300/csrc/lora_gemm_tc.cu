@@ -1064,13 +1064,17 @@ int launch_dual_lora_gemm_tc(const GemmArgs& a, cudaStream_t stream) {
   // pair) cover every m-tile of a few n-columns: x stays in L2 if it fits, else it is read
   // again for each column (a 3072 x 11008 down-projection input of both streams, 135 MB,
   // measured 1026 MB of DRAM reads per launch). Beyond half of L2, m-tiles go in groups
-  // whose inputs total about 48 MB, and W is read once per group instead.
+  // whose inputs total about 48 MB, and W is read once per group instead. From 40 MB of
+  // input (the 50 MB q/k/v, o and gate/up inputs of both streams), groups of about 24 MB:
+  // x then stays while W is read twice (measured DRAM reads per launch: q/k/v 336 -> 280 MB,
+  // o 252 -> 235 MB, gate/up 457 -> 436 MB; groups of 12 MB re-read W too often).
   p.m_group = 0;
   if (pair) {
     const int64_t x_bytes = static_cast<int64_t>(p.streams) * a.M * a.K * 2;
     const int64_t mtile_bytes = static_cast<int64_t>(p.streams) * 256 * a.K * 2;
-    if (x_bytes > (int64_t{64} << 20) && p.m_tiles > 1) {
-      const int64_t g = (int64_t{48} << 20) / mtile_bytes;
+    if (x_bytes > (int64_t{40} << 20) && p.m_tiles > 1) {
+      const int64_t budget = x_bytes > (int64_t{64} << 20) ? (int64_t{48} << 20) : (int64_t{24} << 20);
+      const int64_t g = budget / mtile_bytes;
       p.m_group = static_cast<int>(g < 1 ? 1 : (g > p.m_tiles ? p.m_tiles : g));
       if (p.m_group >= p.m_tiles) p.m_group = 0;
     }

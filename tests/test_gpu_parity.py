@@ -224,8 +224,15 @@ def test_lora_off_switch_is_bitwise(algo):
     assert torch.equal(y_off2, y_on2) and torch.equal(y_off2, y_off)
 
 
-def test_stacked_equals_separate_calls_bitwise():
-    M, K, N, r = 260, 384, 520, 16
+@pytest.mark.parametrize("M,K,N", [
+    (260, 384, 520),
+    (2600, 4096, 1000),   # stacked input 43 MB: groups of 6 m-tiles over 11 (6 + 5)
+    (2600, 11008, 512),   # stacked input 114 MB: groups of 4 over 11 (4 + 4 + 3); each
+])                        # stream's own input 57 MB: groups of 4 in the separate calls
+def test_stacked_equals_separate_calls_bitwise(M, K, N):
+    """Stacked streams, separate calls and the grouped tile orders run the same per-tile
+    arithmetic, so their outputs agree bit for bit."""
+    r = 16
     x, x2, W, A, Bm = _linear_problem(M, K, N, r, seed=24)
     d = [dev_bf16(t) for t in (x, x2, W, A, Bm)]
     st_off, st_on = _run_linear(d[0], d[1], d[2], d[3], d[4], 2.0)
@@ -233,6 +240,11 @@ def test_stacked_equals_separate_calls_bitwise():
     _, sep_on = _run_linear(d[1], None, d[2], d[3], d[4], 2.0)
     assert torch.equal(st_off, sep_off)
     assert torch.equal(st_on, sep_on)
+    if M > 1000:  # the grouped orders against the oracle on sampled rows
+        rows = sample_rows(M + N, M)
+        ref_off, ref_on = O.dual_lora_linear(f64(x[rows]), f64(x2[rows]), f64(W), f64(A), f64(Bm), 2.0)
+        assert_rel(host_f64(st_off[rows]), ref_off, TOL_LINEAR, "y_off")
+        assert_rel(host_f64(st_on[rows]), ref_on, TOL_LINEAR, "y_on")
 
 
 def test_gemv_and_tensor_core_kernel_agree():
