@@ -77,10 +77,8 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
 // scores of the npos = pos + 1 cached keys into shared memory
 // (groups of 8 lanes per key, 32 bytes each, reduced by shuffles), the softmax over them,
 // then the weighted sum of the values (lane = 4 output dimensions, warps split positions).
-// kPrefetch: the key loads of the next iteration are issued before this one's are reduced,
-// for small batches (latency-bound); without it, each iteration loads its own keys (large
-// batches, bound by HBM bandwidth, measured faster that way).
-template <bool kPrefetch>
+// Each iteration loads its own keys: for large batches, bound by HBM bandwidth (small batches
+// take decode_attention_1p_kernel below).
 __global__ void __launch_bounds__(kAttnThreads)
     decode_attention_kernel(const __nv_bfloat16* __restrict__ qkv, int ld, int d, int H,
                             const float2* __restrict__ table, __nv_bfloat16* __restrict__ ck,
@@ -136,8 +134,7 @@ __global__ void __launch_bounds__(kAttnThreads)
     }
   }
   // warp-uniform trip count: all 32 lanes reach the shuffles. Each 8-lane group takes two
-  // keys per iteration, both loaded before either is reduced (with kPrefetch, the next
-  // iteration's keys are loaded before this one's are reduced).
+  // keys per iteration, both loaded before either is reduced.
   constexpr int kKeysPerIter = 2 * 4 * kAttnWarps;
   auto load_keys = [&](int base, uint4 (&kk)[4]) {
     const int q0 = base + g, q1 = base + 4 * kAttnWarps + g;
@@ -153,19 +150,11 @@ __global__ void __launch_bounds__(kAttnThreads)
       kk[3] = __ldcs(reinterpret_cast<const uint4*>(kr + 8));
     }
   };
-  uint4 cur[4], nxt[4];
-#pragma unroll
-  for (int e = 0; e < 4; ++e) nxt[e] = make_uint4(0u, 0u, 0u, 0u);
-  if (kPrefetch) load_keys(warp * 4, cur);
+  uint4 cur[4];
   for (int base = warp * 4; base < npos; base += kKeysPerIter) {
     const int p0 = base + g, p1 = base + 4 * kAttnWarps + g;
-    if (!kPrefetch) load_keys(base, cur);
-    else if (base + kKeysPerIter < npos) load_keys(base + kKeysPerIter, nxt);  // warp-uniform
+    load_keys(base, cur);
     const uint4 a0 = cur[0], b0 = cur[1], a1 = cur[2], b1 = cur[3];
-    if (kPrefetch) {
-#pragma unroll
-      for (int e = 0; e < 4; ++e) cur[e] = nxt[e];
-    }
     const uint32_t w0[8] = {a0.x, a0.y, a0.z, a0.w, b0.x, b0.y, b0.z, b0.w};
     const uint32_t w1[8] = {a1.x, a1.y, a1.z, a1.w, b1.x, b1.y, b1.z, b1.w};
     float acc0 = 0.f, acc1 = 0.f;
@@ -220,6 +209,154 @@ __global__ void __launch_bounds__(kAttnThreads)
   }
 }
 
+
+// Single-pass form for small batches: 32 groups of 8 lanes per block (lane = 16 dimensions of
+// a key or value row); group G takes positions G + 32 t, two per iteration, and the K and V
+// loads of the next iteration are issued before this one's are reduced. Each group keeps a
+// lazily rescaled running maximum (moved only when a score exceeds it by more than 2^8, as in
+// the prefill's flash attention), its sum and its 16-dimension slice of the weighted values;
+// the 32 partial results meet in shared memory at the end.
+constexpr int kAttnGroups = kAttnThreads / 8;
+__global__ void __launch_bounds__(kAttnThreads)
+    decode_attention_1p_kernel(const __nv_bfloat16* __restrict__ qkv, int ld, int d, int H,
+                               const float2* __restrict__ table, __nv_bfloat16* __restrict__ ck,
+                               __nv_bfloat16* __restrict__ cv, int P0,
+                               const int* __restrict__ step, int Pmax, float scale_log2,
+                               __nv_bfloat16* __restrict__ out, int ld_out) {
+  extern __shared__ float part[];  // [kAttnGroups][kDh] partial outputs, then [kAttnGroups][2]
+  __shared__ __align__(16) __nv_bfloat16 qs[kDh];
+  pdl_wait();
+  pdl_launch_dependents();
+  const int h = blockIdx.x, i = blockIdx.y;
+  const int pos = P0 + *step - 1;
+  if (pos < 0 || pos >= Pmax) return;  // the host keeps every step inside the cache
+  const int npos = pos + 1;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  __nv_bfloat16* K = ck + (static_cast<size_t>(i) * H + h) * Pmax * kDh;
+  __nv_bfloat16* Vc = cv + (static_cast<size_t>(i) * H + h) * Pmax * kDh;
+  {
+    constexpr int half = kDh / 2;
+    const __nv_bfloat16* row = qkv + static_cast<size_t>(i) * ld;
+    if (threadIdx.x < 2 * half) {
+      const int j = threadIdx.x & (half - 1), blk = threadIdx.x / half;  // 0: q, 1: k
+      const float2 cs = table[static_cast<size_t>(pos) * half + j];
+      const __nv_bfloat16* x = row + blk * d + h * kDh;
+      const float x1 = __bfloat162float(x[j]), x2 = __bfloat162float(x[j + half]);
+      const __nv_bfloat16 o1 = __float2bfloat16_rn(__fsub_rn(__fmul_rn(x1, cs.x), __fmul_rn(x2, cs.y)));
+      const __nv_bfloat16 o2 = __float2bfloat16_rn(__fadd_rn(__fmul_rn(x1, cs.y), __fmul_rn(x2, cs.x)));
+      __nv_bfloat16* dst = blk == 0 ? qs : K + static_cast<size_t>(pos) * kDh;
+      dst[j] = o1;
+      dst[j + half] = o2;
+    } else if (threadIdx.x < 2 * half + kDh / 8) {
+      const int e = 8 * (threadIdx.x - 2 * half);
+      *reinterpret_cast<uint4*>(Vc + static_cast<size_t>(pos) * kDh + e) =
+          *reinterpret_cast<const uint4*>(row + 2 * d + h * kDh + e);
+    }
+  }
+  __syncthreads();  // q in shared memory, the new k and v visible to the whole block
+  const int g = lane >> 3, sub = lane & 7;
+  const int G = warp * 4 + g;
+  float qf[16];
+  {
+    const uint4 a = *reinterpret_cast<const uint4*>(qs + 16 * sub);
+    const uint4 b = *reinterpret_cast<const uint4*>(qs + 16 * sub + 8);
+    const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const float2 f = unpack_bf16x2(w[k]);
+      qf[2 * k] = f.x * scale_log2;
+      qf[2 * k + 1] = f.y * scale_log2;
+    }
+  }
+  // rows of positions G + 32 (2 t) and G + 32 (2 t + 1): K and V, 2 x 16 bytes each per lane
+  auto load = [&](int t, uint4 (&kk)[4], uint4 (&vv)[4]) {
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      const int p = G + kAttnGroups * (2 * t + e);
+      if (p < npos) {
+        const size_t off = static_cast<size_t>(p) * kDh + 16 * sub;
+        kk[2 * e] = __ldcs(reinterpret_cast<const uint4*>(K + off));
+        kk[2 * e + 1] = __ldcs(reinterpret_cast<const uint4*>(K + off + 8));
+        vv[2 * e] = __ldcs(reinterpret_cast<const uint4*>(Vc + off));
+        vv[2 * e + 1] = __ldcs(reinterpret_cast<const uint4*>(Vc + off + 8));
+      } else {
+        kk[2 * e] = kk[2 * e + 1] = vv[2 * e] = vv[2 * e + 1] = make_uint4(0u, 0u, 0u, 0u);
+      }
+    }
+  };
+  float acc[16];
+#pragma unroll
+  for (int k = 0; k < 16; ++k) acc[k] = 0.f;
+  float m_ref = -INFINITY, l = 0.f;
+  const int iters = (npos + 2 * kAttnGroups - 1) / (2 * kAttnGroups);  // block-uniform
+  uint4 ck4[4], cv4[4], nk4[4], nv4[4];
+  load(0, ck4, cv4);
+  for (int t = 0; t < iters; ++t) {
+    if (t + 1 < iters) load(t + 1, nk4, nv4);
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      const int p = G + kAttnGroups * (2 * t + e);
+      const uint32_t kw[8] = {ck4[2 * e].x, ck4[2 * e].y, ck4[2 * e].z, ck4[2 * e].w,
+                              ck4[2 * e + 1].x, ck4[2 * e + 1].y, ck4[2 * e + 1].z, ck4[2 * e + 1].w};
+      float sdot = 0.f;
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const float2 f = unpack_bf16x2(kw[k]);
+        sdot = fmaf(qf[2 * k], f.x, sdot);
+        sdot = fmaf(qf[2 * k + 1], f.y, sdot);
+      }
+#pragma unroll
+      for (int o = 1; o < 8; o <<= 1) sdot += __shfl_xor_sync(0xffffffffu, sdot, o);
+      if (p < npos) {  // uniform over the 8 lanes of a group
+        if (sdot > m_ref + 8.f) {
+          const float corr = exp2f(m_ref - sdot);
+#pragma unroll
+          for (int k = 0; k < 16; ++k) acc[k] *= corr;
+          l *= corr;
+          m_ref = sdot;
+        }
+        const float wgt = exp2f(sdot - m_ref);
+        l += wgt;
+        const uint32_t vw[8] = {cv4[2 * e].x, cv4[2 * e].y, cv4[2 * e].z, cv4[2 * e].w,
+                                cv4[2 * e + 1].x, cv4[2 * e + 1].y, cv4[2 * e + 1].z, cv4[2 * e + 1].w};
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const float2 f = unpack_bf16x2(vw[k]);
+          acc[2 * k] = fmaf(wgt, f.x, acc[2 * k]);
+          acc[2 * k + 1] = fmaf(wgt, f.y, acc[2 * k + 1]);
+        }
+      }
+    }
+    if (t + 1 < iters) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        ck4[e] = nk4[e];
+        cv4[e] = nv4[e];
+      }
+    }
+  }
+  float* ml = part + kAttnGroups * kDh;
+#pragma unroll
+  for (int k = 0; k < 16; ++k) part[G * kDh + 16 * sub + k] = acc[k];
+  if (sub == 0) {
+    ml[2 * G] = m_ref;
+    ml[2 * G + 1] = l;
+  }
+  __syncthreads();
+  if (threadIdx.x < kDh) {
+    float M = -INFINITY;
+#pragma unroll 8
+    for (int q = 0; q < kAttnGroups; ++q) M = fmaxf(M, ml[2 * q]);
+    float o = 0.f, L = 0.f;
+#pragma unroll 8
+    for (int q = 0; q < kAttnGroups; ++q) {
+      const float f = exp2f(ml[2 * q] - M);  // 0 for a group without positions
+      o = fmaf(f, part[q * kDh + threadIdx.x], o);
+      L = fmaf(f, ml[2 * q + 1], L);
+    }
+    out[static_cast<size_t>(i) * ld_out + h * kDh + threadIdx.x] = __float2bfloat16_rn(o / L);
+  }
+}
 
 // ---------------------------------------------------------------- fused row kernels
 // Thread-block clusters of kCl CTAs share one row: each CTA owns a 1/kCl slice of the columns,
@@ -680,17 +817,30 @@ int launch_decode_attention(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t
                             int64_t Pmax, void* out, int64_t ld_out, cudaStream_t st) {
   if (R == 0) return 0;
   const size_t smem = decode_attention_smem(Pmax);
-  // pipelined key loads up to 16 rows (4 sequences: decode step 3.755 -> 3.617 ms); above, one
-  // iteration's loads at a time (pipelined was slower at 12, 32 and 64 sequences: 4.38 against
-  // 4.18 ms, 5.62 against 5.58 ms, 7.37-7.44 against 7.26 ms)
-  const bool prefetch = R <= kGemvMaxRows;
-  auto kernel = prefetch ? decode_attention_kernel<true> : decode_attention_kernel<false>;
-  static size_t attr[2] = {0, 0};
-  if (smem > 48 * 1024 && smem > attr[prefetch]) {
+  // up to 16 rows the single-pass kernel (4 sequences: decode step 3.685 -> 3.541 ms against
+  // the two-pass kernel with pipelined key loads, which had taken it from 3.755 to 3.617);
+  // above, the two-pass kernel with one iteration's loads at a time (pipelined loads were
+  // slower at 12, 32 and 64 sequences: 4.38 against 4.18 ms, 5.62 against 5.58 ms,
+  // 7.37-7.44 against 7.26 ms)
+  if (R <= kGemvMaxRows) {
+    const size_t smem1 = static_cast<size_t>(kAttnGroups) * (kDh + 2) * 4;
+    const cudaError_t e1 = launch_pdl(
+        decode_attention_1p_kernel, dim3(static_cast<unsigned>(H), static_cast<unsigned>(R)),
+        dim3(kAttnThreads), smem1, st, static_cast<const __nv_bfloat16*>(qkv), static_cast<int>(ld),
+        static_cast<int>(d), static_cast<int>(H), static_cast<const float2*>(table),
+        static_cast<__nv_bfloat16*>(ck), static_cast<__nv_bfloat16*>(cv), static_cast<int>(P0),
+        step, static_cast<int>(Pmax),
+        1.4426950408889634f / sqrtf(static_cast<float>(kDh)), static_cast<__nv_bfloat16*>(out),
+        static_cast<int>(ld_out));
+    return e1 == cudaSuccess ? 0 : -3;
+  }
+  auto kernel = decode_attention_kernel;
+  static size_t attr = 0;
+  if (smem > 48 * 1024 && smem > attr) {
     if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(smem)) != cudaSuccess)
       return -1;
-    attr[prefetch] = smem;
+    attr = smem;
   }
   const cudaError_t e = launch_pdl(
       kernel, dim3(static_cast<unsigned>(H), static_cast<unsigned>(R)),
