@@ -401,7 +401,9 @@ def test_score_llama7b_every_kernel_of_every_layer_against_oracle():
     32 equals, bit for bit, the one the full pass leaves in its workspace (whose first bytes
     hold the fp32 residual stream): every kernel launch of the pass's decoder stack is checked
     at its own full size, without the drift that a chain of bf16 stages accumulates (steps of
-    Algorithm 1's scoring pass; §3 Dynamic LoRA: both streams)."""
+    Algorithm 1's scoring pass; §3 Dynamic LoRA: both streams). The pass's heads (final norm,
+    log-probabilities of both streams, KL-penalised reward, score, values, GAE) are checked
+    from the pass's own residual stream after layer 32 at their stated tolerances."""
     cfg = dict(llama.LLAMA7B)
     nl, d, F, r, nh = cfg["n_layers"], cfg["d_model"], cfg["ffn"], cfg["lora_rank"], cfg["n_heads"]
     P0, L = cfg["prompt_len"], cfg["response_len"]
@@ -514,6 +516,33 @@ def test_score_llama7b_every_kernel_of_every_layer_against_oracle():
     assert torch.equal(h, h_pass), "the per-op composition differs from the pass"
     print("worst relative error per kernel over 32 layers (stated 2e-2): " +
           ", ".join(f"{k} {v:.1e}" for k, v in worst.items()))
+
+    # the pass's heads from its own residual stream after layer 32 (llama_score's steps after
+    # the decoder stack: final RMSNorm, LM head and log-softmax of both streams, KL-penalised
+    # reward, score and values; GAE on the pass's own rewards and values), within the stated
+    # tolerances: log-probabilities and the KL reward 5e-3, score and values 2e-2, GAE 1e-4
+    hp = host_f64(h_pass)
+    rows = np.arange(P0 - 1, P - 1)  # the hidden row that predicts each response token
+    fin = [O.round_bf16(O.rmsnorm(hp[i * T:(i + 1) * T], view["final_norm"], eps)) for i in range(2)]
+    resp = ids[0, P0:].cpu().numpy()
+    lr, _ = O.log_softmax_gather(fin[0][rows] @ view["lm_head"].T, resp)
+    la, _ = O.log_softmax_gather(fin[1][rows] @ view["lm_head"].T, resp)
+    score = float(fin[0][P - 1] @ view["w_rm"])
+    values = fin[1][rows] @ view["w_rm"]
+    reward = O.kl_penalised_reward(la[None], lr[None], [L], [score], cfg["beta"])[0]
+    got = {k: v.cpu().double().numpy() for k, v in out.items()}
+    heads = {
+        "logp_actor": assert_abs(got["logp_actor"][0], la, TOL_LOGP, "logp_actor"),
+        "logp_ref": assert_abs(got["logp_ref"][0], lr, TOL_LOGP, "logp_ref"),
+        "reward": assert_abs(got["reward"][0], reward, TOL_LOGP, "KL-penalised reward"),
+        "score": assert_rel(got["score"][:1], [score], TOL_LINEAR, "score"),
+        "values": assert_rel(got["values"][0], values, TOL_LINEAR, "values"),
+    }
+    adv, ret = O.gae(got["reward"][:1], got["values"][:1], [L], cfg["gamma"], cfg["lam"])
+    heads["advantages"] = assert_rel(got["advantages"][:1], adv, TOL_GAE, "advantages")
+    heads["returns"] = assert_rel(got["returns"][:1], ret, TOL_GAE, "returns")
+    print("heads from the pass's own residual stream: " +
+          ", ".join(f"{k} {v:.1e}" for k, v in heads.items()))
     del w, ws
     torch.cuda.empty_cache()
 
