@@ -410,7 +410,6 @@ __global__ void __launch_bounds__(kThreads)
 // per-warp ring: stage = 16 W rows + 8 NT token rows of 64 bf16, 3 stages
 template <int NT, int W>  // NT n-tiles of 8 token rows, W warps
 struct Gv {
-  static constexpr int kWarps = W;
   static constexpr int kStages = 3;
   static constexpr int kStageBytes = (16 + 8 * NT) * 128;
   static constexpr int kSmem = W * kStages * kStageBytes + W * 16 * 16 * 4;
@@ -432,7 +431,7 @@ __device__ __forceinline__ void gv_ldsm_x4(uint32_t addr, uint32_t (&a)[4]) {
                : "r"(addr));
 }
 
-template <int NT, int kGvWarps>  // n-tiles of 8 token rows (1 or 2), warps per CTA
+template <int NT, int kGvWarps, bool kAlias = false>  // kAlias: partial tiles in the ring
 __global__ void __launch_bounds__(32 * kGvWarps)
     dual_lora_gemv_kernel(const __nv_bfloat16* __restrict__ x_off,
                           const __nv_bfloat16* __restrict__ x_on, int M, int K, int N,
@@ -442,7 +441,7 @@ __global__ void __launch_bounds__(32 * kGvWarps)
   extern __shared__ __align__(1024) uint8_t smem[];
   constexpr int kGvStages = Gv<NT, kGvWarps>::kStages;
   constexpr int kGvStageBytes = Gv<NT, kGvWarps>::kStageBytes;
-  float* red = reinterpret_cast<float*>(smem + kGvWarps * kGvStages * kGvStageBytes);
+  float* red = reinterpret_cast<float*>(kAlias ? smem : smem + kGvWarps * kGvStages * kGvStageBytes);
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int g = lane >> 2, c = lane & 3;
@@ -539,6 +538,7 @@ __global__ void __launch_bounds__(32 * kGvWarps)
     __syncwarp();
   }
   gv_wait<0>();
+  if (kAlias) __syncthreads();  // the ring is free before it holds the partial tiles
 
   // partial [16 rows x 8 NT tokens] of this warp -> shared memory
   float* rw = red + warp * 16 * 16;
@@ -598,16 +598,27 @@ __global__ void __launch_bounds__(32 * kGvWarps)
 }
 
 template <int NT, int W>
-void launch_gemv_t(const GemmArgs& a, cudaStream_t stream) {
-  constexpr int smem = Gv<NT, W>::kSmem;
+void launch_gemv_t(const GemmArgs& a, int nsm, cudaStream_t stream) {
+  constexpr int smem_full = Gv<NT, W>::kSmem;
+  constexpr int smem_ring = W * Gv<NT, W>::kStages * Gv<NT, W>::kStageBytes;
   static bool attr = false;
   if (!attr) {
     cudaFuncSetAttribute(dual_lora_gemv_kernel<NT, W>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         smem);
+                         smem_full);
+    cudaFuncSetAttribute(dual_lora_gemv_kernel<NT, W, true>,
+                         cudaFuncAttributeMaxDynamicSharedMemorySize, smem_ring);
     attr = true;
   }
   const unsigned grid = static_cast<unsigned>((a.N + 15) / 16);
-  launch_pdl(dual_lora_gemv_kernel<NT, W>, dim3(grid), dim3(32 * W), smem, stream,
+  // the partial tiles in the ring, one more CTA per SM, only where that brings a grid that
+  // just misses one wave into one (the 768-CTA q/k/v shape against 5 x 152 = 760 slots)
+  const int per_sm = 227 * 1024 / (smem_full + 1024);
+  const int per_sm_alias = 227 * 1024 / (smem_ring + 1024);
+  const bool alias = per_sm_alias > per_sm && static_cast<int>(grid) > per_sm * nsm &&
+                     static_cast<int>(grid) <= per_sm_alias * nsm;
+  const int smem = alias ? smem_ring : smem_full;
+  launch_pdl(alias ? dual_lora_gemv_kernel<NT, W, true> : dual_lora_gemv_kernel<NT, W>,
+      dim3(grid), dim3(32 * W), smem, stream,
       static_cast<const __nv_bfloat16*>(a.x_off),
       static_cast<const __nv_bfloat16*>(a.shared_x ? a.x_off : a.x_on), static_cast<int>(a.M),
       static_cast<int>(a.K), static_cast<int>(a.N), static_cast<const __nv_bfloat16*>(a.W),
@@ -715,14 +726,14 @@ int launch_dual_lora_gemv(const GemmArgs& a, cudaStream_t stream) {
   const bool narrow = (a.N + 15) / 16 >= 4LL * nsm;  // enough row blocks for 4-warp CTAs
   if (rows <= 8) {
     if (narrow)
-      launch_gemv_t<1, 4>(a, stream);
+      launch_gemv_t<1, 4>(a, nsm, stream);
     else
-      launch_gemv_t<1, 8>(a, stream);
+      launch_gemv_t<1, 8>(a, nsm, stream);
   } else {
     if (narrow)
-      launch_gemv_t<2, 4>(a, stream);
+      launch_gemv_t<2, 4>(a, nsm, stream);
     else
-      launch_gemv_t<2, 8>(a, stream);
+      launch_gemv_t<2, 8>(a, nsm, stream);
   }
   return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
 }

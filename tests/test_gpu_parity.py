@@ -299,8 +299,10 @@ def test_projection_sweep_sampled(K, N, r):
 
 @pytest.mark.parametrize("M", [1, 4, 8, 16])
 def test_decode_gemv_sampled(M):
-    """Decode-shaped inputs through the 4096 -> 32000 LM head and the 11008 -> 4096 down."""
-    for K, N in ((4096, 32000), (11008, 4096)):
+    """Decode-shaped inputs through the 4096 -> 32000 LM head, the 11008 -> 4096 down and the
+    4096 -> 12288 q/k/v projection (whose 768 CTAs, up to 8 token rows, keep their partial
+    tiles in the ring so that six fit on an SM and the grid is one wave)."""
+    for K, N in ((4096, 32000), (11008, 4096), (4096, 12288)):
         x, _, W, A, Bm = _linear_problem(M, K, N, 16, seed=3000 + M + N)
         y_off, y_on = _run_linear(dev_bf16(x), None, dev_bf16(W), dev_bf16(A), dev_bf16(Bm), 2.0)
         ref_off, ref_on = O.dual_lora_linear(f64(x), f64(x), f64(W), f64(A), f64(Bm), 2.0)
