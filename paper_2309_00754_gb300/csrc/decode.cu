@@ -360,8 +360,10 @@ __global__ void __launch_bounds__(kAttnThreads)
 
 // ---------------------------------------------------------------- fused row kernels
 // Thread-block clusters of kCl CTAs share one row: each CTA owns a 1/kCl slice of the columns,
-// partial sums meet through distributed shared memory (mapa + ld.shared::cluster) and are
-// added in CTA-rank order, so the result does not depend on timing.
+// partial sums meet through distributed shared memory and are added in CTA-rank order, so the
+// result does not depend on timing. The one-row kernels push their partials into the CTAs
+// that add them (st.shared::cluster), so one cluster barrier makes them visible and no CTA
+// reads another's shared memory after it; the grouped kernels read them (ld.shared::cluster).
 constexpr int kCl = 8;
 constexpr int kRowThreads = 256;
 constexpr int kRowWarps = kRowThreads / 32;
@@ -396,22 +398,33 @@ __device__ __forceinline__ void prefetch_a_slice(const __nv_bfloat16* __restrict
   asm volatile("cp.async.commit_group;" ::: "memory");
 }
 
-__device__ __forceinline__ void wait_a_slice() {
-  asm volatile("cp.async.wait_group 0;" ::: "memory");
-  __syncthreads();
+// the cluster's CTAs have all started (the arrive at kernel start, the wait before the first
+// store into another CTA's shared memory)
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void st_cluster_f32(float* local, uint32_t rank, float v) {
+  uint32_t raddr;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(raddr) : "r"(smem_u32(local)), "r"(rank));
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(raddr), "f"(v) : "memory");
 }
 
-// Partial LoRA down-projection of this CTA's slice: up[j] = sum_e xs[e] A[j][c0 + e] for
-// j < r2 (warps take j in turn, lanes 4 columns at a time); then rank 0 adds the kCl
-// partials in rank order and writes u = bf16(s * sum). xs holds the slice's bf16 values; As,
-// if not NULL, the prefetched slice of A ([r2][n]).
-__device__ __forceinline__ void lora_slice(const float* xs, int n, int c0, int K,
-                                           const __nv_bfloat16* __restrict__ A,
-                                           const __nv_bfloat16* As, int r2, float s, float* up,
-                                           __nv_bfloat16* __restrict__ u_row, uint32_t rank) {
+// Partial LoRA down-projection of this CTA's slice, pushed into rank 0's shared memory:
+// recv[rank][j] = sum_e xs[e] A[j][c0 + e] for j < r2 (warps take j in turn, lanes 4 columns
+// at a time); after one cluster barrier rank 0 adds the kCl partials in rank order and writes
+// u = bf16(s * sum). xs holds the slice's bf16 values; As, if not NULL, the prefetched slice
+// of A ([r2][n]). No CTA reads another's shared memory after the barrier, so every CTA may
+// leave once it has passed it.
+__device__ __forceinline__ void lora_slice_push(const float* xs, int n, int c0, int K,
+                                                const __nv_bfloat16* __restrict__ A,
+                                                const __nv_bfloat16* As, int r2, float s,
+                                                float* recv, __nv_bfloat16* __restrict__ u_row,
+                                                uint32_t rank) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int j = warp; j < r2; j += kRowWarps) {
-    // the slice from shared memory when it was prefetched, else from global memory
     const __nv_bfloat16* aj = As ? As + static_cast<size_t>(j) * n : A + static_cast<size_t>(j) * K + c0;
     float acc = 0.f;
     for (int e = 4 * lane; e < n; e += 128) {
@@ -424,16 +437,21 @@ __device__ __forceinline__ void lora_slice(const float* xs, int n, int c0, int K
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if (lane == 0) up[j] = acc;
+    if (lane == 0) st_cluster_f32(recv + static_cast<int>(rank) * kMaxR2 + j, 0, acc);
   }
   cluster_sync_all();
   if (rank == 0) {
     for (int j = threadIdx.x; j < r2; j += kRowThreads) {
       float t = 0.f;
-      for (uint32_t q = 0; q < kCl; ++q) t += ld_cluster_f32(up + j, q);
+      for (uint32_t q = 0; q < kCl; ++q) t += recv[q * kMaxR2 + j];
       u_row[j] = __float2bfloat16_rn(s * t);
     }
   }
+}
+
+__device__ __forceinline__ void wait_a_slice() {
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
+  __syncthreads();
 }
 
 // Cluster (kCl, 1, 1) per row of h [R, d]: h += y (RESID), a = bf16(rmsnorm(h) w) and, for the
@@ -447,12 +465,13 @@ __global__ void __launch_bounds__(kRowThreads)
                          int r2, float s, __nv_bfloat16* __restrict__ u) {
   extern __shared__ float xs[];  // this CTA's slice of the row, then the prefetched A slice
   __shared__ float red[kRowWarps];
-  __shared__ float part;
-  __shared__ float up[kMaxR2];
+  __shared__ float parts[kCl];              // every rank's sum of squares, pushed by each rank
+  __shared__ float recv[kCl * kMaxR2];      // rank 0: every rank's LoRA partials
   const uint32_t rank = cluster_rank();
   const int row = blockIdx.y;
   const int n = d / kCl, c0 = static_cast<int>(rank) * n;
   const bool lora = A != nullptr && row >= S;
+  cluster_arrive_relaxed();
   __nv_bfloat16* As = (lora && r2 * n * 2 <= kMaxAPrefetch) ? reinterpret_cast<__nv_bfloat16*>(xs + n)
                                                              : nullptr;
   if (As) prefetch_a_slice(A, d, c0, n, r2, As);
@@ -478,10 +497,11 @@ __global__ void __launch_bounds__(kRowThreads)
     ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
   }
   ss = row_block_sum(ss, red);
-  if (threadIdx.x == 0) part = ss;
+  cluster_wait();  // every CTA of the cluster has started
+  if (threadIdx.x < kCl) st_cluster_f32(&parts[rank], threadIdx.x, ss);
   cluster_sync_all();
   float tot = 0.f;
-  for (uint32_t q = 0; q < kCl; ++q) tot += ld_cluster_f32(&part, q);
+  for (uint32_t q = 0; q < kCl; ++q) tot += parts[q];
   const float inv = rsqrtf(tot / static_cast<float>(d) + eps);
   __nv_bfloat16* ar = a + static_cast<size_t>(row) * d + c0;
   for (int e = 4 * threadIdx.x; e < n; e += 4 * kRowThreads) {
@@ -498,11 +518,8 @@ __global__ void __launch_bounds__(kRowThreads)
   }
   if (As) wait_a_slice();
   else __syncthreads();
-  if (lora)
-    lora_slice(xs, n, c0, d, A, As, r2, s, up, u + static_cast<size_t>(row - S) * r2, rank);
-  else
-    cluster_sync_all();  // the same cluster barriers on every path
-  cluster_sync_all();    // rank 0's remote reads finish before any CTA leaves
+  if (lora)  // the same on every CTA of the cluster (one row)
+    lora_slice_push(xs, n, c0, d, A, As, r2, s, recv, u + static_cast<size_t>(row - S) * r2, rank);
 }
 
 // Cluster (kCl, 1, 1) per row of gu [R, 2F] (gate/up interleaved in blocks of 128):
@@ -513,11 +530,12 @@ __global__ void __launch_bounds__(kRowThreads)
                        int S, const __nv_bfloat16* __restrict__ A, int r, float s,
                        __nv_bfloat16* __restrict__ u) {
   extern __shared__ float xs[];  // this CTA's slice of m, then the prefetched A slice
-  __shared__ float up[kMaxR2];
+  __shared__ float recv[kCl * kMaxR2];  // rank 0: every rank's LoRA partials
   const uint32_t rank = cluster_rank();
   const int row = blockIdx.y;
   const int n = F / kCl, c0 = static_cast<int>(rank) * n;
-  const bool lora = A != nullptr && row >= S;
+  const bool lora = A != nullptr && row >= S;  // the same on every CTA of the cluster
+  if (lora) cluster_arrive_relaxed();
   __nv_bfloat16* As = (lora && r * n * 2 <= kMaxAPrefetch) ? reinterpret_cast<__nv_bfloat16*>(xs + n)
                                                             : nullptr;
   if (As) prefetch_a_slice(A, F, c0, n, r, As);
@@ -545,11 +563,10 @@ __global__ void __launch_bounds__(kRowThreads)
   }
   if (As) wait_a_slice();
   else __syncthreads();
-  if (lora)
-    lora_slice(xs, n, c0, F, A, As, r, s, up, u + static_cast<size_t>(row - S) * r, rank);
-  else
-    cluster_sync_all();
-  cluster_sync_all();
+  if (lora) {
+    cluster_wait();  // every CTA of the cluster has started
+    lora_slice_push(xs, n, c0, F, A, As, r, s, recv, u + static_cast<size_t>(row - S) * r, rank);
+  }
 }
 
 // ---------------------------------------------------------------- grouped row kernels
@@ -557,7 +574,7 @@ __global__ void __launch_bounds__(kRowThreads)
 // of up to kMaxRpc rows (each CTA still owns a 1/kCl slice of the columns). Warp w handles
 // rows w, w + 8, ... of the group, so a row's sums stay inside one warp; the LoRA factor's
 // slice is read once per CTA for all of the group's LoRA-on rows instead of once per row;
-// the group pays the same three cluster barriers as a single row.
+// the group pays three cluster barriers, as the one-row kernels once did.
 // Measured on GB300 (decode step of the 7B model): groups of R / 32 rows gave 7.82 ms against
 // 8.09 ms for one cluster per row at 128 rows, but 6.24 against 6.01 ms at 64 rows. A grouped
 // SwiGLU kernel (slices of 1376 features per warp) was slower than one cluster per row even at
