@@ -212,18 +212,22 @@ __global__ void __launch_bounds__(kAttnThreads)
 
 // Single-pass form for small batches: 32 groups of 8 lanes per block (lane = 16 dimensions of
 // a key or value row); group G takes positions G + 32 t, two per iteration, and the K and V
-// loads of the next iteration are issued before this one's are reduced. Each group keeps a
+// rows of the next two iterations are in flight (cp.async into a shared-memory ring) while
+// this one's are reduced. Each group keeps a
 // lazily rescaled running maximum (moved only when a score exceeds it by more than 2^8, as in
 // the prefill's flash attention), its sum and its 16-dimension slice of the weighted values;
 // the 32 partial results meet in shared memory at the end.
 constexpr int kAttnGroups = kAttnThreads / 8;
+constexpr int kAttnStages = 3;                          // iterations of K / V loads staged
+constexpr int kAttnStageBytes = 2 * kAttnGroups * 512;  // two positions per group, K and V
 __global__ void __launch_bounds__(kAttnThreads)
     decode_attention_1p_kernel(const __nv_bfloat16* __restrict__ qkv, int ld, int d, int H,
                                const float2* __restrict__ table, __nv_bfloat16* __restrict__ ck,
                                __nv_bfloat16* __restrict__ cv, int P0,
                                const int* __restrict__ step, int Pmax, float scale_log2,
                                __nv_bfloat16* __restrict__ out, int ld_out) {
-  extern __shared__ float part[];  // [kAttnGroups][kDh] partial outputs, then [kAttnGroups][2]
+  extern __shared__ float part[];  // the K / V ring; after it, [kAttnGroups][kDh] partial
+                                   // outputs, then [kAttnGroups][2]
   __shared__ __align__(16) __nv_bfloat16 qs[kDh];
   pdl_wait();
   pdl_launch_dependents();
@@ -268,19 +272,30 @@ __global__ void __launch_bounds__(kAttnThreads)
       qf[2 * k + 1] = f.y * scale_log2;
     }
   }
-  // rows of positions G + 32 (2 t) and G + 32 (2 t + 1): K and V, 2 x 16 bytes each per lane
-  auto load = [&](int t, uint4 (&kk)[4], uint4 (&vv)[4]) {
+  // rows of positions G + 32 (2 t + e), e = 0, 1: each lane copies its 32 bytes of K and of V
+  // into stage t % kAttnStages of a shared-memory ring with cp.async (missing positions read
+  // as zeros), so kAttnStages - 1 iterations of loads are in flight while one is reduced; a
+  // lane reads back only the bytes it copied itself
+  const uint32_t ring = smem_u32(part);
+  auto slot = [&](int stage, int e) {
+    return ring + stage * kAttnStageBytes + (e * kAttnGroups + G) * 512 + 32 * sub;
+  };
+  auto load = [&](int t) {
+    const int stage = t % kAttnStages;
 #pragma unroll
     for (int e = 0; e < 2; ++e) {
       const int p = G + kAttnGroups * (2 * t + e);
-      if (p < npos) {
-        const size_t off = static_cast<size_t>(p) * kDh + 16 * sub;
-        kk[2 * e] = __ldcs(reinterpret_cast<const uint4*>(K + off));
-        kk[2 * e + 1] = __ldcs(reinterpret_cast<const uint4*>(K + off + 8));
-        vv[2 * e] = __ldcs(reinterpret_cast<const uint4*>(Vc + off));
-        vv[2 * e + 1] = __ldcs(reinterpret_cast<const uint4*>(Vc + off + 8));
-      } else {
-        kk[2 * e] = kk[2 * e + 1] = vv[2 * e] = vv[2 * e + 1] = make_uint4(0u, 0u, 0u, 0u);
+      const bool ok = p < npos;
+      const size_t off = static_cast<size_t>(ok ? p : 0) * kDh + 16 * sub;
+      const uint32_t dst = slot(stage, e);
+#pragma unroll
+      for (int h2 = 0; h2 < 2; ++h2) {
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst + 16 * h2),
+                     "l"(K + off + 8 * h2), "r"(ok ? 16 : 0)
+                     : "memory");
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst + 256 + 16 * h2),
+                     "l"(Vc + off + 8 * h2), "r"(ok ? 16 : 0)
+                     : "memory");
       }
     }
   };
@@ -289,15 +304,25 @@ __global__ void __launch_bounds__(kAttnThreads)
   for (int k = 0; k < 16; ++k) acc[k] = 0.f;
   float m_ref = -INFINITY, l = 0.f;
   const int iters = (npos + 2 * kAttnGroups - 1) / (2 * kAttnGroups);  // block-uniform
-  uint4 ck4[4], cv4[4], nk4[4], nv4[4];
-  load(0, ck4, cv4);
+  __syncthreads();  // the new key and value are in the cache before any lane copies them
+#pragma unroll
+  for (int t = 0; t < kAttnStages - 1; ++t) {
+    if (t < iters) load(t);
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  }
   for (int t = 0; t < iters; ++t) {
-    if (t + 1 < iters) load(t + 1, nk4, nv4);
+    if (t + kAttnStages - 1 < iters) load(t + kAttnStages - 1);
+    asm volatile("cp.async.commit_group;" ::: "memory");
+    asm volatile("cp.async.wait_group %0;" ::"n"(kAttnStages - 1) : "memory");
+    const int stage = t % kAttnStages;
 #pragma unroll
     for (int e = 0; e < 2; ++e) {
       const int p = G + kAttnGroups * (2 * t + e);
-      const uint32_t kw[8] = {ck4[2 * e].x, ck4[2 * e].y, ck4[2 * e].z, ck4[2 * e].w,
-                              ck4[2 * e + 1].x, ck4[2 * e + 1].y, ck4[2 * e + 1].z, ck4[2 * e + 1].w};
+      const uint32_t src = slot(stage, e);
+      uint4 k0, k1, v0, v1;
+      asm volatile("ld.shared.v4.b32 {%0,%1,%2,%3}, [%4];" : "=r"(k0.x), "=r"(k0.y), "=r"(k0.z), "=r"(k0.w) : "r"(src));
+      asm volatile("ld.shared.v4.b32 {%0,%1,%2,%3}, [%4];" : "=r"(k1.x), "=r"(k1.y), "=r"(k1.z), "=r"(k1.w) : "r"(src + 16));
+      const uint32_t kw[8] = {k0.x, k0.y, k0.z, k0.w, k1.x, k1.y, k1.z, k1.w};
       float sdot = 0.f;
 #pragma unroll
       for (int k = 0; k < 8; ++k) {
@@ -317,8 +342,9 @@ __global__ void __launch_bounds__(kAttnThreads)
         }
         const float wgt = exp2f(sdot - m_ref);
         l += wgt;
-        const uint32_t vw[8] = {cv4[2 * e].x, cv4[2 * e].y, cv4[2 * e].z, cv4[2 * e].w,
-                                cv4[2 * e + 1].x, cv4[2 * e + 1].y, cv4[2 * e + 1].z, cv4[2 * e + 1].w};
+        asm volatile("ld.shared.v4.b32 {%0,%1,%2,%3}, [%4];" : "=r"(v0.x), "=r"(v0.y), "=r"(v0.z), "=r"(v0.w) : "r"(src + 256));
+        asm volatile("ld.shared.v4.b32 {%0,%1,%2,%3}, [%4];" : "=r"(v1.x), "=r"(v1.y), "=r"(v1.z), "=r"(v1.w) : "r"(src + 272));
+        const uint32_t vw[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
           const float2 f = unpack_bf16x2(vw[k]);
@@ -327,14 +353,9 @@ __global__ void __launch_bounds__(kAttnThreads)
         }
       }
     }
-    if (t + 1 < iters) {
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        ck4[e] = nk4[e];
-        cv4[e] = nv4[e];
-      }
-    }
   }
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
+  __syncthreads();  // the ring is free before it holds the partial results
   float* ml = part + kAttnGroups * kDh;
 #pragma unroll
   for (int k = 0; k < 16; ++k) part[G * kDh + 16 * sub + k] = acc[k];
@@ -840,7 +861,14 @@ int launch_decode_attention(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t
   // slower at 12, 32 and 64 sequences: 4.38 against 4.18 ms, 5.62 against 5.58 ms,
   // 7.37-7.44 against 7.26 ms)
   if (R <= kGemvMaxRows) {
-    const size_t smem1 = static_cast<size_t>(kAttnGroups) * (kDh + 2) * 4;
+    const size_t smem1 = static_cast<size_t>(kAttnStages) * kAttnStageBytes;  // > the partials
+    static bool attr1 = false;
+    if (!attr1) {
+      if (cudaFuncSetAttribute(decode_attention_1p_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               static_cast<int>(smem1)) != cudaSuccess)
+        return -1;
+      attr1 = true;
+    }
     const cudaError_t e1 = launch_pdl(
         decode_attention_1p_kernel, dim3(static_cast<unsigned>(H), static_cast<unsigned>(R)),
         dim3(kAttnThreads), smem1, st, static_cast<const __nv_bfloat16*>(qkv), static_cast<int>(ld),
