@@ -127,8 +127,6 @@ __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;"
 __device__ __forceinline__ void pdl_launch_dependents() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
-// Bring [p, p + bytes) into L2 (p and bytes multiples of 16). L2 is the device's point of
-// coherence, so a prefetch issued before pdl_wait() never makes a later read stale.
 // Thread-block clusters: this CTA's rank, a barrier over every thread of every CTA of the
 // cluster (release/acquire: shared-memory writes before it are visible to remote reads after
 // it), and a read of another CTA's shared memory at the address of `local` in this CTA.
@@ -220,6 +218,8 @@ __device__ __forceinline__ void tc_commit_pair(uint32_t bar) {
       : "memory");
 }
 
+// Bring [p, p + bytes) into L2 (p and bytes multiples of 16). L2 is the device's point of
+// coherence, so a prefetch issued before pdl_wait() never makes a later read stale.
 __device__ __forceinline__ void prefetch_l2_bulk(const void* p, uint32_t bytes) {
   asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(p)),
                "r"(bytes)

@@ -220,6 +220,7 @@ __global__ void __launch_bounds__(kAttnThreads)
 constexpr int kAttnGroups = kAttnThreads / 8;
 constexpr int kAttnStages = 3;                          // iterations of K / V loads staged
 constexpr int kAttnStageBytes = 2 * kAttnGroups * 512;  // two positions per group, K and V
+constexpr uint32_t kAttnPrefetchPiece = 4096;           // bytes per L2 prefetch
 __global__ void __launch_bounds__(kAttnThreads)
     decode_attention_1p_kernel(const __nv_bfloat16* __restrict__ qkv, int ld, int d, int H,
                                const float2* __restrict__ table, __nv_bfloat16* __restrict__ ck,
@@ -229,49 +230,31 @@ __global__ void __launch_bounds__(kAttnThreads)
   extern __shared__ float part[];  // the K / V ring; after it, [kAttnGroups][kDh] partial
                                    // outputs, then [kAttnGroups][2]
   __shared__ __align__(16) __nv_bfloat16 qs[kDh];
+  const int h = blockIdx.x, i = blockIdx.y;
+  __nv_bfloat16* K = ck + (static_cast<size_t>(i) * H + h) * Pmax * kDh;
+  __nv_bfloat16* Vc = cv + (static_cast<size_t>(i) * H + h) * Pmax * kDh;
+  {
+    // The cached keys and values of earlier positions are final: this (row, head)'s stream
+    // into L2 while the q/k/v projection finishes. The step counter read here may not have
+    // advanced yet; a prefetch is only a hint, clamped to the cache.
+    const int hint = min(max(P0 + *reinterpret_cast<const volatile int*>(step) - 1, 0), Pmax);
+    const uint32_t bytes = static_cast<uint32_t>(hint) * kDh * 2;  // a multiple of 256
+    const uint32_t pieces = (bytes + kAttnPrefetchPiece - 1) / kAttnPrefetchPiece;
+    for (uint32_t q = threadIdx.x; q < 2 * pieces; q += kAttnThreads) {
+      const bool isv = q >= pieces;
+      const uint32_t off = (isv ? q - pieces : q) * kAttnPrefetchPiece;
+      prefetch_l2_bulk(reinterpret_cast<const uint8_t*>(isv ? Vc : K) + off,
+                       min(kAttnPrefetchPiece, bytes - off));
+    }
+  }
   pdl_wait();
   pdl_launch_dependents();
-  const int h = blockIdx.x, i = blockIdx.y;
   const int pos = P0 + *step - 1;
   if (pos < 0 || pos >= Pmax) return;  // the host keeps every step inside the cache
   const int npos = pos + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  __nv_bfloat16* K = ck + (static_cast<size_t>(i) * H + h) * Pmax * kDh;
-  __nv_bfloat16* Vc = cv + (static_cast<size_t>(i) * H + h) * Pmax * kDh;
-  {
-    constexpr int half = kDh / 2;
-    const __nv_bfloat16* row = qkv + static_cast<size_t>(i) * ld;
-    if (threadIdx.x < 2 * half) {
-      const int j = threadIdx.x & (half - 1), blk = threadIdx.x / half;  // 0: q, 1: k
-      const float2 cs = table[static_cast<size_t>(pos) * half + j];
-      const __nv_bfloat16* x = row + blk * d + h * kDh;
-      const float x1 = __bfloat162float(x[j]), x2 = __bfloat162float(x[j + half]);
-      const __nv_bfloat16 o1 = __float2bfloat16_rn(__fsub_rn(__fmul_rn(x1, cs.x), __fmul_rn(x2, cs.y)));
-      const __nv_bfloat16 o2 = __float2bfloat16_rn(__fadd_rn(__fmul_rn(x1, cs.y), __fmul_rn(x2, cs.x)));
-      __nv_bfloat16* dst = blk == 0 ? qs : K + static_cast<size_t>(pos) * kDh;
-      dst[j] = o1;
-      dst[j + half] = o2;
-    } else if (threadIdx.x < 2 * half + kDh / 8) {
-      const int e = 8 * (threadIdx.x - 2 * half);
-      *reinterpret_cast<uint4*>(Vc + static_cast<size_t>(pos) * kDh + e) =
-          *reinterpret_cast<const uint4*>(row + 2 * d + h * kDh + e);
-    }
-  }
-  __syncthreads();  // q in shared memory, the new k and v visible to the whole block
   const int g = lane >> 3, sub = lane & 7;
   const int G = warp * 4 + g;
-  float qf[16];
-  {
-    const uint4 a = *reinterpret_cast<const uint4*>(qs + 16 * sub);
-    const uint4 b = *reinterpret_cast<const uint4*>(qs + 16 * sub + 8);
-    const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
-#pragma unroll
-    for (int k = 0; k < 8; ++k) {
-      const float2 f = unpack_bf16x2(w[k]);
-      qf[2 * k] = f.x * scale_log2;
-      qf[2 * k + 1] = f.y * scale_log2;
-    }
-  }
   // rows of positions G + 32 (2 t + e), e = 0, 1: each lane copies its 32 bytes of K and of V
   // into stage t % kAttnStages of a shared-memory ring with cp.async (missing positions read
   // as zeros), so kAttnStages - 1 iterations of loads are in flight while one is reduced; a
@@ -299,17 +282,55 @@ __global__ void __launch_bounds__(kAttnThreads)
       }
     }
   };
+  const int iters = (npos + 2 * kAttnGroups - 1) / (2 * kAttnGroups);  // block-uniform
+  auto prologue = [&]() {
+#pragma unroll
+    for (int t = 0; t < kAttnStages - 1; ++t) {
+      if (t < iters) load(t);
+      asm volatile("cp.async.commit_group;" ::: "memory");
+    }
+  };
+  // The first kAttnStages - 1 iterations' loads go out before the rotary and the cache append
+  // when none of their positions is this step's (block-uniform); otherwise after them.
+  const bool early = (kAttnStages - 1) * 2 * kAttnGroups <= pos;
+  if (early) prologue();
+  {
+    constexpr int half = kDh / 2;
+    const __nv_bfloat16* row = qkv + static_cast<size_t>(i) * ld;
+    if (threadIdx.x < 2 * half) {
+      const int j = threadIdx.x & (half - 1), blk = threadIdx.x / half;  // 0: q, 1: k
+      const float2 cs = table[static_cast<size_t>(pos) * half + j];
+      const __nv_bfloat16* x = row + blk * d + h * kDh;
+      const float x1 = __bfloat162float(x[j]), x2 = __bfloat162float(x[j + half]);
+      const __nv_bfloat16 o1 = __float2bfloat16_rn(__fsub_rn(__fmul_rn(x1, cs.x), __fmul_rn(x2, cs.y)));
+      const __nv_bfloat16 o2 = __float2bfloat16_rn(__fadd_rn(__fmul_rn(x1, cs.y), __fmul_rn(x2, cs.x)));
+      __nv_bfloat16* dst = blk == 0 ? qs : K + static_cast<size_t>(pos) * kDh;
+      dst[j] = o1;
+      dst[j + half] = o2;
+    } else if (threadIdx.x < 2 * half + kDh / 8) {
+      const int e = 8 * (threadIdx.x - 2 * half);
+      *reinterpret_cast<uint4*>(Vc + static_cast<size_t>(pos) * kDh + e) =
+          *reinterpret_cast<const uint4*>(row + 2 * d + h * kDh + e);
+    }
+  }
+  __syncthreads();  // q in shared memory, the new k and v in the cache before any lane copies them
+  float qf[16];
+  {
+    const uint4 a = *reinterpret_cast<const uint4*>(qs + 16 * sub);
+    const uint4 b = *reinterpret_cast<const uint4*>(qs + 16 * sub + 8);
+    const uint32_t w[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const float2 f = unpack_bf16x2(w[k]);
+      qf[2 * k] = f.x * scale_log2;
+      qf[2 * k + 1] = f.y * scale_log2;
+    }
+  }
   float acc[16];
 #pragma unroll
   for (int k = 0; k < 16; ++k) acc[k] = 0.f;
   float m_ref = -INFINITY, l = 0.f;
-  const int iters = (npos + 2 * kAttnGroups - 1) / (2 * kAttnGroups);  // block-uniform
-  __syncthreads();  // the new key and value are in the cache before any lane copies them
-#pragma unroll
-  for (int t = 0; t < kAttnStages - 1; ++t) {
-    if (t < iters) load(t);
-    asm volatile("cp.async.commit_group;" ::: "memory");
-  }
+  if (!early) prologue();
   for (int t = 0; t < iters; ++t) {
     if (t + kAttnStages - 1 < iters) load(t + kAttnStages - 1);
     asm volatile("cp.async.commit_group;" ::: "memory");
@@ -751,11 +772,67 @@ __global__ void __launch_bounds__(kRowThreads)
   cluster_sync_all();    // remote reads of up finish before any CTA leaves
 }
 
+// The draw of one step (Algorithm 1: the actor samples each sequence's next token; the
+// reference head's log-probability of it feeds the KL reward, and the critic head's value is
+// kept with it). One thread-block cluster of kSampleCl CTAs per sequence s; CTA `rank` owns a
+// 1/kSampleCl slice of the vocabulary and of the value head's d inputs. In one pass over its
+// slice a thread keeps, for both heads, a running maximum and the sum of exp(z - max) (the
+// sum rescaled when the maximum moves), and the first maximum of z + Gumbel noise. The
+// per-thread, per-warp and per-CTA partials are merged in a fixed order (the CTAs' into rank
+// 0 through distributed shared memory), so the result does not depend on timing; the argmax
+// takes the lowest index among equal keys.
+constexpr int kSampleCl = 8;
 constexpr int kSampleThreads = 512;
+constexpr int kSampleWarps = kSampleThreads / 32;
+constexpr int kSampleBatch = 2;  // float4 loads per array and thread in flight together
 
-// Block s: the drawn token of sequence s at step t = *step from the actor's logits (row
-// S + s) plus the step's Gumbel noise (none: greedy), its log-probability under both heads
-// (the reference head is row s), and the value w_rm . fin[S + s].
+struct SamplePart {
+  float m_on, l_on, m_off, l_off, key, v;
+  int idx;
+};
+
+__device__ __forceinline__ void lse_add(float& m, float& l, float z) {
+  if (z > m) {
+    l = l * expf(m - z) + 1.f;  // 0 * 0 + 1 on the first finite z
+    m = z;
+  } else if (z > -INFINITY) {
+    l += expf(z - m);
+  }
+}
+__device__ __forceinline__ void lse_merge(float& m, float& l, float m2, float l2) {
+  const float M = fmaxf(m, m2);
+  if (M == -INFINITY) return;  // both sides empty
+  l = l * expf(m - M) + l2 * expf(m2 - M);
+  m = M;
+}
+__device__ __forceinline__ void argmax_merge(float& key, int& idx, float k2, int i2) {
+  if (k2 > key || (k2 == key && i2 < idx)) {
+    key = k2;
+    idx = i2;
+  }
+}
+__device__ __forceinline__ void sample_merge(SamplePart& a, const SamplePart& b) {
+  lse_merge(a.m_on, a.l_on, b.m_on, b.l_on);
+  lse_merge(a.m_off, a.l_off, b.m_off, b.l_off);
+  argmax_merge(a.key, a.idx, b.key, b.idx);
+  a.v += b.v;
+}
+__device__ __forceinline__ SamplePart shfl_part(const SamplePart& p, int o) {
+  SamplePart q;
+  q.m_on = __shfl_xor_sync(0xffffffffu, p.m_on, o);
+  q.l_on = __shfl_xor_sync(0xffffffffu, p.l_on, o);
+  q.m_off = __shfl_xor_sync(0xffffffffu, p.m_off, o);
+  q.l_off = __shfl_xor_sync(0xffffffffu, p.l_off, o);
+  q.key = __shfl_xor_sync(0xffffffffu, p.key, o);
+  q.v = __shfl_xor_sync(0xffffffffu, p.v, o);
+  q.idx = __shfl_xor_sync(0xffffffffu, p.idx, o);
+  return q;
+}
+
+// Cluster (kSampleCl, 1, 1) per sequence s: the drawn token of step t = *step from the
+// actor's logits (row S + s) plus the step's Gumbel noise (none: greedy), its log-probability
+// under both heads (the reference head is row s), and the value w_rm . fin[S + s].
+// V % 4 == 0 (16-byte rows).
 __global__ void __launch_bounds__(kSampleThreads)
     sample_tokens_kernel(const float* __restrict__ logits, int S, int V,
                          const float* __restrict__ gumbel, const __nv_bfloat16* __restrict__ fin,
@@ -763,75 +840,91 @@ __global__ void __launch_bounds__(kSampleThreads)
                          const int* __restrict__ step, int n_steps, int32_t* __restrict__ tokens,
                          float* __restrict__ logp_a, float* __restrict__ logp_r,
                          float* __restrict__ values, int32_t* __restrict__ cur_ids) {
-  __shared__ float red[kSampleThreads / 32];
-  __shared__ float bkey[kSampleThreads / 32];
-  __shared__ int bidx[kSampleThreads / 32];
-  const int s = blockIdx.x;
+  __shared__ SamplePart warp_part[kSampleWarps];
+  __shared__ float recv[kSampleCl][8];  // rank 0: every CTA's partial (idx as its bits)
+  pdl_wait();
+  pdl_launch_dependents();
   const int t = *step;
-  if (t < 0 || t >= n_steps) return;  // the host launches exactly n_steps draws
+  if (t < 0 || t >= n_steps) return;  // grid-uniform; the host launches exactly n_steps draws
+  cluster_arrive_relaxed();
+  const uint32_t rank = cluster_rank();
+  const int s = blockIdx.x / kSampleCl;
   const float* zo = logits + static_cast<size_t>(S + s) * V;
   const float* zr = logits + static_cast<size_t>(s) * V;
   const float* gn = gumbel ? gumbel + (static_cast<size_t>(t) * S + s) * V : nullptr;
-  float m_on = -INFINITY, m_off = -INFINITY, key = -INFINITY;
-  int idx = V;
-  for (int k = threadIdx.x; k < V; k += kSampleThreads) {
-    const float a = zo[k], b = zr[k];
-    m_on = fmaxf(m_on, a);
-    m_off = fmaxf(m_off, b);
-    const float kk = gn ? a + gn[k] : a;
-    if (kk > key) {  // k increases: the first maximum of this thread's stripe
-      key = kk;
-      idx = k;
-    }
-  }
-  // argmax across the block, ties to the lowest index
+  const int V4 = V / 4;
+  const int chunk4 = (V4 + kSampleCl - 1) / kSampleCl;
+  const int b4 = min(V4, static_cast<int>(rank) * chunk4), e4 = min(V4, b4 + chunk4);
+
+  SamplePart p = {-INFINITY, 0.f, -INFINITY, 0.f, -INFINITY, 0.f, V};
+  for (int q0 = b4 + threadIdx.x; q0 < e4; q0 += kSampleBatch * kSampleThreads) {
+    float4 a[kSampleBatch], b[kSampleBatch], g[kSampleBatch];
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float k2 = __shfl_xor_sync(0xffffffffu, key, o);
-    const int i2 = __shfl_xor_sync(0xffffffffu, idx, o);
-    if (k2 > key || (k2 == key && i2 < idx)) {
-      key = k2;
-      idx = i2;
+    for (int j = 0; j < kSampleBatch; ++j) {
+      const int q = q0 + j * kSampleThreads;
+      if (q < e4) {
+        a[j] = reinterpret_cast<const float4*>(zo)[q];
+        b[j] = reinterpret_cast<const float4*>(zr)[q];
+        g[j] = gn ? reinterpret_cast<const float4*>(gn)[q] : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < kSampleBatch; ++j) {
+      const int q = q0 + j * kSampleThreads;
+      if (q >= e4) break;
+      const float av[4] = {a[j].x, a[j].y, a[j].z, a[j].w};
+      const float bv[4] = {b[j].x, b[j].y, b[j].z, b[j].w};
+      const float gv[4] = {g[j].x, g[j].y, g[j].z, g[j].w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        lse_add(p.m_on, p.l_on, av[e]);
+        lse_add(p.m_off, p.l_off, bv[e]);
+        const float kk = gn ? av[e] + gv[e] : av[e];
+        if (kk > p.key) {  // indices increase along a thread: the first maximum is kept
+          p.key = kk;
+          p.idx = 4 * q + e;
+        }
+      }
     }
   }
-  const int warp = threadIdx.x >> 5;
-  if ((threadIdx.x & 31) == 0) {
-    bkey[warp] = key;
-    bidx[warp] = idx;
-  }
-  m_on = block_max(m_on, red);
-  m_off = block_max(m_off, red);
-  key = bkey[0];
-  idx = bidx[0];
-  for (int w = 1; w < kSampleThreads / 32; ++w)
-    if (bkey[w] > key || (bkey[w] == key && bidx[w] < idx)) {
-      key = bkey[w];
-      idx = bidx[w];
-    }
-  float l_on = 0.f, l_off = 0.f;
-  for (int k = threadIdx.x; k < V; k += kSampleThreads) {
-    l_on += expf(zo[k] - m_on);
-    l_off += expf(zr[k] - m_off);
-  }
-  l_on = block_sum(l_on, red);
-  l_off = block_sum(l_off, red);
+  // this CTA's slice of the value head
+  const int dchunk = (d + kSampleCl - 1) / kSampleCl;
+  const int d0 = min(d, static_cast<int>(rank) * dchunk), d1 = min(d, d0 + dchunk);
   const __nv_bfloat16* f = fin + static_cast<size_t>(S + s) * d;
-  float v = 0.f;
-  for (int k = threadIdx.x; k < d; k += kSampleThreads)
-    v = fmaf(__bfloat162float(f[k]), __bfloat162float(w_rm[k]), v);
-  v = block_sum(v, red);
+  for (int k = d0 + threadIdx.x; k < d1; k += kSampleThreads)
+    p.v = fmaf(__bfloat162float(f[k]), __bfloat162float(w_rm[k]), p.v);
+
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) sample_merge(p, shfl_part(p, o));
+  const int warp = threadIdx.x >> 5;
+  if ((threadIdx.x & 31) == 0) warp_part[warp] = p;
+  __syncthreads();
+  cluster_wait();  // every CTA of the cluster has started: rank 0's shared memory is live
   if (threadIdx.x == 0) {
-    const int tok = idx < V ? idx : 0;
-    const size_t o = static_cast<size_t>(s) * n_steps + t;
-    tokens[o] = tok;
-    logp_a[o] = zo[tok] - (m_on + logf(l_on));
-    logp_r[o] = zr[tok] - (m_off + logf(l_off));
-    values[o] = v;
-    cur_ids[s] = tok;
+    SamplePart c = warp_part[0];
+    for (int w = 1; w < kSampleWarps; ++w) sample_merge(c, warp_part[w]);
+    const float vals[8] = {c.m_on, c.l_on, c.m_off, c.l_off, c.key, __int_as_float(c.idx), c.v, 0.f};
+#pragma unroll
+    for (int k = 0; k < 7; ++k) st_cluster_f32(&recv[rank][k], 0, vals[k]);
   }
+  cluster_sync_all();
+  if (rank != 0 || threadIdx.x != 0) return;
+  SamplePart c = {recv[0][0], recv[0][1], recv[0][2], recv[0][3], recv[0][4], recv[0][6],
+                  __float_as_int(recv[0][5])};
+  for (int q = 1; q < kSampleCl; ++q) {
+    const SamplePart o = {recv[q][0], recv[q][1], recv[q][2], recv[q][3], recv[q][4], recv[q][6],
+                          __float_as_int(recv[q][5])};
+    sample_merge(c, o);
+  }
+  const int tok = c.idx < V ? c.idx : 0;
+  const size_t o = static_cast<size_t>(s) * n_steps + t;
+  tokens[o] = tok;
+  logp_a[o] = zo[tok] - (c.m_on + logf(c.l_on));
+  logp_r[o] = zr[tok] - (c.m_off + logf(c.l_off));
+  values[o] = c.v;
+  cur_ids[s] = tok;
 }
 
-__global__ void step_advance_kernel(int* step) { *step += 1; }
 
 
 }  // namespace
@@ -899,18 +992,6 @@ int launch_decode_attention(void* qkv, int64_t R, int64_t ld, int64_t d, int64_t
 }
 
 
-int launch_sample_tokens(const float* logits, int64_t S, int64_t V, const float* gumbel,
-                         const void* fin, int64_t d, const void* w_rm, const int* step,
-                         int64_t n_steps, int32_t* tokens, float* logp_a, float* logp_r,
-                         float* values, int32_t* cur_ids, cudaStream_t st) {
-  if (S == 0) return 0;
-  sample_tokens_kernel<<<static_cast<unsigned>(S), kSampleThreads, 0, st>>>(
-      logits, static_cast<int>(S), static_cast<int>(V), gumbel,
-      static_cast<const __nv_bfloat16*>(fin), static_cast<int>(d),
-      static_cast<const __nv_bfloat16*>(w_rm), step, static_cast<int>(n_steps), tokens, logp_a,
-      logp_r, values, cur_ids);
-  return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
-}
 
 // Raise a kernel's dynamic shared-memory limit when a launch needs more than the default
 // (once per kernel and size: `done` remembers the largest limit set).
@@ -923,18 +1004,19 @@ static int set_smem_limit(const void* kernel, size_t bytes, size_t& done) {
   return 0;
 }
 
-// cudaLaunchKernelEx with a (kCl, 1, 1) cluster and programmatic dependent launch
+// cudaLaunchKernelEx with a (cl, 1, 1) cluster of `threads`-thread CTAs (by default the row
+// kernels' kCl CTAs of kRowThreads) and programmatic dependent launch
 template <typename... KArgs, typename... Args>
-static cudaError_t launch_cluster(void (*kernel)(KArgs...), dim3 grid, size_t smem,
-                                  cudaStream_t st, Args&&... args) {
+static cudaError_t launch_cluster_n(void (*kernel)(KArgs...), dim3 grid, unsigned threads,
+                                    unsigned cl, size_t smem, cudaStream_t st, Args&&... args) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
-  cfg.blockDim = dim3(kRowThreads);
+  cfg.blockDim = dim3(threads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = kCl;
+  attr[0].val.clusterDim.x = cl;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -942,6 +1024,26 @@ static cudaError_t launch_cluster(void (*kernel)(KArgs...), dim3 grid, size_t sm
   cfg.attrs = attr;
   cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+template <typename... KArgs, typename... Args>
+static cudaError_t launch_cluster(void (*kernel)(KArgs...), dim3 grid, size_t smem,
+                                  cudaStream_t st, Args&&... args) {
+  return launch_cluster_n(kernel, grid, kRowThreads, kCl, smem, st, std::forward<Args>(args)...);
+}
+
+int launch_sample_tokens(const float* logits, int64_t S, int64_t V, const float* gumbel,
+                         const void* fin, int64_t d, const void* w_rm, const int* step,
+                         int64_t n_steps, int32_t* tokens, float* logp_a, float* logp_r,
+                         float* values, int32_t* cur_ids, cudaStream_t st) {
+  if (S == 0) return 0;
+  if (V % 4 != 0) return -1;
+  const cudaError_t e = launch_cluster_n(
+      sample_tokens_kernel, dim3(static_cast<unsigned>(S * kSampleCl)), kSampleThreads, kSampleCl,
+      0, st, logits, static_cast<int>(S), static_cast<int>(V), gumbel,
+      static_cast<const __nv_bfloat16*>(fin), static_cast<int>(d),
+      static_cast<const __nv_bfloat16*>(w_rm), step, static_cast<int>(n_steps), tokens, logp_a,
+      logp_r, values, cur_ids);
+  return e == cudaSuccess ? 0 : -3;
 }
 
 int launch_row_norm_lora(float* h, const void* y, const void* w, int64_t R, int64_t d, float eps,
@@ -1017,9 +1119,5 @@ int launch_swiglu_lora(const void* gu, int64_t R, int64_t F, void* m, int64_t S,
   return e == cudaSuccess ? 0 : -3;
 }
 
-int launch_step_advance(int* step, cudaStream_t st) {
-  step_advance_kernel<<<1, 1, 0, st>>>(step);
-  return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
-}
 
 }  // namespace hydra

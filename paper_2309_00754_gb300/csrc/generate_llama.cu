@@ -235,12 +235,13 @@ hydra_status hydra_generate_llama(const hydra_llama_config* cfg, const hydra_lla
   const hydra::RowMap last{1, P0, P0 - 1};
   HY_TRY(hydra::launch_rmsnorm(h, w->final_norm, R, d, c.rms_eps, last, find, st));
 
-  // one decode pass of the last drawn token (cur) at position P0 + step - 1, ending in the
-  // final-normed rows find. Eight launches per layer: the residual add, the RMSNorm and the
-  // next projection's LoRA down-projection share one cluster kernel, as do the SwiGLU and
-  // the down projection's LoRA down-projection.
+  // one decode pass of the last drawn token (cur), ending in the final-normed rows find. Its
+  // embedding launch advances the device-side step counter to the number of tokens drawn, so
+  // the pass runs at position P0 + step - 1. Eight launches per layer: the residual add, the
+  // RMSNorm and the next projection's LoRA down-projection share one cluster kernel, as do
+  // the SwiGLU and the down projection's LoRA down-projection.
   auto decode_layers = [&]() -> int {
-    int x = hydra::launch_embed(w->embed, V, d, cur, S, 2, hd, err, st);
+    int x = hydra::launch_embed(w->embed, V, d, cur, S, 2, hd, err, st, step);
     const void* resid = nullptr;  // the previous layer's down projection, added into h
     for (int64_t l = 0; l < c.n_layers && x == 0; ++l) {
       const hydra_llama_layer& ly = w->layers[l];
@@ -267,13 +268,12 @@ hydra_status hydra_generate_llama(const hydra_llama_config* cfg, const hydra_lla
                                       s, nullptr, st);
     return x;
   };
-  // the LM head on both streams' final rows and the draw of step *step
+  // the LM head on both streams' final rows and the draw of step *step (the count so far)
   auto draw = [&]() -> int {
     int x = decode_linear(find, S, d, V, w->lm_head, nullptr, 0, nullptr, logits, true, err, st);
     if (x == 0)
       x = hydra::launch_sample_tokens(logits, S, V, gumbel, find, d, w->w_rm, step, n_steps, tokens,
                                       logp_actor, logp_ref, values, cur, st);
-    if (x == 0) x = hydra::launch_step_advance(step, st);
     return x;
   };
 

@@ -162,7 +162,6 @@ int launch_sample_tokens(const float* logits, int64_t S, int64_t V, const float*
                          const void* fin, int64_t d, const void* w_rm, const int* step,
                          int64_t n_steps, int32_t* tokens, float* logp_a, float* logp_r,
                          float* values, int32_t* cur_ids, cudaStream_t st);
-int launch_step_advance(int* step, cudaStream_t st);
 // Thread-block-cluster row kernels of the decode step (8 CTAs per row): h += y (y may be
 // NULL), a = bf16(rmsnorm(h) w) and, for rows i >= S, u[i - S] = bf16(s a A^T) (A [r2, d] or
 // NULL); and m = SwiGLU(gu) (gate/up interleaved by 128) with u[i - S] = bf16(s m A^T).
@@ -178,8 +177,10 @@ struct RowMap {
   long long g_out, g_in, off;
 };
 
+// h [copies T, d] fp32 = the embedding rows of ids; with `step` (decode), a dependent launch
+// that also advances the device-side step counter by one
 int launch_embed(const void* table, int64_t V, int64_t d, const int32_t* ids, int64_t T,
-                 int copies, float* h, int* err, cudaStream_t st);
+                 int copies, float* h, int* err, cudaStream_t st, int* step = nullptr);
 int launch_rmsnorm(const float* x, const void* w, int64_t rows, int64_t d, float eps,
                    const RowMap& map, void* y, cudaStream_t st);
 // (cos, sin) float2 table [P][Dh / 2] of the rotary angles pos * theta^(-2i/Dh)

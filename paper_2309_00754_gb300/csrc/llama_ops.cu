@@ -24,10 +24,16 @@ __device__ __forceinline__ long long map_row(long long i, const RowMap& m) {
 
 // ---------------------------------------------------------------- embedding
 
+// h[s T + t] = fp32(table[ids[t]]) for s < copies; a NaN row and an error code for an id
+// outside the vocabulary. With `step` (the decode loop's device-side step counter), block 0
+// also advances the counter: the token just drawn moves to the next position.
 __global__ void embed_kernel(const __nv_bfloat16* __restrict__ table, int V, int d,
                              const int32_t* __restrict__ ids, long long T, int copies,
-                             float* __restrict__ h, int* err) {
+                             float* __restrict__ h, int* err, int* step) {
+  pdl_wait();
+  pdl_launch_dependents();
   const long long t = blockIdx.x;
+  if (step != nullptr && t == 0 && threadIdx.x == 0) *step += 1;
   const int id = ids[t];
   const bool bad = id < 0 || id >= V;
   if (bad && threadIdx.x == 0) record_error(err, kDevBadTokenId);
@@ -259,12 +265,19 @@ unsigned grid_for(long long work, int threads) {
 }  // namespace
 
 int launch_embed(const void* table, int64_t V, int64_t d, const int32_t* ids, int64_t T,
-                 int copies, float* h, int* err, cudaStream_t st) {
+                 int copies, float* h, int* err, cudaStream_t st, int* step) {
   if (T == 0) return 0;
-  embed_kernel<<<static_cast<unsigned>(T), 128, 0, st>>>(static_cast<const __nv_bfloat16*>(table),
-                                                          static_cast<int>(V), static_cast<int>(d),
-                                                          ids, T, copies, h, err);
-  return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
+  if (step == nullptr) {
+    embed_kernel<<<static_cast<unsigned>(T), 128, 0, st>>>(
+        static_cast<const __nv_bfloat16*>(table), static_cast<int>(V), static_cast<int>(d), ids,
+        T, copies, h, err, nullptr);
+    return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
+  }
+  const cudaError_t e = launch_pdl(embed_kernel, dim3(static_cast<unsigned>(T)), dim3(128), 0, st,
+                                   static_cast<const __nv_bfloat16*>(table), static_cast<int>(V),
+                                   static_cast<int>(d), ids, static_cast<long long>(T), copies, h,
+                                   err, step);
+  return e == cudaSuccess ? 0 : -3;
 }
 
 int launch_rmsnorm(const float* x, const void* w, int64_t rows, int64_t d, float eps,
