@@ -303,9 +303,10 @@ class HydraScoringLlama7B:
     default_steps, default_warmup = 20, 3
     # DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) per GEMM launch, averaged over
     # the 129 GEMM launches of one pass of this workload (batch 4, two streams): an ncu capture
-    # of one full-width decoder layer (its four GEMMs) and the LM head, scaled to 32 identical
-    # layers; no figure for other shapes or stream counts
-    gemm_dram_bytes_per_launch = 496.7e6
+    # of a three-layer pass (layer 0 with its shared q/k/v products, one full middle layer,
+    # the last layer on its compact rows) and the LM head, the middle layer standing for the
+    # 30 middle layers of the 32; no figure for other shapes or stream counts
+    gemm_dram_bytes_per_launch = 490.4e6
 
     def __init__(self, device, seed=4, reference=False):
         import torch
@@ -334,12 +335,17 @@ class HydraScoringLlama7B:
         d, F, V, r = c["d_model"], c["ffn"], c["vocab"], c["lora_rank"]
         nl = c["n_layers"]
         # algorithmic flops per pass of each projection class (both streams; LoRA-up on the
-        # on stream only)
+        # on stream only). Layer 0's q/k/v products serve both streams (equal inputs); the last
+        # layer's o, gate/up and down run on the Tc rows the heads read (L + 1 per sequence).
+        Tc = self.S * (self.L + 1) if self.L + 1 < P else T
         self.class_flops = {
-            "gemm_qkv": nl * (2 * (2 * T * d * 3 * d) + 2 * T * 2 * r * 3 * d),
-            "gemm_o": nl * 2 * (2 * T * d * d),
-            "gemm_gu": nl * (2 * (2 * T * d * 2 * F) + 2 * T * 2 * r * 2 * F),
-            "gemm_down": nl * (2 * (2 * T * F * d) + 2 * T * r * d),
+            "gemm_qkv": (nl - 1) * (2 * (2 * T * d * 3 * d) + 2 * T * 2 * r * 3 * d)
+                        + (2 * T * d * 3 * d + 2 * T * 2 * r * 3 * d),
+            "gemm_o": (nl - 1) * 2 * (2 * T * d * d) + 2 * (2 * Tc * d * d),
+            "gemm_gu": (nl - 1) * (2 * (2 * T * d * 2 * F) + 2 * T * 2 * r * 2 * F)
+                       + (2 * (2 * Tc * d * 2 * F) + 2 * Tc * 2 * r * 2 * F),
+            "gemm_down": (nl - 1) * (2 * (2 * T * F * d) + 2 * T * r * d)
+                         + (2 * (2 * Tc * F * d) + 2 * Tc * r * d),
             "gemm_lmhead": 2 * (2 * SL * d * V),
         }
         self.gemm_flops = sum(self.class_flops.values())
@@ -499,12 +505,16 @@ class HydraPPOScoringLlama7B(HydraScoringLlama7B):
         P = self.P0 + self.L
         T, SL = self.S * P, self.S * self.L
         d, F, V, r, nl = c["d_model"], c["ffn"], c["vocab"], c["lora_rank"], c["n_layers"]
-        # three streams; the LoRA-up runs on the actor and critic streams
+        # three streams; the LoRA-up runs on the actor and critic streams; the last layer's o,
+        # gate/up and down run on the Tc rows the heads read (L + 1 per sequence)
+        Tc = self.S * (self.L + 1) if self.L + 1 < P else T
         self.class_flops = {
             "gemm_qkv": nl * (3 * (2 * T * d * 3 * d) + 2 * (2 * T * 2 * r * 3 * d)),
-            "gemm_o": nl * 3 * (2 * T * d * d),
-            "gemm_gu": nl * (3 * (2 * T * d * 2 * F) + 2 * (2 * T * 2 * r * 2 * F)),
-            "gemm_down": nl * (3 * (2 * T * F * d) + 2 * (2 * T * r * d)),
+            "gemm_o": (nl - 1) * 3 * (2 * T * d * d) + 3 * (2 * Tc * d * d),
+            "gemm_gu": (nl - 1) * (3 * (2 * T * d * 2 * F) + 2 * (2 * T * 2 * r * 2 * F))
+                       + (3 * (2 * Tc * d * 2 * F) + 2 * (2 * Tc * 2 * r * 2 * F)),
+            "gemm_down": (nl - 1) * (3 * (2 * T * F * d) + 2 * (2 * T * r * d))
+                         + (3 * (2 * Tc * F * d) + 2 * (2 * Tc * r * d)),
             "gemm_lmhead": 2 * (2 * SL * d * V),
         }
         self.gemm_flops = sum(self.class_flops.values())

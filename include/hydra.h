@@ -557,6 +557,9 @@ size_t hydra_score_llama_workspace_size(const hydra_llama_config* cfg, int64_t S
  * Outputs fp32 [S, L] (0 at t >= len): logp_actor, logp_ref, reward, values, advantages,
  * returns; score fp32 [S]. Requirements: head_dim == 128, d == n_heads * 128,
  * ffn % 128 == 0, vocab % 8 == 0, r % 8 == 0, 8 <= r <= 128, P0 >= 1, L >= 1.
+ * Work skipped because nothing reads it: layer 0's q/k/v products are formed once for both
+ * streams (their inputs are equal there), and the last layer's o projection and feed-forward
+ * block run only on positions P0 - 1 .. P0 + L - 1 of each sequence, the rows the heads read.
  */
 hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_weights* w,
                                const int32_t* ids, const int32_t* lengths, int64_t S,
@@ -566,7 +569,8 @@ hydra_status hydra_score_llama(const hydra_llama_config* cfg, const hydra_llama_
 
 /*
  * The Hydra-PPO scoring pass (Algorithm 2; §3 Stage 2: two LoRA sets on one base model):
- * as hydra_score_llama with three stacked streams through every layer, each W read once for
+ * as hydra_score_llama with three stacked streams through every layer (layer 0 included; the
+ * last layer on the rows the heads read), each W read once for
  * all three (hydra_lora_linear_tri): LoRA off (reference log-probabilities, reward score),
  * the actor's LoRA set w->layers (logp_actor) and the critic's LoRA set critic[l] (a HOST
  * array of n_layers entries, same rank r), whose final hidden states give the values through

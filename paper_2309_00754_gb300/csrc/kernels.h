@@ -196,6 +196,9 @@ int launch_seq_score(const float* h, const void* norm, const void* w, int64_t d,
                      float* score, cudaStream_t st);
 int launch_causal_attention(const void* qkv, int64_t nseq, int64_t P, int64_t ld, int64_t n_heads,
                             int64_t head_dim, void* out, int64_t ld_out, cudaStream_t st);
+// dst row i = src row map(i) for i < rows, rows of row_bytes bytes (a multiple of 16)
+int launch_gather_rows(const void* src, int64_t rows, int64_t row_bytes, const RowMap& map,
+                       void* dst, cudaStream_t st);
 
 // Largest sequence length the shared-memory GAE scan accepts.
 constexpr int64_t kGaeMaxL = 16384;

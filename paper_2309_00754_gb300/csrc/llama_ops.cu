@@ -256,6 +256,16 @@ __global__ void __launch_bounds__(128)
   if (threadIdx.x == 0) score[s] = red[0] + red[1] + red[2] + red[3];
 }
 
+// dst row i = src row map(i), one CTA per row, 16-byte pieces
+__global__ void __launch_bounds__(128)
+    gather_rows_kernel(const uint4* __restrict__ src, int chunks, RowMap map,
+                       uint4* __restrict__ dst) {
+  const long long i = blockIdx.x;
+  const uint4* s = src + static_cast<size_t>(map_row(i, map)) * chunks;
+  uint4* o = dst + static_cast<size_t>(i) * chunks;
+  for (int c = threadIdx.x; c < chunks; c += 128) o[c] = s[c];
+}
+
 unsigned grid_for(long long work, int threads) {
   long long b = (work + threads - 1) / threads;
   if (b > 152LL * 16) b = 152LL * 16;
@@ -327,6 +337,16 @@ int launch_head_dot(const void* x, int64_t d, const void* w, const RowMap& map, 
   head_dot_kernel<<<static_cast<unsigned>((n + 7) / 8), 256, 0, st>>>(
       static_cast<const __nv_bfloat16*>(x), static_cast<int>(d),
       static_cast<const __nv_bfloat16*>(w), map, n, lengths, static_cast<int>(L), out);
+  return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
+}
+
+int launch_gather_rows(const void* src, int64_t rows, int64_t row_bytes, const RowMap& map,
+                       void* dst, cudaStream_t st) {
+  if (rows == 0) return 0;
+  if (row_bytes % 16 != 0) return -4;
+  gather_rows_kernel<<<static_cast<unsigned>(rows), 128, 0, st>>>(
+      static_cast<const uint4*>(src), static_cast<int>(row_bytes / 16), map,
+      static_cast<uint4*>(dst));
   return cudaPeekAtLastError() == cudaSuccess ? 0 : -3;
 }
 

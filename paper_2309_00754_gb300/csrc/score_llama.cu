@@ -339,6 +339,17 @@ static hydra_status score_pass(const hydra_llama_config* cfg, const hydra_llama_
   const int64_t SL = S * L;
   const float s = c.lora_scale;
   const hydra::RowMap ident{R, R, 0};
+  // The last layer's output is read only on the rows the heads use: per sequence the L rows
+  // that predict the response tokens (positions P0 - 1 .. P - 2; the actor's and reference
+  // log-probabilities and the values) and the row of the last position P - 1 (the reward
+  // score, at the last valid token). Its q/k/v projection and attention run over every
+  // position (the prompt's keys and values); from the o projection on it runs on those
+  // Lc = L + 1 rows of each sequence, gathered into compact buffers: per row the same
+  // arithmetic, so the same bits.
+  const int64_t Lc = L + 1, Tc = S * Lc;
+  const bool compact = Lc < P;
+  const hydra::RowMap pick{Lc, P, c.prompt_len - 1};  // compact row -> row of the full stream
+  float* hc = reinterpret_cast<float*>(qkv);  // compact residual rows (qkv is free by then)
   int e = 0;
 #define HY_TRY(x)                     \
   do {                                \
@@ -356,27 +367,75 @@ static hydra_status score_pass(const hydra_llama_config* cfg, const hydra_llama_
   for (int64_t l = 0; l < c.n_layers; ++l) {
     const hydra_llama_layer& ly = w->layers[l];
     const hydra_llama_lora* cl = critic != nullptr ? &critic[l] : nullptr;  // critic LoRA set
-    // attention block
-    HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(h, ly.norm_attn, R, d, c.rms_eps, ident, a, st));
-    // q/k/v projection with the rotary embedding of q and k fused into the epilogue
+    // attention block: q/k/v projection with the rotary embedding of q and k fused into the
+    // epilogue
     const hydra::StackRope rope{P, 2 * d, rope_table};
-    HY_TRY(hydra::stacked_linear(HYDRA_PROF_GEMM_QKV, a, T, d, 3 * d, ly.w_qkv, ly.a_qv, ly.b_qkv, 2 * r, s, u, qkv, false,
-                          err, st, hydra::kStackEpiRope, &rope, ns, cl ? cl->a_qv : nullptr, cl ? cl->b_qkv : nullptr, u2));
+    if (l == 0 && ns == 2) {
+      // Both streams enter layer 0 with the same embedding rows, so their normed inputs are
+      // equal: one accumulator per tile serves both outputs (x W^T drained to the off stream,
+      // then the LoRA k-blocks accumulated on top for the on stream), the same bits as the
+      // stacked form for half the products (§3 Dynamic LoRA: one frozen W, LoRA switched)
+      HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(h, ly.norm_attn, T, d, c.rms_eps, ident, a, st));
+      HY_PROF(HYDRA_PROF_LORA_DOWN, hydra::launch_lora_down(a, T, d, ly.a_qv, 2 * r, s, u, st));
+      ProfScope ps(HYDRA_PROF_GEMM_QKV, st);
+      hydra::GemmArgs g;
+      g.x_off = a;
+      g.x_on = a;
+      g.M = T;
+      g.K = d;
+      g.N = 3 * d;
+      g.W = ly.w_qkv;
+      g.u = u;
+      g.B = ly.b_qkv;
+      g.r = 2 * r;
+      g.shared_x = true;
+      g.y_off = qkv;
+      g.y_on = static_cast<uint8_t*>(qkv) + static_cast<size_t>(T) * 3 * d * 2;
+      g.out_f32 = 0;
+      g.err = err;
+      g.epi = hydra::kStackEpiRope;
+      g.rope_P = P;
+      g.rope_cols = 2 * d;
+      g.rope_table = rope_table;
+      HY_TRY(hydra::launch_dual_lora_gemm_tc(g, st));
+    } else {
+      HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(h, ly.norm_attn, R, d, c.rms_eps, ident, a, st));
+      HY_TRY(hydra::stacked_linear(HYDRA_PROF_GEMM_QKV, a, T, d, 3 * d, ly.w_qkv, ly.a_qv, ly.b_qkv, 2 * r, s, u, qkv, false,
+                            err, st, hydra::kStackEpiRope, &rope, ns, cl ? cl->a_qv : nullptr, cl ? cl->b_qkv : nullptr, u2));
+    }
     HY_PROF(HYDRA_PROF_ATTENTION,
             hydra::launch_causal_attention(qkv, ns * S, P, 3 * d, c.n_heads, c.head_dim, attn, d, st));
+    // the rows this layer computes from here on: all, or the compact rows of the last layer
+    // (its attention output gathered into `a`, its residual rows into `hc`)
+    const bool last_c = compact && l == c.n_layers - 1;
+    const int64_t Tl = last_c ? Tc : T;
+    const void* x_o = attn;
+    float* hl = h;
+    void* al = a;
+    if (last_c) {
+      HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_gather_rows(attn, ns * Tc, d * 2, pick, a, st));
+      HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_gather_rows(h, ns * Tc, d * 4, pick, hc, st));
+      x_o = a;
+      hl = hc;
+      al = attn;
+    }
+    const hydra::RowMap ident_l{ns * Tl, ns * Tl, 0};
     // o projection added straight into the residual stream (fused epilogue)
-    HY_TRY(hydra::stacked_linear(HYDRA_PROF_GEMM_O, attn, T, d, d, ly.w_o, nullptr, nullptr, 0, s, u, h, false, err, st,
+    HY_TRY(hydra::stacked_linear(HYDRA_PROF_GEMM_O, x_o, Tl, d, d, ly.w_o, nullptr, nullptr, 0, s, u, hl, false, err, st,
                           HYDRA_EPI_RESIDUAL, nullptr, ns));
-    // feed-forward block: gate/up with the SwiGLU fused into the epilogue, down added into h
-    HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(h, ly.norm_ffn, R, d, c.rms_eps, ident, a, st));
-    HY_TRY(hydra::stacked_linear(HYDRA_PROF_GEMM_GU, a, T, d, 2 * F, ly.w_gu, ly.a_gu, ly.b_gu, 2 * r, s, u, m, false, err, st,
+    // feed-forward block: gate/up with the SwiGLU fused into the epilogue, down added into the
+    // residual stream
+    HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(hl, ly.norm_ffn, ns * Tl, d, c.rms_eps, ident_l, al, st));
+    HY_TRY(hydra::stacked_linear(HYDRA_PROF_GEMM_GU, al, Tl, d, 2 * F, ly.w_gu, ly.a_gu, ly.b_gu, 2 * r, s, u, m, false, err, st,
                           HYDRA_EPI_SWIGLU, nullptr, ns, cl ? cl->a_gu : nullptr, cl ? cl->b_gu : nullptr, u2));
-    HY_TRY(hydra::stacked_linear(HYDRA_PROF_GEMM_DOWN, m, T, F, d, ly.w_down, ly.a_down, ly.b_down, r, s, u, h, false, err, st,
+    HY_TRY(hydra::stacked_linear(HYDRA_PROF_GEMM_DOWN, m, Tl, F, d, ly.w_down, ly.a_down, ly.b_down, r, s, u, hl, false, err, st,
                           HYDRA_EPI_RESIDUAL, nullptr, ns, cl ? cl->a_down : nullptr, cl ? cl->b_down : nullptr, u2));
   }
-  // final norm on the rows that predict response tokens: row P0 - 1 + t of each sequence
-  const hydra::RowMap resp{L, P, c.prompt_len - 1};
-  HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(h, w->final_norm, ns * SL, d, c.rms_eps, resp, fin, st));
+  // final norm on the rows that predict response tokens: row P0 - 1 + t of each sequence (row
+  // t of its compact rows)
+  const float* hf = compact ? hc : h;
+  const hydra::RowMap resp = compact ? hydra::RowMap{L, Lc, 0} : hydra::RowMap{L, P, c.prompt_len - 1};
+  HY_PROF(HYDRA_PROF_ELEMENTWISE, hydra::launch_rmsnorm(hf, w->final_norm, ns * SL, d, c.rms_eps, resp, fin, st));
   // LM head of both streams with the log-softmax reduced in the GEMM epilogue
   const int64_t nt = (V + 255) / 256;
   const int32_t* resp_ids = ids + c.prompt_len;  // token of response row s * L + t: ids[s * P + P0 + t]
@@ -405,8 +464,10 @@ static hydra_status score_pass(const hydra_llama_config* cfg, const hydra_llama_
   }
   // reward-model score on the LoRA-off stream at the last valid token; values on the
   // LoRA-on stream (the same head: r_phi = LO(V))
-  HY_PROF(HYDRA_PROF_HEADS, hydra::launch_seq_score(h, w->final_norm, w->w_rm, d, c.rms_eps,
-                                                    lengths, S, L, P, c.prompt_len, sc, st));
+  // (position P0 + len - 1: compact row len of its sequence)
+  HY_PROF(HYDRA_PROF_HEADS, hydra::launch_seq_score(hf, w->final_norm, w->w_rm, d, c.rms_eps,
+                                                    lengths, S, L, compact ? Lc : P,
+                                                    compact ? 1 : c.prompt_len, sc, st));
   // values from the last stream: the on stream (J-Hydra) or the critic stream (Hydra-PPO)
   const void* fin_on = static_cast<uint8_t*>(fin) + static_cast<size_t>(ns - 1) * SL * d * 2;
   const hydra::RowMap dense{SL, SL, 0};

@@ -397,13 +397,16 @@ def test_score_llama7b_every_kernel_of_every_layer_against_oracle():
     rotary outputs relative to the norm of each rotated pair, the SwiGLU output after the
     propagated one-ulp differences of its two unstored bf16 inputs). The
     layers run through the library's per-op entry points (the kernels
-    and arguments hydra_score_llama launches), and the residual stream they leave after layer
-    32 equals, bit for bit, the one the full pass leaves in its workspace (whose first bytes
-    hold the fp32 residual stream): every kernel launch of the pass's decoder stack is checked
-    at its own full size, without the drift that a chain of bf16 stages accumulates (steps of
-    Algorithm 1's scoring pass; §3 Dynamic LoRA: both streams). The pass's heads (final norm,
+    and arguments hydra_score_llama launches, on every row of both streams), and the residual
+    stream they leave equals, bit for bit, the one the full pass leaves in its workspace: after
+    31 layers the whole stream (the workspace's first bytes; layer 0 there runs both streams
+    from one accumulator), after layer 32 the rows the heads read (the pass runs its last
+    layer's o projection and feed-forward block on those rows alone and keeps them where the
+    q/k/v buffer was). So every kernel launch of the pass's decoder stack is checked at its own
+    full size, without the drift that a chain of bf16 stages accumulates (steps of Algorithm
+    1's scoring pass; §3 Dynamic LoRA: both streams). The pass's heads (final norm,
     log-probabilities of both streams, KL-penalised reward, score, values, GAE) are checked
-    from the pass's own residual stream after layer 32 at their stated tolerances."""
+    from the pass's own residual rows after layer 32 at their stated tolerances."""
     cfg = dict(llama.LLAMA7B)
     nl, d, F, r, nh = cfg["n_layers"], cfg["d_model"], cfg["ffn"], cfg["lora_rank"], cfg["n_heads"]
     P0, L = cfg["prompt_len"], cfg["response_len"]
@@ -419,6 +422,11 @@ def test_score_llama7b_every_kernel_of_every_layer_against_oracle():
     H.hydra_score_llama(cfg, w, ids, None, ws, out)
     torch.cuda.synchronize()
     h_pass = ws[:2 * T * d * 4].view(torch.float32).view(2 * T, d).clone()
+    # the last layer's residual rows: positions P0 - 1 .. P - 1 of each stream, kept in the
+    # workspace after the residual stream h [2T, d] fp32 and the normed activations [2T, d] bf16
+    up256 = lambda v: (v + 255) // 256 * 256  # noqa: E731
+    Lc, off = L + 1, up256(2 * T * d * 4) + up256(2 * T * d * 2)
+    hc_pass = ws[off:off + 2 * Lc * d * 4].view(torch.float32).view(2 * Lc, d).clone()
     # the same layers through the per-op entry points
     h = torch.empty(2 * T, d, device="cuda")
     H.hydra_embed(w["embed"], ids.view(-1), 2, h)
@@ -452,6 +460,8 @@ def test_score_llama7b_every_kernel_of_every_layer_against_oracle():
         return np.concatenate([n, n], axis=-1).reshape(T, nh * Dh)
 
     for l in range(nl):
+        if l == nl - 1:
+            assert torch.equal(h, h_pass), "the per-op composition of 31 layers differs from the pass"
         lw = view["wq"][l]  # noqa: F841  (widens layer l's weights once)
         lo = view["lora"]
         h_in = host_f64(h)
@@ -513,21 +523,22 @@ def test_score_llama7b_every_kernel_of_every_layer_against_oracle():
         check("lora_down down", g_ud, O.lora_down(g_m[T:], lo["wd"][0][l], s))
         dn = O.dual_lora_linear(g_m[:T], g_m[T:], view["wd"][l], lo["wd"][0][l], lo["wd"][1][l], s)
         check("down linear (added into the residual stream)", h_out - h_mid, np.concatenate(dn))
-    assert torch.equal(h, h_pass), "the per-op composition differs from the pass"
+    h_rows = torch.cat([h[P0 - 1:P], h[T + P0 - 1:T + P]])
+    assert torch.equal(h_rows, hc_pass), "the per-op composition's last layer differs from the pass"
     print("worst relative error per kernel over 32 layers (stated 2e-2): " +
           ", ".join(f"{k} {v:.1e}" for k, v in worst.items()))
 
-    # the pass's heads from its own residual stream after layer 32 (llama_score's steps after
+    # the pass's heads from its own residual rows after layer 32 (llama_score's steps after
     # the decoder stack: final RMSNorm, LM head and log-softmax of both streams, KL-penalised
     # reward, score and values; GAE on the pass's own rewards and values), within the stated
     # tolerances: log-probabilities and the KL reward 5e-3, score and values 2e-2, GAE 1e-4
-    hp = host_f64(h_pass)
-    rows = np.arange(P0 - 1, P - 1)  # the hidden row that predicts each response token
-    fin = [O.round_bf16(O.rmsnorm(hp[i * T:(i + 1) * T], view["final_norm"], eps)) for i in range(2)]
+    hp = host_f64(hc_pass)  # row i of a stream: position P0 - 1 + i
+    rows = np.arange(0, L)  # the hidden row that predicts each response token
+    fin = [O.round_bf16(O.rmsnorm(hp[i * Lc:(i + 1) * Lc], view["final_norm"], eps)) for i in range(2)]
     resp = ids[0, P0:].cpu().numpy()
     lr, _ = O.log_softmax_gather(fin[0][rows] @ view["lm_head"].T, resp)
     la, _ = O.log_softmax_gather(fin[1][rows] @ view["lm_head"].T, resp)
-    score = float(fin[0][P - 1] @ view["w_rm"])
+    score = float(fin[0][Lc - 1] @ view["w_rm"])  # position P - 1, the last token
     values = fin[1][rows] @ view["w_rm"]
     reward = O.kl_penalised_reward(la[None], lr[None], [L], [score], cfg["beta"])[0]
     got = {k: v.cpu().double().numpy() for k, v in out.items()}
