@@ -278,6 +278,22 @@ def test_score_llama_several_key_blocks_rank16():
     check_pass(cfg, got, w64, ids, None)
 
 
+@pytest.mark.parametrize("P0", [1, 2])
+def test_score_llama_short_prompts_and_empty_response(P0):
+    """Prompts of one token (the heads read every position: no compact last layer) and two
+    tokens (the last layer drops one position per sequence), with an empty response among
+    the sequences, against the oracle. Layer 0 forms its q/k/v products once for both streams
+    in both cases."""
+    cfg = dict(SMALL, prompt_len=P0)
+    sep, w64 = make_model(cfg, 64 + P0)
+    S, P = 3, cfg["prompt_len"] + cfg["response_len"]
+    ids = synth.randint(641 + P0, (S, P), 0, cfg["vocab"])
+    lengths = np.array([40, 0, 13], dtype=np.int32)
+    got = run_pass(cfg, sep, ids, lengths)
+    check_pass(cfg, got, w64, ids, lengths)
+    assert got["score"][1] == 0.0 and not np.any(got["logp_actor"][1])
+
+
 def test_score_llama_lora_off_streams_agree_bitwise():
     # §3 Dynamic LoRA: with every B = 0 the LoRA-on stream is the LoRA-off stream, so the
     # actor and reference log-probabilities agree exactly and the reward is the score alone
