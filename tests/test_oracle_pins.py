@@ -376,6 +376,36 @@ def test_llama_score_causal_and_lora_changes_actor_only():
     assert np.max(np.abs(out["logp_actor"] - ref0["logp_actor"])) > 1e-6
 
 
+@pytest.mark.parametrize("n", [8, 5, 0])
+def test_llama_score_heads_read_only_the_last_prompt_position_on(monkeypatch, n):
+    """The heads (log-probabilities of both streams, values, reward score) read the final
+    hidden states only at positions P - 1 .. T - 1 of the sequence: the rows that predict the
+    response tokens and the last token's row (Alg. 1 scoring steps). Overwriting every other
+    row changes no output. The GPU pass relies on this reading when it runs its last layer's
+    o projection and feed-forward block on those rows alone."""
+    w, cfg = tiny_llama()
+    rng = np.random.default_rng(16)
+    ids = rng.integers(0, 64, size=12)
+    P = 4
+    ref = O.llama_score(w, ids, P, cfg, seq_lengths=n)
+    real = O.llama_final_hidden
+
+    def scrambled(weights, ids_, cfg_, n_layers=None):
+        f_off, f_on = real(weights, ids_, cfg_, n_layers)
+        junk = np.random.default_rng(17).standard_normal((P - 1, f_off.shape[1]))
+        f_off, f_on = f_off.copy(), f_on.copy()
+        f_off[:P - 1] = junk
+        f_on[:P - 1] = -junk
+        return f_off, f_on
+
+    monkeypatch.setattr(O.hydra_oracle, "llama_final_hidden", scrambled)
+    out = O.llama_score(w, ids, P, cfg, seq_lengths=n)
+    for k in ("logp_actor", "logp_ref", "reward", "values", "advantages", "returns"):
+        assert np.array_equal(out[k], ref[k]), k
+    assert out["score"] == ref["score"]
+    assert not np.array_equal(out["h_off"], ref["h_off"])
+
+
 def test_storage_dither_is_off_by_default_and_bounded():
     x = np.array([1.0, 1.0 + 2 ** -9 + 2 ** -20, 3.0, -0.3])
     base = O.round_bf16(x)
